@@ -1,0 +1,84 @@
+"""Pins of the oracle's forward pass: sign, binary product, Unfolder / Folder (Sec. 5.1, App. C)."""
+import itertools
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import method as om
+
+
+def test_sign_definition():
+    """Sec. 5.1: sign(x) = -1 if x <= 0 else +1 (so 0, -0 and NaN give -1)."""
+    x = np.array([0.0, -0.0, np.nan, 1e-45, -1e-45, 3.0, -2.0, np.inf, -np.inf], dtype=np.float32)
+    assert om.sign(x).tolist() == [-1, -1, -1, 1, -1, 1, -1, 1, -1]
+
+
+def _xnor_popcount_dot(a_bits, b_bits, K):
+    """App. C: SUM(X1 (.) X2) = (bitcount(XNOR(x1, x2)) << 1) - K for K-element words."""
+    mask = (1 << K) - 1
+    return (bin(~(a_bits ^ b_bits) & mask).count("1") << 1) - K
+
+
+@pytest.mark.parametrize("K", [1, 2, 5, 8])
+def test_binary_product_exhaustive_xnor(K):
+    """Every pair of +-1 vectors of length K: oracle product == XNOR-popcount form."""
+    vecs = list(itertools.product([0, 1], repeat=K))
+    a = np.array([[1.0 if b else -1.0 for b in v] for v in vecs], dtype=np.float32)
+    acc, _ = om.forward(a, a, np.ones(len(vecs), dtype=np.float32))
+    bits = [sum(b << i for i, b in enumerate(v)) for v in vecs]
+    for i, bi in enumerate(bits):
+        for j, bj in enumerate(bits):
+            assert acc[i, j] == _xnor_popcount_dot(bi, bj, K)
+
+
+def test_forward_brute_force():
+    rng = np.random.default_rng(3)
+    M, K, D = 5, 37, 7
+    x = rng.standard_normal((M, K)).astype(np.float32)
+    x[0, :3] = 0.0
+    w = rng.standard_normal((D, K)).astype(np.float32)
+    gamma = rng.uniform(0.1, 2, D).astype(np.float32)
+    acc, y = om.forward(x, w, gamma)
+    for m in range(M):
+        for j in range(D):
+            s = 0
+            for k in range(K):
+                sx = 1 if x[m, k] > 0 else -1
+                sw = 1 if w[j, k] > 0 else -1
+                s += sx * sw
+            assert acc[m, j] == s
+            assert y[m, j] == np.float32(gamma[j]) * np.float32(s)
+    assert y.dtype == np.float32
+
+
+@pytest.mark.parametrize("N,C,H,W,k,s,p", [(2, 3, 7, 6, 3, 1, 1), (1, 2, 9, 9, 7, 2, 3), (2, 4, 6, 6, 1, 2, 0),
+                                           (3, 1, 5, 4, 3, 2, 1), (1, 5, 4, 4, 3, 1, 0)])
+def test_unfold_fold_match_torch(N, C, H, W, k, s, p):
+    """Unfolder == torch unfold (rows NHW, columns C*k*k); Folder == torch fold."""
+    rng = np.random.default_rng(N * 100 + C)
+    x = rng.standard_normal((N, C, H, W)).astype(np.float32)
+    xu = om.unfold(x, k, k, s, p)
+    ref = torch.nn.functional.unfold(torch.from_numpy(x), k, padding=p, stride=s)  # [N, C*k*k, L]
+    ref = ref.transpose(1, 2).reshape(-1, C * k * k).numpy()
+    assert np.array_equal(xu, ref)
+    Ho, Wo = om.conv_out_hw(H, W, k, k, s, p)
+    acc = rng.integers(-1000, 1000, size=(N * Ho * Wo, C * k * k))
+    folded = om.fold_int(acc, N, C, H, W, k, k, s, p)
+    t = torch.from_numpy(acc.astype(np.float64)).reshape(N, Ho * Wo, C * k * k).transpose(1, 2)
+    reff = torch.nn.functional.fold(t, (H, W), k, padding=p, stride=s).numpy()
+    assert np.array_equal(folded, reff.astype(np.int64))
+
+
+def test_conv_forward_pads_as_minus_one():
+    """Conv forward through the Unfolder equals a convolution of sign(zero-padded X) (reading R1)."""
+    rng = np.random.default_rng(11)
+    N, C, H, W, D, k, s, p = 2, 3, 6, 5, 4, 3, 2, 1
+    x = rng.standard_normal((N, C, H, W)).astype(np.float32)
+    w = rng.standard_normal((D, C, k, k)).astype(np.float32)
+    acc, _ = om.forward(om.unfold(x, k, k, s, p), w.reshape(D, -1), np.ones(D, np.float32))
+    xp = np.pad(x, ((0, 0), (0, 0), (p, p), (p, p)))
+    sx = torch.from_numpy(np.where(xp > 0, 1.0, -1.0))
+    sw = torch.from_numpy(np.where(w > 0, 1.0, -1.0))
+    ref = torch.nn.functional.conv2d(sx, sw, stride=s).numpy()  # [N, D, Ho, Wo]
+    assert np.array_equal(acc.reshape(N, -1, D), ref.reshape(N, D, -1).transpose(0, 2, 1).astype(np.int64))
