@@ -1,0 +1,184 @@
+/*
+ * libfqt1 -- one fully quantized 1-bit training step of a linear or
+ * convolution layer on an sm_103a GPU (1-Bit FQT, arXiv 2408.14267).
+ *
+ * Conventions for every entry point
+ * ---------------------------------
+ *  - Pointers are DEVICE pointers unless stated otherwise.  The caller owns and
+ *    allocates every buffer; the library allocates nothing, never
+ *    synchronizes, and enqueues all work on `stream` (a cudaStream_t, NULL
+ *    for the legacy default stream).
+ *  - Return value: host-side validation / launch status.  On any error no
+ *    kernel has been launched for that call.
+ *  - Conditions found on the device (non-finite gradient values, an expired
+ *    wait) are OR-ed into `*dev_status` (int32, zeroed by the caller); read it
+ *    after synchronizing.
+ *  - Sizes are element counts; every float / int buffer must be 16-byte
+ *    aligned and rows described by an `ld` must keep that alignment.
+ *
+ * Data layouts
+ * ------------
+ *  Packed signs ("bits"): a [rows, cols] sign matrix is stored as uint32 words
+ *  [rows][fqt1_packed_words(cols)]; bit e % 32 of word e / 32 is 1 iff
+ *  x > 0 (sign +1, Sec. 5.1), least significant bit first.  Padding bits and
+ *  padding words are 0.  "row bits" pack a matrix along its columns, "col
+ *  bits" pack its transpose (one packed row per column).
+ *  Gradient codes: uint8 integers q in [0, 2^b - 1] (Sec. 3.2), rows of
+ *  `ld_codes` bytes.  PSQ codes are [capacity * rows_per_group][ld >= D] in
+ *  kept order; PCQ codes are [capacity][ld >= M] (one row per kept channel,
+ *  samples contiguous).
+ *  Convolutions use the Unfolder of App. C: row m = (n*Ho + oh)*Wo + ow,
+ *  column k = (c*kh + i)*kw + j; the layer output / gradient y, gy are
+ *  [N*Ho*Wo, D] (NHWC rows).
+ */
+#ifndef FQT1_H
+#define FQT1_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  FQT1_OK = 0,
+  FQT1_ERR_INVALID_ARG = 1,  /* null pointer, bad size, bad bits/mode        */
+  FQT1_ERR_MISALIGNED = 2,   /* a pointer or ld breaks 16-byte alignment      */
+  FQT1_ERR_UNSUPPORTED = 3,  /* valid but outside the implemented range       */
+  FQT1_ERR_WORKSPACE = 4,    /* workspace missing or too small                */
+  FQT1_ERR_CUDA = 5          /* a CUDA runtime call failed (see fqt1_last_cuda_error) */
+} fqt1_status;
+
+/* Bits OR-ed into *dev_status by kernels. */
+#define FQT1_DEV_NONFINITE 0x100 /* a gradient value was NaN or +-Inf          */
+#define FQT1_DEV_TIMEOUT 0x200   /* a bounded wait expired; results invalid    */
+
+/* How AGP draws its masks m_i (Sec. 5.2) from the keep probabilities p_i. */
+typedef enum {
+  FQT1_SEL_SYSTEMATIC = 0, /* one uniform offset; P(keep i) = p^_i exactly, kept count
+                              floor or ceil of sum p^ (default)                        */
+  FQT1_SEL_BERNOULLI = 1,  /* independent m_i ~ Bern(p^_i)                             */
+  FQT1_SEL_TOPK = 2        /* the floor(n/b) largest ranges, p^ = 1 (App. B, biased)   */
+} fqt1_select;
+
+/* AGP settings of one gradient branch. */
+typedef struct {
+  int32_t bits;            /* b in {1, 2, 4, 8}: bits of a kept group; keep ratio 1/b   */
+  int32_t mode;            /* fqt1_select                                               */
+  uint64_t seed;           /* key of the counter-based generator (Philox4x32-10)        */
+  int64_t rows_per_group;  /* PSQ only: rows of one sample group (1 for linear layers,
+                              Ho*Wo for convolutions); must divide M                    */
+} fqt1_agp_params;
+
+/* One quantized gradient branch (PSQ or PCQ); every array is caller-owned.
+ * n = number of groups (M / rows_per_group for PSQ, D for PCQ);
+ * capacity = fqt1_kept_capacity(n, bits, mode). */
+typedef struct {
+  float* group_min;        /* [n]  Z_i = min of the group (Sec. 3.2)                  */
+  float* group_range;      /* [n]  R_i = max - min                                    */
+  double* p_hat;           /* [n]  keep probability actually used, P_i / 2^32         */
+  int32_t* slot_of_group;  /* [n]  position of group i in the kept list, -1 if pruned  */
+  int32_t* kept_idx;       /* [capacity] kept group ids, ascending; -1 past the count  */
+  int32_t* kept_count;     /* [1]  number of kept groups                               */
+  float* scale;            /* [capacity] S' = R / (B p^) of each kept group            */
+  float* zero;             /* [capacity] Z' = Z / p^ of each kept group                */
+  uint8_t* codes;          /* codes of the kept groups (layout above)                  */
+  int64_t ld_codes;        /* bytes between code rows, multiple of 16                  */
+} fqt1_qgrad;
+
+/* ---------------------------------------------------------------- helpers */
+/* uint32 words of one packed row of n signs: ceil(n/32) rounded up to a multiple of 4. */
+int64_t fqt1_packed_words(int64_t n);
+/* Upper bound of kept groups: n for b = 1 or BERNOULLI, else ceil(n / b). */
+int64_t fqt1_kept_capacity(int64_t n, int32_t bits, int32_t mode);
+/* Smallest legal ld_codes for rows of n codes (n rounded up to 16). */
+int64_t fqt1_codes_ld(int64_t n);
+/* Workspace bytes for fqt1_scq_quantize / fqt1_agp_quantize_grad (which = 0) and
+ * fqt1_bwd_weight_gemm (which = 1) on an [M, D] gradient / [D, K] weight. */
+size_t fqt1_workspace_size(int32_t which, int64_t M, int64_t D, int64_t K, int32_t rows_per_group);
+/* Text of the last CUDA error seen by the calling host thread. */
+const char* fqt1_last_cuda_error(void);
+/* Number of kernels this library has enqueued since it was loaded (all threads). */
+int64_t fqt1_kernel_launches(void);
+
+/* ------------------------------------------------------------ forward side */
+/* Binarize and pack (Sec. 5.1; row / column encoders of App. C, Algorithm 2).
+ * x: [rows, cols] fp32 with leading dimension ld >= cols.
+ * row_bits: [rows][fqt1_packed_words(cols)] or NULL.
+ * col_bits: [cols][fqt1_packed_words(rows)] or NULL.
+ * colsum:   [cols] int32, colsum[c] = sum_r sign(x[r, c]), or NULL.
+ * At least one output must be given.  For the weight W [D, K] the three
+ * outputs feed the forward GEMM, grad_input GEMM and its dequantization; for
+ * a linear input X [M, K] they feed the forward GEMM, grad_weight GEMM and its
+ * dequantization. */
+fqt1_status fqt1_binarize_pack(const float* x, int64_t rows, int64_t cols, int64_t ld, uint32_t* row_bits,
+                               uint32_t* col_bits, int32_t* colsum, void* stream);
+
+/* Unfolder of App. C fused with sign and pack: x [N, C, H, W] fp32 ->
+ * the packed signs of X_u [M = N*Ho*Wo, K = C*kh*kw]; positions in the zero
+ * padding count as x = 0, i.e. sign -1.  Outputs as in fqt1_binarize_pack
+ * for the matrix X_u (row_bits [M][words(K)], col_bits [K][words(M)],
+ * colsum [K] over all M rows). */
+fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw,
+                        int32_t stride, int32_t pad, uint32_t* row_bits, uint32_t* col_bits, int32_t* colsum,
+                        void* stream);
+
+/* Binarized forward GEMM (Sec. 5.1, App. C "binary multiplication"):
+ * acc[m, j] = sum_k sign(X)[m, k] sign(W)[j, k], y[m, j] = gamma[j] * acc[m, j] (fp32).
+ * sx_row: [M][words(K)], sw_row: [D][words(K)], gamma: [D].
+ * acc: [M][D] int32 or NULL; y: [M][D] fp32 (row stride D). */
+fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D, int64_t K,
+                          const float* gamma, int32_t* acc, float* y, void* stream);
+
+/* ----------------------------------------------------------- gradient side */
+/* AGP on one grouping (Sec. 5.2): ranges of G = gy (.) gamma (gamma may be
+ * NULL), keep probabilities, masks, and stochastic rounding of the kept
+ * groups to `bits`-bit codes with scales S' and zero points Z'.
+ * g: [M, D] fp32 row-major.  group_axis 0 = sample groups (PSQ, stream 0 of
+ * the generator for rounding, 2 for masks), 1 = channels (PCQ, streams 1 / 3).
+ * ws: fqt1_workspace_size(0, ...) bytes. */
+fqt1_status fqt1_agp_quantize_grad(const float* g, int64_t M, int64_t D, int32_t group_axis, const float* gamma,
+                                   const fqt1_agp_params* p, fqt1_qgrad* out, void* ws, size_t ws_bytes,
+                                   int32_t* dev_status, void* stream);
+
+/* Sample-Channel joint Quantization (Sec. 5.3): both AGP branches of one
+ * gradient from a single range pass and a single quantization pass:
+ * psq groups rows (rows_per_group from p_sample), pcq groups columns. */
+fqt1_status fqt1_scq_quantize(const float* g, int64_t M, int64_t D, const float* gamma,
+                              const fqt1_agp_params* p_sample, const fqt1_agp_params* p_channel,
+                              fqt1_qgrad* psq, fqt1_qgrad* pcq, void* ws, size_t ws_bytes, int32_t* dev_status,
+                              void* stream);
+
+/* grad_input side of SCQ (Eq. 21 with Sec. 5.3's per-sample scales):
+ * acc[r, k] = sum_j q[r, j] sign(W)[j, k] over the kept rows r (kept order),
+ * dx[m, k] = S'_g acc + Z'_g colsum_w[k] for rows of kept groups, 0 for
+ * pruned rows.  sw_col: [K][words(D)]; colsum_w: [K] = sum_j sign(W)[j, k].
+ * acc: [capacity * rows_per_group][K] int32 or NULL; dx: [M][K] fp32 or NULL
+ * (a convolution passes acc and folds it with fqt1_col2im). */
+fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t* sw_col, const int32_t* colsum_w, int64_t M,
+                                int64_t D, int64_t K, const fqt1_agp_params* p, int32_t* acc, float* dx,
+                                void* stream);
+
+/* Folder of App. C on the integer accumulators, then dequantization:
+ * dx[n, c, h, w] = S'_n * sum(acc taps) + Z'_n * sum(colsum_w taps) over the
+ * taps of the unfolded matrix that read pixel (h, w); pruned samples get 0.
+ * acc: [capacity * Ho*Wo][K] from fqt1_bwd_input_gemm; dx: [N, C, H, W]. */
+fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, const int32_t* colsum_w, int32_t N, int32_t C,
+                        int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad, float* dx,
+                        void* stream);
+
+/* grad_weight side of SCQ (Eq. 21 with Sec. 5.3's per-channel scales):
+ * acc[c, k] = sum_m q^c[c, m] sign(X)[m, k] for kept channel slots c,
+ * dw[j, k] = S^c'_j acc + Z^c'_j colsum_x[k] for kept channels j, 0 for pruned.
+ * sx_col: [K][words(M)]; colsum_x: [K] = sum_m sign(X)[m, k];
+ * acc: [capacity][K] int32 (required: the integer result, also the reduction
+ * target); dw: [D][K] fp32. */
+fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_t* sx_col, const int32_t* colsum_x, int64_t M,
+                                 int64_t D, int64_t K, const fqt1_agp_params* p, int32_t* acc, float* dw,
+                                 void* ws, size_t ws_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FQT1_H */

@@ -74,10 +74,12 @@ def int_matmul(a, b_t):
 def forward(x_u, w, gamma):
     """Binarized forward of a fully connected layer (Sec. 5.1).
 
-    x_u [M, K] fp32, w [D, K] fp32, gamma [D] fp32.
+    x_u [M, K] fp32, w [D, K] fp32, gamma [D] fp32 (None: Gamma = 1).
     Returns (acc int64 [M, D] = sign(x_u) sign(w)^T, y fp32 = gamma_j * acc).
     """
     acc = int_matmul(sign(x_u), sign(w))
+    if gamma is None:  # no Gamma: unit scale
+        return acc, acc.astype(f32)
     y = (np.asarray(gamma, dtype=f32)[None, :] * acc.astype(f32)).astype(f32)
     return acc, y
 

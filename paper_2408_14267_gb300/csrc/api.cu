@@ -1,0 +1,173 @@
+// C-ABI entry points of the GEMM side, dequantization and the Folder, plus helpers.
+#include <stdio.h>
+
+#include <atomic>
+
+#include "gemm.cuh"
+
+static thread_local char g_last_error[256] = "no error";
+
+void fqt1_set_cuda_error(cudaError_t e) {
+  snprintf(g_last_error, sizeof(g_last_error), "%s: %s", cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+extern "C" const char* fqt1_last_cuda_error(void) { return g_last_error; }
+
+static std::atomic<int64_t> g_launches{0};
+void fqt1_count_launches(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+extern "C" int64_t fqt1_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
+
+extern "C" int64_t fqt1_packed_words(int64_t n) { return n < 1 ? 0 : (((n + 31) / 32 + 3) / 4) * 4; }
+
+extern "C" int64_t fqt1_kept_capacity(int64_t n, int32_t bits, int32_t mode) {
+  if (n < 1 || bits < 1) return 0;
+  if (bits == 1 || mode == FQT1_SEL_BERNOULLI) return n;
+  return (n + bits - 1) / bits;
+}
+
+extern "C" int64_t fqt1_codes_ld(int64_t n) { return n < 1 ? 0 : ((n + 15) / 16) * 16; }
+
+namespace fqt1 {
+
+// out[m, k] = S'_slot * acc[row(m), k] + Z'_slot * cs[k] for rows m of kept groups, 0 otherwise
+// (fp32 multiply, multiply, add; no contraction).  Used for dx (groups of rpg rows) and dw (rpg = 1).
+__global__ void dequant_rows_kernel(const int32_t* __restrict__ acc, int64_t ldacc,
+                                    const int32_t* __restrict__ slot_of_group, const float* __restrict__ scale,
+                                    const float* __restrict__ zero, const int32_t* __restrict__ cs, int64_t M,
+                                    int64_t K, int64_t rpg, float* __restrict__ out) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= M * K) return;
+  const int64_t m = idx / K, k = idx - (idx / K) * K;
+  const int64_t g = m / rpg;
+  const int32_t sl = __ldg(slot_of_group + g);
+  float v = 0.0f;
+  if (sl >= 0) {
+    const int32_t a = __ldg(acc + ((int64_t)sl * rpg + (m - g * rpg)) * ldacc + k);
+    v = __fadd_rn(__fmul_rn(__ldg(scale + sl), __int2float_rn(a)), __fmul_rn(__ldg(zero + sl), __int2float_rn(__ldg(cs + k))));
+  }
+  out[idx] = v;
+}
+
+// Folder of App. C on int32 accumulators + dequantization per sample.
+__global__ void col2im_kernel(const int32_t* __restrict__ acc, const int32_t* __restrict__ slot_of_group,
+                              const float* __restrict__ scale, const float* __restrict__ zero,
+                              const int32_t* __restrict__ cs, int N, int C, int H, int W, int kh, int kw, int stride,
+                              int pad, int Ho, int Wo, float* __restrict__ dx) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t total = (int64_t)N * C * H * W;
+  if (idx >= total) return;
+  const int w = (int)(idx % W);
+  const int h = (int)((idx / W) % H);
+  const int c = (int)((idx / ((int64_t)W * H)) % C);
+  const int n = (int)(idx / ((int64_t)W * H * C));
+  const int32_t sl = __ldg(slot_of_group + n);
+  float v = 0.0f;
+  if (sl >= 0) {
+    const int64_t K = (int64_t)C * kh * kw;
+    const int64_t rbase = (int64_t)sl * Ho * Wo;
+    int32_t a = 0, s = 0;
+    for (int i = 0; i < kh; ++i) {
+      const int hn = h + pad - i;
+      if (hn < 0 || hn % stride) continue;
+      const int oh = hn / stride;
+      if (oh >= Ho) continue;
+      for (int j = 0; j < kw; ++j) {
+        const int wn = w + pad - j;
+        if (wn < 0 || wn % stride) continue;
+        const int ow = wn / stride;
+        if (ow >= Wo) continue;
+        const int64_t k = ((int64_t)c * kh + i) * kw + j;
+        a += __ldg(acc + (rbase + (int64_t)oh * Wo + ow) * K + k);
+        s += __ldg(cs + k);
+      }
+    }
+    v = __fadd_rn(__fmul_rn(__ldg(scale + sl), __int2float_rn(a)), __fmul_rn(__ldg(zero + sl), __int2float_rn(s)));
+  }
+  dx[idx] = v;
+}
+
+}  // namespace fqt1
+
+using namespace fqt1;
+
+static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+static bool valid_bits(int b) { return b == 1 || b == 2 || b == 4 || b == 8; }
+
+extern "C" fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D,
+                                     int64_t K, const float* gamma, int32_t* acc, float* y, void* stream) {
+  if (!sx_row || !sw_row || M < 1 || D < 1 || K < 1 || (!acc && !y) || (y && !gamma)) return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(sx_row) || !aligned16(sw_row) || (acc && !aligned16(acc)) || (y && !aligned16(y)) ||
+      (gamma && !aligned16(gamma)))
+    return FQT1_ERR_MISALIGNED;
+  if (K >= (1ll << 24) || (M + 63) / 64 > 65535) return FQT1_ERR_UNSUPPORTED;
+  FQT1_CUDA_TRY(launch_xnor_gemm_simt(sx_row, sw_row, M, D, K, gamma, acc, y, (cudaStream_t)stream));
+  return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t* sw_col, const int32_t* colsum_w,
+                                           int64_t M, int64_t D, int64_t K, const fqt1_agp_params* p,
+                                           int32_t* acc, float* dx, void* stream) {
+  if (!psq || !sw_col || !p || M < 1 || D < 1 || K < 1 || (!acc && !dx)) return FQT1_ERR_INVALID_ARG;
+  if (!valid_bits(p->bits) || p->rows_per_group < 1 || M % p->rows_per_group) return FQT1_ERR_INVALID_ARG;
+  if (dx && !colsum_w) return FQT1_ERR_INVALID_ARG;
+  if (!psq->codes || !psq->kept_count || !psq->slot_of_group || !psq->scale || !psq->zero ||
+      psq->ld_codes < fqt1_codes_ld(D) || psq->ld_codes % 16)
+    return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(sw_col) || (acc && !aligned16(acc)) || (dx && !aligned16(dx))) return FQT1_ERR_MISALIGNED;
+  const int64_t rpg = p->rows_per_group;
+  const int64_t cap_rows = fqt1_kept_capacity(M / rpg, p->bits, p->mode) * rpg;
+  if ((cap_rows + 63) / 64 > 65535) return FQT1_ERR_UNSUPPORTED;
+  cudaStream_t s = (cudaStream_t)stream;
+  // The CUDA-core path needs the integer result in memory; a conv passes acc.
+  if (!acc) return FQT1_ERR_UNSUPPORTED;
+  FQT1_CUDA_TRY(launch_codes_gemm_simt(p->bits, psq->codes, psq->ld_codes, psq->kept_count, rpg, cap_rows, sw_col, K,
+                                       D, acc, K, s));
+  if (dx) {
+    const int64_t n = M * K;
+    dequant_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(acc, K, psq->slot_of_group, psq->scale,
+                                                                    psq->zero, colsum_w, M, K, rpg, dx);
+    fqt1_count_launches(1);
+    FQT1_CUDA_TRY(cudaGetLastError());
+  }
+  return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, const int32_t* colsum_w, int32_t N,
+                                   int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,
+                                   int32_t pad, float* dx, void* stream) {
+  if (!acc || !psq || !colsum_w || !dx || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 ||
+      pad < 0)
+    return FQT1_ERR_INVALID_ARG;
+  if (!psq->slot_of_group || !psq->scale || !psq->zero) return FQT1_ERR_INVALID_ARG;
+  const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
+  if (H + 2 * pad < kh || W + 2 * pad < kw) return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(acc) || !aligned16(dx)) return FQT1_ERR_MISALIGNED;
+  const int64_t n = (int64_t)N * C * H * W;
+  col2im_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(
+      acc, psq->slot_of_group, psq->scale, psq->zero, colsum_w, N, C, H, W, kh, kw, stride, pad, Ho, Wo, dx);
+  fqt1_count_launches(1);
+  FQT1_CUDA_TRY(cudaGetLastError());
+  return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_t* sx_col, const int32_t* colsum_x,
+                                            int64_t M, int64_t D, int64_t K, const fqt1_agp_params* p, int32_t* acc,
+                                            float* dw, void* ws, size_t ws_bytes, void* stream) {
+  (void)ws; (void)ws_bytes;
+  if (!pcq || !sx_col || !colsum_x || !p || !acc || !dw || M < 1 || D < 1 || K < 1) return FQT1_ERR_INVALID_ARG;
+  if (!valid_bits(p->bits)) return FQT1_ERR_INVALID_ARG;
+  if (!pcq->codes || !pcq->kept_count || !pcq->slot_of_group || !pcq->scale || !pcq->zero ||
+      pcq->ld_codes < fqt1_codes_ld(M) || pcq->ld_codes % 16)
+    return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(sx_col) || !aligned16(acc) || !aligned16(dw) || !aligned16(colsum_x)) return FQT1_ERR_MISALIGNED;
+  const int64_t cap = fqt1_kept_capacity(D, p->bits, p->mode);
+  cudaStream_t s = (cudaStream_t)stream;
+  FQT1_CUDA_TRY(launch_codes_gemm_simt(p->bits, pcq->codes, pcq->ld_codes, pcq->kept_count, 1, cap, sx_col, K, M, acc,
+                                       K, s));
+  const int64_t n = D * K;
+  dequant_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(acc, K, pcq->slot_of_group, pcq->scale, pcq->zero,
+                                                                  colsum_x, D, K, 1, dw);
+  fqt1_count_launches(1);
+  FQT1_CUDA_TRY(cudaGetLastError());
+  return FQT1_OK;
+}

@@ -1,0 +1,572 @@
+// AGP + SCQ gradient quantization (Sec. 3.2, 5.2, 5.3).
+//
+//   range_kernel     one read of G = gY (.) gamma: per-sample-group and per-channel
+//                    min / max through order-preserving integer atomics (exact).
+//   select_kernel    one CTA per grouping: fixed-point ranges, water-filled keep
+//                    probabilities, masks, kept list, scales S' and zero points Z'.
+//   quantize_kernel  second read of G: stochastic rounding of the kept sample
+//                    groups (PSQ codes, row-major) and kept channels (PCQ codes,
+//                    written transposed through shared memory).
+#include "common.cuh"
+
+namespace fqt1 {
+
+// ------------------------------------------------------------------ ranges
+constexpr int kRangeRows = 64, kRangeCols = 128;
+
+struct RangeArgs {
+  const float* g;
+  const float* gamma;
+  int64_t M, D, rpg;
+  uint32_t *smin, *smax;  // [M / rpg] or null
+  uint32_t *cmin, *cmax;  // [D] or null
+  int32_t* dev_status;
+};
+
+template <bool VEC>
+__global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
+  __shared__ uint32_t cmin_s[8][kRangeCols], cmax_s[8][kRangeCols];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t c0 = (int64_t)blockIdx.x * kRangeCols + lane * 4;
+  const int64_t r0 = (int64_t)blockIdx.y * kRangeRows + warp * 8;
+  float gam[4];
+  bool cv[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    cv[q] = c0 + q < a.D;
+    gam[q] = (a.gamma && cv[q]) ? __ldg(a.gamma + c0 + q) : 1.0f;
+  }
+  uint32_t colmin[4] = {0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu}, colmax[4] = {0u, 0u, 0u, 0u};
+  uint32_t gmin = 0xFFFFFFFFu, gmax = 0u;
+  int64_t cur = -1;
+  bool bad = false;
+  for (int i = 0; i < 8; ++i) {
+    const int64_t r = r0 + i;
+    if (r >= a.M) break;
+    const int64_t gi = r / a.rpg;
+    if (a.smin && gi != cur) {
+      if (cur >= 0) {
+        const uint32_t mn = __reduce_min_sync(0xFFFFFFFFu, gmin), mx = __reduce_max_sync(0xFFFFFFFFu, gmax);
+        if (lane == 0) { atomicMin(a.smin + cur, mn); atomicMax(a.smax + cur, mx); }
+      }
+      cur = gi;
+      gmin = 0xFFFFFFFFu;
+      gmax = 0u;
+    }
+    float v[4];
+    if (VEC) {
+      if (cv[0]) {
+        const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + c0));
+        v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+      }
+    } else {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) v[q] = cv[q] ? __ldg(a.g + r * a.D + c0 + q) : 0.0f;
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (!cv[q]) continue;
+      const float x = a.gamma ? __fmul_rn(v[q], gam[q]) : v[q];
+      bad |= !isfinite(x);
+      const uint32_t k = float_to_ordered(x);
+      colmin[q] = min(colmin[q], k);
+      colmax[q] = max(colmax[q], k);
+      gmin = min(gmin, k);
+      gmax = max(gmax, k);
+    }
+  }
+  if (a.smin && cur >= 0) {
+    const uint32_t mn = __reduce_min_sync(0xFFFFFFFFu, gmin), mx = __reduce_max_sync(0xFFFFFFFFu, gmax);
+    if (lane == 0) { atomicMin(a.smin + cur, mn); atomicMax(a.smax + cur, mx); }
+  }
+  if (__any_sync(0xFFFFFFFFu, bad) && lane == 0) atomicOr(a.dev_status, FQT1_DEV_NONFINITE);
+  if (a.cmin) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      cmin_s[warp][lane * 4 + q] = colmin[q];
+      cmax_s[warp][lane * 4 + q] = colmax[q];
+    }
+    __syncthreads();
+    if (threadIdx.x < kRangeCols) {
+      const int64_t c = (int64_t)blockIdx.x * kRangeCols + threadIdx.x;
+      uint32_t mn = 0xFFFFFFFFu, mx = 0u;
+#pragma unroll
+      for (int w = 0; w < 8; ++w) { mn = min(mn, cmin_s[w][threadIdx.x]); mx = max(mx, cmax_s[w][threadIdx.x]); }
+      if (c < a.D && mx != 0u) { atomicMin(a.cmin + c, mn); atomicMax(a.cmax + c, mx); }
+    }
+  }
+}
+
+// --------------------------------------------------------------- selection
+struct SelectArgs {
+  const uint32_t* kmin;
+  const uint32_t* kmax;
+  int32_t n, bits, mode, capacity;
+  uint64_t seed;
+  uint32_t stream;
+  fqt1_qgrad out;
+};
+
+constexpr int kSelThreads = 1024;
+
+// Inclusive scan of one uint64 per thread across the CTA; returns the inclusive value
+// and writes the CTA total to *total.
+__device__ uint64_t block_inclusive_scan(uint64_t v, uint64_t* warp_sums, uint64_t* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint64_t t = __shfl_up_sync(0xFFFFFFFFu, v, o);
+    if (lane >= o) v += t;
+  }
+  if (lane == 31) warp_sums[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    uint64_t s = warp_sums[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint64_t t = __shfl_up_sync(0xFFFFFFFFu, s, o);
+      if (lane >= o) s += t;
+    }
+    warp_sums[lane] = s;
+  }
+  __syncthreads();
+  if (warp > 0) v += warp_sums[warp - 1];
+  const uint64_t tot = warp_sums[31];
+  __syncthreads();
+  *total = tot;
+  return v;
+}
+
+// floor(a * 2^32 / d) for a <= d < 2^60 by base-16 long division (exact).
+__device__ __forceinline__ uint64_t div_shift32(uint64_t a, uint64_t d) {
+  uint64_t q = a / d, r = a % d;
+#pragma unroll
+  for (int s = 0; s < 8; ++s) {
+    r <<= 4;
+    q = (q << 4) | (r / d);
+    r %= d;
+  }
+  return q;
+}
+
+__global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, SelectArgs a1) {
+  const SelectArgs& a = blockIdx.x == 0 ? a0 : a1;
+  extern __shared__ __align__(16) unsigned char sel_smem[];
+  __shared__ uint64_t warp_sums[32];
+  __shared__ uint32_t s_rmax;
+  __shared__ int s_tstar;
+  __shared__ uint64_t s_kth, s_stot;
+  const int n = a.n, tid = threadIdx.x;
+  if (n <= 0) return;
+  int npad = 1;
+  while (npad < n) npad <<= 1;
+  uint64_t* key = reinterpret_cast<uint64_t*>(sel_smem);           // [npad] sort keys, later P
+  float* rf = reinterpret_cast<float*>(sel_smem + 8 * (size_t)npad);  // [n] ranges
+  const fqt1_qgrad& o = a.out;
+
+  // Z = min, R = max - min (fp32)
+  if (tid == 0) s_rmax = 0u;
+  __syncthreads();
+  for (int i = tid; i < n; i += kSelThreads) {
+    const float z = ordered_to_float(a.kmin[i]);
+    const float r = __fsub_rn(ordered_to_float(a.kmax[i]), z);
+    o.group_min[i] = z;
+    o.group_range[i] = r;
+    rf[i] = r;
+    if (r > 0.0f) atomicMax(&s_rmax, __float_as_uint(r));
+  }
+  __syncthreads();
+  const float rmax = __uint_as_float(s_rmax);
+  const uint64_t two32 = 1ull << 32;
+
+  // Fixed-point ranges R~ = floor(R 2^(40 - E)), 2^(E-1) <= max R < 2^E.
+  int e = 0;
+  if (rmax > 0.0f) frexpf(rmax, &e);
+  const double fx = ldexp(1.0, kFixedPointBits - e);
+  auto rtilde = [&](int i) -> uint64_t {
+    const float r = rf[i];
+    return (rmax > 0.0f && r > 0.0f) ? (uint64_t)floor((double)r * fx) : 0ull;
+  };
+
+  if (a.bits > 1) {
+    // sort keys (R~ desc, index asc) descending
+    for (int i = tid; i < npad; i += kSelThreads)
+      key[i] = i < n ? ((rtilde(i) << 24) | (uint64_t)(0xFFFFFFu - (uint32_t)i)) : 0ull;
+    __syncthreads();
+    for (int size = 2; size <= npad; size <<= 1) {
+      for (int stride = size >> 1; stride > 0; stride >>= 1) {
+        for (int i = tid; i < npad / 2; i += kSelThreads) {
+          const int lo = 2 * i - (i & (stride - 1));
+          const int hi = lo + stride;
+          const bool desc = (lo & size) == 0;
+          const uint64_t x = key[lo], y = key[hi];
+          if ((x < y) == desc) { key[lo] = y; key[hi] = x; }
+        }
+        __syncthreads();
+      }
+    }
+    if (a.mode == FQT1_SEL_TOPK) {
+      const int k = max(1, n / a.bits);
+      if (tid == 0) { s_kth = key[k - 1]; s_tstar = k; s_stot = 0; }
+    } else {
+      // suffix sums S_t over sorted positions; t* = first t with (n - b t) R~_(t) <= b S_t
+      const int per = (npad + kSelThreads - 1) / kSelThreads;
+      const int beg = min(npad, tid * per), end = min(npad, beg + per);
+      uint64_t local = 0;
+      for (int t = beg; t < end; ++t) local += key[t] >> 24;
+      // suffix of thread chunks: scan reversed thread order
+      uint64_t total;
+      const uint64_t incl = block_inclusive_scan(local, warp_sums, &total);
+      uint64_t suffix = total - incl + local;  // sum of positions >= beg
+      int best = n;
+      uint64_t best_s = 0;
+      for (int t = beg; t < end && t < n; ++t) {
+        const uint64_t rt = key[t] >> 24;
+        const int64_t lhs = (int64_t)(n - a.bits * t) * (int64_t)rt;
+        const int64_t rhs = (int64_t)a.bits * (int64_t)suffix;
+        if (lhs <= rhs) { best = t; best_s = suffix; break; }
+        suffix -= rt;
+      }
+      if (tid == 0) s_tstar = n;
+      __syncthreads();
+      atomicMin(&s_tstar, best);
+      __syncthreads();
+      if (best == s_tstar && best < n) { s_stot = best_s; s_kth = key[best]; }
+      if (tid == 0 && s_tstar >= n) { s_stot = 0; s_kth = 0; }
+    }
+    __syncthreads();
+    // P_i by group index (reuses the key buffer)
+    const int tstar = s_tstar;
+    const uint64_t kth = s_kth, S = s_stot;
+    for (int i = tid; i < n; i += kSelThreads) {
+      const uint64_t rt = rtilde(i);
+      const uint64_t ki = (rt << 24) | (uint64_t)(0xFFFFFFu - (uint32_t)i);
+      uint64_t P;
+      if (a.mode == FQT1_SEL_TOPK) {
+        P = ki >= kth ? two32 : 0ull;
+      } else if (ki > kth) {
+        P = two32;
+      } else if (S > 0) {
+        const uint64_t num = (uint64_t)(n - a.bits * tstar) * rt;
+        P = min(two32, div_shift32(num, (uint64_t)a.bits * S));
+      } else {
+        P = 0;
+      }
+      key[i] = P;
+    }
+  } else {
+    for (int i = tid; i < n; i += kSelThreads) key[i] = two32;
+  }
+  __syncthreads();
+
+  // masks in index order; each thread owns a contiguous chunk
+  const int per = (n + kSelThreads - 1) / kSelThreads;
+  const int beg = min(n, tid * per), end = min(n, beg + per);
+  uint64_t psum = 0;
+  for (int i = beg; i < end; ++i) psum += key[i];
+  uint64_t total;
+  const uint64_t pincl = block_inclusive_scan(psum, warp_sums, &total);
+  uint64_t c = pincl - psum;
+  uint64_t u = 0;
+  if (a.bits > 1 && a.mode == FQT1_SEL_SYSTEMATIC) u = philox_word(a.seed, a.stream, 0);
+  c += u;
+  uint32_t kept_bits = 0;  // chunk length <= 16 for n <= 16384
+  int nk = 0;
+  for (int i = beg; i < end; ++i) {
+    const uint64_t P = key[i];
+    bool kept;
+    if (a.bits == 1) kept = true;
+    else if (a.mode == FQT1_SEL_SYSTEMATIC) kept = ((c + P) >> 32) > (c >> 32);
+    else if (a.mode == FQT1_SEL_BERNOULLI) kept = (uint64_t)philox_word(a.seed, a.stream, (uint64_t)i) < P;
+    else kept = P == two32;
+    c += P;
+    if (kept) { kept_bits |= 1u << (i - beg); ++nk; }
+  }
+  uint64_t ktot;
+  const uint64_t kincl = block_inclusive_scan((uint64_t)nk, warp_sums, &ktot);
+  int slot = (int)(kincl - nk);
+  const double Bd = (double)((1 << a.bits) - 1);
+  for (int i = beg; i < end; ++i) {
+    const uint64_t P = key[i];
+    const double ph = (double)P * 2.3283064365386963e-10;  // 2^-32, exact
+    o.p_hat[i] = ph;
+    if (kept_bits & (1u << (i - beg))) {
+      o.slot_of_group[i] = slot;
+      o.kept_idx[slot] = i;
+      o.scale[slot] = __double2float_rn(__ddiv_rn((double)rf[i], __dmul_rn(Bd, ph)));
+      o.zero[slot] = __double2float_rn(__ddiv_rn((double)o.group_min[i], ph));
+      ++slot;
+    } else {
+      o.slot_of_group[i] = -1;
+    }
+  }
+  for (int s = (int)ktot + tid; s < a.capacity; s += kSelThreads) o.kept_idx[s] = -1;
+  if (tid == 0) *o.kept_count = (int32_t)ktot;
+}
+
+// --------------------------------------------------------------- quantize
+constexpr int kQRows = 32, kQCols = 128;
+
+struct QBranch {
+  const float* zmin;     // [n] group minima
+  const float* range;    // [n] group ranges
+  const int32_t* slot;   // [n] slot or -1
+  uint8_t* codes;
+  int64_t ld;
+  float B;
+  uint64_t seed;
+};
+
+struct QuantArgs {
+  const float* g;
+  const float* gamma;
+  int64_t M, D, rpg;
+  int do_psq, do_pcq;
+  QBranch s, c;
+};
+
+template <bool VEC>
+__global__ void __launch_bounds__(256) quantize_kernel(QuantArgs a) {
+  __shared__ uint32_t tile[kQCols][kQRows / 4 + 1];  // PCQ codes, 4 rows per word
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t cb = (int64_t)blockIdx.x * kQCols;
+  const int64_t c0 = cb + lane * 4;
+  const int64_t r0 = (int64_t)blockIdx.y * kQRows;
+  float gam[4], zc[4], invc[4];
+  int32_t cslot[4];
+  bool cdeg[4], cv[4];
+  bool any_c = false;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int64_t c = c0 + q;
+    cv[q] = c < a.D;
+    gam[q] = (a.gamma && cv[q]) ? __ldg(a.gamma + c) : 1.0f;
+    cslot[q] = (a.do_pcq && cv[q]) ? __ldg(a.c.slot + c) : -1;
+    zc[q] = 0.f; invc[q] = 0.f; cdeg[q] = true;
+    if (cslot[q] >= 0) {
+      const float r = __ldg(a.c.range + c);
+      zc[q] = __ldg(a.c.zmin + c);
+      invc[q] = __fdiv_rn(a.c.B, r);
+      cdeg[q] = !(r > 0.0f) || !isfinite(invc[q]);
+      any_c = true;
+    }
+  }
+  uint8_t ccode[4][4] = {};  // [row i][col q]
+  for (int i = 0; i < 4; ++i) {
+    const int64_t r = r0 + warp * 4 + i;
+    if (r >= a.M) break;
+    int32_t sslot = -1;
+    int64_t gi = 0;
+    if (a.do_psq) {
+      gi = r / a.rpg;
+      sslot = __ldg(a.s.slot + gi);
+    }
+    if (sslot < 0 && !any_c) continue;
+    float v[4];
+    if (VEC) {
+      if (cv[0]) {
+        const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + c0));
+        v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+      } else {
+        v[0] = v[1] = v[2] = v[3] = 0.f;
+      }
+    } else {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) v[q] = cv[q] ? __ldg(a.g + r * a.D + c0 + q) : 0.0f;
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) v[q] = a.gamma ? __fmul_rn(v[q], gam[q]) : v[q];
+    const uint64_t e0 = (uint64_t)r * (uint64_t)a.D + (uint64_t)c0;
+    if (sslot >= 0) {
+      const float rs = __ldg(a.s.range + gi), zs = __ldg(a.s.zmin + gi);
+      const float inv = __fdiv_rn(a.s.B, rs);
+      const bool deg = !(rs > 0.0f) || !isfinite(inv);
+      uint32_t w[4];
+      if (VEC) {
+        const U32x4 p = philox_block(a.s.seed, kStreamSrPsq, e0 >> 2);
+        w[0] = p.x; w[1] = p.y; w[2] = p.z; w[3] = p.w;
+      } else {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) w[q] = philox_word(a.s.seed, kStreamSrPsq, e0 + q);
+      }
+      uint8_t* dst = a.s.codes + ((int64_t)sslot * a.rpg + (r - gi * a.rpg)) * a.s.ld + c0;
+      if (VEC) {
+        if (cv[0]) {
+          uint32_t packed = 0;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) packed |= sr_code(v[q], zs, inv, a.s.B, deg, w[q]) << (8 * q);
+          *reinterpret_cast<uint32_t*>(dst) = packed;
+        }
+      } else {
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          if (cv[q]) dst[q] = (uint8_t)sr_code(v[q], zs, inv, a.s.B, deg, w[q]);
+      }
+    }
+    if (any_c) {
+      uint32_t w[4];
+      if (VEC) {
+        const U32x4 p = philox_block(a.c.seed, kStreamSrPcq, e0 >> 2);
+        w[0] = p.x; w[1] = p.y; w[2] = p.z; w[3] = p.w;
+      } else {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) w[q] = cslot[q] >= 0 ? philox_word(a.c.seed, kStreamSrPcq, e0 + q) : 0u;
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        if (cslot[q] >= 0) ccode[i][q] = (uint8_t)sr_code(v[q], zc[q], invc[q], a.c.B, cdeg[q], w[q]);
+    }
+  }
+  if (!a.do_pcq) return;
+  // rows warp*4 .. warp*4+3 of each of this lane's columns form one 32-bit word
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint32_t word = (uint32_t)ccode[0][q] | ((uint32_t)ccode[1][q] << 8) | ((uint32_t)ccode[2][q] << 16) |
+                          ((uint32_t)ccode[3][q] << 24);
+    tile[lane * 4 + q][warp] = word;
+  }
+  __syncthreads();
+  // each kept column of the tile: 32 code bytes (rows r0 .. r0+31) -> 2 x 16 bytes
+  const int col = threadIdx.x >> 1, half = threadIdx.x & 1;
+  const int64_t c = cb + col;
+  if (c < a.D) {
+    const int32_t sl = __ldg(a.c.slot + c);
+    const int64_t rb = r0 + 16 * half;
+    if (sl >= 0 && rb < a.M && rb + 16 <= a.c.ld) {
+      uint4 val;
+      val.x = tile[col][4 * half + 0];
+      val.y = tile[col][4 * half + 1];
+      val.z = tile[col][4 * half + 2];
+      val.w = tile[col][4 * half + 3];
+      *reinterpret_cast<uint4*>(a.c.codes + (int64_t)sl * a.c.ld + rb) = val;
+    }
+  }
+}
+
+}  // namespace fqt1
+
+using namespace fqt1;
+
+static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+static bool valid_params(const fqt1_agp_params* p) {
+  return p && (p->bits == 1 || p->bits == 2 || p->bits == 4 || p->bits == 8) && p->mode >= 0 && p->mode <= 2;
+}
+
+static bool valid_qgrad(const fqt1_qgrad* q, int64_t min_ld) {
+  return q && q->group_min && q->group_range && q->p_hat && q->slot_of_group && q->kept_idx && q->kept_count &&
+         q->scale && q->zero && q->codes && q->ld_codes >= min_ld && q->ld_codes % 16 == 0 && aligned16(q->codes);
+}
+
+extern "C" size_t fqt1_workspace_size(int32_t which, int64_t M, int64_t D, int64_t K, int32_t rows_per_group) {
+  if (which == 0) {
+    const int64_t ns = rows_per_group > 0 ? M / rows_per_group : M;
+    return (size_t)(2 * ns + 2 * D) * sizeof(uint32_t);
+  }
+  (void)K;
+  return 0;
+}
+
+// Shared driver of both entry points.
+static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const float* gamma,
+                                 const fqt1_agp_params* ps, fqt1_qgrad* psq, const fqt1_agp_params* pc,
+                                 fqt1_qgrad* pcq, void* ws, size_t ws_bytes, int32_t* dev_status, cudaStream_t s) {
+  if (!g || M < 1 || D < 1 || !dev_status) return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(g) || (gamma && !aligned16(gamma))) return FQT1_ERR_MISALIGNED;
+  int64_t rpg = 1, ns = 0;
+  if (psq) {
+    if (!valid_params(ps) || ps->rows_per_group < 1 || M % ps->rows_per_group != 0) return FQT1_ERR_INVALID_ARG;
+    if (!valid_qgrad(psq, fqt1_codes_ld(D))) return FQT1_ERR_INVALID_ARG;
+    rpg = ps->rows_per_group;
+    ns = M / rpg;
+    if (ns > kMaxGroups) return FQT1_ERR_UNSUPPORTED;
+  }
+  if (pcq) {
+    if (!valid_params(pc) || !valid_qgrad(pcq, fqt1_codes_ld(M))) return FQT1_ERR_INVALID_ARG;
+    if (D > kMaxGroups) return FQT1_ERR_UNSUPPORTED;
+  }
+  const size_t need = (size_t)(2 * ns + 2 * D) * sizeof(uint32_t);  // ns = 0 for a channel-only call
+  if (!ws || ws_bytes < need) return FQT1_ERR_WORKSPACE;
+  if (!aligned16(ws)) return FQT1_ERR_MISALIGNED;
+  if (M * D >= (1ll << 46)) return FQT1_ERR_UNSUPPORTED;
+  if ((M + kQRows - 1) / kQRows > 65535 || (M + kRangeRows - 1) / kRangeRows > 65535) return FQT1_ERR_UNSUPPORTED;
+
+  uint32_t* smin = static_cast<uint32_t*>(ws);
+  uint32_t* cmin = smin + ns;
+  uint32_t* smax = cmin + D;
+  uint32_t* cmax = smax + ns;
+  FQT1_CUDA_TRY(cudaMemsetAsync(smin, 0xFF, sizeof(uint32_t) * (ns + D), s));
+  FQT1_CUDA_TRY(cudaMemsetAsync(smax, 0x00, sizeof(uint32_t) * (ns + D), s));
+
+  const bool vec = (D % 4) == 0;
+  RangeArgs ra{g, gamma, M, D, rpg, psq ? smin : nullptr, psq ? smax : nullptr, pcq ? cmin : nullptr,
+               pcq ? cmax : nullptr, dev_status};
+  dim3 rgrid((unsigned)((D + kRangeCols - 1) / kRangeCols), (unsigned)((M + kRangeRows - 1) / kRangeRows));
+  if (vec) range_kernel<true><<<rgrid, 256, 0, s>>>(ra);
+  else range_kernel<false><<<rgrid, 256, 0, s>>>(ra);
+  fqt1_count_launches(1);
+  FQT1_CUDA_TRY(cudaGetLastError());
+
+  SelectArgs sa[2];
+  int nsel = 0;
+  int npad_max = 1;
+  auto add_sel = [&](const fqt1_agp_params* p, fqt1_qgrad* q, const uint32_t* kmin, const uint32_t* kmax, int n,
+                     uint32_t stream) {
+    SelectArgs x;
+    x.kmin = kmin; x.kmax = kmax; x.n = n; x.bits = p->bits; x.mode = p->mode;
+    x.capacity = (int32_t)fqt1_kept_capacity(n, p->bits, p->mode);
+    x.seed = p->seed; x.stream = stream; x.out = *q;
+    sa[nsel++] = x;
+    int np = 1;
+    while (np < n) np <<= 1;
+    npad_max = np > npad_max ? np : npad_max;
+  };
+  if (psq) add_sel(ps, psq, smin, smax, (int)ns, kStreamSelSample);
+  if (pcq) add_sel(pc, pcq, cmin, cmax, (int)D, kStreamSelChannel);
+  const size_t smem = (size_t)npad_max * 8 + (size_t)npad_max * 4;
+  static bool attr_done = false;
+  if (!attr_done) {
+    FQT1_CUDA_TRY(cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (size_t)kMaxGroups * 12));
+    attr_done = true;
+  }
+  select_kernel<<<nsel, kSelThreads, smem, s>>>(sa[0], nsel > 1 ? sa[1] : sa[0]);
+  fqt1_count_launches(1);
+  FQT1_CUDA_TRY(cudaGetLastError());
+
+  QuantArgs qa;
+  qa.g = g; qa.gamma = gamma; qa.M = M; qa.D = D; qa.rpg = rpg;
+  qa.do_psq = psq != nullptr;
+  qa.do_pcq = pcq != nullptr;
+  if (psq) qa.s = QBranch{psq->group_min, psq->group_range, psq->slot_of_group, psq->codes, psq->ld_codes,
+                          (float)((1 << ps->bits) - 1), ps->seed};
+  else qa.s = QBranch{};
+  if (pcq) qa.c = QBranch{pcq->group_min, pcq->group_range, pcq->slot_of_group, pcq->codes, pcq->ld_codes,
+                          (float)((1 << pc->bits) - 1), pc->seed};
+  else qa.c = QBranch{};
+  dim3 qgrid((unsigned)((D + kQCols - 1) / kQCols), (unsigned)((M + kQRows - 1) / kQRows));
+  if (vec) quantize_kernel<true><<<qgrid, 256, 0, s>>>(qa);
+  else quantize_kernel<false><<<qgrid, 256, 0, s>>>(qa);
+  fqt1_count_launches(1);
+  FQT1_CUDA_TRY(cudaGetLastError());
+  return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_agp_quantize_grad(const float* g, int64_t M, int64_t D, int32_t group_axis,
+                                              const float* gamma, const fqt1_agp_params* p, fqt1_qgrad* out,
+                                              void* ws, size_t ws_bytes, int32_t* dev_status, void* stream) {
+  if (group_axis == 0) return quantize_impl(g, M, D, gamma, p, out, nullptr, nullptr, ws, ws_bytes, dev_status,
+                                            (cudaStream_t)stream);
+  if (group_axis == 1) return quantize_impl(g, M, D, gamma, nullptr, nullptr, p, out, ws, ws_bytes, dev_status,
+                                            (cudaStream_t)stream);
+  return FQT1_ERR_INVALID_ARG;
+}
+
+extern "C" fqt1_status fqt1_scq_quantize(const float* g, int64_t M, int64_t D, const float* gamma,
+                                         const fqt1_agp_params* p_sample, const fqt1_agp_params* p_channel,
+                                         fqt1_qgrad* psq, fqt1_qgrad* pcq, void* ws, size_t ws_bytes,
+                                         int32_t* dev_status, void* stream) {
+  if (!psq || !pcq) return FQT1_ERR_INVALID_ARG;
+  return quantize_impl(g, M, D, gamma, p_sample, psq, p_channel, pcq, ws, ws_bytes, dev_status,
+                       (cudaStream_t)stream);
+}

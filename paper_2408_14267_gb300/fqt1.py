@@ -1,0 +1,185 @@
+"""ctypes binding of libfqt1 (argument marshalling only).
+
+Every function here forwards device pointers and sizes to the C-ABI entry
+point of the same name declared in include/fqt1.h; all arithmetic runs in the
+library's CUDA kernels.  PyTorch supplies device memory and streams.  There is
+no fallback: if libfqt1.so is missing or a call fails, an exception is raised.
+"""
+import ctypes as C
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libfqt1.so")
+
+SYSTEMATIC, BERNOULLI, TOPK = 0, 1, 2
+DEV_NONFINITE, DEV_TIMEOUT = 0x100, 0x200
+STATUS_NAMES = {0: "FQT1_OK", 1: "FQT1_ERR_INVALID_ARG", 2: "FQT1_ERR_MISALIGNED", 3: "FQT1_ERR_UNSUPPORTED",
+                4: "FQT1_ERR_WORKSPACE", 5: "FQT1_ERR_CUDA"}
+
+
+class AgpParams(C.Structure):
+    _fields_ = [("bits", C.c_int32), ("mode", C.c_int32), ("seed", C.c_uint64), ("rows_per_group", C.c_int64)]
+
+
+class QGrad(C.Structure):
+    _fields_ = [("group_min", C.c_void_p), ("group_range", C.c_void_p), ("p_hat", C.c_void_p),
+                ("slot_of_group", C.c_void_p), ("kept_idx", C.c_void_p), ("kept_count", C.c_void_p),
+                ("scale", C.c_void_p), ("zero", C.c_void_p), ("codes", C.c_void_p), ("ld_codes", C.c_int64)]
+
+
+class Fqt1Error(RuntimeError):
+    pass
+
+
+_lib = None
+_VP, _I64, _I32 = C.c_void_p, C.c_int64, C.c_int32
+_SIGS = {
+    "fqt1_packed_words": (_I64, [_I64]),
+    "fqt1_kept_capacity": (_I64, [_I64, _I32, _I32]),
+    "fqt1_codes_ld": (_I64, [_I64]),
+    "fqt1_workspace_size": (C.c_size_t, [_I32, _I64, _I64, _I64, _I32]),
+    "fqt1_last_cuda_error": (C.c_char_p, []),
+    "fqt1_kernel_launches": (_I64, []),
+    "fqt1_binarize_pack": (C.c_int, [_VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
+    "fqt1_im2col": (C.c_int, [_VP] + [_I32] * 8 + [_VP, _VP, _VP, _VP]),
+    "fqt1_fwd_gemm": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
+    "fqt1_agp_quantize_grad": (C.c_int, [_VP, _I64, _I64, _I32, _VP, _VP, _VP, _VP, C.c_size_t, _VP, _VP]),
+    "fqt1_scq_quantize": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, C.c_size_t, _VP, _VP]),
+    "fqt1_bwd_input_gemm": (C.c_int, [_VP, _VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
+    "fqt1_col2im": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
+    "fqt1_bwd_weight_gemm": (C.c_int, [_VP, _VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP, C.c_size_t, _VP]),
+}
+
+
+def lib():
+    """Load libfqt1.so (built by paper_2408_14267_gb300.build)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise Fqt1Error(f"{LIB_PATH} is missing: build it with paper_2408_14267_gb300.build.build()")
+        L = C.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def exported_names():
+    return list(_SIGS)
+
+
+def _check(status, name):
+    if status != 0:
+        msg = STATUS_NAMES.get(status, str(status))
+        if status == 5:
+            msg += " (" + lib().fqt1_last_cuda_error().decode() + ")"
+        raise Fqt1Error(f"{name} failed: {msg}")
+
+
+def _p(t):
+    """Device pointer of a CUDA tensor, or None."""
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise Fqt1Error("libfqt1 takes CUDA tensors only")
+    return t.data_ptr()
+
+
+def _s(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return C.c_void_p(stream.cuda_stream)
+
+
+# ----------------------------------------------------------------- helpers
+def packed_words(n):
+    return lib().fqt1_packed_words(n)
+
+
+def kept_capacity(n, bits, mode):
+    return lib().fqt1_kept_capacity(n, bits, mode)
+
+
+def codes_ld(n):
+    return lib().fqt1_codes_ld(n)
+
+
+def kernel_launches():
+    return lib().fqt1_kernel_launches()
+
+
+def workspace_size(which, M, D, K, rows_per_group):
+    return lib().fqt1_workspace_size(which, M, D, K, rows_per_group)
+
+
+# ------------------------------------------------------------ entry points
+def binarize_pack(x, rows, cols, ld, row_bits=None, col_bits=None, colsum=None, stream=None):
+    _check(lib().fqt1_binarize_pack(_p(x), rows, cols, ld, _p(row_bits), _p(col_bits), _p(colsum), _s(stream)),
+           "fqt1_binarize_pack")
+
+
+def im2col(x, N, Cin, H, W, kh, kw, stride, pad, row_bits=None, col_bits=None, colsum=None, stream=None):
+    _check(lib().fqt1_im2col(_p(x), N, Cin, H, W, kh, kw, stride, pad, _p(row_bits), _p(col_bits), _p(colsum),
+                             _s(stream)), "fqt1_im2col")
+
+
+def fwd_gemm(sx_row, sw_row, M, D, K, gamma, acc, y, stream=None):
+    _check(lib().fqt1_fwd_gemm(_p(sx_row), _p(sw_row), M, D, K, _p(gamma), _p(acc), _p(y), _s(stream)),
+           "fqt1_fwd_gemm")
+
+
+def agp_quantize_grad(g, M, D, group_axis, gamma, params, qgrad, ws, dev_status, stream=None):
+    _check(lib().fqt1_agp_quantize_grad(_p(g), M, D, group_axis, _p(gamma), C.byref(params), C.byref(qgrad.c),
+                                        _p(ws), ws.numel() * ws.element_size(), _p(dev_status), _s(stream)),
+           "fqt1_agp_quantize_grad")
+
+
+def scq_quantize(g, M, D, gamma, p_sample, p_channel, psq, pcq, ws, dev_status, stream=None):
+    _check(lib().fqt1_scq_quantize(_p(g), M, D, _p(gamma), C.byref(p_sample), C.byref(p_channel), C.byref(psq.c),
+                                   C.byref(pcq.c), _p(ws), ws.numel() * ws.element_size(), _p(dev_status),
+                                   _s(stream)), "fqt1_scq_quantize")
+
+
+def bwd_input_gemm(psq, sw_col, colsum_w, M, D, K, params, acc, dx, stream=None):
+    _check(lib().fqt1_bwd_input_gemm(C.byref(psq.c), _p(sw_col), _p(colsum_w), M, D, K, C.byref(params), _p(acc),
+                                     _p(dx), _s(stream)), "fqt1_bwd_input_gemm")
+
+
+def col2im(acc, psq, colsum_w, N, Cin, H, W, kh, kw, stride, pad, dx, stream=None):
+    _check(lib().fqt1_col2im(_p(acc), C.byref(psq.c), _p(colsum_w), N, Cin, H, W, kh, kw, stride, pad, _p(dx),
+                             _s(stream)), "fqt1_col2im")
+
+
+def bwd_weight_gemm(pcq, sx_col, colsum_x, M, D, K, params, acc, dw, ws=None, stream=None):
+    nbytes = 0 if ws is None else ws.numel() * ws.element_size()
+    _check(lib().fqt1_bwd_weight_gemm(C.byref(pcq.c), _p(sx_col), _p(colsum_x), M, D, K, C.byref(params), _p(acc),
+                                      _p(dw), _p(ws), nbytes, _s(stream)), "fqt1_bwd_weight_gemm")
+
+
+# --------------------------------------------------------- buffer holders
+class QGradBuffers:
+    """Device arrays of one fqt1_qgrad branch (n groups, `rows` code rows of `row_len` codes)."""
+
+    def __init__(self, n, capacity, code_rows, row_len, device="cuda"):
+        f = dict(device=device)
+        self.n, self.capacity = n, capacity
+        self.group_min = torch.empty(n, dtype=torch.float32, **f)
+        self.group_range = torch.empty(n, dtype=torch.float32, **f)
+        self.p_hat = torch.empty(n, dtype=torch.float64, **f)
+        self.slot_of_group = torch.empty(n, dtype=torch.int32, **f)
+        self.kept_idx = torch.empty(max(capacity, 1), dtype=torch.int32, **f)
+        self.kept_count = torch.zeros(4, dtype=torch.int32, **f)
+        self.scale = torch.empty(max(capacity, 1), dtype=torch.float32, **f)
+        self.zero = torch.empty(max(capacity, 1), dtype=torch.float32, **f)
+        self.ld = codes_ld(row_len)
+        self.codes = torch.zeros(max(code_rows, 1), self.ld, dtype=torch.uint8, **f)
+        self.c = QGrad(_p(self.group_min), _p(self.group_range), _p(self.p_hat), _p(self.slot_of_group),
+                       _p(self.kept_idx), _p(self.kept_count), _p(self.scale), _p(self.zero), _p(self.codes),
+                       self.ld)
+
+    def count(self):
+        return int(self.kept_count[0].item())

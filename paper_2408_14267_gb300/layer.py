@@ -1,0 +1,104 @@
+"""One fully quantized layer step through the C-ABI (App. C, Algorithm 1).
+
+`LayerStep` owns the device buffers of one linear or convolution layer and
+enqueues, on one CUDA stream and without host synchronisation:
+
+  forward : pack sign(W) (rows, columns, column sums); pack sign(X) or the
+            Unfolder of X fused with sign; binarized GEMM, y = Gamma * acc
+  backward: SCQ quantization of G = gY (.) Gamma (ranges, AGP selection,
+            stochastic rounding of both branches); grad_input GEMM (PSQ side)
+            then, for a convolution, the Folder; grad_weight GEMM (PCQ side)
+
+All arithmetic runs in libfqt1's kernels; this module only allocates and
+passes pointers.  The weight update (Algorithm 1's last step) is not part of
+the layer step.
+"""
+import numpy as np
+import torch
+
+from . import fqt1
+
+
+def conv_out_hw(H, W, kh, kw, stride, pad):
+    return (H + 2 * pad - kh) // stride + 1, (W + 2 * pad - kw) // stride + 1
+
+
+class LayerStep:
+    def __init__(self, wl, device="cuda"):
+        dev = torch.device(device)
+        self.kind = wl["kind"]
+        f32 = dict(dtype=torch.float32, device=dev)
+        i32 = dict(dtype=torch.int32, device=dev)
+        self.x = torch.as_tensor(np.ascontiguousarray(wl["x"]), **f32)
+        self.w = torch.as_tensor(np.ascontiguousarray(wl["w"]), **f32)
+        self.gamma = None if wl.get("gamma") is None else torch.as_tensor(wl["gamma"], **f32)
+        self.gy = torch.as_tensor(np.ascontiguousarray(wl["gy"]), **f32)
+        if self.kind == "conv":
+            N, Cin, H, W = self.x.shape
+            D, _, kh, kw = self.w.shape
+            self.stride, self.pad = wl["stride"], wl["pad"]
+            Ho, Wo = conv_out_hw(H, W, kh, kw, self.stride, self.pad)
+            self.conv = (N, Cin, H, W, kh, kw)
+            M, K, rpg = N * Ho * Wo, Cin * kh * kw, Ho * Wo
+        else:
+            M, K = self.x.shape
+            D = self.w.shape[0]
+            rpg = wl.get("rows_per_group", 1)
+        self.M, self.K, self.D, self.rpg = M, K, D, rpg
+        wK, wM, wD = fqt1.packed_words(K), fqt1.packed_words(M), fqt1.packed_words(D)
+        self.sx_row = torch.empty(M, wK, **i32)
+        self.sx_col = torch.empty(K, wM, **i32)
+        self.cs_x = torch.empty(K, **i32)
+        self.sw_row = torch.empty(D, wK, **i32)
+        self.sw_col = torch.empty(K, wD, **i32)
+        self.cs_w = torch.empty(K, **i32)
+        self.acc_y = torch.empty(M, D, **i32)
+        # without a Gamma the forward uses unit scales and G = gY
+        self.gamma_fwd = self.gamma if self.gamma is not None else torch.ones(D, **f32)
+        self.y = torch.empty(M, D, **f32)
+        self.p_s = fqt1.AgpParams(wl["bits_s"], wl["mode_s"], wl["seed_s"], rpg)
+        self.p_c = fqt1.AgpParams(wl["bits_c"], wl["mode_c"], wl["seed_c"], 1)
+        n_s = M // rpg
+        self.cap_s = fqt1.kept_capacity(n_s, wl["bits_s"], wl["mode_s"])
+        self.cap_c = fqt1.kept_capacity(D, wl["bits_c"], wl["mode_c"])
+        self.psq = fqt1.QGradBuffers(n_s, self.cap_s, self.cap_s * rpg, D, dev)
+        self.pcq = fqt1.QGradBuffers(D, self.cap_c, self.cap_c, M, dev)
+        self.ws = torch.empty(fqt1.workspace_size(0, M, D, K, rpg), dtype=torch.uint8, device=dev)
+        self.dev_status = torch.zeros(4, **i32)
+        self.acc_dx = torch.empty(max(self.cap_s * rpg, 1), K, **i32)
+        self.dx = torch.empty(*(self.x.shape), **f32)
+        self.acc_dw = torch.empty(max(self.cap_c, 1), K, **i32)
+        self.dw = torch.empty(D, K, **f32)
+
+    # dense-equivalent operations of one step: forward, grad_input and grad_weight products
+    def dense_ops(self):
+        return 6.0 * self.M * self.K * self.D
+
+    def forward(self, stream=None):
+        fqt1.binarize_pack(self.w, self.D, self.K, self.K, self.sw_row, self.sw_col, self.cs_w, stream)
+        if self.kind == "conv":
+            N, Cin, H, W, kh, kw = self.conv
+            fqt1.im2col(self.x, N, Cin, H, W, kh, kw, self.stride, self.pad, self.sx_row, self.sx_col, self.cs_x,
+                        stream)
+        else:
+            fqt1.binarize_pack(self.x, self.M, self.K, self.K, self.sx_row, self.sx_col, self.cs_x, stream)
+        fqt1.fwd_gemm(self.sx_row, self.sw_row, self.M, self.D, self.K, self.gamma_fwd, self.acc_y, self.y, stream)
+
+    def backward(self, stream=None):
+        fqt1.scq_quantize(self.gy, self.M, self.D, self.gamma, self.p_s, self.p_c, self.psq, self.pcq, self.ws,
+                          self.dev_status, stream)
+        if self.kind == "conv":
+            N, Cin, H, W, kh, kw = self.conv
+            fqt1.bwd_input_gemm(self.psq, self.sw_col, self.cs_w, self.M, self.D, self.K, self.p_s, self.acc_dx,
+                                None, stream)
+            fqt1.col2im(self.acc_dx, self.psq, self.cs_w, N, Cin, H, W, kh, kw, self.stride, self.pad, self.dx,
+                        stream)
+        else:
+            fqt1.bwd_input_gemm(self.psq, self.sw_col, self.cs_w, self.M, self.D, self.K, self.p_s, self.acc_dx,
+                                self.dx, stream)
+        fqt1.bwd_weight_gemm(self.pcq, self.sx_col, self.cs_x, self.M, self.D, self.K, self.p_c, self.acc_dw,
+                             self.dw, None, stream)
+
+    def step(self, stream=None):
+        self.forward(stream)
+        self.backward(stream)

@@ -1,0 +1,200 @@
+"""GPU parity: the CUDA path through the C-ABI against the CPU oracle.
+
+Integer and byte results (packed signs, column sums, ranges, keep
+probabilities, kept lists, codes, int32 accumulators) must match bit for bit;
+fp32 results within |gpu - ref| <= 1e-5 (|a| + |c|) + 1e-30 where a = S' acc
+and c = Z' colsum are the two terms of the dequantization (1e-5 relative to
+the magnitude of the terms, so cancellation between them cannot hide an error).
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+pytestmark = pytest.mark.gpu
+
+from oracle import method as om  # noqa: E402
+from paper_2408_14267_gb300 import workloads as wl  # noqa: E402
+
+SYS, BER, TOP = om.SYSTEMATIC, om.BERNOULLI, om.TOPK
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2408_14267_gb300 import build
+    build.build()
+
+
+def unpack_bits(words_i32, n):
+    w = words_i32.cpu().numpy().view(np.uint32)
+    bits = ((w[:, :, None] >> np.arange(32, dtype=np.uint32)) & 1).reshape(w.shape[0], -1)
+    return bits[:, :n].astype(np.int8) * 2 - 1, bits[:, n:]
+
+
+def linear_case(M, K, D, rpg, bits, mode, seed=0, gamma=True, bits_c=None, mode_c=None):
+    rng = np.random.default_rng(seed)
+    x = rng.standard_normal((M, K)).astype(np.float32)
+    x[0, : min(3, K)] = 0.0
+    w = rng.standard_normal((D, K)).astype(np.float32)
+    s = 10.0 ** rng.uniform(-2, 2, size=(M // rpg, 1, 1))
+    gy = (rng.laplace(0, 1e-3, (M // rpg, rpg, D)) * s).reshape(M, D).astype(np.float32)
+    g = rng.uniform(0.5, 2.0, D).astype(np.float32) if gamma else None
+    return dict(name=f"linear M{M} K{K} D{D} rpg{rpg} b{bits} m{mode}", kind="linear", x=x, w=w, gamma=g, gy=gy,
+                rows_per_group=rpg, bits_s=bits, mode_s=mode, seed_s=seed + 11, bits_c=bits_c or bits,
+                mode_c=mode if mode_c is None else mode_c, seed_c=seed + 12)
+
+
+def conv_case(N, C, H, W, D, k, s, p, bits, mode, seed=0):
+    d = wl.conv_layer(f"conv N{N} C{C} {H}x{W} D{D} k{k}s{s}p{p} b{bits}", N, C, H, W, D, k, s, p, bits, seed + 5,
+                      seed + 77, sample_sigma=1.5)
+    d["mode_s"] = d["mode_c"] = mode
+    return d
+
+
+def run_oracle(w):
+    if w["kind"] == "conv":
+        return om.layer_step_conv(w["x"], w["w"], w["gamma"], w["gy"], w["stride"], w["pad"], w["bits_s"],
+                                  w["mode_s"], w["seed_s"], w["bits_c"], w["mode_c"], w["seed_c"])
+    return om.layer_step_linear(w["x"], w["w"], w["gamma"], w["gy"], w["bits_s"], w["mode_s"], w["seed_s"],
+                                w["bits_c"], w["mode_c"], w["seed_c"], w["rows_per_group"])
+
+
+def assert_dequant_close(gpu, ref, a_mag, c_mag, what):
+    tol = 1e-5 * (a_mag + c_mag) + 1e-30
+    err = np.abs(gpu.astype(np.float64) - ref.astype(np.float64))
+    bad = err > tol
+    assert not bad.any(), f"{what}: {bad.sum()} elements out of tolerance, max err {err.max()}"
+
+
+def check_branch(gq, rq, code_len, rpg, what):
+    n = gq.n
+    assert np.array_equal(gq.group_min.cpu().numpy(), rq["z"]), what + " Z"
+    assert np.array_equal(gq.group_range.cpu().numpy(), rq["r"]), what + " R"
+    assert np.array_equal(gq.p_hat.cpu().numpy(), rq["p_hat"]), what + " p_hat"
+    cnt = gq.count()
+    kept = rq["kept"]
+    assert cnt == len(kept), what + " kept count"
+    assert gq.kept_idx.cpu().numpy()[:cnt].tolist() == kept.tolist(), what + " kept ids"
+    assert np.all(gq.kept_idx.cpu().numpy()[cnt:gq.capacity] == -1)
+    slots = np.full(n, -1)
+    slots[kept] = np.arange(len(kept))
+    assert np.array_equal(gq.slot_of_group.cpu().numpy(), slots), what + " slots"
+    assert np.array_equal(gq.scale.cpu().numpy()[:cnt], rq["scale"]), what + " scale"
+    assert np.array_equal(gq.zero.cpu().numpy()[:cnt], rq["zero"]), what + " zero"
+    codes = gq.codes.cpu().numpy()[: cnt * rpg, :code_len].astype(np.int64)
+    assert np.array_equal(codes, rq["codes"]), what + " codes"
+
+
+def check_step(w, st, ref):
+    M, K, D, rpg = st.M, st.K, st.D, st.rpg
+    x_u = ref["x_u"] if w["kind"] == "conv" else w["x"]
+    w_u = w["w"].reshape(D, -1)
+    sx, pad_bits = unpack_bits(st.sx_row, K)
+    assert np.array_equal(sx, om.sign(x_u)) and not pad_bits.any(), "sign(X) row bits"
+    sxc, pad_bits = unpack_bits(st.sx_col, M)
+    assert np.array_equal(sxc, om.sign(x_u).T) and not pad_bits.any(), "sign(X) col bits"
+    sw, _ = unpack_bits(st.sw_row, K)
+    assert np.array_equal(sw, om.sign(w_u)), "sign(W) row bits"
+    swc, _ = unpack_bits(st.sw_col, D)
+    assert np.array_equal(swc, om.sign(w_u).T), "sign(W) col bits"
+    assert np.array_equal(st.cs_x.cpu().numpy(), om.colsum_sign(x_u)), "colsum X"
+    assert np.array_equal(st.cs_w.cpu().numpy(), om.colsum_sign(w_u)), "colsum W"
+    assert np.array_equal(st.acc_y.cpu().numpy(), ref["acc_y"]), "forward acc"
+    assert np.array_equal(st.y.cpu().numpy(), ref["y"]), "forward y"
+    assert int(st.dev_status[0].item()) == 0
+    check_branch(st.psq, ref["psq"], D, rpg, "PSQ")
+    check_branch(st.pcq, ref["pcq"], M, 1, "PCQ")
+    cnt_s = st.psq.count()
+    assert np.array_equal(st.acc_dx.cpu().numpy()[: cnt_s * rpg], ref["acc_dx"]), "grad_input acc"
+    cnt_c = st.pcq.count()
+    assert np.array_equal(st.acc_dw.cpu().numpy()[:cnt_c], ref["acc_dw"]), "grad_weight acc"
+    psq, pcq = ref["psq"], ref["pcq"]
+    # magnitudes of the two dequantization terms
+    if w["kind"] == "conv":
+        N = w["x"].shape[0]
+        a_mag = np.zeros(ref["dx"].shape)
+        c_mag = np.zeros(ref["dx"].shape)
+        for s_, g in enumerate(psq["kept"]):
+            a_mag[g] = np.abs(np.float64(psq["scale"][s_]) * ref["acc_fold"][g])
+            c_mag[g] = np.abs(np.float64(psq["zero"][s_]) * ref["cs_fold"])
+        assert ref["dx"].shape == (N,) + tuple(w["x"].shape[1:])
+    else:
+        a_mag = np.zeros((M, K))
+        c_mag = np.zeros((M, K))
+        cs = om.colsum_sign(w_u)
+        for s_, g in enumerate(psq["kept"]):
+            rows = slice(g * rpg, (g + 1) * rpg)
+            a_mag[rows] = np.abs(np.float64(psq["scale"][s_]) * ref["acc_dx"][s_ * rpg:(s_ + 1) * rpg])
+            c_mag[rows] = np.abs(np.float64(psq["zero"][s_]) * cs)[None, :]
+    assert_dequant_close(st.dx.cpu().numpy(), ref["dx"], a_mag, c_mag, "grad_input")
+    aw = np.zeros((D, K))
+    cw = np.zeros((D, K))
+    csx = om.colsum_sign(x_u)
+    for s_, j in enumerate(pcq["kept"]):
+        aw[j] = np.abs(np.float64(pcq["scale"][s_]) * ref["acc_dw"][s_])
+        cw[j] = np.abs(np.float64(pcq["zero"][s_]) * csx)
+    assert_dequant_close(st.dw.cpu().numpy().reshape(D, K), ref["dw"].reshape(D, K), aw, cw, "grad_weight")
+
+
+CASES = [
+    ("linear-64x512x512-b2", lambda: wl.linear_small()),
+    ("conv-resnet18-cifar-8192x2304x256-b4", lambda: wl.resnet18_cifar_conv()),
+    ("linear-ragged-b4", lambda: linear_case(40, 33, 10, 4, 4, SYS)),
+    ("linear-b8-bernoulli", lambda: linear_case(96, 200, 100, 1, 8, BER, seed=3)),
+    ("linear-oddD-b1", lambda: linear_case(50, 70, 30, 5, 1, SYS, seed=4)),
+    ("linear-n-lt-b", lambda: linear_case(3, 64, 16, 1, 8, SYS, seed=5)),
+    ("linear-single-group-topk", lambda: linear_case(64, 96, 48, 64, 2, TOP, seed=6, gamma=False)),
+    ("linear-mixed-bits", lambda: linear_case(128, 300, 64, 2, 4, SYS, seed=7, bits_c=2, mode_c=BER)),
+    ("conv-ragged-s2-topk", lambda: conv_case(3, 5, 7, 6, 12, 3, 2, 1, 2, TOP)),
+    ("conv-7x7-s2-b4", lambda: conv_case(2, 3, 20, 20, 16, 7, 2, 3, 4, SYS, seed=1)),
+    ("conv-1x1-s2-b8", lambda: conv_case(4, 8, 9, 9, 24, 1, 2, 0, 8, SYS, seed=2)),
+]
+
+
+@pytest.mark.parametrize("name,make", CASES, ids=[c[0] for c in CASES])
+def test_layer_step_parity(name, make):
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    ref = run_oracle(w)
+    st = LayerStep(w)
+    st.dev_status.zero_()
+    st.step()
+    torch.cuda.synchronize()
+    check_step(w, st, ref)
+    # a second step on the same buffers reproduces the first (no state leaks between calls)
+    y0, dx0, dw0 = st.y.clone(), st.dx.clone(), st.dw.clone()
+    st.step()
+    torch.cuda.synchronize()
+    assert torch.equal(st.y, y0) and torch.equal(st.dx, dx0) and torch.equal(st.dw, dw0)
+
+
+def test_single_branch_entry_point_matches_scq():
+    """fqt1_agp_quantize_grad on one axis equals that branch of fqt1_scq_quantize."""
+    from paper_2408_14267_gb300 import fqt1
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = linear_case(64, 32, 40, 2, 4, SYS, seed=9)
+    st = LayerStep(w)
+    st.backward()
+    for axis, ref in ((0, st.psq), (1, st.pcq)):
+        n = st.M // st.rpg if axis == 0 else st.D
+        p = st.p_s if axis == 0 else st.p_c
+        rows = ref.capacity * (st.rpg if axis == 0 else 1)
+        q = fqt1.QGradBuffers(n, ref.capacity, rows, st.D if axis == 0 else st.M)
+        fqt1.agp_quantize_grad(st.gy, st.M, st.D, axis, st.gamma, p, q, st.ws, st.dev_status)
+        torch.cuda.synchronize()
+        c = ref.count()
+        assert q.count() == c
+        assert torch.equal(q.codes[:rows], ref.codes[:rows]) and torch.equal(q.p_hat, ref.p_hat)
+
+
+def test_nonfinite_gradient_sets_status():
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = linear_case(32, 32, 16, 1, 2, SYS, seed=10)
+    w["gy"][5, 3] = np.nan
+    st = LayerStep(w)
+    st.dev_status.zero_()
+    st.backward()
+    torch.cuda.synchronize()
+    assert int(st.dev_status[0].item()) & 0x100
