@@ -1,0 +1,345 @@
+"""Benchmark of one 1-bit FQT layer training step (forward + AGP/SCQ backward).
+
+Metric: effective TOPS = 6 M K D (dense-equivalent operations of the forward,
+grad_input and grad_weight products) / device time of the whole step, on the
+ResNet-18 (CIFAR) 3x3 conv 256->256 layer on 8x8 maps, batch 128
+(M = 8192, K = 2304, D = 256; AGP b = 4, keep 1/4 of samples and channels).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl fqt1|reference]
+
+Each GPU runs an independent replica of the step (weak scaling; the layer step
+has no exchange).  The step is captured once in a CUDA graph and replayed; L2
+is flushed (256 MiB write) before every timed step and each step is timed with
+CUDA events on the launching stream.  One JSON line is printed by rank 0.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "effective TOPS of 1-bit FQT layer fwd+bwd step; % of INT8 TC peak / HBM BW"
+UNIT = "TOPS"
+WORKLOAD = "resnet18-cifar conv3x3 256->256 8x8 batch128 (M=8192 K=2304 D=256), AGP b4 keep 1/4, SCQ"
+# Peak used when MEASURED_PEAKS.json is absent.
+FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS = 6800.0, 1900.0
+SMS, POPC_PER_CLK_SM = 152, 16
+
+CPU_SAMPLE_SCRIPT = r"""
+import json, sys, time
+sys.path.insert(0, sys.argv[1])
+from paper_2408_14267_gb300 import workloads as wl
+from oracle import method as om
+w = wl.resnet18_cifar_conv()
+batch, steps = int(sys.argv[2]), int(sys.argv[3])
+N, C, H, W = w["x"].shape
+Ho = Wo = H
+x = w["x"][:batch]
+gy = w["gy"][: batch * Ho * Wo]
+times = []
+for _ in range(steps):
+    t0 = time.perf_counter()
+    om.layer_step_conv(x, w["w"], w["gamma"], gy, w["stride"], w["pad"], w["bits_s"], w["mode_s"], w["seed_s"],
+                       w["bits_c"], w["mode_c"], w["seed_c"])
+    times.append(time.perf_counter() - t0)
+M, K, D = batch * Ho * Wo, C * 9, w["w"].shape[0]
+print(json.dumps({"times": times, "ops": 6.0 * M * K * D, "M": M, "K": K, "D": D}))
+"""
+
+
+def run_oracle_sample(batch, steps):
+    """Time the CPU oracle (as it stands) on `batch` samples of the workload, one thread."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               NUMEXPR_NUM_THREADS="1")
+    p = subprocess.run([sys.executable, "-c", CPU_SAMPLE_SCRIPT, ROOT, str(batch), str(steps)], env=env,
+                       capture_output=True, text=True, timeout=1800)
+    if p.returncode != 0:
+        raise RuntimeError("oracle sample failed: " + p.stderr[-2000:])
+    return json.loads(p.stdout.strip().splitlines()[-1])
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return d.get("hbm_gbs", FALLBACK_HBM_GBS), d.get("bf16_tflops", FALLBACK_BF16_TFLOPS), "measured"
+    return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons, sampled every 100 ms while running."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_gpu{gpu_index}.csv")
+
+    def __enter__(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.Q,
+                                          "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
+                                         stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            self.proc.wait(timeout=10)
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax = float(parts[2])
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def stage_work(st, name):
+    """Algorithmic work of one stage: ('hbm', bytes) or ('alu', 1-bit ops) or ('tensor', ops)."""
+    from paper_2408_14267_gb300 import fqt1
+    M, K, D = st.M, st.K, st.D
+    wK, wM, wD = fqt1.packed_words(K), fqt1.packed_words(M), fqt1.packed_words(D)
+    ks = st.psq.count() * st.rpg
+    kc = st.pcq.count()
+    if name == "pack_w":
+        return "hbm", D * K * 4 + (D * wK + K * wD + K) * 4
+    if name in ("im2col", "pack_x"):
+        return "hbm", st.x.numel() * 4 + (M * wK + K * wM + K) * 4
+    if name == "fwd_gemm":
+        return "alu", 2.0 * M * K * D
+    if name == "scq_quantize":
+        return "hbm", M * D * 4 + ks * D + kc * M
+    if name == "bwd_input_gemm":
+        return "alu", 2.0 * ks * D * K * st.p_s.bits
+    if name == "col2im":
+        return "hbm", ks * K * 4 + st.dx.numel() * 4
+    if name == "bwd_weight_gemm":
+        return "alu", 2.0 * kc * M * K * st.p_c.bits
+    return "hbm", 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="fqt1", choices=["fqt1", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        return reference_arm(args, world, rank)
+
+    import torch
+    import torch.distributed as dist
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local_rank)
+    from paper_2408_14267_gb300 import build, fqt1, workloads
+    if rank == 0 or world == 1:
+        build.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2408_14267_gb300.layer import LayerStep
+
+    wl = workloads.resnet18_cifar_conv()
+    st = LayerStep(wl, device=f"cuda:{local_rank}", keep_acc=False)
+    stream = torch.cuda.Stream()
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device="cuda")  # 256 MiB > 129 MB L2
+    stages = st.stages()
+    with torch.cuda.stream(stream):
+        for _ in range(max(args.warmup, 3)):
+            st.step()
+        stream.synchronize()
+        n0 = fqt1.kernel_launches()
+        st.step()
+        stream.synchronize()
+        launches_per_step = fqt1.kernel_launches() - n0
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            st.step()
+        for _ in range(args.warmup):
+            graph.replay()
+        stream.synchronize()
+
+    def timed_loop(k, sampler_steps=0):
+        times = []
+        with torch.cuda.stream(stream):
+            for i in range(k):
+                flush.zero_()
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                graph.replay()
+                e1.record(stream)
+                times.append((e0, e1))
+            stream.synchronize()
+        return [a.elapsed_time(b) for a, b in times]
+
+    # steady-state pre-roll so that the clock samples bracket a loaded GPU
+    with ClockSampler(local_rank) as clk:
+        t_end = time.time() + 0.8
+        while time.time() < t_end:
+            timed_loop(20)
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        step_ms = timed_loop(args.steps)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        t_end = time.time() + 0.3
+        while time.time() < t_end:
+            timed_loop(20)
+    clocks = clk.summary()
+    total_ms = sum(step_ms)
+    if world > 1:
+        t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    ops = st.dense_ops()
+    value = world * ops * args.steps / (total_ms * 1e-3) / 1e12
+
+    # per-stage device time (eager; the stream is held by a sleep kernel while all launches are queued)
+    per_stage = {n: [] for n, _ in stages}
+    with torch.cuda.stream(stream):
+        for _ in range(max(10, min(args.steps, 50))):
+            flush.zero_()
+            torch.cuda._sleep(2_000_000)
+            evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)]
+            evs[0].record(stream)
+            for i, (n, fn) in enumerate(stages):
+                fn(stream)
+                evs[i + 1].record(stream)
+            stream.synchronize()
+            for i, (n, _) in enumerate(stages):
+                per_stage[n].append(evs[i].elapsed_time(evs[i + 1]))
+    stage_ms = {n: statistics.mean(v) for n, v in per_stage.items()}
+    dom = max(stage_ms, key=stage_ms.get)
+    hbm_peak, bf16_peak, peak_src = load_peaks()
+    bound, work = stage_work(st, dom)
+    dur_s = stage_ms[dom] * 1e-3
+    if bound == "hbm":
+        roof = {"bound": "hbm", "achieved": work / dur_s / 1e9, "peak": hbm_peak, "unit": "GB/s"}
+    elif bound == "tensor":
+        roof = {"bound": "tensor", "achieved": work / dur_s / 1e12, "peak": 2.0 * bf16_peak, "unit": "TFLOP/s"}
+    else:
+        clk_mhz = clocks.get("sm_max_mhz") or 2070.0
+        alu_peak = SMS * POPC_PER_CLK_SM * 32 * 2 * clk_mhz * 1e6 / 1e12
+        roof = {"bound": "alu", "achieved": work / dur_s / 1e12, "peak": alu_peak, "unit": "TOPS"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = None
+    roof["kernel"] = dom
+    roof["peak_source"] = peak_src if bound != "alu" else "derived: 152 SMs x 16 popc/clk x 32 bit x 2 x max clock"
+
+    # end to end: pinned host inputs -> device, step, outputs -> pinned host, all inside the timed region
+    h_in = [t.detach().cpu().pin_memory() for t in (st.x, st.w, st.gy)]
+    d_in = [st.x, st.w, st.gy]
+    if st.gamma is not None:
+        h_in.append(st.gamma.detach().cpu().pin_memory())
+        d_in.append(st.gamma)
+    d_out = [st.y, st.dx, st.dw]
+    h_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in d_out]
+    e2e_ms = []
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup + args.steps):
+            flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for h, d in zip(h_in, d_in):
+                d.copy_(h, non_blocking=True)
+            graph.replay()
+            for h, d in zip(h_out, d_out):
+                h.copy_(d, non_blocking=True)
+            e1.record(stream)
+            stream.synchronize()
+            if i >= args.warmup:
+                e2e_ms.append(e0.elapsed_time(e1))
+    e2e_total = sum(e2e_ms)
+    if world > 1:
+        t = torch.tensor([e2e_total], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_total = float(t.item())
+    e2e = {"value": world * ops * args.steps / (e2e_total * 1e-3) / 1e12, "unit": UNIT,
+           "h2d_bytes_per_step": sum(t.numel() * t.element_size() for t in h_in),
+           "d2h_bytes_per_step": sum(t.numel() * t.element_size() for t in h_out)}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        r = run_oracle_sample(batch=32, steps=2)
+        t = statistics.mean(r["times"])
+        cpu = {"value": r["ops"] / t / 1e12, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"oracle layer step on 32 of the 128 samples (M={r['M']} K={r['K']} D={r['D']}), "
+                         f"mean of 2 runs, {t:.2f} s each, one thread"}
+
+    if world > 1:
+        dist.barrier()
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "b1", "data": "synthetic",
+                "config": {"workload": WORKLOAD, "l2": "flushed before every timed step (256 MiB write)",
+                           "timing": "CUDA-graph replay of the whole step, CUDA events on the launching stream",
+                           "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU"},
+                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
+                "clocks": clocks, "stage_ms": {k: round(v, 5) for k, v in stage_ms.items()}}
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def reference_arm(args, world, rank):
+    """The oracle, as it stands, timed on the host cores (the reference for this build)."""
+    if rank != 0:
+        return
+    batch = 32  # a bounded sample of the workload per step (32 of 128 samples)
+    r = run_oracle_sample(batch=batch, steps=args.warmup + args.steps)
+    times = r["times"][args.warmup:]
+    total = sum(times)
+    value = r["ops"] * len(times) / total / 1e12
+    sample = (f"oracle layer step on {batch} of the 128 samples (M={r['M']} K={r['K']} D={r['D']}) per step, "
+              f"one thread")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(times),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD}, "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1,
+                                                               "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+if __name__ == "__main__":
+    main()

@@ -1,5 +1,7 @@
 // C-ABI entry points of the GEMM side, dequantization and the Folder, plus helpers.
 #include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
 
 #include <atomic>
 
@@ -28,6 +30,23 @@ extern "C" int64_t fqt1_kept_capacity(int64_t n, int32_t bits, int32_t mode) {
 extern "C" int64_t fqt1_codes_ld(int64_t n) { return n < 1 ? 0 : ((n + 15) / 16) * 16; }
 
 namespace fqt1 {
+
+bool use_popcount_path() {
+  static int v = -1;
+  if (v < 0) {
+    const char* e = getenv("FQT1_GEMM_PATH");
+    v = (e && strcmp(e, "popcount") == 0) ? 1 : 0;
+  }
+  return v == 1;
+}
+
+// Rows of pruned groups of an [M][K] fp32 output are exactly zero.
+__global__ void zero_pruned_rows_kernel(const int32_t* __restrict__ slot_of_group, int64_t M, int64_t K, int64_t rpg,
+                                        float* __restrict__ out) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= M * K) return;
+  if (__ldg(slot_of_group + (idx / K) / rpg) < 0) out[idx] = 0.0f;
+}
 
 // out[m, k] = S'_slot * acc[row(m), k] + Z'_slot * cs[k] for rows m of kept groups, 0 otherwise
 // (fp32 multiply, multiply, add; no contraction).  Used for dx (groups of rpg rows) and dw (rpg = 1).
@@ -100,7 +119,11 @@ extern "C" fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_
       (gamma && !aligned16(gamma)))
     return FQT1_ERR_MISALIGNED;
   if (K >= (1ll << 24) || (M + 63) / 64 > 65535) return FQT1_ERR_UNSUPPORTED;
-  FQT1_CUDA_TRY(launch_xnor_gemm_simt(sx_row, sw_row, M, D, K, gamma, acc, y, (cudaStream_t)stream));
+  if (use_popcount_path() || !y) {
+    FQT1_CUDA_TRY(launch_xnor_gemm_simt(sx_row, sw_row, M, D, K, gamma, acc, y, (cudaStream_t)stream));
+  } else {
+    FQT1_CUDA_TRY(launch_fwd_tc(sx_row, sw_row, M, D, K, gamma, acc, y, nullptr, (cudaStream_t)stream));
+  }
   return FQT1_OK;
 }
 
@@ -118,10 +141,25 @@ extern "C" fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t
   const int64_t cap_rows = fqt1_kept_capacity(M / rpg, p->bits, p->mode) * rpg;
   if ((cap_rows + 63) / 64 > 65535) return FQT1_ERR_UNSUPPORTED;
   cudaStream_t s = (cudaStream_t)stream;
-  // The CUDA-core path needs the integer result in memory; a conv passes acc.
-  if (!acc) return FQT1_ERR_UNSUPPORTED;
-  FQT1_CUDA_TRY(launch_codes_gemm_simt(p->bits, psq->codes, psq->ld_codes, psq->kept_count, rpg, cap_rows, sw_col, K,
-                                       D, acc, K, s));
+  if (!use_popcount_path() && !acc) {
+    // dequantization fused into the tensor-core epilogue; pruned rows written as zeros
+    FQT1_CUDA_TRY(launch_codes_tc_simple(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, rpg, sw_col,
+                                         K, D, GEMM_EPI_DX, 1, nullptr, dx, K, psq->kept_idx, psq->scale,
+                                         psq->zero, colsum_w, rpg, nullptr, s));
+    const int64_t n = M * K;
+    zero_pruned_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(psq->slot_of_group, M, K, rpg, dx);
+    fqt1_count_launches(1);
+    FQT1_CUDA_TRY(cudaGetLastError());
+    return FQT1_OK;
+  }
+  if (use_popcount_path()) {
+    FQT1_CUDA_TRY(launch_codes_gemm_simt(p->bits, psq->codes, psq->ld_codes, psq->kept_count, rpg, cap_rows, sw_col,
+                                         K, D, acc, K, s));
+  } else {
+    FQT1_CUDA_TRY(launch_codes_tc_simple(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, rpg, sw_col,
+                                         K, D, GEMM_EPI_ACC32, 1, acc, nullptr, K, nullptr, nullptr, nullptr,
+                                         nullptr, rpg, nullptr, s));
+  }
   if (dx) {
     const int64_t n = M * K;
     dequant_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(acc, K, psq->slot_of_group, psq->scale,
@@ -162,8 +200,24 @@ extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_
   if (!aligned16(sx_col) || !aligned16(acc) || !aligned16(dw) || !aligned16(colsum_x)) return FQT1_ERR_MISALIGNED;
   const int64_t cap = fqt1_kept_capacity(D, p->bits, p->mode);
   cudaStream_t s = (cudaStream_t)stream;
-  FQT1_CUDA_TRY(launch_codes_gemm_simt(p->bits, pcq->codes, pcq->ld_codes, pcq->kept_count, 1, cap, sx_col, K, M, acc,
-                                       K, s));
+  if (use_popcount_path()) {
+    FQT1_CUDA_TRY(launch_codes_gemm_simt(p->bits, pcq->codes, pcq->ld_codes, pcq->kept_count, 1, cap, sx_col, K, M,
+                                         acc, K, s));
+  } else {
+    // split the long contraction over M across CTAs (int32 reduction into acc, exact in any order);
+    // each CTA's fp32 partial sum stays below 2^24
+    const int64_t k_tiles = (M + 127) / 128;
+    const int64_t out_tiles = ((K + 127) / 128) * ((cap + 127) / 128);
+    int64_t splits = (152 + out_tiles - 1) / out_tiles;  // about one wave on 152 SMs
+    const int64_t min_splits = (M + exact_chunk(p->bits) - 1) / exact_chunk(p->bits);
+    if (splits < min_splits) splits = min_splits;
+    if (splits > k_tiles) splits = k_tiles;
+    if ((k_tiles + splits - 1) / splits * 128 > exact_chunk(p->bits)) return FQT1_ERR_UNSUPPORTED;
+    FQT1_CUDA_TRY(cudaMemsetAsync(acc, 0, sizeof(int32_t) * cap * K, s));
+    FQT1_CUDA_TRY(launch_codes_tc_simple(p->bits, pcq->codes, pcq->ld_codes, cap, pcq->kept_count, 1, sx_col, K, M,
+                                         GEMM_EPI_RED, (int)splits, acc, nullptr, K, nullptr, nullptr, nullptr,
+                                         nullptr, 1, nullptr, s));
+  }
   const int64_t n = D * K;
   dequant_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(acc, K, pcq->slot_of_group, pcq->scale, pcq->zero,
                                                                   colsum_x, D, K, 1, dw);

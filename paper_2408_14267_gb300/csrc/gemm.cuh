@@ -10,4 +10,19 @@ cudaError_t launch_codes_gemm_simt(int bits, const uint8_t* Q, int64_t ldq, cons
                                    int64_t rows_per_count, int64_t max_rows, const uint32_t* S, int64_t n_s,
                                    int64_t L, int32_t* out, int64_t ldo, cudaStream_t s);
 
+// tcgen05 path (gemm_tc.cu)
+struct TcArgs;
+cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64_t D, int64_t K, const float* gamma,
+                          int32_t* acc, float* y, int32_t* status, cudaStream_t s);
+cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
+                                   int64_t rows_per_count, const uint32_t* Sg, int64_t n_s, int64_t L, int epi,
+                                   int splits, int32_t* acc, float* out, int64_t ldo, const int32_t* kept_idx,
+                                   const float* scale, const float* zero, const int32_t* cs, int64_t rpg,
+                                   int32_t* status, cudaStream_t s);
+enum : int { GEMM_EPI_ACC32 = 1, GEMM_EPI_RED = 2, GEMM_EPI_DX = 3 };
+// Largest contraction one CTA may sum in fp32 and stay exact: partial sums below 2^24.
+inline int64_t exact_chunk(int bits) { return (int64_t)((1 << 24) / ((1 << bits) - 1)); }
+// 1 if FQT1_GEMM_PATH=popcount selects the CUDA-core kernels (datapath comparison only).
+bool use_popcount_path();
+
 }  // namespace fqt1

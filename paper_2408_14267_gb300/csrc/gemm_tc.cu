@@ -1,0 +1,523 @@
+// Tensor-core integer GEMMs for sm_103a (tcgen05 + TMEM + TMA).
+//
+// C[r, n] = sum_k A[r, k] B[n, k] with both operands K-major:
+//   A: packed +-1 signs (uint32 words) or uint8 gradient codes,
+//   B: packed +-1 signs.
+// The binary product of App. C (XNOR-popcount) and the bit-plane product of
+// Sec. 5.2 are evaluated exactly on the fp8 tensor cores: +-1 and codes
+// 0..15 are exact e4m3 values, a b = 8 code is split into 16*hi + lo with
+// both digits exact, products are exact, and every partial sum is an integer
+// below 2^24 so the fp32 accumulator in TMEM holds it exactly.
+//
+// Pipeline per CTA (one 128 x BN output tile, 128-element K steps):
+//   warp 0 lane 0   TMA: raw tiles (packed words or codes) -> shared memory
+//   warp 1          TMEM allocation; lane 0 issues tcgen05.mma, commits stages
+//   warps 2..5      expand raw tiles into 128B-swizzled e4m3 operand tiles,
+//                   then run the epilogue from TMEM (each warp owns 32 lanes)
+// Every wait is bounded; an expired wait sets FQT1_DEV_TIMEOUT and the CTA
+// drains and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "gemm.cuh"
+
+namespace fqt1 {
+
+constexpr int kBM = 128;           // output rows per CTA (MMA M)
+constexpr int kBK = 128;           // contraction elements per stage (one 128-byte swizzle row of e4m3)
+constexpr int kStages = 4;
+constexpr int kExpWarps = 4;
+constexpr int kThreads = 32 * (2 + kExpWarps);
+constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on every wait
+
+enum : int { EPI_FWD = 0, EPI_ACC32 = 1, EPI_RED = 2, EPI_DX = 3 };
+
+struct TcArgs {
+  int64_t M, N, L;           // rows (capacity), columns, contraction length
+  const int32_t* count;      // valid rows = *count * rows_per_count (null: all M)
+  int64_t rows_per_count;
+  int k_tiles, tiles_per_split;
+  int epi;
+  const float* gamma;        // EPI_FWD: y = gamma[n] * acc
+  float* y;
+  int32_t* acc;              // EPI_FWD (optional), EPI_ACC32, EPI_RED
+  int64_t ldo;
+  const int32_t* kept_idx;   // EPI_DX: dx[kept_idx[r / rpg] * rpg + r % rpg, n] = S' acc + Z' cs[n]
+  const float* scale;
+  const float* zero;
+  const int32_t* cs;
+  int64_t rpg;
+  int32_t* status;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ uint64_t gtimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(b)), "r"(count));
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* b) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(b)) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* b, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(b)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n.reg .pred p;\nmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\nselp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(b)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for phase `parity` of barrier b; false (and the timeout status) if it expired
+// or another role already gave up.
+__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, volatile int* abort_flag, int32_t* status) {
+  if (mbar_test(b, parity)) return true;
+  const uint64_t t0 = gtimer();
+  while (true) {
+    if (mbar_test(b, parity)) return true;
+    if (*abort_flag) return false;
+    if (gtimer() - t0 > kWaitNs) {
+      *abort_flag = 1;
+      if (status) atomicOr(status, FQT1_DEV_TIMEOUT);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
+          smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major operand tile in the 128-byte swizzle layout
+// (rows of 128 bytes, 8-row groups 1024 bytes apart).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFF) >> 4);
+  d |= (uint64_t)1 << 16;              // leading byte offset (unused for this layout)
+  d |= (uint64_t)(1024 >> 4) << 32;    // stride byte offset: next 8-row group
+  d |= (uint64_t)1 << 46;              // descriptor version
+  d |= (uint64_t)2 << 61;              // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor: e4m3 x e4m3 -> f32, both K-major, M = 128, N = bn.
+__host__ __device__ constexpr uint32_t idesc_e4m3(int bn) {
+  return (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(bn >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_e4m3(uint32_t tmem, uint64_t ad, uint64_t bd, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem),
+      "l"(ad), "l"(bd), "r"(idesc), "r"(acc));
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+// Byte offset of 16-byte chunk c of row r in a 128B-swizzled tile.
+__device__ __forceinline__ uint32_t swz(int r, int c) {
+  return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
+}
+
+// 4 sign bits -> 4 e4m3 bytes (+1 = 0x38, -1 = 0xB8).
+__device__ __forceinline__ uint32_t signs4(uint32_t nib) {
+  const uint32_t spread = (nib * 0x00204081u) & 0x01010101u;
+  return 0xB8B8B8B8u ^ (spread << 7);
+}
+// 16 sign bits -> 16 e4m3 bytes.
+__device__ __forceinline__ uint4 signs16(uint32_t h) {
+  return make_uint4(signs4(h & 15u), signs4((h >> 4) & 15u), signs4((h >> 8) & 15u), signs4((h >> 12) & 15u));
+}
+// 4 codes (one per byte, each < 16) -> 4 e4m3 bytes of the same integers.
+__device__ __forceinline__ uint32_t codes4(uint32_t c) {
+  const uint32_t sel = (c & 0x7u) | ((c >> 4) & 0x70u) | ((c >> 8) & 0x700u) | ((c >> 12) & 0x7000u);
+  const uint32_t lo = __byte_perm(0x44403800u, 0x4E4C4A48u, sel);  // e4m3 of 0..7
+  const uint32_t hi = __byte_perm(0x53525150u, 0x57565554u, sel);  // e4m3 of 8..15
+  const uint32_t m = ((c >> 3) & 0x01010101u) * 0xFFu;
+  return (lo & ~m) | (hi & m);
+}
+// e4m3 of 16*h for digits h < 16 (exponent raised by 4; zero stays zero).
+__device__ __forceinline__ uint32_t codes4_x16(uint32_t h) {
+  const uint32_t e = codes4(h);
+  const uint32_t nz = (((h | (h >> 1) | (h >> 2) | (h >> 3)) & 0x01010101u)) * 0x20u;
+  return e + nz;
+}
+
+template <bool A_CODES, bool BITS8, int BN>
+struct TcSmem {
+  static constexpr int kOpA = kBM * kBK;              // bytes of one e4m3 A tile
+  static constexpr int kOpB = BN * kBK;
+  static constexpr int kRawA = A_CODES ? 0 : kBM * 16;  // packed words of A (4 per row)
+  static constexpr int kRawB = BN * 16;
+  static constexpr int kStage = kOpA * (BITS8 ? 2 : 1) + kOpB + kRawA + kRawB;
+  static constexpr int kBytes = kStages * kStage + 1024;  // + alignment slack
+};
+
+template <bool A_CODES, bool BITS8, int BN>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, TcArgs a) {
+  using S = TcSmem<A_CODES, BITS8, BN>;
+  extern __shared__ unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t raw_full[kStages], raw_empty[kStages], op_full[kStages], op_empty[kStages];
+  __shared__ __align__(8) uint64_t acc_full;
+  __shared__ uint32_t tmem_slot;
+  __shared__ volatile int abort_flag;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t m0 = (int64_t)blockIdx.y * kBM, n0 = (int64_t)blockIdx.x * BN;
+  const int64_t valid_rows = a.count ? (int64_t)__ldg(a.count) * a.rows_per_count : a.M;
+  if (m0 >= valid_rows) return;
+  const int kt0 = blockIdx.z * a.tiles_per_split;
+  const int kt1 = min(a.k_tiles, kt0 + a.tiles_per_split);
+  if (kt0 >= kt1) return;
+  const int nk = kt1 - kt0;
+
+  unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  auto opA = [&](int s) { return base + s * S::kStage; };
+  auto opA2 = [&](int s) { return base + s * S::kStage + S::kOpA; };
+  auto opB = [&](int s) { return base + s * S::kStage + S::kOpA * (BITS8 ? 2 : 1); };
+  auto rawA = [&](int s) { return opB(s) + S::kOpB; };
+  auto rawB = [&](int s) { return rawA(s) + S::kRawA; };
+
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&raw_full[s], 1);
+      mbar_init(&raw_empty[s], kExpWarps);
+      mbar_init(&op_full[s], kExpWarps);
+      mbar_init(&op_empty[s], 1);
+    }
+    mbar_init(&acc_full, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
+                 "r"(BN));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = tmem_slot;
+
+  constexpr uint32_t kTxA = A_CODES ? (uint32_t)S::kOpA : (uint32_t)S::kRawA;
+  constexpr uint32_t kTx = kTxA + (uint32_t)S::kRawB;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      int issued = 0;
+      for (int i = 0; i < nk; ++i) {
+        const int s = i % kStages, it = i / kStages;
+        if (it > 0) {
+          if (!mbar_wait(&raw_empty[s], (it - 1) & 1, &abort_flag, a.status)) break;
+          if (A_CODES && !mbar_wait(&op_empty[s], (it - 1) & 1, &abort_flag, a.status)) break;
+        }
+        const int kt = kt0 + i;
+        mbar_expect_tx(&raw_full[s], kTx);
+        if (A_CODES) tma_load_2d(opA(s), &tmA, &raw_full[s], kt * kBK, (int)m0);
+        else tma_load_2d(rawA(s), &tmA, &raw_full[s], kt * (kBK / 32), (int)m0);
+        tma_load_2d(rawB(s), &tmB, &raw_full[s], kt * (kBK / 32), (int)n0);
+        ++issued;
+      }
+      // drain: every issued copy must land before the CTA may exit
+      for (int i = (issued > kStages ? issued - kStages : 0); i < issued; ++i) {
+        const int s = i % kStages, it = i / kStages;
+        const uint64_t t0 = gtimer();
+        while (!mbar_test(&raw_full[s], it & 1) && gtimer() - t0 < kWaitNs) {
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_e4m3(BN);
+      bool ok = true;
+      for (int i = 0; i < nk; ++i) {
+        const int s = i % kStages, it = i / kStages;
+        if (!mbar_wait(&op_full[s], it & 1, &abort_flag, a.status)) { ok = false; break; }
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t aaddr = smem_u32(opA(s)), a2addr = smem_u32(opA2(s)), baddr = smem_u32(opB(s));
+#pragma unroll
+        for (int k = 0; k < kBK / 32; ++k) {
+          const uint64_t bd = sw128_desc(baddr + 32 * k);
+          mma_e4m3(tmem, sw128_desc(aaddr + 32 * k), bd, idesc, (i > 0 || k > 0) ? 1u : 0u);
+          if (BITS8) mma_e4m3(tmem, sw128_desc(a2addr + 32 * k), bd, idesc, 1u);
+        }
+        mma_commit(&op_empty[s]);
+      }
+      (void)ok;
+      mma_commit(&acc_full);
+    }
+  } else {
+    // ---------------------------------------------------------------- expansion
+    const int t = threadIdx.x - 64;  // 0..127
+    for (int i = 0; i < nk; ++i) {
+      const int s = i % kStages, it = i / kStages;
+      if (it > 0 && !mbar_wait(&op_empty[s], (it - 1) & 1, &abort_flag, a.status)) break;
+      if (!mbar_wait(&raw_full[s], it & 1, &abort_flag, a.status)) break;
+      const int kt = kt0 + i;
+      // A tile: row t
+      if (A_CODES) {
+        unsigned char* ta = opA(s);
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const uint32_t off = swz(t, c);
+          uint4 v = *reinterpret_cast<uint4*>(ta + off);
+          if (BITS8) {
+            uint4 lo, hi;
+            lo.x = codes4(v.x & 0x0F0F0F0Fu); hi.x = codes4_x16((v.x >> 4) & 0x0F0F0F0Fu);
+            lo.y = codes4(v.y & 0x0F0F0F0Fu); hi.y = codes4_x16((v.y >> 4) & 0x0F0F0F0Fu);
+            lo.z = codes4(v.z & 0x0F0F0F0Fu); hi.z = codes4_x16((v.z >> 4) & 0x0F0F0F0Fu);
+            lo.w = codes4(v.w & 0x0F0F0F0Fu); hi.w = codes4_x16((v.w >> 4) & 0x0F0F0F0Fu);
+            *reinterpret_cast<uint4*>(ta + off) = hi;
+            *reinterpret_cast<uint4*>(opA2(s) + off) = lo;
+          } else {
+            v.x = codes4(v.x); v.y = codes4(v.y); v.z = codes4(v.z); v.w = codes4(v.w);
+            *reinterpret_cast<uint4*>(ta + off) = v;
+          }
+        }
+      } else {
+        const uint4 w4 = *reinterpret_cast<const uint4*>(rawA(s) + 16 * t);
+        const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+        unsigned char* ta = opA(s);
+        const int64_t kbase = (int64_t)kt * kBK;
+        const bool full = kbase + kBK <= a.L;
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            uint4 v = signs16(wv[w] >> (16 * h));
+            if (!full) {  // elements past the contraction length contribute 0
+              const int64_t e0 = kbase + 32 * w + 16 * h;
+              uint32_t* vv = reinterpret_cast<uint32_t*>(&v);
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                for (int bb = 0; bb < 4; ++bb)
+                  if (e0 + 4 * q + bb >= a.L) vv[q] &= ~(0xFFu << (8 * bb));
+              }
+            }
+            *reinterpret_cast<uint4*>(ta + swz(t, 2 * w + h)) = v;
+          }
+        }
+      }
+      // B tile: rows t, t + 128, ...
+#pragma unroll
+      for (int rr = 0; rr < BN / kBM; ++rr) {
+        const int r = t + kBM * rr;
+        const uint4 w4 = *reinterpret_cast<const uint4*>(rawB(s) + 16 * r);
+        const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+        unsigned char* tb = opB(s);
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          *reinterpret_cast<uint4*>(tb + swz(r, 2 * w)) = signs16(wv[w]);
+          *reinterpret_cast<uint4*>(tb + swz(r, 2 * w + 1)) = signs16(wv[w] >> 16);
+        }
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&op_full[s]);
+        mbar_arrive(&raw_empty[s]);
+      }
+    }
+
+    // ---------------------------------------------------------------- epilogue
+    const bool have_acc = mbar_wait(&acc_full, 0, &abort_flag, a.status);
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const int q = warp & 3;  // TMEM lane quarter of this warp
+    const int64_t r = m0 + 32 * q + lane;
+    const bool row_ok = have_acc && r < valid_rows && r < a.M;
+    int64_t out_row = r;
+    float sc = 0.f, ze = 0.f;
+    if (a.epi == EPI_DX && row_ok) {
+      const int64_t slot = r / a.rpg;
+      out_row = (int64_t)__ldg(a.kept_idx + slot) * a.rpg + (r - slot * a.rpg);
+      sc = __ldg(a.scale + slot);
+      ze = __ldg(a.zero + slot);
+    }
+    const bool vec = (a.ldo % 4) == 0;
+    for (int c0 = 0; c0 < BN; c0 += 32) {
+      __syncwarp();
+      uint32_t v[32];
+      const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)c0;
+      asm volatile(
+          "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,"
+          "%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+          : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+            "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
+            "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
+            "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+          : "r"(taddr));
+      asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+      if (!row_ok) continue;
+      const int64_t nb = n0 + c0;
+      if (nb >= a.N) continue;
+      int32_t iv[32];
+#pragma unroll
+      for (int j = 0; j < 32; ++j) iv[j] = __float2int_rn(__uint_as_float(v[j]));
+      const bool full = nb + 32 <= a.N && vec;
+      if (a.epi == EPI_FWD) {
+        float* yrow = a.y + out_row * a.ldo + nb;
+        if (full) {
+#pragma unroll
+          for (int j = 0; j < 32; j += 4) {
+            float4 o;
+            o.x = __fmul_rn(__ldg(a.gamma + nb + j + 0), (float)iv[j + 0]);
+            o.y = __fmul_rn(__ldg(a.gamma + nb + j + 1), (float)iv[j + 1]);
+            o.z = __fmul_rn(__ldg(a.gamma + nb + j + 2), (float)iv[j + 2]);
+            o.w = __fmul_rn(__ldg(a.gamma + nb + j + 3), (float)iv[j + 3]);
+            *reinterpret_cast<float4*>(yrow + j) = o;
+            if (a.acc) *reinterpret_cast<int4*>(a.acc + out_row * a.ldo + nb + j) = make_int4(iv[j], iv[j + 1], iv[j + 2], iv[j + 3]);
+          }
+        } else {
+          for (int j = 0; j < 32 && nb + j < a.N; ++j) {
+            yrow[j] = __fmul_rn(__ldg(a.gamma + nb + j), (float)iv[j]);
+            if (a.acc) a.acc[out_row * a.ldo + nb + j] = iv[j];
+          }
+        }
+      } else if (a.epi == EPI_ACC32) {
+        int32_t* orow = a.acc + out_row * a.ldo + nb;
+        if (full) {
+#pragma unroll
+          for (int j = 0; j < 32; j += 4) *reinterpret_cast<int4*>(orow + j) = make_int4(iv[j], iv[j + 1], iv[j + 2], iv[j + 3]);
+        } else {
+          for (int j = 0; j < 32 && nb + j < a.N; ++j) orow[j] = iv[j];
+        }
+      } else if (a.epi == EPI_RED) {
+        int32_t* orow = a.acc + out_row * a.ldo + nb;
+        for (int j = 0; j < 32 && nb + j < a.N; ++j) atomicAdd(orow + j, iv[j]);
+      } else {  // EPI_DX
+        float* orow = a.y + out_row * a.ldo + nb;
+        if (full) {
+#pragma unroll
+          for (int j = 0; j < 32; j += 4) {
+            float4 o;
+            o.x = __fadd_rn(__fmul_rn(sc, (float)iv[j + 0]), __fmul_rn(ze, (float)__ldg(a.cs + nb + j + 0)));
+            o.y = __fadd_rn(__fmul_rn(sc, (float)iv[j + 1]), __fmul_rn(ze, (float)__ldg(a.cs + nb + j + 1)));
+            o.z = __fadd_rn(__fmul_rn(sc, (float)iv[j + 2]), __fmul_rn(ze, (float)__ldg(a.cs + nb + j + 2)));
+            o.w = __fadd_rn(__fmul_rn(sc, (float)iv[j + 3]), __fmul_rn(ze, (float)__ldg(a.cs + nb + j + 3)));
+            *reinterpret_cast<float4*>(orow + j) = o;
+          }
+        } else {
+          for (int j = 0; j < 32 && nb + j < a.N; ++j)
+            orow[j] = __fadd_rn(__fmul_rn(sc, (float)iv[j]), __fmul_rn(ze, (float)__ldg(a.cs + nb + j)));
+        }
+      }
+    }
+  }
+
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  if (warp == 1) {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(BN));
+  }
+}
+
+// ------------------------------------------------------------------ host side
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D map of a row-major matrix: inner extent `cols` elements, `rows` rows, row stride `ld_bytes`.
+static bool make_map(CUtensorMap* m, const void* ptr, CUtensorMapDataType type, int64_t cols, int64_t rows,
+                     int64_t ld_bytes, uint32_t box_cols, uint32_t box_rows, CUtensorMapSwizzle swz_mode) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)ld_bytes};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, type, 2, const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz_mode,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <bool A_CODES, bool BITS8, int BN>
+static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const TcArgs& a, int splits,
+                             cudaStream_t s) {
+  using S = TcSmem<A_CODES, BITS8, BN>;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<A_CODES, BITS8, BN>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  dim3 grid((unsigned)((a.N + BN - 1) / BN), (unsigned)((a.M + kBM - 1) / kBM), (unsigned)splits);
+  tc_gemm_kernel<A_CODES, BITS8, BN><<<grid, kThreads, S::kBytes, s>>>(ma, mb, a);
+  fqt1_count_launches(1);
+  return cudaGetLastError();
+}
+
+// Forward: A = sign(X) rows [M][words(K)], B = sign(W) rows [D][words(K)].
+cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64_t D, int64_t K, const float* gamma,
+                          int32_t* acc, float* y, int32_t* status, cudaStream_t s) {
+  const int64_t ldw = fqt1_packed_words(K);
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, A, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, M, ldw * 4, 4, kBM, CU_TENSOR_MAP_SWIZZLE_NONE) ||
+      !make_map(&mb, B, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, D, ldw * 4, 4, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+    return cudaErrorInvalidValue;
+  TcArgs a{};
+  a.M = M; a.N = D; a.L = K; a.count = nullptr; a.rows_per_count = 1;
+  a.k_tiles = (int)((K + kBK - 1) / kBK); a.tiles_per_split = a.k_tiles;
+  a.epi = EPI_FWD; a.gamma = gamma; a.y = y; a.acc = acc; a.ldo = D; a.status = status;
+  return launch_tc<false, false, 128>(ma, mb, a, 1, s);
+}
+
+// Codes x signs: out[r, n] = sum_j Q[r, j] S[n, j], Q [rows][ld] uint8 (valid rows *count * rpc),
+// S [n_s][words(L)] packed signs.  epi: EPI_ACC32 (store), EPI_RED (split-K add), EPI_DX (dequantize).
+cudaError_t launch_codes_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
+                            int64_t rows_per_count, const uint32_t* Sg, int64_t n_s, int64_t L, int epi, int splits,
+                            const TcArgs& epi_args, cudaStream_t s) {
+  const int64_t lds = fqt1_packed_words(L);
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, L, max_rows, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, n_s, lds * 4, 4, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+    return cudaErrorInvalidValue;
+  TcArgs a = epi_args;
+  a.M = max_rows; a.N = n_s; a.L = L; a.count = count; a.rows_per_count = rows_per_count;
+  a.k_tiles = (int)((L + kBK - 1) / kBK);
+  a.tiles_per_split = (a.k_tiles + splits - 1) / splits;
+  a.epi = epi;
+  const int z = (a.k_tiles + a.tiles_per_split - 1) / a.tiles_per_split;
+  if (bits == 8) return launch_tc<true, true, 128>(ma, mb, a, z, s);
+  return launch_tc<true, false, 128>(ma, mb, a, z, s);
+}
+
+cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
+                                   int64_t rows_per_count, const uint32_t* Sg, int64_t n_s, int64_t L, int epi,
+                                   int splits, int32_t* acc, float* out, int64_t ldo, const int32_t* kept_idx,
+                                   const float* scale, const float* zero, const int32_t* cs, int64_t rpg,
+                                   int32_t* status, cudaStream_t s) {
+  TcArgs a{};
+  a.acc = acc; a.y = out; a.ldo = ldo; a.kept_idx = kept_idx; a.scale = scale; a.zero = zero; a.cs = cs;
+  a.rpg = rpg; a.status = status;
+  return launch_codes_tc(bits, Q, ldq, max_rows, count, rows_per_count, Sg, n_s, L, epi, splits, a, s);
+}
+
+}  // namespace fqt1

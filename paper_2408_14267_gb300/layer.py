@@ -24,9 +24,13 @@ def conv_out_hw(H, W, kh, kw, stride, pad):
 
 
 class LayerStep:
-    def __init__(self, wl, device="cuda"):
+    """Buffers and launches of one layer step.  keep_acc=False skips the optional
+    int32 copy of the forward accumulators (the benchmark's configuration)."""
+
+    def __init__(self, wl, device="cuda", keep_acc=True):
         dev = torch.device(device)
         self.kind = wl["kind"]
+        self.keep_acc = keep_acc
         f32 = dict(dtype=torch.float32, device=dev)
         i32 = dict(dtype=torch.int32, device=dev)
         self.x = torch.as_tensor(np.ascontiguousarray(wl["x"]), **f32)
@@ -52,7 +56,7 @@ class LayerStep:
         self.sw_row = torch.empty(D, wK, **i32)
         self.sw_col = torch.empty(K, wD, **i32)
         self.cs_w = torch.empty(K, **i32)
-        self.acc_y = torch.empty(M, D, **i32)
+        self.acc_y = torch.empty(M, D, **i32) if keep_acc else None
         # without a Gamma the forward uses unit scales and G = gY
         self.gamma_fwd = self.gamma if self.gamma is not None else torch.ones(D, **f32)
         self.y = torch.empty(M, D, **f32)
@@ -74,31 +78,47 @@ class LayerStep:
     def dense_ops(self):
         return 6.0 * self.M * self.K * self.D
 
-    def forward(self, stream=None):
-        fqt1.binarize_pack(self.w, self.D, self.K, self.K, self.sw_row, self.sw_col, self.cs_w, stream)
+    def stages(self):
+        """The step as (name, launch(stream)) pairs, in stream order."""
+        st = [("pack_w", lambda s: fqt1.binarize_pack(self.w, self.D, self.K, self.K, self.sw_row, self.sw_col,
+                                                       self.cs_w, s))]
         if self.kind == "conv":
             N, Cin, H, W, kh, kw = self.conv
-            fqt1.im2col(self.x, N, Cin, H, W, kh, kw, self.stride, self.pad, self.sx_row, self.sx_col, self.cs_x,
-                        stream)
+            st.append(("im2col", lambda s: fqt1.im2col(self.x, N, Cin, H, W, kh, kw, self.stride, self.pad,
+                                                       self.sx_row, self.sx_col, self.cs_x, s)))
         else:
-            fqt1.binarize_pack(self.x, self.M, self.K, self.K, self.sx_row, self.sx_col, self.cs_x, stream)
-        fqt1.fwd_gemm(self.sx_row, self.sw_row, self.M, self.D, self.K, self.gamma_fwd, self.acc_y, self.y, stream)
+            st.append(("pack_x", lambda s: fqt1.binarize_pack(self.x, self.M, self.K, self.K, self.sx_row,
+                                                              self.sx_col, self.cs_x, s)))
+        st.append(("fwd_gemm", lambda s: fqt1.fwd_gemm(self.sx_row, self.sw_row, self.M, self.D, self.K,
+                                                       self.gamma_fwd, self.acc_y, self.y, s)))
+        st.append(("scq_quantize", lambda s: fqt1.scq_quantize(self.gy, self.M, self.D, self.gamma, self.p_s,
+                                                               self.p_c, self.psq, self.pcq, self.ws,
+                                                               self.dev_status, s)))
+        if self.kind == "conv":
+            N, Cin, H, W, kh, kw = self.conv
+            st.append(("bwd_input_gemm", lambda s: fqt1.bwd_input_gemm(self.psq, self.sw_col, self.cs_w, self.M,
+                                                                       self.D, self.K, self.p_s, self.acc_dx, None,
+                                                                       s)))
+            st.append(("col2im", lambda s: fqt1.col2im(self.acc_dx, self.psq, self.cs_w, N, Cin, H, W, kh, kw,
+                                                       self.stride, self.pad, self.dx, s)))
+        else:
+            # without keep_acc the dequantization runs in the GEMM epilogue (no int32 round trip)
+            acc = self.acc_dx if self.keep_acc else None
+            st.append(("bwd_input_gemm", lambda s: fqt1.bwd_input_gemm(self.psq, self.sw_col, self.cs_w, self.M,
+                                                                       self.D, self.K, self.p_s, acc, self.dx, s)))
+        st.append(("bwd_weight_gemm", lambda s: fqt1.bwd_weight_gemm(self.pcq, self.sx_col, self.cs_x, self.M,
+                                                                     self.D, self.K, self.p_c, self.acc_dw, self.dw,
+                                                                     None, s)))
+        return st
+
+    def forward(self, stream=None):
+        for name, fn in self.stages()[:3]:
+            fn(stream)
 
     def backward(self, stream=None):
-        fqt1.scq_quantize(self.gy, self.M, self.D, self.gamma, self.p_s, self.p_c, self.psq, self.pcq, self.ws,
-                          self.dev_status, stream)
-        if self.kind == "conv":
-            N, Cin, H, W, kh, kw = self.conv
-            fqt1.bwd_input_gemm(self.psq, self.sw_col, self.cs_w, self.M, self.D, self.K, self.p_s, self.acc_dx,
-                                None, stream)
-            fqt1.col2im(self.acc_dx, self.psq, self.cs_w, N, Cin, H, W, kh, kw, self.stride, self.pad, self.dx,
-                        stream)
-        else:
-            fqt1.bwd_input_gemm(self.psq, self.sw_col, self.cs_w, self.M, self.D, self.K, self.p_s, self.acc_dx,
-                                self.dx, stream)
-        fqt1.bwd_weight_gemm(self.pcq, self.sx_col, self.cs_x, self.M, self.D, self.K, self.p_c, self.acc_dw,
-                             self.dw, None, stream)
+        for name, fn in self.stages()[3:]:
+            fn(stream)
 
     def step(self, stream=None):
-        self.forward(stream)
-        self.backward(stream)
+        for name, fn in self.stages():
+            fn(stream)

@@ -170,6 +170,34 @@ def test_layer_step_parity(name, make):
     assert torch.equal(st.y, y0) and torch.equal(st.dx, dx0) and torch.equal(st.dw, dw0)
 
 
+LINEAR_CASES = [c for c in CASES if c[0].startswith("linear")]
+
+
+@pytest.mark.parametrize("name,make", LINEAR_CASES, ids=[c[0] for c in LINEAR_CASES])
+def test_linear_fused_dequant_parity(name, make):
+    """Without the int32 copy, grad_input is dequantized in the GEMM epilogue; same results."""
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    ref = run_oracle(w)
+    st = LayerStep(w, keep_acc=False)
+    st.step()
+    torch.cuda.synchronize()
+    assert np.array_equal(st.y.cpu().numpy(), ref["y"])
+    a_mag = np.zeros(ref["dx"].shape)
+    c_mag = np.zeros(ref["dx"].shape)
+    psq, rpg = ref["psq"], st.rpg
+    cs = om.colsum_sign(w["w"])
+    for s_, g in enumerate(psq["kept"]):
+        rows = slice(g * rpg, (g + 1) * rpg)
+        a_mag[rows] = np.abs(np.float64(psq["scale"][s_]) * ref["acc_dx"][s_ * rpg:(s_ + 1) * rpg])
+        c_mag[rows] = np.abs(np.float64(psq["zero"][s_]) * cs)[None, :]
+    assert_dequant_close(st.dx.cpu().numpy(), ref["dx"], a_mag, c_mag, "grad_input (fused)")
+    pruned = np.setdiff1d(np.arange(st.M // rpg), psq["kept"])
+    dx = st.dx.cpu().numpy()
+    for g in pruned:
+        assert np.all(dx[g * rpg:(g + 1) * rpg] == 0)
+
+
 def test_single_branch_entry_point_matches_scq():
     """fqt1_agp_quantize_grad on one axis equals that branch of fqt1_scq_quantize."""
     from paper_2408_14267_gb300 import fqt1
