@@ -150,6 +150,28 @@ fqt1_status fqt1_scq_quantize(const float* g, int64_t M, int64_t D, const float*
                               fqt1_qgrad* psq, fqt1_qgrad* pcq, void* ws, size_t ws_bytes, int32_t* dev_status,
                               void* stream);
 
+/* Allocation-free fqt1_scq_quantize.  The paper has no counterpart: this only
+ * changes where the scratch memory lives.  It is meant for callers that cannot
+ * allocate device memory when they quantize (a plugin interface that only
+ * passes in the tensors, or a memory pool frozen after warm-up), so they cannot
+ * supply `ws`.  The range-pass scratch is instead a fixed array of
+ * FQT1_NOALLOC_SCRATCH_KEYS uint32 (64 KiB) inside the library, held on every
+ * device that loads it until the process exits.
+ *  - Sizes: 2 * (M / rows_per_group) + 2 * D must not exceed
+ *    FQT1_NOALLOC_SCRATCH_KEYS; larger calls return FQT1_ERR_UNSUPPORTED and
+ *    fqt1_last_cuda_error() names the limit.
+ *  - The first call on a device (the device current on the calling thread,
+ *    which must own `stream`) looks up the array's device address; make that
+ *    first call before any stream capture.
+ *  - Every call uses the same array and resets the part it needs; calls whose
+ *    work overlaps on the GPU (concurrent streams) race on it.
+ *  - Allocates nothing: no cudaMalloc / cudaFree or allocating library call.
+ * All other arguments, results and errors are those of fqt1_scq_quantize. */
+#define FQT1_NOALLOC_SCRATCH_KEYS 16384
+fqt1_status fqt1_scq_quantize_noalloc(const float* g, int64_t M, int64_t D, const float* gamma,
+                                      const fqt1_agp_params* p_sample, const fqt1_agp_params* p_channel,
+                                      fqt1_qgrad* psq, fqt1_qgrad* pcq, int32_t* dev_status, void* stream);
+
 /* grad_input side of SCQ (Eq. 21 with Sec. 5.3's per-sample scales):
  * acc[r, k] = sum_j q[r, j] sign(W)[j, k] over the kept rows r (kept order),
  * dx[m, k] = S'_g acc + Z'_g colsum_w[k] for rows of kept groups, 0 for

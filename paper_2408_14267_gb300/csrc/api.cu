@@ -15,6 +15,8 @@ void fqt1_set_cuda_error(cudaError_t e) {
 
 extern "C" const char* fqt1_last_cuda_error(void) { return g_last_error; }
 
+void fqt1_set_error_text(const char* msg) { snprintf(g_last_error, sizeof(g_last_error), "%s", msg); }
+
 static std::atomic<int64_t> g_launches{0};
 void fqt1_count_launches(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 extern "C" int64_t fqt1_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }

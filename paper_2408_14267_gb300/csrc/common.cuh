@@ -81,5 +81,7 @@ __device__ __forceinline__ uint32_t sr_code(float x, float z, float inv, float B
   } while (0)
 
 void fqt1_set_cuda_error(cudaError_t e);
+// Replaces the text returned by fqt1_last_cuda_error() with msg.
+void fqt1_set_error_text(const char* msg);
 // Adds n to the count returned by fqt1_kernel_launches().
 void fqt1_count_launches(int n);

@@ -7,6 +7,9 @@
 //   quantize_kernel  second read of G: stochastic rounding of the kept sample
 //                    groups (PSQ codes, row-major) and kept channels (PCQ codes,
 //                    written transposed through shared memory).
+#include <mutex>
+#include <stdio.h>
+
 #include "common.cuh"
 
 namespace fqt1 {
@@ -569,4 +572,59 @@ extern "C" fqt1_status fqt1_scq_quantize(const float* g, int64_t M, int64_t D, c
   if (!psq || !pcq) return FQT1_ERR_INVALID_ARG;
   return quantize_impl(g, M, D, gamma, p_sample, psq, p_channel, pcq, ws, ws_bytes, dev_status,
                        (cudaStream_t)stream);
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of fqt1_scq_quantize.
+//
+// Some callers cannot hand this library a workspace: a plugin interface that
+// passes only the input and output tensors, or a training loop whose device
+// memory pool is frozen after warm-up so that nothing may call cudaMalloc on
+// the step path.  For them the scratch of the range pass (the ordered min / max
+// keys of every sample group and channel) lives in a fixed array compiled into
+// this library instead of a caller buffer.  The array is shared by every call on
+// a device and keeps what the last call left in it; the keys are reset at the
+// start of each call, so only calls that overlap on the GPU (e.g. on two
+// streams at once) interfere, and such calls race.
+static __device__ __align__(256) uint32_t g_scq_scratch[FQT1_NOALLOC_SCRATCH_KEYS];
+
+static std::mutex g_scq_scratch_mu;
+static void* g_scq_scratch_dev[64];  // device address of g_scq_scratch, per device ordinal
+
+// Device address of the scratch array on the calling thread's current device.
+// The first call on a device looks it up (cudaGetSymbolAddress) and caches it.
+static fqt1_status scq_scratch_address(void** out) {
+  int dev = -1;
+  FQT1_CUDA_TRY(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= 64) return FQT1_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_scq_scratch_mu);
+  if (!g_scq_scratch_dev[dev]) {
+    void* p = nullptr;
+    FQT1_CUDA_TRY(cudaGetSymbolAddress(&p, g_scq_scratch));
+    g_scq_scratch_dev[dev] = p;
+  }
+  *out = g_scq_scratch_dev[dev];
+  return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_scq_quantize_noalloc(const float* g, int64_t M, int64_t D, const float* gamma,
+                                                 const fqt1_agp_params* p_sample, const fqt1_agp_params* p_channel,
+                                                 fqt1_qgrad* psq, fqt1_qgrad* pcq, int32_t* dev_status,
+                                                 void* stream) {
+  if (!psq || !pcq || !p_sample || !p_channel || M < 1 || D < 1 || p_sample->rows_per_group < 1)
+    return FQT1_ERR_INVALID_ARG;
+  const int64_t keys = 2 * (M / p_sample->rows_per_group) + 2 * D;
+  if (keys > FQT1_NOALLOC_SCRATCH_KEYS) {
+    char msg[200];
+    snprintf(msg, sizeof(msg),
+             "fqt1_scq_quantize_noalloc: 2*(M/rows_per_group) + 2*D = %lld keys exceed the built-in scratch of %d",
+             (long long)keys, (int)FQT1_NOALLOC_SCRATCH_KEYS);
+    fqt1_set_error_text(msg);
+    return FQT1_ERR_UNSUPPORTED;
+  }
+  void* scratch = nullptr;
+  const fqt1_status st = scq_scratch_address(&scratch);
+  if (st != FQT1_OK) return st;
+  return quantize_impl(g, M, D, gamma, p_sample, psq, p_channel, pcq, scratch,
+                       sizeof(uint32_t) * FQT1_NOALLOC_SCRATCH_KEYS, dev_status, (cudaStream_t)stream);
 }

@@ -47,6 +47,7 @@ _SIGS = {
     "fqt1_fwd_gemm": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
     "fqt1_agp_quantize_grad": (C.c_int, [_VP, _I64, _I64, _I32, _VP, _VP, _VP, _VP, C.c_size_t, _VP, _VP]),
     "fqt1_scq_quantize": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, C.c_size_t, _VP, _VP]),
+    "fqt1_scq_quantize_noalloc": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, _VP]),
     "fqt1_bwd_input_gemm": (C.c_int, [_VP, _VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
     "fqt1_col2im": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
     "fqt1_bwd_weight_gemm": (C.c_int, [_VP, _VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP, C.c_size_t, _VP]),
@@ -142,6 +143,14 @@ def scq_quantize(g, M, D, gamma, p_sample, p_channel, psq, pcq, ws, dev_status, 
     _check(lib().fqt1_scq_quantize(_p(g), M, D, _p(gamma), C.byref(p_sample), C.byref(p_channel), C.byref(psq.c),
                                    C.byref(pcq.c), _p(ws), ws.numel() * ws.element_size(), _p(dev_status),
                                    _s(stream)), "fqt1_scq_quantize")
+
+
+def scq_quantize_noalloc(g, M, D, gamma, p_sample, p_channel, psq, pcq, dev_status, stream=None):
+    """fqt1_scq_quantize without a workspace argument: the scratch is a fixed array inside
+    the library, for callers that cannot allocate device memory at this point."""
+    _check(lib().fqt1_scq_quantize_noalloc(_p(g), M, D, _p(gamma), C.byref(p_sample), C.byref(p_channel),
+                                           C.byref(psq.c), C.byref(pcq.c), _p(dev_status), _s(stream)),
+           "fqt1_scq_quantize_noalloc")
 
 
 def bwd_input_gemm(psq, sw_col, colsum_w, M, D, K, params, acc, dx, stream=None):

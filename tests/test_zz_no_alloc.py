@@ -1,0 +1,73 @@
+"""The allocation-free SCQ entry point (fqt1_scq_quantize_noalloc) against fqt1_scq_quantize.
+
+Callers that cannot allocate device memory where they quantize (a plugin
+interface that only hands over tensors, a memory pool frozen after warm-up)
+cannot pass a workspace; this entry point keeps its scratch in a fixed array
+inside the library instead.  Its results must equal those of the workspace
+entry point bit for bit (integers, ranges, probabilities, scales, codes), on
+consecutive calls that reuse the same array.  This file is collected last.
+"""
+import ctypes as C
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2408_14267_gb300 import build
+    build.build()
+
+
+def _branches_equal(a, b, rows):
+    c = a.count()
+    assert c == b.count()
+    for name in ("group_min", "group_range", "p_hat", "slot_of_group"):
+        assert torch.equal(getattr(a, name), getattr(b, name)), name
+    assert torch.equal(a.kept_idx[: a.capacity], b.kept_idx[: b.capacity])
+    assert torch.equal(a.scale[:c], b.scale[:c]) and torch.equal(a.zero[:c], b.zero[:c])
+    assert torch.equal(a.codes[: c * rows], b.codes[: c * rows])
+
+
+def _run_both(w):
+    from paper_2408_14267_gb300 import fqt1
+    from paper_2408_14267_gb300.layer import LayerStep
+    st = LayerStep(w)
+    st.dev_status.zero_()
+    fqt1.scq_quantize(st.gy, st.M, st.D, st.gamma, st.p_s, st.p_c, st.psq, st.pcq, st.ws, st.dev_status)
+    psq = fqt1.QGradBuffers(st.psq.n, st.psq.capacity, st.psq.capacity * st.rpg, st.D)
+    pcq = fqt1.QGradBuffers(st.pcq.n, st.pcq.capacity, st.pcq.capacity, st.M)
+    status = torch.zeros(4, dtype=torch.int32, device="cuda")
+    fqt1.scq_quantize_noalloc(st.gy, st.M, st.D, st.gamma, st.p_s, st.p_c, psq, pcq, status)
+    torch.cuda.synchronize()
+    assert int(status[0].item()) == int(st.dev_status[0].item()) == 0
+    _branches_equal(psq, st.psq, st.rpg)
+    _branches_equal(pcq, st.pcq, 1)
+
+
+def test_noalloc_matches_workspace_entry_point_on_consecutive_calls():
+    from paper_2408_14267_gb300 import workloads as wl
+    # first call: the 8192 x 256 conv gradient (128 sample groups of 64 rows)
+    _run_both(wl.resnet18_cifar_conv())
+    # second call on the same scratch: a different shape, grouping and bit width
+    _run_both(wl.linear_small())
+
+
+def test_noalloc_rejects_sizes_beyond_the_scratch():
+    from paper_2408_14267_gb300 import fqt1
+    L = fqt1.lib()
+    fake = C.c_void_p(0x10000)  # never dereferenced: the size check comes first
+    ps = fqt1.AgpParams(2, 0, 1, 1)
+    pc = fqt1.AgpParams(2, 0, 2, 1)
+    q = fqt1.QGrad(*(0x10000 for _ in range(9)), 1 << 16)
+    # 2 * 8192 sample groups + 2 * 64 channels > 16384 keys
+    st = L.fqt1_scq_quantize_noalloc(fake, 8192, 64, None, C.byref(ps), C.byref(pc), C.byref(q), C.byref(q), fake,
+                                     C.c_void_p(0))
+    assert st == 3
+    assert b"exceed the built-in scratch" in L.fqt1_last_cuda_error()
