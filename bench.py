@@ -153,6 +153,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="fqt1", choices=["fqt1", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile", type=int, default=0, metavar="N",
+                    help="only run --warmup + N eager steps (for ncu), print nothing")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -176,6 +178,12 @@ def main():
     wl = workloads.resnet18_cifar_conv()
     st = LayerStep(wl, device=f"cuda:{local_rank}", keep_acc=False)
     stream = torch.cuda.Stream()
+    if args.profile:
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup + args.profile):
+                st.step()
+        torch.cuda.synchronize()
+        return
     flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device="cuda")  # 256 MiB > 129 MB L2
     stages = st.stages()
     with torch.cuda.stream(stream):
@@ -188,7 +196,7 @@ def main():
         launches_per_step = fqt1.kernel_launches() - n0
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph, stream=stream):
-            st.step()
+            st.step_concurrent(stream)
         for _ in range(args.warmup):
             graph.replay()
         stream.synchronize()
@@ -312,7 +320,9 @@ def main():
                 "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "b1", "data": "synthetic",
                 "config": {"workload": WORKLOAD, "l2": "flushed before every timed step (256 MiB write)",
-                           "timing": "CUDA-graph replay of the whole step, CUDA events on the launching stream",
+                           "timing": "CUDA-graph replay of the whole step (three stream branches: pack W | "
+                                     "pack X + forward + grad_weight | SCQ + grad_input + Folder), CUDA events "
+                                     "on the launching stream",
                            "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU"},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
                 "clocks": clocks, "stage_ms": {k: round(v, 5) for k, v in stage_ms.items()}}

@@ -107,6 +107,102 @@ __global__ void col2im_kernel(const int32_t* __restrict__ acc, const int32_t* __
   dx[idx] = v;
 }
 
+// Folder with the accumulators staged in shared memory.  A CTA owns sample n, channels
+// [c0, c0+cb) and input rows [h0, h0+hb): it loads, coalesced, the int32 accumulator rows of
+// every output pixel whose window touches those input rows (their k-range of the block's
+// channels), then sums the taps of each input pixel from shared memory.  Row stride of the
+// tile is odd so that neighbouring pixels fall in different banks.
+struct FoldArgs {
+  const int32_t* acc;
+  const int32_t* slot_of_group;
+  const float* scale;
+  const float* zero;
+  const int32_t* cs;
+  float* dx;
+  int N, C, H, W, kh, kw, stride, pad, Ho, Wo;
+  int cb, hb, ncb, max_rows, kstride;
+  int64_t K;
+};
+
+__global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
+  extern __shared__ int32_t fold_smem[];
+  const int n = blockIdx.y;
+  const int cblk = blockIdx.x % a.ncb, hblk = blockIdx.x / a.ncb;
+  const int c0 = cblk * a.cb, h0 = hblk * a.hb;
+  const int c1 = min(a.C, c0 + a.cb), h1 = min(a.H, h0 + a.hb);
+  const int nc = c1 - c0, nh = h1 - h0;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int32_t slot = __ldg(a.slot_of_group + n);
+  const int plane = nh * a.W;  // contiguous floats of one channel inside the block
+  if (slot < 0) {
+    for (int cl = 0; cl < nc; ++cl) {
+      float* dst = a.dx + (((int64_t)n * a.C + c0 + cl) * a.H + h0) * a.W;
+      for (int x = threadIdx.x; x < plane; x += blockDim.x) dst[x] = 0.0f;
+    }
+    return;
+  }
+  const int khw = a.kh * a.kw;
+  int oh_lo = h0 + a.pad - (a.kh - 1);
+  oh_lo = oh_lo <= 0 ? 0 : (oh_lo + a.stride - 1) / a.stride;
+  const int oh_hi = min(a.Ho - 1, (h1 - 1 + a.pad) / a.stride);
+  const int nrows = oh_hi - oh_lo + 1;
+  const int kb = nc * khw;
+  int32_t* tile = fold_smem;                                   // [max_rows * Wo][kstride]
+  int32_t* hrow = tile + a.max_rows * a.Wo * a.kstride;        // [hb * kh]: pixel-row offset or -1
+  int32_t* wcol = hrow + a.hb * a.kh;                          // [W * kw]: output column or -1
+  int32_t* css = wcol + a.W * a.kw;                            // [cb * khw]: colsum of the block
+  for (int x = threadIdx.x; x < nh * a.kh; x += blockDim.x) {
+    const int hl = x / a.kh, i = x - hl * a.kh;
+    const int hn = h0 + hl + a.pad - i;
+    int v = -1;
+    if (hn >= 0 && hn % a.stride == 0) {
+      const int oh = hn / a.stride;
+      if (oh >= oh_lo && oh <= oh_hi) v = (oh - oh_lo) * a.Wo;
+    }
+    hrow[x] = v;
+  }
+  for (int x = threadIdx.x; x < a.W * a.kw; x += blockDim.x) {
+    const int w = x / a.kw, j = x - w * a.kw;
+    const int wn = w + a.pad - j;
+    int v = -1;
+    if (wn >= 0 && wn % a.stride == 0 && wn / a.stride < a.Wo) v = wn / a.stride;
+    wcol[x] = v;
+  }
+  const int64_t kbase = (int64_t)c0 * khw;
+  for (int x = threadIdx.x; x < kb; x += blockDim.x) css[x] = __ldg(a.cs + kbase + x);
+  if (nrows > 0) {
+    const int npix = nrows * a.Wo;
+    const int64_t rbase = (int64_t)slot * a.Ho * a.Wo + (int64_t)oh_lo * a.Wo;
+    for (int pix = warp; pix < npix; pix += blockDim.x >> 5) {
+      const int32_t* src = a.acc + (rbase + pix) * a.K + kbase;
+      int32_t* dst = tile + pix * a.kstride;
+      for (int kk = lane; kk < kb; kk += 32) dst[kk] = __ldg(src + kk);
+    }
+  }
+  __syncthreads();
+  const float sc = __ldg(a.scale + slot), ze = __ldg(a.zero + slot);
+  const int outs = nc * plane;
+  for (int e = threadIdx.x; e < outs; e += blockDim.x) {
+    const int cl = e / plane, rem = e - cl * plane;
+    const int hl = rem / a.W, w = rem - hl * a.W;
+    const int kc = cl * khw;
+    int32_t acc = 0, csum = 0;
+    for (int i = 0; i < a.kh; ++i) {
+      const int ro = hrow[hl * a.kh + i];
+      if (ro < 0) continue;
+      for (int j = 0; j < a.kw; ++j) {
+        const int co = wcol[w * a.kw + j];
+        if (co < 0) continue;
+        const int kk = kc + i * a.kw + j;
+        acc += tile[(ro + co) * a.kstride + kk];
+        csum += css[kk];
+      }
+    }
+    a.dx[(((int64_t)n * a.C + c0 + cl) * a.H + h0 + hl) * a.W + w] =
+        __fadd_rn(__fmul_rn(sc, __int2float_rn(acc)), __fmul_rn(ze, __int2float_rn(csum)));
+  }
+}
+
 }  // namespace fqt1
 
 using namespace fqt1;
@@ -135,6 +231,7 @@ extern "C" fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t
   if (!psq || !sw_col || !p || M < 1 || D < 1 || K < 1 || (!acc && !dx)) return FQT1_ERR_INVALID_ARG;
   if (!valid_bits(p->bits) || p->rows_per_group < 1 || M % p->rows_per_group) return FQT1_ERR_INVALID_ARG;
   if (dx && !colsum_w) return FQT1_ERR_INVALID_ARG;
+  if (colsum_w && !aligned16(colsum_w)) return FQT1_ERR_MISALIGNED;
   if (!psq->codes || !psq->kept_count || !psq->slot_of_group || !psq->scale || !psq->zero ||
       psq->ld_codes < fqt1_codes_ld(D) || psq->ld_codes % 16)
     return FQT1_ERR_INVALID_ARG;
@@ -182,9 +279,43 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
   const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
   if (H + 2 * pad < kh || W + 2 * pad < kw) return FQT1_ERR_INVALID_ARG;
   if (!aligned16(acc) || !aligned16(dx)) return FQT1_ERR_MISALIGNED;
-  const int64_t n = (int64_t)N * C * H * W;
-  col2im_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(
-      acc, psq->slot_of_group, psq->scale, psq->zero, colsum_w, N, C, H, W, kh, kw, stride, pad, Ho, Wo, dx);
+  // tiled Folder: choose input rows and channels per CTA so that the staged accumulators fit
+  constexpr int64_t kMaxTile = 96 * 1024;
+  const int khw = kh * kw;
+  int hb = H < 8 ? H : 8, cb = 0;
+  int max_rows = 0, kstride = 0;
+  for (; hb >= 1 && cb == 0; hb /= 2) {
+    max_rows = (hb - 1 + kh - 1) / stride + 1;
+    if (max_rows > Ho) max_rows = Ho;
+    for (int c = (C < 32 ? C : 32); c >= 1; c = (c > 1 ? c / 2 : 0)) {
+      const int ks = (c * khw) | 1;
+      const int64_t words = (int64_t)max_rows * Wo * ks + (int64_t)hb * kh + (int64_t)W * kw + (int64_t)c * khw;
+      if (words * 4 <= kMaxTile) { cb = c; kstride = ks; break; }
+    }
+    if (cb) break;
+  }
+  if (cb > 0) {
+    static bool attr = false;
+    if (!attr) {
+      FQT1_CUDA_TRY(cudaFuncSetAttribute(col2im_tiled_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kMaxTile));
+      attr = true;
+    }
+    FoldArgs fa;
+    fa.acc = acc; fa.slot_of_group = psq->slot_of_group; fa.scale = psq->scale; fa.zero = psq->zero;
+    fa.cs = colsum_w; fa.dx = dx; fa.N = N; fa.C = C; fa.H = H; fa.W = W; fa.kh = kh; fa.kw = kw;
+    fa.stride = stride; fa.pad = pad; fa.Ho = Ho; fa.Wo = Wo; fa.cb = cb; fa.hb = hb;
+    fa.ncb = (C + cb - 1) / cb; fa.max_rows = max_rows; fa.kstride = kstride; fa.K = (int64_t)C * khw;
+    const int64_t nblk = (int64_t)fa.ncb * ((H + hb - 1) / hb);
+    if (nblk > 0x7FFFFFFF || N > 65535) return FQT1_ERR_UNSUPPORTED;
+    const size_t smem =
+        ((size_t)max_rows * Wo * kstride + (size_t)hb * kh + (size_t)W * kw + (size_t)cb * khw) * 4;
+    col2im_tiled_kernel<<<dim3((unsigned)nblk, (unsigned)N), 256, smem, (cudaStream_t)stream>>>(fa);
+  } else {
+    const int64_t n = (int64_t)N * C * H * W;
+    col2im_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(
+        acc, psq->slot_of_group, psq->scale, psq->zero, colsum_w, N, C, H, W, kh, kw, stride, pad, Ho, Wo, dx);
+  }
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
   return FQT1_OK;

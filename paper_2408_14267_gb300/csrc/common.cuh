@@ -47,6 +47,20 @@ __device__ __forceinline__ uint32_t philox_word(uint64_t seed, uint32_t stream, 
   }
 }
 
+// Division of 32-bit unsigned n < 2^31 by an invariant d >= 1 with one multiply-high
+// (Granlund and Montgomery, "Division by invariant integers using multiplication",
+// PLDI'94): with l = ceil(log2 d) and m = floor(2^32 (2^l - d) / d) + 1,
+// n / d = (umulhi(n, m) + n) >> l.  The host computes m and l.
+struct FastDiv {
+  uint32_t d, mul, shr;
+  FastDiv() : d(1), mul(1), shr(0) {}
+  explicit FastDiv(uint32_t divisor) : d(divisor), mul(0), shr(0) {
+    while (shr < 31 && (1u << shr) < d) ++shr;
+    mul = (uint32_t)((((uint64_t)1 << 32) * (((uint64_t)1 << shr) - d)) / d + 1);
+  }
+  __device__ __forceinline__ uint32_t div(uint32_t n) const { return (__umulhi(n, mul) + n) >> shr; }
+};
+
 // Order-preserving map float -> uint32 (so atomicMin/atomicMax give float min/max).
 __device__ __forceinline__ uint32_t float_to_ordered(float f) {
   const uint32_t b = __float_as_uint(f);

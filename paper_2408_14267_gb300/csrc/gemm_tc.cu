@@ -9,11 +9,16 @@
 // both digits exact, products are exact, and every partial sum is an integer
 // below 2^24 so the fp32 accumulator in TMEM holds it exactly.
 //
-// Pipeline per CTA (one 128 x BN output tile, 128-element K steps):
-//   warp 0 lane 0   TMA: raw tiles (packed words or codes) -> shared memory
-//   warp 1          TMEM allocation; lane 0 issues tcgen05.mma, commits stages
-//   warps 2..5      expand raw tiles into 128B-swizzled e4m3 operand tiles,
-//                   then run the epilogue from TMEM (each warp owns 32 lanes)
+// Pipeline per CTA (one 128 x BN output tile, 128-element K steps), two rings:
+//   raw ring (deep)    TMA writes the raw tiles: packed sign words (16 bytes per row)
+//                      or uint8 codes (128B-swizzled box)
+//   operand ring       e4m3 tiles in the 128B-swizzle K-major layout the MMA reads
+//   warp 0 lane 0   TMA producer of the raw ring
+//   warp 1          TMEM allocation; lane 0 issues tcgen05.mma, commits operand stages
+//   warps 2..9      expand raw -> operand tiles (one row per thread and stage), then
+//                   the epilogue: TMEM -> registers -> swizzled per-warp staging ->
+//                   coalesced row stores (warp w owns TMEM lanes 32 (w % 4) .. +31 and
+//                   half of the columns)
 // Every wait is bounded; an expired wait sets FQT1_DEV_TIMEOUT and the CTA
 // drains and returns.
 #include <cuda.h>
@@ -25,8 +30,8 @@ namespace fqt1 {
 
 constexpr int kBM = 128;           // output rows per CTA (MMA M)
 constexpr int kBK = 128;           // contraction elements per stage (one 128-byte swizzle row of e4m3)
-constexpr int kStages = 4;
-constexpr int kExpWarps = 4;
+constexpr int kMaxStages = 8;
+constexpr int kExpWarps = 8;       // two expansion / epilogue warps per SM sub-partition
 constexpr int kThreads = 32 * (2 + kExpWarps);
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on every wait
 
@@ -81,13 +86,15 @@ __device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
 __device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, volatile int* abort_flag, int32_t* status) {
   if (mbar_test(b, parity)) return true;
   const uint64_t t0 = gtimer();
-  while (true) {
+  for (uint32_t n = 1;; ++n) {
     if (mbar_test(b, parity)) return true;
-    if (*abort_flag) return false;
-    if (gtimer() - t0 > kWaitNs) {
-      *abort_flag = 1;
-      if (status) atomicOr(status, FQT1_DEV_TIMEOUT);
-      return false;
+    if ((n & 1023u) == 0) {  // the timer and the abort flag are checked every 1024 polls
+      if (*abort_flag) return false;
+      if (gtimer() - t0 > kWaitNs) {
+        *abort_flag = 1;
+        if (status) atomicOr(status, FQT1_DEV_TIMEOUT);
+        return false;
+      }
     }
   }
 }
@@ -159,20 +166,27 @@ __device__ __forceinline__ uint32_t codes4_x16(uint32_t h) {
 
 template <bool A_CODES, bool BITS8, int BN>
 struct TcSmem {
-  static constexpr int kOpA = kBM * kBK;              // bytes of one e4m3 A tile
+  static constexpr int kOpA = kBM * kBK;                        // bytes of one e4m3 A tile
   static constexpr int kOpB = BN * kBK;
-  static constexpr int kRawA = A_CODES ? 0 : kBM * 16;  // packed words of A (4 per row)
+  static constexpr int kOpStage = kOpA * (BITS8 ? 2 : 1) + kOpB;
+  static constexpr int kRawA = A_CODES ? kBM * kBK : kBM * 16;  // codes, or packed words (4 per row)
   static constexpr int kRawB = BN * 16;
-  static constexpr int kStage = kOpA * (BITS8 ? 2 : 1) + kOpB + kRawA + kRawB;
-  static constexpr int kBytes = kStages * kStage + 1024;  // + alignment slack
+  static constexpr int kRawStage = kRawA + kRawB;
+  static constexpr int kOpStages = BITS8 ? 2 : (A_CODES ? 3 : 4);
+  static constexpr int kRawStages = A_CODES ? 4 : 8;
+  static constexpr int kBytes = kOpStages * kOpStage + kRawStages * kRawStage + 1024;  // + alignment slack
+  static_assert(kOpStage % 1024 == 0 && kRawStage % 1024 == 0, "stages keep 1024-byte alignment");
+  static_assert(kOpStages * kOpStage >= kExpWarps * 4096, "epilogue staging fits in the operand ring");
 };
 
 template <bool A_CODES, bool BITS8, int BN>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, TcArgs a) {
   using S = TcSmem<A_CODES, BITS8, BN>;
+  constexpr int OS = S::kOpStages, RS = S::kRawStages;
   extern __shared__ unsigned char smem_raw[];
-  __shared__ __align__(8) uint64_t raw_full[kStages], raw_empty[kStages], op_full[kStages], op_empty[kStages];
+  __shared__ __align__(8) uint64_t raw_full[kMaxStages], raw_empty[kMaxStages], op_full[kMaxStages],
+      op_empty[kMaxStages];
   __shared__ __align__(8) uint64_t acc_full;
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
@@ -187,20 +201,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nk = kt1 - kt0;
 
   unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  auto opA = [&](int s) { return base + s * S::kStage; };
-  auto opA2 = [&](int s) { return base + s * S::kStage + S::kOpA; };
-  auto opB = [&](int s) { return base + s * S::kStage + S::kOpA * (BITS8 ? 2 : 1); };
-  auto rawA = [&](int s) { return opB(s) + S::kOpB; };
-  auto rawB = [&](int s) { return rawA(s) + S::kRawA; };
+  auto opA = [&](int s) { return base + s * S::kOpStage; };
+  auto opA2 = [&](int s) { return base + s * S::kOpStage + S::kOpA; };
+  auto opB = [&](int s) { return base + s * S::kOpStage + S::kOpA * (BITS8 ? 2 : 1); };
+  unsigned char* raw_base = base + OS * S::kOpStage;
+  auto rawA = [&](int s) { return raw_base + s * S::kRawStage; };
+  auto rawB = [&](int s) { return raw_base + s * S::kRawStage + S::kRawA; };
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&raw_full[s], 1);
-      mbar_init(&raw_empty[s], kExpWarps);
-      mbar_init(&op_full[s], kExpWarps);
-      mbar_init(&op_empty[s], 1);
-    }
+    for (int s = 0; s < RS; ++s) { mbar_init(&raw_full[s], 1); mbar_init(&raw_empty[s], kExpWarps); }
+    for (int s = 0; s < OS; ++s) { mbar_init(&op_full[s], kExpWarps); mbar_init(&op_empty[s], 1); }
     mbar_init(&acc_full, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -214,42 +225,37 @@ __global__ void __launch_bounds__(kThreads, 1)
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = tmem_slot;
 
-  constexpr uint32_t kTxA = A_CODES ? (uint32_t)S::kOpA : (uint32_t)S::kRawA;
-  constexpr uint32_t kTx = kTxA + (uint32_t)S::kRawB;
+  constexpr uint32_t kTx = (uint32_t)S::kRawStage;
 
   if (warp == 0) {
-    // ---------------------------------------------------------------- TMA producer
+    // ---------------------------------------------------------------- TMA producer (raw ring)
     if (lane == 0) {
       int issued = 0;
       for (int i = 0; i < nk; ++i) {
-        const int s = i % kStages, it = i / kStages;
-        if (it > 0) {
-          if (!mbar_wait(&raw_empty[s], (it - 1) & 1, &abort_flag, a.status)) break;
-          if (A_CODES && !mbar_wait(&op_empty[s], (it - 1) & 1, &abort_flag, a.status)) break;
-        }
+        const int s = i % RS, it = i / RS;
+        if (it > 0 && !mbar_wait(&raw_empty[s], (it - 1) & 1, &abort_flag, a.status)) break;
         const int kt = kt0 + i;
         mbar_expect_tx(&raw_full[s], kTx);
-        if (A_CODES) tma_load_2d(opA(s), &tmA, &raw_full[s], kt * kBK, (int)m0);
+        if (A_CODES) tma_load_2d(rawA(s), &tmA, &raw_full[s], kt * kBK, (int)m0);
         else tma_load_2d(rawA(s), &tmA, &raw_full[s], kt * (kBK / 32), (int)m0);
         tma_load_2d(rawB(s), &tmB, &raw_full[s], kt * (kBK / 32), (int)n0);
         ++issued;
       }
       // drain: every issued copy must land before the CTA may exit
-      for (int i = (issued > kStages ? issued - kStages : 0); i < issued; ++i) {
-        const int s = i % kStages, it = i / kStages;
+      for (int i = (issued > RS ? issued - RS : 0); i < issued; ++i) {
+        const int s = i % RS, it = i / RS;
         const uint64_t t0 = gtimer();
         while (!mbar_test(&raw_full[s], it & 1) && gtimer() - t0 < kWaitNs) {
         }
       }
     }
   } else if (warp == 1) {
-    // ---------------------------------------------------------------- MMA issuer
+    // ---------------------------------------------------------------- MMA issuer (operand ring)
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_e4m3(BN);
-      bool ok = true;
       for (int i = 0; i < nk; ++i) {
-        const int s = i % kStages, it = i / kStages;
-        if (!mbar_wait(&op_full[s], it & 1, &abort_flag, a.status)) { ok = false; break; }
+        const int s = i % OS, it = i / OS;
+        if (!mbar_wait(&op_full[s], it & 1, &abort_flag, a.status)) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const uint32_t aaddr = smem_u32(opA(s)), a2addr = smem_u32(opA2(s)), baddr = smem_u32(opB(s));
 #pragma unroll
@@ -260,99 +266,95 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mma_commit(&op_empty[s]);
       }
-      (void)ok;
       mma_commit(&acc_full);
     }
   } else {
-    // ---------------------------------------------------------------- expansion
-    const int t = threadIdx.x - 64;  // 0..127
+    // ---------------------------------------------------------------- expansion (raw -> operand)
+    // threads 0..127 expand A row t, threads 128..255 expand B row t - 128 (BN = 128)
+    const int t = threadIdx.x - 64;  // 0..255
     for (int i = 0; i < nk; ++i) {
-      const int s = i % kStages, it = i / kStages;
-      if (it > 0 && !mbar_wait(&op_empty[s], (it - 1) & 1, &abort_flag, a.status)) break;
-      if (!mbar_wait(&raw_full[s], it & 1, &abort_flag, a.status)) break;
+      const int so = i % OS, ito = i / OS, sr = i % RS, itr = i / RS;
+      if (ito > 0 && !mbar_wait(&op_empty[so], (ito - 1) & 1, &abort_flag, a.status)) break;
+      if (!mbar_wait(&raw_full[sr], itr & 1, &abort_flag, a.status)) break;
       const int kt = kt0 + i;
-      // A tile: row t
-      if (A_CODES) {
-        unsigned char* ta = opA(s);
+      if (t < kBM) {
+        if (A_CODES) {
+          const unsigned char* ra = rawA(sr);
+          unsigned char* ta = opA(so);
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const uint32_t off = swz(t, c);
-          uint4 v = *reinterpret_cast<uint4*>(ta + off);
-          if (BITS8) {
-            uint4 lo, hi;
-            lo.x = codes4(v.x & 0x0F0F0F0Fu); hi.x = codes4_x16((v.x >> 4) & 0x0F0F0F0Fu);
-            lo.y = codes4(v.y & 0x0F0F0F0Fu); hi.y = codes4_x16((v.y >> 4) & 0x0F0F0F0Fu);
-            lo.z = codes4(v.z & 0x0F0F0F0Fu); hi.z = codes4_x16((v.z >> 4) & 0x0F0F0F0Fu);
-            lo.w = codes4(v.w & 0x0F0F0F0Fu); hi.w = codes4_x16((v.w >> 4) & 0x0F0F0F0Fu);
-            *reinterpret_cast<uint4*>(ta + off) = hi;
-            *reinterpret_cast<uint4*>(opA2(s) + off) = lo;
-          } else {
-            v.x = codes4(v.x); v.y = codes4(v.y); v.z = codes4(v.z); v.w = codes4(v.w);
-            *reinterpret_cast<uint4*>(ta + off) = v;
+          for (int c = 0; c < 8; ++c) {
+            const uint32_t off = swz(t, c);  // TMA wrote the codes with the same 128B swizzle
+            uint4 v = *reinterpret_cast<const uint4*>(ra + off);
+            if (BITS8) {
+              uint4 lo, hi;
+              lo.x = codes4(v.x & 0x0F0F0F0Fu); hi.x = codes4_x16((v.x >> 4) & 0x0F0F0F0Fu);
+              lo.y = codes4(v.y & 0x0F0F0F0Fu); hi.y = codes4_x16((v.y >> 4) & 0x0F0F0F0Fu);
+              lo.z = codes4(v.z & 0x0F0F0F0Fu); hi.z = codes4_x16((v.z >> 4) & 0x0F0F0F0Fu);
+              lo.w = codes4(v.w & 0x0F0F0F0Fu); hi.w = codes4_x16((v.w >> 4) & 0x0F0F0F0Fu);
+              *reinterpret_cast<uint4*>(ta + off) = hi;
+              *reinterpret_cast<uint4*>(opA2(so) + off) = lo;
+            } else {
+              v.x = codes4(v.x); v.y = codes4(v.y); v.z = codes4(v.z); v.w = codes4(v.w);
+              *reinterpret_cast<uint4*>(ta + off) = v;
+            }
+          }
+        } else {
+          const uint4 w4 = *reinterpret_cast<const uint4*>(rawA(sr) + 16 * t);
+          const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+          unsigned char* ta = opA(so);
+          const int64_t kbase = (int64_t)kt * kBK;
+          const bool full = kbase + kBK <= a.L;
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              uint4 v = signs16(wv[w] >> (16 * h));
+              if (!full) {  // elements past the contraction length contribute 0
+                const int64_t e0 = kbase + 32 * w + 16 * h;
+                uint32_t* vv = reinterpret_cast<uint32_t*>(&v);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                  for (int bb = 0; bb < 4; ++bb)
+                    if (e0 + 4 * q + bb >= a.L) vv[q] &= ~(0xFFu << (8 * bb));
+                }
+              }
+              *reinterpret_cast<uint4*>(ta + swz(t, 2 * w + h)) = v;
+            }
           }
         }
       } else {
-        const uint4 w4 = *reinterpret_cast<const uint4*>(rawA(s) + 16 * t);
-        const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
-        unsigned char* ta = opA(s);
-        const int64_t kbase = (int64_t)kt * kBK;
-        const bool full = kbase + kBK <= a.L;
 #pragma unroll
-        for (int w = 0; w < 4; ++w) {
+        for (int rr = 0; rr < BN / kBM; ++rr) {
+          const int r = t - kBM + kBM * rr;
+          const uint4 w4 = *reinterpret_cast<const uint4*>(rawB(sr) + 16 * r);
+          const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+          unsigned char* tb = opB(so);
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            uint4 v = signs16(wv[w] >> (16 * h));
-            if (!full) {  // elements past the contraction length contribute 0
-              const int64_t e0 = kbase + 32 * w + 16 * h;
-              uint32_t* vv = reinterpret_cast<uint32_t*>(&v);
-#pragma unroll
-              for (int q = 0; q < 4; ++q) {
-#pragma unroll
-                for (int bb = 0; bb < 4; ++bb)
-                  if (e0 + 4 * q + bb >= a.L) vv[q] &= ~(0xFFu << (8 * bb));
-              }
-            }
-            *reinterpret_cast<uint4*>(ta + swz(t, 2 * w + h)) = v;
+          for (int w = 0; w < 4; ++w) {
+            *reinterpret_cast<uint4*>(tb + swz(r, 2 * w)) = signs16(wv[w]);
+            *reinterpret_cast<uint4*>(tb + swz(r, 2 * w + 1)) = signs16(wv[w] >> 16);
           }
-        }
-      }
-      // B tile: rows t, t + 128, ...
-#pragma unroll
-      for (int rr = 0; rr < BN / kBM; ++rr) {
-        const int r = t + kBM * rr;
-        const uint4 w4 = *reinterpret_cast<const uint4*>(rawB(s) + 16 * r);
-        const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
-        unsigned char* tb = opB(s);
-#pragma unroll
-        for (int w = 0; w < 4; ++w) {
-          *reinterpret_cast<uint4*>(tb + swz(r, 2 * w)) = signs16(wv[w]);
-          *reinterpret_cast<uint4*>(tb + swz(r, 2 * w + 1)) = signs16(wv[w] >> 16);
         }
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       __syncwarp();
       if (lane == 0) {
-        mbar_arrive(&op_full[s]);
-        mbar_arrive(&raw_empty[s]);
+        mbar_arrive(&op_full[so]);
+        mbar_arrive(&raw_empty[sr]);
       }
     }
 
     // ---------------------------------------------------------------- epilogue
+    // TMEM -> registers (thread = row) -> per-warp swizzled staging (32 x 32 words) ->
+    // one coalesced 128-byte row per store instruction (lane = column).
     const bool have_acc = mbar_wait(&acc_full, 0, &abort_flag, a.status);
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    const int q = warp & 3;  // TMEM lane quarter of this warp
-    const int64_t r = m0 + 32 * q + lane;
-    const bool row_ok = have_acc && r < valid_rows && r < a.M;
-    int64_t out_row = r;
-    float sc = 0.f, ze = 0.f;
-    if (a.epi == EPI_DX && row_ok) {
-      const int64_t slot = r / a.rpg;
-      out_row = (int64_t)__ldg(a.kept_idx + slot) * a.rpg + (r - slot * a.rpg);
-      sc = __ldg(a.scale + slot);
-      ze = __ldg(a.zero + slot);
-    }
-    const bool vec = (a.ldo % 4) == 0;
-    for (int c0 = 0; c0 < BN; c0 += 32) {
+    const int q = warp & 3;                         // TMEM lane quarter of this warp
+    const int cbeg = ((warp - 2) >> 2) * (BN / 2);  // its half of the accumulator columns
+    uint32_t* stage = reinterpret_cast<uint32_t*>(base) + (warp - 2) * 1024;  // 4 KB per warp (operand ring is idle)
+    const int64_t row_base = m0 + 32 * q;
+    for (int c0 = cbeg; c0 < cbeg + BN / 2; c0 += 32) {
       __syncwarp();
       uint32_t v[32];
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)c0;
@@ -365,58 +367,88 @@ __global__ void __launch_bounds__(kThreads, 1)
             "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
           : "r"(taddr));
       asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-      if (!row_ok) continue;
-      const int64_t nb = n0 + c0;
-      if (nb >= a.N) continue;
-      int32_t iv[32];
+      if (!have_acc) continue;
+      if (a.epi != EPI_RED) {
+        // direct stores: this thread's row, 32 consecutive columns
+        const int64_t r = row_base + lane;
+        const int64_t nb = n0 + c0;
+        if (r >= valid_rows || r >= a.M || nb >= a.N) continue;
+        int32_t iv[32];
 #pragma unroll
-      for (int j = 0; j < 32; ++j) iv[j] = __float2int_rn(__uint_as_float(v[j]));
-      const bool full = nb + 32 <= a.N && vec;
-      if (a.epi == EPI_FWD) {
-        float* yrow = a.y + out_row * a.ldo + nb;
-        if (full) {
+        for (int j = 0; j < 32; ++j) iv[j] = __float2int_rn(__uint_as_float(v[j]));
+        const bool full = nb + 32 <= a.N && (a.ldo % 4) == 0;
+        int64_t out_row = r;
+        float sc = 0.f, ze = 0.f;
+        if (a.epi == EPI_DX) {
+          const int64_t slot = r / a.rpg;
+          out_row = (int64_t)__ldg(a.kept_idx + slot) * a.rpg + (r - slot * a.rpg);
+          sc = __ldg(a.scale + slot);
+          ze = __ldg(a.zero + slot);
+        }
+        if (a.epi == EPI_FWD) {
+          float* yrow = a.y + out_row * a.ldo + nb;
+          if (full) {
 #pragma unroll
-          for (int j = 0; j < 32; j += 4) {
-            float4 o;
-            o.x = __fmul_rn(__ldg(a.gamma + nb + j + 0), (float)iv[j + 0]);
-            o.y = __fmul_rn(__ldg(a.gamma + nb + j + 1), (float)iv[j + 1]);
-            o.z = __fmul_rn(__ldg(a.gamma + nb + j + 2), (float)iv[j + 2]);
-            o.w = __fmul_rn(__ldg(a.gamma + nb + j + 3), (float)iv[j + 3]);
-            *reinterpret_cast<float4*>(yrow + j) = o;
-            if (a.acc) *reinterpret_cast<int4*>(a.acc + out_row * a.ldo + nb + j) = make_int4(iv[j], iv[j + 1], iv[j + 2], iv[j + 3]);
+            for (int j = 0; j < 32; j += 4) {
+              const float4 g4 = __ldg(reinterpret_cast<const float4*>(a.gamma + nb + j));
+              *reinterpret_cast<float4*>(yrow + j) =
+                  make_float4(__fmul_rn(g4.x, (float)iv[j]), __fmul_rn(g4.y, (float)iv[j + 1]),
+                              __fmul_rn(g4.z, (float)iv[j + 2]), __fmul_rn(g4.w, (float)iv[j + 3]));
+              if (a.acc)
+                *reinterpret_cast<int4*>(a.acc + out_row * a.ldo + nb + j) = make_int4(iv[j], iv[j + 1], iv[j + 2], iv[j + 3]);
+            }
+          } else {
+            for (int j = 0; j < 32 && nb + j < a.N; ++j) {
+              yrow[j] = __fmul_rn(__ldg(a.gamma + nb + j), (float)iv[j]);
+              if (a.acc) a.acc[out_row * a.ldo + nb + j] = iv[j];
+            }
           }
-        } else {
-          for (int j = 0; j < 32 && nb + j < a.N; ++j) {
-            yrow[j] = __fmul_rn(__ldg(a.gamma + nb + j), (float)iv[j]);
-            if (a.acc) a.acc[out_row * a.ldo + nb + j] = iv[j];
+        } else if (a.epi == EPI_ACC32) {
+          int32_t* orow = a.acc + out_row * a.ldo + nb;
+          if (full) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) *reinterpret_cast<int4*>(orow + j) = make_int4(iv[j], iv[j + 1], iv[j + 2], iv[j + 3]);
+          } else {
+            for (int j = 0; j < 32 && nb + j < a.N; ++j) orow[j] = iv[j];
+          }
+        } else {  // EPI_DX
+          float* orow = a.y + out_row * a.ldo + nb;
+          if (full) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) {
+              const int4 c4 = __ldg(reinterpret_cast<const int4*>(a.cs + nb + j));
+              *reinterpret_cast<float4*>(orow + j) = make_float4(
+                  __fadd_rn(__fmul_rn(sc, (float)iv[j + 0]), __fmul_rn(ze, (float)c4.x)),
+                  __fadd_rn(__fmul_rn(sc, (float)iv[j + 1]), __fmul_rn(ze, (float)c4.y)),
+                  __fadd_rn(__fmul_rn(sc, (float)iv[j + 2]), __fmul_rn(ze, (float)c4.z)),
+                  __fadd_rn(__fmul_rn(sc, (float)iv[j + 3]), __fmul_rn(ze, (float)c4.w)));
+            }
+          } else {
+            for (int j = 0; j < 32 && nb + j < a.N; ++j)
+              orow[j] = __fadd_rn(__fmul_rn(sc, (float)iv[j]), __fmul_rn(ze, (float)__ldg(a.cs + nb + j)));
           }
         }
-      } else if (a.epi == EPI_ACC32) {
-        int32_t* orow = a.acc + out_row * a.ldo + nb;
-        if (full) {
+        continue;
+      }
+      // split-K reduction: stage the 32 x 32 block (row `lane`, 16-byte chunk c stored at
+      // chunk c ^ (lane & 7)), then add one coalesced 128-byte row per instruction
 #pragma unroll
-          for (int j = 0; j < 32; j += 4) *reinterpret_cast<int4*>(orow + j) = make_int4(iv[j], iv[j + 1], iv[j + 2], iv[j + 3]);
-        } else {
-          for (int j = 0; j < 32 && nb + j < a.N; ++j) orow[j] = iv[j];
-        }
-      } else if (a.epi == EPI_RED) {
-        int32_t* orow = a.acc + out_row * a.ldo + nb;
-        for (int j = 0; j < 32 && nb + j < a.N; ++j) atomicAdd(orow + j, iv[j]);
-      } else {  // EPI_DX
-        float* orow = a.y + out_row * a.ldo + nb;
-        if (full) {
-#pragma unroll
-          for (int j = 0; j < 32; j += 4) {
-            float4 o;
-            o.x = __fadd_rn(__fmul_rn(sc, (float)iv[j + 0]), __fmul_rn(ze, (float)__ldg(a.cs + nb + j + 0)));
-            o.y = __fadd_rn(__fmul_rn(sc, (float)iv[j + 1]), __fmul_rn(ze, (float)__ldg(a.cs + nb + j + 1)));
-            o.z = __fadd_rn(__fmul_rn(sc, (float)iv[j + 2]), __fmul_rn(ze, (float)__ldg(a.cs + nb + j + 2)));
-            o.w = __fadd_rn(__fmul_rn(sc, (float)iv[j + 3]), __fmul_rn(ze, (float)__ldg(a.cs + nb + j + 3)));
-            *reinterpret_cast<float4*>(orow + j) = o;
-          }
-        } else {
-          for (int j = 0; j < 32 && nb + j < a.N; ++j)
-            orow[j] = __fadd_rn(__fmul_rn(sc, (float)iv[j]), __fmul_rn(ze, (float)__ldg(a.cs + nb + j)));
+      for (int c = 0; c < 8; ++c) {
+        uint4 w;
+        w.x = (uint32_t)__float2int_rn(__uint_as_float(v[4 * c + 0]));
+        w.y = (uint32_t)__float2int_rn(__uint_as_float(v[4 * c + 1]));
+        w.z = (uint32_t)__float2int_rn(__uint_as_float(v[4 * c + 2]));
+        w.w = (uint32_t)__float2int_rn(__uint_as_float(v[4 * c + 3]));
+        *reinterpret_cast<uint4*>(stage + lane * 32 + ((c ^ (lane & 7)) << 2)) = w;
+      }
+      __syncwarp();
+      const int64_t n = n0 + c0 + lane;  // this lane's column
+      if (n < a.N) {
+#pragma unroll 4
+        for (int rr = 0; rr < 32; ++rr) {
+          const int64_t r = row_base + rr;
+          if (r >= valid_rows || r >= a.M) break;
+          atomicAdd(a.acc + r * a.ldo + n, (int32_t)stage[rr * 32 + ((((lane >> 2) ^ (rr & 7))) << 2) + (lane & 3)]);
         }
       }
     }

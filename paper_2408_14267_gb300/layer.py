@@ -122,3 +122,41 @@ class LayerStep:
     def step(self, stream=None):
         for name, fn in self.stages():
             fn(stream)
+
+    def step_concurrent(self, stream=None):
+        """The same step as three stream branches joined by events (capturable in one graph).
+
+        The packing of W, the packing / Unfolder of X and the SCQ quantization of gY are
+        independent; each product waits only for its own operands:
+          calling stream: pack X -> (wait W) forward -> (wait SCQ) grad_weight -> join
+          branch 1      : pack W
+          branch 2      : SCQ quantize -> (wait W) grad_input (-> Folder)
+        """
+        main = stream if stream is not None else torch.cuda.current_stream()
+        if not hasattr(self, "_branches"):
+            self._branches = (torch.cuda.Stream(device=main.device), torch.cuda.Stream(device=main.device))
+        b1, b2 = self._branches
+        st = dict(self.stages())
+        fork = torch.cuda.Event()
+        fork.record(main)
+        b1.wait_event(fork)
+        b2.wait_event(fork)
+        st["pack_w"](b1)
+        w_ready = torch.cuda.Event()
+        w_ready.record(b1)
+        st["scq_quantize"](b2)
+        q_ready = torch.cuda.Event()
+        q_ready.record(b2)
+        b2.wait_event(w_ready)
+        st["bwd_input_gemm"](b2)
+        if "col2im" in st:
+            st["col2im"](b2)
+        x_name = "im2col" if "im2col" in st else "pack_x"
+        st[x_name](main)
+        main.wait_event(w_ready)
+        st["fwd_gemm"](main)
+        main.wait_event(q_ready)
+        st["bwd_weight_gemm"](main)
+        b2_done = torch.cuda.Event()
+        b2_done.record(b2)
+        main.wait_event(b2_done)

@@ -198,6 +198,25 @@ def test_linear_fused_dequant_parity(name, make):
         assert np.all(dx[g * rpg:(g + 1) * rpg] == 0)
 
 
+@pytest.mark.parametrize("name,make", [CASES[0], CASES[1], CASES[9]], ids=[CASES[0][0], CASES[1][0], CASES[9][0]])
+def test_concurrent_step_matches_serial(name, make):
+    """The three-branch schedule (also captured in a CUDA graph) gives the serial step's results."""
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    a = LayerStep(w, keep_acc=False)
+    a.step()
+    b = LayerStep(w, keep_acc=False)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        b.step_concurrent(s)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            b.step_concurrent(s)
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(a.y, b.y) and torch.equal(a.dx, b.dx) and torch.equal(a.dw, b.dw)
+
+
 def test_single_branch_entry_point_matches_scq():
     """fqt1_agp_quantize_grad on one axis equals that branch of fqt1_scq_quantize."""
     from paper_2408_14267_gb300 import fqt1
