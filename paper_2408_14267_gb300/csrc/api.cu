@@ -42,12 +42,26 @@ bool use_popcount_path() {
   return v == 1;
 }
 
-// Rows of pruned groups of an [M][K] fp32 output are exactly zero.
+// Rows of pruned groups of an [M][K] fp32 output are exactly zero.  Grid: x covers a row in
+// chunks of 1024 floats, y (and z for more than 65535 rows) the rows.
 __global__ void zero_pruned_rows_kernel(const int32_t* __restrict__ slot_of_group, int64_t M, int64_t K, int64_t rpg,
                                         float* __restrict__ out) {
-  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= M * K) return;
-  if (__ldg(slot_of_group + (idx / K) / rpg) < 0) out[idx] = 0.0f;
+  const int64_t row = (int64_t)blockIdx.z * 65535 + blockIdx.y;
+  if (row >= M || __ldg(slot_of_group + row / rpg) >= 0) return;
+  float* dst = out + row * K;
+  const int64_t c = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 4;
+  if (c + 4 <= K && (K % 4) == 0) {
+    *reinterpret_cast<float4*>(dst + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+  } else {
+    for (int64_t j = c; j < c + 4 && j < K; ++j) dst[j] = 0.0f;
+  }
+}
+
+static void launch_zero_pruned_rows(const int32_t* slot_of_group, int64_t M, int64_t K, int64_t rpg, float* out,
+                                    cudaStream_t s) {
+  const dim3 grid((unsigned)((K + 1023) / 1024), (unsigned)(M < 65535 ? M : 65535), (unsigned)((M + 65534) / 65535));
+  zero_pruned_rows_kernel<<<grid, 256, 0, s>>>(slot_of_group, M, K, rpg, out);
+  fqt1_count_launches(1);
 }
 
 // out[m, k] = S'_slot * acc[row(m), k] + Z'_slot * cs[k] for rows m of kept groups, 0 otherwise
@@ -114,7 +128,8 @@ __global__ void col2im_kernel(const int32_t* __restrict__ acc, const int32_t* __
 // tile is odd so that neighbouring pixels fall in different banks.
 struct FoldArgs {
   const int32_t* acc;
-  const int32_t* slot_of_group;
+  const int32_t* kept_idx;
+  const int32_t* kept_count;
   const float* scale;
   const float* zero;
   const int32_t* cs;
@@ -126,21 +141,15 @@ struct FoldArgs {
 
 __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
   extern __shared__ int32_t fold_smem[];
-  const int n = blockIdx.y;
+  const int32_t slot = (int32_t)blockIdx.y;  // one kept sample per grid row
+  if (slot >= __ldg(a.kept_count)) return;
+  const int n = __ldg(a.kept_idx + slot);
   const int cblk = blockIdx.x % a.ncb, hblk = blockIdx.x / a.ncb;
   const int c0 = cblk * a.cb, h0 = hblk * a.hb;
   const int c1 = min(a.C, c0 + a.cb), h1 = min(a.H, h0 + a.hb);
   const int nc = c1 - c0, nh = h1 - h0;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int32_t slot = __ldg(a.slot_of_group + n);
   const int plane = nh * a.W;  // contiguous floats of one channel inside the block
-  if (slot < 0) {
-    for (int cl = 0; cl < nc; ++cl) {
-      float* dst = a.dx + (((int64_t)n * a.C + c0 + cl) * a.H + h0) * a.W;
-      for (int x = threadIdx.x; x < plane; x += blockDim.x) dst[x] = 0.0f;
-    }
-    return;
-  }
   const int khw = a.kh * a.kw;
   int oh_lo = h0 + a.pad - (a.kh - 1);
   oh_lo = oh_lo <= 0 ? 0 : (oh_lo + a.stride - 1) / a.stride;
@@ -171,31 +180,44 @@ __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
   const int64_t kbase = (int64_t)c0 * khw;
   for (int x = threadIdx.x; x < kb; x += blockDim.x) css[x] = __ldg(a.cs + kbase + x);
   if (nrows > 0) {
+    // one accumulator row segment (kb ints) per warp iteration; 8 loads in flight per lane
     const int npix = nrows * a.Wo;
     const int64_t rbase = (int64_t)slot * a.Ho * a.Wo + (int64_t)oh_lo * a.Wo;
     for (int pix = warp; pix < npix; pix += blockDim.x >> 5) {
       const int32_t* src = a.acc + (rbase + pix) * a.K + kbase;
       int32_t* dst = tile + pix * a.kstride;
-      for (int kk = lane; kk < kb; kk += 32) dst[kk] = __ldg(src + kk);
+      for (int k0 = 0; k0 < kb; k0 += 256) {
+        int32_t v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int kk = k0 + 32 * u + lane;
+          v[u] = kk < kb ? __ldg(src + kk) : 0;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int kk = k0 + 32 * u + lane;
+          if (kk < kb) dst[kk] = v[u];
+        }
+      }
     }
   }
   __syncthreads();
   const float sc = __ldg(a.scale + slot), ze = __ldg(a.zero + slot);
-  const int outs = nc * plane;
-  for (int e = threadIdx.x; e < outs; e += blockDim.x) {
-    const int cl = e / plane, rem = e - cl * plane;
-    const int hl = rem / a.W, w = rem - hl * a.W;
+  const FastDiv div_plane((uint32_t)plane), div_w((uint32_t)a.W);
+  for (int e = threadIdx.x; e < nc * plane; e += blockDim.x) {  // output (channel, row, column) of the block
+    const int cl = (int)div_plane.div((uint32_t)e), pos = e - cl * plane;
+    const int hl = (int)div_w.div((uint32_t)pos), w = pos - hl * a.W;
     const int kc = cl * khw;
     int32_t acc = 0, csum = 0;
     for (int i = 0; i < a.kh; ++i) {
       const int ro = hrow[hl * a.kh + i];
       if (ro < 0) continue;
+      const int32_t* trow = tile + kc + i * a.kw;
       for (int j = 0; j < a.kw; ++j) {
         const int co = wcol[w * a.kw + j];
         if (co < 0) continue;
-        const int kk = kc + i * a.kw + j;
-        acc += tile[(ro + co) * a.kstride + kk];
-        csum += css[kk];
+        acc += trow[(ro + co) * a.kstride + j];
+        csum += css[kc + i * a.kw + j];
       }
     }
     a.dx[(((int64_t)n * a.C + c0 + cl) * a.H + h0 + hl) * a.W + w] =
@@ -245,9 +267,7 @@ extern "C" fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t
     FQT1_CUDA_TRY(launch_codes_tc_simple(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, rpg, sw_col,
                                          K, D, GEMM_EPI_DX, 1, nullptr, dx, K, psq->kept_idx, psq->scale,
                                          psq->zero, colsum_w, rpg, nullptr, s));
-    const int64_t n = M * K;
-    zero_pruned_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(psq->slot_of_group, M, K, rpg, dx);
-    fqt1_count_launches(1);
+    launch_zero_pruned_rows(psq->slot_of_group, M, K, rpg, dx, s);
     FQT1_CUDA_TRY(cudaGetLastError());
     return FQT1_OK;
   }
@@ -275,12 +295,14 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
   if (!acc || !psq || !colsum_w || !dx || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 ||
       pad < 0)
     return FQT1_ERR_INVALID_ARG;
-  if (!psq->slot_of_group || !psq->scale || !psq->zero) return FQT1_ERR_INVALID_ARG;
+  if (!psq->slot_of_group || !psq->scale || !psq->zero || !psq->kept_idx || !psq->kept_count)
+    return FQT1_ERR_INVALID_ARG;
   const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
   if (H + 2 * pad < kh || W + 2 * pad < kw) return FQT1_ERR_INVALID_ARG;
   if (!aligned16(acc) || !aligned16(dx)) return FQT1_ERR_MISALIGNED;
   // tiled Folder: choose input rows and channels per CTA so that the staged accumulators fit
   constexpr int64_t kMaxTile = 96 * 1024;
+  constexpr int64_t kPreferTile = 48 * 1024;  // >= 4 resident CTAs per SM
   const int khw = kh * kw;
   int hb = H < 8 ? H : 8, cb = 0;
   int max_rows = 0, kstride = 0;
@@ -290,7 +312,7 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
     for (int c = (C < 32 ? C : 32); c >= 1; c = (c > 1 ? c / 2 : 0)) {
       const int ks = (c * khw) | 1;
       const int64_t words = (int64_t)max_rows * Wo * ks + (int64_t)hb * kh + (int64_t)W * kw + (int64_t)c * khw;
-      if (words * 4 <= kMaxTile) { cb = c; kstride = ks; break; }
+      if (words * 4 <= (c > 1 ? kPreferTile : kMaxTile)) { cb = c; kstride = ks; break; }
     }
     if (cb) break;
   }
@@ -302,7 +324,8 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
       attr = true;
     }
     FoldArgs fa;
-    fa.acc = acc; fa.slot_of_group = psq->slot_of_group; fa.scale = psq->scale; fa.zero = psq->zero;
+    fa.acc = acc; fa.kept_idx = psq->kept_idx; fa.kept_count = psq->kept_count; fa.scale = psq->scale;
+    fa.zero = psq->zero;
     fa.cs = colsum_w; fa.dx = dx; fa.N = N; fa.C = C; fa.H = H; fa.W = W; fa.kh = kh; fa.kw = kw;
     fa.stride = stride; fa.pad = pad; fa.Ho = Ho; fa.Wo = Wo; fa.cb = cb; fa.hb = hb;
     fa.ncb = (C + cb - 1) / cb; fa.max_rows = max_rows; fa.kstride = kstride; fa.K = (int64_t)C * khw;
@@ -310,7 +333,10 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
     if (nblk > 0x7FFFFFFF || N > 65535) return FQT1_ERR_UNSUPPORTED;
     const size_t smem =
         ((size_t)max_rows * Wo * kstride + (size_t)hb * kh + (size_t)W * kw + (size_t)cb * khw) * 4;
-    col2im_tiled_kernel<<<dim3((unsigned)nblk, (unsigned)N), 256, smem, (cudaStream_t)stream>>>(fa);
+    // pruned samples: zeros; kept samples: the tiled fold (one grid row per kept slot)
+    launch_zero_pruned_rows(psq->slot_of_group, N, (int64_t)C * H * W, 1, dx, (cudaStream_t)stream);
+    const int64_t cap = fqt1_kept_capacity(N, 8, FQT1_SEL_BERNOULLI);  // upper bound: all samples
+    col2im_tiled_kernel<<<dim3((unsigned)nblk, (unsigned)cap), 256, smem, (cudaStream_t)stream>>>(fa);
   } else {
     const int64_t n = (int64_t)N * C * H * W;
     col2im_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(

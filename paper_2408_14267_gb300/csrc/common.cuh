@@ -53,8 +53,8 @@ __device__ __forceinline__ uint32_t philox_word(uint64_t seed, uint32_t stream, 
 // n / d = (umulhi(n, m) + n) >> l.  The host computes m and l.
 struct FastDiv {
   uint32_t d, mul, shr;
-  FastDiv() : d(1), mul(1), shr(0) {}
-  explicit FastDiv(uint32_t divisor) : d(divisor), mul(0), shr(0) {
+  __host__ __device__ FastDiv() : d(1), mul(1), shr(0) {}
+  __host__ __device__ explicit FastDiv(uint32_t divisor) : d(divisor), mul(0), shr(0) {
     while (shr < 31 && (1u << shr) < d) ++shr;
     mul = (uint32_t)((((uint64_t)1 << 32) * (((uint64_t)1 << shr) - d)) / d + 1);
   }

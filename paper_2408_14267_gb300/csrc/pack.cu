@@ -1,6 +1,8 @@
 // Sign + pack kernels: the row / column encoders of App. C (Algorithm 2) and the
 // Unfolder fused with them.  One pass over the input writes both packings and
 // the column sums of the signs.
+#include <algorithm>
+
 #include "common.cuh"
 
 namespace fqt1 {
@@ -130,6 +132,202 @@ __global__ void zero_col_pad_kernel(uint32_t* col_bits, int64_t cols, int64_t co
   if (i < cols * npad) col_bits[(i / npad) * col_words + first_pad + (i % npad)] = 0u;
 }
 
+// ---------------------------------------------------------------------------
+// Bit-level Unfolder.  A CTA owns tm output pixels x 256 columns of X_u.
+//  1. It sign-packs the part of the input those entries read into shared memory: for
+//     every (image, channel) pair of the region, input rows h_lo..h_hi form one bit
+//     stream (bit e = sign of the e-th float of those rows, behind one zero guard word
+//     and followed by another).
+//  2. Warp w builds the 32 x 32 bit blocks of columns k0 + 32 w .. + 31.  For stride 1
+//     a lane builds the column word of one k (a run of output pixels on one output row
+//     reads a run of consecutive stream bits); otherwise a lane builds the row word of
+//     one pixel (a run of kernel taps on one input row reads consecutive stream bits).
+//     A 5-step shuffle butterfly transposes each block into the other packing.
+//  3. Row words and column words are staged in shared memory and written as 32-byte runs.
+constexpr int kUnfoldMaxStreamWords = 24576;  // 96 KB of input bit streams per CTA
+
+struct UnfoldArgs {
+  const float* x;
+  uint32_t* row_bits;
+  uint32_t* col_bits;
+  int32_t* colsum;
+  int64_t row_words, col_words;
+  int C, H, W, kh, kw, stride, pad, Wo, M, K, khw, HWo;
+  int tm;  // output pixels per CTA: 32, 64, 128 or 256
+  FastDiv div_khw, div_kw, div_hwo, div_wo;
+};
+
+// 32 x 32 bit transpose across a warp: lane r holds row r (bit c = column c); afterwards
+// lane c holds column c (bit r = row r).  Each step swaps the off-diagonal j x j blocks.
+__device__ __forceinline__ uint32_t warp_transpose32(uint32_t x, int lane) {
+#pragma unroll
+  for (int j = 16; j >= 1; j >>= 1) {
+    const uint32_t m = j == 16 ? 0x0000FFFFu : j == 8 ? 0x00FF00FFu : j == 4 ? 0x0F0F0F0Fu : j == 2 ? 0x33333333u
+                                                                                                      : 0x55555555u;
+    const uint32_t p = __shfl_xor_sync(0xFFFFFFFFu, x, j);
+    x = (lane & j) ? ((x & ~m) | ((p >> j) & m)) : ((x & m) | ((p & m) << j));
+  }
+  return x;
+}
+
+// cnt (1..32) bits of a stream starting at bit pos; the guard words keep both reads inside.
+__device__ __forceinline__ uint32_t stream_bits(const uint32_t* st, int pos, int cnt) {
+  const int w = pos >> 5, o = pos & 31;
+  const uint64_t v = ((uint64_t)st[w + 1] << 32) | st[w];
+  const uint32_t bits = (uint32_t)(v >> o);
+  return cnt >= 32 ? bits : bits & ((1u << cnt) - 1u);
+}
+
+__global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
+  extern __shared__ uint32_t stream[];
+  __shared__ uint32_t rw_s[256][9];  // row words [pixel in tile][k-word in tile]
+  __shared__ uint32_t cw_s[256][9];  // column words [k in tile][pixel-word in tile]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.y * a.tm, m1 = min(a.M, m0 + a.tm);
+  const int k0 = blockIdx.x * 256, k1 = min(a.K, k0 + 256);
+  const int nsub = a.tm / 32;
+  const bool have_k = k0 < a.K;
+  // region of the input read by this tile
+  int c_lo = 0, nc = 1, n_lo = 0, h_lo = 0, nrows = 0, plane_words = 2, nplanes = 0;
+  if (have_k) {
+    c_lo = (int)a.div_khw.div((uint32_t)k0);
+    nc = (int)a.div_khw.div((uint32_t)(k1 - 1)) - c_lo + 1;
+    n_lo = (int)a.div_hwo.div((uint32_t)m0);
+    const int n_hi = (int)a.div_hwo.div((uint32_t)(m1 - 1));
+    int h_hi = a.H - 1;
+    if (n_lo == n_hi) {
+      const int oh_lo = (int)a.div_wo.div((uint32_t)(m0 - n_lo * a.HWo));
+      const int oh_hi = (int)a.div_wo.div((uint32_t)(m1 - 1 - n_lo * a.HWo));
+      h_lo = max(0, oh_lo * a.stride - a.pad);
+      h_hi = min(a.H - 1, oh_hi * a.stride - a.pad + a.kh - 1);
+    }
+    nrows = max(0, h_hi - h_lo + 1);
+    plane_words = (nrows * a.W + 31) / 32 + 2;
+    nplanes = (n_hi - n_lo + 1) * nc;
+  }
+  // 1. sign-pack the region (one warp per 32 stream bits: coalesced 128-byte loads + ballot)
+  const int plane_bits = nrows * a.W, data_words = plane_words - 2;
+  for (int pl = warp; pl < nplanes; pl += 8) {  // one (image, channel) plane per warp iteration
+    const int nn = pl / nc;
+    const float* src = a.x + (((int64_t)(n_lo + nn) * a.C + c_lo + (pl - nn * nc)) * a.H + h_lo) * a.W;
+    uint32_t* dst = stream + pl * plane_words + 1;
+    for (int q0 = 0; q0 < data_words; q0 += 4) {  // 4 loads in flight per lane, then 4 ballots
+      float v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int e = 32 * (q0 + u) + lane;
+        v[u] = (q0 + u < data_words && e < plane_bits) ? __ldg(src + e) : 0.0f;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const uint32_t word = __ballot_sync(0xFFFFFFFFu, v[u] > 0.0f);
+        if (lane == 0 && q0 + u < data_words) dst[q0 + u] = word;
+      }
+    }
+  }
+  for (int pl = threadIdx.x; pl < nplanes; pl += 256) {
+    stream[pl * plane_words] = 0u;
+    stream[pl * plane_words + plane_words - 1] = 0u;
+  }
+  __syncthreads();
+  // 2. the 32 x 32 blocks of columns kb .. kb + 31
+  const int kb = k0 + 32 * warp;
+  // column k = kb + lane as (channel, kernel row, kernel column), fixed for the whole tile
+  const int kl = min(kb + lane, a.K - 1);
+  const int cl_ = (int)a.div_khw.div((uint32_t)kl), tl_ = kl - cl_ * a.khw;
+  const int il_ = (int)a.div_kw.div((uint32_t)tl_), jl_ = tl_ - il_ * a.kw;
+  const int Ho = a.HWo / a.Wo;
+  for (int sub = 0; sub < nsub; ++sub) {
+    const int ms = m0 + 32 * sub;
+    uint32_t roww = 0, colw = 0;
+    if (kb < a.K && ms < a.M) {  // warp-uniform
+      if (a.stride == 1) {
+        // column word of k = kb + lane over pixels ms .. ms + 31: runs along output rows
+        const int mend = min(a.M, ms + 32);
+        int n = (int)a.div_hwo.div((uint32_t)ms), rem = ms - n * a.HWo;
+        int oh = (int)a.div_wo.div((uint32_t)rem), ow = rem - oh * a.Wo;
+        const uint32_t* st_c = stream + (cl_ - c_lo) * plane_words;
+        const bool kvalid = kb + lane < a.K;
+        for (int m = ms; m < mend;) {
+          const int cnt = min(a.Wo - ow, mend - m);  // pixels left on this output row
+          const int h = oh - a.pad + il_;
+          const int wa = ow - a.pad + jl_;  // input column of the run's first pixel
+          const int lo = max(0, -wa), hi = min(cnt, a.W - wa);
+          if (kvalid && h >= 0 && h < a.H && hi > lo) {
+            const uint32_t* st = st_c + (n - n_lo) * nc * plane_words;
+            colw |= stream_bits(st, 32 + (h - h_lo) * a.W + wa + lo, hi - lo) << (m - ms + lo);
+          }
+          m += cnt;
+          ow += cnt;
+          if (ow == a.Wo) {
+            ow = 0;
+            if (++oh == Ho) { oh = 0; ++n; }
+          }
+        }
+        roww = warp_transpose32(colw, lane);
+      } else {
+        // row word of pixel ms + lane over columns kb .. kb + 31: runs along kernel rows
+        const int mr = ms + lane;
+        if (mr < a.M) {
+          const int n = (int)a.div_hwo.div((uint32_t)mr), rem = mr - n * a.HWo;
+          const int oh = (int)a.div_wo.div((uint32_t)rem), ow = rem - oh * a.Wo;
+          const int h0 = oh * a.stride - a.pad, w0 = ow * a.stride - a.pad;
+          int c = (int)a.div_khw.div((uint32_t)kb), t = kb - c * a.khw;
+          int i = (int)a.div_kw.div((uint32_t)t), j = t - i * a.kw;
+          const int kend = min(a.K, kb + 32);
+          const uint32_t* st_n = stream + (n - n_lo) * nc * plane_words;
+          for (int k = kb; k < kend;) {
+            const int cnt = min(a.kw - j, kend - k);  // taps left on this kernel row
+            const int h = h0 + i;
+            const int wa = w0 + j;
+            const int lo = max(0, -wa), hi = min(cnt, a.W - wa);
+            if (h >= 0 && h < a.H && hi > lo)
+              roww |= stream_bits(st_n + (c - c_lo) * plane_words, 32 + (h - h_lo) * a.W + wa + lo, hi - lo)
+                      << (k - kb + lo);
+            k += cnt;
+            j += cnt;
+            if (j == a.kw) {
+              j = 0;
+              if (++i == a.kh) { i = 0; ++c; }
+            }
+          }
+        }
+        colw = warp_transpose32(roww, lane);
+      }
+    }
+    rw_s[32 * sub + lane][warp] = roww;
+    cw_s[32 * warp + lane][sub] = colw;
+  }
+  __syncthreads();
+  // 3. outputs
+  if (a.row_bits) {
+    const int64_t w0 = (int64_t)blockIdx.x * 8;
+    for (int e = threadIdx.x; e < (m1 - m0) * 8; e += 256) {
+      const int r = e >> 3, q = e & 7;
+      if (w0 + q < a.row_words) a.row_bits[(int64_t)(m0 + r) * a.row_words + w0 + q] = rw_s[r][q];
+    }
+  }
+  if (have_k && (a.col_bits || a.colsum)) {
+    const int64_t wbase = m0 / 32;
+    if (a.col_bits) {
+      for (int e = threadIdx.x; e < (k1 - k0) * nsub; e += 256) {
+        const int kk = e / nsub, sub = e - kk * nsub;
+        if (wbase + sub < a.col_words) a.col_bits[(int64_t)(k0 + kk) * a.col_words + wbase + sub] = cw_s[kk][sub];
+      }
+    }
+    if (a.colsum) {
+      for (int kk = threadIdx.x; kk < k1 - k0; kk += 256) {
+        int sum = 0;
+        for (int sub = 0; sub < nsub; ++sub) {
+          const int valid = min(32, max(0, a.M - (m0 + 32 * sub)));
+          sum += 2 * __popc(cw_s[kk][sub]) - valid;
+        }
+        atomicAdd(a.colsum + k0 + kk, sum);
+      }
+    }
+  }
+}
+
 template <class Loader>
 static fqt1_status launch_pack(const Loader& L, uint32_t* row_bits, uint32_t* col_bits, int32_t* colsum,
                                cudaStream_t s) {
@@ -184,10 +382,50 @@ extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t
       (colsum && !aligned16(colsum)))
     return FQT1_ERR_MISALIGNED;
   if ((int64_t)N * C * H * W >= (1ll << 31) || (int64_t)N * Ho * Wo >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
+  cudaStream_t s = (cudaStream_t)stream;
+  // Bit-level Unfolder when the input region of a tile fits in shared memory.  Bound on the
+  // region of a tile of tm pixels: images it may touch x channels of 256 columns x whole planes.
+  const int64_t Mi = (int64_t)N * Ho * Wo, Ki = (int64_t)C * kh * kw;
+  if (pad <= 32 && Ki < (1ll << 31)) {
+    const int tm_first = Mi >= 64 * 152 * 4 ? 128 : 64;  // smaller tiles: more resident CTAs
+    for (int tm = tm_first; tm >= 32; tm /= 2) {
+      const int64_t imgs = std::min<int64_t>(N, tm / (Ho * Wo) + 2);
+      const int64_t chans = std::min<int64_t>(C, 256 / (kh * kw) + 2);
+      const int64_t words = imgs * chans * (((int64_t)H * W + 31) / 32 + 2);
+      if (words > kUnfoldMaxStreamWords) continue;
+      UnfoldArgs u;
+      u.x = x; u.row_bits = row_bits; u.col_bits = col_bits; u.colsum = colsum;
+      u.row_words = fqt1_packed_words(Ki); u.col_words = fqt1_packed_words(Mi);
+      u.C = C; u.H = H; u.W = W; u.kh = kh; u.kw = kw; u.stride = stride; u.pad = pad; u.Wo = Wo;
+      u.M = (int)Mi; u.K = (int)Ki; u.khw = kh * kw; u.HWo = Ho * Wo; u.tm = tm;
+      u.div_khw = FastDiv((uint32_t)(kh * kw)); u.div_kw = FastDiv((uint32_t)kw);
+      u.div_hwo = FastDiv((uint32_t)(Ho * Wo)); u.div_wo = FastDiv((uint32_t)Wo);
+      const int64_t row_tiles = (Mi + tm - 1) / tm, word_tiles = (u.row_words + 7) / 8;
+      if (row_tiles > 65535) break;
+      static bool attr = false;
+      if (!attr) {
+        FQT1_CUDA_TRY(cudaFuncSetAttribute(unfold_bits_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           kUnfoldMaxStreamWords * 4));
+        attr = true;
+      }
+      if (colsum) FQT1_CUDA_TRY(cudaMemsetAsync(colsum, 0, sizeof(int32_t) * Ki, s));
+      unfold_bits_kernel<<<dim3((unsigned)word_tiles, (unsigned)row_tiles), 256, (size_t)words * 4, s>>>(u);
+      fqt1_count_launches(1);
+      FQT1_CUDA_TRY(cudaGetLastError());
+      const int64_t written = row_tiles * (tm / 32);
+      if (col_bits && u.col_words > written) {
+        const int64_t n = Ki * (u.col_words - written);
+        zero_col_pad_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(col_bits, Ki, u.col_words, written);
+        fqt1_count_launches(1);
+        FQT1_CUDA_TRY(cudaGetLastError());
+      }
+      return FQT1_OK;
+    }
+  }
   Im2colLoader L;
   L.x = x; L.rows = (int64_t)N * Ho * Wo; L.cols = (int64_t)C * kh * kw;
   L.H = H; L.W = W; L.stride = stride; L.pad = pad; L.CHW = C * H * W; L.HW = H * W;
   L.div_hw_out = FastDiv((uint32_t)(Ho * Wo)); L.div_wo = FastDiv((uint32_t)Wo);
   L.div_khw = FastDiv((uint32_t)(kh * kw)); L.div_kw = FastDiv((uint32_t)kw);
-  return launch_pack(L, row_bits, col_bits, colsum, (cudaStream_t)stream);
+  return launch_pack(L, row_bits, col_bits, colsum, s);
 }

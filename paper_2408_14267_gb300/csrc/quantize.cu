@@ -15,7 +15,7 @@
 namespace fqt1 {
 
 // ------------------------------------------------------------------ ranges
-constexpr int kRangeRows = 64, kRangeCols = 128;
+constexpr int kRangeRows = 32, kRangeCols = 128;  // 8 warps x 4 rows x (32 lanes x 4 columns)
 
 struct RangeArgs {
   const float* g;
@@ -31,7 +31,7 @@ __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
   __shared__ uint32_t cmin_s[8][kRangeCols], cmax_s[8][kRangeCols];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t c0 = (int64_t)blockIdx.x * kRangeCols + lane * 4;
-  const int64_t r0 = (int64_t)blockIdx.y * kRangeRows + warp * 8;
+  const int64_t r0 = (int64_t)blockIdx.y * kRangeRows + warp * (kRangeRows / 8);
   float gam[4];
   bool cv[4];
 #pragma unroll
@@ -43,7 +43,25 @@ __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
   uint32_t gmin = 0xFFFFFFFFu, gmax = 0u;
   int64_t cur = -1;
   bool bad = false;
-  for (int i = 0; i < 8; ++i) {
+  constexpr int kR = kRangeRows / 8;  // rows per warp
+  float v[kR][4];
+#pragma unroll
+  for (int i = 0; i < kR; ++i) {  // all loads of this warp's rows first
+    const int64_t r = r0 + i;
+    if (VEC) {
+      if (cv[0] && r < a.M) {
+        const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + c0));
+        v[i][0] = t.x; v[i][1] = t.y; v[i][2] = t.z; v[i][3] = t.w;
+      } else {
+        v[i][0] = v[i][1] = v[i][2] = v[i][3] = 0.f;
+      }
+    } else {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) v[i][q] = (cv[q] && r < a.M) ? __ldg(a.g + r * a.D + c0 + q) : 0.0f;
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < kR; ++i) {
     const int64_t r = r0 + i;
     if (r >= a.M) break;
     const int64_t gi = r / a.rpg;
@@ -56,20 +74,10 @@ __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
       gmin = 0xFFFFFFFFu;
       gmax = 0u;
     }
-    float v[4];
-    if (VEC) {
-      if (cv[0]) {
-        const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + c0));
-        v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
-      }
-    } else {
-#pragma unroll
-      for (int q = 0; q < 4; ++q) v[q] = cv[q] ? __ldg(a.g + r * a.D + c0 + q) : 0.0f;
-    }
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       if (!cv[q]) continue;
-      const float x = a.gamma ? __fmul_rn(v[q], gam[q]) : v[q];
+      const float x = a.gamma ? __fmul_rn(v[i][q], gam[q]) : v[i][q];
       bad |= !isfinite(x);
       const uint32_t k = float_to_ordered(x);
       colmin[q] = min(colmin[q], k);
@@ -140,15 +148,14 @@ __device__ uint64_t block_inclusive_scan(uint64_t v, uint64_t* warp_sums, uint64
   return v;
 }
 
-// floor(a * 2^32 / d) for a <= d < 2^60 by base-16 long division (exact).
+// floor(a * 2^32 / d) for 0 < d < 2^60, a < 2^60 (exact): a float64 estimate, then the
+// remainder a * 2^32 - q d in 128-bit integers moves q to the exact quotient.
 __device__ __forceinline__ uint64_t div_shift32(uint64_t a, uint64_t d) {
-  uint64_t q = a / d, r = a % d;
-#pragma unroll
-  for (int s = 0; s < 8; ++s) {
-    r <<= 4;
-    q = (q << 4) | (r / d);
-    r %= d;
-  }
+  const unsigned __int128 num = (unsigned __int128)a << 32;
+  double est = __ddiv_rn(__ull2double_rn(a) * 4294967296.0, __ull2double_rn(d));
+  uint64_t q = est <= 0.0 ? 0ull : (uint64_t)est;
+  while ((unsigned __int128)q * d > num) --q;
+  while ((unsigned __int128)(q + 1) * d <= num) ++q;
   return q;
 }
 
@@ -191,7 +198,54 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
     return (rmax > 0.0f && r > 0.0f) ? (uint64_t)floor((double)r * fx) : 0ull;
   };
 
-  if (a.bits > 1) {
+  if (a.bits > 1 && n <= kSelThreads) {
+    // rank of each key (R~ desc, index asc) by comparison with all others: no sort needed
+    uint64_t myk = 0, myrt = 0;
+    if (tid < n) {
+      myrt = rtilde(tid);
+      myk = (myrt << 24) | (uint64_t)(0xFFFFFFu - (uint32_t)tid);
+      key[tid] = myk;
+    }
+    __syncthreads();
+    int rank = 0;
+    if (tid < n)
+      for (int j = 0; j < n; ++j) rank += key[j] > myk ? 1 : 0;
+    __syncthreads();
+    if (tid < n) key[rank] = myrt;  // fixed-point ranges in sorted (descending) order
+    __syncthreads();
+    int tstar;
+    uint64_t S = 0;
+    if (a.mode == FQT1_SEL_TOPK) {
+      tstar = max(1, n / a.bits);
+    } else {
+      // thread u holds position t = n - 1 - u; its inclusive scan is the suffix sum S_t
+      const int t = n - 1 - tid;
+      const uint64_t v = (tid < n) ? key[t] : 0ull;
+      uint64_t total;
+      const uint64_t suffix = block_inclusive_scan(v, warp_sums, &total);
+      if (tid == 0) s_tstar = n;
+      __syncthreads();
+      if (tid < n) {
+        const int64_t lhs = (int64_t)(n - a.bits * t) * (int64_t)v;
+        if (lhs <= (int64_t)a.bits * (int64_t)suffix) atomicMin(&s_tstar, t);
+      }
+      __syncthreads();
+      tstar = s_tstar;
+      if (tid < n && t == tstar) s_stot = suffix;
+      if (tid == 0 && tstar >= n) s_stot = 0;
+      __syncthreads();
+      S = s_stot;
+    }
+    __syncthreads();
+    if (tid < n) {
+      uint64_t P;
+      if (a.mode == FQT1_SEL_TOPK) P = rank < tstar ? two32 : 0ull;
+      else if (rank < tstar) P = two32;
+      else if (S > 0) P = min(two32, div_shift32((uint64_t)(n - a.bits * tstar) * myrt, (uint64_t)a.bits * S));
+      else P = 0;
+      key[tid] = P;
+    }
+  } else if (a.bits > 1) {
     // sort keys (R~ desc, index asc) descending
     for (int i = tid; i < npad; i += kSelThreads)
       key[i] = i < n ? ((rtilde(i) << 24) | (uint64_t)(0xFFFFFFu - (uint32_t)i)) : 0ull;
@@ -329,7 +383,7 @@ struct QuantArgs {
 };
 
 template <bool VEC>
-__global__ void __launch_bounds__(256) quantize_kernel(QuantArgs a) {
+__global__ void __launch_bounds__(256, 4) quantize_kernel(QuantArgs a) {
   __shared__ uint32_t tile[kQCols][kQRows / 4 + 1];  // PCQ codes, 4 rows per word
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t cb = (int64_t)blockIdx.x * kQCols;
@@ -355,30 +409,35 @@ __global__ void __launch_bounds__(256) quantize_kernel(QuantArgs a) {
     }
   }
   uint8_t ccode[4][4] = {};  // [row i][col q]
-  for (int i = 0; i < 4; ++i) {
+  float vv[4][4];
+  int32_t sslots[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {  // slots and loads of this warp's 4 rows first
     const int64_t r = r0 + warp * 4 + i;
-    if (r >= a.M) break;
-    int32_t sslot = -1;
-    int64_t gi = 0;
-    if (a.do_psq) {
-      gi = r / a.rpg;
-      sslot = __ldg(a.s.slot + gi);
-    }
-    if (sslot < 0 && !any_c) continue;
-    float v[4];
+    sslots[i] = (a.do_psq && r < a.M) ? __ldg(a.s.slot + r / a.rpg) : -1;
+    const bool need = r < a.M && (sslots[i] >= 0 || any_c);
     if (VEC) {
-      if (cv[0]) {
+      if (need && cv[0]) {
         const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + c0));
-        v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+        vv[i][0] = t.x; vv[i][1] = t.y; vv[i][2] = t.z; vv[i][3] = t.w;
       } else {
-        v[0] = v[1] = v[2] = v[3] = 0.f;
+        vv[i][0] = vv[i][1] = vv[i][2] = vv[i][3] = 0.f;
       }
     } else {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) v[q] = cv[q] ? __ldg(a.g + r * a.D + c0 + q) : 0.0f;
+      for (int q = 0; q < 4; ++q) vv[i][q] = (need && cv[q]) ? __ldg(a.g + r * a.D + c0 + q) : 0.0f;
     }
+  }
 #pragma unroll
-    for (int q = 0; q < 4; ++q) v[q] = a.gamma ? __fmul_rn(v[q], gam[q]) : v[q];
+  for (int i = 0; i < 4; ++i) {
+    const int64_t r = r0 + warp * 4 + i;
+    if (r >= a.M) break;
+    const int32_t sslot = sslots[i];
+    const int64_t gi = r / a.rpg;
+    if (sslot < 0 && !any_c) continue;
+    float v[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) v[q] = a.gamma ? __fmul_rn(vv[i][q], gam[q]) : vv[i][q];
     const uint64_t e0 = (uint64_t)r * (uint64_t)a.D + (uint64_t)c0;
     if (sslot >= 0) {
       const float rs = __ldg(a.s.range + gi), zs = __ldg(a.s.zmin + gi);

@@ -150,6 +150,10 @@ CASES = [
     ("conv-ragged-s2-topk", lambda: conv_case(3, 5, 7, 6, 12, 3, 2, 1, 2, TOP)),
     ("conv-7x7-s2-b4", lambda: conv_case(2, 3, 20, 20, 16, 7, 2, 3, 4, SYS, seed=1)),
     ("conv-1x1-s2-b8", lambda: conv_case(4, 8, 9, 9, 24, 1, 2, 0, 8, SYS, seed=2)),
+    # region of a 256-column tile too large for the bit-level Unfolder: the generic gather path
+    ("conv-1x1-256ch-56x56-gather", lambda: conv_case(2, 256, 56, 56, 16, 1, 1, 0, 4, SYS, seed=3)),
+    ("conv-3x3-s1-multi-image-tiles", lambda: conv_case(9, 20, 5, 7, 40, 3, 1, 1, 2, BER, seed=4)),
+    ("conv-5x5-s3-p2", lambda: conv_case(3, 6, 17, 13, 8, 5, 3, 2, 4, SYS, seed=5)),
 ]
 
 
