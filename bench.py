@@ -30,6 +30,27 @@ WORKLOAD = "resnet18-cifar conv3x3 256->256 8x8 batch128 (M=8192 K=2304 D=256), 
 FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS = 6800.0, 1900.0
 SMS, POPC_PER_CLK_SM = 152, 16
 
+# DRAM bytes (read + write) per launch of each stage's kernels, from one ncu capture of
+# `bench.py --profile 2 --warmup 1` (profiles/kernels_resnet18_cifar_conv_full.md).  They are
+# valid only for the kernel sources they were taken on: TRAFFIC_SOURCES is the sha256 prefix of
+# paper_2408_14267_gb300/csrc at that capture; any other source tree reports traffic = null.
+TRAFFIC_SOURCES = "a731c2adfbbf5134"
+TRAFFIC_BYTES = {"pack_w": 2.379264e6, "im2col": 8.428288e6, "fwd_gemm": 2.492160e6,
+                 "scq_quantize": 8.414720e6 + 0.059904e6 + 8.434944e6, "bwd_input_gemm": 0.650752e6 + 256,
+                 "col2im": 0.007168e6 + 18.904064e6, "bwd_weight_gemm": 3.525888e6 + 0.606464e6}
+
+
+def sources_sha():
+    import glob
+    import hashlib
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2408_14267_gb300", "csrc")
+    for f in sorted(glob.glob(os.path.join(csrc, "*.cu")) + glob.glob(os.path.join(csrc, "*.cuh"))):
+        h.update(os.path.basename(f).encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
 CPU_SAMPLE_SCRIPT = r"""
 import json, sys, time
 sys.path.insert(0, sys.argv[1])
@@ -123,7 +144,10 @@ class ClockSampler:
 
 
 def stage_work(st, name):
-    """Algorithmic work of one stage: ('hbm', bytes) or ('alu', 1-bit ops) or ('tensor', ops)."""
+    """Algorithmic work of one stage: ('hbm', bytes) or ('tensor', dense-equivalent operations).
+
+    The products run on e4m3 tensor cores, so their peak is the fp8 dense rate (twice the
+    measured bf16 rate, the nominal ratio)."""
     from paper_2408_14267_gb300 import fqt1
     M, K, D = st.M, st.K, st.D
     wK, wM, wD = fqt1.packed_words(K), fqt1.packed_words(M), fqt1.packed_words(D)
@@ -134,15 +158,15 @@ def stage_work(st, name):
     if name in ("im2col", "pack_x"):
         return "hbm", st.x.numel() * 4 + (M * wK + K * wM + K) * 4
     if name == "fwd_gemm":
-        return "alu", 2.0 * M * K * D
+        return "tensor", 2.0 * M * K * D
     if name == "scq_quantize":
         return "hbm", M * D * 4 + ks * D + kc * M
     if name == "bwd_input_gemm":
-        return "alu", 2.0 * ks * D * K * st.p_s.bits
+        return "tensor", 2.0 * ks * D * K
     if name == "col2im":
         return "hbm", ks * K * 4 + st.dx.numel() * 4
     if name == "bwd_weight_gemm":
-        return "alu", 2.0 * kc * M * K * st.p_c.bits
+        return "tensor", 2.0 * kc * M * K
     return "hbm", 0
 
 
@@ -262,13 +286,14 @@ def main():
     if bound == "hbm":
         roof = {"bound": "hbm", "achieved": work / dur_s / 1e9, "peak": hbm_peak, "unit": "GB/s"}
     elif bound == "tensor":
-        roof = {"bound": "tensor", "achieved": work / dur_s / 1e12, "peak": 2.0 * bf16_peak, "unit": "TFLOP/s"}
+        roof = {"bound": "tensor", "achieved": work / dur_s / 1e12, "peak": 2.0 * bf16_peak, "unit": "TFLOP/s",
+                "peak_note": "fp8 dense = 2 x measured bf16 (nominal fp8/bf16 ratio)"}
     else:
         clk_mhz = clocks.get("sm_max_mhz") or 2070.0
         alu_peak = SMS * POPC_PER_CLK_SM * 32 * 2 * clk_mhz * 1e6 / 1e12
         roof = {"bound": "alu", "achieved": work / dur_s / 1e12, "peak": alu_peak, "unit": "TOPS"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = None
+    roof["traffic"] = TRAFFIC_BYTES.get(dom) if sources_sha() == TRAFFIC_SOURCES else None
     roof["kernel"] = dom
     roof["peak_source"] = peak_src if bound != "alu" else "derived: 152 SMs x 16 popc/clk x 32 bit x 2 x max clock"
 
@@ -318,7 +343,7 @@ def main():
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
-                "vs_baseline": None, "dtype": "b1", "data": "synthetic",
+                "vs_baseline": None, "dtype": "e4m3", "data": "synthetic",
                 "config": {"workload": WORKLOAD, "l2": "flushed before every timed step (256 MiB write)",
                            "timing": "CUDA-graph replay of the whole step (three stream branches: pack W | "
                                      "pack X + forward + grad_weight | SCQ + grad_input + Folder), CUDA events "
