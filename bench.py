@@ -161,7 +161,7 @@ def stage_work(st, name):
         return "tensor", 2.0 * M * K * D
     if name == "scq_quantize":
         return "hbm", M * D * 4 + ks * D + kc * M
-    if name == "bwd_input_gemm":
+    if name in ("bwd_input_gemm", "bwd_input_fold"):
         return "tensor", 2.0 * ks * D * K
     if name == "col2im":
         return "hbm", ks * K * 4 + st.dx.numel() * 4
@@ -346,8 +346,8 @@ def main():
                 "vs_baseline": None, "dtype": "e4m3", "data": "synthetic",
                 "config": {"workload": WORKLOAD, "l2": "flushed before every timed step (256 MiB write)",
                            "timing": "CUDA-graph replay of the whole step (three stream branches: pack W | "
-                                     "pack X + forward + grad_weight | SCQ + grad_input + Folder), CUDA events "
-                                     "on the launching stream",
+                                     "pack X + forward + grad_weight | SCQ + grad_input with the Folder in its "
+                                     "epilogue), CUDA events on the launching stream",
                            "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU"},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
                 "clocks": clocks, "stage_ms": {k: round(v, 5) for k, v in stage_ms.items()}}

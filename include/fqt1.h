@@ -190,6 +190,17 @@ fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, const int32_t
                         int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad, float* dx,
                         void* stream);
 
+/* grad_input of a convolution with the Folder fused into the product (Eq. 21 with
+ * Sec. 5.3's per-sample scales, App. C Folder): the same dx as fqt1_bwd_input_gemm
+ * followed by fqt1_col2im, without the int32 accumulators in memory.  A tile of 128
+ * accumulator rows holds whole samples, so this call requires Ho*Wo to divide 128
+ * (maps of 8x8, 4x4, 2x2 ... pixels) and kh*kw <= 256; other shapes return
+ * FQT1_ERR_UNSUPPORTED (use the two-call path).  p->rows_per_group must be Ho*Wo.
+ * sw_col: [K = C*kh*kw][words(D)]; colsum_w: [K]; dx: [N, C, H, W] (pruned samples 0). */
+fqt1_status fqt1_bwd_input_fold(const fqt1_qgrad* psq, const uint32_t* sw_col, const int32_t* colsum_w, int32_t N,
+                                int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad,
+                                int64_t D, const fqt1_agp_params* p, float* dx, void* stream);
+
 /* grad_weight side of SCQ (Eq. 21 with Sec. 5.3's per-channel scales):
  * acc[c, k] = sum_m q^c[c, m] sign(X)[m, k] for kept channel slots c,
  * dw[j, k] = S^c'_j acc + Z^c'_j colsum_x[k] for kept channels j, 0 for pruned.

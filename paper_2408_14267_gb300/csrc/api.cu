@@ -46,6 +46,8 @@ bool use_popcount_path() {
 // chunks of 1024 floats, y (and z for more than 65535 rows) the rows.
 __global__ void zero_pruned_rows_kernel(const int32_t* __restrict__ slot_of_group, int64_t M, int64_t K, int64_t rpg,
                                         float* __restrict__ out) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   const int64_t row = (int64_t)blockIdx.z * 65535 + blockIdx.y;
   if (row >= M || __ldg(slot_of_group + row / rpg) >= 0) return;
   float* dst = out + row * K;
@@ -60,7 +62,7 @@ __global__ void zero_pruned_rows_kernel(const int32_t* __restrict__ slot_of_grou
 static void launch_zero_pruned_rows(const int32_t* slot_of_group, int64_t M, int64_t K, int64_t rpg, float* out,
                                     cudaStream_t s) {
   const dim3 grid((unsigned)((K + 1023) / 1024), (unsigned)(M < 65535 ? M : 65535), (unsigned)((M + 65534) / 65535));
-  zero_pruned_rows_kernel<<<grid, 256, 0, s>>>(slot_of_group, M, K, rpg, out);
+  launch_k(zero_pruned_rows_kernel, dim3(grid), dim3(256), 0, s, slot_of_group, M, K, rpg, out);
   fqt1_count_launches(1);
 }
 
@@ -70,6 +72,8 @@ __global__ void dequant_rows_kernel(const int32_t* __restrict__ acc, int64_t lda
                                     const int32_t* __restrict__ slot_of_group, const float* __restrict__ scale,
                                     const float* __restrict__ zero, const int32_t* __restrict__ cs, int64_t M,
                                     int64_t K, int64_t rpg, float* __restrict__ out) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= M * K) return;
   const int64_t m = idx / K, k = idx - (idx / K) * K;
@@ -88,6 +92,8 @@ __global__ void col2im_kernel(const int32_t* __restrict__ acc, const int32_t* __
                               const float* __restrict__ scale, const float* __restrict__ zero,
                               const int32_t* __restrict__ cs, int N, int C, int H, int W, int kh, int kw, int stride,
                               int pad, int Ho, int Wo, float* __restrict__ dx) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t total = (int64_t)N * C * H * W;
   if (idx >= total) return;
@@ -140,6 +146,8 @@ struct FoldArgs {
 };
 
 __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   extern __shared__ int32_t fold_smem[];
   const int32_t slot = (int32_t)blockIdx.y;  // one kept sample per grid row
   if (slot >= __ldg(a.kept_count)) return;
@@ -281,7 +289,7 @@ extern "C" fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t
   }
   if (dx) {
     const int64_t n = M * K;
-    dequant_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(acc, K, psq->slot_of_group, psq->scale,
+    launch_k(dequant_rows_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, acc, K, psq->slot_of_group, psq->scale,
                                                                     psq->zero, colsum_w, M, K, rpg, dx);
     fqt1_count_launches(1);
     FQT1_CUDA_TRY(cudaGetLastError());
@@ -336,14 +344,41 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
     // pruned samples: zeros; kept samples: the tiled fold (one grid row per kept slot)
     launch_zero_pruned_rows(psq->slot_of_group, N, (int64_t)C * H * W, 1, dx, (cudaStream_t)stream);
     const int64_t cap = fqt1_kept_capacity(N, 8, FQT1_SEL_BERNOULLI);  // upper bound: all samples
-    col2im_tiled_kernel<<<dim3((unsigned)nblk, (unsigned)cap), 256, smem, (cudaStream_t)stream>>>(fa);
+    launch_k(col2im_tiled_kernel, dim3((unsigned)nblk, (unsigned)cap), dim3(256), smem, (cudaStream_t)stream, fa);
   } else {
     const int64_t n = (int64_t)N * C * H * W;
-    col2im_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(
+    launch_k(col2im_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, (cudaStream_t)stream, 
         acc, psq->slot_of_group, psq->scale, psq->zero, colsum_w, N, C, H, W, kh, kw, stride, pad, Ho, Wo, dx);
   }
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
+  return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_bwd_input_fold(const fqt1_qgrad* psq, const uint32_t* sw_col, const int32_t* colsum_w,
+                                           int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw,
+                                           int32_t stride, int32_t pad, int64_t D, const fqt1_agp_params* p,
+                                           float* dx, void* stream) {
+  if (!psq || !sw_col || !colsum_w || !p || !dx || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 ||
+      stride < 1 || pad < 0 || D < 1)
+    return FQT1_ERR_INVALID_ARG;
+  if (!valid_bits(p->bits) || !psq->codes || !psq->kept_count || !psq->kept_idx || !psq->slot_of_group ||
+      !psq->scale || !psq->zero || psq->ld_codes < fqt1_codes_ld(D) || psq->ld_codes % 16)
+    return FQT1_ERR_INVALID_ARG;
+  if (H + 2 * pad < kh || W + 2 * pad < kw) return FQT1_ERR_INVALID_ARG;
+  const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
+  if (p->rows_per_group != (int64_t)Ho * Wo) return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(sw_col) || !aligned16(dx) || !aligned16(colsum_w)) return FQT1_ERR_MISALIGNED;
+  // whole samples per 128-row tile and at least one channel's taps per 256-column tile
+  if (128 % (Ho * Wo) != 0 || kh * kw > 256 || (int64_t)N * C * H * W >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
+  cudaStream_t s = (cudaStream_t)stream;
+  const int64_t rpg = (int64_t)Ho * Wo;
+  const int64_t cap_rows = fqt1_kept_capacity(N, p->bits, p->mode) * rpg;
+  launch_zero_pruned_rows(psq->slot_of_group, N, (int64_t)C * H * W, 1, dx, s);
+  FQT1_CUDA_TRY(cudaGetLastError());
+  FQT1_CUDA_TRY(launch_fold_tc(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, sw_col,
+                               (int64_t)C * kh * kw, D, psq->kept_idx, psq->scale, psq->zero, colsum_w, dx, C, H, W,
+                               kh, kw, stride, pad, Ho, Wo, nullptr, s));
   return FQT1_OK;
 }
 
@@ -378,7 +413,7 @@ extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_
                                          nullptr, 1, nullptr, s));
   }
   const int64_t n = D * K;
-  dequant_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(acc, K, pcq->slot_of_group, pcq->scale, pcq->zero,
+  launch_k(dequant_rows_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, acc, K, pcq->slot_of_group, pcq->scale, pcq->zero,
                                                                   colsum_x, D, K, 1, dw);
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());

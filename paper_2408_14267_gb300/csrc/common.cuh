@@ -94,6 +94,31 @@ __device__ __forceinline__ uint32_t sr_code(float x, float z, float inv, float B
     }                                                    \
   } while (0)
 
+// Programmatic dependent launch: every kernel of the library is launched with programmatic
+// stream serialization, so its launch and prologue may overlap the tail of the kernel before
+// it in the stream.  A kernel calls FQT1_PDL_WAIT() before it touches memory written by
+// earlier work (it then sees all of it), and FQT1_PDL_TRIGGER() to let the next kernel start.
+#define FQT1_PDL_WAIT() asm volatile("griddepcontrol.wait;" ::: "memory")
+#define FQT1_PDL_TRIGGER() asm volatile("griddepcontrol.launch_dependents;" ::: "memory")
+
+namespace fqt1 {
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                            Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+}  // namespace fqt1
+
 void fqt1_set_cuda_error(cudaError_t e);
 // Replaces the text returned by fqt1_last_cuda_error() with msg.
 void fqt1_set_error_text(const char* msg);

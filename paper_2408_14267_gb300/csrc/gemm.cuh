@@ -20,6 +20,10 @@ cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int6
                                    const float* scale, const float* zero, const int32_t* cs, int64_t rpg,
                                    int32_t* status, cudaStream_t s);
 enum : int { GEMM_EPI_ACC32 = 1, GEMM_EPI_RED = 2, GEMM_EPI_DX = 3 };
+cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
+                           const uint32_t* Sg, int64_t K, int64_t D, const int32_t* kept_idx, const float* scale,
+                           const float* zero, const int32_t* cs, float* dx, int C, int H, int W, int kh, int kw,
+                           int stride, int pad, int Ho, int Wo, int32_t* status, cudaStream_t s);
 // Largest contraction one CTA may sum in fp32 and stay exact: partial sums below 2^24.
 inline int64_t exact_chunk(int bits) { return (int64_t)((1 << 24) / ((1 << bits) - 1)); }
 // 1 if FQT1_GEMM_PATH=popcount selects the CUDA-core kernels (datapath comparison only).

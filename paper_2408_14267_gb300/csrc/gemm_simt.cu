@@ -14,6 +14,8 @@ __global__ void __launch_bounds__(256) xnor_gemm_simt_kernel(const uint32_t* __r
                                                              const uint32_t* __restrict__ B, int64_t M, int64_t N,
                                                              int64_t K, int64_t ldw, const float* __restrict__ gamma,
                                                              int32_t* __restrict__ acc_out, float* __restrict__ y) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   __shared__ uint32_t As[kSW][kST + 1], Bs[kSW][kST + 1];
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
   const int64_t m0 = (int64_t)blockIdx.y * kST, n0 = (int64_t)blockIdx.x * kST;
@@ -62,6 +64,8 @@ __global__ void __launch_bounds__(256) codes_gemm_simt_kernel(const uint8_t* __r
                                                               const uint32_t* __restrict__ S, int64_t lds,
                                                               int64_t n_s, int64_t L, int32_t* __restrict__ out,
                                                               int64_t ldo) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   __shared__ uint32_t Ap[BITS][kSW][kST + 1], Bs[kSW][kST + 1];
   const int64_t n_r = (int64_t)__ldg(count) * rows_per_count;
   const int64_t r0 = (int64_t)blockIdx.y * kST, s0 = (int64_t)blockIdx.x * kST;
@@ -124,7 +128,7 @@ cudaError_t launch_xnor_gemm_simt(const uint32_t* A, const uint32_t* B, int64_t 
                                   const float* gamma, int32_t* acc, float* y, cudaStream_t s) {
   const int64_t ldw = fqt1_packed_words(K);
   dim3 grid((unsigned)((N + kST - 1) / kST), (unsigned)((M + kST - 1) / kST));
-  xnor_gemm_simt_kernel<<<grid, 256, 0, s>>>(A, B, M, N, K, ldw, gamma, acc, y);
+  launch_k(xnor_gemm_simt_kernel, dim3(grid), dim3(256), 0, s, A, B, M, N, K, ldw, gamma, acc, y);
   fqt1_count_launches(1);
   return cudaGetLastError();
 }
@@ -135,10 +139,10 @@ cudaError_t launch_codes_gemm_simt(int bits, const uint8_t* Q, int64_t ldq, cons
   const int64_t lds = fqt1_packed_words(L);
   dim3 grid((unsigned)((n_s + kST - 1) / kST), (unsigned)((max_rows + kST - 1) / kST));
   switch (bits) {
-    case 1: codes_gemm_simt_kernel<1><<<grid, 256, 0, s>>>(Q, ldq, count, rows_per_count, S, lds, n_s, L, out, ldo); break;
-    case 2: codes_gemm_simt_kernel<2><<<grid, 256, 0, s>>>(Q, ldq, count, rows_per_count, S, lds, n_s, L, out, ldo); break;
-    case 4: codes_gemm_simt_kernel<4><<<grid, 256, 0, s>>>(Q, ldq, count, rows_per_count, S, lds, n_s, L, out, ldo); break;
-    default: codes_gemm_simt_kernel<8><<<grid, 256, 0, s>>>(Q, ldq, count, rows_per_count, S, lds, n_s, L, out, ldo); break;
+    case 1: launch_k(codes_gemm_simt_kernel<1>, dim3(grid), dim3(256), 0, s, Q, ldq, count, rows_per_count, S, lds, n_s, L, out, ldo); break;
+    case 2: launch_k(codes_gemm_simt_kernel<2>, dim3(grid), dim3(256), 0, s, Q, ldq, count, rows_per_count, S, lds, n_s, L, out, ldo); break;
+    case 4: launch_k(codes_gemm_simt_kernel<4>, dim3(grid), dim3(256), 0, s, Q, ldq, count, rows_per_count, S, lds, n_s, L, out, ldo); break;
+    default: launch_k(codes_gemm_simt_kernel<8>, dim3(grid), dim3(256), 0, s, Q, ldq, count, rows_per_count, S, lds, n_s, L, out, ldo); break;
   }
   fqt1_count_launches(1);
   return cudaGetLastError();

@@ -35,7 +35,7 @@ constexpr int kExpWarps = 8;       // two expansion / epilogue warps per SM sub-
 constexpr int kThreads = 32 * (2 + kExpWarps);
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on every wait
 
-enum : int { EPI_FWD = 0, EPI_ACC32 = 1, EPI_RED = 2, EPI_DX = 3 };
+enum : int { EPI_FWD = 0, EPI_ACC32 = 1, EPI_RED = 2, EPI_DX = 3, EPI_FOLD = 4 };
 
 struct TcArgs {
   int64_t M, N, L;           // rows (capacity), columns, contraction length
@@ -53,6 +53,11 @@ struct TcArgs {
   const int32_t* cs;
   int64_t rpg;
   int32_t* status;
+  // EPI_FOLD: grad_input of a convolution with the Folder in the epilogue.  A CTA's rows are
+  // whole samples (rpg = Ho*Wo divides 128) and its columns the kernel taps of fcb channels
+  // starting at channel blockIdx.x * fcb (column offset n_step = fcb * kh * kw).
+  int n_step, grid_x;
+  int fC, fH, fW, fkh, fkw, fstride, fpad, fHo, fWo, fcb;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -192,13 +197,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ volatile int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t m0 = (int64_t)blockIdx.y * kBM, n0 = (int64_t)blockIdx.x * BN;
-  const int64_t valid_rows = a.count ? (int64_t)__ldg(a.count) * a.rows_per_count : a.M;
-  if (m0 >= valid_rows) return;
+  const int64_t m0 = (int64_t)blockIdx.y * kBM, n0 = (int64_t)blockIdx.x * (a.n_step > 0 ? a.n_step : BN);
   const int kt0 = blockIdx.z * a.tiles_per_split;
   const int kt1 = min(a.k_tiles, kt0 + a.tiles_per_split);
-  if (kt0 >= kt1) return;
-  const int nk = kt1 - kt0;
+  if (kt0 >= kt1) {
+    FQT1_PDL_TRIGGER();
+    return;
+  }
 
   unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   auto opA = [&](int s) { return base + s * S::kOpStage; };
@@ -220,10 +225,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                  "r"(BN));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
+  if (threadIdx.x == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+  }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = tmem_slot;
+  // the setup above overlaps the previous kernel; operands and the kept count are read after this
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  const int64_t valid_rows = a.count ? (int64_t)__ldg(a.count) * a.rows_per_count : a.M;
+  const int nk = m0 < valid_rows ? kt1 - kt0 : 0;  // a tile past the kept rows has no work
 
   constexpr uint32_t kTx = (uint32_t)S::kRawStage;
 
@@ -350,6 +364,72 @@ __global__ void __launch_bounds__(kThreads, 1)
     // one coalesced 128-byte row per store instruction (lane = column).
     const bool have_acc = mbar_wait(&acc_full, 0, &abort_flag, a.status);
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    if (a.epi == EPI_FOLD) {
+      // 1. the whole 128 x BN accumulator tile -> shared memory as int32 (rings are idle);
+      //    row stride BN + 1 keeps the 32 rows of a warp in distinct banks
+      constexpr int TS = BN + 1;
+      int32_t* T = reinterpret_cast<int32_t*>(base);
+      const int qf = warp & 3, cbegf = ((warp - 2) >> 2) * (BN / 2);
+      for (int c0 = cbegf; c0 < cbegf + BN / 2; c0 += 32) {
+        __syncwarp();
+        uint32_t v[32];
+        const uint32_t taddr = tmem + ((uint32_t)(32 * qf) << 16) + (uint32_t)c0;
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,"
+            "%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+            : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+              "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
+              "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
+              "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+            : "r"(taddr));
+        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        int32_t* trow = T + (32 * qf + lane) * TS + c0;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) trow[j] = __float2int_rn(__uint_as_float(v[j]));
+      }
+      // tap tables: hrow[h*kh + i] = oh*Wo or -1, wcol[w*kw + j] = ow or -1 (input pixel -> output pixel)
+      int32_t* hrow = T + kBM * TS;
+      int32_t* wcol = hrow + a.fH * a.fkh;
+      for (int x = threadIdx.x - 64; x < a.fH * a.fkh; x += 256) {
+        const int h = x / a.fkh, i = x - h * a.fkh, hn = h + a.fpad - i;
+        hrow[x] = (hn >= 0 && hn % a.fstride == 0 && hn / a.fstride < a.fHo) ? (hn / a.fstride) * a.fWo : -1;
+      }
+      for (int x = threadIdx.x - 64; x < a.fW * a.fkw; x += 256) {
+        const int w = x / a.fkw, j = x - w * a.fkw, wn = w + a.fpad - j;
+        wcol[x] = (wn >= 0 && wn % a.fstride == 0 && wn / a.fstride < a.fWo) ? wn / a.fstride : -1;
+      }
+      asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
+      // 2. Folder: dx[n, c, h, w] = S'_n sum(acc taps) + Z'_n sum(colsum taps)
+      const int rpg = (int)a.rpg, imgs = kBM / rpg, khw = a.fkh * a.fkw, HW = a.fH * a.fW;
+      const int c_first = blockIdx.x * a.fcb, nc = min(a.fcb, a.fC - c_first);
+      const int64_t slot0 = m0 / rpg, nslots = valid_rows / rpg;
+      const int per_img = nc * HW;
+      const FastDiv div_img((uint32_t)per_img), div_hw((uint32_t)HW), div_w((uint32_t)a.fW);
+      const int32_t* csb = a.cs + (int64_t)c_first * khw;
+      for (int e = threadIdx.x - 64; have_acc && e < imgs * per_img; e += 256) {
+        const int img = (int)div_img.div((uint32_t)e), rem = e - img * per_img;
+        const int64_t slot = slot0 + img;
+        if (slot >= nslots) break;
+        const int cl = (int)div_hw.div((uint32_t)rem), pos = rem - cl * HW;
+        const int h = (int)div_w.div((uint32_t)pos), w = pos - h * a.fW;
+        int32_t acc = 0, csum = 0;
+        const int32_t* timg = T + img * rpg * TS + cl * khw;
+        for (int i = 0; i < a.fkh; ++i) {
+          const int ro = hrow[h * a.fkh + i];
+          if (ro < 0) continue;
+          for (int j = 0; j < a.fkw; ++j) {
+            const int co = wcol[w * a.fkw + j];
+            if (co < 0) continue;
+            const int tap = i * a.fkw + j;
+            acc += timg[(ro + co) * TS + tap];
+            csum += __ldg(csb + cl * khw + tap);
+          }
+        }
+        const int64_t n = __ldg(a.kept_idx + slot);
+        a.y[((n * a.fC + c_first + cl) * a.fH + h) * a.fW + w] =
+            __fadd_rn(__fmul_rn(__ldg(a.scale + slot), (float)acc), __fmul_rn(__ldg(a.zero + slot), (float)csum));
+      }
+    } else {
     const int q = warp & 3;                         // TMEM lane quarter of this warp
     const int cbeg = ((warp - 2) >> 2) * (BN / 2);  // its half of the accumulator columns
     uint32_t* stage = reinterpret_cast<uint32_t*>(base) + (warp - 2) * 1024;  // 4 KB per warp (operand ring is idle)
@@ -452,6 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+    }  // epilogue modes other than EPI_FOLD
   }
 
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -500,8 +581,9 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  dim3 grid((unsigned)((a.N + BN - 1) / BN), (unsigned)((a.M + kBM - 1) / kBM), (unsigned)splits);
-  tc_gemm_kernel<A_CODES, BITS8, BN><<<grid, kThreads, S::kBytes, s>>>(ma, mb, a);
+  dim3 grid((unsigned)(a.grid_x > 0 ? a.grid_x : (a.N + BN - 1) / BN), (unsigned)((a.M + kBM - 1) / kBM),
+            (unsigned)splits);
+  launch_k(tc_gemm_kernel<A_CODES, BITS8, BN>, dim3(grid), dim3(kThreads), S::kBytes, s, ma, mb, a);
   fqt1_count_launches(1);
   return cudaGetLastError();
 }
@@ -539,6 +621,29 @@ cudaError_t launch_codes_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max
   const int z = (a.k_tiles + a.tiles_per_split - 1) / a.tiles_per_split;
   if (bits == 8) return launch_tc<true, true, 128>(ma, mb, a, z, s);
   return launch_tc<true, false, 128>(ma, mb, a, z, s);
+}
+
+// grad_input of a convolution with the Folder in the epilogue (EPI_FOLD, 256-column tiles).
+cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
+                           const uint32_t* Sg, int64_t K, int64_t D, const int32_t* kept_idx, const float* scale,
+                           const float* zero, const int32_t* cs, float* dx, int C, int H, int W, int kh, int kw,
+                           int stride, int pad, int Ho, int Wo, int32_t* status, cudaStream_t s) {
+  const int64_t lds = fqt1_packed_words(D);
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, D, max_rows, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, 4, 256, CU_TENSOR_MAP_SWIZZLE_NONE))
+    return cudaErrorInvalidValue;
+  TcArgs a{};
+  const int khw = kh * kw, cb = 256 / khw;
+  a.M = max_rows; a.N = K; a.L = D; a.count = count; a.rows_per_count = (int64_t)Ho * Wo;
+  a.k_tiles = (int)((D + kBK - 1) / kBK); a.tiles_per_split = a.k_tiles;
+  a.epi = EPI_FOLD; a.y = dx; a.kept_idx = kept_idx; a.scale = scale; a.zero = zero; a.cs = cs;
+  a.rpg = (int64_t)Ho * Wo; a.status = status;
+  a.n_step = cb * khw; a.grid_x = (C + cb - 1) / cb;
+  a.fC = C; a.fH = H; a.fW = W; a.fkh = kh; a.fkw = kw; a.fstride = stride; a.fpad = pad; a.fHo = Ho; a.fWo = Wo;
+  a.fcb = cb;
+  if (bits == 8) return launch_tc<true, true, 256>(ma, mb, a, 1, s);
+  return launch_tc<true, false, 256>(ma, mb, a, 1, s);
 }
 
 cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,

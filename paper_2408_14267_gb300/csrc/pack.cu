@@ -73,6 +73,8 @@ template <class Loader>
 __global__ void __launch_bounds__(256) pack_kernel(Loader L, uint32_t* __restrict__ row_bits, int64_t row_words,
                                                    uint32_t* __restrict__ col_bits, int64_t col_words,
                                                    int32_t* __restrict__ colsum) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   constexpr int R = Loader::kRows;
   __shared__ uint32_t rw[R][kPackWordsPerCta];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -127,6 +129,8 @@ __global__ void __launch_bounds__(256) pack_kernel(Loader L, uint32_t* __restric
 
 // Column-packed words past ceil(rows/32) (the alignment padding) are zero.
 __global__ void zero_col_pad_kernel(uint32_t* col_bits, int64_t cols, int64_t col_words, int64_t first_pad) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   const int64_t npad = col_words - first_pad;
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i < cols * npad) col_bits[(i / npad) * col_words + first_pad + (i % npad)] = 0u;
@@ -179,6 +183,8 @@ __device__ __forceinline__ uint32_t stream_bits(const uint32_t* st, int pos, int
 }
 
 __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   extern __shared__ uint32_t stream[];
   __shared__ uint32_t rw_s[256][9];  // row words [pixel in tile][k-word in tile]
   __shared__ uint32_t cw_s[256][9];  // column words [k in tile][pixel-word in tile]
@@ -339,12 +345,12 @@ static fqt1_status launch_pack(const Loader& L, uint32_t* row_bits, uint32_t* co
   if (row_tiles > 65535) return FQT1_ERR_UNSUPPORTED;
   if (colsum) FQT1_CUDA_TRY(cudaMemsetAsync(colsum, 0, sizeof(int32_t) * L.cols, s));
   dim3 grid((unsigned)word_tiles, (unsigned)row_tiles);
-  pack_kernel<Loader><<<grid, 256, 0, s>>>(L, row_bits, row_words, col_bits, col_words, colsum);
+  launch_k(pack_kernel<Loader>, dim3(grid), dim3(256), 0, s, L, row_bits, row_words, col_bits, col_words, colsum);
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
   if (col_bits && col_words > col_words_written) {
     const int64_t n = L.cols * (col_words - col_words_written);
-    zero_col_pad_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(col_bits, L.cols, col_words,
+    launch_k(zero_col_pad_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, col_bits, L.cols, col_words,
                                                                     col_words_written);
     fqt1_count_launches(1);
     FQT1_CUDA_TRY(cudaGetLastError());
@@ -409,13 +415,13 @@ extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t
         attr = true;
       }
       if (colsum) FQT1_CUDA_TRY(cudaMemsetAsync(colsum, 0, sizeof(int32_t) * Ki, s));
-      unfold_bits_kernel<<<dim3((unsigned)word_tiles, (unsigned)row_tiles), 256, (size_t)words * 4, s>>>(u);
+      launch_k(unfold_bits_kernel, dim3((unsigned)word_tiles, (unsigned)row_tiles), dim3(256), (size_t)words * 4, s, u);
       fqt1_count_launches(1);
       FQT1_CUDA_TRY(cudaGetLastError());
       const int64_t written = row_tiles * (tm / 32);
       if (col_bits && u.col_words > written) {
         const int64_t n = Ki * (u.col_words - written);
-        zero_col_pad_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(col_bits, Ki, u.col_words, written);
+        launch_k(zero_col_pad_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, col_bits, Ki, u.col_words, written);
         fqt1_count_launches(1);
         FQT1_CUDA_TRY(cudaGetLastError());
       }

@@ -21,13 +21,15 @@ struct RangeArgs {
   const float* g;
   const float* gamma;
   int64_t M, D, rpg;
-  uint32_t *smin, *smax;  // [M / rpg] or null
-  uint32_t *cmin, *cmax;  // [D] or null
+  uint32_t *smin, *smax;  // [M / rpg] or null (smax holds complemented keys)
+  uint32_t *cmin, *cmax;  // [D] or null (cmax holds complemented keys)
   int32_t* dev_status;
 };
 
 template <bool VEC>
 __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   __shared__ uint32_t cmin_s[8][kRangeCols], cmax_s[8][kRangeCols];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t c0 = (int64_t)blockIdx.x * kRangeCols + lane * 4;
@@ -68,7 +70,7 @@ __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
     if (a.smin && gi != cur) {
       if (cur >= 0) {
         const uint32_t mn = __reduce_min_sync(0xFFFFFFFFu, gmin), mx = __reduce_max_sync(0xFFFFFFFFu, gmax);
-        if (lane == 0) { atomicMin(a.smin + cur, mn); atomicMax(a.smax + cur, mx); }
+        if (lane == 0) { atomicMin(a.smin + cur, mn); atomicMin(a.smax + cur, ~mx); }
       }
       cur = gi;
       gmin = 0xFFFFFFFFu;
@@ -88,7 +90,7 @@ __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
   }
   if (a.smin && cur >= 0) {
     const uint32_t mn = __reduce_min_sync(0xFFFFFFFFu, gmin), mx = __reduce_max_sync(0xFFFFFFFFu, gmax);
-    if (lane == 0) { atomicMin(a.smin + cur, mn); atomicMax(a.smax + cur, mx); }
+    if (lane == 0) { atomicMin(a.smin + cur, mn); atomicMin(a.smax + cur, ~mx); }
   }
   if (__any_sync(0xFFFFFFFFu, bad) && lane == 0) atomicOr(a.dev_status, FQT1_DEV_NONFINITE);
   if (a.cmin) {
@@ -103,7 +105,7 @@ __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
       uint32_t mn = 0xFFFFFFFFu, mx = 0u;
 #pragma unroll
       for (int w = 0; w < 8; ++w) { mn = min(mn, cmin_s[w][threadIdx.x]); mx = max(mx, cmax_s[w][threadIdx.x]); }
-      if (c < a.D && mx != 0u) { atomicMin(a.cmin + c, mn); atomicMax(a.cmax + c, mx); }
+      if (c < a.D && mx != 0u) { atomicMin(a.cmin + c, mn); atomicMin(a.cmax + c, ~mx); }
     }
   }
 }
@@ -160,6 +162,8 @@ __device__ __forceinline__ uint64_t div_shift32(uint64_t a, uint64_t d) {
 }
 
 __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, SelectArgs a1) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   const SelectArgs& a = blockIdx.x == 0 ? a0 : a1;
   extern __shared__ __align__(16) unsigned char sel_smem[];
   __shared__ uint64_t warp_sums[32];
@@ -179,7 +183,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
   __syncthreads();
   for (int i = tid; i < n; i += kSelThreads) {
     const float z = ordered_to_float(a.kmin[i]);
-    const float r = __fsub_rn(ordered_to_float(a.kmax[i]), z);
+    const float r = __fsub_rn(ordered_to_float(~a.kmax[i]), z);
     o.group_min[i] = z;
     o.group_range[i] = r;
     rf[i] = r;
@@ -384,6 +388,8 @@ struct QuantArgs {
 
 template <bool VEC>
 __global__ void __launch_bounds__(256, 4) quantize_kernel(QuantArgs a) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
   __shared__ uint32_t tile[kQCols][kQRows / 4 + 1];  // PCQ codes, 4 rows per word
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t cb = (int64_t)blockIdx.x * kQCols;
@@ -557,15 +563,15 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
   uint32_t* cmin = smin + ns;
   uint32_t* smax = cmin + D;
   uint32_t* cmax = smax + ns;
-  FQT1_CUDA_TRY(cudaMemsetAsync(smin, 0xFF, sizeof(uint32_t) * (ns + D), s));
-  FQT1_CUDA_TRY(cudaMemsetAsync(smax, 0x00, sizeof(uint32_t) * (ns + D), s));
+  // min keys and complemented max keys both start at 0xFFFFFFFF and both take atomicMin
+  FQT1_CUDA_TRY(cudaMemsetAsync(smin, 0xFF, sizeof(uint32_t) * 2 * (ns + D), s));
 
   const bool vec = (D % 4) == 0;
   RangeArgs ra{g, gamma, M, D, rpg, psq ? smin : nullptr, psq ? smax : nullptr, pcq ? cmin : nullptr,
                pcq ? cmax : nullptr, dev_status};
   dim3 rgrid((unsigned)((D + kRangeCols - 1) / kRangeCols), (unsigned)((M + kRangeRows - 1) / kRangeRows));
-  if (vec) range_kernel<true><<<rgrid, 256, 0, s>>>(ra);
-  else range_kernel<false><<<rgrid, 256, 0, s>>>(ra);
+  if (vec) launch_k(range_kernel<true>, dim3(rgrid), dim3(256), 0, s, ra);
+  else launch_k(range_kernel<false>, dim3(rgrid), dim3(256), 0, s, ra);
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
 
@@ -592,7 +598,7 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
                                        (size_t)kMaxGroups * 12));
     attr_done = true;
   }
-  select_kernel<<<nsel, kSelThreads, smem, s>>>(sa[0], nsel > 1 ? sa[1] : sa[0]);
+  launch_k(select_kernel, dim3(nsel), dim3(kSelThreads), smem, s, sa[0], nsel > 1 ? sa[1] : sa[0]);
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
 
@@ -607,8 +613,8 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
                           (float)((1 << pc->bits) - 1), pc->seed};
   else qa.c = QBranch{};
   dim3 qgrid((unsigned)((D + kQCols - 1) / kQCols), (unsigned)((M + kQRows - 1) / kQRows));
-  if (vec) quantize_kernel<true><<<qgrid, 256, 0, s>>>(qa);
-  else quantize_kernel<false><<<qgrid, 256, 0, s>>>(qa);
+  if (vec) launch_k(quantize_kernel<true>, dim3(qgrid), dim3(256), 0, s, qa);
+  else launch_k(quantize_kernel<false>, dim3(qgrid), dim3(256), 0, s, qa);
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
   return FQT1_OK;

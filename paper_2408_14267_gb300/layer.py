@@ -27,7 +27,7 @@ class LayerStep:
     """Buffers and launches of one layer step.  keep_acc=False skips the optional
     int32 copy of the forward accumulators (the benchmark's configuration)."""
 
-    def __init__(self, wl, device="cuda", keep_acc=True):
+    def __init__(self, wl, device="cuda", keep_acc=True, fold=None):
         dev = torch.device(device)
         self.kind = wl["kind"]
         self.keep_acc = keep_acc
@@ -49,6 +49,13 @@ class LayerStep:
             D = self.w.shape[0]
             rpg = wl.get("rows_per_group", 1)
         self.M, self.K, self.D, self.rpg = M, K, D, rpg
+        # convolutions whose samples fit a 128-row tile fold grad_input in the GEMM epilogue,
+        # unless the int32 accumulators are kept (keep_acc) or fold is forced off
+        if self.kind == "conv":
+            ok = fqt1.fold_supported(Ho, Wo, kh, kw)
+            self.fold = (not keep_acc and ok) if fold is None else (fold and ok)
+        else:
+            self.fold = False
         wK, wM, wD = fqt1.packed_words(K), fqt1.packed_words(M), fqt1.packed_words(D)
         self.sx_row = torch.empty(M, wK, **i32)
         self.sx_col = torch.empty(K, wM, **i32)
@@ -94,7 +101,12 @@ class LayerStep:
         st.append(("scq_quantize", lambda s: fqt1.scq_quantize(self.gy, self.M, self.D, self.gamma, self.p_s,
                                                                self.p_c, self.psq, self.pcq, self.ws,
                                                                self.dev_status, s)))
-        if self.kind == "conv":
+        if self.kind == "conv" and self.fold:
+            N, Cin, H, W, kh, kw = self.conv
+            st.append(("bwd_input_fold", lambda s: fqt1.bwd_input_fold(self.psq, self.sw_col, self.cs_w, N, Cin, H, W,
+                                                                       kh, kw, self.stride, self.pad, self.D,
+                                                                       self.p_s, self.dx, s)))
+        elif self.kind == "conv":
             N, Cin, H, W, kh, kw = self.conv
             st.append(("bwd_input_gemm", lambda s: fqt1.bwd_input_gemm(self.psq, self.sw_col, self.cs_w, self.M,
                                                                        self.D, self.K, self.p_s, self.acc_dx, None,
@@ -148,9 +160,12 @@ class LayerStep:
         q_ready = torch.cuda.Event()
         q_ready.record(b2)
         b2.wait_event(w_ready)
-        st["bwd_input_gemm"](b2)
-        if "col2im" in st:
-            st["col2im"](b2)
+        if "bwd_input_fold" in st:
+            st["bwd_input_fold"](b2)
+        else:
+            st["bwd_input_gemm"](b2)
+            if "col2im" in st:
+                st["col2im"](b2)
         x_name = "im2col" if "im2col" in st else "pack_x"
         st[x_name](main)
         main.wait_event(w_ready)

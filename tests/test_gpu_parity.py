@@ -176,6 +176,38 @@ def test_layer_step_parity(name, make):
 
 LINEAR_CASES = [c for c in CASES if c[0].startswith("linear")]
 
+FOLD_CASES = [
+    ("fold-resnet18-cifar-8192x2304x256-b4", lambda: wl.resnet18_cifar_conv()),
+    ("fold-4x4-3x3-8-samples-per-tile", lambda: conv_case(6, 10, 4, 4, 20, 3, 1, 1, 4, SYS, seed=7)),
+    ("fold-8x8-b8", lambda: conv_case(5, 40, 8, 8, 24, 3, 1, 1, 8, SYS, seed=8)),
+    ("fold-2x2-topk", lambda: conv_case(40, 16, 2, 2, 8, 3, 1, 1, 2, TOP, seed=9)),
+    ("fold-5x5-kernel-4x4-map", lambda: conv_case(5, 30, 4, 4, 16, 5, 1, 2, 4, BER, seed=10)),
+    ("fold-stride2-16x16-to-8x8", lambda: conv_case(3, 12, 16, 16, 32, 3, 2, 1, 4, SYS, seed=11)),
+]
+
+
+@pytest.mark.parametrize("name,make", FOLD_CASES, ids=[c[0] for c in FOLD_CASES])
+def test_conv_fold_parity(name, make):
+    """grad_input with the Folder fused into the product equals the oracle's folded gradient."""
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    ref = run_oracle(w)
+    st = LayerStep(w, keep_acc=False)
+    assert st.fold
+    st.step()
+    torch.cuda.synchronize()
+    psq = ref["psq"]
+    a_mag = np.zeros(ref["dx"].shape)
+    c_mag = np.zeros(ref["dx"].shape)
+    for s_, g in enumerate(psq["kept"]):
+        a_mag[g] = np.abs(np.float64(psq["scale"][s_]) * ref["acc_fold"][g])
+        c_mag[g] = np.abs(np.float64(psq["zero"][s_]) * ref["cs_fold"])
+    assert_dequant_close(st.dx.cpu().numpy(), ref["dx"], a_mag, c_mag, "grad_input (fold)")
+    dx = st.dx.cpu().numpy()
+    for g in np.setdiff1d(np.arange(w["x"].shape[0]), psq["kept"]):
+        assert np.all(dx[g] == 0)
+    assert np.array_equal(st.y.cpu().numpy(), ref["y"])
+
 
 @pytest.mark.parametrize("name,make", LINEAR_CASES, ids=[c[0] for c in LINEAR_CASES])
 def test_linear_fused_dequant_parity(name, make):
