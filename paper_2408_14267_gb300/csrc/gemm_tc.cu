@@ -169,7 +169,7 @@ __device__ __forceinline__ uint32_t codes4_x16(uint32_t h) {
   return e + nz;
 }
 
-template <bool A_CODES, bool BITS8, int BN>
+template <bool A_CODES, bool BITS8, int BN, bool SHORT = false>
 struct TcSmem {
   static constexpr int kOpA = kBM * kBK;                        // bytes of one e4m3 A tile
   static constexpr int kOpB = BN * kBK;
@@ -177,17 +177,18 @@ struct TcSmem {
   static constexpr int kRawA = A_CODES ? kBM * kBK : kBM * 16;  // codes, or packed words (4 per row)
   static constexpr int kRawB = BN * 16;
   static constexpr int kRawStage = kRawA + kRawB;
-  static constexpr int kOpStages = BITS8 ? 2 : (A_CODES ? 3 : 4);
-  static constexpr int kRawStages = A_CODES ? 4 : 8;
+  // SHORT: two-stage rings for short contractions (two CTAs per SM)
+  static constexpr int kOpStages = SHORT ? 2 : (BITS8 ? 2 : (A_CODES ? 3 : 4));
+  static constexpr int kRawStages = SHORT ? 2 : (A_CODES ? 4 : 8);
   static constexpr int kBytes = kOpStages * kOpStage + kRawStages * kRawStage + 1024;  // + alignment slack
   static_assert(kOpStage % 1024 == 0 && kRawStage % 1024 == 0, "stages keep 1024-byte alignment");
   static_assert(kOpStages * kOpStage >= kExpWarps * 4096, "epilogue staging fits in the operand ring");
 };
 
-template <bool A_CODES, bool BITS8, int BN>
+template <bool A_CODES, bool BITS8, int BN, bool SHORT>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, TcArgs a) {
-  using S = TcSmem<A_CODES, BITS8, BN>;
+  using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
   constexpr int OS = S::kOpStages, RS = S::kRawStages;
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t raw_full[kMaxStages], raw_empty[kMaxStages], op_full[kMaxStages],
@@ -387,47 +388,62 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int j = 0; j < 32; ++j) trow[j] = __float2int_rn(__uint_as_float(v[j]));
       }
-      // tap tables: hrow[h*kh + i] = oh*Wo or -1, wcol[w*kw + j] = ow or -1 (input pixel -> output pixel)
-      int32_t* hrow = T + kBM * TS;
-      int32_t* wcol = hrow + a.fH * a.fkh;
-      for (int x = threadIdx.x - 64; x < a.fH * a.fkh; x += 256) {
-        const int h = x / a.fkh, i = x - h * a.fkh, hn = h + a.fpad - i;
-        hrow[x] = (hn >= 0 && hn % a.fstride == 0 && hn / a.fstride < a.fHo) ? (hn / a.fstride) * a.fWo : -1;
-      }
-      for (int x = threadIdx.x - 64; x < a.fW * a.fkw; x += 256) {
-        const int w = x / a.fkw, j = x - w * a.fkw, wn = w + a.fpad - j;
-        wcol[x] = (wn >= 0 && wn % a.fstride == 0 && wn / a.fstride < a.fWo) ? wn / a.fstride : -1;
-      }
-      asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
-      // 2. Folder: dx[n, c, h, w] = S'_n sum(acc taps) + Z'_n sum(colsum taps)
+      // per-CTA tables: for input position pos = h*W + w and tap t = i*kw + j, the tile offset
+      // (output pixel row * TS + t) of the accumulator that lands on it, or -1; the folded
+      // colsum of each (channel, position); each sample's kept id, scale and zero point
       const int rpg = (int)a.rpg, imgs = kBM / rpg, khw = a.fkh * a.fkw, HW = a.fH * a.fW;
       const int c_first = blockIdx.x * a.fcb, nc = min(a.fcb, a.fC - c_first);
-      const int64_t slot0 = m0 / rpg, nslots = valid_rows / rpg;
-      const int per_img = nc * HW;
-      const FastDiv div_img((uint32_t)per_img), div_hw((uint32_t)HW), div_w((uint32_t)a.fW);
-      const int32_t* csb = a.cs + (int64_t)c_first * khw;
-      for (int e = threadIdx.x - 64; have_acc && e < imgs * per_img; e += 256) {
-        const int img = (int)div_img.div((uint32_t)e), rem = e - img * per_img;
-        const int64_t slot = slot0 + img;
-        if (slot >= nslots) break;
-        const int cl = (int)div_hw.div((uint32_t)rem), pos = rem - cl * HW;
-        const int h = (int)div_w.div((uint32_t)pos), w = pos - h * a.fW;
-        int32_t acc = 0, csum = 0;
-        const int32_t* timg = T + img * rpg * TS + cl * khw;
-        for (int i = 0; i < a.fkh; ++i) {
-          const int ro = hrow[h * a.fkh + i];
-          if (ro < 0) continue;
-          for (int j = 0; j < a.fkw; ++j) {
-            const int co = wcol[w * a.fkw + j];
-            if (co < 0) continue;
-            const int tap = i * a.fkw + j;
-            acc += timg[(ro + co) * TS + tap];
-            csum += __ldg(csb + cl * khw + tap);
-          }
+      int32_t* tap_off = T + kBM * TS;                 // [HW][khw]
+      int32_t* csf = tap_off + HW * khw;               // [nc][HW]
+      float* s_scale = reinterpret_cast<float*>(csf + nc * HW);
+      float* s_zero = s_scale + imgs;
+      int32_t* s_n = reinterpret_cast<int32_t*>(s_zero + imgs);
+      const int tt = threadIdx.x - 64;
+      for (int x = tt; x < HW * khw; x += 256) {
+        const int pos = x / khw, t = x - pos * khw;
+        const int h = pos / a.fW, w = pos - h * a.fW, i = t / a.fkw, j = t - i * a.fkw;
+        const int hn = h + a.fpad - i, wn = w + a.fpad - j;
+        int v = -1;
+        if (hn >= 0 && wn >= 0 && hn % a.fstride == 0 && wn % a.fstride == 0) {
+          const int oh = hn / a.fstride, ow = wn / a.fstride;
+          if (oh < a.fHo && ow < a.fWo) v = (oh * a.fWo + ow) * TS + t;
         }
-        const int64_t n = __ldg(a.kept_idx + slot);
-        a.y[((n * a.fC + c_first + cl) * a.fH + h) * a.fW + w] =
-            __fadd_rn(__fmul_rn(__ldg(a.scale + slot), (float)acc), __fmul_rn(__ldg(a.zero + slot), (float)csum));
+        tap_off[x] = v;
+      }
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+      const int32_t* csb = a.cs + (int64_t)c_first * khw;
+      for (int x = tt; x < nc * HW; x += 256) {
+        const int cl = x / HW, pos = x - cl * HW;
+        int32_t cs = 0;
+        for (int t = 0; t < khw; ++t)
+          if (tap_off[pos * khw + t] >= 0) cs += __ldg(csb + cl * khw + t);
+        csf[x] = cs;
+      }
+      const int64_t slot0 = m0 / rpg, nslots = valid_rows / rpg;
+      if (tt < imgs) {
+        const int64_t slot = slot0 + tt;
+        s_n[tt] = slot < nslots ? __ldg(a.kept_idx + slot) : -1;
+        s_scale[tt] = slot < nslots ? __ldg(a.scale + slot) : 0.f;
+        s_zero[tt] = slot < nslots ? __ldg(a.zero + slot) : 0.f;
+      }
+      asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
+      // Folder: dx[n, c, h, w] = S'_n sum(acc taps) + Z'_n sum(colsum taps)
+      const int per_img = nc * HW;
+      const FastDiv div_img((uint32_t)per_img), div_hw((uint32_t)HW);
+      for (int e = tt; have_acc && e < imgs * per_img; e += 256) {
+        const int img = (int)div_img.div((uint32_t)e), rem = e - img * per_img;
+        const int n = s_n[img];
+        if (n < 0) break;
+        const int cl = (int)div_hw.div((uint32_t)rem), pos = rem - cl * HW;
+        const int32_t* tim = T + img * rpg * TS + cl * khw;
+        const int32_t* to = tap_off + pos * khw;
+        int32_t acc = 0;
+        for (int t = 0; t < khw; ++t) {
+          const int o = to[t];
+          if (o >= 0) acc += tim[o];
+        }
+        a.y[((int64_t)n * a.fC + c_first + cl) * HW + pos] =
+            __fadd_rn(__fmul_rn(s_scale[img], (float)acc), __fmul_rn(s_zero[img], (float)csf[rem]));
       }
     } else {
     const int q = warp & 3;                         // TMEM lane quarter of this warp
@@ -570,20 +586,20 @@ static bool make_map(CUtensorMap* m, const void* ptr, CUtensorMapDataType type, 
             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <bool A_CODES, bool BITS8, int BN>
+template <bool A_CODES, bool BITS8, int BN, bool SHORT = false>
 static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const TcArgs& a, int splits,
                              cudaStream_t s) {
-  using S = TcSmem<A_CODES, BITS8, BN>;
+  using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<A_CODES, BITS8, BN>,
+    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   dim3 grid((unsigned)(a.grid_x > 0 ? a.grid_x : (a.N + BN - 1) / BN), (unsigned)((a.M + kBM - 1) / kBM),
             (unsigned)splits);
-  launch_k(tc_gemm_kernel<A_CODES, BITS8, BN>, dim3(grid), dim3(kThreads), S::kBytes, s, ma, mb, a);
+  launch_k(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT>, dim3(grid), dim3(kThreads), S::kBytes, s, ma, mb, a);
   fqt1_count_launches(1);
   return cudaGetLastError();
 }
@@ -631,10 +647,10 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
   const int64_t lds = fqt1_packed_words(D);
   CUtensorMap ma, mb;
   if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, D, max_rows, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, 4, 256, CU_TENSOR_MAP_SWIZZLE_NONE))
+      !make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, 4, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
     return cudaErrorInvalidValue;
   TcArgs a{};
-  const int khw = kh * kw, cb = 256 / khw;
+  const int khw = kh * kw, cb = 128 / khw;
   a.M = max_rows; a.N = K; a.L = D; a.count = count; a.rows_per_count = (int64_t)Ho * Wo;
   a.k_tiles = (int)((D + kBK - 1) / kBK); a.tiles_per_split = a.k_tiles;
   a.epi = EPI_FOLD; a.y = dx; a.kept_idx = kept_idx; a.scale = scale; a.zero = zero; a.cs = cs;
@@ -642,8 +658,8 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
   a.n_step = cb * khw; a.grid_x = (C + cb - 1) / cb;
   a.fC = C; a.fH = H; a.fW = W; a.fkh = kh; a.fkw = kw; a.fstride = stride; a.fpad = pad; a.fHo = Ho; a.fWo = Wo;
   a.fcb = cb;
-  if (bits == 8) return launch_tc<true, true, 256>(ma, mb, a, 1, s);
-  return launch_tc<true, false, 256>(ma, mb, a, 1, s);
+  if (bits == 8) return launch_tc<true, true, 128, true>(ma, mb, a, 1, s);
+  return launch_tc<true, false, 128, true>(ma, mb, a, 1, s);
 }
 
 cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,

@@ -169,9 +169,11 @@ def bwd_input_fold(psq, sw_col, colsum_w, N, Cin, H, W, kh, kw, stride, pad, D, 
                                      C.byref(params), _p(dx), _s(stream)), "fqt1_bwd_input_fold")
 
 
-def fold_supported(Ho, Wo, kh, kw):
+def fold_supported(Ho, Wo, kh, kw, H, W):
     """The fused grad_input + Folder needs whole samples per 128-row tile (Ho*Wo divides 128)."""
-    return 128 % (Ho * Wo) == 0 and kh * kw <= 256
+    if 128 % (Ho * Wo) != 0 or kh * kw > 128:
+        return False
+    return 128 * 129 * 4 + 4 * H * W * kh * kw + 4 * (128 // (kh * kw)) * H * W + 64 <= 100 * 1024
 
 
 def bwd_weight_gemm(pcq, sx_col, colsum_x, M, D, K, params, acc, dw, ws=None, stream=None):

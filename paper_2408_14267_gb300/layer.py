@@ -52,7 +52,7 @@ class LayerStep:
         # convolutions whose samples fit a 128-row tile fold grad_input in the GEMM epilogue,
         # unless the int32 accumulators are kept (keep_acc) or fold is forced off
         if self.kind == "conv":
-            ok = fqt1.fold_supported(Ho, Wo, kh, kw)
+            ok = fqt1.fold_supported(Ho, Wo, kh, kw, H, W)
             self.fold = (not keep_acc and ok) if fold is None else (fold and ok)
         else:
             self.fold = False
