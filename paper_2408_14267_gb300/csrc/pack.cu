@@ -14,20 +14,8 @@ namespace fqt1 {
 constexpr int kPackWordsPerCta = 8;
 
 // A loader splits element (r, c) into a per-row part and a per-column part, so that a
-// warp computes its row part once per row and a lane its column parts once per CTA.
-struct DenseLoader {
-  static constexpr int kRows = 32;  // rows per CTA
-  const float* x;
-  int64_t rows, cols, ld;
-  struct Col { int64_t c; bool ok; };
-  struct Row { const float* p; bool ok; };
-  __device__ __forceinline__ Col col(int64_t c) const { return {c, c < cols}; }
-  __device__ __forceinline__ Row row(int64_t r) const { return {x + r * ld, r < rows}; }
-  __device__ __forceinline__ float load(const Row& r, const Col& c) const {
-    return (r.ok && c.ok) ? __ldg(r.p + c.c) : 0.0f;
-  }
-};
-
+// warp computes its row part once per row and a lane its column parts once per CTA.  The
+// gather path below serves unfolds whose input region does not fit the bit-level kernel.
 // Element (m, k) of the unfolded matrix X_u = Unfolder(x); outside the image it is 0.
 // Column k = (c*kh + i)*kw + j, row m = (n*Ho + oh)*Wo + ow.  All indices fit in 32 bits
 // (checked on the host); divisions by the layer's constants use FastDiv.
@@ -124,6 +112,39 @@ __global__ void __launch_bounds__(256) pack_kernel(Loader L, uint32_t* __restric
       if (nvalid > 0) sum += 2 * __popc(cw) - (int)nvalid;
     }
     if (colsum) atomicAdd(colsum + c, sum);
+  }
+}
+
+// Dense sign-pack: one warp per 32 x 32 block of x.  Lane l loads column c0 + l of the
+// block's 32 rows (32 independent coalesced loads), forms that column's word with shifts,
+// and the 32 ballots give the block's row words (lane i keeps row i's word).
+__global__ void __launch_bounds__(128) pack_dense_kernel(const float* __restrict__ x, int64_t rows, int64_t cols,
+                                                         int64_t ld, uint32_t* __restrict__ row_bits,
+                                                         int64_t row_words, uint32_t* __restrict__ col_bits,
+                                                         int64_t col_words, int32_t* __restrict__ colsum) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  const int lane = threadIdx.x & 31;
+  const int64_t wb = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);  // word column of the block
+  const int64_t rb = blockIdx.y;                                    // 32-row band
+  if (wb >= row_words) return;
+  const int64_t c = wb * 32 + lane, r0 = rb * 32;
+  const bool cok = c < cols;
+  float v[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = (cok && r0 + i < rows) ? __ldg(x + (r0 + i) * ld + c) : 0.0f;
+  uint32_t cw = 0, rw = 0;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const uint32_t bit = v[i] > 0.0f ? 1u : 0u;
+    cw |= bit << i;
+    const uint32_t b = __ballot_sync(0xFFFFFFFFu, bit);
+    if (lane == i) rw = b;
+  }
+  if (row_bits && r0 + lane < rows) row_bits[(r0 + lane) * row_words + wb] = rw;
+  if (cok) {
+    if (col_bits) col_bits[c * col_words + rb] = cw;
+    if (colsum) atomicAdd(colsum + c, 2 * __popc(cw) - (int)min((int64_t)32, rows - r0));
   }
 }
 
@@ -372,8 +393,21 @@ extern "C" fqt1_status fqt1_binarize_pack(const float* x, int64_t rows, int64_t 
   if (!aligned16(x) || (row_bits && !aligned16(row_bits)) || (col_bits && !aligned16(col_bits)) ||
       (colsum && !aligned16(colsum)))
     return FQT1_ERR_MISALIGNED;
-  DenseLoader L{x, rows, cols, ld};
-  return launch_pack(L, row_bits, col_bits, colsum, (cudaStream_t)stream);
+  cudaStream_t s = (cudaStream_t)stream;
+  const int64_t row_words = fqt1_packed_words(cols), col_words = fqt1_packed_words(rows);
+  const int64_t bands = (rows + 31) / 32;
+  if (bands > 65535) return FQT1_ERR_UNSUPPORTED;
+  if (colsum) FQT1_CUDA_TRY(cudaMemsetAsync(colsum, 0, sizeof(int32_t) * cols, s));
+  FQT1_CUDA_TRY(launch_k(pack_dense_kernel, dim3((unsigned)((row_words + 3) / 4), (unsigned)bands), dim3(128), 0, s,
+                         x, rows, cols, ld, row_bits, row_words, col_bits, col_words, colsum));
+  fqt1_count_launches(1);
+  if (col_bits && col_words > bands) {
+    const int64_t n = cols * (col_words - bands);
+    FQT1_CUDA_TRY(launch_k(zero_col_pad_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, col_bits, cols,
+                           col_words, bands));
+    fqt1_count_launches(1);
+  }
+  return FQT1_OK;
 }
 
 extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh,
