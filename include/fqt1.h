@@ -135,8 +135,9 @@ fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_row, int64_
 /* AGP on one grouping (Sec. 5.2): ranges of G = gy (.) gamma (gamma may be
  * NULL), keep probabilities, masks, and stochastic rounding of the kept
  * groups to `bits`-bit codes with scales S' and zero points Z'.
- * g: [M, D] fp32 row-major.  group_axis 0 = sample groups (PSQ, stream 0 of
- * the generator for rounding, 2 for masks), 1 = channels (PCQ, streams 1 / 3).
+ * g: [M, D] fp32 row-major.  group_axis 0 = sample groups (PSQ: rounding takes
+ * word m*D + j of generator stream 0, masks stream 2), 1 = channels (PCQ: word
+ * j*M + m of stream 1, masks stream 3).
  * ws: fqt1_workspace_size(0, ...) bytes. */
 fqt1_status fqt1_agp_quantize_grad(const float* g, int64_t M, int64_t D, int32_t group_axis, const float* gamma,
                                    const fqt1_agp_params* p, fqt1_qgrad* out, void* ws, size_t ws_bytes,

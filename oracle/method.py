@@ -36,8 +36,10 @@ R4  masks: SYSTEMATIC (default) draws one uniform offset and keeps group i iff
     TOPK keeps the floor(n/b) largest ranges with p^ = 1 (App. B analysis, biased).
 R5  stochastic rounding in fp32: inv = B / R, t = (x - Z) * inv, q = floor(t)
     + [u < t - floor(t)], u = (w >> 8) 2^-24 with w a Philox word, q clamped
-    to [0, B]; groups with R = 0 (or B / R not finite) get q = 0.  Codes do not
-    depend on p; p enters the scale S' = R / (B p^) and zero point Z' = Z / p^.
+    to [0, B]; groups with R = 0 (or B / R not finite) get q = 0.  The word of
+    element (m, j) is number m*D + j of stream 0 for PSQ (row-major) and number
+    j*M + m of stream 1 for PCQ (column-major).  Codes do not depend on p; p
+    enters the scale S' = R / (B p^) and zero point Z' = Z / p^.
 R6  dequantization is fp32: a = S' * float(acc), c = Z' * float(colsum),
     out = a + c; pruned rows / channels are exactly 0.
 """
@@ -253,7 +255,8 @@ def sr_codes(x, z, r, bits, seed, stream, flat_index):
     """Unbiased b-bit codes of x under zero point z and range r (fp32 ops).
 
     x, z, r broadcast together; flat_index gives the Philox word index of each
-    element (its flat position in G = [M, D]).
+    element (its row-major position m*D + j in G = [M, D] for PSQ, its
+    column-major position j*M + m for PCQ).
     """
     B = f32((1 << bits) - 1)
     x = np.asarray(x, dtype=f32)
@@ -306,7 +309,7 @@ def agp_quantize(g, group_axis, rows_per_group, bits, mode, seed):
         flat = rows[:, None].astype(np.uint64) * np.uint64(D) + np.arange(D, dtype=np.uint64)[None, :]
         codes = sr_codes(g[rows, :], z[grp][:, None], r[grp][:, None], bits, seed, stream_sr, flat)
     else:
-        flat = np.arange(M, dtype=np.uint64)[None, :] * np.uint64(D) + kept.astype(np.uint64)[:, None]
+        flat = kept.astype(np.uint64)[:, None] * np.uint64(M) + np.arange(M, dtype=np.uint64)[None, :]
         codes = sr_codes(g[:, kept].T, z[kept][:, None], r[kept][:, None], bits, seed, stream_sr, flat)
     return dict(z=z, r=r, P=P, p_hat=p_hat, kept=kept, scale=scale, zero=zero, codes=codes,
                 bits=bits, group_axis=group_axis, rows_per_group=rows_per_group)

@@ -414,12 +414,13 @@ __global__ void __launch_bounds__(256, 4) quantize_kernel(QuantArgs a) {
       any_c = true;
     }
   }
-  uint8_t ccode[4][4] = {};  // [row i][col q]
+  // this warp's 4 rows: slots and loads first
+  const int64_t rb = r0 + warp * 4;
   float vv[4][4];
   int32_t sslots[4];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {  // slots and loads of this warp's 4 rows first
-    const int64_t r = r0 + warp * 4 + i;
+  for (int i = 0; i < 4; ++i) {
+    const int64_t r = rb + i;
     sslots[i] = (a.do_psq && r < a.M) ? __ldg(a.s.slot + r / a.rpg) : -1;
     const bool need = r < a.M && (sslots[i] >= 0 || any_c);
     if (VEC) {
@@ -433,64 +434,56 @@ __global__ void __launch_bounds__(256, 4) quantize_kernel(QuantArgs a) {
 #pragma unroll
       for (int q = 0; q < 4; ++q) vv[i][q] = (need && cv[q]) ? __ldg(a.g + r * a.D + c0 + q) : 0.0f;
     }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) vv[i][q] = a.gamma ? __fmul_rn(vv[i][q], gam[q]) : vv[i][q];
   }
+  // PSQ: kept rows; element (m, j) takes word m*D + j of stream 0 (one block = 4 columns)
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const int64_t r = r0 + warp * 4 + i;
-    if (r >= a.M) break;
+    const int64_t r = rb + i;
     const int32_t sslot = sslots[i];
+    if (sslot < 0) continue;
     const int64_t gi = r / a.rpg;
-    if (sslot < 0 && !any_c) continue;
-    float v[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) v[q] = a.gamma ? __fmul_rn(vv[i][q], gam[q]) : vv[i][q];
+    const float rs = __ldg(a.s.range + gi), zs = __ldg(a.s.zmin + gi);
+    const float inv = __fdiv_rn(a.s.B, rs);
+    const bool deg = !(rs > 0.0f) || !isfinite(inv);
     const uint64_t e0 = (uint64_t)r * (uint64_t)a.D + (uint64_t)c0;
-    if (sslot >= 0) {
-      const float rs = __ldg(a.s.range + gi), zs = __ldg(a.s.zmin + gi);
-      const float inv = __fdiv_rn(a.s.B, rs);
-      const bool deg = !(rs > 0.0f) || !isfinite(inv);
-      uint32_t w[4];
-      if (VEC) {
+    uint8_t* dst = a.s.codes + ((int64_t)sslot * a.rpg + (r - gi * a.rpg)) * a.s.ld + c0;
+    if (VEC) {
+      if (cv[0]) {
         const U32x4 p = philox_block(a.s.seed, kStreamSrPsq, e0 >> 2);
-        w[0] = p.x; w[1] = p.y; w[2] = p.z; w[3] = p.w;
-      } else {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) w[q] = philox_word(a.s.seed, kStreamSrPsq, e0 + q);
+        const uint32_t packed = sr_code(vv[i][0], zs, inv, a.s.B, deg, p.x) |
+                                (sr_code(vv[i][1], zs, inv, a.s.B, deg, p.y) << 8) |
+                                (sr_code(vv[i][2], zs, inv, a.s.B, deg, p.z) << 16) |
+                                (sr_code(vv[i][3], zs, inv, a.s.B, deg, p.w) << 24);
+        *reinterpret_cast<uint32_t*>(dst) = packed;
       }
-      uint8_t* dst = a.s.codes + ((int64_t)sslot * a.rpg + (r - gi * a.rpg)) * a.s.ld + c0;
-      if (VEC) {
-        if (cv[0]) {
-          uint32_t packed = 0;
-#pragma unroll
-          for (int q = 0; q < 4; ++q) packed |= sr_code(v[q], zs, inv, a.s.B, deg, w[q]) << (8 * q);
-          *reinterpret_cast<uint32_t*>(dst) = packed;
-        }
-      } else {
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-          if (cv[q]) dst[q] = (uint8_t)sr_code(v[q], zs, inv, a.s.B, deg, w[q]);
-      }
-    }
-    if (any_c) {
-      uint32_t w[4];
-      if (VEC) {
-        const U32x4 p = philox_block(a.c.seed, kStreamSrPcq, e0 >> 2);
-        w[0] = p.x; w[1] = p.y; w[2] = p.z; w[3] = p.w;
-      } else {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) w[q] = cslot[q] >= 0 ? philox_word(a.c.seed, kStreamSrPcq, e0 + q) : 0u;
-      }
+    } else {
 #pragma unroll
       for (int q = 0; q < 4; ++q)
-        if (cslot[q] >= 0) ccode[i][q] = (uint8_t)sr_code(v[q], zc[q], invc[q], a.c.B, cdeg[q], w[q]);
+        if (cv[q]) dst[q] = (uint8_t)sr_code(vv[i][q], zs, inv, a.s.B, deg, philox_word(a.s.seed, kStreamSrPsq, e0 + q));
     }
   }
   if (!a.do_pcq) return;
-  // rows warp*4 .. warp*4+3 of each of this lane's columns form one 32-bit word
+  // PCQ: kept columns; element (m, j) takes word j*M + m of stream 1, so one Philox block
+  // gives the 4 rows of this warp; the 4 codes form the column's staging word directly
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    const uint32_t word = (uint32_t)ccode[0][q] | ((uint32_t)ccode[1][q] << 8) | ((uint32_t)ccode[2][q] << 16) |
-                          ((uint32_t)ccode[3][q] << 24);
+    uint32_t word = 0;
+    if (cslot[q] >= 0) {
+      const uint64_t e = (uint64_t)(c0 + q) * (uint64_t)a.M + (uint64_t)rb;
+      uint32_t w[4];
+      if ((a.M & 3) == 0) {
+        const U32x4 p = philox_block(a.c.seed, kStreamSrPcq, e >> 2);
+        w[0] = p.x; w[1] = p.y; w[2] = p.z; w[3] = p.w;
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) w[i] = philox_word(a.c.seed, kStreamSrPcq, e + i);
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (rb + i < a.M) word |= sr_code(vv[i][q], zc[q], invc[q], a.c.B, cdeg[q], w[i]) << (8 * i);
+    }
     tile[lane * 4 + q][warp] = word;
   }
   __syncthreads();

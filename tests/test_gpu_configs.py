@@ -130,7 +130,7 @@ def test_sweep_16384_sampled():
     dw = st.dw.cpu().numpy()
     for slot in rng.choice(len(kept_c), 3, replace=False):
         j = kept_c[slot]
-        flat = np.arange(M, dtype=np.uint64) * np.uint64(D) + np.uint64(j)
+        flat = np.uint64(j) * np.uint64(M) + np.arange(M, dtype=np.uint64)
         q = om.sr_codes(g[:, j], zc[j], rc[j], 4, w["seed_c"], om.STREAM_SR_PCQ, flat)
         a = (q.astype(np.float32) @ sxf).astype(np.int64)
         ref = om.dequant(sc_c[slot], a, ze_c[slot], cs_x)
