@@ -143,6 +143,25 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def max_over_ranks(x, device="cpu"):
+    """The largest x over all ranks of the default process group (x itself without one).
+
+    Replicas time their own K steps; the job took as long as its slowest rank."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tops(ops_per_step, steps, world, total_ms):
+    """Whole-job throughput (tera-ops/s): each of `world` replicas ran `steps` steps of
+    `ops_per_step` operations, and the slowest rank needed `total_ms`."""
+    return world * ops_per_step * steps / (total_ms * 1e-3) / 1e12
+
+
 def stage_work(st, name):
     """Algorithmic work of one stage: ('hbm', bytes) or ('tensor', dense-equivalent operations).
 
@@ -255,14 +274,10 @@ def main():
         while time.time() < t_end:
             timed_loop(20)
     clocks = clk.summary()
-    total_ms = sum(step_ms)
-    if world > 1:
-        t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(sum(step_ms), "cuda")
     ms_per_step = total_ms / args.steps
     ops = st.dense_ops()
-    value = world * ops * args.steps / (total_ms * 1e-3) / 1e12
+    value = job_tops(ops, args.steps, world, total_ms)
 
     # per-stage device time (eager; the stream is held by a sleep kernel while all launches are queued)
     per_stage = {n: [] for n, _ in stages}
@@ -321,12 +336,8 @@ def main():
             stream.synchronize()
             if i >= args.warmup:
                 e2e_ms.append(e0.elapsed_time(e1))
-    e2e_total = sum(e2e_ms)
-    if world > 1:
-        t = torch.tensor([e2e_total], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_total = float(t.item())
-    e2e = {"value": world * ops * args.steps / (e2e_total * 1e-3) / 1e12, "unit": UNIT,
+    e2e_total = max_over_ranks(sum(e2e_ms), "cuda")
+    e2e = {"value": job_tops(ops, args.steps, world, e2e_total), "unit": UNIT,
            "h2d_bytes_per_step": sum(t.numel() * t.element_size() for t in h_in),
            "d2h_bytes_per_step": sum(t.numel() * t.element_size() for t in h_out)}
 
