@@ -370,8 +370,10 @@ extern "C" fqt1_status fqt1_bwd_input_fold(const fqt1_qgrad* psq, const uint32_t
   if (p->rows_per_group != (int64_t)Ho * Wo) return FQT1_ERR_INVALID_ARG;
   if (!aligned16(sw_col) || !aligned16(dx) || !aligned16(colsum_w)) return FQT1_ERR_MISALIGNED;
   // whole samples per 128-row tile and at least one channel's taps per 256-column tile
-  // epilogue shared memory: 128 x 129 int32 tile, tap table, folded colsums of 128 / (kh kw) channels
-  const int64_t fold_bytes = 128 * 129 * 4 + 4ll * H * W * kh * kw + 4ll * (128 / (kh * kw)) * H * W + 64;
+  // epilogue shared memory: 128 x 129 int32 tile, tap table, folded colsums of 128 / (kh kw)
+  // channels, scale / zero / sample id of the 128 / (Ho Wo) samples, the block's colsums
+  const int64_t fold_bytes = 128 * 129 * 4 + 4ll * H * W * kh * kw + 4ll * (128 / (kh * kw)) * H * W +
+                             12ll * (128 / ((int64_t)Ho * Wo)) + 512;
   if (128 % (Ho * Wo) != 0 || kh * kw > 128 || fold_bytes > 100 * 1024 || (int64_t)N * C * H * W >= (1ll << 31))
     return FQT1_ERR_UNSUPPORTED;
   cudaStream_t s = (cudaStream_t)stream;

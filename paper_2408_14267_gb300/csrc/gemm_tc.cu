@@ -145,10 +145,11 @@ __device__ __forceinline__ uint32_t swz(int r, int c) {
   return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
 }
 
-// 4 sign bits -> 4 e4m3 bytes (+1 = 0x38, -1 = 0xB8).
+// 4 sign bits (bits 0..3 of nib) -> 4 e4m3 bytes (+1 = 0x38, -1 = 0xB8).  The product holds
+// four copies of nib shifted by 7, 14, 21 and 28 bits; they do not overlap, and bit k of the
+// copy shifted by 7 (k + 1) lands on bit 8k + 7, the sign bit of byte k.
 __device__ __forceinline__ uint32_t signs4(uint32_t nib) {
-  const uint32_t spread = (nib * 0x00204081u) & 0x01010101u;
-  return 0xB8B8B8B8u ^ (spread << 7);
+  return ((nib * 0x10204080u) & 0x80808080u) ^ 0xB8B8B8B8u;
 }
 // 16 sign bits -> 16 e4m3 bytes.
 __device__ __forceinline__ uint4 signs16(uint32_t h) {
@@ -156,16 +157,23 @@ __device__ __forceinline__ uint4 signs16(uint32_t h) {
 }
 // 4 codes (one per byte, each < 16) -> 4 e4m3 bytes of the same integers.
 __device__ __forceinline__ uint32_t codes4(uint32_t c) {
-  const uint32_t sel = (c & 0x7u) | ((c >> 4) & 0x70u) | ((c >> 8) & 0x700u) | ((c >> 12) & 0x7000u);
+  const uint32_t y = c & 0x07070707u;
+  // low 3 bits of byte i -> selector nibble i (bytes 0 and 2 of y | y >> 4 hold two nibbles each)
+  const uint32_t sel = __byte_perm(y | (y >> 4), 0u, 0x0020u);
   const uint32_t lo = __byte_perm(0x44403800u, 0x4E4C4A48u, sel);  // e4m3 of 0..7
   const uint32_t hi = __byte_perm(0x53525150u, 0x57565554u, sel);  // e4m3 of 8..15
-  const uint32_t m = ((c >> 3) & 0x01010101u) * 0xFFu;
+  // 0xFF in the bytes whose code is >= 8: bit 3 moved to the byte's sign bit, then replicated
+  // over the byte by prmt.b32 (a selector nibble with its top bit set sign-extends the byte;
+  // __byte_perm ignores that bit, hence the inline PTX)
+  uint32_t m;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(m) : "r"(c << 4), "r"(0u), "r"(0xBA98u));
   return (lo & ~m) | (hi & m);
 }
 // e4m3 of 16*h for digits h < 16 (exponent raised by 4; zero stays zero).
 __device__ __forceinline__ uint32_t codes4_x16(uint32_t h) {
   const uint32_t e = codes4(h);
-  const uint32_t nz = (((h | (h >> 1) | (h >> 2) | (h >> 3)) & 0x01010101u)) * 0x20u;
+  // every nonzero byte of e is in 0x38..0x57, so adding 0x7F sets its top bit without a carry
+  const uint32_t nz = ((e + 0x7F7F7F7Fu) & 0x80808080u) >> 2;  // 0x20 per nonzero byte
   return e + nz;
 }
 
@@ -230,6 +238,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
   }
+  // lane 0 of warp 0 ran alone above; __syncthreads is an aligned barrier (all lanes of a
+  // warp must reach it together), so reconverge first
+  __syncwarp();
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -287,13 +298,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------------------------------------------------------- expansion (raw -> operand)
     // threads 0..127 expand A row t, threads 128..255 expand B row t - 128 (BN = 128)
     const int t = threadIdx.x - 64;  // 0..255
+    // A rows past the kept rows are not expanded: an accumulator row depends only on its own
+    // A row, and the epilogue drops those rows
+    const bool a_live = t < kBM && m0 + t < valid_rows;
     for (int i = 0; i < nk; ++i) {
       const int so = i % OS, ito = i / OS, sr = i % RS, itr = i / RS;
       if (ito > 0 && !mbar_wait(&op_empty[so], (ito - 1) & 1, &abort_flag, a.status)) break;
       if (!mbar_wait(&raw_full[sr], itr & 1, &abort_flag, a.status)) break;
       const int kt = kt0 + i;
       if (t < kBM) {
-        if (A_CODES) {
+        if (!a_live) {
+        } else if (A_CODES) {
           const unsigned char* ra = rawA(sr);
           unsigned char* ta = opA(so);
 #pragma unroll
@@ -398,7 +413,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       float* s_scale = reinterpret_cast<float*>(csf + nc * HW);
       float* s_zero = s_scale + imgs;
       int32_t* s_n = reinterpret_cast<int32_t*>(s_zero + imgs);
+      int32_t* cs_s = s_n + imgs;                      // [nc * khw] colsums of this block's columns
       const int tt = threadIdx.x - 64;
+      const int32_t* csb = a.cs + (int64_t)c_first * khw;
+      if (tt < nc * khw) cs_s[tt] = __ldg(csb + tt);   // nc * khw <= 128: one load per thread
       for (int x = tt; x < HW * khw; x += 256) {
         const int pos = x / khw, t = x - pos * khw;
         const int h = pos / a.fW, w = pos - h * a.fW, i = t / a.fkw, j = t - i * a.fkw;
@@ -411,12 +429,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         tap_off[x] = v;
       }
       asm volatile("bar.sync 1, 256;" ::: "memory");
-      const int32_t* csb = a.cs + (int64_t)c_first * khw;
       for (int x = tt; x < nc * HW; x += 256) {
         const int cl = x / HW, pos = x - cl * HW;
         int32_t cs = 0;
         for (int t = 0; t < khw; ++t)
-          if (tap_off[pos * khw + t] >= 0) cs += __ldg(csb + cl * khw + t);
+          if (tap_off[pos * khw + t] >= 0) cs += cs_s[cl * khw + t];
         csf[x] = cs;
       }
       const int64_t slot0 = m0 / rpg, nslots = valid_rows / rpg;
@@ -551,6 +568,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }  // epilogue modes other than EPI_FOLD
   }
 
+  // The producer and MMA roles ran on lane 0 only; reconverge before the aligned barrier
+  // that orders the epilogue's TMEM reads before warp 1 frees TMEM.
+  __syncwarp();
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   if (warp == 1) {
