@@ -193,8 +193,9 @@ struct TcSmem {
   static_assert(kOpStages * kOpStage >= kExpWarps * 4096, "epilogue staging fits in the operand ring");
 };
 
+// SHORT tiles run two CTAs per SM, which caps the registers at 65536 / (2 * 320) per thread.
 template <bool A_CODES, bool BITS8, int BN, bool SHORT>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, TcArgs a) {
   using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
   constexpr int OS = S::kOpStages, RS = S::kRawStages;
