@@ -12,13 +12,15 @@
 // Pipeline per CTA (one 128 x BN output tile, 128-element K steps), two rings:
 //   raw ring (deep)    TMA writes the raw tiles: packed sign words (16 bytes per row)
 //                      or uint8 codes (128B-swizzled box)
-//   operand ring       e4m3 tiles in the 128B-swizzle K-major layout the MMA reads
+//   operand ring       e4m3 A stages in TMEM (row = lane, 4 elements per column), e4m3 B
+//                      tiles in shared memory in the 128B-swizzle K-major layout
 //   warp 0 lane 0   TMA producer of the raw ring
-//   warp 1          TMEM allocation; lane 0 issues tcgen05.mma, commits operand stages
-//   warps 2..9      expand raw -> operand tiles (one row per thread and stage), then
-//                   the epilogue: TMEM -> registers -> swizzled per-warp staging ->
-//                   coalesced row stores (warp w owns TMEM lanes 32 (w % 4) .. +31 and
-//                   half of the columns)
+//   warp 1          TMEM allocation; lane 0 issues tcgen05.mma (A from TMEM, B from shared
+//                   memory) and commits operand stages
+//   warps 2..5      expand A rows of their TMEM lane quarter and store them with tcgen05.st
+//   warps 6..9      expand B rows into the shared tile
+//   warps 2..9      then the epilogue: TMEM -> registers -> global memory (warp w owns TMEM
+//                   lanes 32 (w % 4) .. +31 and half of the columns)
 // Every wait is bounded; an expired wait sets FQT1_DEV_TIMEOUT and the CTA
 // drains and returns.
 #include <cuda.h>
@@ -34,6 +36,7 @@ constexpr int kMaxStages = 8;
 constexpr int kExpWarps = 8;       // two expansion / epilogue warps per SM sub-partition
 constexpr int kThreads = 32 * (2 + kExpWarps);
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on every wait
+constexpr int kFoldSmem = 102400;  // Folder epilogue: accumulator tile and tables (bytes)
 
 enum : int { EPI_FWD = 0, EPI_ACC32 = 1, EPI_RED = 2, EPI_DX = 3, EPI_FOLD = 4 };
 
@@ -129,15 +132,30 @@ __host__ __device__ constexpr uint32_t idesc_e4m3(int bn) {
   return (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(bn >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
 }
 
-__device__ __forceinline__ void mma_e4m3(uint32_t tmem, uint64_t ad, uint64_t bd, uint32_t idesc, uint32_t acc) {
-  asm volatile(
-      "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
-      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem),
-      "l"(ad), "l"(bd), "r"(idesc), "r"(acc));
-}
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
+}
+
+// A operand in TMEM (row = lane, 4 e4m3 per 32-bit column), B from a shared-memory descriptor.
+__device__ __forceinline__ void mma_e4m3_ta(uint32_t tmem_d, uint32_t tmem_a, uint64_t bd, uint32_t idesc,
+                                            uint32_t acc) {
+  asm volatile(
+      "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "r"(tmem_a), "l"(bd), "r"(idesc), "r"(acc));
+}
+
+// 32 consecutive TMEM columns of this thread's lane <- v (the warp writes its 32 lanes).
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,"
+      "%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
+      "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]), "r"(v[17]),
+      "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]),
+      "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+      : "memory");
 }
 
 // Byte offset of 16-byte chunk c of row r in a 128B-swizzled tile.
@@ -179,18 +197,25 @@ __device__ __forceinline__ uint32_t codes4_x16(uint32_t h) {
 
 template <bool A_CODES, bool BITS8, int BN, bool SHORT = false>
 struct TcSmem {
-  static constexpr int kOpA = kBM * kBK;                        // bytes of one e4m3 A tile
-  static constexpr int kOpB = BN * kBK;
-  static constexpr int kOpStage = kOpA * (BITS8 ? 2 : 1) + kOpB;
-  static constexpr int kRawA = A_CODES ? kBM * kBK : kBM * 16;  // codes, or packed words (4 per row)
+  static_assert(BN == 128, "one B row per expansion thread");
+  static constexpr int kOpB = BN * kBK;                          // bytes of one e4m3 B tile (shared)
+  static constexpr int kAcols = (kBK / 4) * (BITS8 ? 2 : 1);      // TMEM columns of one e4m3 A stage
+  static constexpr int kRawA = A_CODES ? kBM * kBK : kBM * 16;    // codes, or packed words (4 per row)
   static constexpr int kRawB = BN * 16;
   static constexpr int kRawStage = kRawA + kRawB;
   // SHORT: two-stage rings for short contractions (two CTAs per SM)
-  static constexpr int kOpStages = SHORT ? 2 : (BITS8 ? 2 : (A_CODES ? 3 : 4));
+  static constexpr int kOpStages = SHORT ? 2 : (BITS8 ? 3 : 4);
   static constexpr int kRawStages = SHORT ? 2 : (A_CODES ? 4 : 8);
-  static constexpr int kBytes = kOpStages * kOpStage + kRawStages * kRawStage + 1024;  // + alignment slack
-  static_assert(kOpStage % 1024 == 0 && kRawStage % 1024 == 0, "stages keep 1024-byte alignment");
-  static_assert(kOpStages * kOpStage >= kExpWarps * 4096, "epilogue staging fits in the operand ring");
+  // TMEM: the BN accumulator columns, then the A stages
+  static constexpr int kTmemUsed = BN + kOpStages * kAcols;
+  static constexpr int kTmemCols = kTmemUsed <= 256 ? 256 : 512;
+  static constexpr int kRing = kOpStages * kOpB + kRawStages * kRawStage;
+  // the epilogue reuses the rings: per-warp staging, or the Folder's tile and tables
+  static constexpr int kEpi = SHORT ? kFoldSmem : kExpWarps * 4096;
+  static constexpr int kBytes = (kRing > kEpi ? kRing : kEpi) + 1024;  // + alignment slack
+  static_assert(kOpB % 1024 == 0 && kRawStage % 1024 == 0, "stages keep 1024-byte alignment");
+  static_assert(kTmemUsed <= 512, "TMEM holds 512 columns");
+  static_assert(!SHORT || kTmemCols <= 256, "two CTAs per SM share the TMEM columns");
 };
 
 // SHORT tiles run two CTAs per SM, which caps the registers at 65536 / (2 * 320) per thread.
@@ -216,10 +241,8 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   }
 
   unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  auto opA = [&](int s) { return base + s * S::kOpStage; };
-  auto opA2 = [&](int s) { return base + s * S::kOpStage + S::kOpA; };
-  auto opB = [&](int s) { return base + s * S::kOpStage + S::kOpA * (BITS8 ? 2 : 1); };
-  unsigned char* raw_base = base + OS * S::kOpStage;
+  auto opB = [&](int s) { return base + s * S::kOpB; };
+  unsigned char* raw_base = base + OS * S::kOpB;
   auto rawA = [&](int s) { return raw_base + s * S::kRawStage; };
   auto rawB = [&](int s) { return raw_base + s * S::kRawStage + S::kRawA; };
 
@@ -232,7 +255,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
-                 "r"(BN));
+                 "r"(S::kTmemCols));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
   if (threadIdx.x == 0) {
@@ -284,91 +307,90 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         const int s = i % OS, it = i / OS;
         if (!mbar_wait(&op_full[s], it & 1, &abort_flag, a.status)) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const uint32_t aaddr = smem_u32(opA(s)), a2addr = smem_u32(opA2(s)), baddr = smem_u32(opB(s));
+        const uint32_t acol = tmem + BN + s * S::kAcols, baddr = smem_u32(opB(s));
 #pragma unroll
         for (int k = 0; k < kBK / 32; ++k) {
           const uint64_t bd = sw128_desc(baddr + 32 * k);
-          mma_e4m3(tmem, sw128_desc(aaddr + 32 * k), bd, idesc, (i > 0 || k > 0) ? 1u : 0u);
-          if (BITS8) mma_e4m3(tmem, sw128_desc(a2addr + 32 * k), bd, idesc, 1u);
+          mma_e4m3_ta(tmem, acol + 8 * k, bd, idesc, (i > 0 || k > 0) ? 1u : 0u);
+          if (BITS8) mma_e4m3_ta(tmem, acol + kBK / 4 + 8 * k, bd, idesc, 1u);
         }
         mma_commit(&op_empty[s]);
       }
       mma_commit(&acc_full);
     }
   } else {
-    // ---------------------------------------------------------------- expansion (raw -> operand)
-    // threads 0..127 expand A row t, threads 128..255 expand B row t - 128 (BN = 128)
-    const int t = threadIdx.x - 64;  // 0..255
-    // A rows past the kept rows are not expanded: an accumulator row depends only on its own
-    // A row, and the epilogue drops those rows
-    const bool a_live = t < kBM && m0 + t < valid_rows;
+    // ---------------------------------------------------------------- expansion (raw -> operands)
+    // warps 2..5: the 32 A rows of their TMEM lane quarter -> e4m3 in TMEM (one row per thread);
+    // warps 6..9: B row 32 (warp - 6) + lane -> e4m3 in the 128B-swizzled shared tile
+    const bool a_warp = warp < 6;
+    const int quarter = warp & 3;
+    const int arow = 32 * quarter + lane, brow = 32 * (warp - 6) + lane;
+    // a warp whose 32 A rows all lie past the kept rows skips its work: an accumulator row
+    // depends only on its own A row, and the epilogue drops those rows
+    const bool a_live = a_warp && m0 + 32 * quarter < valid_rows;
+    const uint32_t a_lanes = tmem + ((uint32_t)(32 * quarter) << 16);
     for (int i = 0; i < nk; ++i) {
       const int so = i % OS, ito = i / OS, sr = i % RS, itr = i / RS;
       if (ito > 0 && !mbar_wait(&op_empty[so], (ito - 1) & 1, &abort_flag, a.status)) break;
       if (!mbar_wait(&raw_full[sr], itr & 1, &abort_flag, a.status)) break;
       const int kt = kt0 + i;
-      if (t < kBM) {
-        if (!a_live) {
-        } else if (A_CODES) {
-          const unsigned char* ra = rawA(sr);
-          unsigned char* ta = opA(so);
-#pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            const uint32_t off = swz(t, c);  // TMA wrote the codes with the same 128B swizzle
-            uint4 v = *reinterpret_cast<const uint4*>(ra + off);
+      if (a_warp) {
+        if (a_live) {
+          const uint32_t acol = a_lanes + BN + so * S::kAcols;
+          uint32_t o[32];
+          if (A_CODES) {
+            const unsigned char* ra = rawA(sr);
             if (BITS8) {
-              uint4 lo, hi;
-              lo.x = codes4(v.x & 0x0F0F0F0Fu); hi.x = codes4_x16((v.x >> 4) & 0x0F0F0F0Fu);
-              lo.y = codes4(v.y & 0x0F0F0F0Fu); hi.y = codes4_x16((v.y >> 4) & 0x0F0F0F0Fu);
-              lo.z = codes4(v.z & 0x0F0F0F0Fu); hi.z = codes4_x16((v.z >> 4) & 0x0F0F0F0Fu);
-              lo.w = codes4(v.w & 0x0F0F0F0Fu); hi.w = codes4_x16((v.w >> 4) & 0x0F0F0F0Fu);
-              *reinterpret_cast<uint4*>(ta + off) = hi;
-              *reinterpret_cast<uint4*>(opA2(so) + off) = lo;
-            } else {
-              v.x = codes4(v.x); v.y = codes4(v.y); v.z = codes4(v.z); v.w = codes4(v.w);
-              *reinterpret_cast<uint4*>(ta + off) = v;
-            }
-          }
-        } else {
-          const uint4 w4 = *reinterpret_cast<const uint4*>(rawA(sr) + 16 * t);
-          const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
-          unsigned char* ta = opA(so);
-          const int64_t kbase = (int64_t)kt * kBK;
-          const bool full = kbase + kBK <= a.L;
+              uint32_t o2[32];
 #pragma unroll
-          for (int w = 0; w < 4; ++w) {
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              uint4 v = signs16(wv[w] >> (16 * h));
-              if (!full) {  // elements past the contraction length contribute 0
-                const int64_t e0 = kbase + 32 * w + 16 * h;
-                uint32_t* vv = reinterpret_cast<uint32_t*>(&v);
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-#pragma unroll
-                  for (int bb = 0; bb < 4; ++bb)
-                    if (e0 + 4 * q + bb >= a.L) vv[q] &= ~(0xFFu << (8 * bb));
-                }
+              for (int c = 0; c < 8; ++c) {  // TMA wrote the codes with the 128B swizzle
+                const uint4 v = *reinterpret_cast<const uint4*>(ra + swz(arow, c));
+                o[4 * c + 0] = codes4_x16((v.x >> 4) & 0x0F0F0F0Fu); o2[4 * c + 0] = codes4(v.x & 0x0F0F0F0Fu);
+                o[4 * c + 1] = codes4_x16((v.y >> 4) & 0x0F0F0F0Fu); o2[4 * c + 1] = codes4(v.y & 0x0F0F0F0Fu);
+                o[4 * c + 2] = codes4_x16((v.z >> 4) & 0x0F0F0F0Fu); o2[4 * c + 2] = codes4(v.z & 0x0F0F0F0Fu);
+                o[4 * c + 3] = codes4_x16((v.w >> 4) & 0x0F0F0F0Fu); o2[4 * c + 3] = codes4(v.w & 0x0F0F0F0Fu);
               }
-              *reinterpret_cast<uint4*>(ta + swz(t, 2 * w + h)) = v;
+              tmem_st32(acol, o);
+              tmem_st32(acol + kBK / 4, o2);
+            } else {
+#pragma unroll
+              for (int c = 0; c < 8; ++c) {
+                const uint4 v = *reinterpret_cast<const uint4*>(ra + swz(arow, c));
+                o[4 * c + 0] = codes4(v.x); o[4 * c + 1] = codes4(v.y);
+                o[4 * c + 2] = codes4(v.z); o[4 * c + 3] = codes4(v.w);
+              }
+              tmem_st32(acol, o);
             }
+          } else {
+            const uint4 w4 = *reinterpret_cast<const uint4*>(rawA(sr) + 16 * arow);
+            const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+            for (int j = 0; j < 32; ++j) o[j] = signs4((wv[j >> 3] >> (4 * (j & 7))) & 15u);
+            const int64_t kbase = (int64_t)kt * kBK;
+            if (kbase + kBK > a.L) {  // elements past the contraction length contribute 0
+#pragma unroll
+              for (int j = 0; j < 32; ++j) {
+#pragma unroll
+                for (int bb = 0; bb < 4; ++bb)
+                  if (kbase + 4 * j + bb >= a.L) o[j] &= ~(0xFFu << (8 * bb));
+              }
+            }
+            tmem_st32(acol, o);
           }
+          asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         }
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       } else {
+        const uint4 w4 = *reinterpret_cast<const uint4*>(rawB(sr) + 16 * brow);
+        const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+        unsigned char* tb = opB(so);
 #pragma unroll
-        for (int rr = 0; rr < BN / kBM; ++rr) {
-          const int r = t - kBM + kBM * rr;
-          const uint4 w4 = *reinterpret_cast<const uint4*>(rawB(sr) + 16 * r);
-          const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
-          unsigned char* tb = opB(so);
-#pragma unroll
-          for (int w = 0; w < 4; ++w) {
-            *reinterpret_cast<uint4*>(tb + swz(r, 2 * w)) = signs16(wv[w]);
-            *reinterpret_cast<uint4*>(tb + swz(r, 2 * w + 1)) = signs16(wv[w] >> 16);
-          }
+        for (int w = 0; w < 4; ++w) {
+          *reinterpret_cast<uint4*>(tb + swz(brow, 2 * w)) = signs16(wv[w]);
+          *reinterpret_cast<uint4*>(tb + swz(brow, 2 * w + 1)) = signs16(wv[w] >> 16);
         }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       __syncwarp();
       if (lane == 0) {
         mbar_arrive(&op_full[so]);
@@ -576,7 +598,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   __syncthreads();
   if (warp == 1) {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(BN));
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(S::kTmemCols));
   }
 }
 

@@ -130,9 +130,14 @@ __global__ void __launch_bounds__(128) pack_dense_kernel(const float* __restrict
   if (wb >= row_words) return;
   const int64_t c = wb * 32 + lane, r0 = rb * 32;
   const bool cok = c < cols;
+  // unconditional loads from clamped addresses (masked afterwards): all 32 are issued before
+  // the first ballot instead of one dependent round trip per row
+  const float* xc = x + min(c, cols - 1);
   float v[32];
 #pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = (cok && r0 + i < rows) ? __ldg(x + (r0 + i) * ld + c) : 0.0f;
+  for (int i = 0; i < 32; ++i) v[i] = __ldg(xc + min(r0 + i, rows - 1) * ld);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = (cok && r0 + i < rows) ? v[i] : 0.0f;
   uint32_t cw = 0, rw = 0;
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
@@ -178,7 +183,9 @@ struct UnfoldArgs {
   int32_t* colsum;
   int64_t row_words, col_words;
   int C, H, W, kh, kw, stride, pad, Wo, M, K, khw, HWo;
-  int tm;  // output pixels per CTA: 32, 64, 128 or 256
+  int tm;     // output pixels per CTA: 32, 64, 128 or 256
+  int guard;  // zero words before and after every plane stream
+  int same;   // stride 1, kh = kw = 2 pad + 1, Ho Wo a multiple of 32 (fast column words)
   FastDiv div_khw, div_kw, div_hwo, div_wo;
 };
 
@@ -229,15 +236,15 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
       h_hi = min(a.H - 1, oh_hi * a.stride - a.pad + a.kh - 1);
     }
     nrows = max(0, h_hi - h_lo + 1);
-    plane_words = (nrows * a.W + 31) / 32 + 2;
+    plane_words = (nrows * a.W + 31) / 32 + 2 * a.guard;
     nplanes = (n_hi - n_lo + 1) * nc;
   }
   // 1. sign-pack the region (one warp per 32 stream bits: coalesced 128-byte loads + ballot)
-  const int plane_bits = nrows * a.W, data_words = plane_words - 2;
+  const int plane_bits = nrows * a.W, data_words = plane_words - 2 * a.guard, gbits = 32 * a.guard;
   for (int pl = warp; pl < nplanes; pl += 8) {  // one (image, channel) plane per warp iteration
     const int nn = pl / nc;
     const float* src = a.x + (((int64_t)(n_lo + nn) * a.C + c_lo + (pl - nn * nc)) * a.H + h_lo) * a.W;
-    uint32_t* dst = stream + pl * plane_words + 1;
+    uint32_t* dst = stream + pl * plane_words + a.guard;
     for (int q0 = 0; q0 < data_words; q0 += 4) {  // 4 loads in flight per lane, then 4 ballots
       float v[4];
 #pragma unroll
@@ -252,9 +259,9 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
       }
     }
   }
-  for (int pl = threadIdx.x; pl < nplanes; pl += 256) {
-    stream[pl * plane_words] = 0u;
-    stream[pl * plane_words + plane_words - 1] = 0u;
+  for (int e = threadIdx.x; e < nplanes * 2 * a.guard; e += 256) {
+    const int pl = e / (2 * a.guard), g = e - pl * 2 * a.guard;
+    stream[pl * plane_words + (g < a.guard ? g : data_words + g)] = 0u;
   }
   __syncthreads();
   // 2. the 32 x 32 blocks of columns kb .. kb + 31
@@ -268,7 +275,36 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
     const int ms = m0 + 32 * sub;
     uint32_t roww = 0, colw = 0;
     if (kb < a.K && ms < a.M) {  // warp-uniform
-      if (a.stride == 1) {
+      if (a.same) {
+        // "same" convolution: pixel p of an image reads input position p + (i - pad) W + (j - pad)
+        // for tap (i, j), so the column word of k over 32 pixels of one image is one 32-bit window
+        // of the plane stream (rows outside the image fall in the zero guards), masked where
+        // the tap's input column leaves the image row
+        const int n = (int)a.div_hwo.div((uint32_t)ms), p0 = ms - n * a.HWo;
+        if (kb + lane < a.K) {
+          const int lo = max(0, a.pad - jl_), hi = min(a.W, a.W + a.pad - jl_);  // valid output columns
+          uint32_t mask;
+          if (32 % a.W == 0) {
+            const uint32_t row = (a.W == 32 ? 0xFFFFFFFFu : ((1u << hi) - (1u << lo)));
+            mask = a.W == 32 ? (hi >= 32 ? 0xFFFFFFFFu << lo : ((1u << hi) - 1u) & (0xFFFFFFFFu << lo))
+                             : row * (0xFFFFFFFFu / ((1u << a.W) - 1u));
+          } else {
+            mask = 0u;
+            int t = p0 - (int)a.div_wo.div((uint32_t)p0) * a.Wo;  // output column of bit 0
+            for (int b = 0; b < 32;) {
+              const int seg = min(a.W - t, 32 - b);
+              const int s0 = max(lo - t, 0), s1 = min(hi - t, seg);
+              if (s1 > s0) mask |= ((s1 - s0 >= 32) ? 0xFFFFFFFFu : ((1u << (s1 - s0)) - 1u)) << (b + s0);
+              b += seg;
+              t = 0;
+            }
+          }
+          const uint32_t* st = stream + ((n - n_lo) * nc + (cl_ - c_lo)) * plane_words;
+          const int pos = gbits + p0 - h_lo * a.W + (il_ - a.pad) * a.W + (jl_ - a.pad);
+          colw = stream_bits(st, pos, 32) & mask;
+        }
+        roww = warp_transpose32(colw, lane);
+      } else if (a.stride == 1) {
         // column word of k = kb + lane over pixels ms .. ms + 31: runs along output rows
         const int mend = min(a.M, ms + 32);
         int n = (int)a.div_hwo.div((uint32_t)ms), rem = ms - n * a.HWo;
@@ -282,7 +318,7 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
           const int lo = max(0, -wa), hi = min(cnt, a.W - wa);
           if (kvalid && h >= 0 && h < a.H && hi > lo) {
             const uint32_t* st = st_c + (n - n_lo) * nc * plane_words;
-            colw |= stream_bits(st, 32 + (h - h_lo) * a.W + wa + lo, hi - lo) << (m - ms + lo);
+            colw |= stream_bits(st, gbits + (h - h_lo) * a.W + wa + lo, hi - lo) << (m - ms + lo);
           }
           m += cnt;
           ow += cnt;
@@ -309,7 +345,7 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
             const int wa = w0 + j;
             const int lo = max(0, -wa), hi = min(cnt, a.W - wa);
             if (h >= 0 && h < a.H && hi > lo)
-              roww |= stream_bits(st_n + (c - c_lo) * plane_words, 32 + (h - h_lo) * a.W + wa + lo, hi - lo)
+              roww |= stream_bits(st_n + (c - c_lo) * plane_words, gbits + (h - h_lo) * a.W + wa + lo, hi - lo)
                       << (k - kb + lo);
             k += cnt;
             j += cnt;
@@ -428,16 +464,20 @@ extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t
   const int64_t Mi = (int64_t)N * Ho * Wo, Ki = (int64_t)C * kh * kw;
   if (pad <= 32 && Ki < (1ll << 31)) {
     const int tm_first = Mi >= 64 * 152 * 4 ? 128 : 64;  // smaller tiles: more resident CTAs
+    const bool same = stride == 1 && kh == kw && kh == 2 * pad + 1 && (Ho * Wo) % 32 == 0;
+    // the fast path reads a 32-bit window up to pad W + pad bits before or after the plane
+    const int guard = same ? (pad * W + pad + 63) / 32 : 1;
     for (int tm = tm_first; tm >= 32; tm /= 2) {
       const int64_t imgs = std::min<int64_t>(N, tm / (Ho * Wo) + 2);
       const int64_t chans = std::min<int64_t>(C, 256 / (kh * kw) + 2);
-      const int64_t words = imgs * chans * (((int64_t)H * W + 31) / 32 + 2);
+      const int64_t words = imgs * chans * (((int64_t)H * W + 31) / 32 + 2 * guard);
       if (words > kUnfoldMaxStreamWords) continue;
       UnfoldArgs u;
       u.x = x; u.row_bits = row_bits; u.col_bits = col_bits; u.colsum = colsum;
       u.row_words = fqt1_packed_words(Ki); u.col_words = fqt1_packed_words(Mi);
       u.C = C; u.H = H; u.W = W; u.kh = kh; u.kw = kw; u.stride = stride; u.pad = pad; u.Wo = Wo;
       u.M = (int)Mi; u.K = (int)Ki; u.khw = kh * kw; u.HWo = Ho * Wo; u.tm = tm;
+      u.guard = guard; u.same = same ? 1 : 0;
       u.div_khw = FastDiv((uint32_t)(kh * kw)); u.div_kw = FastDiv((uint32_t)kw);
       u.div_hwo = FastDiv((uint32_t)(Ho * Wo)); u.div_wo = FastDiv((uint32_t)Wo);
       const int64_t row_tiles = (Mi + tm - 1) / tm, word_tiles = (u.row_words + 7) / 8;
