@@ -150,15 +150,32 @@ __device__ uint64_t block_inclusive_scan(uint64_t v, uint64_t* warp_sums, uint64
   return v;
 }
 
-// floor(a * 2^32 / d) for 0 < d < 2^60, a < 2^60 (exact): a float64 estimate, then the
-// remainder a * 2^32 - q d in 128-bit integers moves q to the exact quotient.
+// floor(a * 2^32 / d) for 0 < d < 2^62, a < 2^60 (exact; quotients of 2^34 or more return ~0,
+// the callers clamp at 2^32).  An fp32 estimate (relative error below 2^-22) is corrected with
+// exact 128-bit remainders; float64 is avoided (its division is slow on this part).
 __device__ __forceinline__ uint64_t div_shift32(uint64_t a, uint64_t d) {
-  const unsigned __int128 num = (unsigned __int128)a << 32;
-  double est = __ddiv_rn(__ull2double_rn(a) * 4294967296.0, __ull2double_rn(d));
-  uint64_t q = est <= 0.0 ? 0ull : (uint64_t)est;
-  while ((unsigned __int128)q * d > num) --q;
-  while ((unsigned __int128)(q + 1) * d <= num) ++q;
+  typedef unsigned __int128 u128;
+  const u128 num = (u128)a << 32;
+  if ((num >> 34) >= d) return ~0ull;
+  uint64_t q = (uint64_t)__fdiv_rn(__ull2float_rn(a), __fmul_rn(__ull2float_rn(d), 2.3283064365386963e-10f));
+  // |q - quotient| < 2^13: one float step on the remainder, scaled so that d keeps 24 bits
+  const int sh = max(0, 40 - __clzll(d));
+  const float df = __ull2float_rn(d >> sh);
+  const u128 qd = (u128)q * d;
+  if (qd > num) q -= (uint64_t)__fdiv_rn(__ull2float_rn((uint64_t)((qd - num) >> sh)), df);
+  else q += (uint64_t)__fdiv_rn(__ull2float_rn((uint64_t)((num - qd) >> sh)), df);
+  while ((u128)q * d > num) --q;
+  while ((u128)(q + 1) * d <= num) ++q;
   return q;
+}
+
+// p^ = P 2^-32 as a float64, built from its bits (P <= 2^33).
+__device__ __forceinline__ double p_hat_of(uint64_t P) {
+  if (P == 0) return 0.0;
+  const int lz = __clzll(P);
+  const uint64_t frac = ((P << lz) << 1) >> 12;  // fraction bits below the leading one
+  const uint64_t ex = (uint64_t)(1023 + 63 - lz - 32);
+  return __longlong_as_double((long long)((ex << 52) | frac));
 }
 
 __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, SelectArgs a1) {
@@ -170,6 +187,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
   __shared__ uint32_t s_rmax;
   __shared__ int s_tstar;
   __shared__ uint64_t s_kth, s_stot;
+  __shared__ int rank_s[kSelThreads];
+  __shared__ uint64_t sorted_s[kSelThreads];
   const int n = a.n, tid = threadIdx.x;
   if (n <= 0) return;
   int npad = 1;
@@ -196,10 +215,15 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
   // Fixed-point ranges R~ = floor(R 2^(40 - E)), 2^(E-1) <= max R < 2^E.
   int e = 0;
   if (rmax > 0.0f) frexpf(rmax, &e);
-  const double fx = ldexp(1.0, kFixedPointBits - e);
+  // R~ = floor(R 2^(40 - E)) from the bits of R = m 2^x (exact integer shifts)
   auto rtilde = [&](int i) -> uint64_t {
     const float r = rf[i];
-    return (rmax > 0.0f && r > 0.0f) ? (uint64_t)floor((double)r * fx) : 0ull;
+    if (!(rmax > 0.0f) || !(r > 0.0f)) return 0ull;
+    const uint32_t b = __float_as_uint(r);
+    const int eb = (int)((b >> 23) & 0xFFu);
+    const uint64_t m = eb ? ((b & 0x7FFFFFu) | 0x800000u) : (b & 0x7FFFFFu);
+    const int sh = min((eb ? eb - 150 : -149) + kFixedPointBits - e, kFixedPointBits);
+    return sh >= 0 ? (m << sh) : (sh <= -32 ? 0ull : (m >> -sh));
   };
 
   if (a.bits > 1 && n <= kSelThreads) {
@@ -210,11 +234,40 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
       myk = (myrt << 24) | (uint64_t)(0xFFFFFFu - (uint32_t)tid);
       key[tid] = myk;
     }
+    // rank of each key: every warp sorts its 32 keys (bitonic, shuffles), then a key's rank is
+    // the number of larger keys in all the sorted lists (a 5-step binary search in each)
+    {
+      const int lane = tid & 31, nw = (n + 31) >> 5;
+      if ((tid >> 5) < nw) {
+        uint64_t k = tid < n ? myk : 0ull;
+#pragma unroll
+        for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+          for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            const uint64_t o = __shfl_xor_sync(0xFFFFFFFFu, k, stride);
+            const bool take_max = ((lane & stride) == 0) == ((lane & size) == 0);
+            k = take_max ? (k > o ? k : o) : (k < o ? k : o);
+          }
+        }
+        sorted_s[tid] = k;
+      }
+      __syncthreads();
+      if (tid < n) {
+        int r = 0;
+        for (int w = 0; w < nw; ++w) {
+          const uint64_t* L = sorted_s + 32 * w;
+          int idx = 0;
+#pragma unroll
+          for (int step = 16; step >= 1; step >>= 1)
+            if (L[idx + step - 1] > myk) idx += step;
+          if (idx == 31 && L[31] > myk) idx = 32;  // the five steps reach at most 31
+          r += idx;
+        }
+        rank_s[tid] = r;
+      }
+    }
     __syncthreads();
-    int rank = 0;
-    if (tid < n)
-      for (int j = 0; j < n; ++j) rank += key[j] > myk ? 1 : 0;
-    __syncthreads();
+    const int rank = tid < n ? rank_s[tid] : 0;
     if (tid < n) key[rank] = myrt;  // fixed-point ranges in sorted (descending) order
     __syncthreads();
     int tstar;
@@ -346,16 +399,13 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
   uint64_t ktot;
   const uint64_t kincl = block_inclusive_scan((uint64_t)nk, warp_sums, &ktot);
   int slot = (int)(kincl - nk);
-  const double Bd = (double)((1 << a.bits) - 1);
+  // the per-slot scale and zero point are computed by the quantize kernel
   for (int i = beg; i < end; ++i) {
     const uint64_t P = key[i];
-    const double ph = (double)P * 2.3283064365386963e-10;  // 2^-32, exact
-    o.p_hat[i] = ph;
+    o.p_hat[i] = p_hat_of(P);
     if (kept_bits & (1u << (i - beg))) {
       o.slot_of_group[i] = slot;
       o.kept_idx[slot] = i;
-      o.scale[slot] = __double2float_rn(__ddiv_rn((double)rf[i], __dmul_rn(Bd, ph)));
-      o.zero[slot] = __double2float_rn(__ddiv_rn((double)o.group_min[i], ph));
       ++slot;
     } else {
       o.slot_of_group[i] = -1;
@@ -376,7 +426,32 @@ struct QBranch {
   int64_t ld;
   float B;
   uint64_t seed;
+  const int32_t* kept_idx;    // [capacity] group of each slot
+  const int32_t* kept_count;  // [1]
+  const double* p_hat;        // [n]
+  float* scale;               // [capacity] S' = R / (B p^)
+  float* zero;                // [capacity] Z' = Z / p^
 };
+
+constexpr int kQWarps = 8;  // quantizing warps; one more warp computes the per-slot constants
+
+// Dequantization constants of the kept slots (Sec. 5.3): S' = R / (B p^) and Z' = Z / p^ in
+// float64, rounded to float, for slots cta, cta + ncta, ...  Lanes 0 / 1 compute the sample
+// branch's S' / Z', lanes 2 / 3 the channel branch's, all four in the same instructions.
+__device__ void slot_constants(const QBranch& bs, const QBranch& bc, bool do_s, bool do_c, int64_t cta,
+                               int64_t ncta, int lane) {
+  const bool chan = lane >= 2, zero_pt = (lane & 1) != 0;
+  if (lane >= 4 || !(chan ? do_c : do_s)) return;
+  const QBranch& q = chan ? bc : bs;
+  const int32_t count = __ldg(q.kept_count);
+  for (int64_t s = cta; s < count; s += ncta) {
+    const int32_t i = __ldg(q.kept_idx + s);
+    const double ph = __ldg(q.p_hat + i);
+    const double num = (double)__ldg((zero_pt ? q.zmin : q.range) + i);
+    const double den = zero_pt ? ph : __dmul_rn((double)q.B, ph);
+    (zero_pt ? q.zero : q.scale)[s] = __double2float_rn(__ddiv_rn(num, den));
+  }
+}
 
 struct QuantArgs {
   const float* g;
@@ -387,11 +462,19 @@ struct QuantArgs {
 };
 
 template <bool VEC>
-__global__ void __launch_bounds__(256, 4) quantize_kernel(QuantArgs a) {
+__global__ void __launch_bounds__(32 * (kQWarps + 1), 4) quantize_kernel(QuantArgs a) {
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
   __shared__ uint32_t tile[kQCols][kQRows / 4 + 1];  // PCQ codes, 4 rows per word
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (warp == kQWarps) {
+    // the float64 divisions run beside the quantizing warps of this CTA
+    const int64_t cta = (int64_t)blockIdx.y * gridDim.x + blockIdx.x, ncta = (int64_t)gridDim.x * gridDim.y;
+    slot_constants(a.s, a.c, a.do_psq != 0, a.do_pcq != 0, cta, ncta, lane);
+    __syncwarp();
+    if (a.do_pcq) __syncthreads();  // the PCQ tile barrier below
+    return;
+  }
   const int64_t cb = (int64_t)blockIdx.x * kQCols;
   const int64_t c0 = cb + lane * 4;
   const int64_t r0 = (int64_t)blockIdx.y * kQRows;
@@ -600,14 +683,16 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
   qa.do_psq = psq != nullptr;
   qa.do_pcq = pcq != nullptr;
   if (psq) qa.s = QBranch{psq->group_min, psq->group_range, psq->slot_of_group, psq->codes, psq->ld_codes,
-                          (float)((1 << ps->bits) - 1), ps->seed};
+                          (float)((1 << ps->bits) - 1), ps->seed, psq->kept_idx, psq->kept_count, psq->p_hat,
+                          psq->scale, psq->zero};
   else qa.s = QBranch{};
   if (pcq) qa.c = QBranch{pcq->group_min, pcq->group_range, pcq->slot_of_group, pcq->codes, pcq->ld_codes,
-                          (float)((1 << pc->bits) - 1), pc->seed};
+                          (float)((1 << pc->bits) - 1), pc->seed, pcq->kept_idx, pcq->kept_count, pcq->p_hat,
+                          pcq->scale, pcq->zero};
   else qa.c = QBranch{};
   dim3 qgrid((unsigned)((D + kQCols - 1) / kQCols), (unsigned)((M + kQRows - 1) / kQRows));
-  if (vec) launch_k(quantize_kernel<true>, dim3(qgrid), dim3(256), 0, s, qa);
-  else launch_k(quantize_kernel<false>, dim3(qgrid), dim3(256), 0, s, qa);
+  if (vec) launch_k(quantize_kernel<true>, dim3(qgrid), dim3(32 * (kQWarps + 1)), 0, s, qa);
+  else launch_k(quantize_kernel<false>, dim3(qgrid), dim3(32 * (kQWarps + 1)), 0, s, qa);
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
   return FQT1_OK;
