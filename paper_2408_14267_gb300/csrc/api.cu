@@ -3,6 +3,7 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <algorithm>
 #include <atomic>
 
 #include "gemm.cuh"
@@ -403,9 +404,21 @@ extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_
     FQT1_CUDA_TRY(launch_codes_gemm_simt(p->bits, pcq->codes, pcq->ld_codes, pcq->kept_count, 1, cap, sx_col, K, M,
                                          acc, K, s));
   } else {
-    // split the long contraction over M across CTAs (int32 reduction into acc, exact in any order);
-    // each CTA's fp32 partial sum stays below 2^24
+    // split the long contraction over M across a cluster of CTAs that reduce their int32
+    // partial tiles in shared memory and dequantize in the same kernel; each CTA's fp32 partial
+    // sum stays below 2^24 and no split is empty (every CTA of a cluster takes part)
     const int64_t k_tiles = (M + 127) / 128;
+    const int64_t out_tiles_c = ((K + 127) / 128) * ((cap + 127) / 128);
+    int64_t cs = wgrad_cluster_size(p->bits, out_tiles_c, k_tiles);
+    int64_t tps = (k_tiles + cs - 1) / cs;
+    cs = (k_tiles + tps - 1) / tps;
+    if (tps * 128 <= exact_chunk(p->bits)) {
+      FQT1_CUDA_TRY(launch_wgrad_cluster_tc(p->bits, pcq->codes, pcq->ld_codes, cap, pcq->kept_count, sx_col, K, M,
+                                            (int)cs, acc, dw, D, pcq->kept_idx, pcq->slot_of_group, pcq->scale,
+                                            pcq->zero, colsum_x, nullptr, s));
+      return FQT1_OK;
+    }
+    // contractions too long for eight exact splits: int32 atomics across CTAs, then dequantize
     const int64_t out_tiles = ((K + 127) / 128) * ((cap + 127) / 128);
     int64_t splits = (152 + out_tiles - 1) / out_tiles;  // about one wave on 152 SMs
     const int64_t min_splits = (M + exact_chunk(p->bits) - 1) / exact_chunk(p->bits);

@@ -24,6 +24,18 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
                            const uint32_t* Sg, int64_t K, int64_t D, const int32_t* kept_idx, const float* scale,
                            const float* zero, const int32_t* cs, float* dx, int C, int H, int W, int kh, int kw,
                            int stride, int pad, int Ho, int Wo, int32_t* status, cudaStream_t s);
+// grad_weight with the split-K reduction and the dequantization in the kernel: the splits of
+// an output tile form a thread-block cluster of `splits` (<= 8) CTAs that add their partial
+// tiles through distributed shared memory.  acc [capacity][K] receives the int32 sums (rows past
+// the kept count 0), dw [D][K] the dequantized rows (pruned channels 0).
+cudaError_t launch_wgrad_cluster_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t capacity, const int32_t* count,
+                                    const uint32_t* Sx, int64_t K, int64_t M, int splits, int32_t* acc, float* dw,
+                                    int64_t D, const int32_t* kept_idx, const int32_t* slot_of_group,
+                                    const float* scale, const float* zero, const int32_t* cs, int32_t* status,
+                                    cudaStream_t s);
+// Cluster size for launch_wgrad_cluster_tc: the largest (<= 8, <= k_tiles) whose out_tiles
+// clusters fit on the GPU at once.
+int wgrad_cluster_size(int bits, int64_t out_tiles, int64_t k_tiles);
 // Largest contraction one CTA may sum in fp32 and stay exact: partial sums below 2^24.
 inline int64_t exact_chunk(int bits) { return (int64_t)((1 << 24) / ((1 << bits) - 1)); }
 // 1 if FQT1_GEMM_PATH=popcount selects the CUDA-core kernels (datapath comparison only).

@@ -38,7 +38,7 @@ constexpr int kThreads = 32 * (2 + kExpWarps);
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on every wait
 constexpr int kFoldSmem = 102400;  // Folder epilogue: accumulator tile and tables (bytes)
 
-enum : int { EPI_FWD = 0, EPI_ACC32 = 1, EPI_RED = 2, EPI_DX = 3, EPI_FOLD = 4 };
+enum : int { EPI_FWD = 0, EPI_ACC32 = 1, EPI_RED = 2, EPI_DX = 3, EPI_FOLD = 4, EPI_CRED = 5 };
 
 struct TcArgs {
   int64_t M, N, L;           // rows (capacity), columns, contraction length
@@ -61,6 +61,12 @@ struct TcArgs {
   // starting at channel blockIdx.x * fcb (column offset n_step = fcb * kh * kw).
   int n_step, grid_x;
   int fC, fH, fW, fkh, fkw, fstride, fpad, fHo, fWo, fcb;
+  // EPI_FWD / EPI_ACC32: bit 0 = y, bit 1 = acc leave through TMA stores (tmY / tmAcc)
+  int tma_out;
+  // EPI_CRED: the cluster's partial tiles are summed into acc (int32, ldo) and dequantized into
+  // y = dw[D][ldo] (kept channel kept_idx[r]: scale[r] acc + zero[r] cs[n]; pruned channels 0)
+  const int32_t* slot_of_group;
+  int64_t D;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -114,6 +120,42 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
       "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y)
       : "memory");
 }
+
+// Shared -> global tile store through TMA (bulk group; the caller commits and waits).
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(smem_u32(src)), "r"(x), "r"(y)
+               : "memory");
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_size() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+// 16 bytes of CTA `rank`'s shared memory at this CTA's shared address saddr.
+__device__ __forceinline__ int4 ld_cluster_v4(uint32_t saddr, uint32_t rank) {
+  uint32_t ra;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(saddr), "r"(rank));
+  int4 v;
+  asm volatile("ld.shared::cluster.v4.s32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(ra)
+               : "memory");
+  return v;
+}
+// Byte offset of 16-byte chunk ch (0..31) of row r (0..127) of a 128 x 128 int32 tile, the
+// chunk index swizzled with r & 7 so that a warp's 32 rows hit distinct banks.
+__device__ __forceinline__ uint32_t ptile_off(int r, int ch) { return (uint32_t)(r * 512 + ((ch ^ (r & 7)) << 4)); }
 
 // Shared-memory matrix descriptor of a K-major operand tile in the 128-byte swizzle layout
 // (rows of 128 bytes, 8-row groups 1024 bytes apart).
@@ -211,7 +253,7 @@ struct TcSmem {
   static constexpr int kTmemCols = kTmemUsed <= 256 ? 256 : 512;
   static constexpr int kRing = kOpStages * kOpB + kRawStages * kRawStage;
   // the epilogue reuses the rings: per-warp staging, or the Folder's tile and tables
-  static constexpr int kEpi = SHORT ? kFoldSmem : kExpWarps * 4096;
+  static constexpr int kEpi = SHORT ? kFoldSmem : kExpWarps * 8192;
   static constexpr int kBytes = (kRing > kEpi ? kRing : kEpi) + 1024;  // + alignment slack
   static_assert(kOpB % 1024 == 0 && kRawStage % 1024 == 0, "stages keep 1024-byte alignment");
   static_assert(kTmemUsed <= 512, "TMEM holds 512 columns");
@@ -221,7 +263,8 @@ struct TcSmem {
 // SHORT tiles run two CTAs per SM, which caps the registers at 65536 / (2 * 320) per thread.
 template <bool A_CODES, bool BITS8, int BN, bool SHORT>
 __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
-    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, TcArgs a) {
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmAcc, TcArgs a) {
   using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
   constexpr int OS = S::kOpStages, RS = S::kRawStages;
   extern __shared__ unsigned char smem_raw[];
@@ -503,7 +546,63 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
             "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
           : "r"(taddr));
       asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+      if (a.epi == EPI_CRED) {
+        // this CTA's partial sums -> its shared tile, read by the whole cluster below
+        const int r = 32 * q + lane;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          int4 w;
+          w.x = __float2int_rn(__uint_as_float(v[4 * c + 0]));
+          w.y = __float2int_rn(__uint_as_float(v[4 * c + 1]));
+          w.z = __float2int_rn(__uint_as_float(v[4 * c + 2]));
+          w.w = __float2int_rn(__uint_as_float(v[4 * c + 3]));
+          *reinterpret_cast<int4*>(base + ptile_off(r, (c0 >> 2) + c)) = w;
+        }
+        continue;
+      }
       if (!have_acc) continue;
+      if (a.tma_out && row_base + 32 <= valid_rows) {
+        // stage the warp's 32 x 32 block (row = lane; 16-byte chunk c of a row at chunk
+        // c ^ (row & 7), the 128-byte swizzle of the output maps), then one TMA store per
+        // output; TMA clips columns past the tensor
+        float* sy = reinterpret_cast<float*>(base + (warp - 2) * 8192);
+        int32_t* sacc = reinterpret_cast<int32_t*>(base + (warp - 2) * 8192 + 4096);
+        if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+        __syncwarp();
+        const int64_t nb = n0 + c0;
+        const bool fullc = nb + 32 <= a.N;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const int32_t i0 = __float2int_rn(__uint_as_float(v[4 * c + 0]));
+          const int32_t i1 = __float2int_rn(__uint_as_float(v[4 * c + 1]));
+          const int32_t i2 = __float2int_rn(__uint_as_float(v[4 * c + 2]));
+          const int32_t i3 = __float2int_rn(__uint_as_float(v[4 * c + 3]));
+          const int off = lane * 32 + ((c ^ (lane & 7)) << 2);
+          if (a.tma_out & 1) {
+            float4 g4;
+            if (fullc) {
+              g4 = __ldg(reinterpret_cast<const float4*>(a.gamma + nb + 4 * c));
+            } else {
+              const int64_t nc = nb + 4 * c;
+              g4.x = nc + 0 < a.N ? __ldg(a.gamma + nc + 0) : 0.f;
+              g4.y = nc + 1 < a.N ? __ldg(a.gamma + nc + 1) : 0.f;
+              g4.z = nc + 2 < a.N ? __ldg(a.gamma + nc + 2) : 0.f;
+              g4.w = nc + 3 < a.N ? __ldg(a.gamma + nc + 3) : 0.f;
+            }
+            *reinterpret_cast<float4*>(sy + off) = make_float4(__fmul_rn(g4.x, (float)i0), __fmul_rn(g4.y, (float)i1),
+                                                               __fmul_rn(g4.z, (float)i2), __fmul_rn(g4.w, (float)i3));
+          }
+          if (a.tma_out & 2) *reinterpret_cast<int4*>(sacc + off) = make_int4(i0, i1, i2, i3);
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+        if (lane == 0) {
+          if (a.tma_out & 1) tma_store_2d(&tmY, sy, (int)nb, (int)row_base);
+          if (a.tma_out & 2) tma_store_2d(&tmAcc, sacc, (int)nb, (int)row_base);
+          asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+        }
+        continue;
+      }
       if (a.epi != EPI_RED) {
         // direct stores: this thread's row, 32 consecutive columns
         const int64_t r = row_base + lane;
@@ -588,12 +687,62 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         }
       }
     }
+    if (a.tma_out && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
     }  // epilogue modes other than EPI_FOLD
   }
 
-  // The producer and MMA roles ran on lane 0 only; reconverge before the aligned barrier
-  // that orders the epilogue's TMEM reads before warp 1 frees TMEM.
+  // The producer and MMA roles ran on lane 0 only; reconverge before the aligned barriers
+  // (the cluster's, and the one that orders the epilogue's TMEM reads before warp 1 frees TMEM).
   __syncwarp();
+  if (a.epi == EPI_CRED) {
+    // every CTA of the cluster reaches both barriers, also after an expired wait
+    cluster_sync_all();
+    const uint32_t rank = cluster_rank(), nr = cluster_size();
+    const int rpr = (kBM + (int)nr - 1) / (int)nr;  // tile rows summed by each CTA
+    const int r_lo = (int)rank * rpr, r_hi = min(kBM, r_lo + rpr);
+    const uint32_t pbase = smem_u32(base);
+    const bool ok = !abort_flag;
+    const bool vec = (a.ldo % 4) == 0;
+    for (int e = threadIdx.x; e < (r_hi - r_lo) * 32; e += kThreads) {
+      const int r = r_lo + (e >> 5), ch = e & 31;
+      const int64_t grow = m0 + r, n = n0 + 4 * ch;
+      if (grow >= a.M || n >= a.N) continue;
+      int4 sum = make_int4(0, 0, 0, 0);
+      const bool kept = ok && grow < valid_rows;
+      if (kept) {
+        for (uint32_t src = 0; src < nr; ++src) {
+          const int4 t = ld_cluster_v4(pbase + ptile_off(r, ch), src);
+          sum.x += t.x; sum.y += t.y; sum.z += t.z; sum.w += t.w;
+        }
+      }
+      const int32_t sv[4] = {sum.x, sum.y, sum.z, sum.w};
+      int32_t* arow = a.acc + grow * a.ldo + n;
+      if (vec && n + 4 <= a.N) *reinterpret_cast<int4*>(arow) = sum;
+      else for (int t = 0; t < 4 && n + t < a.N; ++t) arow[t] = sv[t];
+      if (kept) {
+        const int64_t j = __ldg(a.kept_idx + grow);
+        const float sc = __ldg(a.scale + grow), ze = __ldg(a.zero + grow);
+        float* wrow = a.y + j * a.ldo + n;
+        float o[4];
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+          o[t] = n + t < a.N ? __fadd_rn(__fmul_rn(sc, (float)sv[t]), __fmul_rn(ze, (float)__ldg(a.cs + n + t))) : 0.f;
+        if (vec && n + 4 <= a.N) *reinterpret_cast<float4*>(wrow) = make_float4(o[0], o[1], o[2], o[3]);
+        else for (int t = 0; t < 4 && n + t < a.N; ++t) wrow[t] = o[t];
+      }
+    }
+    if (blockIdx.y == 0) {
+      // pruned channels: zero rows of dw over this tile's columns, shared by the cluster
+      for (int64_t e = (int64_t)rank * kThreads + threadIdx.x; e < a.D * 32; e += (int64_t)nr * kThreads) {
+        const int64_t j = e >> 5, n = n0 + 4 * (e & 31);
+        if (n >= a.N || __ldg(a.slot_of_group + j) >= 0) continue;
+        float* wrow = a.y + j * a.ldo + n;
+        if (vec && n + 4 <= a.N) *reinterpret_cast<float4*>(wrow) = make_float4(0.f, 0.f, 0.f, 0.f);
+        else for (int t = 0; t < 4 && n + t < a.N; ++t) wrow[t] = 0.f;
+      }
+    }
+    cluster_sync_all();  // no CTA leaves while another still reads its tile
+  }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   if (warp == 1) {
@@ -631,7 +780,9 @@ static bool make_map(CUtensorMap* m, const void* ptr, CUtensorMapDataType type, 
 
 template <bool A_CODES, bool BITS8, int BN, bool SHORT = false>
 static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const TcArgs& a, int splits,
-                             cudaStream_t s) {
+                             cudaStream_t s, const CUtensorMap* my = nullptr, const CUtensorMap* macc = nullptr,
+                             bool cluster = false) {
+  static const CUtensorMap unused{};  // never read: the matching tma_out bit is clear
   using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
   static bool attr = false;
   if (!attr) {
@@ -642,7 +793,12 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
   }
   dim3 grid((unsigned)(a.grid_x > 0 ? a.grid_x : (a.N + BN - 1) / BN), (unsigned)((a.M + kBM - 1) / kBM),
             (unsigned)splits);
-  launch_k(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT>, dim3(grid), dim3(kThreads), S::kBytes, s, ma, mb, a);
+  if (cluster)
+    launch_k_cluster(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT>, dim3(grid), dim3(kThreads), S::kBytes, s,
+                     (unsigned)splits, ma, mb, my ? *my : unused, macc ? *macc : unused, a);
+  else
+    launch_k(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT>, dim3(grid), dim3(kThreads), S::kBytes, s, ma, mb,
+             my ? *my : unused, macc ? *macc : unused, a);
   fqt1_count_launches(1);
   return cudaGetLastError();
 }
@@ -659,7 +815,19 @@ cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64
   a.M = M; a.N = D; a.L = K; a.count = nullptr; a.rows_per_count = 1;
   a.k_tiles = (int)((K + kBK - 1) / kBK); a.tiles_per_split = a.k_tiles;
   a.epi = EPI_FWD; a.gamma = gamma; a.y = y; a.acc = acc; a.ldo = D; a.status = status;
-  return launch_tc<false, false, 128>(ma, mb, a, 1, s);
+  // outputs leave through TMA stores when their rows are 16-byte multiples
+  CUtensorMap my{}, macc{};
+  if (D % 4 == 0 && make_map(&my, y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, D, M, D * 4, 32, 32,
+                             CU_TENSOR_MAP_SWIZZLE_128B)) {
+    a.tma_out = 1;
+    if (acc) {
+      if (make_map(&macc, acc, CU_TENSOR_MAP_DATA_TYPE_INT32, D, M, D * 4, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B))
+        a.tma_out |= 2;
+      else
+        a.tma_out = 0;
+    }
+  }
+  return launch_tc<false, false, 128>(ma, mb, a, 1, s, &my, &macc);
 }
 
 // Codes x signs: out[r, n] = sum_j Q[r, j] S[n, j], Q [rows][ld] uint8 (valid rows *count * rpc),
@@ -703,6 +871,65 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
   a.fcb = cb;
   if (bits == 8) return launch_tc<true, true, 128, true>(ma, mb, a, 1, s);
   return launch_tc<true, false, 128, true>(ma, mb, a, 1, s);
+}
+
+// Clusters of `cs` CTAs of this kernel that fit on the GPU at once (0 if unknown).
+template <bool BITS8>
+static int max_active_clusters(int cs) {
+  using S = TcSmem<true, BITS8, 128>;
+  static int cache[9] = {-1, -1, -1, -1, -1, -1, -1, -1, -1};
+  if (cs < 1 || cs > 8) return 0;
+  if (cache[cs] >= 0) return cache[cs];
+  auto kern = tc_gemm_kernel<true, BITS8, 128, false>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes) != cudaSuccess) return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(1, 1, (unsigned)cs);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = S::kBytes;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = (unsigned)cs;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, (const void*)kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    n = 0;
+  }
+  cache[cs] = n;
+  return n;
+}
+
+int wgrad_cluster_size(int bits, int64_t out_tiles, int64_t k_tiles) {
+  // the largest cluster (<= 8 splits) whose out_tiles clusters all run in one wave
+  for (int cs = 8; cs >= 1; --cs) {
+    if (cs > k_tiles) continue;
+    const int fit = bits == 8 ? max_active_clusters<true>(cs) : max_active_clusters<false>(cs);
+    if (fit >= out_tiles) return cs;
+  }
+  return 1;
+}
+
+cudaError_t launch_wgrad_cluster_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t capacity, const int32_t* count,
+                                    const uint32_t* Sx, int64_t K, int64_t M, int splits, int32_t* acc, float* dw,
+                                    int64_t D, const int32_t* kept_idx, const int32_t* slot_of_group,
+                                    const float* scale, const float* zero, const int32_t* cs, int32_t* status,
+                                    cudaStream_t s) {
+  const int64_t lds = fqt1_packed_words(M);
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, M, capacity, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&mb, Sx, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, 4, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+    return cudaErrorInvalidValue;
+  TcArgs a{};
+  a.M = capacity; a.N = K; a.L = M; a.count = count; a.rows_per_count = 1;
+  a.k_tiles = (int)((M + kBK - 1) / kBK);
+  a.tiles_per_split = (a.k_tiles + splits - 1) / splits;
+  a.epi = EPI_CRED; a.acc = acc; a.y = dw; a.ldo = K; a.kept_idx = kept_idx; a.scale = scale; a.zero = zero;
+  a.cs = cs; a.status = status; a.slot_of_group = slot_of_group; a.D = D;
+  if (bits == 8) return launch_tc<true, true, 128>(ma, mb, a, splits, s, nullptr, nullptr, true);
+  return launch_tc<true, false, 128>(ma, mb, a, splits, s, nullptr, nullptr, true);
 }
 
 cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
