@@ -195,9 +195,9 @@ fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, const int32_t
  * Sec. 5.3's per-sample scales, App. C Folder): the same dx as fqt1_bwd_input_gemm
  * followed by fqt1_col2im, without the int32 accumulators in memory.  A tile of 128
  * accumulator rows holds whole samples, so this call requires Ho*Wo to divide 128
- * (maps of 8x8, 4x4, 2x2 ... pixels), kh*kw <= 128 and
- * 66048 + 4 H W kh kw + 4 floor(128 / (kh kw)) H W + 12 (128 / (Ho Wo)) + 512 <= 102400
- * (its shared-memory tables); other shapes return
+ * (maps of 8x8, 4x4, 2x2 ... pixels), kh*kw <= 128 and, with cb = floor(128 / (kh kw)),
+ * 4 (H W kh kw + cb H W + cb kh kw) + 12 (128 / (Ho Wo)) <= 36864 (its shared-memory
+ * tables); other shapes return
  * FQT1_ERR_UNSUPPORTED (use the two-call path).  p->rows_per_group must be Ho*Wo.
  * sw_col: [K = C*kh*kw][words(D)]; colsum_w: [K]; dx: [N, C, H, W] (pruned samples 0). */
 fqt1_status fqt1_bwd_input_fold(const fqt1_qgrad* psq, const uint32_t* sw_col, const int32_t* colsum_w, int32_t N,

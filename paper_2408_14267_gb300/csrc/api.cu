@@ -370,21 +370,18 @@ extern "C" fqt1_status fqt1_bwd_input_fold(const fqt1_qgrad* psq, const uint32_t
   const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
   if (p->rows_per_group != (int64_t)Ho * Wo) return FQT1_ERR_INVALID_ARG;
   if (!aligned16(sw_col) || !aligned16(dx) || !aligned16(colsum_w)) return FQT1_ERR_MISALIGNED;
-  // whole samples per 128-row tile and at least one channel's taps per 256-column tile
-  // epilogue shared memory: 128 x 129 int32 tile, tap table, folded colsums of 128 / (kh kw)
-  // channels, scale / zero / sample id of the 128 / (Ho Wo) samples, the block's colsums
-  const int64_t fold_bytes = 128 * 129 * 4 + 4ll * H * W * kh * kw + 4ll * (128 / (kh * kw)) * H * W +
-                             12ll * (128 / ((int64_t)Ho * Wo)) + 512;
-  if (128 % (Ho * Wo) != 0 || kh * kw > 128 || fold_bytes > 100 * 1024 || (int64_t)N * C * H * W >= (1ll << 31))
+  // whole samples per 128-row tile, at least one channel's taps per tile, and the Folder's
+  // tables (tap offsets, folded colsums of 128 / (kh kw) channels, per-sample constants) in
+  // their 36 KB of shared memory
+  if (128 % (Ho * Wo) != 0 || kh * kw > 128 || fold_table_bytes(H, W, kh, kw, Ho, Wo) > 36864 ||
+      (int64_t)N * C * H * W >= (1ll << 31))
     return FQT1_ERR_UNSUPPORTED;
   cudaStream_t s = (cudaStream_t)stream;
   const int64_t rpg = (int64_t)Ho * Wo;
   const int64_t cap_rows = fqt1_kept_capacity(N, p->bits, p->mode) * rpg;
-  launch_zero_pruned_rows(psq->slot_of_group, N, (int64_t)C * H * W, 1, dx, s);
-  FQT1_CUDA_TRY(cudaGetLastError());
   FQT1_CUDA_TRY(launch_fold_tc(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, sw_col,
-                               (int64_t)C * kh * kw, D, psq->kept_idx, psq->scale, psq->zero, colsum_w, dx, C, H, W,
-                               kh, kw, stride, pad, Ho, Wo, nullptr, s));
+                               (int64_t)C * kh * kw, D, psq->kept_idx, psq->scale, psq->zero, colsum_w,
+                               psq->slot_of_group, dx, N, C, H, W, kh, kw, stride, pad, Ho, Wo, nullptr, s));
   return FQT1_OK;
 }
 

@@ -22,8 +22,15 @@ cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int6
 enum : int { GEMM_EPI_ACC32 = 1, GEMM_EPI_RED = 2, GEMM_EPI_DX = 3 };
 cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
                            const uint32_t* Sg, int64_t K, int64_t D, const int32_t* kept_idx, const float* scale,
-                           const float* zero, const int32_t* cs, float* dx, int C, int H, int W, int kh, int kw,
-                           int stride, int pad, int Ho, int Wo, int32_t* status, cudaStream_t s);
+                           const float* zero, const int32_t* cs, const int32_t* slot_of_group, float* dx, int N, int C,
+                           int H, int W, int kh, int kw, int stride, int pad, int Ho, int Wo, int32_t* status,
+                           cudaStream_t s);
+// Bytes of the fused Folder's tables (tap offsets, folded colsums, per-sample constants); the
+// fused path needs this to be at most 36864.
+inline int64_t fold_table_bytes(int64_t H, int64_t W, int64_t kh, int64_t kw, int64_t Ho, int64_t Wo) {
+  const int64_t khw = kh * kw, cb = 128 / khw;
+  return 4 * (H * W * khw + cb * H * W + cb * khw) + 12 * (128 / (Ho * Wo));
+}
 // grad_weight with the split-K reduction and the dequantization in the kernel: the splits of
 // an output tile form a thread-block cluster of `splits` (<= 8) CTAs that add their partial
 // tiles through distributed shared memory.  acc [capacity][K] receives the int32 sums (rows past

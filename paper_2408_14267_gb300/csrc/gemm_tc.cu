@@ -36,7 +36,9 @@ constexpr int kMaxStages = 8;
 constexpr int kExpWarps = 8;       // two expansion / epilogue warps per SM sub-partition
 constexpr int kThreads = 32 * (2 + kExpWarps);
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on every wait
-constexpr int kFoldSmem = 102400;  // Folder epilogue: accumulator tile and tables (bytes)
+constexpr int kFoldTile = 128 * 129 * 4;  // Folder epilogue: int32 accumulator tile (aliases the rings)
+constexpr int kFoldTab = 40960;           // Folder tables, a region of their own (bytes)
+constexpr int kFoldZero = 4096;           // its last 4 KB: zeros, the source of bulk stores
 
 enum : int { EPI_FWD = 0, EPI_ACC32 = 1, EPI_RED = 2, EPI_DX = 3, EPI_FOLD = 4, EPI_CRED = 5 };
 
@@ -63,6 +65,9 @@ struct TcArgs {
   int fC, fH, fW, fkh, fkw, fstride, fpad, fHo, fWo, fcb;
   // EPI_FWD / EPI_ACC32: bit 0 = y, bit 1 = acc leave through TMA stores (tmY / tmAcc)
   int tma_out;
+  int fN;  // EPI_FOLD: samples (pruned ones are zeroed by the kernel)
+  // EPI_FOLD divisors (host-built): kh kw, W, kw, H W, stride, fcb H W
+  FastDiv fd_khw, fd_w, fd_kw, fd_hw, fd_s, fd_cbhw;
   // EPI_CRED: the cluster's partial tiles are summed into acc (int32, ldo) and dequantized into
   // y = dw[D][ldo] (kept channel kept_idx[r]: scale[r] acc + zero[r] cs[n]; pruned channels 0)
   const int32_t* slot_of_group;
@@ -126,6 +131,13 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void*
   asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
                    reinterpret_cast<uint64_t>(map)),
                "r"(smem_u32(src)), "r"(x), "r"(y)
+               : "memory");
+}
+
+// Untiled bulk copy shared -> global (both addresses 16-byte aligned, bytes a multiple of 16).
+__device__ __forceinline__ void bulk_store(void* gdst, const void* ssrc, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(reinterpret_cast<uint64_t>(gdst)),
+               "r"(smem_u32(ssrc)), "r"(bytes)
                : "memory");
 }
 
@@ -252,9 +264,12 @@ struct TcSmem {
   static constexpr int kTmemUsed = BN + kOpStages * kAcols;
   static constexpr int kTmemCols = kTmemUsed <= 256 ? 256 : 512;
   static constexpr int kRing = kOpStages * kOpB + kRawStages * kRawStage;
-  // the epilogue reuses the rings: per-warp staging, or the Folder's tile and tables
-  static constexpr int kEpi = SHORT ? kFoldSmem : kExpWarps * 8192;
-  static constexpr int kBytes = (kRing > kEpi ? kRing : kEpi) + 1024;  // + alignment slack
+  // the epilogue reuses the rings (per-warp staging, or the Folder's accumulator tile); the
+  // Folder's tables have a region of their own after the rings (built while the rings are busy)
+  static constexpr int kEpi = SHORT ? kFoldTile : kExpWarps * 8192;
+  static constexpr int kMain = kRing > kEpi ? kRing : kEpi;
+  static constexpr int kTab = SHORT ? kFoldTab : 0;
+  static constexpr int kBytes = kMain + kTab + 1024;  // + alignment slack
   static_assert(kOpB % 1024 == 0 && kRawStage % 1024 == 0, "stages keep 1024-byte alignment");
   static_assert(kTmemUsed <= 512, "TMEM holds 512 columns");
   static_assert(!SHORT || kTmemCols <= 256, "two CTAs per SM share the TMEM columns");
@@ -304,6 +319,29 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   if (threadIdx.x == 0) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+  }
+  // Folder tap table (geometry only, so it is built before the dependency wait): for input
+  // position pos = h W + w and tap t = i kw + j, the accumulator tile offset
+  // (output pixel * 129 + t) of the product that lands there, or -1
+  int32_t* const fold_tab = reinterpret_cast<int32_t*>(base + S::kMain);
+  if (SHORT && a.epi == EPI_FOLD && threadIdx.x >= 64) {
+    int4* zb = reinterpret_cast<int4*>(base + S::kMain + kFoldTab - kFoldZero);
+    for (int x = threadIdx.x - 64; x < kFoldZero / 16; x += 256) zb[x] = make_int4(0, 0, 0, 0);
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the bulk stores read it later
+    const int khw = a.fkh * a.fkw, HW = a.fH * a.fW;
+    for (int x = threadIdx.x - 64; x < HW * khw; x += 256) {
+      const int pos = (int)a.fd_khw.div((uint32_t)x), t = x - pos * khw;
+      const int h = (int)a.fd_w.div((uint32_t)pos), w = pos - h * a.fW;
+      const int i = (int)a.fd_kw.div((uint32_t)t), j = t - i * a.fkw;
+      const int hn = h + a.fpad - i, wn = w + a.fpad - j;
+      int v = -1;
+      if (hn >= 0 && wn >= 0) {
+        const int oh = (int)a.fd_s.div((uint32_t)hn), ow = (int)a.fd_s.div((uint32_t)wn);
+        if (oh * a.fstride == hn && ow * a.fstride == wn && oh < a.fHo && ow < a.fWo)
+          v = (oh * a.fWo + ow) * (BN + 1) + t;
+      }
+      fold_tab[x] = v;
+    }
   }
   // lane 0 of warp 0 ran alone above; __syncthreads is an aligned barrier (all lanes of a
   // warp must reach it together), so reconverge first
@@ -444,6 +482,36 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     // ---------------------------------------------------------------- epilogue
     // TMEM -> registers (thread = row) -> per-warp swizzled staging (32 x 32 words) ->
     // one coalesced 128-byte row per store instruction (lane = column).
+    // Folder tables that read inputs (after the dependency wait, before the accumulator is
+    // ready): this block's colsums, the folded colsum of each (channel, position), and each
+    // sample's kept id, scale and zero point
+    const int f_khw = a.fkh * a.fkw, f_HW = a.fH * a.fW, f_imgs = a.rpg > 0 ? kBM / (int)a.rpg : 0;
+    const int f_c0 = blockIdx.x * a.fcb, f_nc = min(a.fcb, a.fC - f_c0);
+    int32_t* const f_tap = fold_tab;                   // [HW][khw]
+    int32_t* const f_csf = f_tap + f_HW * f_khw;       // [nc][HW]
+    int32_t* const f_cs = f_csf + f_nc * f_HW;         // [nc * khw]
+    float* const f_scale = reinterpret_cast<float*>(f_cs + f_nc * f_khw);
+    float* const f_zero = f_scale + f_imgs;
+    int32_t* const f_n = reinterpret_cast<int32_t*>(f_zero + f_imgs);
+    if (SHORT && a.epi == EPI_FOLD) {
+      const int tt = threadIdx.x - 64;
+      if (tt < f_nc * f_khw) f_cs[tt] = __ldg(a.cs + (int64_t)f_c0 * f_khw + tt);  // nc * khw <= 128
+      const int64_t slot0 = (int64_t)blockIdx.y * f_imgs, nslots = __ldg(a.count);  // rpg divides 128
+      if (tt < f_imgs) {
+        const int64_t slot = slot0 + tt;
+        f_n[tt] = slot < nslots ? __ldg(a.kept_idx + slot) : -1;
+        f_scale[tt] = slot < nslots ? __ldg(a.scale + slot) : 0.f;
+        f_zero[tt] = slot < nslots ? __ldg(a.zero + slot) : 0.f;
+      }
+      asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
+      for (int x = tt; x < f_nc * f_HW; x += 256) {
+        const int cl = (int)a.fd_hw.div((uint32_t)x), pos = x - cl * f_HW;
+        int32_t cs = 0;
+        for (int t = 0; t < f_khw; ++t)
+          if (f_tap[pos * f_khw + t] >= 0) cs += f_cs[cl * f_khw + t];
+        f_csf[x] = cs;
+      }
+    }
     const bool have_acc = mbar_wait(&acc_full, 0, &abort_flag, a.status);
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     if (a.epi == EPI_FOLD) {
@@ -469,64 +537,72 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
 #pragma unroll
         for (int j = 0; j < 32; ++j) trow[j] = __float2int_rn(__uint_as_float(v[j]));
       }
-      // per-CTA tables: for input position pos = h*W + w and tap t = i*kw + j, the tile offset
-      // (output pixel row * TS + t) of the accumulator that lands on it, or -1; the folded
-      // colsum of each (channel, position); each sample's kept id, scale and zero point
-      const int rpg = (int)a.rpg, imgs = kBM / rpg, khw = a.fkh * a.fkw, HW = a.fH * a.fW;
-      const int c_first = blockIdx.x * a.fcb, nc = min(a.fcb, a.fC - c_first);
-      int32_t* tap_off = T + kBM * TS;                 // [HW][khw]
-      int32_t* csf = tap_off + HW * khw;               // [nc][HW]
-      float* s_scale = reinterpret_cast<float*>(csf + nc * HW);
-      float* s_zero = s_scale + imgs;
-      int32_t* s_n = reinterpret_cast<int32_t*>(s_zero + imgs);
-      int32_t* cs_s = s_n + imgs;                      // [nc * khw] colsums of this block's columns
+      const int rpg = (int)a.rpg, imgs = f_imgs, khw = f_khw, HW = f_HW;
+      const int c_first = f_c0, nc = f_nc;
+      const int32_t* tap_off = f_tap;
+      const int32_t* csf = f_csf;
+      const float* s_scale = f_scale;
+      const float* s_zero = f_zero;
+      const int32_t* s_n = f_n;
       const int tt = threadIdx.x - 64;
-      const int32_t* csb = a.cs + (int64_t)c_first * khw;
-      if (tt < nc * khw) cs_s[tt] = __ldg(csb + tt);   // nc * khw <= 128: one load per thread
-      for (int x = tt; x < HW * khw; x += 256) {
-        const int pos = x / khw, t = x - pos * khw;
-        const int h = pos / a.fW, w = pos - h * a.fW, i = t / a.fkw, j = t - i * a.fkw;
-        const int hn = h + a.fpad - i, wn = w + a.fpad - j;
-        int v = -1;
-        if (hn >= 0 && wn >= 0 && hn % a.fstride == 0 && wn % a.fstride == 0) {
-          const int oh = hn / a.fstride, ow = wn / a.fstride;
-          if (oh < a.fHo && ow < a.fWo) v = (oh * a.fWo + ow) * TS + t;
-        }
-        tap_off[x] = v;
-      }
-      asm volatile("bar.sync 1, 256;" ::: "memory");
-      for (int x = tt; x < nc * HW; x += 256) {
-        const int cl = x / HW, pos = x - cl * HW;
-        int32_t cs = 0;
-        for (int t = 0; t < khw; ++t)
-          if (tap_off[pos * khw + t] >= 0) cs += cs_s[cl * khw + t];
-        csf[x] = cs;
-      }
-      const int64_t slot0 = m0 / rpg, nslots = valid_rows / rpg;
-      if (tt < imgs) {
-        const int64_t slot = slot0 + tt;
-        s_n[tt] = slot < nslots ? __ldg(a.kept_idx + slot) : -1;
-        s_scale[tt] = slot < nslots ? __ldg(a.scale + slot) : 0.f;
-        s_zero[tt] = slot < nslots ? __ldg(a.zero + slot) : 0.f;
-      }
       asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
-      // Folder: dx[n, c, h, w] = S'_n sum(acc taps) + Z'_n sum(colsum taps)
-      const int per_img = nc * HW;
-      const FastDiv div_img((uint32_t)per_img), div_hw((uint32_t)HW);
+      // Folder: dx[n, c, h, w] = S'_n sum(acc taps) + Z'_n sum(colsum taps); entries of fcb
+      // channels per sample (a last, narrower channel block skips the missing ones)
+      const int per_img = a.fcb * HW;
       for (int e = tt; have_acc && e < imgs * per_img; e += 256) {
-        const int img = (int)div_img.div((uint32_t)e), rem = e - img * per_img;
+        const int img = (int)a.fd_cbhw.div((uint32_t)e), rem = e - img * per_img;
         const int n = s_n[img];
         if (n < 0) break;
-        const int cl = (int)div_hw.div((uint32_t)rem), pos = rem - cl * HW;
+        const int cl = (int)a.fd_hw.div((uint32_t)rem), pos = rem - cl * HW;
+        if (cl >= nc) continue;
         const int32_t* tim = T + img * rpg * TS + cl * khw;
         const int32_t* to = tap_off + pos * khw;
         int32_t acc = 0;
-        for (int t = 0; t < khw; ++t) {
-          const int o = to[t];
-          if (o >= 0) acc += tim[o];
+        if (khw == 9) {  // 3 x 3 kernels: all table and tile loads in flight together
+          int o[9];
+#pragma unroll
+          for (int t = 0; t < 9; ++t) o[t] = to[t];
+#pragma unroll
+          for (int t = 0; t < 9; ++t) acc += o[t] >= 0 ? tim[o[t]] : 0;
+        } else {
+          for (int t = 0; t < khw; ++t) {
+            const int o = to[t];
+            if (o >= 0) acc += tim[o];
+          }
         }
         a.y[((int64_t)n * a.fC + c_first + cl) * HW + pos] =
             __fadd_rn(__fmul_rn(s_scale[img], (float)acc), __fmul_rn(s_zero[img], (float)csf[rem]));
+      }
+      // pruned samples: this CTA zeroes its channel block (nc HW contiguous floats) of samples
+      // blockIdx.y, + gridDim.y, ...: bulk stores from a zero buffer, one thread per 4 KB piece
+      const int nsamp = a.fN > (int)blockIdx.y ? (a.fN - (int)blockIdx.y + (int)gridDim.y - 1) / (int)gridDim.y : 0;
+      const int64_t blk_bytes = (int64_t)nc * HW * 4;
+      if (HW % 4 == 0) {
+        const int pieces = (int)((blk_bytes + kFoldZero - 1) / kFoldZero);
+        const unsigned char* zb = base + S::kMain + kFoldTab - kFoldZero;
+        bool issued = false;
+        for (int e = tt; e < nsamp * pieces; e += 256) {
+          const int k = e / pieces, pc = e - k * pieces;
+          const int64_t n = (int64_t)blockIdx.y + (int64_t)k * gridDim.y;
+          if (__ldg(a.slot_of_group + n) >= 0) continue;
+          unsigned char* dst = reinterpret_cast<unsigned char*>(a.y + ((int64_t)n * a.fC + c_first) * HW) +
+                               (int64_t)pc * kFoldZero;
+          const int64_t left = blk_bytes - (int64_t)pc * kFoldZero;
+          bulk_store(dst, zb, (uint32_t)(left < kFoldZero ? left : kFoldZero));
+          issued = true;
+        }
+        if (issued) {
+          asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+          asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        }
+      } else {
+        for (int e = tt; e < nsamp * per_img; e += 256) {
+          const int k = (int)a.fd_cbhw.div((uint32_t)e), x = e - k * per_img;
+          if (x >= nc * HW) continue;
+          const int64_t n = (int64_t)blockIdx.y + (int64_t)k * gridDim.y;
+          if (__ldg(a.slot_of_group + n) >= 0) continue;
+          a.y[((int64_t)n * a.fC + c_first) * HW + x] = 0.f;
+        }
       }
     } else {
     const int q = warp & 3;                         // TMEM lane quarter of this warp
@@ -853,8 +929,9 @@ cudaError_t launch_codes_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max
 // grad_input of a convolution with the Folder in the epilogue (EPI_FOLD, 256-column tiles).
 cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
                            const uint32_t* Sg, int64_t K, int64_t D, const int32_t* kept_idx, const float* scale,
-                           const float* zero, const int32_t* cs, float* dx, int C, int H, int W, int kh, int kw,
-                           int stride, int pad, int Ho, int Wo, int32_t* status, cudaStream_t s) {
+                           const float* zero, const int32_t* cs, const int32_t* slot_of_group, float* dx, int N, int C,
+                           int H, int W, int kh, int kw, int stride, int pad, int Ho, int Wo, int32_t* status,
+                           cudaStream_t s) {
   const int64_t lds = fqt1_packed_words(D);
   CUtensorMap ma, mb;
   if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, D, max_rows, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
@@ -868,7 +945,9 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
   a.rpg = (int64_t)Ho * Wo; a.status = status;
   a.n_step = cb * khw; a.grid_x = (C + cb - 1) / cb;
   a.fC = C; a.fH = H; a.fW = W; a.fkh = kh; a.fkw = kw; a.fstride = stride; a.fpad = pad; a.fHo = Ho; a.fWo = Wo;
-  a.fcb = cb;
+  a.fcb = cb; a.fN = N; a.slot_of_group = slot_of_group;
+  a.fd_khw = FastDiv((uint32_t)khw); a.fd_w = FastDiv((uint32_t)W); a.fd_kw = FastDiv((uint32_t)kw);
+  a.fd_hw = FastDiv((uint32_t)(H * W)); a.fd_s = FastDiv((uint32_t)stride); a.fd_cbhw = FastDiv((uint32_t)(cb * H * W));
   if (bits == 8) return launch_tc<true, true, 128, true>(ma, mb, a, 1, s);
   return launch_tc<true, false, 128, true>(ma, mb, a, 1, s);
 }

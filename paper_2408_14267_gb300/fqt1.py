@@ -173,8 +173,9 @@ def fold_supported(Ho, Wo, kh, kw, H, W):
     """The fused grad_input + Folder needs whole samples per 128-row tile (Ho*Wo divides 128)."""
     if 128 % (Ho * Wo) != 0 or kh * kw > 128:
         return False
-    return (128 * 129 * 4 + 4 * H * W * kh * kw + 4 * (128 // (kh * kw)) * H * W + 12 * (128 // (Ho * Wo)) + 512
-            <= 100 * 1024)
+    khw = kh * kw
+    cb = 128 // khw
+    return 4 * (H * W * khw + cb * H * W + cb * khw) + 12 * (128 // (Ho * Wo)) <= 36864
 
 
 def bwd_weight_gemm(pcq, sx_col, colsum_x, M, D, K, params, acc, dw, ws=None, stream=None):
