@@ -31,13 +31,14 @@ FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS = 6800.0, 1900.0
 SMS, POPC_PER_CLK_SM = 152, 16
 
 # DRAM bytes (read + write) per launch of each stage's kernels, from one ncu capture of
-# `bench.py --profile 2 --warmup 1` (profiles/kernels_resnet18_cifar_conv_full.md).  They are
+# `bench.py --profile 2 --warmup 1` (profiles/kernels_resnet18_cifar_conv_full.md; the SCQ
+# stage is the sum of its range, selection and quantize kernels).  They are
 # valid only for the kernel sources they were taken on: TRAFFIC_SOURCES is the sha256 prefix of
 # paper_2408_14267_gb300/csrc at that capture; any other source tree reports traffic = null.
-TRAFFIC_SOURCES = "a731c2adfbbf5134"
-TRAFFIC_BYTES = {"pack_w": 2.379264e6, "im2col": 8.428288e6, "fwd_gemm": 2.492160e6,
-                 "scq_quantize": 8.414720e6 + 0.059904e6 + 8.434944e6, "bwd_input_gemm": 0.650752e6 + 256,
-                 "col2im": 0.007168e6 + 18.904064e6, "bwd_weight_gemm": 3.525888e6 + 0.606464e6}
+TRAFFIC_SOURCES = "2dc6bca3edf7472b"
+TRAFFIC_BYTES = {"pack_w": 2.384640e+06, "im2col": 8.435456e+06, "fwd_gemm": 2.508800e+06,
+                 "scq_quantize": 1.694387e+07, "bwd_input_fold": 6.832640e+05,
+                 "bwd_weight_gemm": 2.977792e+06}
 
 
 def sources_sha():
