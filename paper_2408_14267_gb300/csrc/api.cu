@@ -404,12 +404,12 @@ extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_
     // split the long contraction over M across a cluster of CTAs that reduce their int32
     // partial tiles in shared memory and dequantize in the same kernel; each CTA's fp32 partial
     // sum stays below 2^24 and no split is empty (every CTA of a cluster takes part)
-    const int64_t k_tiles = (M + 127) / 128;
+    const int64_t k_tiles = (M + kCodesStageK - 1) / kCodesStageK;  // pipeline stages
     const int64_t out_tiles_c = ((K + 127) / 128) * ((cap + 127) / 128);
     int64_t cs = wgrad_cluster_size(p->bits, out_tiles_c, k_tiles);
     int64_t tps = (k_tiles + cs - 1) / cs;
     cs = (k_tiles + tps - 1) / tps;
-    if (tps * 128 <= exact_chunk(p->bits)) {
+    if (tps * kCodesStageK <= exact_chunk(p->bits)) {
       FQT1_CUDA_TRY(launch_wgrad_cluster_tc(p->bits, pcq->codes, pcq->ld_codes, cap, pcq->kept_count, sx_col, K, M,
                                             (int)cs, acc, dw, D, pcq->kept_idx, pcq->slot_of_group, pcq->scale,
                                             pcq->zero, colsum_x, nullptr, s));
@@ -421,7 +421,7 @@ extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_
     const int64_t min_splits = (M + exact_chunk(p->bits) - 1) / exact_chunk(p->bits);
     if (splits < min_splits) splits = min_splits;
     if (splits > k_tiles) splits = k_tiles;
-    if ((k_tiles + splits - 1) / splits * 128 > exact_chunk(p->bits)) return FQT1_ERR_UNSUPPORTED;
+    if ((k_tiles + splits - 1) / splits * kCodesStageK > exact_chunk(p->bits)) return FQT1_ERR_UNSUPPORTED;
     FQT1_CUDA_TRY(cudaMemsetAsync(acc, 0, sizeof(int32_t) * cap * K, s));
     FQT1_CUDA_TRY(launch_codes_tc_simple(p->bits, pcq->codes, pcq->ld_codes, cap, pcq->kept_count, 1, sx_col, K, M,
                                          GEMM_EPI_RED, (int)splits, acc, nullptr, K, nullptr, nullptr, nullptr,

@@ -43,6 +43,9 @@ cudaError_t launch_wgrad_cluster_tc(int bits, const uint8_t* Q, int64_t ldq, int
 // Cluster size for launch_wgrad_cluster_tc: the largest (<= 8, <= k_tiles) whose out_tiles
 // clusters fit on the GPU at once.
 int wgrad_cluster_size(int bits, int64_t out_tiles, int64_t k_tiles);
+// Contraction elements per pipeline stage of the code x sign products (the grad_input and
+// grad_weight GEMMs): split counts and the exactness bound are counted in these stages.
+constexpr int kCodesStageK = 256;
 // Largest contraction one CTA may sum in fp32 and stay exact: partial sums below 2^24.
 inline int64_t exact_chunk(int bits) { return (int64_t)((1 << 24) / ((1 << bits) - 1)); }
 // 1 if FQT1_GEMM_PATH=popcount selects the CUDA-core kernels (datapath comparison only).

@@ -31,7 +31,7 @@
 namespace fqt1 {
 
 constexpr int kBM = 128;           // output rows per CTA (MMA M)
-constexpr int kBK = 128;           // contraction elements per stage (one 128-byte swizzle row of e4m3)
+constexpr int kBK = 128;           // contraction elements per sub-tile (one 128-byte swizzle row of e4m3)
 constexpr int kMaxStages = 8;
 constexpr int kExpWarps = 8;       // two expansion / epilogue warps per SM sub-partition
 constexpr int kThreads = 32 * (2 + kExpWarps);
@@ -212,6 +212,14 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32
       : "memory");
 }
 
+// Sub-tiles of stage kt that hold contraction elements below L (1..KSUB for a stage that
+// starts below L).
+template <int KSUB>
+__device__ __forceinline__ int valid_subtiles(int64_t L, int kt) {
+  const int64_t left = L - (int64_t)kt * KSUB * kBK;
+  return left >= (int64_t)KSUB * kBK ? KSUB : (int)((left + kBK - 1) / kBK);
+}
+
 // Byte offset of 16-byte chunk c of row r in a 128B-swizzled tile.
 __device__ __forceinline__ uint32_t swz(int r, int c) {
   return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
@@ -252,27 +260,33 @@ __device__ __forceinline__ uint32_t codes4_x16(uint32_t h) {
 template <bool A_CODES, bool BITS8, int BN, bool SHORT = false>
 struct TcSmem {
   static_assert(BN == 128, "one B row per expansion thread");
-  static constexpr int kOpB = BN * kBK;                          // bytes of one e4m3 B tile (shared)
-  static constexpr int kAcols = (kBK / 4) * (BITS8 ? 2 : 1);      // TMEM columns of one e4m3 A stage
-  static constexpr int kRawA = A_CODES ? kBM * kBK : kBM * 16;    // codes, or packed words (4 per row)
-  static constexpr int kRawB = BN * 16;
+  // a stage carries KSUB sub-tiles of kBK contraction elements (fewer ring hand-offs per element)
+  static constexpr int KSUB = A_CODES ? 2 : 4;
+  static constexpr int kSub = BN * kBK;                          // bytes of one e4m3 B sub-tile
+  static constexpr int kOpB = kSub * KSUB;                        // bytes of one B stage (shared)
+  static constexpr int kAcols = (kBK / 4) * KSUB * (BITS8 ? 2 : 1);  // TMEM columns of one A stage
+  static constexpr int kRawRow = 16 * KSUB;                       // packed-sign bytes per row per stage
+  static constexpr int kRawA = A_CODES ? kBM * kBK * KSUB : kBM * kRawRow;
+  static constexpr int kRawB = BN * kRawRow;
   static constexpr int kRawStage = kRawA + kRawB;
-  // SHORT: two-stage rings for short contractions (two CTAs per SM)
-  static constexpr int kOpStages = SHORT ? 2 : (BITS8 ? 3 : 4);
-  static constexpr int kRawStages = SHORT ? 2 : (A_CODES ? 4 : 8);
+  // SHORT: single-buffered rings for short contractions (two CTAs per SM)
+  static constexpr int kOpStages = SHORT ? 1 : 2;
+  static constexpr int kRawStages = SHORT ? 1 : (A_CODES ? 3 : 4);
   // TMEM: the BN accumulator columns, then the A stages
   static constexpr int kTmemUsed = BN + kOpStages * kAcols;
   static constexpr int kTmemCols = kTmemUsed <= 256 ? 256 : 512;
   static constexpr int kRing = kOpStages * kOpB + kRawStages * kRawStage;
   // the epilogue reuses the rings (per-warp staging, or the Folder's accumulator tile); the
   // Folder's tables have a region of their own after the rings (built while the rings are busy)
-  static constexpr int kEpi = SHORT ? kFoldTile : kExpWarps * 8192;
+  static constexpr int kEpi = SHORT ? kFoldTile : kExpWarps * 16384;
   static constexpr int kMain = kRing > kEpi ? kRing : kEpi;
   static constexpr int kTab = SHORT ? kFoldTab : 0;
   static constexpr int kBytes = kMain + kTab + 1024;  // + alignment slack
-  static_assert(kOpB % 1024 == 0 && kRawStage % 1024 == 0, "stages keep 1024-byte alignment");
+  static_assert(kSub % 1024 == 0 && kRawStage % 1024 == 0, "stages keep 1024-byte alignment");
   static_assert(kTmemUsed <= 512, "TMEM holds 512 columns");
   static_assert(!SHORT || kTmemCols <= 256, "two CTAs per SM share the TMEM columns");
+  static_assert(kBytes <= 227 * 1024, "shared memory per CTA");
+  static_assert(!A_CODES || kBK * KSUB == kCodesStageK, "the host sizes code stages with kCodesStageK");
 };
 
 // SHORT tiles run two CTAs per SM, which caps the registers at 65536 / (2 * 320) per thread.
@@ -281,13 +295,14 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmAcc, TcArgs a) {
   using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
-  constexpr int OS = S::kOpStages, RS = S::kRawStages;
+  constexpr int OS = S::kOpStages, RS = S::kRawStages, KSUB = S::KSUB;
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t raw_full[kMaxStages], raw_empty[kMaxStages], op_full[kMaxStages],
       op_empty[kMaxStages];
   __shared__ __align__(8) uint64_t acc_full;
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
+  __shared__ __align__(16) float gamma_s[BN];  // EPI_FWD: Gamma of this tile's columns (read as float4)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t m0 = (int64_t)blockIdx.y * kBM, n0 = (int64_t)blockIdx.x * (a.n_step > 0 ? a.n_step : BN);
@@ -367,9 +382,14 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         if (it > 0 && !mbar_wait(&raw_empty[s], (it - 1) & 1, &abort_flag, a.status)) break;
         const int kt = kt0 + i;
         mbar_expect_tx(&raw_full[s], kTx);
-        if (A_CODES) tma_load_2d(rawA(s), &tmA, &raw_full[s], kt * kBK, (int)m0);
-        else tma_load_2d(rawA(s), &tmA, &raw_full[s], kt * (kBK / 32), (int)m0);
-        tma_load_2d(rawB(s), &tmB, &raw_full[s], kt * (kBK / 32), (int)n0);
+        if (A_CODES) {
+#pragma unroll
+          for (int h = 0; h < KSUB; ++h)  // one 128-byte-swizzled box per sub-tile
+            tma_load_2d(rawA(s) + h * (kBM * kBK), &tmA, &raw_full[s], (kt * KSUB + h) * kBK, (int)m0);
+        } else {
+          tma_load_2d(rawA(s), &tmA, &raw_full[s], kt * KSUB * (kBK / 32), (int)m0);
+        }
+        tma_load_2d(rawB(s), &tmB, &raw_full[s], kt * KSUB * (kBK / 32), (int)n0);
         ++issued;
       }
       // drain: every issued copy must land before the CTA may exit
@@ -389,11 +409,16 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         if (!mbar_wait(&op_full[s], it & 1, &abort_flag, a.status)) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const uint32_t acol = tmem + BN + s * S::kAcols, baddr = smem_u32(opB(s));
+        const int nsub = valid_subtiles<KSUB>(a.L, kt0 + i);
 #pragma unroll
-        for (int k = 0; k < kBK / 32; ++k) {
-          const uint64_t bd = sw128_desc(baddr + 32 * k);
-          mma_e4m3_ta(tmem, acol + 8 * k, bd, idesc, (i > 0 || k > 0) ? 1u : 0u);
-          if (BITS8) mma_e4m3_ta(tmem, acol + kBK / 4 + 8 * k, bd, idesc, 1u);
+        for (int h = 0; h < KSUB; ++h) {
+          if (h >= nsub) break;  // sub-tiles past the contraction length hold no products
+#pragma unroll
+          for (int k = 0; k < kBK / 32; ++k) {
+            const uint64_t bd = sw128_desc(baddr + h * S::kSub + 32 * k);
+            mma_e4m3_ta(tmem, acol + (kBK / 4) * h + 8 * k, bd, idesc, (i > 0 || h > 0 || k > 0) ? 1u : 0u);
+            if (BITS8) mma_e4m3_ta(tmem, acol + (kBK / 4) * (KSUB + h) + 8 * k, bd, idesc, 1u);
+          }
         }
         mma_commit(&op_empty[s]);
       }
@@ -418,57 +443,66 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       if (a_warp) {
         if (a_live) {
           const uint32_t acol = a_lanes + BN + so * S::kAcols;
-          uint32_t o[32];
-          if (A_CODES) {
-            const unsigned char* ra = rawA(sr);
-            if (BITS8) {
-              uint32_t o2[32];
+          const int nsub = valid_subtiles<KSUB>(a.L, kt);
+#pragma unroll 1
+          for (int h = 0; h < nsub; ++h) {  // one sub-tile's registers live at a time
+            uint32_t o[32];
+            if (A_CODES) {
+              const unsigned char* ra = rawA(sr) + h * (kBM * kBK);
+              if (BITS8) {
+                uint32_t o2[32];
 #pragma unroll
-              for (int c = 0; c < 8; ++c) {  // TMA wrote the codes with the 128B swizzle
-                const uint4 v = *reinterpret_cast<const uint4*>(ra + swz(arow, c));
-                o[4 * c + 0] = codes4_x16((v.x >> 4) & 0x0F0F0F0Fu); o2[4 * c + 0] = codes4(v.x & 0x0F0F0F0Fu);
-                o[4 * c + 1] = codes4_x16((v.y >> 4) & 0x0F0F0F0Fu); o2[4 * c + 1] = codes4(v.y & 0x0F0F0F0Fu);
-                o[4 * c + 2] = codes4_x16((v.z >> 4) & 0x0F0F0F0Fu); o2[4 * c + 2] = codes4(v.z & 0x0F0F0F0Fu);
-                o[4 * c + 3] = codes4_x16((v.w >> 4) & 0x0F0F0F0Fu); o2[4 * c + 3] = codes4(v.w & 0x0F0F0F0Fu);
+                for (int c = 0; c < 8; ++c) {  // TMA wrote the codes with the 128B swizzle
+                  const uint4 v = *reinterpret_cast<const uint4*>(ra + swz(arow, c));
+                  o[4 * c + 0] = codes4_x16((v.x >> 4) & 0x0F0F0F0Fu); o2[4 * c + 0] = codes4(v.x & 0x0F0F0F0Fu);
+                  o[4 * c + 1] = codes4_x16((v.y >> 4) & 0x0F0F0F0Fu); o2[4 * c + 1] = codes4(v.y & 0x0F0F0F0Fu);
+                  o[4 * c + 2] = codes4_x16((v.z >> 4) & 0x0F0F0F0Fu); o2[4 * c + 2] = codes4(v.z & 0x0F0F0F0Fu);
+                  o[4 * c + 3] = codes4_x16((v.w >> 4) & 0x0F0F0F0Fu); o2[4 * c + 3] = codes4(v.w & 0x0F0F0F0Fu);
+                }
+                tmem_st32(acol + (kBK / 4) * h, o);
+                tmem_st32(acol + (kBK / 4) * (KSUB + h), o2);
+              } else {
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                  const uint4 v = *reinterpret_cast<const uint4*>(ra + swz(arow, c));
+                  o[4 * c + 0] = codes4(v.x); o[4 * c + 1] = codes4(v.y);
+                  o[4 * c + 2] = codes4(v.z); o[4 * c + 3] = codes4(v.w);
+                }
+                tmem_st32(acol + (kBK / 4) * h, o);
               }
-              tmem_st32(acol, o);
-              tmem_st32(acol + kBK / 4, o2);
             } else {
+              const uint4 w4 = *reinterpret_cast<const uint4*>(rawA(sr) + arow * S::kRawRow + 16 * h);
+              const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
-              for (int c = 0; c < 8; ++c) {
-                const uint4 v = *reinterpret_cast<const uint4*>(ra + swz(arow, c));
-                o[4 * c + 0] = codes4(v.x); o[4 * c + 1] = codes4(v.y);
-                o[4 * c + 2] = codes4(v.z); o[4 * c + 3] = codes4(v.w);
+              for (int j = 0; j < 32; ++j) o[j] = signs4((wv[j >> 3] >> (4 * (j & 7))) & 15u);
+              const int64_t kbase = ((int64_t)kt * KSUB + h) * kBK;
+              if (kbase + kBK > a.L) {  // elements past the contraction length contribute 0
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+#pragma unroll
+                  for (int bb = 0; bb < 4; ++bb)
+                    if (kbase + 4 * j + bb >= a.L) o[j] &= ~(0xFFu << (8 * bb));
+                }
               }
-              tmem_st32(acol, o);
+              tmem_st32(acol + (kBK / 4) * h, o);
             }
-          } else {
-            const uint4 w4 = *reinterpret_cast<const uint4*>(rawA(sr) + 16 * arow);
-            const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
-#pragma unroll
-            for (int j = 0; j < 32; ++j) o[j] = signs4((wv[j >> 3] >> (4 * (j & 7))) & 15u);
-            const int64_t kbase = (int64_t)kt * kBK;
-            if (kbase + kBK > a.L) {  // elements past the contraction length contribute 0
-#pragma unroll
-              for (int j = 0; j < 32; ++j) {
-#pragma unroll
-                for (int bb = 0; bb < 4; ++bb)
-                  if (kbase + 4 * j + bb >= a.L) o[j] &= ~(0xFFu << (8 * bb));
-              }
-            }
-            tmem_st32(acol, o);
           }
           asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         }
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       } else {
-        const uint4 w4 = *reinterpret_cast<const uint4*>(rawB(sr) + 16 * brow);
-        const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
-        unsigned char* tb = opB(so);
+        const int nsub = valid_subtiles<KSUB>(a.L, kt);
 #pragma unroll
-        for (int w = 0; w < 4; ++w) {
-          *reinterpret_cast<uint4*>(tb + swz(brow, 2 * w)) = signs16(wv[w]);
-          *reinterpret_cast<uint4*>(tb + swz(brow, 2 * w + 1)) = signs16(wv[w] >> 16);
+        for (int h = 0; h < KSUB; ++h) {
+          if (h >= nsub) break;
+          const uint4 w4 = *reinterpret_cast<const uint4*>(rawB(sr) + brow * S::kRawRow + 16 * h);
+          const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+          unsigned char* tb = opB(so) + h * S::kSub;
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            *reinterpret_cast<uint4*>(tb + swz(brow, 2 * w)) = signs16(wv[w]);
+            *reinterpret_cast<uint4*>(tb + swz(brow, 2 * w + 1)) = signs16(wv[w] >> 16);
+          }
         }
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       }
@@ -511,6 +545,11 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
           if (f_tap[pos * f_khw + t] >= 0) cs += f_cs[cl * f_khw + t];
         f_csf[x] = cs;
       }
+    }
+    if (a.tma_out & 1) {  // Gamma of this tile's columns, before the accumulator is ready
+      const int tt = threadIdx.x - 64;
+      if (tt < BN) gamma_s[tt] = n0 + tt < a.N ? __ldg(a.gamma + n0 + tt) : 0.f;
+      asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
     }
     const bool have_acc = mbar_wait(&acc_full, 0, &abort_flag, a.status);
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -641,12 +680,11 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         // stage the warp's 32 x 32 block (row = lane; 16-byte chunk c of a row at chunk
         // c ^ (row & 7), the 128-byte swizzle of the output maps), then one TMA store per
         // output; TMA clips columns past the tensor
-        float* sy = reinterpret_cast<float*>(base + (warp - 2) * 8192);
-        int32_t* sacc = reinterpret_cast<int32_t*>(base + (warp - 2) * 8192 + 4096);
-        if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-        __syncwarp();
+        // 8 KB per warp and 32-column chunk (y then acc): no wait between the warp's chunks
+        unsigned char* stg = base + (warp - 2) * 16384 + ((c0 - cbeg) >> 5) * 8192;
+        float* sy = reinterpret_cast<float*>(stg);
+        int32_t* sacc = reinterpret_cast<int32_t*>(stg + 4096);
         const int64_t nb = n0 + c0;
-        const bool fullc = nb + 32 <= a.N;
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
           const int32_t i0 = __float2int_rn(__uint_as_float(v[4 * c + 0]));
@@ -655,16 +693,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
           const int32_t i3 = __float2int_rn(__uint_as_float(v[4 * c + 3]));
           const int off = lane * 32 + ((c ^ (lane & 7)) << 2);
           if (a.tma_out & 1) {
-            float4 g4;
-            if (fullc) {
-              g4 = __ldg(reinterpret_cast<const float4*>(a.gamma + nb + 4 * c));
-            } else {
-              const int64_t nc = nb + 4 * c;
-              g4.x = nc + 0 < a.N ? __ldg(a.gamma + nc + 0) : 0.f;
-              g4.y = nc + 1 < a.N ? __ldg(a.gamma + nc + 1) : 0.f;
-              g4.z = nc + 2 < a.N ? __ldg(a.gamma + nc + 2) : 0.f;
-              g4.w = nc + 3 < a.N ? __ldg(a.gamma + nc + 3) : 0.f;
-            }
+            const float4 g4 = *reinterpret_cast<const float4*>(gamma_s + c0 + 4 * c);
             *reinterpret_cast<float4*>(sy + off) = make_float4(__fmul_rn(g4.x, (float)i0), __fmul_rn(g4.y, (float)i1),
                                                                __fmul_rn(g4.z, (float)i2), __fmul_rn(g4.w, (float)i3));
           }
@@ -763,7 +792,8 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         }
       }
     }
-    if (a.tma_out && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+    // the stores must have read the staging buffers before the CTA exits
+    if (a.tma_out && lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
     }  // epilogue modes other than EPI_FOLD
   }
 
@@ -882,14 +912,16 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
 // Forward: A = sign(X) rows [M][words(K)], B = sign(W) rows [D][words(K)].
 cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64_t D, int64_t K, const float* gamma,
                           int32_t* acc, float* y, int32_t* status, cudaStream_t s) {
+  using S = TcSmem<false, false, 128>;
   const int64_t ldw = fqt1_packed_words(K);
   CUtensorMap ma, mb;
-  if (!make_map(&ma, A, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, M, ldw * 4, 4, kBM, CU_TENSOR_MAP_SWIZZLE_NONE) ||
-      !make_map(&mb, B, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, D, ldw * 4, 4, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+  if (!make_map(&ma, A, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, M, ldw * 4, 4 * S::KSUB, kBM,
+                CU_TENSOR_MAP_SWIZZLE_NONE) ||
+      !make_map(&mb, B, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, D, ldw * 4, 4 * S::KSUB, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
     return cudaErrorInvalidValue;
   TcArgs a{};
   a.M = M; a.N = D; a.L = K; a.count = nullptr; a.rows_per_count = 1;
-  a.k_tiles = (int)((K + kBK - 1) / kBK); a.tiles_per_split = a.k_tiles;
+  a.k_tiles = (int)((K + kBK * S::KSUB - 1) / (kBK * S::KSUB)); a.tiles_per_split = a.k_tiles;
   a.epi = EPI_FWD; a.gamma = gamma; a.y = y; a.acc = acc; a.ldo = D; a.status = status;
   // outputs leave through TMA stores when their rows are 16-byte multiples
   CUtensorMap my{}, macc{};
@@ -914,11 +946,12 @@ cudaError_t launch_codes_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max
   const int64_t lds = fqt1_packed_words(L);
   CUtensorMap ma, mb;
   if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, L, max_rows, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, n_s, lds * 4, 4, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+      !make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, n_s, lds * 4, kCodesStageK / 32, 128,
+                CU_TENSOR_MAP_SWIZZLE_NONE))
     return cudaErrorInvalidValue;
   TcArgs a = epi_args;
   a.M = max_rows; a.N = n_s; a.L = L; a.count = count; a.rows_per_count = rows_per_count;
-  a.k_tiles = (int)((L + kBK - 1) / kBK);
+  a.k_tiles = (int)((L + kCodesStageK - 1) / kCodesStageK);
   a.tiles_per_split = (a.k_tiles + splits - 1) / splits;
   a.epi = epi;
   const int z = (a.k_tiles + a.tiles_per_split - 1) / a.tiles_per_split;
@@ -935,12 +968,13 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
   const int64_t lds = fqt1_packed_words(D);
   CUtensorMap ma, mb;
   if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, D, max_rows, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, 4, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+      !make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, kCodesStageK / 32, 128,
+                CU_TENSOR_MAP_SWIZZLE_NONE))
     return cudaErrorInvalidValue;
   TcArgs a{};
   const int khw = kh * kw, cb = 128 / khw;
   a.M = max_rows; a.N = K; a.L = D; a.count = count; a.rows_per_count = (int64_t)Ho * Wo;
-  a.k_tiles = (int)((D + kBK - 1) / kBK); a.tiles_per_split = a.k_tiles;
+  a.k_tiles = (int)((D + kCodesStageK - 1) / kCodesStageK); a.tiles_per_split = a.k_tiles;
   a.epi = EPI_FOLD; a.y = dx; a.kept_idx = kept_idx; a.scale = scale; a.zero = zero; a.cs = cs;
   a.rpg = (int64_t)Ho * Wo; a.status = status;
   a.n_step = cb * khw; a.grid_x = (C + cb - 1) / cb;
@@ -999,11 +1033,12 @@ cudaError_t launch_wgrad_cluster_tc(int bits, const uint8_t* Q, int64_t ldq, int
   const int64_t lds = fqt1_packed_words(M);
   CUtensorMap ma, mb;
   if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, M, capacity, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&mb, Sx, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, 4, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+      !make_map(&mb, Sx, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, kCodesStageK / 32, 128,
+                CU_TENSOR_MAP_SWIZZLE_NONE))
     return cudaErrorInvalidValue;
   TcArgs a{};
   a.M = capacity; a.N = K; a.L = M; a.count = count; a.rows_per_count = 1;
-  a.k_tiles = (int)((M + kBK - 1) / kBK);
+  a.k_tiles = (int)((M + kCodesStageK - 1) / kCodesStageK);
   a.tiles_per_split = (a.k_tiles + splits - 1) / splits;
   a.epi = EPI_CRED; a.acc = acc; a.y = dw; a.ldo = K; a.kept_idx = kept_idx; a.scale = scale; a.zero = zero;
   a.cs = cs; a.status = status; a.slot_of_group = slot_of_group; a.D = D;
