@@ -428,9 +428,18 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     // ---------------------------------------------------------------- expansion (raw -> operands)
     // warps 2..5: the 32 A rows of their TMEM lane quarter -> e4m3 in TMEM (one row per thread);
     // warps 6..9: B row 32 (warp - 6) + lane -> e4m3 in the 128B-swizzled shared tile
-    const bool a_warp = warp < 6;
+    // (the split below changes this for tiles with few live rows)
+    // A tile with at most two live lane quarters (e.g. 64 kept channels) and two sub-tiles per
+    // stage splits its A work by sub-tile over the two warps of each live quarter (4 / 8 and
+    // 5 / 9); warps 2, 3, 6 and 7 then take the B rows.
+    const int64_t tile_rows = valid_rows - m0;  // may exceed kBM or be negative
+    const int live_q = tile_rows >= kBM ? 4 : (tile_rows <= 0 ? 0 : (int)((tile_rows + 31) / 32));
+    const bool split = KSUB == 2 && live_q <= 2;
+    const bool a_warp = split ? (warp == 4 || warp == 5 || warp >= 8) : warp < 6;
+    const int a_h0 = split && warp >= 8 ? 1 : 0, a_h1 = split ? a_h0 + 1 : KSUB;
+    const int bblk = split ? (warp == 2 ? 0 : warp == 3 ? 1 : warp == 6 ? 2 : 3) : warp - 6;
     const int quarter = warp & 3;
-    const int arow = 32 * quarter + lane, brow = 32 * (warp - 6) + lane;
+    const int arow = 32 * quarter + lane, brow = 32 * bblk + lane;
     // a warp whose 32 A rows all lie past the kept rows skips its work: an accumulator row
     // depends only on its own A row, and the epilogue drops those rows
     const bool a_live = a_warp && m0 + 32 * quarter < valid_rows;
@@ -443,9 +452,9 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       if (a_warp) {
         if (a_live) {
           const uint32_t acol = a_lanes + BN + so * S::kAcols;
-          const int nsub = valid_subtiles<KSUB>(a.L, kt);
+          const int nsub = min(valid_subtiles<KSUB>(a.L, kt), a_h1);
 #pragma unroll 1
-          for (int h = 0; h < nsub; ++h) {  // one sub-tile's registers live at a time
+          for (int h = a_h0; h < nsub; ++h) {  // one sub-tile's registers live at a time
             uint32_t o[32];
             if (A_CODES) {
               const unsigned char* ra = rawA(sr) + h * (kBM * kBK);
