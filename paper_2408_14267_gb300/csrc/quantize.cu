@@ -478,36 +478,43 @@ __global__ void __launch_bounds__(32 * (kQWarps + 1), 4) quantize_kernel(QuantAr
   const int64_t cb = (int64_t)blockIdx.x * kQCols;
   const int64_t c0 = cb + lane * 4;
   const int64_t r0 = (int64_t)blockIdx.y * kQRows;
-  float gam[4], zc[4], invc[4];
+  // every load first (column and row slots, ranges, zero points and the 4 x 4 gradient
+  // values), so that they are in flight together instead of one dependent round trip each
+  float gam[4], zc[4], invc[4], crg[4];
   int32_t cslot[4];
   bool cdeg[4], cv[4];
-  bool any_c = false;
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const int64_t c = c0 + q;
     cv[q] = c < a.D;
+    const bool lc = a.do_pcq && cv[q];
     gam[q] = (a.gamma && cv[q]) ? __ldg(a.gamma + c) : 1.0f;
-    cslot[q] = (a.do_pcq && cv[q]) ? __ldg(a.c.slot + c) : -1;
-    zc[q] = 0.f; invc[q] = 0.f; cdeg[q] = true;
-    if (cslot[q] >= 0) {
-      const float r = __ldg(a.c.range + c);
-      zc[q] = __ldg(a.c.zmin + c);
-      invc[q] = __fdiv_rn(a.c.B, r);
-      cdeg[q] = !(r > 0.0f) || !isfinite(invc[q]);
-      any_c = true;
+    cslot[q] = lc ? __ldg(a.c.slot + c) : -1;
+    crg[q] = lc ? __ldg(a.c.range + c) : 0.f;
+    zc[q] = lc ? __ldg(a.c.zmin + c) : 0.f;
+  }
+  const int64_t rb = r0 + warp * 4;  // this warp's 4 rows
+  int32_t sslots[4];
+  int32_t srem[4];  // row within its sample group
+  float srg[4], szm[4];
+  {
+    int64_t gi = rb / a.rpg, rem = rb - gi * a.rpg;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (i > 0 && ++rem == a.rpg) { rem = 0; ++gi; }
+      srem[i] = (int32_t)rem;
+      const bool ls = a.do_psq && rb + i < a.M;
+      sslots[i] = ls ? __ldg(a.s.slot + gi) : -1;
+      srg[i] = ls ? __ldg(a.s.range + gi) : 0.f;
+      szm[i] = ls ? __ldg(a.s.zmin + gi) : 0.f;
     }
   }
-  // this warp's 4 rows: slots and loads first
-  const int64_t rb = r0 + warp * 4;
   float vv[4][4];
-  int32_t sslots[4];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const int64_t r = rb + i;
-    sslots[i] = (a.do_psq && r < a.M) ? __ldg(a.s.slot + r / a.rpg) : -1;
-    const bool need = r < a.M && (sslots[i] >= 0 || any_c);
     if (VEC) {
-      if (need && cv[0]) {
+      if (r < a.M && cv[0]) {
         const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + c0));
         vv[i][0] = t.x; vv[i][1] = t.y; vv[i][2] = t.z; vv[i][3] = t.w;
       } else {
@@ -515,8 +522,20 @@ __global__ void __launch_bounds__(32 * (kQWarps + 1), 4) quantize_kernel(QuantAr
       }
     } else {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) vv[i][q] = (need && cv[q]) ? __ldg(a.g + r * a.D + c0 + q) : 0.0f;
+      for (int q = 0; q < 4; ++q) vv[i][q] = (r < a.M && cv[q]) ? __ldg(a.g + r * a.D + c0 + q) : 0.0f;
     }
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    invc[q] = 0.f;
+    cdeg[q] = true;
+    if (cslot[q] >= 0) {
+      invc[q] = __fdiv_rn(a.c.B, crg[q]);
+      cdeg[q] = !(crg[q] > 0.0f) || !isfinite(invc[q]);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
 #pragma unroll
     for (int q = 0; q < 4; ++q) vv[i][q] = a.gamma ? __fmul_rn(vv[i][q], gam[q]) : vv[i][q];
   }
@@ -526,12 +545,11 @@ __global__ void __launch_bounds__(32 * (kQWarps + 1), 4) quantize_kernel(QuantAr
     const int64_t r = rb + i;
     const int32_t sslot = sslots[i];
     if (sslot < 0) continue;
-    const int64_t gi = r / a.rpg;
-    const float rs = __ldg(a.s.range + gi), zs = __ldg(a.s.zmin + gi);
+    const float rs = srg[i], zs = szm[i];
     const float inv = __fdiv_rn(a.s.B, rs);
     const bool deg = !(rs > 0.0f) || !isfinite(inv);
     const uint64_t e0 = (uint64_t)r * (uint64_t)a.D + (uint64_t)c0;
-    uint8_t* dst = a.s.codes + ((int64_t)sslot * a.rpg + (r - gi * a.rpg)) * a.s.ld + c0;
+    uint8_t* dst = a.s.codes + ((int64_t)sslot * a.rpg + srem[i]) * a.s.ld + c0;
     if (VEC) {
       if (cv[0]) {
         const U32x4 p = philox_block(a.s.seed, kStreamSrPsq, e0 >> 2);
