@@ -463,7 +463,9 @@ extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t
   // region of a tile of tm pixels: images it may touch x channels of 256 columns x whole planes.
   const int64_t Mi = (int64_t)N * Ho * Wo, Ki = (int64_t)C * kh * kw;
   if (pad <= 32 && Ki < (1ll << 31)) {
-    const int tm_first = Mi >= 64 * 152 * 4 ? 128 : 64;  // smaller tiles: more resident CTAs
+    // 128-pixel tiles (smaller only when the input region does not fit): fewer CTAs, each
+    // amortizing its region set-up over more output words
+    const int tm_first = 128;
     const bool same = stride == 1 && kh == kw && kh == 2 * pad + 1 && (Ho * Wo) % 32 == 0;
     // the fast path reads a 32-bit window up to pad W + pad bits before or after the plane
     const int guard = same ? (pad * W + pad + 63) / 32 : 1;
