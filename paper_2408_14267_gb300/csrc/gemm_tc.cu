@@ -813,8 +813,11 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     // every CTA of the cluster reaches both barriers, also after an expired wait
     cluster_sync_all();
     const uint32_t rank = cluster_rank(), nr = cluster_size();
-    const int rpr = (kBM + (int)nr - 1) / (int)nr;  // tile rows summed by each CTA
-    const int r_lo = (int)rank * rpr, r_hi = min(kBM, r_lo + rpr);
+    // the tile rows that exist (up to the capacity) are divided over the cluster's CTAs
+    const int64_t rows_here = a.M - m0;
+    const int nrows = rows_here >= kBM ? kBM : (rows_here <= 0 ? 0 : (int)rows_here);
+    const int rpr = (nrows + (int)nr - 1) / (int)nr;  // tile rows summed by each CTA
+    const int r_lo = min(nrows, (int)rank * rpr), r_hi = min(nrows, r_lo + rpr);
     const uint32_t pbase = smem_u32(base);
     const bool ok = !abort_flag;
     const bool vec = (a.ldo % 4) == 0;
@@ -825,10 +828,14 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       int4 sum = make_int4(0, 0, 0, 0);
       const bool kept = ok && grow < valid_rows;
       if (kept) {
-        for (uint32_t src = 0; src < nr; ++src) {
-          const int4 t = ld_cluster_v4(pbase + ptile_off(r, ch), src);
-          sum.x += t.x; sum.y += t.y; sum.z += t.z; sum.w += t.w;
-        }
+        // all of the cluster's partial chunks in flight together (clusters have <= 8 CTAs)
+        int4 t[8];
+#pragma unroll
+        for (uint32_t src = 0; src < 8; ++src)
+          if (src < nr) t[src] = ld_cluster_v4(pbase + ptile_off(r, ch), src);
+#pragma unroll
+        for (uint32_t src = 0; src < 8; ++src)
+          if (src < nr) { sum.x += t[src].x; sum.y += t[src].y; sum.z += t[src].z; sum.w += t[src].w; }
       }
       const int32_t sv[4] = {sum.x, sum.y, sum.z, sum.w};
       int32_t* arow = a.acc + grow * a.ldo + n;
