@@ -212,6 +212,12 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32
       : "memory");
 }
 
+// Folder of a 3 x 3, stride-1, pad-1 convolution (Ho = H, Wo = W): tap offsets are computed,
+// not looked up.
+__device__ __forceinline__ bool fold_same3(const TcArgs& a) {
+  return a.fkh == 3 && a.fkw == 3 && a.fstride == 1 && a.fpad == 1;
+}
+
 // Sub-tiles of stage kt that hold contraction elements below L (1..KSUB for a stage that
 // starts below L).
 template <int KSUB>
@@ -343,6 +349,8 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     int4* zb = reinterpret_cast<int4*>(base + S::kMain + kFoldTab - kFoldZero);
     for (int x = threadIdx.x - 64; x < kFoldZero / 16; x += 256) zb[x] = make_int4(0, 0, 0, 0);
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the bulk stores read it later
+  }
+  if (SHORT && a.epi == EPI_FOLD && threadIdx.x >= 64 && !fold_same3(a)) {  // same 3x3: offsets computed
     const int khw = a.fkh * a.fkw, HW = a.fH * a.fW;
     for (int x = threadIdx.x - 64; x < HW * khw; x += 256) {
       const int pos = (int)a.fd_khw.div((uint32_t)x), t = x - pos * khw;
@@ -550,8 +558,16 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       for (int x = tt; x < f_nc * f_HW; x += 256) {
         const int cl = (int)a.fd_hw.div((uint32_t)x), pos = x - cl * f_HW;
         int32_t cs = 0;
-        for (int t = 0; t < f_khw; ++t)
-          if (f_tap[pos * f_khw + t] >= 0) cs += f_cs[cl * f_khw + t];
+        if (fold_same3(a)) {  // tap (i, j) of input (h, w) lands on output (h + 1 - i, w + 1 - j)
+          const int h = (int)a.fd_w.div((uint32_t)pos), w = pos - h * a.fW;
+#pragma unroll
+          for (int t = 0; t < 9; ++t)
+            if ((unsigned)(h + 1 - t / 3) < (unsigned)a.fH && (unsigned)(w + 1 - t % 3) < (unsigned)a.fW)
+              cs += f_cs[cl * 9 + t];
+        } else {
+          for (int t = 0; t < f_khw; ++t)
+            if (f_tap[pos * f_khw + t] >= 0) cs += f_cs[cl * f_khw + t];
+        }
         f_csf[x] = cs;
       }
     }
@@ -606,7 +622,18 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         const int32_t* tim = T + img * rpg * TS + cl * khw;
         const int32_t* to = tap_off + pos * khw;
         int32_t acc = 0;
-        if (khw == 9) {  // 3 x 3 kernels: all table and tile loads in flight together
+        if (fold_same3(a)) {
+          // 3 x 3, stride 1, pad 1: tap (i, j) of input (h, w) is the product of output pixel
+          // (h + 1 - i, w + 1 - j), i.e. tile row pos + (1 - i) W + (1 - j), column 3 i + j
+          const int h = (int)a.fd_w.div((uint32_t)pos), w = pos - h * a.fW;
+          const int32_t* tp = tim + pos * TS;
+#pragma unroll
+          for (int t = 0; t < 9; ++t) {
+            const int di = 1 - t / 3, dj = 1 - t % 3;
+            const bool v = (unsigned)(h + di) < (unsigned)a.fH && (unsigned)(w + dj) < (unsigned)a.fW;
+            acc += v ? tp[(di * a.fW + dj) * TS + t] : 0;
+          }
+        } else if (khw == 9) {  // other 3 x 3 kernels: all table and tile loads in flight together
           int o[9];
 #pragma unroll
           for (int t = 0; t < 9; ++t) o[t] = to[t];
