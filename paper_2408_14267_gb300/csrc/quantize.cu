@@ -122,8 +122,9 @@ struct SelectArgs {
 
 constexpr int kSelThreads = 1024;
 
-// Inclusive scan of one uint64 per thread across the CTA; returns the inclusive value
-// and writes the CTA total to *total.
+// Inclusive scan of one uint64 per thread across the CTA's NT threads; returns the inclusive
+// value and writes the CTA total to *total.
+template <int NT>
 __device__ uint64_t block_inclusive_scan(uint64_t v, uint64_t* warp_sums, uint64_t* total) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
@@ -134,7 +135,7 @@ __device__ uint64_t block_inclusive_scan(uint64_t v, uint64_t* warp_sums, uint64
   if (lane == 31) warp_sums[warp] = v;
   __syncthreads();
   if (warp == 0) {
-    uint64_t s = warp_sums[lane];
+    uint64_t s = lane < NT / 32 ? warp_sums[lane] : 0ull;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const uint64_t t = __shfl_up_sync(0xFFFFFFFFu, s, o);
@@ -178,7 +179,9 @@ __device__ __forceinline__ double p_hat_of(uint64_t P) {
   return __longlong_as_double((long long)((ex << 52) | frac));
 }
 
-__global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, SelectArgs a1) {
+// NT threads per CTA (256 when every grouping has at most 256 groups, else 1024).
+template <int NT>
+__global__ void __launch_bounds__(NT) select_kernel(SelectArgs a0, SelectArgs a1) {
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
   const SelectArgs& a = blockIdx.x == 0 ? a0 : a1;
@@ -187,8 +190,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
   __shared__ uint32_t s_rmax;
   __shared__ int s_tstar;
   __shared__ uint64_t s_kth, s_stot;
-  __shared__ int rank_s[kSelThreads];
-  __shared__ uint64_t sorted_s[kSelThreads];
+  __shared__ int rank_s[NT];
+  __shared__ uint64_t sorted_s[NT];
   const int n = a.n, tid = threadIdx.x;
   if (n <= 0) return;
   int npad = 1;
@@ -200,7 +203,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
   // Z = min, R = max - min (fp32)
   if (tid == 0) s_rmax = 0u;
   __syncthreads();
-  for (int i = tid; i < n; i += kSelThreads) {
+  for (int i = tid; i < n; i += NT) {
     const float z = ordered_to_float(a.kmin[i]);
     const float r = __fsub_rn(ordered_to_float(~a.kmax[i]), z);
     o.group_min[i] = z;
@@ -226,7 +229,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
     return sh >= 0 ? (m << sh) : (sh <= -32 ? 0ull : (m >> -sh));
   };
 
-  if (a.bits > 1 && n <= kSelThreads) {
+  if (a.bits > 1 && n <= NT) {
     // rank of each key (R~ desc, index asc) by comparison with all others: no sort needed
     uint64_t myk = 0, myrt = 0;
     if (tid < n) {
@@ -279,7 +282,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
       const int t = n - 1 - tid;
       const uint64_t v = (tid < n) ? key[t] : 0ull;
       uint64_t total;
-      const uint64_t suffix = block_inclusive_scan(v, warp_sums, &total);
+      const uint64_t suffix = block_inclusive_scan<NT>(v, warp_sums, &total);
       if (tid == 0) s_tstar = n;
       __syncthreads();
       if (tid < n) {
@@ -304,12 +307,12 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
     }
   } else if (a.bits > 1) {
     // sort keys (R~ desc, index asc) descending
-    for (int i = tid; i < npad; i += kSelThreads)
+    for (int i = tid; i < npad; i += NT)
       key[i] = i < n ? ((rtilde(i) << 24) | (uint64_t)(0xFFFFFFu - (uint32_t)i)) : 0ull;
     __syncthreads();
     for (int size = 2; size <= npad; size <<= 1) {
       for (int stride = size >> 1; stride > 0; stride >>= 1) {
-        for (int i = tid; i < npad / 2; i += kSelThreads) {
+        for (int i = tid; i < npad / 2; i += NT) {
           const int lo = 2 * i - (i & (stride - 1));
           const int hi = lo + stride;
           const bool desc = (lo & size) == 0;
@@ -324,13 +327,13 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
       if (tid == 0) { s_kth = key[k - 1]; s_tstar = k; s_stot = 0; }
     } else {
       // suffix sums S_t over sorted positions; t* = first t with (n - b t) R~_(t) <= b S_t
-      const int per = (npad + kSelThreads - 1) / kSelThreads;
+      const int per = (npad + NT - 1) / NT;
       const int beg = min(npad, tid * per), end = min(npad, beg + per);
       uint64_t local = 0;
       for (int t = beg; t < end; ++t) local += key[t] >> 24;
       // suffix of thread chunks: scan reversed thread order
       uint64_t total;
-      const uint64_t incl = block_inclusive_scan(local, warp_sums, &total);
+      const uint64_t incl = block_inclusive_scan<NT>(local, warp_sums, &total);
       uint64_t suffix = total - incl + local;  // sum of positions >= beg
       int best = n;
       uint64_t best_s = 0;
@@ -352,7 +355,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
     // P_i by group index (reuses the key buffer)
     const int tstar = s_tstar;
     const uint64_t kth = s_kth, S = s_stot;
-    for (int i = tid; i < n; i += kSelThreads) {
+    for (int i = tid; i < n; i += NT) {
       const uint64_t rt = rtilde(i);
       const uint64_t ki = (rt << 24) | (uint64_t)(0xFFFFFFu - (uint32_t)i);
       uint64_t P;
@@ -369,22 +372,22 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
       key[i] = P;
     }
   } else {
-    for (int i = tid; i < n; i += kSelThreads) key[i] = two32;
+    for (int i = tid; i < n; i += NT) key[i] = two32;
   }
   __syncthreads();
 
   // masks in index order; each thread owns a contiguous chunk
-  const int per = (n + kSelThreads - 1) / kSelThreads;
+  const int per = (n + NT - 1) / NT;
   const int beg = min(n, tid * per), end = min(n, beg + per);
   uint64_t psum = 0;
   for (int i = beg; i < end; ++i) psum += key[i];
   uint64_t total;
-  const uint64_t pincl = block_inclusive_scan(psum, warp_sums, &total);
+  const uint64_t pincl = block_inclusive_scan<NT>(psum, warp_sums, &total);
   uint64_t c = pincl - psum;
   uint64_t u = 0;
   if (a.bits > 1 && a.mode == FQT1_SEL_SYSTEMATIC) u = philox_word(a.seed, a.stream, 0);
   c += u;
-  uint32_t kept_bits = 0;  // chunk length <= 16 for n <= 16384
+  uint64_t kept_bits = 0;  // chunk length <= 64 for n <= 16384 and NT >= 256
   int nk = 0;
   for (int i = beg; i < end; ++i) {
     const uint64_t P = key[i];
@@ -394,16 +397,16 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
     else if (a.mode == FQT1_SEL_BERNOULLI) kept = (uint64_t)philox_word(a.seed, a.stream, (uint64_t)i) < P;
     else kept = P == two32;
     c += P;
-    if (kept) { kept_bits |= 1u << (i - beg); ++nk; }
+    if (kept) { kept_bits |= 1ull << (i - beg); ++nk; }
   }
   uint64_t ktot;
-  const uint64_t kincl = block_inclusive_scan((uint64_t)nk, warp_sums, &ktot);
+  const uint64_t kincl = block_inclusive_scan<NT>((uint64_t)nk, warp_sums, &ktot);
   int slot = (int)(kincl - nk);
   // the per-slot scale and zero point are computed by the quantize kernel
   for (int i = beg; i < end; ++i) {
     const uint64_t P = key[i];
     o.p_hat[i] = p_hat_of(P);
-    if (kept_bits & (1u << (i - beg))) {
+    if (kept_bits & (1ull << (i - beg))) {
       o.slot_of_group[i] = slot;
       o.kept_idx[slot] = i;
       ++slot;
@@ -411,7 +414,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelectArgs a0, Sele
       o.slot_of_group[i] = -1;
     }
   }
-  for (int s = (int)ktot + tid; s < a.capacity; s += kSelThreads) o.kept_idx[s] = -1;
+  for (int s = (int)ktot + tid; s < a.capacity; s += NT) o.kept_idx[s] = -1;
   if (tid == 0) *o.kept_count = (int32_t)ktot;
 }
 
@@ -688,11 +691,16 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
   const size_t smem = (size_t)npad_max * 8 + (size_t)npad_max * 4;
   static bool attr_done = false;
   if (!attr_done) {
-    FQT1_CUDA_TRY(cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    FQT1_CUDA_TRY(cudaFuncSetAttribute(select_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (size_t)kMaxGroups * 12));
+    FQT1_CUDA_TRY(cudaFuncSetAttribute(select_kernel<kSelThreads>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (size_t)kMaxGroups * 12));
     attr_done = true;
   }
-  launch_k(select_kernel, dim3(nsel), dim3(kSelThreads), smem, s, sa[0], nsel > 1 ? sa[1] : sa[0]);
+  if (npad_max <= 256)  // fewer warps per barrier when every grouping has at most 256 groups
+    launch_k(select_kernel<256>, dim3(nsel), dim3(256), smem, s, sa[0], nsel > 1 ? sa[1] : sa[0]);
+  else
+    launch_k(select_kernel<kSelThreads>, dim3(nsel), dim3(kSelThreads), smem, s, sa[0], nsel > 1 ? sa[1] : sa[0]);
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
 
