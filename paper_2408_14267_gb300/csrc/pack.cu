@@ -190,14 +190,21 @@ struct UnfoldArgs {
 };
 
 // 32 x 32 bit transpose across a warp: lane r holds row r (bit c = column c); afterwards
-// lane c holds column c (bit r = row r).  Each step swaps the off-diagonal j x j blocks.
+// lane c holds column c (bit r = row r).  Step j swaps the off-diagonal j x j blocks: the
+// lower lane of a pair keeps the low block of every 2j-bit field (mask m) and takes the
+// partner's low block moved up by j; the upper lane keeps the high blocks and takes the
+// partner's high blocks moved down.  A rotation by +-j followed by one bit select does
+// either (the bits that wrap around land in the half that is not taken).
 __device__ __forceinline__ uint32_t warp_transpose32(uint32_t x, int lane) {
 #pragma unroll
   for (int j = 16; j >= 1; j >>= 1) {
     const uint32_t m = j == 16 ? 0x0000FFFFu : j == 8 ? 0x00FF00FFu : j == 4 ? 0x0F0F0F0Fu : j == 2 ? 0x33333333u
                                                                                                       : 0x55555555u;
+    const bool up = (lane & j) != 0;
     const uint32_t p = __shfl_xor_sync(0xFFFFFFFFu, x, j);
-    x = (lane & j) ? ((x & ~m) | ((p >> j) & m)) : ((x & m) | ((p & m) << j));
+    const uint32_t r = __funnelshift_l(p, p, up ? 32 - j : j);
+    const uint32_t take = up ? m : ~m;
+    x = (x & ~take) | (r & take);
   }
   return x;
 }
@@ -248,9 +255,10 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
     for (int q0 = 0; q0 < data_words; q0 += 4) {  // 4 loads in flight per lane, then 4 ballots
       float v[4];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
+      for (int u = 0; u < 4; ++u) {  // unconditional loads from clamped indices, masked afterwards
         const int e = 32 * (q0 + u) + lane;
-        v[u] = (q0 + u < data_words && e < plane_bits) ? __ldg(src + e) : 0.0f;
+        v[u] = __ldg(src + min(e, plane_bits - 1));
+        if (q0 + u >= data_words || e >= plane_bits) v[u] = 0.0f;
       }
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
@@ -391,6 +399,167 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
   }
 }
 
+// ---------------------------------------------------------------------------
+// Unfolder for "same" convolutions (stride 1, kh = kw = 2 pad + 1, so Ho = H and Wo = W)
+// whose planes hold a multiple of 32 pixels and whose tiles hold whole images: a tile is
+// 32 NSUB pixels = ipt images x 256 columns.
+//  1. The input region of a tile (ipt images x nc channels, whole planes) is, per image,
+//     one contiguous run of x, so sign-packing it is a linear copy into shared memory:
+//     word f of the region is the ballot of 32 consecutive floats.  Planes lie back to back
+//     (dw = H W / 32 words each); zero guard words sit only before and after the region.
+//  2. Pixel p reads input pixel p + (i - pad) W + (j - pad) for tap (i, j), so the column
+//     word of k over 32 pixels of one image is a 32-bit window of its channel's plane.  It
+//     is masked to the pixels whose tap lands inside the image: a pixel interval for the
+//     input row (reads that cross into a neighbouring plane fall outside it) and a per-j
+//     pattern for the input column.  The shuffle transpose gives the row words.
+//  3. Row words and column words go through XOR-swizzled shared memory (conflict-free
+//     32-lane writes) and leave as 16-byte stores; the column sums come from the same reads.
+struct UnfoldSameArgs {
+  const float* x;
+  uint32_t* row_bits;
+  uint32_t* col_bits;
+  int32_t* colsum;
+  int64_t row_words, col_words;
+  int N, C, H, W, pad, kw, khw, K, HW;
+  int dw;        // words per plane, H W / 32
+  int ipt;       // images per tile, 32 NSUB / (H W)
+  int guard;     // zero words before and after the region
+  uint32_t rep;  // W divides 32: replicates a W-bit row pattern over 32 bits (1 for W = 32); else 0
+  FastDiv div_khw, div_kw;
+};
+
+__device__ __forceinline__ uint32_t bit_range(int lo, int hi) {  // bits lo .. hi - 1 of a word
+  lo = max(lo, 0);
+  hi = min(hi, 32);
+  if (hi <= lo) return 0u;
+  return (hi - lo == 32 ? 0xFFFFFFFFu : ((1u << (hi - lo)) - 1u)) << lo;
+}
+
+// 4 words read as one 16-byte vector from a chunk whose words were stored at index ^ z
+// (z in 0..3): word e of the result is the vector's word e ^ z.
+__device__ __forceinline__ uint4 unswizzle4(uint4 v, int z) {
+  if (z & 2) v = make_uint4(v.z, v.w, v.x, v.y);
+  if (z & 1) v = make_uint4(v.y, v.x, v.w, v.z);
+  return v;
+}
+
+template <int NSUB>
+__global__ void __launch_bounds__(256) unfold_same_kernel(UnfoldSameArgs a) {
+  static_assert(NSUB == 4 || NSUB == 8, "tiles of 128 or 256 pixels");
+  constexpr int TM = 32 * NSUB;
+  constexpr int kZShift = NSUB == 4 ? 3 : 2;  // column-word swizzle: (k >> kZShift) & (NSUB - 1)
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  extern __shared__ uint32_t region[];
+  __shared__ __align__(16) uint32_t rw_s[TM * 8];     // [pixel][8 k-words], word q at q ^ ((pixel >> 2) & 7)
+  __shared__ __align__(16) uint32_t cw_s[256 * NSUB];  // [k][NSUB pixel-words], word s at s ^ z(k)
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_lo = blockIdx.y * a.ipt;
+  const int nimg = min(a.ipt, a.N - n_lo);
+  const int k0 = blockIdx.x * 256, k1 = min(a.K, k0 + 256);
+  const int c_lo = (int)a.div_khw.div((uint32_t)k0);
+  const int nc = (int)a.div_khw.div((uint32_t)(k1 - 1)) - c_lo + 1;
+  const int span = nc * a.dw;  // region words per image
+  const int total = nimg * span;
+  uint32_t* st = region + a.guard;
+  // 1. sign-pack; f / span by a multiply-high with ceil(2^32 / span) (exact for f, span < 2^16)
+  {
+    const uint32_t inv = (uint32_t)(0xFFFFFFFFu / (uint32_t)span) + 1u;
+    const float* src = a.x + ((int64_t)n_lo * a.C + c_lo) * a.HW + lane;
+    const int64_t img_stride = (int64_t)a.C * a.HW;
+    for (int f0 = warp; f0 < total; f0 += 8 * 16) {
+      // unconditional loads from clamped word indices (the ballots of words past the region are
+      // not stored): a load under a condition is not hoisted, and the 16 round trips serialize
+      float v[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const int f = min(f0 + 8 * u, total - 1);
+        const int img = (int)__umulhi((uint32_t)f, inv);
+        v[u] = __ldg(src + img * img_stride + (int64_t)(f - img * span) * 32);
+      }
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const uint32_t word = __ballot_sync(0xFFFFFFFFu, v[u] > 0.0f);
+        if (lane == 0 && f0 + 8 * u < total) st[f0 + 8 * u] = word;
+      }
+    }
+    for (int e = threadIdx.x; e < 2 * a.guard; e += 256) region[e < a.guard ? e : total + e] = 0u;
+  }
+  __syncthreads();
+  // 2. column word of k = kb + lane over each 32-pixel sub-tile, and its transpose
+  const int kb = k0 + 32 * warp;
+  const int k = kb + lane;
+  const bool kvalid = k < k1;
+  const int kk = min(k, a.K - 1);
+  const int c = (int)a.div_khw.div((uint32_t)kk), t = kk - c * a.khw;
+  const int i = (int)a.div_kw.div((uint32_t)t), j = t - i * a.kw;
+  const int plo = max(0, a.pad - i) * a.W, phi = min(a.H, a.H + a.pad - i) * a.W;  // pixels with the row inside
+  const int olo = max(0, a.pad - j), ohi = min(a.W, a.W + a.pad - j);              // output columns inside
+  const uint32_t cmask_rep = a.rep ? bit_range(olo, ohi) * a.rep : 0u;
+  // bit position, relative to st, of the window of pixel 0 of image 0
+  const int pos0 = 32 * (c - c_lo) * a.dw + (i - a.pad) * a.W + (j - a.pad);
+  int img = 0, q = 0, ow0 = 0;  // sub-tile s = img dw + q; ow0 = output column of its bit 0
+#pragma unroll 1
+  for (int s = 0; s < NSUB; ++s) {
+    uint32_t colw = 0;
+    if (kvalid && img < nimg) {
+      const int p0 = 32 * q;
+      const int pos = pos0 + 32 * img * span + p0;
+      const int w = pos >> 5, o = pos & 31;
+      const uint64_t v = ((uint64_t)st[w + 1] << 32) | st[w];
+      uint32_t cmask = cmask_rep;
+      if (!a.rep) {
+        for (int b = 0, tt = ow0; b < 32;) {
+          const int seg = min(a.W - tt, 32 - b);
+          cmask |= bit_range(b + max(olo - tt, 0), b + min(ohi - tt, seg));
+          b += seg;
+          tt = 0;
+        }
+      }
+      colw = (uint32_t)(v >> o) & bit_range(plo - p0, phi - p0) & cmask;
+    }
+    const uint32_t roww = warp_transpose32(colw, lane);
+    const int px = 32 * s + lane;
+    rw_s[px * 8 + (warp ^ ((px >> 2) & 7))] = roww;
+    const int kl = 32 * warp + lane;
+    cw_s[kl * NSUB + (s ^ ((kl >> kZShift) & (NSUB - 1)))] = colw;
+    if (!a.rep) {
+      ow0 += 32;
+      while (ow0 >= a.W) ow0 -= a.W;
+    }
+    if (++q == a.dw) { q = 0; ++img; ow0 = 0; }
+  }
+  __syncthreads();
+  // 3. outputs as 16-byte chunks
+  if (a.row_bits) {
+    const int64_t wbase = (int64_t)k0 / 32;
+    for (int e = threadIdx.x; e < 2 * TM; e += 256) {
+      const int px = e >> 1, h = e & 1;
+      const int sw = (px >> 2) & 7;
+      if (px < nimg * a.HW && wbase + 4 * h < a.row_words) {
+        const uint4 v = unswizzle4(*reinterpret_cast<const uint4*>(rw_s + px * 8 + 4 * (h ^ (sw >> 2))), sw & 3);
+        *reinterpret_cast<uint4*>(a.row_bits + ((int64_t)n_lo * a.HW + px) * a.row_words + wbase + 4 * h) = v;
+      }
+    }
+  }
+  {
+    const int kl = threadIdx.x;
+    if (k0 + kl < k1) {
+      const int z = (kl >> kZShift) & (NSUB - 1);
+      const int64_t wbase = (int64_t)blockIdx.y * NSUB;
+      int ones = 0;
+#pragma unroll
+      for (int h = 0; h < NSUB / 4; ++h) {
+        const uint4 v = unswizzle4(*reinterpret_cast<const uint4*>(cw_s + kl * NSUB + 4 * (h ^ (z >> 2))), z & 3);
+        ones += __popc(v.x) + __popc(v.y) + __popc(v.z) + __popc(v.w);
+        if (a.col_bits && wbase + 4 * h < a.col_words)
+          *reinterpret_cast<uint4*>(a.col_bits + (int64_t)(k0 + kl) * a.col_words + wbase + 4 * h) = v;
+      }
+      if (a.colsum) atomicAdd(a.colsum + k0 + kl, 2 * ones - nimg * a.HW);
+    }
+  }
+}
+
 template <class Loader>
 static fqt1_status launch_pack(const Loader& L, uint32_t* row_bits, uint32_t* col_bits, int32_t* colsum,
                                cudaStream_t s) {
@@ -462,11 +631,45 @@ extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t
   // Bit-level Unfolder when the input region of a tile fits in shared memory.  Bound on the
   // region of a tile of tm pixels: images it may touch x channels of 256 columns x whole planes.
   const int64_t Mi = (int64_t)N * Ho * Wo, Ki = (int64_t)C * kh * kw;
+  const bool same = stride == 1 && kh == kw && kh == 2 * pad + 1 && (Ho * Wo) % 32 == 0;
+  if (same && pad <= 32 && Ki < (1ll << 31) && (128 % (H * W) == 0 || H * W == 256)) {
+    // whole images per tile: the contiguous-region Unfolder
+    UnfoldSameArgs u;
+    u.x = x; u.row_bits = row_bits; u.col_bits = col_bits; u.colsum = colsum;
+    u.row_words = fqt1_packed_words(Ki); u.col_words = fqt1_packed_words(Mi);
+    u.N = N; u.C = C; u.H = H; u.W = W; u.pad = pad; u.kw = kw; u.khw = kh * kw; u.K = (int)Ki; u.HW = H * W;
+    u.dw = H * W / 32;
+    const int nsub = H * W == 256 ? 8 : 4;
+    u.ipt = 32 * nsub / (H * W);
+    u.guard = (pad * W + pad + 63) / 32;
+    u.rep = 32 % W == 0 ? (W == 32 ? 1u : 0xFFFFFFFFu / ((1u << W) - 1u)) : 0u;
+    u.div_khw = FastDiv((uint32_t)(kh * kw)); u.div_kw = FastDiv((uint32_t)kw);
+    const int64_t nc_max = std::min<int64_t>(C, 256 / (kh * kw) + 2);
+    const size_t smem = (size_t)(2 * u.guard + u.ipt * nc_max * u.dw) * 4;
+    const int64_t row_tiles = (N + u.ipt - 1) / u.ipt, word_tiles = (Ki + 255) / 256;
+    if (row_tiles <= 65535 && smem <= 32 * 1024) {
+      if (colsum) FQT1_CUDA_TRY(cudaMemsetAsync(colsum, 0, sizeof(int32_t) * Ki, s));
+      if (nsub == 4)
+        launch_k(unfold_same_kernel<4>, dim3((unsigned)word_tiles, (unsigned)row_tiles), dim3(256), smem, s, u);
+      else
+        launch_k(unfold_same_kernel<8>, dim3((unsigned)word_tiles, (unsigned)row_tiles), dim3(256), smem, s, u);
+      fqt1_count_launches(1);
+      FQT1_CUDA_TRY(cudaGetLastError());
+      const int64_t written = row_tiles * nsub;
+      if (col_bits && u.col_words > written) {
+        const int64_t n = Ki * (u.col_words - written);
+        launch_k(zero_col_pad_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, col_bits, Ki, u.col_words,
+                 written);
+        fqt1_count_launches(1);
+        FQT1_CUDA_TRY(cudaGetLastError());
+      }
+      return FQT1_OK;
+    }
+  }
   if (pad <= 32 && Ki < (1ll << 31)) {
     // 128-pixel tiles (smaller only when the input region does not fit): fewer CTAs, each
     // amortizing its region set-up over more output words
     const int tm_first = 128;
-    const bool same = stride == 1 && kh == kw && kh == 2 * pad + 1 && (Ho * Wo) % 32 == 0;
     // the fast path reads a 32-bit window up to pad W + pad bits before or after the plane
     const int guard = same ? (pad * W + pad + 63) / 32 : 1;
     for (int tm = tm_first; tm >= 32; tm /= 2) {

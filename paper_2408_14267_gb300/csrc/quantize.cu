@@ -24,7 +24,18 @@ struct RangeArgs {
   uint32_t *smin, *smax;  // [M / rpg] or null (smax holds complemented keys)
   uint32_t *cmin, *cmax;  // [D] or null (cmax holds complemented keys)
   int32_t* dev_status;
+  FastDiv div_rpg;        // row -> sample group (rows < 2^31)
 };
+
+// Loads of a kernel's prologue are issued unconditionally, from a clamped index (or from
+// `any`, a valid address, when the array is absent), and the result is selected afterwards:
+// a load under a condition is not hoisted above the code before it, and a chain of them
+// costs one memory round trip each.
+template <class T>
+__device__ __forceinline__ T ldg_sel(const T* p, int64_t i, bool ok, T dflt, const void* any) {
+  const T v = __ldg(p ? p + (ok ? i : 0) : reinterpret_cast<const T*>(any));
+  return ok ? v : dflt;
+}
 
 template <bool VEC>
 __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
@@ -39,7 +50,7 @@ __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     cv[q] = c0 + q < a.D;
-    gam[q] = (a.gamma && cv[q]) ? __ldg(a.gamma + c0 + q) : 1.0f;
+    gam[q] = ldg_sel(a.gamma, c0 + q, a.gamma && cv[q], 1.0f, a.g);
   }
   uint32_t colmin[4] = {0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu}, colmax[4] = {0u, 0u, 0u, 0u};
   uint32_t gmin = 0xFFFFFFFFu, gmax = 0u;
@@ -48,25 +59,23 @@ __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
   constexpr int kR = kRangeRows / 8;  // rows per warp
   float v[kR][4];
 #pragma unroll
-  for (int i = 0; i < kR; ++i) {  // all loads of this warp's rows first
-    const int64_t r = r0 + i;
+  for (int i = 0; i < kR; ++i) {  // all loads of this warp's rows first, unconditional (clamped)
+    const int64_t r = min(r0 + i, a.M - 1);
     if (VEC) {
-      if (cv[0] && r < a.M) {
-        const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + c0));
-        v[i][0] = t.x; v[i][1] = t.y; v[i][2] = t.z; v[i][3] = t.w;
-      } else {
-        v[i][0] = v[i][1] = v[i][2] = v[i][3] = 0.f;
-      }
+      const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + (cv[0] ? c0 : 0)));
+      v[i][0] = t.x; v[i][1] = t.y; v[i][2] = t.z; v[i][3] = t.w;
     } else {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) v[i][q] = (cv[q] && r < a.M) ? __ldg(a.g + r * a.D + c0 + q) : 0.0f;
+      for (int q = 0; q < 4; ++q) v[i][q] = __ldg(a.g + r * a.D + min(c0 + q, a.D - 1));
     }
   }
+  // sample group of the first row; the next rows step through it
+  int64_t gi = a.div_rpg.div((uint32_t)min(r0, a.M - 1)), grem = min(r0, a.M - 1) - gi * a.rpg;
 #pragma unroll
   for (int i = 0; i < kR; ++i) {
     const int64_t r = r0 + i;
     if (r >= a.M) break;
-    const int64_t gi = r / a.rpg;
+    if (i > 0 && ++grem == a.rpg) { grem = 0; ++gi; }
     if (a.smin && gi != cur) {
       if (cur >= 0) {
         const uint32_t mn = __reduce_min_sync(0xFFFFFFFFu, gmin), mx = __reduce_max_sync(0xFFFFFFFFu, gmax);
@@ -462,79 +471,110 @@ struct QuantArgs {
   int64_t M, D, rpg;
   int do_psq, do_pcq;
   QBranch s, c;
+  FastDiv div_rpg;  // row -> sample group (rows < 2^31)
 };
 
+// Quantization of one 32 x 128 tile of G = gY * gamma for both branches (Sec. 5.3).
+//  - Warps 0-7 load the tile (warp w: rows 4w .. 4w+3, lane l: columns 4l .. 4l+3) and the
+//    per-row and per-column constants, every load unconditional so that all are in flight
+//    together.
+//  - PSQ: rows of kept sample groups; element (m, j) takes word m D + j of stream 0, so one
+//    Philox block gives a lane's 4 columns of a row.
+//  - PCQ: the tile goes to shared memory and the kept columns of the tile are listed; one
+//    thread per (kept column, 4 rows) draws one Philox block (words j M + m .. + 3 of stream
+//    1) and forms the 4 codes, so no rounding is spent on pruned channels.
+//  - Warp 8 lists the kept columns with their constants (and signals barrier 1 without
+//    waiting), then computes the per-slot S' and Z' in float64 beside the quantizing warps.
 template <bool VEC>
 __global__ void __launch_bounds__(32 * (kQWarps + 1), 4) quantize_kernel(QuantArgs a) {
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
-  __shared__ uint32_t tile[kQCols][kQRows / 4 + 1];  // PCQ codes, 4 rows per word
+  __shared__ __align__(16) float gt[kQRows][kQCols + 4];  // the tile of G * gamma
+  __shared__ uint32_t tile[kQCols][kQRows / 4 + 1];       // codes of kept column j, 4 rows per word
+  __shared__ int32_t klist[kQCols], kslot[kQCols];        // kept column j: tile column, slot
+  __shared__ float kz[kQCols], kinv[kQCols];              // its Z and B / R (negative: degenerate)
+  __shared__ int32_t nk_s;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (warp == kQWarps) {
-    // the float64 divisions run beside the quantizing warps of this CTA
-    const int64_t cta = (int64_t)blockIdx.y * gridDim.x + blockIdx.x, ncta = (int64_t)gridDim.x * gridDim.y;
-    slot_constants(a.s, a.c, a.do_psq != 0, a.do_pcq != 0, cta, ncta, lane);
-    __syncwarp();
-    if (a.do_pcq) __syncthreads();  // the PCQ tile barrier below
-    return;
-  }
   const int64_t cb = (int64_t)blockIdx.x * kQCols;
   const int64_t c0 = cb + lane * 4;
   const int64_t r0 = (int64_t)blockIdx.y * kQRows;
-  // every load first (column and row slots, ranges, zero points and the 4 x 4 gradient
+  if (warp == kQWarps) {
+    if (a.do_pcq) {
+      // the kept columns of the tile in ascending order (lane l: columns 4l .. 4l+3)
+      int32_t cslot[4];
+      float crg[4], zc[4];
+      int mine = 0;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const bool lc = c0 + q < a.D;
+        cslot[q] = ldg_sel(a.c.slot, c0 + q, lc, -1, a.g);
+        crg[q] = ldg_sel(a.c.range, c0 + q, lc, 0.f, a.g);
+        zc[q] = ldg_sel(a.c.zmin, c0 + q, lc, 0.f, a.g);
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) mine += cslot[q] >= 0 ? 1 : 0;
+      int incl = mine;
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const int t = __shfl_up_sync(0xFFFFFFFFu, incl, d);
+        if (lane >= d) incl += t;
+      }
+      int j = incl - mine;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        if (cslot[q] < 0) continue;
+        const float inv = __fdiv_rn(a.c.B, crg[q]);
+        klist[j] = 4 * lane + q;
+        kslot[j] = cslot[q];
+        kz[j] = zc[q];
+        kinv[j] = (!(crg[q] > 0.0f) || !isfinite(inv)) ? -1.0f : inv;
+        ++j;
+      }
+      if (lane == 31) nk_s = incl;
+      asm volatile("bar.arrive 1, %0;" ::"n"(32 * (kQWarps + 1)) : "memory");
+    }
+    // the float64 divisions run beside the quantizing warps of this CTA
+    const int64_t cta = (int64_t)blockIdx.y * gridDim.x + blockIdx.x, ncta = (int64_t)gridDim.x * gridDim.y;
+    slot_constants(a.s, a.c, a.do_psq != 0, a.do_pcq != 0, cta, ncta, lane);
+    return;
+  }
+  // every load first (gamma, the row slots, ranges and zero points, the 4 x 4 gradient
   // values), so that they are in flight together instead of one dependent round trip each
-  float gam[4], zc[4], invc[4], crg[4];
-  int32_t cslot[4];
-  bool cdeg[4], cv[4];
+  float gam[4];
+  bool cv[4];
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const int64_t c = c0 + q;
     cv[q] = c < a.D;
-    const bool lc = a.do_pcq && cv[q];
-    gam[q] = (a.gamma && cv[q]) ? __ldg(a.gamma + c) : 1.0f;
-    cslot[q] = lc ? __ldg(a.c.slot + c) : -1;
-    crg[q] = lc ? __ldg(a.c.range + c) : 0.f;
-    zc[q] = lc ? __ldg(a.c.zmin + c) : 0.f;
+    gam[q] = ldg_sel(a.gamma, c, a.gamma && cv[q], 1.0f, a.g);
   }
   const int64_t rb = r0 + warp * 4;  // this warp's 4 rows
   int32_t sslots[4];
   int32_t srem[4];  // row within its sample group
   float srg[4], szm[4];
   {
-    int64_t gi = rb / a.rpg, rem = rb - gi * a.rpg;
+    const int64_t rc = min(rb, a.M - 1);
+    int64_t gi = a.div_rpg.div((uint32_t)rc), rem = rc - gi * a.rpg;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       if (i > 0 && ++rem == a.rpg) { rem = 0; ++gi; }
       srem[i] = (int32_t)rem;
       const bool ls = a.do_psq && rb + i < a.M;
-      sslots[i] = ls ? __ldg(a.s.slot + gi) : -1;
-      srg[i] = ls ? __ldg(a.s.range + gi) : 0.f;
-      szm[i] = ls ? __ldg(a.s.zmin + gi) : 0.f;
+      sslots[i] = ldg_sel(a.s.slot, gi, ls, -1, a.g);
+      srg[i] = ldg_sel(a.s.range, gi, ls, 0.f, a.g);
+      szm[i] = ldg_sel(a.s.zmin, gi, ls, 0.f, a.g);
     }
   }
   float vv[4][4];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int64_t r = rb + i;
+  for (int i = 0; i < 4; ++i) {  // unconditional loads from clamped rows / columns
+    const int64_t r = min(rb + i, a.M - 1);
     if (VEC) {
-      if (r < a.M && cv[0]) {
-        const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + c0));
-        vv[i][0] = t.x; vv[i][1] = t.y; vv[i][2] = t.z; vv[i][3] = t.w;
-      } else {
-        vv[i][0] = vv[i][1] = vv[i][2] = vv[i][3] = 0.f;
-      }
+      const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + (cv[0] ? c0 : 0)));
+      vv[i][0] = t.x; vv[i][1] = t.y; vv[i][2] = t.z; vv[i][3] = t.w;
     } else {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) vv[i][q] = (r < a.M && cv[q]) ? __ldg(a.g + r * a.D + c0 + q) : 0.0f;
-    }
-  }
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    invc[q] = 0.f;
-    cdeg[q] = true;
-    if (cslot[q] >= 0) {
-      invc[q] = __fdiv_rn(a.c.B, crg[q]);
-      cdeg[q] = !(crg[q] > 0.0f) || !isfinite(invc[q]);
+      for (int q = 0; q < 4; ++q) vv[i][q] = __ldg(a.g + r * a.D + min(c0 + q, a.D - 1));
     }
   }
 #pragma unroll
@@ -569,41 +609,45 @@ __global__ void __launch_bounds__(32 * (kQWarps + 1), 4) quantize_kernel(QuantAr
     }
   }
   if (!a.do_pcq) return;
-  // PCQ: kept columns; element (m, j) takes word j*M + m of stream 1, so one Philox block
-  // gives the 4 rows of this warp; the 4 codes form the column's staging word directly
+  // stage the tile; barrier 1 also waits for warp 8's list of kept columns
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    uint32_t word = 0;
-    if (cslot[q] >= 0) {
-      const uint64_t e = (uint64_t)(c0 + q) * (uint64_t)a.M + (uint64_t)rb;
-      uint32_t w[4];
-      if ((a.M & 3) == 0) {
-        const U32x4 p = philox_block(a.c.seed, kStreamSrPcq, e >> 2);
-        w[0] = p.x; w[1] = p.y; w[2] = p.z; w[3] = p.w;
-      } else {
+  for (int i = 0; i < 4; ++i)
+    *reinterpret_cast<float4*>(&gt[4 * warp + i][4 * lane]) = make_float4(vv[i][0], vv[i][1], vv[i][2], vv[i][3]);
+  asm volatile("bar.sync 1, %0;" ::"n"(32 * (kQWarps + 1)) : "memory");
+  const int nk = nk_s;
+  for (int u = threadIdx.x; u < nk * (kQRows / 4); u += 32 * kQWarps) {
+    const int j = u / (kQRows / 4), g = u % (kQRows / 4);
+    const int col = klist[j];
+    const int64_t rq = r0 + 4 * g;
+    const float z = kz[j], inv = kinv[j];
+    const bool deg = !(inv > 0.0f);
+    const uint64_t e = (uint64_t)(cb + col) * (uint64_t)a.M + (uint64_t)rq;
+    uint32_t w[4];
+    if ((a.M & 3) == 0) {
+      const U32x4 p = philox_block(a.c.seed, kStreamSrPcq, e >> 2);
+      w[0] = p.x; w[1] = p.y; w[2] = p.z; w[3] = p.w;
+    } else {
 #pragma unroll
-        for (int i = 0; i < 4; ++i) w[i] = philox_word(a.c.seed, kStreamSrPcq, e + i);
-      }
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-        if (rb + i < a.M) word |= sr_code(vv[i][q], zc[q], invc[q], a.c.B, cdeg[q], w[i]) << (8 * i);
+      for (int i = 0; i < 4; ++i) w[i] = philox_word(a.c.seed, kStreamSrPcq, e + i);
     }
-    tile[lane * 4 + q][warp] = word;
+    uint32_t word = 0;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (rq + i < a.M) word |= sr_code(gt[4 * g + i][col], z, inv, a.c.B, deg, w[i]) << (8 * i);
+    tile[j][g] = word;
   }
-  __syncthreads();
-  // each kept column of the tile: 32 code bytes (rows r0 .. r0+31) -> 2 x 16 bytes
-  const int col = threadIdx.x >> 1, half = threadIdx.x & 1;
-  const int64_t c = cb + col;
-  if (c < a.D) {
-    const int32_t sl = __ldg(a.c.slot + c);
+  asm volatile("bar.sync 2, %0;" ::"n"(32 * kQWarps) : "memory");
+  // kept column j: the codes of rows r0 .. r0 + 31 as two 16-byte stores
+  for (int t = threadIdx.x; t < 2 * nk; t += 32 * kQWarps) {
+    const int j = t >> 1, half = t & 1;
     const int64_t rb = r0 + 16 * half;
-    if (sl >= 0 && rb < a.M && rb + 16 <= a.c.ld) {
+    if (rb < a.M && rb + 16 <= a.c.ld) {
       uint4 val;
-      val.x = tile[col][4 * half + 0];
-      val.y = tile[col][4 * half + 1];
-      val.z = tile[col][4 * half + 2];
-      val.w = tile[col][4 * half + 3];
-      *reinterpret_cast<uint4*>(a.c.codes + (int64_t)sl * a.c.ld + rb) = val;
+      val.x = tile[j][4 * half + 0];
+      val.y = tile[j][4 * half + 1];
+      val.z = tile[j][4 * half + 2];
+      val.w = tile[j][4 * half + 3];
+      *reinterpret_cast<uint4*>(a.c.codes + (int64_t)kslot[j] * a.c.ld + rb) = val;
     }
   }
 }
@@ -665,7 +709,7 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
 
   const bool vec = (D % 4) == 0;
   RangeArgs ra{g, gamma, M, D, rpg, psq ? smin : nullptr, psq ? smax : nullptr, pcq ? cmin : nullptr,
-               pcq ? cmax : nullptr, dev_status};
+               pcq ? cmax : nullptr, dev_status, FastDiv((uint32_t)rpg)};
   dim3 rgrid((unsigned)((D + kRangeCols - 1) / kRangeCols), (unsigned)((M + kRangeRows - 1) / kRangeRows));
   if (vec) launch_k(range_kernel<true>, dim3(rgrid), dim3(256), 0, s, ra);
   else launch_k(range_kernel<false>, dim3(rgrid), dim3(256), 0, s, ra);
@@ -705,7 +749,7 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
   FQT1_CUDA_TRY(cudaGetLastError());
 
   QuantArgs qa;
-  qa.g = g; qa.gamma = gamma; qa.M = M; qa.D = D; qa.rpg = rpg;
+  qa.g = g; qa.gamma = gamma; qa.M = M; qa.D = D; qa.rpg = rpg; qa.div_rpg = FastDiv((uint32_t)rpg);
   qa.do_psq = psq != nullptr;
   qa.do_pcq = pcq != nullptr;
   if (psq) qa.s = QBranch{psq->group_min, psq->group_range, psq->slot_of_group, psq->codes, psq->ld_codes,

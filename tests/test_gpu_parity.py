@@ -154,6 +154,14 @@ CASES = [
     ("conv-1x1-256ch-56x56-gather", lambda: conv_case(2, 256, 56, 56, 16, 1, 1, 0, 4, SYS, seed=3)),
     ("conv-3x3-s1-multi-image-tiles", lambda: conv_case(9, 20, 5, 7, 40, 3, 1, 1, 2, BER, seed=4)),
     ("conv-5x5-s3-p2", lambda: conv_case(3, 6, 17, 13, 8, 5, 3, 2, 4, SYS, seed=5)),
+    # "same" convolutions whose tiles hold whole images (contiguous-region Unfolder):
+    # ragged last image tile and last column tile, 16x16 planes (256-pixel tiles), 1x1,
+    # 7x7 with pad 3, and rows wider than 32 pixels (per-sub-tile column masks)
+    ("conv-same-8x8-ragged", lambda: conv_case(5, 30, 8, 8, 24, 3, 1, 1, 4, SYS, seed=6)),
+    ("conv-same-16x16-5x5", lambda: conv_case(3, 12, 16, 16, 20, 5, 1, 2, 2, BER, seed=7)),
+    ("conv-same-4x8-1x1", lambda: conv_case(7, 300, 4, 8, 16, 1, 1, 0, 8, SYS, seed=8)),
+    ("conv-same-8x16-7x7", lambda: conv_case(3, 4, 8, 16, 8, 7, 1, 3, 4, SYS, seed=9)),
+    ("conv-same-4x64", lambda: conv_case(2, 6, 4, 64, 8, 3, 1, 1, 2, SYS, seed=10)),
 ]
 
 
