@@ -209,6 +209,62 @@ __device__ __forceinline__ uint32_t warp_transpose32(uint32_t x, int lane) {
   return x;
 }
 
+// Dense sign-pack through shared memory, for rows of a multiple of 4 floats: a CTA loads a
+// 32-row x 128-column tile with coalesced 16-byte loads (8 per thread, all in flight), lane l
+// of warp w forms the column word of column 32 w + l from shared memory, the warp transpose
+// gives the row words, and the row words leave as 16-byte stores.
+constexpr int kPackTileWarps = 4;
+
+__global__ void __launch_bounds__(32 * kPackTileWarps) pack_tile_kernel(
+    const float* __restrict__ x, int64_t rows, int64_t cols, int64_t ld, uint32_t* __restrict__ row_bits,
+    int64_t row_words, uint32_t* __restrict__ col_bits, int64_t col_words, int32_t* __restrict__ colsum) {
+  constexpr int NW = kPackTileWarps, TC = 32 * NW, F4 = TC / 4;
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  __shared__ __align__(16) float t[32][TC];
+  __shared__ __align__(16) uint32_t rws[32][NW];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t r0 = (int64_t)blockIdx.y * 32, cb = (int64_t)blockIdx.x * TC;
+  float4 v[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {  // unconditional loads from clamped positions, masked below
+    const int idx = threadIdx.x + 32 * NW * k, r = idx / F4, c4 = idx % F4;
+    v[k] = __ldg(reinterpret_cast<const float4*>(x + min(r0 + r, rows - 1) * ld + min(cb + 4 * c4, cols - 4)));
+  }
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const int idx = threadIdx.x + 32 * NW * k, r = idx / F4, c4 = idx % F4;
+    const int64_t c = cb + 4 * c4;
+    float4 w = v[k];
+    if (r0 + r >= rows) w = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (c + 0 >= cols) w.x = 0.f;
+    if (c + 1 >= cols) w.y = 0.f;
+    if (c + 2 >= cols) w.z = 0.f;
+    if (c + 3 >= cols) w.w = 0.f;
+    *reinterpret_cast<float4*>(&t[r][4 * c4]) = w;
+  }
+  __syncthreads();
+  const int cl = 32 * warp + lane;
+  uint32_t cw = 0;
+#pragma unroll
+  for (int r = 0; r < 32; ++r) cw |= (t[r][cl] > 0.0f ? 1u : 0u) << r;
+  rws[lane][warp] = warp_transpose32(cw, lane);
+  const int64_t c = cb + cl;
+  if (c < cols) {
+    if (col_bits) col_bits[c * col_words + blockIdx.y] = cw;
+    if (colsum) atomicAdd(colsum + c, 2 * __popc(cw) - (int)min((int64_t)32, rows - r0));
+  }
+  __syncthreads();
+  if (row_bits) {  // row r: words cb / 32 .. + NW - 1
+    for (int e = threadIdx.x; e < 32 * (NW / 4); e += 32 * NW) {
+      const int r = e / (NW / 4), h = e % (NW / 4);
+      const int64_t w0 = cb / 32 + 4 * h;
+      if (r0 + r < rows && w0 < row_words)
+        *reinterpret_cast<uint4*>(row_bits + (r0 + r) * row_words + w0) = *reinterpret_cast<const uint4*>(&rws[r][4 * h]);
+    }
+  }
+}
+
 // cnt (1..32) bits of a stream starting at bit pos; the guard words keep both reads inside.
 __device__ __forceinline__ uint32_t stream_bits(const uint32_t* st, int pos, int cnt) {
   const int w = pos >> 5, o = pos & 31;
@@ -603,8 +659,14 @@ extern "C" fqt1_status fqt1_binarize_pack(const float* x, int64_t rows, int64_t 
   const int64_t bands = (rows + 31) / 32;
   if (bands > 65535) return FQT1_ERR_UNSUPPORTED;
   if (colsum) FQT1_CUDA_TRY(cudaMemsetAsync(colsum, 0, sizeof(int32_t) * cols, s));
-  FQT1_CUDA_TRY(launch_k(pack_dense_kernel, dim3((unsigned)((row_words + 3) / 4), (unsigned)bands), dim3(128), 0, s,
-                         x, rows, cols, ld, row_bits, row_words, col_bits, col_words, colsum));
+  if (cols % 4 == 0 && ld % 4 == 0)
+    FQT1_CUDA_TRY(launch_k(pack_tile_kernel, dim3((unsigned)((cols + 32 * kPackTileWarps - 1) / (32 * kPackTileWarps)),
+                                                  (unsigned)bands),
+                           dim3(32 * kPackTileWarps), 0, s, x, rows, cols, ld, row_bits, row_words, col_bits, col_words,
+                           colsum));
+  else
+    FQT1_CUDA_TRY(launch_k(pack_dense_kernel, dim3((unsigned)((row_words + 3) / 4), (unsigned)bands), dim3(128), 0,
+                           s, x, rows, cols, ld, row_bits, row_words, col_bits, col_words, colsum));
   fqt1_count_launches(1);
   if (col_bits && col_words > bands) {
     const int64_t n = cols * (col_words - bands);

@@ -289,3 +289,27 @@ def test_nonfinite_gradient_sets_status():
     st.backward()
     torch.cuda.synchronize()
     assert int(st.dev_status[0].item()) & 0x100
+
+
+@pytest.mark.parametrize("rows,cols,ld", [(77, 300, 304), (40, 128, 132), (3, 4, 8), (64, 256, 256), (33, 100, 103),
+                                          (70, 45, 45)])
+def test_binarize_pack_strided(rows, cols, ld):
+    """Row bits, column bits and column sums of sign(x) for a strided [rows, cols] view (Sec. 5.1):
+    rows of a multiple of 4 floats take the shared-memory tile path, the others the per-warp path."""
+    from paper_2408_14267_gb300 import fqt1
+    rng = np.random.default_rng(rows * 1000 + cols)
+    full = rng.standard_normal((rows, ld)).astype(np.float32)
+    full[:, :cols][rng.random((rows, cols)) < 0.05] = 0.0
+    x = full[:, :cols]
+    dev = torch.from_numpy(full).cuda()
+    rw, cw = fqt1.packed_words(cols), fqt1.packed_words(rows)
+    row_bits = torch.full((rows, rw), -1, dtype=torch.int32, device="cuda")
+    col_bits = torch.full((cols, cw), -1, dtype=torch.int32, device="cuda")
+    colsum = torch.full((cols,), 12345, dtype=torch.int32, device="cuda")
+    fqt1.binarize_pack(dev, rows, cols, ld, row_bits, col_bits, colsum)
+    torch.cuda.synchronize()
+    s, pad = unpack_bits(row_bits, cols)
+    assert np.array_equal(s, om.sign(x)) and not pad.any()
+    sc, pad = unpack_bits(col_bits, rows)
+    assert np.array_equal(sc, om.sign(x).T) and not pad.any()
+    assert np.array_equal(colsum.cpu().numpy(), om.colsum_sign(x))
