@@ -544,15 +544,34 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     float* const f_scale = reinterpret_cast<float*>(f_cs + f_nc * f_khw);
     float* const f_zero = f_scale + f_imgs;
     int32_t* const f_n = reinterpret_cast<int32_t*>(f_zero + f_imgs);
+    bool fold_zero_issued = false;  // bulk stores of zeros in flight (read from shared memory)
     if (SHORT && a.epi == EPI_FOLD) {
       const int tt = threadIdx.x - 64;
-      if (tt < f_nc * f_khw) f_cs[tt] = __ldg(a.cs + (int64_t)f_c0 * f_khw + tt);  // nc * khw <= 128
-      const int64_t slot0 = (int64_t)blockIdx.y * f_imgs, nslots = __ldg(a.count);  // rpg divides 128
+      // every global load of the tables (column sums, kept count, kept ids, scales, zero
+      // points, and the kept flags of this thread's first zeroing pieces below) is issued
+      // together from clamped indices; the results are selected afterwards
+      const int ncs = f_nc * f_khw;  // <= 128
+      const int32_t cs_v = __ldg(a.cs + (int64_t)f_c0 * f_khw + min(tt, ncs - 1));
+      const int64_t slot0 = (int64_t)blockIdx.y * f_imgs, cap = a.M / a.rpg;  // rpg divides 128
+      const int64_t slot = min(slot0 + min(tt, f_imgs - 1), cap - 1);
+      const int64_t nslots = __ldg(a.count);
+      const int32_t kid = __ldg(a.kept_idx + slot);
+      const float ksc = __ldg(a.scale + slot), kze = __ldg(a.zero + slot);
+      const int nsamp = a.fN > (int)blockIdx.y ? (a.fN - (int)blockIdx.y + (int)gridDim.y - 1) / (int)gridDim.y : 0;
+      const int64_t blk_bytes = (int64_t)f_nc * f_HW * 4;
+      const int pieces = (int)((blk_bytes + kFoldZero - 1) / kFoldZero);
+      int32_t sl[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int k = nsamp > 0 ? min(tt + 256 * u, nsamp * pieces - 1) / pieces : 0;
+        sl[u] = __ldg(a.slot_of_group + min((int64_t)blockIdx.y + (int64_t)k * gridDim.y, (int64_t)a.fN - 1));
+      }
+      if (tt < ncs) f_cs[tt] = cs_v;
       if (tt < f_imgs) {
-        const int64_t slot = slot0 + tt;
-        f_n[tt] = slot < nslots ? __ldg(a.kept_idx + slot) : -1;
-        f_scale[tt] = slot < nslots ? __ldg(a.scale + slot) : 0.f;
-        f_zero[tt] = slot < nslots ? __ldg(a.zero + slot) : 0.f;
+        const bool kept = slot0 + tt < nslots;
+        f_n[tt] = kept ? kid : -1;
+        f_scale[tt] = kept ? ksc : 0.f;
+        f_zero[tt] = kept ? kze : 0.f;
       }
       asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
       for (int x = tt; x < f_nc * f_HW; x += 256) {
@@ -569,6 +588,44 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
             if (f_tap[pos * f_khw + t] >= 0) cs += f_cs[cl * f_khw + t];
         }
         f_csf[x] = cs;
+      }
+      // pruned samples (they do not depend on the products, so before the accumulator is
+      // ready): this CTA zeroes its channel block (nc HW contiguous floats) of samples
+      // blockIdx.y, + gridDim.y, ...: bulk stores from a zero buffer, one thread per 4 KB piece;
+      // the kept flags of a thread's pieces are loaded together first
+      if (f_HW % 4 == 0) {
+        const unsigned char* zb = base + S::kMain + kFoldTab - kFoldZero;
+        for (int e0 = tt; e0 < nsamp * pieces; e0 += 4 * 256) {
+          if (e0 != tt) {  // later pieces (the first ones' flags were loaded with the tables)
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const int k = min(e0 + 256 * u, nsamp * pieces - 1) / pieces;
+              sl[u] = __ldg(a.slot_of_group + (int64_t)blockIdx.y + (int64_t)k * gridDim.y);
+            }
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int e = e0 + 256 * u;
+            if (e >= nsamp * pieces || sl[u] >= 0) continue;
+            const int k = e / pieces, pc = e - k * pieces;
+            const int64_t n = (int64_t)blockIdx.y + (int64_t)k * gridDim.y;
+            unsigned char* dst = reinterpret_cast<unsigned char*>(a.y + ((int64_t)n * a.fC + f_c0) * f_HW) +
+                                 (int64_t)pc * kFoldZero;
+            const int64_t left = blk_bytes - (int64_t)pc * kFoldZero;
+            bulk_store(dst, zb, (uint32_t)(left < kFoldZero ? left : kFoldZero));
+            fold_zero_issued = true;
+          }
+        }
+        if (fold_zero_issued) asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+      } else {
+        const int per_img = a.fcb * f_HW;
+        for (int e = tt; e < nsamp * per_img; e += 256) {
+          const int k = (int)a.fd_cbhw.div((uint32_t)e), x = e - k * per_img;
+          if (x >= f_nc * f_HW) continue;
+          const int64_t n = (int64_t)blockIdx.y + (int64_t)k * gridDim.y;
+          if (__ldg(a.slot_of_group + n) >= 0) continue;
+          a.y[((int64_t)n * a.fC + f_c0) * f_HW + x] = 0.f;
+        }
       }
     }
     if (a.tma_out & 1) {  // Gamma of this tile's columns, before the accumulator is ready
@@ -648,37 +705,8 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         a.y[((int64_t)n * a.fC + c_first + cl) * HW + pos] =
             __fadd_rn(__fmul_rn(s_scale[img], (float)acc), __fmul_rn(s_zero[img], (float)csf[rem]));
       }
-      // pruned samples: this CTA zeroes its channel block (nc HW contiguous floats) of samples
-      // blockIdx.y, + gridDim.y, ...: bulk stores from a zero buffer, one thread per 4 KB piece
-      const int nsamp = a.fN > (int)blockIdx.y ? (a.fN - (int)blockIdx.y + (int)gridDim.y - 1) / (int)gridDim.y : 0;
-      const int64_t blk_bytes = (int64_t)nc * HW * 4;
-      if (HW % 4 == 0) {
-        const int pieces = (int)((blk_bytes + kFoldZero - 1) / kFoldZero);
-        const unsigned char* zb = base + S::kMain + kFoldTab - kFoldZero;
-        bool issued = false;
-        for (int e = tt; e < nsamp * pieces; e += 256) {
-          const int k = e / pieces, pc = e - k * pieces;
-          const int64_t n = (int64_t)blockIdx.y + (int64_t)k * gridDim.y;
-          if (__ldg(a.slot_of_group + n) >= 0) continue;
-          unsigned char* dst = reinterpret_cast<unsigned char*>(a.y + ((int64_t)n * a.fC + c_first) * HW) +
-                               (int64_t)pc * kFoldZero;
-          const int64_t left = blk_bytes - (int64_t)pc * kFoldZero;
-          bulk_store(dst, zb, (uint32_t)(left < kFoldZero ? left : kFoldZero));
-          issued = true;
-        }
-        if (issued) {
-          asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-          asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
-        }
-      } else {
-        for (int e = tt; e < nsamp * per_img; e += 256) {
-          const int k = (int)a.fd_cbhw.div((uint32_t)e), x = e - k * per_img;
-          if (x >= nc * HW) continue;
-          const int64_t n = (int64_t)blockIdx.y + (int64_t)k * gridDim.y;
-          if (__ldg(a.slot_of_group + n) >= 0) continue;
-          a.y[((int64_t)n * a.fC + c_first) * HW + x] = 0.f;
-        }
-      }
+      // the bulk stores of zeros must have read the zero buffer before the CTA exits
+      if (fold_zero_issued) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
     } else {
     const int q = warp & 3;                         // TMEM lane quarter of this warp
     const int cbeg = ((warp - 2) >> 2) * (BN / 2);  // its half of the accumulator columns
@@ -838,17 +866,54 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   __syncwarp();
   if (a.epi == EPI_CRED) {
     // every CTA of the cluster reaches both barriers, also after an expired wait
-    cluster_sync_all();
     const uint32_t rank = cluster_rank(), nr = cluster_size();
+    const bool vec = (a.ldo % 4) == 0;
+    if (blockIdx.y == 0) {
+      // pruned channels (independent of the products, so before the cluster barrier): zero
+      // rows of dw over this tile's columns, shared by the cluster; the slots of a thread's
+      // next 4 elements are loaded together first
+      const int64_t step = (int64_t)nr * kThreads;
+      for (int64_t e0 = (int64_t)rank * kThreads + threadIdx.x; e0 < a.D * 32; e0 += 4 * step) {
+        int32_t sl[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) sl[u] = __ldg(a.slot_of_group + (min(e0 + u * step, a.D * 32 - 1) >> 5));
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int64_t e = e0 + u * step;
+          const int64_t j = e >> 5, n = n0 + 4 * (e & 31);
+          if (e >= a.D * 32 || n >= a.N || sl[u] >= 0) continue;
+          float* wrow = a.y + j * a.ldo + n;
+          if (vec && n + 4 <= a.N) *reinterpret_cast<float4*>(wrow) = make_float4(0.f, 0.f, 0.f, 0.f);
+          else for (int t = 0; t < 4 && n + t < a.N; ++t) wrow[t] = 0.f;
+        }
+      }
+    }
     // the tile rows that exist (up to the capacity) are divided over the cluster's CTAs
     const int64_t rows_here = a.M - m0;
     const int nrows = rows_here >= kBM ? kBM : (rows_here <= 0 ? 0 : (int)rows_here);
     const int rpr = (nrows + (int)nr - 1) / (int)nr;  // tile rows summed by each CTA
     const int r_lo = min(nrows, (int)rank * rpr), r_hi = min(nrows, r_lo + rpr);
+    const int nel = (r_hi - r_lo) * 32;
+    // the row and column inputs of the dequantization (kept channel, S', Z', column sums of
+    // sign(X)) of a chunk, loaded together from clamped indices; the first chunk's before
+    // the cluster barrier
+    int64_t kj = 0;
+    float ksc = 0.f, kze = 0.f;
+    int32_t kcs[4] = {0, 0, 0, 0};
+    auto chunk_inputs = [&](int e) {
+      const int64_t grow = min(m0 + r_lo + (e >> 5), a.M - 1), n = n0 + 4 * (e & 31);
+      kj = __ldg(a.kept_idx + grow);
+      ksc = __ldg(a.scale + grow);
+      kze = __ldg(a.zero + grow);
+#pragma unroll
+      for (int t = 0; t < 4; ++t) kcs[t] = __ldg(a.cs + min(n + t, a.N - 1));
+    };
+    if ((int)threadIdx.x < nel) chunk_inputs(threadIdx.x);
+    cluster_sync_all();
     const uint32_t pbase = smem_u32(base);
     const bool ok = !abort_flag;
-    const bool vec = (a.ldo % 4) == 0;
-    for (int e = threadIdx.x; e < (r_hi - r_lo) * 32; e += kThreads) {
+    for (int e = threadIdx.x; e < nel; e += kThreads) {
+      if (e != (int)threadIdx.x) chunk_inputs(e);
       const int r = r_lo + (e >> 5), ch = e & 31;
       const int64_t grow = m0 + r, n = n0 + 4 * ch;
       if (grow >= a.M || n >= a.N) continue;
@@ -869,25 +934,13 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       if (vec && n + 4 <= a.N) *reinterpret_cast<int4*>(arow) = sum;
       else for (int t = 0; t < 4 && n + t < a.N; ++t) arow[t] = sv[t];
       if (kept) {
-        const int64_t j = __ldg(a.kept_idx + grow);
-        const float sc = __ldg(a.scale + grow), ze = __ldg(a.zero + grow);
-        float* wrow = a.y + j * a.ldo + n;
+        float* wrow = a.y + kj * a.ldo + n;
         float o[4];
 #pragma unroll
         for (int t = 0; t < 4; ++t)
-          o[t] = n + t < a.N ? __fadd_rn(__fmul_rn(sc, (float)sv[t]), __fmul_rn(ze, (float)__ldg(a.cs + n + t))) : 0.f;
+          o[t] = n + t < a.N ? __fadd_rn(__fmul_rn(ksc, (float)sv[t]), __fmul_rn(kze, (float)kcs[t])) : 0.f;
         if (vec && n + 4 <= a.N) *reinterpret_cast<float4*>(wrow) = make_float4(o[0], o[1], o[2], o[3]);
         else for (int t = 0; t < 4 && n + t < a.N; ++t) wrow[t] = o[t];
-      }
-    }
-    if (blockIdx.y == 0) {
-      // pruned channels: zero rows of dw over this tile's columns, shared by the cluster
-      for (int64_t e = (int64_t)rank * kThreads + threadIdx.x; e < a.D * 32; e += (int64_t)nr * kThreads) {
-        const int64_t j = e >> 5, n = n0 + 4 * (e & 31);
-        if (n >= a.N || __ldg(a.slot_of_group + j) >= 0) continue;
-        float* wrow = a.y + j * a.ldo + n;
-        if (vec && n + 4 <= a.N) *reinterpret_cast<float4*>(wrow) = make_float4(0.f, 0.f, 0.f, 0.f);
-        else for (int t = 0; t < 4 && n + t < a.N; ++t) wrow[t] = 0.f;
       }
     }
     cluster_sync_all();  // no CTA leaves while another still reads its tile

@@ -191,8 +191,10 @@ __device__ __forceinline__ double p_hat_of(uint64_t P) {
 // NT threads per CTA (256 when every grouping has at most 256 groups, else 1024).
 template <int NT>
 __global__ void __launch_bounds__(NT) select_kernel(SelectArgs a0, SelectArgs a1) {
+  // The dependents (the quantize grid, one CTA per tile of G) are released only when this
+  // kernel ends: launched early they would occupy every SM in their dependency wait while
+  // these two CTAs run, keeping the other branches' kernels off the GPU.
   FQT1_PDL_WAIT();
-  FQT1_PDL_TRIGGER();
   const SelectArgs& a = blockIdx.x == 0 ? a0 : a1;
   extern __shared__ __align__(16) unsigned char sel_smem[];
   __shared__ uint64_t warp_sums[32];
@@ -487,8 +489,10 @@ struct QuantArgs {
 //    waiting), then computes the per-slot S' and Z' in float64 beside the quantizing warps.
 template <bool VEC>
 __global__ void __launch_bounds__(32 * (kQWarps + 1), 4) quantize_kernel(QuantArgs a) {
+  // the dependent (the grad_input product, a leaf of the step) is not released early either:
+  // its CTAs would wait on SMs that the grad_weight product, which also waits for this
+  // kernel, can use
   FQT1_PDL_WAIT();
-  FQT1_PDL_TRIGGER();
   __shared__ __align__(16) float gt[kQRows][kQCols + 4];  // the tile of G * gamma
   __shared__ uint32_t tile[kQCols][kQRows / 4 + 1];       // codes of kept column j, 4 rows per word
   __shared__ int32_t klist[kQCols], kslot[kQCols];        // kept column j: tile column, slot
