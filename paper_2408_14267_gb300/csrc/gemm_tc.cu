@@ -319,7 +319,10 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     return;
   }
 
-  unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // 1024-byte aligned start of the dynamic shared memory, derived from smem_raw by an offset
+  // (not by a round trip through an integer) so that accesses through it stay shared-memory
+  // accesses instead of generic ones
+  unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   auto opB = [&](int s) { return base + s * S::kOpB; };
   unsigned char* raw_base = base + OS * S::kOpB;
   auto rawA = [&](int s) { return raw_base + s * S::kRawStage; };
@@ -574,7 +577,22 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         f_zero[tt] = kept ? kze : 0.f;
       }
       asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
-      for (int x = tt; x < f_nc * f_HW; x += 256) {
+      if (fold_same3(a) && 256 % f_HW == 0) {
+        // one input position per thread (H W divides 256): its 9-tap validity mask once
+        const int pos = tt & (f_HW - 1);
+        const int h = (int)a.fd_w.div((uint32_t)pos), w = pos - h * a.fW;
+        uint32_t msk = 0;
+#pragma unroll
+        for (int t = 0; t < 9; ++t)
+          if ((unsigned)(h + 1 - t / 3) < (unsigned)a.fH && (unsigned)(w + 1 - t % 3) < (unsigned)a.fW) msk |= 1u << t;
+        for (int cl = tt / f_HW; cl < f_nc; cl += 256 / f_HW) {
+          int32_t cs = 0;
+#pragma unroll
+          for (int t = 0; t < 9; ++t) cs += (msk >> t) & 1u ? f_cs[cl * 9 + t] : 0;
+          f_csf[cl * f_HW + pos] = cs;
+        }
+      }
+      for (int x = tt; !(fold_same3(a) && 256 % f_HW == 0) && x < f_nc * f_HW; x += 256) {
         const int cl = (int)a.fd_hw.div((uint32_t)x), pos = x - cl * f_HW;
         int32_t cs = 0;
         if (fold_same3(a)) {  // tap (i, j) of input (h, w) lands on output (h + 1 - i, w + 1 - j)
@@ -669,8 +687,42 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
       // Folder: dx[n, c, h, w] = S'_n sum(acc taps) + Z'_n sum(colsum taps); entries of fcb
       // channels per sample (a last, narrower channel block skips the missing ones)
+      const bool fixed_pos = fold_same3(a) && 256 % HW == 0;
+      if (fixed_pos && have_acc) {
+        // 3 x 3, stride 1, pad 1 with H W dividing 256: one input position per thread, its tap
+        // offsets (tile row pos + (1 - i) W + (1 - j), column 3 i + j) and validity computed
+        // once; the 9 shared loads of an output are independent (a tap outside reads offset 0
+        // and is masked)
+        const int pos = tt & (HW - 1);
+        const int h = (int)a.fd_w.div((uint32_t)pos), w = pos - h * a.fW;
+        int off[9];
+        uint32_t msk = 0;
+#pragma unroll
+        for (int t = 0; t < 9; ++t) {
+          const int di = 1 - t / 3, dj = 1 - t % 3;
+          const bool v = (unsigned)(h + di) < (unsigned)a.fH && (unsigned)(w + dj) < (unsigned)a.fW;
+          off[t] = v ? (di * a.fW + dj) * TS + t : 0;
+          msk |= v ? 1u << t : 0u;
+        }
+        for (int img = 0; img < imgs; ++img) {
+          const int n = s_n[img];
+          if (n < 0) break;
+          const float sc = s_scale[img], ze = s_zero[img];
+          for (int cl = tt / HW; cl < nc; cl += 256 / HW) {
+            const int32_t* tp = T + (img * rpg + pos) * TS + cl * 9;
+            int32_t v[9];
+#pragma unroll
+            for (int t = 0; t < 9; ++t) v[t] = tp[off[t]];
+            int32_t acc = 0;
+#pragma unroll
+            for (int t = 0; t < 9; ++t) acc += (msk >> t) & 1u ? v[t] : 0;
+            a.y[((int64_t)n * a.fC + c_first + cl) * HW + pos] =
+                __fadd_rn(__fmul_rn(sc, (float)acc), __fmul_rn(ze, (float)csf[cl * HW + pos]));
+          }
+        }
+      }
       const int per_img = a.fcb * HW;
-      for (int e = tt; have_acc && e < imgs * per_img; e += 256) {
+      for (int e = tt; !fixed_pos && have_acc && e < imgs * per_img; e += 256) {
         const int img = (int)a.fd_cbhw.div((uint32_t)e), rem = e - img * per_img;
         const int n = s_n[img];
         if (n < 0) break;
