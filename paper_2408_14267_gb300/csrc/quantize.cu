@@ -161,19 +161,20 @@ __device__ uint64_t block_inclusive_scan(uint64_t v, uint64_t* warp_sums, uint64
 }
 
 // floor(a * 2^32 / d) for 0 < d < 2^62, a < 2^60 (exact; quotients of 2^34 or more return ~0,
-// the callers clamp at 2^32).  An fp32 estimate (relative error below 2^-22) is corrected with
-// exact 128-bit remainders; float64 is avoided (its division is slow on this part).
+// the callers clamp at 2^32).  An fp32 estimate (relative error below 2^-20) is corrected with
+// exact 128-bit remainders; float64 is avoided (its division is slow on this part).  The float
+// quotients are the fast approximate ones: the integer steps after them make the result exact.
 __device__ __forceinline__ uint64_t div_shift32(uint64_t a, uint64_t d) {
   typedef unsigned __int128 u128;
   const u128 num = (u128)a << 32;
   if ((num >> 34) >= d) return ~0ull;
-  uint64_t q = (uint64_t)__fdiv_rn(__ull2float_rn(a), __fmul_rn(__ull2float_rn(d), 2.3283064365386963e-10f));
-  // |q - quotient| < 2^13: one float step on the remainder, scaled so that d keeps 24 bits
+  uint64_t q = (uint64_t)__fdividef(__ull2float_rn(a), __fmul_rn(__ull2float_rn(d), 2.3283064365386963e-10f));
+  // |q - quotient| < 2^15: one float step on the remainder, scaled so that d keeps 24 bits
   const int sh = max(0, 40 - __clzll(d));
   const float df = __ull2float_rn(d >> sh);
   const u128 qd = (u128)q * d;
-  if (qd > num) q -= (uint64_t)__fdiv_rn(__ull2float_rn((uint64_t)((qd - num) >> sh)), df);
-  else q += (uint64_t)__fdiv_rn(__ull2float_rn((uint64_t)((num - qd) >> sh)), df);
+  if (qd > num) q -= (uint64_t)__fdividef(__ull2float_rn((uint64_t)((qd - num) >> sh)), df);
+  else q += (uint64_t)__fdividef(__ull2float_rn((uint64_t)((num - qd) >> sh)), df);
   while ((u128)q * d > num) --q;
   while ((u128)(q + 1) * d <= num) ++q;
   return q;
