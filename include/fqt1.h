@@ -131,6 +131,33 @@ fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t H, int32_t
 fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D, int64_t K,
                           const float* gamma, int32_t* acc, float* y, void* stream);
 
+/* fqt1_fwd_gemm with a per-channel bias: y[m, j] = gamma[j] * acc[m, j] + bias[j]
+ * (fp32 multiply, then fp32 add).  The paper's layer (Sec. 5.1) has the scale
+ * Gamma only; the bias is the usual extension of a linear or convolution layer
+ * (Algorithm 1 omits it).  bias: [D] fp32, 16-byte aligned, or NULL (then the
+ * call equals fqt1_fwd_gemm); a bias needs y. */
+fqt1_status fqt1_fwd_gemm_bias(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D, int64_t K,
+                               const float* gamma, const float* bias, int32_t* acc, float* y, void* stream);
+
+/* ------------------------------------------------ layer parameters and STE */
+/* Gradients of the layer's scale Gamma (Sec. 5.1: y = (sign(X) sign(W)^T) (.)
+ * Gamma, Gamma learnable) and of its bias:
+ *   dgamma[j] = sum_m gy[m, j] acc[m, j],   dbias[j] = sum_m gy[m, j].
+ * gy: [M][D] fp32 (the gradient of y); acc: [M][D] int32, the forward
+ * accumulators (fqt1_fwd_gemm's acc), needed for dgamma; dgamma, dbias: [D]
+ * fp32, either may be NULL, overwritten.  The sums run in a fixed order (fp32
+ * over 64-row chunks, fp64 over the chunks), so the results are reproducible.
+ * ws: fqt1_scale_bias_workspace(M, D) bytes, 16-byte aligned, caller-owned. */
+size_t fqt1_scale_bias_workspace(int64_t M, int64_t D);
+fqt1_status fqt1_scale_bias_grad(const float* gy, const int32_t* acc, int64_t M, int64_t D, float* dgamma,
+                                 float* dbias, void* ws, size_t ws_bytes, void* stream);
+
+/* Clipped straight-through estimator of sign() (the STE cited in Sec. 3.1):
+ * dx[i] = dx[i] if |x[i]| <= t else 0, in place, for i < n.  Without this call
+ * the gradient passes sign() unchanged (the identity STE).  x, dx: [n] fp32,
+ * 16-byte aligned; t >= 0 (NaN x gives 0). */
+fqt1_status fqt1_ste_clip(const float* x, float* dx, int64_t n, float t, void* stream);
+
 /* ----------------------------------------------------------- gradient side */
 /* AGP on one grouping (Sec. 5.2): ranges of G = gy (.) gamma (gamma may be
  * NULL), keep probabilities, masks, and stochastic rounding of the kept

@@ -42,6 +42,11 @@ R5  stochastic rounding in fp32: inv = B / R, t = (x - Z) * inv, q = floor(t)
     enters the scale S' = R / (B p^) and zero point Z' = Z / p^.
 R6  dequantization is fp32: a = S' * float(acc), c = Z' * float(colsum),
     out = a + c; pruned rows / channels are exactly 0.
+R10 a layer may add a per-channel bias after the scale (y = Gamma * acc + bias,
+    fp32 multiply then add); the gradients of Gamma and of the bias are the
+    exact sums over the rows of gY * acc and gY (float64 here).  The
+    straight-through estimator of sign() is the identity; its clipped form
+    keeps the gradient where |x| <= t.
 """
 import numpy as np
 
@@ -84,6 +89,30 @@ def forward(x_u, w, gamma):
         return acc, acc.astype(f32)
     y = (np.asarray(gamma, dtype=f32)[None, :] * acc.astype(f32)).astype(f32)
     return acc, y
+
+
+def forward_bias(x_u, w, gamma, bias):
+    """Forward of Sec. 5.1 with a per-channel bias after the scale (reading R10):
+    y = fp32(Gamma * acc) + bias, both operations rounded to fp32."""
+    acc, y = forward(x_u, w, gamma)
+    if bias is None:
+        return acc, y
+    return acc, (y + np.asarray(bias, dtype=f32)[None, :]).astype(f32)
+
+
+def scale_bias_grad(gy, acc):
+    """Gradients of the layer's learnable scale Gamma (Sec. 5.1, y = acc (.) Gamma) and of
+    its bias (reading R10): dGamma_j = sum_m gY[m, j] acc[m, j], dbias_j = sum_m gY[m, j],
+    in float64."""
+    g = np.asarray(gy, dtype=np.float64)
+    return (g * np.asarray(acc, dtype=np.float64)).sum(axis=0), g.sum(axis=0)
+
+
+def ste_clip(x, dx, t=1.0):
+    """Clipped straight-through estimator of sign() (reading R10): the gradient passes
+    where |x| <= t and is 0 elsewhere (also where x is NaN)."""
+    x = np.asarray(x)
+    return np.where(np.abs(x) <= t, dx, 0).astype(np.asarray(dx).dtype)
 
 
 def colsum_sign(a):

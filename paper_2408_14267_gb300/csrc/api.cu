@@ -241,19 +241,26 @@ using namespace fqt1;
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 static bool valid_bits(int b) { return b == 1 || b == 2 || b == 4 || b == 8; }
 
-extern "C" fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D,
-                                     int64_t K, const float* gamma, int32_t* acc, float* y, void* stream) {
-  if (!sx_row || !sw_row || M < 1 || D < 1 || K < 1 || (!acc && !y) || (y && !gamma)) return FQT1_ERR_INVALID_ARG;
+extern "C" fqt1_status fqt1_fwd_gemm_bias(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D,
+                                          int64_t K, const float* gamma, const float* bias, int32_t* acc, float* y,
+                                          void* stream) {
+  if (!sx_row || !sw_row || M < 1 || D < 1 || K < 1 || (!acc && !y) || (y && !gamma) || (bias && !y))
+    return FQT1_ERR_INVALID_ARG;
   if (!aligned16(sx_row) || !aligned16(sw_row) || (acc && !aligned16(acc)) || (y && !aligned16(y)) ||
-      (gamma && !aligned16(gamma)))
+      (gamma && !aligned16(gamma)) || (bias && !aligned16(bias)))
     return FQT1_ERR_MISALIGNED;
   if (K >= (1ll << 24) || (M + 63) / 64 > 65535) return FQT1_ERR_UNSUPPORTED;
   if (use_popcount_path() || !y) {
-    FQT1_CUDA_TRY(launch_xnor_gemm_simt(sx_row, sw_row, M, D, K, gamma, acc, y, (cudaStream_t)stream));
+    FQT1_CUDA_TRY(launch_xnor_gemm_simt(sx_row, sw_row, M, D, K, gamma, bias, acc, y, (cudaStream_t)stream));
   } else {
-    FQT1_CUDA_TRY(launch_fwd_tc(sx_row, sw_row, M, D, K, gamma, acc, y, nullptr, (cudaStream_t)stream));
+    FQT1_CUDA_TRY(launch_fwd_tc(sx_row, sw_row, M, D, K, gamma, bias, acc, y, nullptr, (cudaStream_t)stream));
   }
   return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D,
+                                     int64_t K, const float* gamma, int32_t* acc, float* y, void* stream) {
+  return fqt1_fwd_gemm_bias(sx_row, sw_row, M, D, K, gamma, nullptr, acc, y, stream);
 }
 
 extern "C" fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t* sw_col, const int32_t* colsum_w,

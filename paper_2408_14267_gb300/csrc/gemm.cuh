@@ -5,7 +5,7 @@
 namespace fqt1 {
 
 cudaError_t launch_xnor_gemm_simt(const uint32_t* A, const uint32_t* B, int64_t M, int64_t N, int64_t K,
-                                  const float* gamma, int32_t* acc, float* y, cudaStream_t s);
+                                  const float* gamma, const float* bias, int32_t* acc, float* y, cudaStream_t s);
 cudaError_t launch_codes_gemm_simt(int bits, const uint8_t* Q, int64_t ldq, const int32_t* count,
                                    int64_t rows_per_count, int64_t max_rows, const uint32_t* S, int64_t n_s,
                                    int64_t L, int32_t* out, int64_t ldo, cudaStream_t s);
@@ -13,7 +13,7 @@ cudaError_t launch_codes_gemm_simt(int bits, const uint8_t* Q, int64_t ldq, cons
 // tcgen05 path (gemm_tc.cu)
 struct TcArgs;
 cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64_t D, int64_t K, const float* gamma,
-                          int32_t* acc, float* y, int32_t* status, cudaStream_t s);
+                          const float* bias, int32_t* acc, float* y, int32_t* status, cudaStream_t s);
 cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
                                    int64_t rows_per_count, const uint32_t* Sg, int64_t n_s, int64_t L, int epi,
                                    int splits, int32_t* acc, float* out, int64_t ldo, const int32_t* kept_idx,

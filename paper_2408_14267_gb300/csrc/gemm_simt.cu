@@ -13,6 +13,7 @@ constexpr int kSW = 8;      // packed words per K step (256 elements)
 __global__ void __launch_bounds__(256) xnor_gemm_simt_kernel(const uint32_t* __restrict__ A,
                                                              const uint32_t* __restrict__ B, int64_t M, int64_t N,
                                                              int64_t K, int64_t ldw, const float* __restrict__ gamma,
+                                                             const float* __restrict__ bias,
                                                              int32_t* __restrict__ acc_out, float* __restrict__ y) {
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
@@ -50,7 +51,10 @@ __global__ void __launch_bounds__(256) xnor_gemm_simt_kernel(const uint32_t* __r
       if (n >= N) continue;
       const int32_t v = (int32_t)K - 2 * pc[i][j];
       if (acc_out) acc_out[m * N + n] = v;
-      if (y) y[m * N + n] = __fmul_rn(__ldg(gamma + n), __int2float_rn(v));
+      if (y) {
+        const float g = __fmul_rn(__ldg(gamma + n), __int2float_rn(v));
+        y[m * N + n] = bias ? __fadd_rn(g, __ldg(bias + n)) : g;
+      }
     }
   }
 }
@@ -125,10 +129,10 @@ __global__ void __launch_bounds__(256) codes_gemm_simt_kernel(const uint8_t* __r
 }
 
 cudaError_t launch_xnor_gemm_simt(const uint32_t* A, const uint32_t* B, int64_t M, int64_t N, int64_t K,
-                                  const float* gamma, int32_t* acc, float* y, cudaStream_t s) {
+                                  const float* gamma, const float* bias, int32_t* acc, float* y, cudaStream_t s) {
   const int64_t ldw = fqt1_packed_words(K);
   dim3 grid((unsigned)((N + kST - 1) / kST), (unsigned)((M + kST - 1) / kST));
-  launch_k(xnor_gemm_simt_kernel, dim3(grid), dim3(256), 0, s, A, B, M, N, K, ldw, gamma, acc, y);
+  launch_k(xnor_gemm_simt_kernel, dim3(grid), dim3(256), 0, s, A, B, M, N, K, ldw, gamma, bias, acc, y);
   fqt1_count_launches(1);
   return cudaGetLastError();
 }

@@ -48,7 +48,8 @@ struct TcArgs {
   int64_t rows_per_count;
   int k_tiles, tiles_per_split;
   int epi;
-  const float* gamma;        // EPI_FWD: y = gamma[n] * acc
+  const float* gamma;        // EPI_FWD: y = gamma[n] * acc (+ bias[n])
+  const float* bias;         // EPI_FWD: per-column bias or null
   float* y;
   int32_t* acc;              // EPI_FWD (optional), EPI_ACC32, EPI_RED
   int64_t ldo;
@@ -309,6 +310,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
   __shared__ __align__(16) float gamma_s[BN];  // EPI_FWD: Gamma of this tile's columns (read as float4)
+  __shared__ __align__(16) float bias_s[BN];   // EPI_FWD with a bias: the bias of those columns
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t m0 = (int64_t)blockIdx.y * kBM, n0 = (int64_t)blockIdx.x * (a.n_step > 0 ? a.n_step : BN);
@@ -649,6 +651,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     if (a.tma_out & 1) {  // Gamma of this tile's columns, before the accumulator is ready
       const int tt = threadIdx.x - 64;
       if (tt < BN) gamma_s[tt] = n0 + tt < a.N ? __ldg(a.gamma + n0 + tt) : 0.f;
+      if (a.bias && tt < BN) bias_s[tt] = n0 + tt < a.N ? __ldg(a.bias + n0 + tt) : 0.f;
       asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
     }
     const bool have_acc = mbar_wait(&acc_full, 0, &abort_flag, a.status);
@@ -810,8 +813,14 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
           const int off = lane * 32 + ((c ^ (lane & 7)) << 2);
           if (a.tma_out & 1) {
             const float4 g4 = *reinterpret_cast<const float4*>(gamma_s + c0 + 4 * c);
-            *reinterpret_cast<float4*>(sy + off) = make_float4(__fmul_rn(g4.x, (float)i0), __fmul_rn(g4.y, (float)i1),
-                                                               __fmul_rn(g4.z, (float)i2), __fmul_rn(g4.w, (float)i3));
+            float4 y4 = make_float4(__fmul_rn(g4.x, (float)i0), __fmul_rn(g4.y, (float)i1),
+                                    __fmul_rn(g4.z, (float)i2), __fmul_rn(g4.w, (float)i3));
+            if (a.bias) {
+              const float4 b4 = *reinterpret_cast<const float4*>(bias_s + c0 + 4 * c);
+              y4 = make_float4(__fadd_rn(y4.x, b4.x), __fadd_rn(y4.y, b4.y), __fadd_rn(y4.z, b4.z),
+                               __fadd_rn(y4.w, b4.w));
+            }
+            *reinterpret_cast<float4*>(sy + off) = y4;
           }
           if (a.tma_out & 2) *reinterpret_cast<int4*>(sacc + off) = make_int4(i0, i1, i2, i3);
         }
@@ -847,15 +856,21 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
 #pragma unroll
             for (int j = 0; j < 32; j += 4) {
               const float4 g4 = __ldg(reinterpret_cast<const float4*>(a.gamma + nb + j));
-              *reinterpret_cast<float4*>(yrow + j) =
-                  make_float4(__fmul_rn(g4.x, (float)iv[j]), __fmul_rn(g4.y, (float)iv[j + 1]),
-                              __fmul_rn(g4.z, (float)iv[j + 2]), __fmul_rn(g4.w, (float)iv[j + 3]));
+              float4 y4 = make_float4(__fmul_rn(g4.x, (float)iv[j]), __fmul_rn(g4.y, (float)iv[j + 1]),
+                                      __fmul_rn(g4.z, (float)iv[j + 2]), __fmul_rn(g4.w, (float)iv[j + 3]));
+              if (a.bias) {
+                const float4 b4 = __ldg(reinterpret_cast<const float4*>(a.bias + nb + j));
+                y4 = make_float4(__fadd_rn(y4.x, b4.x), __fadd_rn(y4.y, b4.y), __fadd_rn(y4.z, b4.z),
+                                 __fadd_rn(y4.w, b4.w));
+              }
+              *reinterpret_cast<float4*>(yrow + j) = y4;
               if (a.acc)
                 *reinterpret_cast<int4*>(a.acc + out_row * a.ldo + nb + j) = make_int4(iv[j], iv[j + 1], iv[j + 2], iv[j + 3]);
             }
           } else {
             for (int j = 0; j < 32 && nb + j < a.N; ++j) {
-              yrow[j] = __fmul_rn(__ldg(a.gamma + nb + j), (float)iv[j]);
+              const float g = __fmul_rn(__ldg(a.gamma + nb + j), (float)iv[j]);
+              yrow[j] = a.bias ? __fadd_rn(g, __ldg(a.bias + nb + j)) : g;
               if (a.acc) a.acc[out_row * a.ldo + nb + j] = iv[j];
             }
           }
@@ -1059,7 +1074,7 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
 
 // Forward: A = sign(X) rows [M][words(K)], B = sign(W) rows [D][words(K)].
 cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64_t D, int64_t K, const float* gamma,
-                          int32_t* acc, float* y, int32_t* status, cudaStream_t s) {
+                          const float* bias, int32_t* acc, float* y, int32_t* status, cudaStream_t s) {
   using S = TcSmem<false, false, 128>;
   const int64_t ldw = fqt1_packed_words(K);
   CUtensorMap ma, mb;
@@ -1070,7 +1085,7 @@ cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64
   TcArgs a{};
   a.M = M; a.N = D; a.L = K; a.count = nullptr; a.rows_per_count = 1;
   a.k_tiles = (int)((K + kBK * S::KSUB - 1) / (kBK * S::KSUB)); a.tiles_per_split = a.k_tiles;
-  a.epi = EPI_FWD; a.gamma = gamma; a.y = y; a.acc = acc; a.ldo = D; a.status = status;
+  a.epi = EPI_FWD; a.gamma = gamma; a.bias = bias; a.y = y; a.acc = acc; a.ldo = D; a.status = status;
   // outputs leave through TMA stores when their rows are 16-byte multiples
   CUtensorMap my{}, macc{};
   if (D % 4 == 0 && make_map(&my, y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, D, M, D * 4, 32, 32,

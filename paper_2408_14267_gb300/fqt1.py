@@ -45,6 +45,10 @@ _SIGS = {
     "fqt1_binarize_pack": (C.c_int, [_VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
     "fqt1_im2col": (C.c_int, [_VP] + [_I32] * 8 + [_VP, _VP, _VP, _VP]),
     "fqt1_fwd_gemm": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
+    "fqt1_fwd_gemm_bias": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP, _VP]),
+    "fqt1_scale_bias_workspace": (C.c_size_t, [_I64, _I64]),
+    "fqt1_scale_bias_grad": (C.c_int, [_VP, _VP, _I64, _I64, _VP, _VP, _VP, C.c_size_t, _VP]),
+    "fqt1_ste_clip": (C.c_int, [_VP, _VP, _I64, C.c_float, _VP]),
     "fqt1_agp_quantize_grad": (C.c_int, [_VP, _I64, _I64, _I32, _VP, _VP, _VP, _VP, C.c_size_t, _VP, _VP]),
     "fqt1_scq_quantize": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, C.c_size_t, _VP, _VP]),
     "fqt1_scq_quantize_noalloc": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, _VP]),
@@ -132,6 +136,24 @@ def im2col(x, N, Cin, H, W, kh, kw, stride, pad, row_bits=None, col_bits=None, c
 def fwd_gemm(sx_row, sw_row, M, D, K, gamma, acc, y, stream=None):
     _check(lib().fqt1_fwd_gemm(_p(sx_row), _p(sw_row), M, D, K, _p(gamma), _p(acc), _p(y), _s(stream)),
            "fqt1_fwd_gemm")
+
+
+def fwd_gemm_bias(sx_row, sw_row, M, D, K, gamma, bias, acc, y, stream=None):
+    _check(lib().fqt1_fwd_gemm_bias(_p(sx_row), _p(sw_row), M, D, K, _p(gamma), _p(bias), _p(acc), _p(y),
+                                    _s(stream)), "fqt1_fwd_gemm_bias")
+
+
+def scale_bias_workspace(M, D):
+    return lib().fqt1_scale_bias_workspace(M, D)
+
+
+def scale_bias_grad(gy, acc, M, D, dgamma, dbias, ws, stream=None):
+    _check(lib().fqt1_scale_bias_grad(_p(gy), _p(acc), M, D, _p(dgamma), _p(dbias), _p(ws),
+                                      ws.numel() * ws.element_size(), _s(stream)), "fqt1_scale_bias_grad")
+
+
+def ste_clip(x, dx, n, t, stream=None):
+    _check(lib().fqt1_ste_clip(_p(x), _p(dx), n, float(t), _s(stream)), "fqt1_ste_clip")
 
 
 def agp_quantize_grad(g, M, D, group_axis, gamma, params, qgrad, ws, dev_status, stream=None):

@@ -82,3 +82,49 @@ def test_conv_forward_pads_as_minus_one():
     sw = torch.from_numpy(np.where(w > 0, 1.0, -1.0))
     ref = torch.nn.functional.conv2d(sx, sw, stride=s).numpy()  # [N, D, Ho, Wo]
     assert np.array_equal(acc.reshape(N, -1, D), ref.reshape(N, D, -1).transpose(0, 2, 1).astype(np.int64))
+
+
+def test_scale_bias_grad_matches_autograd():
+    """dGamma and dbias of y = (sign(X) sign(W)^T) (.) Gamma + bias (Sec. 5.1 with a bias):
+    the oracle's closed sums against torch autograd of the plain float64 formula."""
+    rng = np.random.default_rng(21)
+    M, K, D = 37, 45, 19
+    x = rng.standard_normal((M, K))
+    w = rng.standard_normal((D, K))
+    gy = rng.standard_normal((M, D))
+    sx = torch.tensor(om.sign(x), dtype=torch.float64)
+    sw = torch.tensor(om.sign(w), dtype=torch.float64)
+    gamma = torch.tensor(rng.uniform(0.5, 2.0, D), dtype=torch.float64, requires_grad=True)
+    bias = torch.tensor(rng.standard_normal(D), dtype=torch.float64, requires_grad=True)
+    y = (sx @ sw.T) * gamma + bias
+    (y * torch.tensor(gy)).sum().backward()
+    acc, _ = om.forward(x, w, np.ones(D, np.float32))
+    dgamma, dbias = om.scale_bias_grad(gy, acc)
+    assert np.allclose(dgamma, gamma.grad.numpy(), rtol=1e-12, atol=1e-12)
+    assert np.allclose(dbias, bias.grad.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_forward_bias_adds_after_the_scale():
+    rng = np.random.default_rng(22)
+    x, w = rng.standard_normal((5, 40)), rng.standard_normal((7, 40))
+    gamma = rng.uniform(0.5, 2.0, 7).astype(np.float32)
+    bias = rng.standard_normal(7).astype(np.float32)
+    acc, y0 = om.forward(x, w, gamma)
+    acc1, y1 = om.forward_bias(x, w, gamma, bias)
+    assert np.array_equal(acc, acc1)
+    assert np.array_equal(y1, (y0 + bias[None, :]).astype(np.float32))
+    assert np.array_equal(om.forward_bias(x, w, gamma, None)[1], y0)
+
+
+def test_ste_clip_matches_hardtanh_gradient():
+    """Clipped STE: the gradient of hardtanh(x) = clip(x, -1, 1) is 1 strictly inside (-1, 1)
+    and 0 outside; the boundary |x| = 1 and NaN are the reading's own choices (pass, zero)."""
+    rng = np.random.default_rng(23)
+    x = rng.uniform(-3, 3, 1000)
+    x = x[np.abs(np.abs(x) - 1) > 1e-9]
+    g = rng.standard_normal(x.shape)
+    xt = torch.tensor(x, requires_grad=True)
+    torch.nn.functional.hardtanh(xt).backward(torch.tensor(g))
+    assert np.array_equal(om.ste_clip(x, g, 1.0), xt.grad.numpy())
+    assert np.array_equal(om.ste_clip(np.array([1.0, -1.0, np.nan, 0.5]), np.ones(4), 1.0), [1.0, 1.0, 0.0, 1.0])
+    assert np.array_equal(om.ste_clip(np.array([0.3, 0.6]), np.array([2.0, 3.0]), 0.5), [2.0, 0.0])
