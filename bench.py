@@ -199,6 +199,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile", type=int, default=0, metavar="N",
                     help="only run --warmup + N eager steps (for ncu), print nothing")
+    ap.add_argument("--table5", action="store_true",
+                    help="GEMM-only comparison of average 1-bit and 1-bit products on the Table 5 shapes")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -206,6 +208,8 @@ def main():
 
     if args.impl == "reference":
         return reference_arm(args, world, rank)
+    if args.table5:
+        return table5(args)
 
     import torch
     import torch.distributed as dist
@@ -366,6 +370,79 @@ def main():
         print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
+
+
+TABLE5_SHAPES = [(512, 512, 512), (512, 512, 1024), (1024, 512, 512), (1024, 512, 1024), (2048, 512, 512),
+                 (2048, 512, 1024)]
+
+
+def table5(args):
+    """Table 5's comparison on this datapath: the product of sign(A) [M, K] and sign(B) [N, K]
+    (1-bit, the forward product) against the product of the kept quarter of A's rows as 4-bit
+    codes with sign(B) (average 1-bit, b = 4: the grad_input product on a PSQ branch with one
+    row per group).  Each product is one graph-captured launch, timed with CUDA events after an
+    L2 flush; both write 4-byte outputs (fp32 y, int32 accumulators)."""
+    import torch
+    from paper_2408_14267_gb300 import build, fqt1
+    build.build()
+    dev = torch.device("cuda")
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)
+    stream = torch.cuda.Stream()
+    gen = torch.Generator(device="cpu").manual_seed(5)
+
+    def timed(fn, reps):
+        with torch.cuda.stream(stream):
+            fn(stream)
+            stream.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                fn(stream)
+            for _ in range(max(args.warmup, 3)):
+                g.replay()
+            ts = []
+            for _ in range(reps):
+                flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                g.replay()
+                e1.record(stream)
+                ts.append((e0, e1))
+            stream.synchronize()
+        return statistics.median(a.elapsed_time(b) * 1e3 for a, b in ts)
+
+    rows = []
+    for M, K, N in TABLE5_SHAPES:
+        a = torch.randn(M, K, generator=gen).to(dev)
+        b = torch.randn(N, K, generator=gen).to(dev)
+        wK = fqt1.packed_words(K)
+        sa = torch.empty(M, wK, dtype=torch.int32, device=dev)
+        sb_row = torch.empty(N, wK, dtype=torch.int32, device=dev)
+        fqt1.binarize_pack(a, M, K, K, sa, None, None)
+        fqt1.binarize_pack(b, N, K, K, sb_row, None, None)
+        ones = torch.ones(N, device=dev)
+        y = torch.empty(M, N, device=dev)
+        one_bit = timed(lambda s: fqt1.fwd_gemm(sa, sb_row, M, N, K, ones, None, y, s), args.steps)
+        # average 1-bit: the kept quarter of A's rows (b = 4) as 4-bit codes
+        g = (torch.randn(M, K, generator=gen) * torch.exp(2 * torch.randn(M, 1, generator=gen))).to(dev)
+        p = fqt1.AgpParams(4, 0, 11, 1)
+        cap = fqt1.kept_capacity(M, 4, 0)
+        q = fqt1.QGradBuffers(M, cap, cap, K, dev)
+        ws = torch.empty(fqt1.workspace_size(0, M, K, N, 1), dtype=torch.uint8, device=dev)
+        status = torch.zeros(4, dtype=torch.int32, device=dev)
+        fqt1.agp_quantize_grad(g, M, K, 0, None, p, q, ws, status)
+        acc = torch.empty(cap, N, dtype=torch.int32, device=dev)
+        # contraction over K: the product's second operand is sign(B) packed along K, as for the forward
+        avg = timed(lambda s: fqt1.bwd_input_gemm(q, sb_row, None, M, K, N, p, acc, None, s), args.steps)
+        rows.append({"M": M, "K": K, "N": N, "kept_rows": q.count(), "one_bit_us": round(one_bit, 2),
+                     "avg_1bit_us": round(avg, 2)})
+    ratio = statistics.mean(r["avg_1bit_us"] / r["one_bit_us"] for r in rows)
+    print(json.dumps({"metric": "GEMM time, average 1-bit (b=4, kept quarter, 4-bit codes) / 1-bit, Table 5 shapes",
+                      "value": ratio, "unit": "ratio", "higher_is_better": False, "steps": args.steps,
+                      "warmup": args.warmup, "dtype": "e4m3", "data": "synthetic",
+                      "config": {"workload": "Table 5 shapes M x K x N, K the contraction",
+                                 "l2": "flushed before every timed launch (256 MiB write)",
+                                 "timing": "one graph-captured launch, CUDA events, median"},
+                      "shapes": rows}))
 
 
 def reference_arm(args, world, rank):

@@ -313,3 +313,36 @@ def test_binarize_pack_strided(rows, cols, ld):
     sc, pad = unpack_bits(col_bits, rows)
     assert np.array_equal(sc, om.sign(x).T) and not pad.any()
     assert np.array_equal(colsum.cpu().numpy(), om.colsum_sign(x))
+
+
+@pytest.mark.parametrize("M,K,N", [(512, 512, 512), (1024, 512, 1024), (2048, 512, 512)])
+def test_table5_shapes_exact(M, K, N):
+    """The two products bench.py --table5 times, on Table 5 shapes: sign(A) sign(B)^T (1-bit) and
+    the kept quarter of A's rows as 4-bit codes times sign(B)^T (average 1-bit), int32 exact."""
+    from paper_2408_14267_gb300 import fqt1
+    rng = np.random.default_rng(M + N)
+    a = rng.standard_normal((M, K)).astype(np.float32)
+    b = rng.standard_normal((N, K)).astype(np.float32)
+    g = (rng.standard_normal((M, K)) * np.exp(2 * rng.standard_normal((M, 1)))).astype(np.float32)
+    dev = torch.device("cuda")
+    wK = fqt1.packed_words(K)
+    sa = torch.empty(M, wK, dtype=torch.int32, device=dev)
+    sb = torch.empty(N, wK, dtype=torch.int32, device=dev)
+    fqt1.binarize_pack(torch.from_numpy(a).cuda(), M, K, K, sa, None, None)
+    fqt1.binarize_pack(torch.from_numpy(b).cuda(), N, K, K, sb, None, None)
+    acc1 = torch.empty(M, N, dtype=torch.int32, device=dev)
+    y = torch.empty(M, N, device=dev)
+    fqt1.fwd_gemm(sa, sb, M, N, K, torch.ones(N, device=dev), acc1, y)
+    assert np.array_equal(acc1.cpu().numpy(), om.int_matmul(om.sign(a), om.sign(b)))
+    p = fqt1.AgpParams(4, SYS, 11, 1)
+    cap = fqt1.kept_capacity(M, 4, SYS)
+    q = fqt1.QGradBuffers(M, cap, cap, K, dev)
+    ws = torch.empty(fqt1.workspace_size(0, M, K, N, 1), dtype=torch.uint8, device=dev)
+    status = torch.zeros(4, dtype=torch.int32, device=dev)
+    fqt1.agp_quantize_grad(torch.from_numpy(g).cuda(), M, K, 0, None, p, q, ws, status)
+    acc4 = torch.empty(cap, N, dtype=torch.int32, device=dev)
+    fqt1.bwd_input_gemm(q, sb, None, M, K, N, p, acc4, None)
+    ref = om.agp_quantize(g, 0, 1, 4, SYS, 11)
+    cnt = q.count()
+    assert cnt == len(ref["kept"])
+    assert np.array_equal(acc4.cpu().numpy()[:cnt], om.int_matmul(ref["codes"], om.sign(b)))
