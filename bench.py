@@ -201,6 +201,10 @@ def main():
                     help="only run --warmup + N eager steps (for ncu), print nothing")
     ap.add_argument("--table5", action="store_true",
                     help="GEMM-only comparison of average 1-bit and 1-bit products on the Table 5 shapes")
+    ap.add_argument("--model", choices=["vgg16", "resnet18"],
+                    help="training step of a synthetic model built from binop layers against FP32 PyTorch")
+    ap.add_argument("--res", type=int, default=32, help="input resolution of --model")
+    ap.add_argument("--batch", type=int, default=128, help="batch of --model")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -210,6 +214,8 @@ def main():
         return reference_arm(args, world, rank)
     if args.table5:
         return table5(args)
+    if args.model:
+        return model_step(args)
 
     import torch
     import torch.distributed as dist
@@ -443,6 +449,137 @@ def table5(args):
                                  "l2": "flushed before every timed launch (256 MiB write)",
                                  "timing": "one graph-captured launch, CUDA events, median"},
                       "shapes": rows}))
+
+
+def build_model(name, res, binary, classes=10):
+    """VGG-16 or ResNet-18 for res x res inputs.  binary: the hidden convolutions and fully
+    connected layers are binop layers (1-bit forward, 1-bit FQT backward); the first convolution
+    and the classifier stay full precision, as in binary networks; BatchNorm and Hardtanh between
+    layers.  Otherwise every layer is a float32 torch layer."""
+    import torch
+    from paper_2408_14267_gb300 import binop
+    nn = torch.nn
+
+    def conv(cin, cout, k, s, p, first=False):
+        if binary and not first:
+            return binop.Conv2d(cin, cout, k, stride=s, padding=p, qcfg=binop.QuantConfig(4))
+        return nn.Conv2d(cin, cout, k, stride=s, padding=p, bias=False)
+
+    def fc(fin, fout, last=False):
+        if binary and not last:
+            return binop.Linear(fin, fout, qcfg=binop.QuantConfig(4))
+        return nn.Linear(fin, fout)
+
+    if name == "vgg16":
+        cfg = [64, 64, "M", 128, 128, "M", 256, 256, 256, "M", 512, 512, 512, "M", 512, 512, 512, "M"]
+        layers, cin = [], 3
+        for v in cfg:
+            if v == "M":
+                layers.append(nn.MaxPool2d(2))
+            else:
+                layers += [conv(cin, v, 3, 1, 1, first=cin == 3), nn.BatchNorm2d(v), nn.Hardtanh()]
+                cin = v
+        feat = 512 * (res // 32) ** 2
+        layers += [nn.Flatten(), fc(feat, 512), nn.BatchNorm1d(512), nn.Hardtanh(), fc(512, 512),
+                   nn.BatchNorm1d(512), nn.Hardtanh(), fc(512, classes, last=True)]
+        return nn.Sequential(*layers)
+
+    class Block(nn.Module):
+        def __init__(self, cin, cout, stride):
+            super().__init__()
+            self.c1, self.b1 = conv(cin, cout, 3, stride, 1), nn.BatchNorm2d(cout)
+            self.c2, self.b2 = conv(cout, cout, 3, 1, 1), nn.BatchNorm2d(cout)
+            self.down = None
+            if stride != 1 or cin != cout:
+                self.down = nn.Sequential(conv(cin, cout, 1, stride, 0), nn.BatchNorm2d(cout))
+            self.act = nn.Hardtanh()
+
+        def forward(self, x):
+            y = self.act(self.b1(self.c1(x)))
+            y = self.b2(self.c2(y))
+            return self.act(y + (x if self.down is None else self.down(x)))
+
+    if res <= 64:  # CIFAR-style stem
+        stem = [conv(3, 64, 3, 1, 1, first=True), nn.BatchNorm2d(64), nn.Hardtanh()]
+    else:
+        stem = [conv(3, 64, 7, 2, 3, first=True), nn.BatchNorm2d(64), nn.Hardtanh(), nn.MaxPool2d(3, 2, 1)]
+    blocks, cin = [], 64
+    for cout, stride in ((64, 1), (128, 2), (256, 2), (512, 2)):
+        blocks += [Block(cin, cout, stride), Block(cout, cout, 1)]
+        cin = cout
+    return nn.Sequential(*stem, *blocks, nn.AdaptiveAvgPool2d(1), nn.Flatten(), fc(512, classes, last=True))
+
+
+def model_step(args):
+    """One training step (forward, cross-entropy, backward, SGD update) of a synthetic VGG-16 or
+    ResNet-18 on random data, graph-captured, with binop layers against float32 torch layers
+    (TF32 off): the GPU analogue of Table 3's speedup over FP32 PyTorch."""
+    import torch
+    from paper_2408_14267_gb300 import build
+    build.build()
+    torch.backends.cudnn.allow_tf32 = False
+    torch.backends.cuda.matmul.allow_tf32 = False
+    torch.backends.cudnn.benchmark = True
+    dev = torch.device("cuda")
+    gen = torch.Generator(device="cpu").manual_seed(1)
+    x = torch.randn(args.batch, 3, args.res, args.res, generator=gen).to(dev)
+    t = torch.randint(0, 10, (args.batch,), generator=gen).to(dev)
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)
+    out = {}
+    if args.profile:  # eager steps of the binop model only (for a kernel launch list)
+        torch.backends.cudnn.benchmark = False  # no algorithm search among the launches
+        torch.manual_seed(2)
+        net = build_model(args.model, args.res, True).to(dev)
+        opt = torch.optim.SGD(net.parameters(), lr=1e-3)
+        for _ in range(args.warmup + args.profile):
+            opt.zero_grad(set_to_none=False)
+            torch.nn.functional.cross_entropy(net(x), t).backward()
+            opt.step()
+        torch.cuda.synchronize()
+        return
+    for arm, binary in (("fp32", False), ("fqt1", True)):
+        torch.manual_seed(2)
+        net = build_model(args.model, args.res, binary).to(dev)
+        opt = torch.optim.SGD(net.parameters(), lr=1e-3)
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            for _ in range(3):  # warm-up before capture (allocator, cuDNN algorithms)
+                opt.zero_grad(set_to_none=False)
+                torch.nn.functional.cross_entropy(net(x), t).backward()
+                opt.step()
+        torch.cuda.current_stream().wait_stream(side)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            opt.zero_grad(set_to_none=False)
+            loss = torch.nn.functional.cross_entropy(net(x), t)
+            loss.backward()
+            opt.step()
+        for _ in range(max(args.warmup, 3)):
+            g.replay()
+        ts = []
+        for _ in range(args.steps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            g.replay()
+            e1.record()
+            ts.append((e0, e1))
+        torch.cuda.synchronize()
+        out[arm] = statistics.median(a.elapsed_time(b) for a, b in ts)
+        assert torch.isfinite(loss).item(), "non-finite loss"
+    print(json.dumps({"metric": f"training step speedup over FP32 PyTorch, synthetic {args.model}",
+                      "value": out["fp32"] / out["fqt1"], "unit": "x", "higher_is_better": True,
+                      "steps": args.steps, "warmup": args.warmup, "dtype": "e4m3", "data": "synthetic",
+                      "ms_per_step": {"fqt1": round(out["fqt1"], 4), "fp32": round(out["fp32"], 4)},
+                      "config": {"workload": f"{args.model}, batch {args.batch}, {args.res}x{args.res} inputs, "
+                                             "10 classes; hidden convolutions and fully connected layers binop "
+                                             "(1-bit forward, AGP b=4 SCQ backward), first convolution and "
+                                             "classifier float32; the fp32 arm has float32 layers (TF32 off)",
+                                 "l2": "flushed before every timed step (256 MiB write)",
+                                 "timing": "one CUDA graph per arm (forward, loss, backward, SGD step), CUDA "
+                                           "events, median; the graph repeats its quantizer seeds"}}))
 
 
 def reference_arm(args, world, rank):

@@ -146,7 +146,7 @@ fqt1_status fqt1_fwd_gemm_bias(const uint32_t* sx_row, const uint32_t* sw_row, i
  * gy: [M][D] fp32 (the gradient of y); acc: [M][D] int32, the forward
  * accumulators (fqt1_fwd_gemm's acc), needed for dgamma; dgamma, dbias: [D]
  * fp32, either may be NULL, overwritten.  The sums run in a fixed order (fp32
- * over 64-row chunks, fp64 over the chunks), so the results are reproducible.
+ * within 256-row chunks, fp64 over the chunks), so the results are reproducible.
  * ws: fqt1_scale_bias_workspace(M, D) bytes, 16-byte aligned, caller-owned. */
 size_t fqt1_scale_bias_workspace(int64_t M, int64_t D);
 fqt1_status fqt1_scale_bias_grad(const float* gy, const int32_t* acc, int64_t M, int64_t D, float* dgamma,

@@ -4,7 +4,7 @@
 // Gamma in R^D shared by weights and activations; a bias is an extension, the paper's
 // Algorithm 1 omits it).  With acc = sign(x) sign(W)^T the int32 forward accumulators:
 //   dGamma[j] = sum_m gY[m, j] acc[m, j],   dbias[j] = sum_m gY[m, j].
-// Both sums run in a fixed order (fp32 over chunks of kChunkRows rows, then fp64 over the
+// Both sums run in a fixed order (fp32 within chunks of kChunkRows rows, float64 over the
 // chunks), so the results do not depend on the launch.
 //
 // The straight-through estimator (cited in Sec. 3.1 for QAT) passes the gradient of sign()
@@ -15,57 +15,86 @@
 
 namespace fqt1 {
 
-constexpr int kChunkRows = 64;   // rows of gY per partial sum
-constexpr int kGradCols = 128;   // columns per CTA (one per thread)
+constexpr int kChunkRows = 256;  // rows of gY per partial sum
+constexpr int kGradCols = 32;    // columns per CTA (one per lane)
+constexpr int kRowLanes = 8;     // warps of a CTA; warp w takes rows w, w + 8, ... of a chunk
 
-// partial[c][j] (and partial[chunks + c][j]) = the fp32 sums over rows c kChunkRows ..
+// part[c][j] and part[chunks + c][j] = the fp32 sums of gY acc and gY over rows c kChunkRows ..
+// (c + 1) kChunkRows - 1: each warp sums its rows in order, then the 8 warp sums are added in
+// warp order.
 template <bool ACC>
-__global__ void __launch_bounds__(kGradCols) scale_bias_partial_kernel(const float* __restrict__ gy,
-                                                                       const int32_t* __restrict__ acc, int64_t M,
-                                                                       int64_t D, int64_t chunks,
-                                                                       float* __restrict__ part) {
+__global__ void __launch_bounds__(kGradCols * kRowLanes) scale_bias_partial_kernel(
+    const float* __restrict__ gy, const int32_t* __restrict__ acc, int64_t M, int64_t D, int64_t chunks,
+    float* __restrict__ part) {
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
-  const int64_t j = (int64_t)blockIdx.x * kGradCols + threadIdx.x;
-  const int64_t c = blockIdx.y, r0 = c * kChunkRows;
-  if (j >= D) return;
-  const int64_t jc = j;
+  __shared__ float sg_s[kRowLanes][kGradCols], sb_s[kRowLanes][kGradCols];
+  const int lane = threadIdx.x & 31, rl = threadIdx.x >> 5;
+  const int64_t j = (int64_t)blockIdx.x * kGradCols + lane;
+  const int64_t jc = min(j, D - 1);
+  const int64_t c = blockIdx.y, r0 = c * kChunkRows + rl;
   float sg = 0.f, sb = 0.f;
-  for (int rr = 0; rr < kChunkRows; rr += 8) {
+#pragma unroll 1
+  for (int i0 = 0; i0 < kChunkRows / kRowLanes; i0 += 8) {
     // 8 rows in flight (unconditional loads from clamped rows, masked below)
     float g[8];
     int32_t q[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
-      const int64_t r = min(r0 + rr + u, M - 1);
+      const int64_t r = min(r0 + (int64_t)kRowLanes * (i0 + u), M - 1);
       g[u] = __ldg(gy + r * D + jc);
       q[u] = ACC ? __ldg(acc + r * D + jc) : 0;
     }
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
-      if (r0 + rr + u >= M) break;
+      if (r0 + (int64_t)kRowLanes * (i0 + u) >= M) break;
       sg = __fadd_rn(sg, __fmul_rn(g[u], (float)q[u]));
       sb = __fadd_rn(sb, g[u]);
     }
   }
-  part[c * D + j] = sg;
-  part[(chunks + c) * D + j] = sb;
+  sg_s[rl][lane] = sg;
+  sb_s[rl][lane] = sb;
+  __syncthreads();
+  if (rl == 0 && j < D) {
+    float tg = 0.f, tb = 0.f;
+#pragma unroll
+    for (int w = 0; w < kRowLanes; ++w) {
+      tg = __fadd_rn(tg, sg_s[w][lane]);
+      tb = __fadd_rn(tb, sb_s[w][lane]);
+    }
+    part[c * D + j] = tg;
+    part[(chunks + c) * D + j] = tb;
+  }
 }
 
-__global__ void __launch_bounds__(kGradCols) scale_bias_final_kernel(const float* __restrict__ part, int64_t D,
-                                                                     int64_t chunks, float* __restrict__ dgamma,
-                                                                     float* __restrict__ dbias) {
+// dgamma[j], dbias[j]: warp w adds chunks w, w + 8, ... in float64, then the 8 warp sums are
+// added in warp order.
+__global__ void __launch_bounds__(kGradCols * kRowLanes) scale_bias_final_kernel(
+    const float* __restrict__ part, int64_t D, int64_t chunks, float* __restrict__ dgamma, float* __restrict__ dbias) {
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
-  const int64_t j = (int64_t)blockIdx.x * kGradCols + threadIdx.x;
-  if (j >= D) return;
+  __shared__ double sg_s[kRowLanes][kGradCols], sb_s[kRowLanes][kGradCols];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t j = (int64_t)blockIdx.x * kGradCols + lane;
+  const int64_t jc = min(j, D - 1);
   double sg = 0.0, sb = 0.0;
-  for (int64_t c = 0; c < chunks; ++c) {
-    sg += (double)part[c * D + j];
-    sb += (double)part[(chunks + c) * D + j];
+  for (int64_t c = w; c < chunks; c += kRowLanes) {
+    sg += (double)__ldg(part + c * D + jc);
+    sb += (double)__ldg(part + (chunks + c) * D + jc);
   }
-  if (dgamma) dgamma[j] = (float)sg;
-  if (dbias) dbias[j] = (float)sb;
+  sg_s[w][lane] = sg;
+  sb_s[w][lane] = sb;
+  __syncthreads();
+  if (w == 0 && j < D) {
+    double tg = 0.0, tb = 0.0;
+#pragma unroll
+    for (int u = 0; u < kRowLanes; ++u) {
+      tg += sg_s[u][lane];
+      tb += sb_s[u][lane];
+    }
+    if (dgamma) dgamma[j] = (float)tg;
+    if (dbias) dbias[j] = (float)tb;
+  }
 }
 
 __global__ void __launch_bounds__(256) ste_clip_kernel(const float* __restrict__ x, float* __restrict__ dx,
@@ -110,14 +139,15 @@ extern "C" fqt1_status fqt1_scale_bias_grad(const float* gy, const int32_t* acc,
   cudaStream_t s = (cudaStream_t)stream;
   float* part = static_cast<float*>(ws);
   const unsigned gx = (unsigned)((D + kGradCols - 1) / kGradCols);
+  const dim3 block(kGradCols * kRowLanes);
   if (dgamma)
-    FQT1_CUDA_TRY(launch_k(scale_bias_partial_kernel<true>, dim3(gx, (unsigned)chunks), dim3(kGradCols), 0, s, gy,
-                           acc, M, D, chunks, part));
+    FQT1_CUDA_TRY(launch_k(scale_bias_partial_kernel<true>, dim3(gx, (unsigned)chunks), block, 0, s, gy, acc, M, D,
+                           chunks, part));
   else
-    FQT1_CUDA_TRY(launch_k(scale_bias_partial_kernel<false>, dim3(gx, (unsigned)chunks), dim3(kGradCols), 0, s, gy,
-                           acc, M, D, chunks, part));
+    FQT1_CUDA_TRY(launch_k(scale_bias_partial_kernel<false>, dim3(gx, (unsigned)chunks), block, 0, s, gy, acc, M, D,
+                           chunks, part));
   fqt1_count_launches(1);
-  FQT1_CUDA_TRY(launch_k(scale_bias_final_kernel, dim3(gx), dim3(kGradCols), 0, s, part, D, chunks, dgamma, dbias));
+  FQT1_CUDA_TRY(launch_k(scale_bias_final_kernel, dim3(gx), block, 0, s, part, D, chunks, dgamma, dbias));
   fqt1_count_launches(1);
   return FQT1_OK;
 }
