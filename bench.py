@@ -203,6 +203,8 @@ def main():
                     help="GEMM-only comparison of average 1-bit and 1-bit products on the Table 5 shapes")
     ap.add_argument("--model", choices=["vgg16", "resnet18"],
                     help="training step of a synthetic model built from binop layers against FP32 PyTorch")
+    ap.add_argument("--variance", action="store_true",
+                    help="empirical variance of the AGP quantizer (b = 2, 4, 8) and of 1-bit PSQ against Eq. 24")
     ap.add_argument("--res", type=int, default=32, help="input resolution of --model")
     ap.add_argument("--batch", type=int, default=128, help="batch of --model")
     args = ap.parse_args()
@@ -216,6 +218,8 @@ def main():
         return table5(args)
     if args.model:
         return model_step(args)
+    if args.variance:
+        return variance_study(args)
 
     import torch
     import torch.distributed as dist
@@ -580,6 +584,64 @@ def model_step(args):
                                  "l2": "flushed before every timed step (256 MiB write)",
                                  "timing": "one CUDA graph per arm (forward, loss, backward, SGD step), CUDA "
                                            "events, median; the graph repeats its quantizer seeds"}}))
+
+
+def variance_study(args):
+    """Quantizer variance on heterogeneous synthetic gradients (the mechanism of Sec. 5.2 and the
+    quantizer-variance comparison of the experiments): G [M, D] of 128 samples x 64 rows, per-sample
+    scales exp(2 N(0,1)), groups = samples.  For each setting, `steps` seeds of the library's AGP
+    quantizer (fqt1_agp_quantize_grad) give E||Q(G) - G||^2, summed over elements, next to the bound
+    of Eq. 24, D_g / (4 B^2) sum over the N/b largest ranges of R_i^2 (D_g = elements per group),
+    and the 1-bit PSQ bound D_g / 4 sum_i R_i^2.  The dequantization Q = S' q + Z' (0 for pruned
+    groups) is evaluated here in float64 for the measurement only."""
+    import numpy as np
+    import torch
+    from paper_2408_14267_gb300 import build, fqt1
+    build.build()
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(31)
+    N, rpg, D = 128, 64, 256
+    M = N * rpg
+    g_np = (1e-3 * rng.standard_normal((N, rpg, D)) * np.exp(2 * rng.standard_normal((N, 1, 1)))).reshape(M, D)
+    g = torch.from_numpy(g_np.astype(np.float32)).to(dev)
+    g64 = g.double()
+    ws = torch.empty(fqt1.workspace_size(0, M, D, 0, rpg), dtype=torch.uint8, device=dev)
+    status = torch.zeros(4, dtype=torch.int32, device=dev)
+    settings = [("PSQ 1-bit", 1, 0), ("AGP b=2", 2, 0), ("AGP b=4", 4, 0), ("AGP b=8", 8, 0),
+                ("AGP b=4, Bernoulli masks", 4, 1), ("AGP b=4, top-N/b (biased)", 4, 2)]
+    results = []
+    for name, bits, mode in settings:
+        cap = fqt1.kept_capacity(N, bits, mode)
+        q = fqt1.QGradBuffers(N, cap, cap * rpg, D, dev)
+        sq = torch.zeros(M, D, dtype=torch.float64, device=dev)
+        mean = torch.zeros(M, D, dtype=torch.float64, device=dev)
+        for seed in range(args.steps):
+            fqt1.agp_quantize_grad(g, M, D, 0, None, fqt1.AgpParams(bits, mode, 1000 + seed, rpg), q, ws, status)
+            cnt = q.count()
+            kept = q.kept_idx[:cnt].long()
+            codes = q.codes[:cnt * rpg, :D].double().view(cnt, rpg, D)
+            deq = torch.zeros(N, rpg, D, dtype=torch.float64, device=dev)
+            deq[kept] = codes * q.scale[:cnt].double().view(cnt, 1, 1) + q.zero[:cnt].double().view(cnt, 1, 1)
+            deq = deq.view(M, D)
+            sq += (deq - g64) ** 2
+            mean += deq
+        assert int(status[0].item()) == 0
+        r = q.group_range.double().cpu().numpy()
+        B = (1 << bits) - 1
+        top = np.sort(r)[::-1][:max(1, N // bits) if bits > 1 else N]
+        d_g = rpg * D
+        var = float(sq.sum().item()) / args.steps
+        bias = float(((mean / args.steps - g64) ** 2).sum().item())
+        results.append({"setting": name, "bits": bits, "E_sq_error": var, "sq_bias_of_mean": bias,
+                        "eq24_bound": d_g / (4 * B * B) * float(np.sum(top ** 2)),
+                        "psq_1bit_bound": d_g / 4 * float(np.sum(r ** 2))})
+    agp4 = next(x for x in results if x["setting"] == "AGP b=4")["E_sq_error"]
+    psq = results[0]["E_sq_error"]
+    print(json.dumps({"metric": "quantizer variance E||Q(G) - G||^2, AGP b=4 / 1-bit PSQ", "value": agp4 / psq,
+                      "unit": "ratio", "higher_is_better": False, "steps": args.steps, "data": "synthetic",
+                      "config": {"workload": f"G [{M}, {D}]: {N} samples x {rpg} rows, N(0,1) x 1e-3 x exp(2 N(0,1)) "
+                                             "per sample; groups = samples; seeds 1000 .. 1000 + steps - 1"},
+                      "settings": results}))
 
 
 def reference_arm(args, world, rank):

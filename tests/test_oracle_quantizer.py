@@ -151,3 +151,24 @@ def test_conv_grad_input_matches_transposed_conv():
     scale[res["psq"]["kept"]] = np.abs(res["psq"]["scale"])
     tol = 1e-6 * (scale[:, None, None, None] * np.abs(res["acc_fold"]) + np.abs(ref)) + 1e-30
     assert np.all(np.abs(res["dx"] - ref) <= tol)
+
+
+def test_agp_variance_below_one_bit_psq():
+    """Sec. 5.2 / App. B: on groups with heterogeneous ranges, AGP with b = 4 (a quarter of the
+    groups kept at 4 bits, systematic masks) has a much smaller variance E||Q(G) - G||^2 than
+    1-bit PSQ (every group at 1 bit), whose exact variance is sum R_i^2 p(1 - p) over the
+    elements (SR variance with B = 1)."""
+    rng = np.random.default_rng(12)
+    M, D, rpg, trials = 32, 8, 1, 1500
+    g = (rng.standard_normal((M, D)) * np.exp(2 * rng.standard_normal((M, 1)))).astype(f32)
+    agp = np.stack([_dequant_psq(om.agp_quantize(g, 0, rpg, 4, om.SYSTEMATIC, s), M, D) for s in range(trials)])
+    var_agp = ((agp - g.astype(np.float64)) ** 2).sum(axis=(1, 2)).mean()
+    qd = om.agp_quantize(g, 0, rpg, 1, om.SYSTEMATIC, 0)
+    t = ((g - qd["z"][:, None]) * (f32(1) / qd["r"])[:, None]).astype(np.float64)
+    p = t - np.floor(t)
+    var_psq = np.sum(qd["r"].astype(np.float64)[:, None] ** 2 * p * (1 - p))
+    assert var_agp < 0.25 * var_psq
+    # and the 1-bit PSQ variance formula itself against sampling
+    psq = np.stack([_dequant_psq(om.agp_quantize(g, 0, rpg, 1, om.SYSTEMATIC, s), M, D) for s in range(400)])
+    emp = ((psq - g.astype(np.float64)) ** 2).sum(axis=(1, 2)).mean()
+    assert abs(emp - var_psq) <= 0.1 * var_psq
