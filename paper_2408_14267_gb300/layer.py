@@ -175,3 +175,76 @@ class LayerStep:
         b2_done = torch.cuda.Event()
         b2_done.record(b2)
         main.wait_event(b2_done)
+
+    def step_concurrent_host(self, h_in, h_out, stream=None):
+        """step_concurrent with the host copies of one step, capturable in one graph.
+
+        h_in: pinned host tensors (x, w, gy[, gamma]) copied into the layer's inputs; h_out:
+        pinned host tensors (y, dx, dw) that receive the outputs.  The host link carries one
+        copy at a time at full rate (parallel copies share it), so the copies run in a fixed
+        order on two streams and each branch starts as soon as its own input has landed:
+          copies in : W, Gamma (if any), gY, X
+          branch 1  : (W in) pack W
+          branch 2  : (gY in) SCQ quantize -> (W packed) grad_input (-> Folder)
+          calling   : (X in) pack / Unfolder -> (W packed) forward -> (SCQ) grad_weight
+          copies out: (all in, grad_input done) dx, (forward done) y, (grad_weight done) dw
+        """
+        main = stream if stream is not None else torch.cuda.current_stream()
+        if not hasattr(self, "_branches4"):
+            self._branches4 = tuple(torch.cuda.Stream(device=main.device) for _ in range(4))
+        b1, b2, cin, cout = self._branches4
+        st = dict(self.stages())
+
+        def ev(s):
+            e = torch.cuda.Event()
+            e.record(s)
+            return e
+
+        fork = ev(main)
+        for b in (b1, b2, cin, cout):
+            b.wait_event(fork)
+        x_h, w_h, gy_h = h_in[0], h_in[1], h_in[2]
+        g_h = h_in[3] if len(h_in) > 3 else None
+        with torch.cuda.stream(cin):
+            self.w.copy_(w_h, non_blocking=True)
+            w_in = ev(cin)
+            if g_h is not None:
+                self.gamma.copy_(g_h, non_blocking=True)
+            self.gy.copy_(gy_h, non_blocking=True)
+            gy_in = ev(cin)
+            self.x.copy_(x_h, non_blocking=True)
+            x_in = ev(cin)
+        b1.wait_event(w_in)
+        st["pack_w"](b1)
+        w_ready = ev(b1)
+        b2.wait_event(gy_in)
+        st["scq_quantize"](b2)
+        q_ready = ev(b2)
+        b2.wait_event(w_ready)
+        if "bwd_input_fold" in st:
+            st["bwd_input_fold"](b2)
+        else:
+            st["bwd_input_gemm"](b2)
+            if "col2im" in st:
+                st["col2im"](b2)
+        dx_ready = ev(b2)
+        main.wait_event(x_in)
+        x_name = "im2col" if "im2col" in st else "pack_x"
+        st[x_name](main)
+        main.wait_event(w_ready)
+        main.wait_event(gy_in)  # Gamma (copied before gY) scales the forward
+        st["fwd_gemm"](main)
+        y_ready = ev(main)
+        main.wait_event(q_ready)
+        st["bwd_weight_gemm"](main)
+        dw_ready = ev(main)
+        cout.wait_event(x_in)  # the outputs follow the inputs on the link
+        with torch.cuda.stream(cout):
+            cout.wait_event(dx_ready)
+            h_out[1].copy_(self.dx, non_blocking=True)
+            cout.wait_event(y_ready)
+            h_out[0].copy_(self.y, non_blocking=True)
+            cout.wait_event(dw_ready)
+            h_out[2].copy_(self.dw, non_blocking=True)
+        main.wait_event(ev(cout))
+        main.wait_event(ev(b2))

@@ -346,3 +346,26 @@ def test_table5_shapes_exact(M, K, N):
     cnt = q.count()
     assert cnt == len(ref["kept"])
     assert np.array_equal(acc4.cpu().numpy()[:cnt], om.int_matmul(ref["codes"], om.sign(b)))
+
+
+@pytest.mark.parametrize("name,make", [CASES[0], CASES[1]], ids=[CASES[0][0], CASES[1][0]])
+def test_host_copy_step_matches_serial(name, make):
+    """The step with its host copies (LayerStep.step_concurrent_host, the end-to-end form) gives
+    the outputs of the serial step bit for bit, from inputs that reach the device only through
+    its copies."""
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    st = LayerStep(w, keep_acc=False)
+    st.step()
+    torch.cuda.synchronize()
+    ref = [t.clone() for t in (st.y, st.dx, st.dw)]
+    h_in = [t.detach().cpu().pin_memory() for t in (st.x, st.w, st.gy)]
+    if st.gamma is not None:
+        h_in.append(st.gamma.detach().cpu().pin_memory())
+    for t in (st.x, st.w, st.gy, st.y, st.dx, st.dw):
+        t.zero_()
+    h_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in ref]
+    st.step_concurrent_host(h_in, h_out)
+    torch.cuda.synchronize()
+    for h, r, what in zip(h_out, ref, ("y", "dx", "dw")):
+        assert torch.equal(h, r.cpu()), what
