@@ -443,7 +443,7 @@ def table5(args):
         p = fqt1.AgpParams(4, 0, 11, 1)
         cap = fqt1.kept_capacity(M, 4, 0)
         q = fqt1.QGradBuffers(M, cap, cap, K, dev)
-        ws = torch.empty(fqt1.workspace_size(0, M, K, N, 1), dtype=torch.uint8, device=dev)
+        ws = fqt1.scq_workspace(M, K, N, 1, dev)
         status = torch.zeros(4, dtype=torch.int32, device=dev)
         fqt1.agp_quantize_grad(g, M, K, 0, None, p, q, ws, status)
         acc = torch.empty(cap, N, dtype=torch.int32, device=dev)
@@ -611,7 +611,7 @@ def variance_study(args):
     g_np = (1e-3 * rng.standard_normal((N, rpg, D)) * np.exp(2 * rng.standard_normal((N, 1, 1)))).reshape(M, D)
     g = torch.from_numpy(g_np.astype(np.float32)).to(dev)
     g64 = g.double()
-    ws = torch.empty(fqt1.workspace_size(0, M, D, 0, rpg), dtype=torch.uint8, device=dev)
+    ws = fqt1.scq_workspace(M, D, 0, rpg, dev)
     status = torch.zeros(4, dtype=torch.int32, device=dev)
     settings = [("PSQ 1-bit", 1, 0), ("AGP b=2", 2, 0), ("AGP b=4", 4, 0), ("AGP b=8", 8, 0),
                 ("AGP b=4, Bernoulli masks", 4, 1), ("AGP b=4, top-N/b (biased)", 4, 2)]

@@ -159,13 +159,25 @@ fqt1_status fqt1_scale_bias_grad(const float* gy, const int32_t* acc, int64_t M,
 fqt1_status fqt1_ste_clip(const float* x, float* dx, int64_t n, float t, void* stream);
 
 /* ----------------------------------------------------------- gradient side */
+/* Prepare a workspace of fqt1_agp_quantize_grad / fqt1_scq_quantize: fill its
+ * ws_bytes bytes with 0xFF on `stream` (the initial value of the range keys,
+ * which both take atomicMin).  Needed once per buffer: every call that returns
+ * FQT1_OK leaves the keys it used at 0xFF again (the selection kernel resets
+ * each key after reading it), so one workspace serves any sequence of calls and
+ * shapes that fit it.  Call it again after a call that failed once its kernels
+ * had been launched (a launch error), as that may leave keys behind.
+ * Errors: FQT1_ERR_INVALID_ARG for a null ws or ws_bytes 0; FQT1_ERR_CUDA if
+ * the fill cannot be queued. */
+fqt1_status fqt1_scq_workspace_init(void* ws, size_t ws_bytes, void* stream);
+
 /* AGP on one grouping (Sec. 5.2): ranges of G = gy (.) gamma (gamma may be
  * NULL), keep probabilities, masks, and stochastic rounding of the kept
  * groups to `bits`-bit codes with scales S' and zero points Z'.
  * g: [M, D] fp32 row-major.  group_axis 0 = sample groups (PSQ: rounding takes
  * word m*D + j of generator stream 0, masks stream 2), 1 = channels (PCQ: word
  * j*M + m of stream 1, masks stream 3).
- * ws: fqt1_workspace_size(0, ...) bytes. */
+ * ws: fqt1_workspace_size(0, ...) bytes, initialised by fqt1_scq_workspace_init
+ * (a workspace holding anything else gives wrong ranges). */
 fqt1_status fqt1_agp_quantize_grad(const float* g, int64_t M, int64_t D, int32_t group_axis, const float* gamma,
                                    const fqt1_agp_params* p, fqt1_qgrad* out, void* ws, size_t ws_bytes,
                                    int32_t* dev_status, void* stream);
@@ -191,8 +203,11 @@ fqt1_status fqt1_scq_quantize(const float* g, int64_t M, int64_t D, const float*
  *  - The first call on a device (the device current on the calling thread,
  *    which must own `stream`) looks up the array's device address; make that
  *    first call before any stream capture.
- *  - Every call uses the same array and resets the part it needs; calls whose
- *    work overlaps on the GPU (concurrent streams) race on it.
+ *  - The array is filled with 0xFF by the first call on the device that is not
+ *    captured into a graph (until then by each captured call, as a node of its
+ *    graph); every call leaves the part it used at 0xFF, as a workspace after
+ *    fqt1_scq_workspace_init.  Calls whose work overlaps on the GPU (concurrent
+ *    streams) race on it.
  *  - Allocates nothing: no cudaMalloc / cudaFree or allocating library call.
  * All other arguments, results and errors are those of fqt1_scq_quantize. */
 #define FQT1_NOALLOC_SCRATCH_KEYS 16384

@@ -106,7 +106,7 @@ class _BinaryProduct(torch.autograd.Function):
         cap_c = fqt1.kept_capacity(D, q.bits_c, q.mode_c)
         psq = fqt1.QGradBuffers(M // rpg, cap_s, cap_s * rpg, D, dev)
         pcq = fqt1.QGradBuffers(D, cap_c, cap_c, M, dev)
-        ws = torch.empty(fqt1.workspace_size(0, M, D, K, rpg), dtype=torch.uint8, device=dev)
+        ws = fqt1.scq_workspace(M, D, K, rpg, dev)
         status = torch.zeros(4, dtype=torch.int32, device=dev)
         fqt1.scq_quantize(gy2, M, D, g, p_s, p_c, psq, pcq, ws, status)
         dx = dw = dgamma = dbias = None

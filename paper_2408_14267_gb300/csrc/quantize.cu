@@ -121,8 +121,8 @@ __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
 
 // --------------------------------------------------------------- selection
 struct SelectArgs {
-  const uint32_t* kmin;
-  const uint32_t* kmax;
+  uint32_t* kmin;  // the range keys of the grouping; reset to 0xFFFFFFFF once read
+  uint32_t* kmax;
   int32_t n, bits, mode, capacity;
   uint64_t seed;
   uint32_t stream;
@@ -218,6 +218,10 @@ __global__ void __launch_bounds__(NT) select_kernel(SelectArgs a0, SelectArgs a1
   for (int i = tid; i < n; i += NT) {
     const float z = ordered_to_float(a.kmin[i]);
     const float r = __fsub_rn(ordered_to_float(~a.kmax[i]), z);
+    // the keys go back to their initial value for the next call's range pass (the only other
+    // reader of them, which runs before this kernel), so no call needs to fill them first
+    a.kmin[i] = 0xFFFFFFFFu;
+    a.kmax[i] = 0xFFFFFFFFu;
     o.group_min[i] = z;
     o.group_range[i] = r;
     rf[i] = r;
@@ -709,8 +713,8 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
   uint32_t* cmin = smin + ns;
   uint32_t* smax = cmin + D;
   uint32_t* cmax = smax + ns;
-  // min keys and complemented max keys both start at 0xFFFFFFFF and both take atomicMin
-  FQT1_CUDA_TRY(cudaMemsetAsync(smin, 0xFF, sizeof(uint32_t) * 2 * (ns + D), s));
+  // min keys and complemented max keys start at 0xFFFFFFFF (fqt1_scq_workspace_init, then the
+  // selection kernel of every call resets the keys it read) and both take atomicMin
 
   const bool vec = (D % 4) == 0;
   RangeArgs ra{g, gamma, M, D, rpg, psq ? smin : nullptr, psq ? smax : nullptr, pcq ? cmin : nullptr,
@@ -724,7 +728,7 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
   SelectArgs sa[2];
   int nsel = 0;
   int npad_max = 1;
-  auto add_sel = [&](const fqt1_agp_params* p, fqt1_qgrad* q, const uint32_t* kmin, const uint32_t* kmax, int n,
+  auto add_sel = [&](const fqt1_agp_params* p, fqt1_qgrad* q, uint32_t* kmin, uint32_t* kmax, int n,
                      uint32_t stream) {
     SelectArgs x;
     x.kmin = kmin; x.kmax = kmax; x.n = n; x.bits = p->bits; x.mode = p->mode;
@@ -773,6 +777,12 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
   return FQT1_OK;
 }
 
+extern "C" fqt1_status fqt1_scq_workspace_init(void* ws, size_t ws_bytes, void* stream) {
+  if (!ws || ws_bytes == 0) return FQT1_ERR_INVALID_ARG;
+  FQT1_CUDA_TRY(cudaMemsetAsync(ws, 0xFF, ws_bytes, (cudaStream_t)stream));
+  return FQT1_OK;
+}
+
 extern "C" fqt1_status fqt1_agp_quantize_grad(const float* g, int64_t M, int64_t D, int32_t group_axis,
                                               const float* gamma, const fqt1_agp_params* p, fqt1_qgrad* out,
                                               void* ws, size_t ws_bytes, int32_t* dev_status, void* stream) {
@@ -801,17 +811,21 @@ extern "C" fqt1_status fqt1_scq_quantize(const float* g, int64_t M, int64_t D, c
 // the step path.  For them the scratch of the range pass (the ordered min / max
 // keys of every sample group and channel) lives in a fixed array compiled into
 // this library instead of a caller buffer.  The array is shared by every call on
-// a device and keeps what the last call left in it; the keys are reset at the
-// start of each call, so only calls that overlap on the GPU (e.g. on two
-// streams at once) interfere, and such calls race.
+// a device; it is filled with 0xFF once (by the first call on the device that is
+// not being captured into a graph, or by each captured call until then) and every
+// call leaves it so, like a workspace after fqt1_scq_workspace_init.  Only calls
+// that overlap on the GPU (e.g. on two streams at once) interfere, and such calls
+// race.
 static __device__ __align__(256) uint32_t g_scq_scratch[FQT1_NOALLOC_SCRATCH_KEYS];
 
 static std::mutex g_scq_scratch_mu;
 static void* g_scq_scratch_dev[64];  // device address of g_scq_scratch, per device ordinal
+static bool g_scq_scratch_ready[64];  // filled with 0xFF outside a graph capture
 
-// Device address of the scratch array on the calling thread's current device.
-// The first call on a device looks it up (cudaGetSymbolAddress) and caches it.
-static fqt1_status scq_scratch_address(void** out) {
+// Device address of the scratch array on the calling thread's current device, filled with
+// 0xFF on stream s until a fill has run outside a graph capture.  The first call on a device
+// looks the address up (cudaGetSymbolAddress) and caches it.
+static fqt1_status scq_scratch_address(void** out, cudaStream_t s) {
   int dev = -1;
   FQT1_CUDA_TRY(cudaGetDevice(&dev));
   if (dev < 0 || dev >= 64) return FQT1_ERR_UNSUPPORTED;
@@ -820,6 +834,12 @@ static fqt1_status scq_scratch_address(void** out) {
     void* p = nullptr;
     FQT1_CUDA_TRY(cudaGetSymbolAddress(&p, g_scq_scratch));
     g_scq_scratch_dev[dev] = p;
+  }
+  if (!g_scq_scratch_ready[dev]) {
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    FQT1_CUDA_TRY(cudaStreamIsCapturing(s, &cap));
+    FQT1_CUDA_TRY(cudaMemsetAsync(g_scq_scratch_dev[dev], 0xFF, sizeof(g_scq_scratch), s));
+    if (cap == cudaStreamCaptureStatusNone) g_scq_scratch_ready[dev] = true;
   }
   *out = g_scq_scratch_dev[dev];
   return FQT1_OK;
@@ -841,7 +861,7 @@ extern "C" fqt1_status fqt1_scq_quantize_noalloc(const float* g, int64_t M, int6
     return FQT1_ERR_UNSUPPORTED;
   }
   void* scratch = nullptr;
-  const fqt1_status st = scq_scratch_address(&scratch);
+  const fqt1_status st = scq_scratch_address(&scratch, (cudaStream_t)stream);
   if (st != FQT1_OK) return st;
   return quantize_impl(g, M, D, gamma, p_sample, psq, p_channel, pcq, scratch,
                        sizeof(uint32_t) * FQT1_NOALLOC_SCRATCH_KEYS, dev_status, (cudaStream_t)stream);

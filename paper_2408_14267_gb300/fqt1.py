@@ -50,6 +50,7 @@ _SIGS = {
     "fqt1_scale_bias_grad": (C.c_int, [_VP, _VP, _I64, _I64, _VP, _VP, _VP, C.c_size_t, _VP]),
     "fqt1_ste_clip": (C.c_int, [_VP, _VP, _I64, C.c_float, _VP]),
     "fqt1_agp_quantize_grad": (C.c_int, [_VP, _I64, _I64, _I32, _VP, _VP, _VP, _VP, C.c_size_t, _VP, _VP]),
+    "fqt1_scq_workspace_init": (C.c_int, [_VP, C.c_size_t, _VP]),
     "fqt1_scq_quantize": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, C.c_size_t, _VP, _VP]),
     "fqt1_scq_quantize_noalloc": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, _VP]),
     "fqt1_bwd_input_gemm": (C.c_int, [_VP, _VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
@@ -120,6 +121,20 @@ def kernel_launches():
 
 def workspace_size(which, M, D, K, rows_per_group):
     return lib().fqt1_workspace_size(which, M, D, K, rows_per_group)
+
+
+def scq_workspace(M, D, K, rows_per_group, device, stream=None):
+    """A workspace of fqt1_agp_quantize_grad / fqt1_scq_quantize, filled with 0xFF by
+    fqt1_scq_workspace_init; the calls leave it so, and it can be reused for any shape it fits."""
+    import torch
+    ws = torch.empty(workspace_size(0, M, D, K, rows_per_group), dtype=torch.uint8, device=device)
+    scq_workspace_init(ws, stream)
+    return ws
+
+
+def scq_workspace_init(ws, stream=None):
+    _check(lib().fqt1_scq_workspace_init(_p(ws), ws.numel() * ws.element_size(), _s(stream)),
+           "fqt1_scq_workspace_init")
 
 
 # ------------------------------------------------------------ entry points

@@ -74,7 +74,7 @@ class LayerStep:
         self.cap_c = fqt1.kept_capacity(D, wl["bits_c"], wl["mode_c"])
         self.psq = fqt1.QGradBuffers(n_s, self.cap_s, self.cap_s * rpg, D, dev)
         self.pcq = fqt1.QGradBuffers(D, self.cap_c, self.cap_c, M, dev)
-        self.ws = torch.empty(fqt1.workspace_size(0, M, D, K, rpg), dtype=torch.uint8, device=dev)
+        self.ws = fqt1.scq_workspace(M, D, K, rpg, dev)
         self.dev_status = torch.zeros(4, **i32)
         self.acc_dx = torch.empty(max(self.cap_s * rpg, 1), K, **i32)
         self.dx = torch.empty(*(self.x.shape), **f32)

@@ -280,6 +280,42 @@ def test_single_branch_entry_point_matches_scq():
         assert torch.equal(q.codes[:rows], ref.codes[:rows]) and torch.equal(q.p_hat, ref.p_hat)
 
 
+def test_workspace_keys_restored_after_each_call():
+    """Every quantizer call leaves its range keys at the 0xFF of fqt1_scq_workspace_init
+    (the selection kernel resets each key it reads), so one workspace, initialised once,
+    gives the results of a fresh one on repeated calls, other shapes and single branches."""
+    from paper_2408_14267_gb300 import fqt1
+    from paper_2408_14267_gb300 import workloads as wl
+    from paper_2408_14267_gb300.layer import LayerStep
+    steps = [LayerStep(wl.resnet18_cifar_conv()), LayerStep(wl.linear_small()),
+             LayerStep(linear_case(100, 48, 72, 4, 2, SYS, seed=11))]
+    ws = fqt1.scq_workspace(max(s.M for s in steps), max(s.D for s in steps), 0, 1, "cuda")
+
+    def same(a, b, rows):
+        c = a.count()
+        assert c == b.count()
+        for name in ("group_min", "group_range", "p_hat", "slot_of_group"):
+            assert torch.equal(getattr(a, name), getattr(b, name)), name
+        assert torch.equal(a.scale[:c], b.scale[:c]) and torch.equal(a.zero[:c], b.zero[:c])
+        assert torch.equal(a.codes[: c * rows], b.codes[: c * rows])
+
+    for st in steps + steps[:1]:
+        st.dev_status.zero_()
+        fqt1.scq_quantize(st.gy, st.M, st.D, st.gamma, st.p_s, st.p_c, st.psq, st.pcq, st.ws, st.dev_status)
+        psq = fqt1.QGradBuffers(st.psq.n, st.psq.capacity, st.psq.capacity * st.rpg, st.D)
+        pcq = fqt1.QGradBuffers(st.pcq.n, st.pcq.capacity, st.pcq.capacity, st.M)
+        fqt1.scq_quantize(st.gy, st.M, st.D, st.gamma, st.p_s, st.p_c, psq, pcq, ws, st.dev_status)
+        torch.cuda.synchronize()
+        assert bool((ws == 255).all()) and bool((st.ws == 255).all())
+        same(psq, st.psq, st.rpg)
+        same(pcq, st.pcq, 1)
+        q = fqt1.QGradBuffers(st.pcq.n, st.pcq.capacity, st.pcq.capacity, st.M)
+        fqt1.agp_quantize_grad(st.gy, st.M, st.D, 1, st.gamma, st.p_c, q, ws, st.dev_status)
+        torch.cuda.synchronize()
+        assert bool((ws == 255).all())
+        same(q, st.pcq, 1)
+
+
 def test_nonfinite_gradient_sets_status():
     from paper_2408_14267_gb300.layer import LayerStep
     w = linear_case(32, 32, 16, 1, 2, SYS, seed=10)
@@ -337,7 +373,7 @@ def test_table5_shapes_exact(M, K, N):
     p = fqt1.AgpParams(4, SYS, 11, 1)
     cap = fqt1.kept_capacity(M, 4, SYS)
     q = fqt1.QGradBuffers(M, cap, cap, K, dev)
-    ws = torch.empty(fqt1.workspace_size(0, M, K, N, 1), dtype=torch.uint8, device=dev)
+    ws = fqt1.scq_workspace(M, K, N, 1, dev)
     status = torch.zeros(4, dtype=torch.int32, device=dev)
     fqt1.agp_quantize_grad(torch.from_numpy(g).cuda(), M, K, 0, None, p, q, ws, status)
     acc4 = torch.empty(cap, N, dtype=torch.int32, device=dev)
