@@ -35,10 +35,10 @@ SMS, POPC_PER_CLK_SM = 152, 16
 # stage is the sum of its range, selection and quantize kernels).  They are
 # valid only for the kernel sources they were taken on: TRAFFIC_SOURCES is the sha256 prefix of
 # paper_2408_14267_gb300/csrc at that capture; any other source tree reports traffic = null.
-TRAFFIC_SOURCES = "8858dee0c727824d"
-TRAFFIC_BYTES = {"pack_w": 2.378752e+06, "im2col": 8.418304e+06, "fwd_gemm": 2.512384e+06,
-                 "scq_quantize": 1.693261e+07, "bwd_input_fold": 6.845440e+05,
-                 "bwd_weight_gemm": 2.977280e+06}
+TRAFFIC_SOURCES = "4f6e3a0bc012d230"
+TRAFFIC_BYTES = {"pack_w": 2.379264e+06, "im2col": 8.418304e+06, "fwd_gemm": 2.512384e+06,
+                 "scq_quantize": 1.693517e+07, "bwd_input_fold": 6.835200e+05,
+                 "bwd_weight_gemm": 2.980096e+06}
 
 
 def sources_sha():
