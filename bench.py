@@ -197,6 +197,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="fqt1", choices=["fqt1", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--implicit", action="store_true",
+                    help="implicit-GEMM forward (pixel-major sign(X), no unfolded row packing)")
     ap.add_argument("--profile", type=int, default=0, metavar="N",
                     help="only run --warmup + N eager steps (for ncu), print nothing")
     ap.add_argument("--table5", action="store_true",
@@ -234,7 +236,7 @@ def main():
     from paper_2408_14267_gb300.layer import LayerStep
 
     wl = workloads.resnet18_cifar_conv()
-    st = LayerStep(wl, device=f"cuda:{local_rank}", keep_acc=False)
+    st = LayerStep(wl, device=f"cuda:{local_rank}", keep_acc=False, implicit=args.implicit)
     stream = torch.cuda.Stream()
     if args.profile:
         with torch.cuda.stream(stream):
@@ -380,7 +382,9 @@ def main():
                            "timing": "CUDA-graph replay of the whole step (three stream branches: pack W | "
                                      "pack X + forward + grad_weight | SCQ + grad_input with the Folder in its "
                                      "epilogue), CUDA events on the launching stream",
-                           "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU"},
+                           "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU",
+                           "forward": "implicit GEMM (pixel-major sign(X))" if st.implicit
+                           else "1-bit unfolded X_u"},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
                 "clocks": clocks, "stage_ms": {k: round(v, 5) for k, v in stage_ms.items()}}
         print(json.dumps(line))

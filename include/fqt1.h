@@ -124,7 +124,43 @@ fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t H, int32_t
                         int32_t stride, int32_t pad, uint32_t* row_bits, uint32_t* col_bits, int32_t* colsum,
                         void* stream);
 
-/* Binarized forward GEMM (Sec. 5.1, App. C "binary multiplication"):
+/* Implicit-GEMM convolution forward (the Unfolder of App. C left implicit).
+ * The binary product of a stride-1 "same" convolution (kh = kw = 2 pad + 1) is
+ * computed without materializing X_u: the contraction runs over kernel taps
+ * and channels, k' = t C + c for tap t = i kw + j.  Each A tile is read from
+ * pixel-major sign words, shifted by the tap, and taps in the zero padding read
+ * sign -1 (as in fqt1_im2col).  The integer result equals fqt1_fwd_gemm on the
+ * unfolded matrix, since it is the same sum in another order.
+ *
+ * fqt1_pack_pixels: x [N, C, H, W] fp32 -> x_pix [N*H*W][fqt1_packed_words(C)];
+ *   word b of pixel p = (n H + h) W + w has bit e set iff x[n, 32 b + e, h, w] > 0.
+ *   C must be a multiple of 128 (FQT1_ERR_UNSUPPORTED otherwise); x_pix 16-byte
+ *   aligned.
+ * fqt1_pack_weight_taps: w [D, C, kh, kw] fp32 -> w_taps
+ *   [D][fqt1_packed_words(kh*kw*C)]; bit e of word t C / 32 + b of row d is set
+ *   iff w[d, 32 b + e, i, j] > 0 (t = i kw + j); padding words are 0.  C must be
+ *   a multiple of 32.
+ * fqt1_conv_implicit_supported: 1 if fqt1_conv_fwd_implicit accepts the shape:
+ *   stride 1, kh = kw = 2 pad + 1, C a multiple of 128, kh kw C < 2^24, and the
+ *   output pixels tile by 128 rows as whole images (H W divides 128) or as whole
+ *   image rows (W divides 128 and 128 / W divides H).  Otherwise 0.
+ * fqt1_conv_fwd_implicit: acc[m, d] = sum_k sign(X_u)[m, k] sign(W)[d, k] for
+ *   output pixel m = (n H + h) W + w; y = gamma[d] acc (+ bias[d]) as in
+ *   fqt1_fwd_gemm_bias.  acc may be NULL; gamma and y are required.
+ *   FQT1_ERR_UNSUPPORTED for a shape that fqt1_conv_implicit_supported rejects.
+ * Buffers are caller-owned device memory and all three calls are asynchronous
+ * on `stream`. */
+fqt1_status fqt1_pack_pixels(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, uint32_t* x_pix,
+                             void* stream);
+fqt1_status fqt1_pack_weight_taps(const float* w, int64_t D, int32_t C, int32_t kh, int32_t kw, uint32_t* w_taps,
+                                  void* stream);
+int32_t fqt1_conv_implicit_supported(int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw,
+                                     int32_t stride, int32_t pad);
+fqt1_status fqt1_conv_fwd_implicit(const uint32_t* x_pix, const uint32_t* w_taps, int32_t N, int32_t C, int32_t H,
+                                   int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad, int64_t D,
+                                   const float* gamma, const float* bias, int32_t* acc, float* y, void* stream);
+
+/* Binarized forward GEMM (Sec. 5.1, App. C "binary multiplication"):/* Binarized forward GEMM (Sec. 5.1, App. C "binary multiplication"):
  * acc[m, j] = sum_k sign(X)[m, k] sign(W)[j, k], y[m, j] = gamma[j] * acc[m, j] (fp32).
  * sx_row: [M][words(K)], sw_row: [D][words(K)], gamma: [D].
  * acc: [M][D] int32 or NULL; y: [M][D] fp32 (row stride D). */

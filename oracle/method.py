@@ -162,7 +162,42 @@ def fold_int(acc_u, N, C, H, W, kh, kw, stride, pad):
     return out[:, :, pad:pad + H, pad:pad + W]
 
 
+def pixel_signs(x):
+    """Pixel-major signs of x [N, C, H, W]: row p = (n H + h) W + w is sign(x[n, :, h, w]).
+    The operand layout of the implicit convolution product below."""
+    x = np.asarray(x, dtype=f32)
+    N, C, H, W = x.shape
+    return sign(x.transpose(0, 2, 3, 1).reshape(N * H * W, C))
+
+
+def tap_major_signs(w):
+    """Signs of w [D, C, kh, kw] with the contraction index k' = t C + c of tap t = i kw + j."""
+    w = np.asarray(w, dtype=f32)
+    D, C, kh, kw = w.shape
+    return sign(w.transpose(0, 2, 3, 1).reshape(D, kh * kw * C))
+
+
+def implicit_conv_acc(x, w, pad):
+    """Binary product of a stride-1 convolution with the Unfolder of App. C left implicit:
+    acc[(n Ho + oh) Wo + ow, d] = sum over taps (i, j), then channels c, of
+    sign(x)[n, c, oh + i - pad, ow + j - pad] sign(w)[d, c, i, j], where a tap in the
+    zero padding has sign -1 (R1).  Exact int64."""
+    x = np.asarray(x, dtype=f32)
+    N, C, H, W = x.shape
+    D, _, kh, kw = np.asarray(w).shape
+    Ho, Wo = conv_out_hw(H, W, kh, kw, 1, pad)
+    sx = np.full((N, C, H + 2 * pad, W + 2 * pad), -1, dtype=np.int64)
+    sx[:, :, pad:pad + H, pad:pad + W] = sign(x)
+    sw = sign(w).astype(np.int64)
+    acc = np.zeros((N, Ho, Wo, D), dtype=np.int64)
+    for i in range(kh):
+        for j in range(kw):
+            acc += np.einsum("nchw,dc->nhwd", sx[:, :, i:i + Ho, j:j + Wo], sw[:, :, i, j])
+    return acc.reshape(N * Ho * Wo, D)
+
+
 # --------------------------------------------------------------------------
+# Backward, step 1: group ranges# --------------------------------------------------------------------------
 # Backward, step 1: group ranges (Sec. 3.2, PSQ Sec. 5.2, PCQ Sec. 5.3)
 # --------------------------------------------------------------------------
 def grad_to_quantize(gy, gamma):

@@ -263,6 +263,27 @@ extern "C" fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_
   return fqt1_fwd_gemm_bias(sx_row, sw_row, M, D, K, gamma, nullptr, acc, y, stream);
 }
 
+extern "C" int32_t fqt1_conv_implicit_supported(int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw,
+                                                int32_t stride, int32_t pad) {
+  return implicit_conv_supported(N, C, H, W, kh, kw, stride, pad) ? 1 : 0;
+}
+
+extern "C" fqt1_status fqt1_conv_fwd_implicit(const uint32_t* x_pix, const uint32_t* w_taps, int32_t N, int32_t C,
+                                              int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,
+                                              int32_t pad, int64_t D, const float* gamma, const float* bias,
+                                              int32_t* acc, float* y, void* stream) {
+  if (!x_pix || !w_taps || !gamma || !y || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 ||
+      pad < 0 || D < 1)
+    return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(x_pix) || !aligned16(w_taps) || !aligned16(gamma) || !aligned16(y) || (acc && !aligned16(acc)) ||
+      (bias && !aligned16(bias)))
+    return FQT1_ERR_MISALIGNED;
+  if (use_popcount_path() || !implicit_conv_supported(N, C, H, W, kh, kw, stride, pad)) return FQT1_ERR_UNSUPPORTED;
+  FQT1_CUDA_TRY(launch_fwd_implicit_tc(x_pix, w_taps, N, C, H, W, kh, pad, D, gamma, bias, acc, y, nullptr,
+                                       (cudaStream_t)stream));
+  return FQT1_OK;
+}
+
 extern "C" fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t* sw_col, const int32_t* colsum_w,
                                            int64_t M, int64_t D, int64_t K, const fqt1_agp_params* p,
                                            int32_t* acc, float* dx, void* stream) {

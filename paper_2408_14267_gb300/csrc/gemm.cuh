@@ -14,6 +14,14 @@ cudaError_t launch_codes_gemm_simt(int bits, const uint8_t* Q, int64_t ldq, cons
 struct TcArgs;
 cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64_t D, int64_t K, const float* gamma,
                           const float* bias, int32_t* acc, float* y, int32_t* status, cudaStream_t s);
+// Implicit-GEMM forward of a stride-1 "same" convolution from pixel-major sign words xp
+// [N][H][W][C / 32] and tap-major weight signs wt [D][words(k k C)] (k' = t C + c); the shapes
+// implicit_conv_supported accepts.
+bool implicit_conv_supported(int64_t N, int64_t C, int64_t H, int64_t W, int64_t kh, int64_t kw, int64_t stride,
+                             int64_t pad);
+cudaError_t launch_fwd_implicit_tc(const uint32_t* xp, const uint32_t* wt, int N, int C, int H, int W, int k, int pad,
+                                   int64_t D, const float* gamma, const float* bias, int32_t* acc, float* y,
+                                   int32_t* status, cudaStream_t s);
 cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
                                    int64_t rows_per_count, const uint32_t* Sg, int64_t n_s, int64_t L, int epi,
                                    int splits, int32_t* acc, float* out, int64_t ldo, const int32_t* kept_idx,

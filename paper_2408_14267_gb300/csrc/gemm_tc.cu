@@ -67,6 +67,11 @@ struct TcArgs {
   // EPI_FWD / EPI_ACC32: bit 0 = y, bit 1 = acc leave through TMA stores (tmY / tmAcc)
   int tma_out;
   int fN;  // EPI_FOLD: samples (pruned ones are zeroed by the kernel)
+  // implicit-GEMM forward of a stride-1 "same" convolution (impl = 1): A comes from the
+  // pixel-major sign words [N][H][W][C / 32] through a 4-D tensor map, one box per 128-channel
+  // sub-tile of one kernel tap, shifted by the tap; the contraction index is k' = t C + c.
+  // A box covers 2^isb consecutive sub-tiles of one tap (rows of 16 * 2^isb bytes).
+  int impl, iC, ikw, ikhw, ipad, iW, iHW, isb;
   // EPI_FOLD divisors (host-built): kh kw, W, kw, H W, stride, fcb H W
   FastDiv fd_khw, fd_w, fd_kw, fd_hw, fd_s, fd_cbhw;
   // EPI_CRED: the cluster's partial tiles are summed into acc (int32, ldo) and dequantized into
@@ -124,6 +129,16 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
           smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+
+// 4-D tile load (coordinates innermost first; a box reaching outside the tensor reads zeros).
+__device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, uint64_t* bar, int c0, int c1, int c2,
+                                            int c3) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5, %6}], "
+      "[%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
       : "memory");
 }
 
@@ -399,6 +414,21 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
 #pragma unroll
           for (int h = 0; h < KSUB; ++h)  // one 128-byte-swizzled box per sub-tile
             tma_load_2d(rawA(s) + h * (kBM * kBK), &tmA, &raw_full[s], (kt * KSUB + h) * kBK, (int)m0);
+        } else if (!A_CODES && a.impl) {
+          // implicit convolution: box b = sub-tiles b 2^isb .. + 2^isb - 1, 128 2^isb channels
+          // of one tap t; the box of the tile's output pixels shifted by (i - pad, j - pad), so
+          // that a tap in the padding reads the fill value 0 (sign -1).  Boxes past the
+          // contraction length load a valid box whose products are never issued.
+          const int64_t pix_n0 = m0 / a.iHW, pix_h0 = (m0 - pix_n0 * a.iHW) / a.iW;
+          const int sb = 1 << a.isb;
+          for (int h = 0; h < KSUB; h += sb) {
+            const int64_t kq = ((int64_t)kt * KSUB + h) * kBK;
+            const int t = kq < a.L ? (int)(kq / a.iC) : a.ikhw - 1;
+            const int cw = kq < a.L ? (int)((kq - (int64_t)t * a.iC) >> 5) : 0;
+            const int ti = t / a.ikw, tj = t - ti * a.ikw;
+            tma_load_4d(rawA(s) + h * (kBM * 16), &tmA, &raw_full[s], cw, tj - a.ipad,
+                        (int)pix_h0 + ti - a.ipad, (int)pix_n0);
+          }
         } else {
           tma_load_2d(rawA(s), &tmA, &raw_full[s], kt * KSUB * (kBK / 32), (int)m0);
         }
@@ -493,7 +523,12 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
                 tmem_st32(acol + (kBK / 4) * h, o);
               }
             } else {
-              const uint4 w4 = *reinterpret_cast<const uint4*>(rawA(sr) + arow * S::kRawRow + 16 * h);
+              // raw rows: 16 bytes per sub-tile, interleaved per row (2-D box), or per row of a
+              // box of 2^isb sub-tiles (implicit convolution)
+              const int hb = (h >> a.isb) << a.isb;
+              const unsigned char* rp = a.impl ? rawA(sr) + hb * (kBM * 16) + (arow << (4 + a.isb)) + 16 * (h - hb)
+                                               : rawA(sr) + arow * S::kRawRow + 16 * h;
+              const uint4 w4 = *reinterpret_cast<const uint4*>(rp);
               const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
               for (int j = 0; j < 32; ++j) o[j] = signs4((wv[j >> 3] >> (4 * (j & 7))) & 15u);
@@ -1072,17 +1107,16 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
   return cudaGetLastError();
 }
 
-// Forward: A = sign(X) rows [M][words(K)], B = sign(W) rows [D][words(K)].
-cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64_t D, int64_t K, const float* gamma,
-                          const float* bias, int32_t* acc, float* y, int32_t* status, cudaStream_t s) {
+// Forward with a prepared A map: B = sign(W) rows [D][words(K)]; a carries the implicit-
+// convolution fields (impl = 0 for a plain A = sign(X) rows map).
+static cudaError_t launch_fwd_common(const CUtensorMap& ma, TcArgs a, const uint32_t* B, int64_t M, int64_t D,
+                                     int64_t K, const float* gamma, const float* bias, int32_t* acc, float* y,
+                                     int32_t* status, cudaStream_t s) {
   using S = TcSmem<false, false, 128>;
   const int64_t ldw = fqt1_packed_words(K);
-  CUtensorMap ma, mb;
-  if (!make_map(&ma, A, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, M, ldw * 4, 4 * S::KSUB, kBM,
-                CU_TENSOR_MAP_SWIZZLE_NONE) ||
-      !make_map(&mb, B, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, D, ldw * 4, 4 * S::KSUB, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+  CUtensorMap mb;
+  if (!make_map(&mb, B, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, D, ldw * 4, 4 * S::KSUB, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
     return cudaErrorInvalidValue;
-  TcArgs a{};
   a.M = M; a.N = D; a.L = K; a.count = nullptr; a.rows_per_count = 1;
   a.k_tiles = (int)((K + kBK * S::KSUB - 1) / (kBK * S::KSUB)); a.tiles_per_split = a.k_tiles;
   a.epi = EPI_FWD; a.gamma = gamma; a.bias = bias; a.y = y; a.acc = acc; a.ldo = D; a.status = status;
@@ -1099,6 +1133,57 @@ cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64
     }
   }
   return launch_tc<false, false, 128>(ma, mb, a, 1, s, &my, &macc);
+}
+
+// Forward: A = sign(X) rows [M][words(K)], B = sign(W) rows [D][words(K)].
+cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64_t D, int64_t K, const float* gamma,
+                          const float* bias, int32_t* acc, float* y, int32_t* status, cudaStream_t s) {
+  using S = TcSmem<false, false, 128>;
+  const int64_t ldw = fqt1_packed_words(K);
+  CUtensorMap ma;
+  if (!make_map(&ma, A, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, M, ldw * 4, 4 * S::KSUB, kBM,
+                CU_TENSOR_MAP_SWIZZLE_NONE))
+    return cudaErrorInvalidValue;
+  return launch_fwd_common(ma, TcArgs{}, B, M, D, K, gamma, bias, acc, y, status, s);
+}
+
+// Implicit-GEMM forward of a stride-1 "same" convolution (kh = kw = 2 pad + 1, C a multiple of
+// 128).  A tile of 128 output pixels is whole images (H W divides 128) or whole image rows (W
+// divides 128 and the rows of a tile divide H); its A sub-tiles are 4-D boxes of the pixel-major
+// sign words xp [N][H][W][C / 32], one per (tap, 128 channels).  B = tap-major sign(W) rows.
+bool implicit_conv_supported(int64_t N, int64_t C, int64_t H, int64_t W, int64_t kh, int64_t kw, int64_t stride,
+                             int64_t pad) {
+  if (N < 1 || C < 1 || H < 1 || W < 1 || stride != 1 || kh != kw || kh != 2 * pad + 1 || C % 128 != 0) return false;
+  if (C * kh * kw >= (1ll << 24) || N * H * W >= (1ll << 31) || (N * H * W + kBM - 1) / kBM > 65535) return false;
+  const int64_t HW = H * W;
+  if (HW <= kBM) return kBM % HW == 0;
+  return W <= kBM && kBM % W == 0 && H % (kBM / W) == 0;
+}
+
+cudaError_t launch_fwd_implicit_tc(const uint32_t* xp, const uint32_t* wt, int N, int C, int H, int W, int k, int pad,
+                                   int64_t D, const float* gamma, const float* bias, int32_t* acc, float* y,
+                                   int32_t* status, cudaStream_t s) {
+  auto fn = encode_fn();
+  if (!fn) return cudaErrorInvalidValue;
+  const int64_t cw = fqt1_packed_words(C), HW = (int64_t)H * W;
+  const uint32_t box_h = HW <= kBM ? (uint32_t)H : (uint32_t)(kBM / W);
+  const uint32_t box_n = HW <= kBM ? (uint32_t)(kBM / HW) : 1u;
+  // sub-tiles per box: the largest power of two (<= KSUB) dividing the 128-channel blocks of a tap
+  using S = TcSmem<false, false, 128>;
+  int isb = 0;
+  while ((1 << (isb + 1)) <= S::KSUB && (C / 128) % (1 << (isb + 1)) == 0) ++isb;
+  cuuint64_t dims[4] = {(cuuint64_t)cw, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
+  cuuint64_t strides[3] = {(cuuint64_t)(cw * 4), (cuuint64_t)(cw * 4 * W), (cuuint64_t)(cw * 4 * HW)};
+  cuuint32_t box[4] = {4u << isb, (cuuint32_t)W, box_h, box_n};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUtensorMap ma;
+  if (fn(&ma, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, const_cast<uint32_t*>(xp), dims, strides, box, estr,
+         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
+  TcArgs a{};
+  a.impl = 1; a.iC = C; a.ikw = k; a.ikhw = k * k; a.ipad = pad; a.iW = W; a.iHW = (int)HW; a.isb = isb;
+  return launch_fwd_common(ma, a, wt, (int64_t)N * HW, D, (int64_t)C * k * k, gamma, bias, acc, y, status, s);
 }
 
 // Codes x signs: out[r, n] = sum_j Q[r, j] S[n, j], Q [rows][ld] uint8 (valid rows *count * rpc),

@@ -574,9 +574,11 @@ __global__ void __launch_bounds__(256) unfold_same_kernel(UnfoldSameArgs a) {
       }
       colw = (uint32_t)(v >> o) & bit_range(plo - p0, phi - p0) & cmask;
     }
-    const uint32_t roww = warp_transpose32(colw, lane);
-    const int px = 32 * s + lane;
-    rw_s[px * 8 + (warp ^ ((px >> 2) & 7))] = roww;
+    if (a.row_bits) {  // uniform: a caller that needs only the column packing skips the transposes
+      const uint32_t roww = warp_transpose32(colw, lane);
+      const int px = 32 * s + lane;
+      rw_s[px * 8 + (warp ^ ((px >> 2) & 7))] = roww;
+    }
     const int kl = 32 * warp + lane;
     cw_s[kl * NSUB + (s ^ ((kl >> kZShift) & (NSUB - 1)))] = colw;
     if (!a.rep) {
@@ -640,6 +642,76 @@ static fqt1_status launch_pack(const Loader& L, uint32_t* row_bits, uint32_t* co
   return FQT1_OK;
 }
 
+
+// ------------------------------------------------------------------ implicit-convolution packings
+// Pixel-major signs of x [N, C, H, W] for the implicit-GEMM forward: word b of pixel
+// p = (n H + h) W + w holds sign(x[n, 32 b + e, h, w]) > 0 at bit e.  A CTA takes 32
+// consecutive pixels (lane = pixel) and 4 blocks of 32 channels (warp = block): 32 loads
+// per lane, each a contiguous run of the plane across the warp, then one word per lane; the
+// 4 words of a pixel leave as one 16-byte store.
+constexpr int kPixBlocks = 4;
+__global__ void __launch_bounds__(32 * kPixBlocks) pack_pixels_kernel(const float* __restrict__ x, int64_t P, int C,
+                                                                      int HW, FastDiv div_hw, int64_t words,
+                                                                      uint32_t* __restrict__ out) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  __shared__ __align__(16) uint32_t w_s[32][kPixBlocks];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t p = (int64_t)blockIdx.x * 32 + lane;
+  const uint32_t pc = (uint32_t)min(p, P - 1);
+  const uint32_t n = div_hw.div(pc);
+  const int cb = blockIdx.y * kPixBlocks + warp;  // C is a multiple of 32 kPixBlocks
+  const float* src = x + ((int64_t)n * C + 32 * cb) * HW + (pc - n * (uint32_t)HW);
+  float v[32];
+#pragma unroll
+  for (int u = 0; u < 32; ++u) v[u] = __ldg(src + (int64_t)u * HW);
+  uint32_t wd = 0;
+#pragma unroll
+  for (int u = 0; u < 32; ++u) wd |= (v[u] > 0.0f ? 1u : 0u) << u;
+  w_s[lane][warp] = wd;
+  __syncthreads();
+  const int64_t q = (int64_t)blockIdx.x * 32 + threadIdx.x;  // one pixel per thread of warp 0
+  if (threadIdx.x < 32 && q < P)
+    *reinterpret_cast<uint4*>(out + q * words + (int64_t)blockIdx.y * kPixBlocks) =
+        *reinterpret_cast<const uint4*>(&w_s[threadIdx.x][0]);
+}
+
+// Tap-major signs of w [D, C, kh, kw] for the implicit-GEMM forward: row d, contraction index
+// k' = t C + c for tap t = i kw + j, i.e. word t C / 32 + b holds sign(w[d, 32 b + e, i, j]) at
+// bit e.  One warp per (d, t); lane = channel within a block of 32, one ballot per block (8
+// loads in flight per lane), lane b keeps word b of its group of 32 blocks.  Words past
+// kh kw C / 32 (the row padding to 16 bytes) are written as 0.
+__global__ void __launch_bounds__(256) pack_weight_taps_kernel(const float* __restrict__ w, int64_t D, int C, int khw,
+                                                               int64_t words, uint32_t* __restrict__ out) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t g = (int64_t)blockIdx.x * 8 + warp;
+  const int64_t d = g / khw;
+  const int t = (int)(g - d * khw);
+  if (d >= D) return;  // warp-uniform
+  const float* src = w + d * (int64_t)C * khw + t;
+  uint32_t* dst = out + d * words + (int64_t)t * (C / 32);
+  const int nb = C / 32;
+  for (int b0 = 0; b0 < nb; b0 += 32) {
+    uint32_t mine = 0;
+    for (int b1 = b0; b1 < min(nb, b0 + 32); b1 += 8) {
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = __ldg(src + (int64_t)(min(b1 + u, nb - 1) * 32 + lane) * khw);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const uint32_t wd = __ballot_sync(0xFFFFFFFFu, v[u] > 0.0f);
+        if (lane == b1 + u - b0) mine = wd;
+      }
+    }
+    if (b0 + lane < nb) dst[b0 + lane] = mine;
+  }
+  if (t == khw - 1) {
+    const int64_t used = (int64_t)khw * nb;
+    for (int64_t e = used + lane; e < words; e += 32) out[d * words + e] = 0u;
+  }
+}
 }  // namespace fqt1
 
 using namespace fqt1;
@@ -775,4 +847,33 @@ extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t
   L.div_hw_out = FastDiv((uint32_t)(Ho * Wo)); L.div_wo = FastDiv((uint32_t)Wo);
   L.div_khw = FastDiv((uint32_t)(kh * kw)); L.div_kw = FastDiv((uint32_t)kw);
   return launch_pack(L, row_bits, col_bits, colsum, s);
+}
+
+extern "C" fqt1_status fqt1_pack_pixels(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, uint32_t* x_pix,
+                                        void* stream) {
+  if (!x || !x_pix || N < 1 || C < 1 || H < 1 || W < 1) return FQT1_ERR_INVALID_ARG;
+  if (C % (32 * kPixBlocks) != 0) return FQT1_ERR_UNSUPPORTED;
+  if (!aligned16(x_pix)) return FQT1_ERR_MISALIGNED;
+  const int64_t P = (int64_t)N * H * W;
+  if ((int64_t)N * C * H * W >= (1ll << 31) || (P + 31) / 32 >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
+  const int64_t words = fqt1_packed_words(C);
+  FQT1_CUDA_TRY(launch_k(pack_pixels_kernel, dim3((unsigned)((P + 31) / 32), (unsigned)(C / (32 * kPixBlocks))),
+                         dim3(32 * kPixBlocks), 0, (cudaStream_t)stream, x, P, (int)C, H * W,
+                         FastDiv((uint32_t)(H * W)), words, x_pix));
+  fqt1_count_launches(1);
+  return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_pack_weight_taps(const float* w, int64_t D, int32_t C, int32_t kh, int32_t kw,
+                                             uint32_t* w_taps, void* stream) {
+  if (!w || !w_taps || D < 1 || C < 1 || kh < 1 || kw < 1) return FQT1_ERR_INVALID_ARG;
+  if (C % 32 != 0) return FQT1_ERR_UNSUPPORTED;
+  if (!aligned16(w_taps)) return FQT1_ERR_MISALIGNED;
+  const int64_t khw = (int64_t)kh * kw;
+  if (D * C * khw >= (1ll << 40) || (D * khw + 7) / 8 >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
+  const int64_t words = fqt1_packed_words(khw * C);
+  FQT1_CUDA_TRY(launch_k(pack_weight_taps_kernel, dim3((unsigned)((D * khw + 7) / 8)), dim3(256), 0,
+                         (cudaStream_t)stream, w, D, (int)C, (int)khw, words, w_taps));
+  fqt1_count_launches(1);
+  return FQT1_OK;
 }

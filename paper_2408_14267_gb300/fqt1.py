@@ -51,6 +51,10 @@ _SIGS = {
     "fqt1_ste_clip": (C.c_int, [_VP, _VP, _I64, C.c_float, _VP]),
     "fqt1_agp_quantize_grad": (C.c_int, [_VP, _I64, _I64, _I32, _VP, _VP, _VP, _VP, C.c_size_t, _VP, _VP]),
     "fqt1_scq_workspace_init": (C.c_int, [_VP, C.c_size_t, _VP]),
+    "fqt1_pack_pixels": (C.c_int, [_VP, _I32, _I32, _I32, _I32, _VP, _VP]),
+    "fqt1_pack_weight_taps": (C.c_int, [_VP, _I64, _I32, _I32, _I32, _VP, _VP]),
+    "fqt1_conv_implicit_supported": (_I32, [_I32] * 8),
+    "fqt1_conv_fwd_implicit": (C.c_int, [_VP, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP, _VP, _VP]),
     "fqt1_scq_quantize": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, C.c_size_t, _VP, _VP]),
     "fqt1_scq_quantize_noalloc": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, _VP]),
     "fqt1_bwd_input_gemm": (C.c_int, [_VP, _VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
@@ -151,6 +155,23 @@ def im2col(x, N, Cin, H, W, kh, kw, stride, pad, row_bits=None, col_bits=None, c
 def fwd_gemm(sx_row, sw_row, M, D, K, gamma, acc, y, stream=None):
     _check(lib().fqt1_fwd_gemm(_p(sx_row), _p(sw_row), M, D, K, _p(gamma), _p(acc), _p(y), _s(stream)),
            "fqt1_fwd_gemm")
+
+
+def pack_pixels(x, N, Cin, H, W, x_pix, stream=None):
+    _check(lib().fqt1_pack_pixels(_p(x), N, Cin, H, W, _p(x_pix), _s(stream)), "fqt1_pack_pixels")
+
+
+def pack_weight_taps(w, D, Cin, kh, kw, w_taps, stream=None):
+    _check(lib().fqt1_pack_weight_taps(_p(w), D, Cin, kh, kw, _p(w_taps), _s(stream)), "fqt1_pack_weight_taps")
+
+
+def conv_implicit_supported(N, Cin, H, W, kh, kw, stride, pad):
+    return bool(lib().fqt1_conv_implicit_supported(N, Cin, H, W, kh, kw, stride, pad))
+
+
+def conv_fwd_implicit(x_pix, w_taps, N, Cin, H, W, kh, kw, stride, pad, D, gamma, bias, acc, y, stream=None):
+    _check(lib().fqt1_conv_fwd_implicit(_p(x_pix), _p(w_taps), N, Cin, H, W, kh, kw, stride, pad, D, _p(gamma),
+                                        _p(bias), _p(acc), _p(y), _s(stream)), "fqt1_conv_fwd_implicit")
 
 
 def fwd_gemm_bias(sx_row, sw_row, M, D, K, gamma, bias, acc, y, stream=None):

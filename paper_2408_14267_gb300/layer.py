@@ -4,7 +4,11 @@
 enqueues, on one CUDA stream and without host synchronisation:
 
   forward : pack sign(W) (rows, columns, column sums); pack sign(X) or the
-            Unfolder of X fused with sign; binarized GEMM, y = Gamma * acc
+            Unfolder of X fused with sign; binarized GEMM, y = Gamma * acc.
+            A stride-1 "same" convolution with C a multiple of 128 runs the
+            implicit-GEMM forward instead: sign(X) packed per pixel, sign(W)
+            packed tap-major, and the Unfolder writes only the column packing
+            that grad_weight reads
   backward: SCQ quantization of G = gY (.) Gamma (ranges, AGP selection,
             stochastic rounding of both branches); grad_input GEMM (PSQ side)
             then, for a convolution, the Folder; grad_weight GEMM (PCQ side)
@@ -27,7 +31,7 @@ class LayerStep:
     """Buffers and launches of one layer step.  keep_acc=False skips the optional
     int32 copy of the forward accumulators (the benchmark's configuration)."""
 
-    def __init__(self, wl, device="cuda", keep_acc=True, fold=None):
+    def __init__(self, wl, device="cuda", keep_acc=True, fold=None, implicit=False):
         dev = torch.device(device)
         self.kind = wl["kind"]
         self.keep_acc = keep_acc
@@ -56,11 +60,22 @@ class LayerStep:
             self.fold = (not keep_acc and ok) if fold is None else (fold and ok)
         else:
             self.fold = False
+        # implicit-GEMM forward on request, where the library supports the convolution (off by
+        # default: on the 8 x 8, 256-channel layer its two extra packing kernels cost more than
+        # the Unfolder's row packing they replace)
+        if self.kind == "conv":
+            self.implicit = bool(implicit) and fqt1.conv_implicit_supported(N, Cin, H, W, kh, kw, self.stride,
+                                                                              self.pad)
+        else:
+            self.implicit = False
         wK, wM, wD = fqt1.packed_words(K), fqt1.packed_words(M), fqt1.packed_words(D)
-        self.sx_row = torch.empty(M, wK, **i32)
+        if self.implicit:
+            self.x_pix = torch.empty(N * H * W, fqt1.packed_words(Cin), **i32)
+            self.w_taps = torch.empty(D, wK, **i32)
+        self.sx_row = None if self.implicit else torch.empty(M, wK, **i32)
         self.sx_col = torch.empty(K, wM, **i32)
         self.cs_x = torch.empty(K, **i32)
-        self.sw_row = torch.empty(D, wK, **i32)
+        self.sw_row = None if self.implicit else torch.empty(D, wK, **i32)
         self.sw_col = torch.empty(K, wD, **i32)
         self.cs_w = torch.empty(K, **i32)
         self.acc_y = torch.empty(M, D, **i32) if keep_acc else None
@@ -85,19 +100,36 @@ class LayerStep:
     def dense_ops(self):
         return 6.0 * self.M * self.K * self.D
 
+    FORWARD_STAGES = ("pack_w", "pack_xp", "pack_x", "im2col", "fwd_gemm")
+
     def stages(self):
         """The step as (name, launch(stream)) pairs, in stream order."""
-        st = [("pack_w", lambda s: fqt1.binarize_pack(self.w, self.D, self.K, self.K, self.sw_row, self.sw_col,
-                                                       self.cs_w, s))]
-        if self.kind == "conv":
+        if self.implicit:
             N, Cin, H, W, kh, kw = self.conv
-            st.append(("im2col", lambda s: fqt1.im2col(self.x, N, Cin, H, W, kh, kw, self.stride, self.pad,
-                                                       self.sx_row, self.sx_col, self.cs_x, s)))
+
+            def pack_w(s):
+                fqt1.binarize_pack(self.w, self.D, self.K, self.K, None, self.sw_col, self.cs_w, s)
+                fqt1.pack_weight_taps(self.w, self.D, Cin, kh, kw, self.w_taps, s)
+
+            st = [("pack_w", pack_w),
+                  ("pack_xp", lambda s: fqt1.pack_pixels(self.x, N, Cin, H, W, self.x_pix, s)),
+                  ("im2col", lambda s: fqt1.im2col(self.x, N, Cin, H, W, kh, kw, self.stride, self.pad, None,
+                                                   self.sx_col, self.cs_x, s)),
+                  ("fwd_gemm", lambda s: fqt1.conv_fwd_implicit(self.x_pix, self.w_taps, N, Cin, H, W, kh, kw,
+                                                                self.stride, self.pad, self.D, self.gamma_fwd, None,
+                                                                self.acc_y, self.y, s))]
         else:
-            st.append(("pack_x", lambda s: fqt1.binarize_pack(self.x, self.M, self.K, self.K, self.sx_row,
-                                                              self.sx_col, self.cs_x, s)))
-        st.append(("fwd_gemm", lambda s: fqt1.fwd_gemm(self.sx_row, self.sw_row, self.M, self.D, self.K,
-                                                       self.gamma_fwd, self.acc_y, self.y, s)))
+            st = [("pack_w", lambda s: fqt1.binarize_pack(self.w, self.D, self.K, self.K, self.sw_row, self.sw_col,
+                                                           self.cs_w, s))]
+            if self.kind == "conv":
+                N, Cin, H, W, kh, kw = self.conv
+                st.append(("im2col", lambda s: fqt1.im2col(self.x, N, Cin, H, W, kh, kw, self.stride, self.pad,
+                                                           self.sx_row, self.sx_col, self.cs_x, s)))
+            else:
+                st.append(("pack_x", lambda s: fqt1.binarize_pack(self.x, self.M, self.K, self.K, self.sx_row,
+                                                                  self.sx_col, self.cs_x, s)))
+            st.append(("fwd_gemm", lambda s: fqt1.fwd_gemm(self.sx_row, self.sw_row, self.M, self.D, self.K,
+                                                           self.gamma_fwd, self.acc_y, self.y, s)))
         st.append(("scq_quantize", lambda s: fqt1.scq_quantize(self.gy, self.M, self.D, self.gamma, self.p_s,
                                                                self.p_c, self.psq, self.pcq, self.ws,
                                                                self.dev_status, s)))
@@ -124,12 +156,14 @@ class LayerStep:
         return st
 
     def forward(self, stream=None):
-        for name, fn in self.stages()[:3]:
-            fn(stream)
+        for name, fn in self.stages():
+            if name in self.FORWARD_STAGES:
+                fn(stream)
 
     def backward(self, stream=None):
-        for name, fn in self.stages()[3:]:
-            fn(stream)
+        for name, fn in self.stages():
+            if name not in self.FORWARD_STAGES:
+                fn(stream)
 
     def step(self, stream=None):
         for name, fn in self.stages():
@@ -143,6 +177,8 @@ class LayerStep:
           calling stream: pack X -> (wait W) forward -> (wait SCQ) grad_weight -> join
           branch 1      : pack W
           branch 2      : SCQ quantize -> (wait W) grad_input (-> Folder)
+        With the implicit-GEMM forward the calling stream packs X per pixel, and the Unfolder
+        (only grad_weight reads its column packing) runs on branch 1 after pack W.
         """
         main = stream if stream is not None else torch.cuda.current_stream()
         if not hasattr(self, "_branches"):
@@ -166,11 +202,18 @@ class LayerStep:
             st["bwd_input_gemm"](b2)
             if "col2im" in st:
                 st["col2im"](b2)
-        x_name = "im2col" if "im2col" in st else "pack_x"
-        st[x_name](main)
+        if self.implicit:
+            st["im2col"](b1)
+            x_ready = torch.cuda.Event()
+            x_ready.record(b1)
+            st["pack_xp"](main)
+        else:
+            st["im2col" if "im2col" in st else "pack_x"](main)
         main.wait_event(w_ready)
         st["fwd_gemm"](main)
         main.wait_event(q_ready)
+        if self.implicit:
+            main.wait_event(x_ready)
         st["bwd_weight_gemm"](main)
         b2_done = torch.cuda.Event()
         b2_done.record(b2)
@@ -187,6 +230,8 @@ class LayerStep:
           branch 1  : (W in) pack W
           branch 2  : (gY in) SCQ quantize -> (W packed) grad_input (-> Folder)
           calling   : (X in) pack / Unfolder -> (W packed) forward -> (SCQ) grad_weight
+          (implicit-GEMM forward: the calling stream packs X per pixel and branch 1 runs the
+          Unfolder after pack W and X in; grad_weight also waits for it)
           copies out: (all in, grad_input done) dx, (forward done) y, (grad_weight done) dw
         """
         main = stream if stream is not None else torch.cuda.current_stream()
@@ -229,13 +274,20 @@ class LayerStep:
                 st["col2im"](b2)
         dx_ready = ev(b2)
         main.wait_event(x_in)
-        x_name = "im2col" if "im2col" in st else "pack_x"
-        st[x_name](main)
+        if self.implicit:  # the Unfolder feeds only grad_weight: branch 1, after pack W
+            b1.wait_event(x_in)
+            st["im2col"](b1)
+            x_ready = ev(b1)
+            st["pack_xp"](main)
+        else:
+            st["im2col" if "im2col" in st else "pack_x"](main)
         main.wait_event(w_ready)
         main.wait_event(gy_in)  # Gamma (copied before gY) scales the forward
         st["fwd_gemm"](main)
         y_ready = ev(main)
         main.wait_event(q_ready)
+        if self.implicit:
+            main.wait_event(x_ready)
         st["bwd_weight_gemm"](main)
         dw_ready = ev(main)
         cout.wait_event(x_in)  # the outputs follow the inputs on the link

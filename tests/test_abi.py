@@ -74,3 +74,39 @@ def test_argument_validation_without_launch(lib):
     assert lib.fqt1_bwd_input_gemm(C.byref(q), fake, fake, 8, 8, 8, C.byref(bad_bits), fake, fake, s) == 1
     assert lib.fqt1_bwd_weight_gemm(C.byref(q), fake, fake, 8, 8, 8, C.byref(ok), None, fake, None, 0, s) == 1
     assert lib.fqt1_col2im(fake, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 0, 1, fake, s) == 1  # stride 0
+
+
+def test_implicit_conv_support_rules(lib):
+    """Shapes the implicit-GEMM forward accepts: stride-1 "same" kernels, C a multiple of 128,
+    and 128-pixel tiles of whole images or whole image rows (host logic, no GPU)."""
+    ok = lambda *a: bool(lib.fqt1_conv_implicit_supported(*a))  # N, C, H, W, kh, kw, stride, pad
+    assert ok(128, 256, 8, 8, 3, 3, 1, 1)           # whole images, 2 per tile
+    assert ok(9, 128, 4, 4, 1, 1, 1, 0)             # 1x1, 8 images per tile
+    assert ok(2, 128, 16, 16, 3, 3, 1, 1)           # 8 rows of 16 per tile
+    assert ok(1, 512, 32, 32, 5, 5, 1, 2)           # 4 rows of 32, 5x5
+    assert ok(64, 128, 2, 2, 3, 3, 1, 1)            # 32 images per tile
+    assert not ok(2, 96, 8, 8, 3, 3, 1, 1)          # C not a multiple of 128
+    assert not ok(2, 128, 8, 8, 3, 3, 2, 1)         # stride 2
+    assert not ok(2, 128, 8, 8, 3, 3, 1, 0)         # not "same"
+    assert not ok(2, 128, 8, 8, 3, 1, 1, 1)         # kh != kw
+    assert not ok(2, 128, 12, 12, 3, 3, 1, 1)       # 144 pixels, rows of 12 do not tile 128
+    assert not ok(2, 128, 12, 16, 3, 3, 1, 1)       # 8 rows per tile do not divide 12
+    assert not ok(2, 128, 3, 3, 3, 3, 1, 1)         # 9 pixels do not divide 128
+
+
+def test_implicit_conv_validation_without_launch(lib):
+    fake = C.c_void_p(0x10000)
+    odd = C.c_void_p(0x10004)
+    s = C.c_void_p(0)
+    assert lib.fqt1_pack_pixels(fake, 2, 96, 8, 8, fake, s) == 3                   # C % 128
+    assert lib.fqt1_pack_pixels(fake, 2, 128, 8, 8, odd, s) == 2                   # misaligned output
+    assert lib.fqt1_pack_pixels(None, 2, 128, 8, 8, fake, s) == 1
+    assert lib.fqt1_pack_weight_taps(fake, 4, 48, 3, 3, fake, s) == 3              # C % 32
+    assert lib.fqt1_pack_weight_taps(fake, 0, 64, 3, 3, fake, s) == 1
+    args = [fake, fake, 2, 128, 8, 8, 3, 3, 2, 1, C.c_int64(16), fake, None, None, fake, s]
+    assert lib.fqt1_conv_fwd_implicit(*args) == 3                                  # stride 2
+    args[8] = 1
+    args[11] = None
+    assert lib.fqt1_conv_fwd_implicit(*args) == 1                                  # no gamma
+    args[11] = odd
+    assert lib.fqt1_conv_fwd_implicit(*args) == 2                                  # misaligned gamma

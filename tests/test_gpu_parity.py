@@ -91,12 +91,18 @@ def check_step(w, st, ref):
     M, K, D, rpg = st.M, st.K, st.D, st.rpg
     x_u = ref["x_u"] if w["kind"] == "conv" else w["x"]
     w_u = w["w"].reshape(D, -1)
-    sx, pad_bits = unpack_bits(st.sx_row, K)
-    assert np.array_equal(sx, om.sign(x_u)) and not pad_bits.any(), "sign(X) row bits"
+    if st.implicit:  # implicit-GEMM forward: pixel-major sign(X), tap-major sign(W)
+        sp, pad_bits = unpack_bits(st.x_pix, w["x"].shape[1])
+        assert np.array_equal(sp, om.pixel_signs(w["x"])) and not pad_bits.any(), "sign(X) pixel bits"
+        swt, pad_bits = unpack_bits(st.w_taps, K)
+        assert np.array_equal(swt, om.tap_major_signs(w["w"])) and not pad_bits.any(), "sign(W) tap-major bits"
+    else:
+        sx, pad_bits = unpack_bits(st.sx_row, K)
+        assert np.array_equal(sx, om.sign(x_u)) and not pad_bits.any(), "sign(X) row bits"
+        sw, _ = unpack_bits(st.sw_row, K)
+        assert np.array_equal(sw, om.sign(w_u)), "sign(W) row bits"
     sxc, pad_bits = unpack_bits(st.sx_col, M)
     assert np.array_equal(sxc, om.sign(x_u).T) and not pad_bits.any(), "sign(X) col bits"
-    sw, _ = unpack_bits(st.sw_row, K)
-    assert np.array_equal(sw, om.sign(w_u)), "sign(W) row bits"
     swc, _ = unpack_bits(st.sw_col, D)
     assert np.array_equal(swc, om.sign(w_u).T), "sign(W) col bits"
     assert np.array_equal(st.cs_x.cpu().numpy(), om.colsum_sign(x_u)), "colsum X"
@@ -162,6 +168,13 @@ CASES = [
     ("conv-same-4x8-1x1", lambda: conv_case(7, 300, 4, 8, 16, 1, 1, 0, 8, SYS, seed=8)),
     ("conv-same-8x16-7x7", lambda: conv_case(3, 4, 8, 16, 8, 7, 1, 3, 4, SYS, seed=9)),
     ("conv-same-4x64", lambda: conv_case(2, 6, 4, 64, 8, 3, 1, 1, 2, SYS, seed=10)),
+    # implicit-GEMM forward (C a multiple of 128): a ragged last tile of whole images, tiles of
+    # image rows, 1x1 with 8 images per tile, and 5x5 taps over 32-pixel rows with a partial
+    # last contraction stage (K = 3200)
+    ("conv-implicit-8x8-ragged", lambda: conv_case(5, 128, 8, 8, 48, 3, 1, 1, 4, SYS, seed=12)),
+    ("conv-implicit-16x16-rows", lambda: conv_case(2, 128, 16, 16, 40, 3, 1, 1, 2, BER, seed=13)),
+    ("conv-implicit-4x4-1x1", lambda: conv_case(9, 256, 4, 4, 24, 1, 1, 0, 8, SYS, seed=14)),
+    ("conv-implicit-32x32-5x5", lambda: conv_case(1, 128, 32, 32, 16, 5, 1, 2, 4, SYS, seed=15)),
 ]
 
 
@@ -170,7 +183,9 @@ def test_layer_step_parity(name, make):
     from paper_2408_14267_gb300.layer import LayerStep
     w = make()
     ref = run_oracle(w)
-    st = LayerStep(w)
+    st = LayerStep(w, implicit="implicit" in name)
+    if "implicit" in name:
+        assert st.implicit
     st.dev_status.zero_()
     st.step()
     torch.cuda.synchronize()
@@ -183,6 +198,22 @@ def test_layer_step_parity(name, make):
 
 
 LINEAR_CASES = [c for c in CASES if c[0].startswith("linear")]
+
+
+@pytest.mark.parametrize("name,make", [CASES[1], CASES[-4]], ids=[CASES[1][0], CASES[-4][0]])
+def test_implicit_and_unfolded_forward_steps_agree(name, make):
+    """The bench layer with the implicit forward and an implicit case with it switched off
+    (materialized 1-bit unfolding, row-packed operands) both match the oracle's step."""
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    ref = run_oracle(w)
+    want = "implicit" not in name
+    st = LayerStep(w, implicit=want)
+    assert st.implicit == want
+    st.dev_status.zero_()
+    st.step()
+    torch.cuda.synchronize()
+    check_step(w, st, ref)
 
 FOLD_CASES = [
     ("fold-resnet18-cifar-8192x2304x256-b4", lambda: wl.resnet18_cifar_conv()),

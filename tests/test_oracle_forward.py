@@ -84,6 +84,55 @@ def test_conv_forward_pads_as_minus_one():
     assert np.array_equal(acc.reshape(N, -1, D), ref.reshape(N, D, -1).transpose(0, 2, 1).astype(np.int64))
 
 
+def _direct_conv_signs(x, w, pad):
+    """Brute-force stride-1 convolution of sign(zero-padded x) with sign(w), plain loops."""
+    N, C, H, W = x.shape
+    D, _, kh, kw = w.shape
+    Ho, Wo = H + 2 * pad - kh + 1, W + 2 * pad - kw + 1
+    out = np.zeros((N * Ho * Wo, D), dtype=np.int64)
+    for n in range(N):
+        for oh in range(Ho):
+            for ow in range(Wo):
+                for d in range(D):
+                    s = 0
+                    for c in range(C):
+                        for i in range(kh):
+                            for j in range(kw):
+                                h, ww = oh + i - pad, ow + j - pad
+                                v = x[n, c, h, ww] if 0 <= h < H and 0 <= ww < W else 0.0
+                                s += (1 if v > 0 else -1) * (1 if w[d, c, i, j] > 0 else -1)
+                    out[(n * Ho + oh) * Wo + ow, d] = s
+    return out
+
+
+@pytest.mark.parametrize("N,C,H,W,D,k,p", [(2, 3, 4, 5, 3, 3, 1), (1, 4, 3, 3, 2, 1, 0), (2, 2, 5, 4, 2, 5, 2),
+                                           (1, 3, 4, 4, 2, 3, 0)])
+def test_implicit_conv_matches_direct_convolution(N, C, H, W, D, k, p):
+    """The tap-by-tap implicit product equals a brute-force convolution of the signs and the
+    Unfolder product; regathering the pixel-major rows by tap against the tap-major weight
+    signs gives the same integers (pins both layouts: a transposed one fails)."""
+    rng = np.random.default_rng(N * 31 + C * 7 + k)
+    x = rng.standard_normal((N, C, H, W)).astype(np.float32)
+    x[0, 0, 0, :2] = 0.0
+    w = rng.standard_normal((D, C, k, k)).astype(np.float32)
+    ref = _direct_conv_signs(x, w, p)
+    assert np.array_equal(om.implicit_conv_acc(x, w, p), ref)
+    acc_u, _ = om.forward(om.unfold(x, k, k, 1, p), w.reshape(D, -1), None)
+    assert np.array_equal(acc_u, ref)
+    Ho, Wo = H + 2 * p - k + 1, W + 2 * p - k + 1
+    px = om.pixel_signs(x).astype(np.int64).reshape(N, H, W, C)
+    a = np.full((N, Ho, Wo, k * k, C), -1, dtype=np.int64)  # row m, k' = t C + c
+    for i in range(k):
+        for j in range(k):
+            for oh in range(Ho):
+                for ow in range(Wo):
+                    h, ww = oh + i - p, ow + j - p
+                    if 0 <= h < H and 0 <= ww < W:
+                        a[:, oh, ow, i * k + j, :] = px[:, h, ww, :]
+    acc_t = om.int_matmul(a.reshape(N * Ho * Wo, k * k * C), om.tap_major_signs(w))
+    assert np.array_equal(acc_t, ref)
+
+
 def test_scale_bias_grad_matches_autograd():
     """dGamma and dbias of y = (sign(X) sign(W)^T) (.) Gamma + bias (Sec. 5.1 with a bias):
     the oracle's closed sums against torch autograd of the plain float64 formula."""
