@@ -32,25 +32,37 @@ SMS, POPC_PER_CLK_SM = 152, 16
 
 # DRAM bytes (read + write) per launch of each stage's kernels, from one ncu capture of
 # `bench.py --profile 2 --warmup 1` (profiles/kernels_resnet18_cifar_conv_full.md; the SCQ
-# stage is the sum of its range, selection and quantize kernels).  They are
-# valid only for the kernel sources they were taken on: TRAFFIC_SOURCES is the sha256 prefix of
-# paper_2408_14267_gb300/csrc at that capture; any other source tree reports traffic = null.
-TRAFFIC_SOURCES = "4f6e3a0bc012d230"
+# stage is the sum of its range, selection and quantize kernels).  A figure is valid only for
+# the kernel sources it was taken on: TRAFFIC_SOURCES holds, per stage, the sha256 prefix of the
+# files that define that stage's kernels (STAGE_SOURCES) at the capture; a stage whose sources
+# have changed since reports traffic = null.
+STAGE_SOURCES = {"pack": ("common.cuh", "pack.cu"), "gemm": ("api.cu", "common.cuh", "gemm.cuh", "gemm_tc.cu"),
+                 "scq": ("common.cuh", "quantize.cu")}
+STAGE_GROUP = {"pack_w": "pack", "pack_xp": "pack", "im2col": "pack", "fwd_gemm": "gemm", "scq_quantize": "scq",
+               "bwd_input_fold": "gemm", "bwd_weight_gemm": "gemm"}
+TRAFFIC_SOURCES = {"pack": "3ddd9ed0cf4ec421", "gemm": "25bd0f246f63f95b", "scq": "4c3011fadca46d05"}
 TRAFFIC_BYTES = {"pack_w": 2.379264e+06, "im2col": 8.418304e+06, "fwd_gemm": 2.512384e+06,
                  "scq_quantize": 1.693517e+07, "bwd_input_fold": 6.835200e+05,
                  "bwd_weight_gemm": 2.980096e+06}
 
 
-def sources_sha():
-    import glob
+def sources_sha(group):
+    """sha256 prefix of the kernel sources of one stage group (file names and contents)."""
     import hashlib
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2408_14267_gb300", "csrc")
-    for f in sorted(glob.glob(os.path.join(csrc, "*.cu")) + glob.glob(os.path.join(csrc, "*.cuh"))):
-        h.update(os.path.basename(f).encode())
-        with open(f, "rb") as fh:
+    for f in sorted(STAGE_SOURCES[group]):
+        h.update(f.encode())
+        with open(os.path.join(csrc, f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
+
+
+def stage_traffic(stage):
+    g = STAGE_GROUP.get(stage)
+    if g is None or stage not in TRAFFIC_BYTES or sources_sha(g) != TRAFFIC_SOURCES.get(g):
+        return None
+    return TRAFFIC_BYTES[stage]
 
 CPU_SAMPLE_SCRIPT = r"""
 import json, sys, time
@@ -325,7 +337,7 @@ def main():
         alu_peak = SMS * POPC_PER_CLK_SM * 32 * 2 * clk_mhz * 1e6 / 1e12
         roof = {"bound": "alu", "achieved": work / dur_s / 1e12, "peak": alu_peak, "unit": "TOPS"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = TRAFFIC_BYTES.get(dom) if sources_sha() == TRAFFIC_SOURCES else None
+    roof["traffic"] = stage_traffic(dom)
     roof["kernel"] = dom
     roof["peak_source"] = peak_src if bound != "alu" else "derived: 152 SMs x 16 popc/clk x 32 bit x 2 x max clock"
 
