@@ -322,6 +322,9 @@ def test_workspace_keys_restored_after_each_call():
              LayerStep(linear_case(100, 48, 72, 4, 2, SYS, seed=11))]
     ws = fqt1.scq_workspace(max(s.M for s in steps), max(s.D for s in steps), 0, 1, "cuda")
 
+    def initialised(w):  # range keys 0xFF
+        return bool((w == 255).all())
+
     def same(a, b, rows):
         c = a.count()
         assert c == b.count()
@@ -337,14 +340,49 @@ def test_workspace_keys_restored_after_each_call():
         pcq = fqt1.QGradBuffers(st.pcq.n, st.pcq.capacity, st.pcq.capacity, st.M)
         fqt1.scq_quantize(st.gy, st.M, st.D, st.gamma, st.p_s, st.p_c, psq, pcq, ws, st.dev_status)
         torch.cuda.synchronize()
-        assert bool((ws == 255).all()) and bool((st.ws == 255).all())
+        assert initialised(ws) and initialised(st.ws)
         same(psq, st.psq, st.rpg)
         same(pcq, st.pcq, 1)
         q = fqt1.QGradBuffers(st.pcq.n, st.pcq.capacity, st.pcq.capacity, st.M)
         fqt1.agp_quantize_grad(st.gy, st.M, st.D, 1, st.gamma, st.p_c, q, ws, st.dev_status)
         torch.cuda.synchronize()
-        assert bool((ws == 255).all())
+        assert initialised(ws)
         same(q, st.pcq, 1)
+
+
+@pytest.mark.parametrize("M,D,rpg,bits,mode", [(8192, 256, 64, 4, SYS), (250, 100, 5, 8, BER), (1024, 256, 4, 2, SYS),
+                                              (60, 16, 60, 2, TOP)])
+def test_scq_matches_single_branch_calls(M, D, rpg, bits, mode):
+    """One fqt1_scq_quantize call (both groupings from one range pass and one rounding pass)
+    equals two single-branch fqt1_agp_quantize_grad calls bit for bit, all outputs, also for M
+    not a multiple of 4 (per-word rounding draws) and for every mask law."""
+    from paper_2408_14267_gb300 import fqt1
+    rng = np.random.default_rng(M + D)
+    s_ = 10.0 ** rng.uniform(-2, 2, size=(M // rpg, 1, 1))
+    g = torch.from_numpy((rng.laplace(0, 1e-3, (M // rpg, rpg, D)) * s_).reshape(M, D).astype(np.float32)).cuda()
+    gamma = torch.from_numpy(rng.uniform(0.5, 2.0, D).astype(np.float32)).cuda()
+    p_s, p_c = fqt1.AgpParams(bits, mode, 31, rpg), fqt1.AgpParams(bits, mode, 32, 1)
+    cap_s, cap_c = fqt1.kept_capacity(M // rpg, bits, mode), fqt1.kept_capacity(D, bits, mode)
+    bufs = lambda: (fqt1.QGradBuffers(M // rpg, cap_s, cap_s * rpg, D), fqt1.QGradBuffers(D, cap_c, cap_c, M))
+    ws = fqt1.scq_workspace(M, D, 0, rpg, "cuda")
+    st = torch.zeros(4, dtype=torch.int32, device="cuda")
+    psq, pcq = bufs()
+    for q in (psq, pcq):
+        q.codes.fill_(0x5A)
+    fqt1.scq_quantize(g, M, D, gamma, p_s, p_c, psq, pcq, ws, st)
+    rs, rc = bufs()
+    for q in (rs, rc):
+        q.codes.fill_(0x5A)
+    fqt1.agp_quantize_grad(g, M, D, 0, gamma, p_s, rs, ws, st)
+    fqt1.agp_quantize_grad(g, M, D, 1, gamma, p_c, rc, ws, st)
+    torch.cuda.synchronize()
+    assert int(st[0].item()) == 0
+    assert bool((ws == 255).all())
+    for a, b in ((psq, rs), (pcq, rc)):
+        for name in ("group_min", "group_range", "p_hat", "slot_of_group", "kept_idx", "kept_count", "codes"):
+            assert torch.equal(getattr(a, name), getattr(b, name)), name
+        c = a.count()
+        assert torch.equal(a.scale[:c], b.scale[:c]) and torch.equal(a.zero[:c], b.zero[:c])
 
 
 def test_nonfinite_gradient_sets_status():
