@@ -302,24 +302,35 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
     plane_words = (nrows * a.W + 31) / 32 + 2 * a.guard;
     nplanes = (n_hi - n_lo + 1) * nc;
   }
-  // 1. sign-pack the region (one warp per 32 stream bits: coalesced 128-byte loads + ballot)
+  // 1. sign-pack the region: word f of the region (plane f / data_words, word f % data_words of
+  //    it) is the ballot of 32 consecutive floats of one plane row run; a warp takes words
+  //    warp, warp + 8, ... with 16 loads in flight per lane (unconditional, from clamped
+  //    indices), so the region costs one memory round trip per 128 words, not one per plane
   const int plane_bits = nrows * a.W, data_words = plane_words - 2 * a.guard, gbits = 32 * a.guard;
-  for (int pl = warp; pl < nplanes; pl += 8) {  // one (image, channel) plane per warp iteration
-    const int nn = pl / nc;
-    const float* src = a.x + (((int64_t)(n_lo + nn) * a.C + c_lo + (pl - nn * nc)) * a.H + h_lo) * a.W;
-    uint32_t* dst = stream + pl * plane_words + a.guard;
-    for (int q0 = 0; q0 < data_words; q0 += 4) {  // 4 loads in flight per lane, then 4 ballots
-      float v[4];
+  {
+    const int total = nplanes * data_words;
+    const FastDiv div_dw((uint32_t)max(data_words, 1)), div_nc((uint32_t)nc);
+    const int64_t img_stride = (int64_t)a.C * a.H * a.W;
+    const float* base = a.x + ((int64_t)n_lo * a.C + c_lo) * a.H * a.W + (int64_t)h_lo * a.W;
+    for (int f0 = warp; f0 < total; f0 += 8 * 16) {
+      float v[16];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {  // unconditional loads from clamped indices, masked afterwards
-        const int e = 32 * (q0 + u) + lane;
-        v[u] = __ldg(src + min(e, plane_bits - 1));
-        if (q0 + u >= data_words || e >= plane_bits) v[u] = 0.0f;
+      for (int u = 0; u < 16; ++u) {
+        const int f = min(f0 + 8 * u, total - 1);
+        const int pl = (int)div_dw.div((uint32_t)f), q = f - pl * data_words;
+        const int nn = (int)div_nc.div((uint32_t)pl), c = pl - nn * nc;
+        const int e = 32 * q + lane;
+        v[u] = __ldg(base + nn * img_stride + (int64_t)c * a.H * a.W + min(e, plane_bits - 1));
+        if (e >= plane_bits) v[u] = 0.0f;
       }
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
+      for (int u = 0; u < 16; ++u) {
         const uint32_t word = __ballot_sync(0xFFFFFFFFu, v[u] > 0.0f);
-        if (lane == 0 && q0 + u < data_words) dst[q0 + u] = word;
+        const int f = f0 + 8 * u;
+        if (lane == 0 && f < total) {
+          const int pl = (int)div_dw.div((uint32_t)f);
+          stream[pl * plane_words + a.guard + (f - pl * data_words)] = word;
+        }
       }
     }
   }
