@@ -40,10 +40,10 @@ STAGE_SOURCES = {"pack": ("common.cuh", "pack.cu"), "gemm": ("api.cu", "common.c
                  "scq": ("common.cuh", "quantize.cu")}
 STAGE_GROUP = {"pack_w": "pack", "pack_xp": "pack", "im2col": "pack", "fwd_gemm": "gemm", "scq_quantize": "scq",
                "bwd_input_fold": "gemm", "bwd_weight_gemm": "gemm"}
-TRAFFIC_SOURCES = {"pack": "3ddd9ed0cf4ec421", "gemm": "25bd0f246f63f95b", "scq": "4c3011fadca46d05"}
-TRAFFIC_BYTES = {"pack_w": 2.379264e+06, "im2col": 8.418304e+06, "fwd_gemm": 2.512384e+06,
-                 "scq_quantize": 1.693517e+07, "bwd_input_fold": 6.835200e+05,
-                 "bwd_weight_gemm": 2.980096e+06}
+TRAFFIC_SOURCES = {"pack": "8df06b7aa9f13c7d", "gemm": "85572ab8238d2e95", "scq": "4c3011fadca46d05"}
+TRAFFIC_BYTES = {"pack_w": 2.379008e+06, "im2col": 8.418304e+06, "fwd_gemm": 2.511872e+06,
+                 "scq_quantize": 1.693030e+07, "bwd_input_fold": 6.840320e+05,
+                 "bwd_weight_gemm": 2.979840e+06}
 
 
 def sources_sha(group):
