@@ -175,6 +175,38 @@ fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_row, int64_
 fqt1_status fqt1_fwd_gemm_bias(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D, int64_t K,
                                const float* gamma, const float* bias, int32_t* acc, float* y, void* stream);
 
+/* e4m3 copies of sign(W) for the products' B operand (no counterpart in the
+ * paper: the same +-1 values in the tensor cores' byte format, so that the
+ * products load B with TMA instead of expanding packed bits in every CTA).
+ * fqt1_expand_signs_e4m3: packed signs bits [rows][fqt1_packed_words(n)] (as
+ *   written by fqt1_binarize_pack) -> out [rows][ld_out] bytes: 0x38 (+1) where
+ *   the bit is set, 0xB8 (-1) where it is clear, 0 for columns n .. ld_out - 1.
+ *   ld_out >= n and a multiple of 16; both pointers 16-byte aligned.
+ * fqt1_fwd_gemm_e4m3w: fqt1_fwd_gemm_bias with sign(W) given as w_e4m3
+ *   [D][ld_w] (the row packing expanded); gamma and y required, acc and bias
+ *   may be NULL.  Results equal fqt1_fwd_gemm_bias bit for bit.
+ * fqt1_bwd_input_fold_e4m3w: fqt1_bwd_input_fold with sign(W)^T given as
+ *   wt_e4m3 [K][ld_wt] (the column packing expanded, ld_wt >= D).  Results
+ *   equal fqt1_bwd_input_fold bit for bit. */
+fqt1_status fqt1_expand_signs_e4m3(const uint32_t* bits, int64_t rows, int64_t n, uint8_t* out, int64_t ld_out,
+                                   void* stream);
+/* fqt1_binarize_pack with the e4m3 bytes of the signs as two more optional
+ * outputs, written by the same pass over x where its rows are a multiple of 4
+ * floats (otherwise the packed outputs, which must then be given, are expanded
+ * by fqt1_expand_signs_e4m3): row_e4m3 [rows][ld_re] (ld_re >= cols, columns
+ * past cols 0) and col_e4m3 [cols][ld_ce] (ld_ce >= rows, rows past `rows` 0);
+ * ld_re and ld_ce multiples of 16, all pointers 16-byte aligned. */
+fqt1_status fqt1_binarize_pack_e4m3(const float* x, int64_t rows, int64_t cols, int64_t ld, uint32_t* row_bits,
+                                    uint32_t* col_bits, int32_t* colsum, uint8_t* row_e4m3, int64_t ld_re,
+                                    uint8_t* col_e4m3, int64_t ld_ce, void* stream);
+fqt1_status fqt1_fwd_gemm_e4m3w(const uint32_t* sx_row, const uint8_t* w_e4m3, int64_t ld_w, int64_t M, int64_t D,
+                                int64_t K, const float* gamma, const float* bias, int32_t* acc, float* y,
+                                void* stream);
+fqt1_status fqt1_bwd_input_fold_e4m3w(const fqt1_qgrad* psq, const uint8_t* wt_e4m3, int64_t ld_wt,
+                                      const int32_t* colsum_w, int32_t N, int32_t C, int32_t H, int32_t W,
+                                      int32_t kh, int32_t kw, int32_t stride, int32_t pad, int64_t D,
+                                      const fqt1_agp_params* p, float* dx, void* stream);
+
 /* ------------------------------------------------ layer parameters and STE */
 /* Gradients of the layer's scale Gamma (Sec. 5.1: y = (sign(X) sign(W)^T) (.)
  * Gamma, Gamma learnable) and of its bias:

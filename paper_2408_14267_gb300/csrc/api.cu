@@ -258,6 +258,19 @@ extern "C" fqt1_status fqt1_fwd_gemm_bias(const uint32_t* sx_row, const uint32_t
   return FQT1_OK;
 }
 
+extern "C" fqt1_status fqt1_fwd_gemm_e4m3w(const uint32_t* sx_row, const uint8_t* w_e4m3, int64_t ld_w, int64_t M,
+                                           int64_t D, int64_t K, const float* gamma, const float* bias, int32_t* acc,
+                                           float* y, void* stream) {
+  if (!sx_row || !w_e4m3 || !gamma || !y || M < 1 || D < 1 || K < 1 || ld_w < K || ld_w % 16)
+    return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(sx_row) || !aligned16(w_e4m3) || (acc && !aligned16(acc)) || !aligned16(y) || !aligned16(gamma) ||
+      (bias && !aligned16(bias)))
+    return FQT1_ERR_MISALIGNED;
+  if (K >= (1ll << 24) || (M + 63) / 64 > 65535 || use_popcount_path()) return FQT1_ERR_UNSUPPORTED;
+  FQT1_CUDA_TRY(launch_fwd_e4m3w_tc(sx_row, w_e4m3, ld_w, M, D, K, gamma, bias, acc, y, nullptr, (cudaStream_t)stream));
+  return FQT1_OK;
+}
+
 extern "C" fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D,
                                      int64_t K, const float* gamma, int32_t* acc, float* y, void* stream) {
   return fqt1_fwd_gemm_bias(sx_row, sw_row, M, D, K, gamma, nullptr, acc, y, stream);
@@ -384,20 +397,24 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
   return FQT1_OK;
 }
 
-extern "C" fqt1_status fqt1_bwd_input_fold(const fqt1_qgrad* psq, const uint32_t* sw_col, const int32_t* colsum_w,
-                                           int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw,
-                                           int32_t stride, int32_t pad, int64_t D, const fqt1_agp_params* p,
-                                           float* dx, void* stream) {
-  if (!psq || !sw_col || !colsum_w || !p || !dx || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 ||
-      stride < 1 || pad < 0 || D < 1)
+// Shared by the two Folder entry points: B is the packed sign(W) columns sw_col, or (wt_e4m3
+// non-null) the e4m3 bytes of sign(W)^T with rows of ld_wt bytes.
+static fqt1_status bwd_input_fold_impl(const fqt1_qgrad* psq, const uint32_t* sw_col, const uint8_t* wt_e4m3,
+                                       int64_t ld_wt, const int32_t* colsum_w, int32_t N, int32_t C, int32_t H,
+                                       int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad, int64_t D,
+                                       const fqt1_agp_params* p, float* dx, void* stream) {
+  if (!psq || (!sw_col && !wt_e4m3) || !colsum_w || !p || !dx || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 ||
+      kw < 1 || stride < 1 || pad < 0 || D < 1)
     return FQT1_ERR_INVALID_ARG;
+  if (wt_e4m3 && (ld_wt < D || ld_wt % 16)) return FQT1_ERR_INVALID_ARG;
+  if (wt_e4m3 && !aligned16(wt_e4m3)) return FQT1_ERR_MISALIGNED;
   if (!valid_bits(p->bits) || !psq->codes || !psq->kept_count || !psq->kept_idx || !psq->slot_of_group ||
       !psq->scale || !psq->zero || psq->ld_codes < fqt1_codes_ld(D) || psq->ld_codes % 16)
     return FQT1_ERR_INVALID_ARG;
   if (H + 2 * pad < kh || W + 2 * pad < kw) return FQT1_ERR_INVALID_ARG;
   const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
   if (p->rows_per_group != (int64_t)Ho * Wo) return FQT1_ERR_INVALID_ARG;
-  if (!aligned16(sw_col) || !aligned16(dx) || !aligned16(colsum_w)) return FQT1_ERR_MISALIGNED;
+  if ((sw_col && !aligned16(sw_col)) || !aligned16(dx) || !aligned16(colsum_w)) return FQT1_ERR_MISALIGNED;
   // whole samples per 128-row tile, at least one channel's taps per tile, and the Folder's
   // tables (tap offsets, folded colsums of 128 / (kh kw) channels, per-sample constants) in
   // their 36 KB of shared memory
@@ -409,8 +426,26 @@ extern "C" fqt1_status fqt1_bwd_input_fold(const fqt1_qgrad* psq, const uint32_t
   const int64_t cap_rows = fqt1_kept_capacity(N, p->bits, p->mode) * rpg;
   FQT1_CUDA_TRY(launch_fold_tc(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, sw_col,
                                (int64_t)C * kh * kw, D, psq->kept_idx, psq->scale, psq->zero, colsum_w,
-                               psq->slot_of_group, dx, N, C, H, W, kh, kw, stride, pad, Ho, Wo, nullptr, s));
+                               psq->slot_of_group, dx, N, C, H, W, kh, kw, stride, pad, Ho, Wo, nullptr, s,
+                               wt_e4m3, ld_wt));
   return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_bwd_input_fold(const fqt1_qgrad* psq, const uint32_t* sw_col, const int32_t* colsum_w,
+                                           int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw,
+                                           int32_t stride, int32_t pad, int64_t D, const fqt1_agp_params* p,
+                                           float* dx, void* stream) {
+  if (!sw_col) return FQT1_ERR_INVALID_ARG;
+  return bwd_input_fold_impl(psq, sw_col, nullptr, 0, colsum_w, N, C, H, W, kh, kw, stride, pad, D, p, dx, stream);
+}
+
+extern "C" fqt1_status fqt1_bwd_input_fold_e4m3w(const fqt1_qgrad* psq, const uint8_t* wt_e4m3, int64_t ld_wt,
+                                                 const int32_t* colsum_w, int32_t N, int32_t C, int32_t H, int32_t W,
+                                                 int32_t kh, int32_t kw, int32_t stride, int32_t pad, int64_t D,
+                                                 const fqt1_agp_params* p, float* dx, void* stream) {
+  if (!wt_e4m3) return FQT1_ERR_INVALID_ARG;
+  return bwd_input_fold_impl(psq, nullptr, wt_e4m3, ld_wt, colsum_w, N, C, H, W, kh, kw, stride, pad, D, p, dx,
+                             stream);
 }
 
 extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_t* sx_col, const int32_t* colsum_x,

@@ -72,6 +72,10 @@ struct TcArgs {
   // sub-tile of one kernel tap, shifted by the tap; the contraction index is k' = t C + c.
   // A box covers 2^isb consecutive sub-tiles of one tap (rows of 16 * 2^isb bytes).
   int impl, iC, ikw, ikhw, ipad, iW, iHW, isb;
+  // b_tma = 1: B is given as e4m3 bytes (+1 = 0x38, -1 = 0xB8, K-major rows, tmB a 128B-swizzled
+  // map of 128 x 128 boxes) and goes by TMA straight into the operand ring; all eight expansion
+  // warps then expand A, each half of a stage's sub-tiles.
+  int b_tma;
   // EPI_FOLD divisors (host-built): kh kw, W, kw, H W, stride, fcb H W
   FastDiv fd_khw, fd_w, fd_kw, fd_hw, fd_s, fd_cbhw;
   // EPI_CRED: the cluster's partial tiles are summed into acc (int32, ldo) and dequantized into
@@ -322,6 +326,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   __shared__ __align__(8) uint64_t raw_full[kMaxStages], raw_empty[kMaxStages], op_full[kMaxStages],
       op_empty[kMaxStages];
   __shared__ __align__(8) uint64_t acc_full;
+  __shared__ __align__(8) uint64_t b_full[kMaxStages];  // b_tma: the B boxes of an operand stage landed
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
   __shared__ __align__(16) float gamma_s[BN];  // EPI_FWD: Gamma of this tile's columns (read as float4)
@@ -348,7 +353,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   if (threadIdx.x == 0) {
     abort_flag = 0;
     for (int s = 0; s < RS; ++s) { mbar_init(&raw_full[s], 1); mbar_init(&raw_empty[s], kExpWarps); }
-    for (int s = 0; s < OS; ++s) { mbar_init(&op_full[s], kExpWarps); mbar_init(&op_empty[s], 1); }
+    for (int s = 0; s < OS; ++s) { mbar_init(&op_full[s], kExpWarps); mbar_init(&op_empty[s], 1); mbar_init(&b_full[s], 1); }
     mbar_init(&acc_full, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -399,7 +404,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   const int64_t valid_rows = a.count ? (int64_t)__ldg(a.count) * a.rows_per_count : a.M;
   const int nk = m0 < valid_rows ? kt1 - kt0 : 0;  // a tile past the kept rows has no work
 
-  constexpr uint32_t kTx = (uint32_t)S::kRawStage;
+  const uint32_t kTx = a.b_tma ? (uint32_t)S::kRawA : (uint32_t)S::kRawStage;
 
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer (raw ring)
@@ -432,7 +437,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         } else {
           tma_load_2d(rawA(s), &tmA, &raw_full[s], kt * KSUB * (kBK / 32), (int)m0);
         }
-        tma_load_2d(rawB(s), &tmB, &raw_full[s], kt * KSUB * (kBK / 32), (int)n0);
+        if (!a.b_tma) tma_load_2d(rawB(s), &tmB, &raw_full[s], kt * KSUB * (kBK / 32), (int)n0);
         ++issued;
       }
       // drain: every issued copy must land before the CTA may exit
@@ -450,6 +455,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       for (int i = 0; i < nk; ++i) {
         const int s = i % OS, it = i / OS;
         if (!mbar_wait(&op_full[s], it & 1, &abort_flag, a.status)) break;
+        if (a.b_tma && !mbar_wait(&b_full[s], it & 1, &abort_flag, a.status)) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const uint32_t acol = tmem + BN + s * S::kAcols, baddr = smem_u32(opB(s));
         const int nsub = valid_subtiles<KSUB>(a.L, kt0 + i);
@@ -478,8 +484,9 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     const int64_t tile_rows = valid_rows - m0;  // may exceed kBM or be negative
     const int live_q = tile_rows >= kBM ? 4 : (tile_rows <= 0 ? 0 : (int)((tile_rows + 31) / 32));
     const bool split = KSUB == 2 && live_q <= 2;
-    const bool a_warp = split ? (warp == 4 || warp == 5 || warp >= 8) : warp < 6;
-    const int a_h0 = split && warp >= 8 ? 1 : 0, a_h1 = split ? a_h0 + 1 : KSUB;
+    const bool a_warp = a.b_tma ? true : split ? (warp == 4 || warp == 5 || warp >= 8) : warp < 6;
+    const int a_h0 = a.b_tma ? (warp >= 6 ? KSUB / 2 : 0) : (split && warp >= 8 ? 1 : 0);
+    const int a_h1 = a.b_tma ? a_h0 + KSUB / 2 : (split ? a_h0 + 1 : KSUB);
     const int bblk = split ? (warp == 2 ? 0 : warp == 3 ? 1 : warp == 6 ? 2 : 3) : warp - 6;
     const int quarter = warp & 3;
     const int arow = 32 * quarter + lane, brow = 32 * bblk + lane;
@@ -487,9 +494,20 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     // depends only on its own A row, and the epilogue drops those rows
     const bool a_live = a_warp && m0 + 32 * quarter < valid_rows;
     const uint32_t a_lanes = tmem + ((uint32_t)(32 * quarter) << 16);
+    int b_issued = 0;  // b_tma: operand stages whose B boxes this thread (warp 2, lane 0) issued
     for (int i = 0; i < nk; ++i) {
       const int so = i % OS, ito = i / OS, sr = i % RS, itr = i / RS;
       if (ito > 0 && !mbar_wait(&op_empty[so], (ito - 1) & 1, &abort_flag, a.status)) break;
+      if (a.b_tma) {  // the stage's B boxes, as soon as the MMAs of its previous use are done
+        if (warp == 2 && lane == 0) {
+          mbar_expect_tx(&b_full[so], (uint32_t)S::kOpB);
+#pragma unroll
+          for (int h = 0; h < KSUB; ++h)
+            tma_load_2d(opB(so) + h * S::kSub, &tmB, &b_full[so], ((kt0 + i) * KSUB + h) * kBK, (int)n0);
+          ++b_issued;
+        }
+        __syncwarp();
+      }
       if (!mbar_wait(&raw_full[sr], itr & 1, &abort_flag, a.status)) break;
       const int kt = kt0 + i;
       if (a_warp) {
@@ -569,6 +587,18 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         mbar_arrive(&raw_empty[sr]);
       }
     }
+
+    // every B box this thread issued must land before the epilogue reuses the ring or the CTA
+    // exits (normally the MMA issuer has already seen them land)
+    if (a.b_tma && warp == 2 && lane == 0) {
+      for (int i = (b_issued > OS ? b_issued - OS : 0); i < b_issued; ++i) {
+        const int so = i % OS, ito = i / OS;
+        const uint64_t t0 = gtimer();
+        while (!mbar_test(&b_full[so], ito & 1) && gtimer() - t0 < kWaitNs) {
+        }
+      }
+    }
+    __syncwarp();
 
     // ---------------------------------------------------------------- epilogue
     // TMEM -> registers (thread = row) -> per-warp swizzled staging (32 x 32 words) ->
@@ -1111,12 +1141,18 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
 // convolution fields (impl = 0 for a plain A = sign(X) rows map).
 static cudaError_t launch_fwd_common(const CUtensorMap& ma, TcArgs a, const uint32_t* B, int64_t M, int64_t D,
                                      int64_t K, const float* gamma, const float* bias, int32_t* acc, float* y,
-                                     int32_t* status, cudaStream_t s) {
+                                     int32_t* status, cudaStream_t s, const uint8_t* Be = nullptr, int64_t ldbe = 0) {
   using S = TcSmem<false, false, 128>;
   const int64_t ldw = fqt1_packed_words(K);
   CUtensorMap mb;
-  if (!make_map(&mb, B, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, D, ldw * 4, 4 * S::KSUB, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+  if (Be) {  // e4m3 sign(W) rows [D][ldbe] bytes: 128 x 128 boxes, 128-byte swizzle
+    if (!make_map(&mb, Be, CU_TENSOR_MAP_DATA_TYPE_UINT8, K, D, ldbe, kBK, 128, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+    a.b_tma = 1;
+  } else if (!make_map(&mb, B, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, D, ldw * 4, 4 * S::KSUB, 128,
+                       CU_TENSOR_MAP_SWIZZLE_NONE)) {
     return cudaErrorInvalidValue;
+  }
   a.M = M; a.N = D; a.L = K; a.count = nullptr; a.rows_per_count = 1;
   a.k_tiles = (int)((K + kBK * S::KSUB - 1) / (kBK * S::KSUB)); a.tiles_per_split = a.k_tiles;
   a.epi = EPI_FWD; a.gamma = gamma; a.bias = bias; a.y = y; a.acc = acc; a.ldo = D; a.status = status;
@@ -1145,6 +1181,19 @@ cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64
                 CU_TENSOR_MAP_SWIZZLE_NONE))
     return cudaErrorInvalidValue;
   return launch_fwd_common(ma, TcArgs{}, B, M, D, K, gamma, bias, acc, y, status, s);
+}
+
+// Forward with B = e4m3 sign(W) rows [D][ldbe] bytes (ldbe a multiple of 16, bytes past K zero).
+cudaError_t launch_fwd_e4m3w_tc(const uint32_t* A, const uint8_t* Be, int64_t ldbe, int64_t M, int64_t D, int64_t K,
+                                const float* gamma, const float* bias, int32_t* acc, float* y, int32_t* status,
+                                cudaStream_t s) {
+  using S = TcSmem<false, false, 128>;
+  const int64_t ldw = fqt1_packed_words(K);
+  CUtensorMap ma;
+  if (!make_map(&ma, A, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, M, ldw * 4, 4 * S::KSUB, kBM,
+                CU_TENSOR_MAP_SWIZZLE_NONE))
+    return cudaErrorInvalidValue;
+  return launch_fwd_common(ma, TcArgs{}, nullptr, M, D, K, gamma, bias, acc, y, status, s, Be, ldbe);
 }
 
 // Implicit-GEMM forward of a stride-1 "same" convolution (kh = kw = 2 pad + 1, C a multiple of
@@ -1212,14 +1261,20 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
                            const uint32_t* Sg, int64_t K, int64_t D, const int32_t* kept_idx, const float* scale,
                            const float* zero, const int32_t* cs, const int32_t* slot_of_group, float* dx, int N, int C,
                            int H, int W, int kh, int kw, int stride, int pad, int Ho, int Wo, int32_t* status,
-                           cudaStream_t s) {
+                           cudaStream_t s, const uint8_t* Bte, int64_t ldbte) {
   const int64_t lds = fqt1_packed_words(D);
   CUtensorMap ma, mb;
-  if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, D, max_rows, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, kCodesStageK / 32, 128,
-                CU_TENSOR_MAP_SWIZZLE_NONE))
+  if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, D, max_rows, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B))
     return cudaErrorInvalidValue;
+  if (Bte) {  // e4m3 sign(W)^T rows [K][ldbte] bytes: 128 x 128 boxes, 128-byte swizzle
+    if (!make_map(&mb, Bte, CU_TENSOR_MAP_DATA_TYPE_UINT8, D, K, ldbte, kBK, 128, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+  } else if (!make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, kCodesStageK / 32, 128,
+                       CU_TENSOR_MAP_SWIZZLE_NONE)) {
+    return cudaErrorInvalidValue;
+  }
   TcArgs a{};
+  a.b_tma = Bte ? 1 : 0;
   const int khw = kh * kw, cb = 128 / khw;
   a.M = max_rows; a.N = K; a.L = D; a.count = count; a.rows_per_count = (int64_t)Ho * Wo;
   a.k_tiles = (int)((D + kCodesStageK - 1) / kCodesStageK); a.tiles_per_split = a.k_tiles;

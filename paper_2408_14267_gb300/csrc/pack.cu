@@ -215,9 +215,17 @@ __device__ __forceinline__ uint32_t warp_transpose32(uint32_t x, int lane) {
 // gives the row words, and the row words leave as 16-byte stores.
 constexpr int kPackTileWarps = 4;
 
+// e4m3 bytes of 4 sign bits (bit k of nib -> byte k): +1 = 0x38, -1 = 0xB8.
+__device__ __forceinline__ uint32_t e4m3_signs4(uint32_t nib) {
+  return ((nib & 15u) * 0x10204080u & 0x80808080u) ^ 0xB8B8B8B8u;
+}
+
+// Optional outputs: the e4m3 bytes of the signs, rows [rows][ld_re] (columns cols .. ld_re - 1
+// zero) and columns [cols][ld_ce] (rows rows .. ld_ce - 1 zero).
 __global__ void __launch_bounds__(32 * kPackTileWarps) pack_tile_kernel(
     const float* __restrict__ x, int64_t rows, int64_t cols, int64_t ld, uint32_t* __restrict__ row_bits,
-    int64_t row_words, uint32_t* __restrict__ col_bits, int64_t col_words, int32_t* __restrict__ colsum) {
+    int64_t row_words, uint32_t* __restrict__ col_bits, int64_t col_words, int32_t* __restrict__ colsum,
+    uint8_t* __restrict__ row_e4m3, int64_t ld_re, uint8_t* __restrict__ col_e4m3, int64_t ld_ce) {
   constexpr int NW = kPackTileWarps, TC = 32 * NW, F4 = TC / 4;
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
@@ -253,6 +261,43 @@ __global__ void __launch_bounds__(32 * kPackTileWarps) pack_tile_kernel(
   if (c < cols) {
     if (col_bits) col_bits[c * col_words + blockIdx.y] = cw;
     if (colsum) atomicAdd(colsum + c, 2 * __popc(cw) - (int)min((int64_t)32, rows - r0));
+    if (col_e4m3) {  // column c, rows r0 .. r0 + 31 (up to ld_ce): 32 bytes from the column word
+      const int nvalid = (int)min((int64_t)32, rows - r0);
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        if (r0 + 16 * h >= ld_ce) break;
+        uint32_t wv[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          uint32_t v = e4m3_signs4(cw >> (16 * h + 4 * q));
+#pragma unroll
+          for (int b = 0; b < 4; ++b)
+            if (16 * h + 4 * q + b >= nvalid) v &= ~(0xFFu << (8 * b));
+          wv[q] = v;
+        }
+        *reinterpret_cast<uint4*>(col_e4m3 + c * ld_ce + r0 + 16 * h) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+      }
+    }
+  }
+  if (row_e4m3) {  // rows r0 .. r0 + 31, columns cb .. cb + TC - 1 (up to ld_re): 16 bytes per thread
+    for (int e = threadIdx.x; e < 32 * (TC / 16); e += 32 * NW) {
+      const int r = e / (TC / 16), q16 = e % (TC / 16);
+      const int64_t c0 = cb + 16 * q16;
+      if (r0 + r >= rows || c0 >= ld_re) continue;
+      uint32_t wv[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        uint32_t nib = 0;
+#pragma unroll
+        for (int b = 0; b < 4; ++b) nib |= (t[r][16 * q16 + 4 * q + b] > 0.0f ? 1u : 0u) << b;
+        uint32_t v = e4m3_signs4(nib);
+#pragma unroll
+        for (int b = 0; b < 4; ++b)
+          if (c0 + 4 * q + b >= cols) v &= ~(0xFFu << (8 * b));
+        wv[q] = v;
+      }
+      *reinterpret_cast<uint4*>(row_e4m3 + (r0 + r) * ld_re + c0) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+    }
   }
   __syncthreads();
   if (row_bits) {  // row r: words cb / 32 .. + NW - 1
@@ -723,6 +768,32 @@ __global__ void __launch_bounds__(256) pack_weight_taps_kernel(const float* __re
     for (int64_t e = used + lane; e < words; e += 32) out[d * words + e] = 0u;
   }
 }
+
+// ------------------------------------------------------------------ e4m3 signs
+// e4m3 bytes of packed signs (the B operand of the products when it is loaded as bytes):
+// out[r][e] = 0x38 (+1) where bit e of row r is set, 0xB8 (-1) where it is clear, for e < n,
+// and 0 for n <= e < ld_out (so that no byte past the contraction is a NaN pattern).  One thread
+// per 16 output bytes; bit k of a nibble lands on the sign bit of byte k through one multiply.
+__global__ void __launch_bounds__(256) expand_signs_kernel(const uint32_t* __restrict__ bits, int64_t rows, int64_t n,
+                                                           int64_t ld_words, uint8_t* __restrict__ out, int64_t ld_out) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  const int64_t chunks = ld_out / 16;
+  const int64_t t = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  if (t >= rows * chunks) return;
+  const int64_t r = t / chunks, e0 = 16 * (t - r * chunks);
+  const uint32_t h = e0 < n ? (__ldg(bits + r * ld_words + (e0 >> 5)) >> (e0 & 16)) & 0xFFFFu : 0u;
+  uint32_t wv[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint32_t v = (((h >> (4 * q)) & 15u) * 0x10204080u & 0x80808080u) ^ 0xB8B8B8B8u;
+#pragma unroll
+    for (int b = 0; b < 4; ++b)
+      if (e0 + 4 * q + b >= n) v &= ~(0xFFu << (8 * b));
+    wv[q] = v;
+  }
+  *reinterpret_cast<uint4*>(out + r * ld_out + e0) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+}
 }  // namespace fqt1
 
 using namespace fqt1;
@@ -746,7 +817,7 @@ extern "C" fqt1_status fqt1_binarize_pack(const float* x, int64_t rows, int64_t 
     FQT1_CUDA_TRY(launch_k(pack_tile_kernel, dim3((unsigned)((cols + 32 * kPackTileWarps - 1) / (32 * kPackTileWarps)),
                                                   (unsigned)bands),
                            dim3(32 * kPackTileWarps), 0, s, x, rows, cols, ld, row_bits, row_words, col_bits, col_words,
-                           colsum));
+                           colsum, (uint8_t*)nullptr, (int64_t)0, (uint8_t*)nullptr, (int64_t)0));
   else
     FQT1_CUDA_TRY(launch_k(pack_dense_kernel, dim3((unsigned)((row_words + 3) / 4), (unsigned)bands), dim3(128), 0,
                            s, x, rows, cols, ld, row_bits, row_words, col_bits, col_words, colsum));
@@ -886,5 +957,58 @@ extern "C" fqt1_status fqt1_pack_weight_taps(const float* w, int64_t D, int32_t 
   FQT1_CUDA_TRY(launch_k(pack_weight_taps_kernel, dim3((unsigned)((D * khw + 7) / 8)), dim3(256), 0,
                          (cudaStream_t)stream, w, D, (int)C, (int)khw, words, w_taps));
   fqt1_count_launches(1);
+  return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_expand_signs_e4m3(const uint32_t* bits, int64_t rows, int64_t n, uint8_t* out,
+                                              int64_t ld_out, void* stream) {
+  if (!bits || !out || rows < 1 || n < 1 || ld_out < n || ld_out % 16) return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(bits) || !aligned16(out)) return FQT1_ERR_MISALIGNED;
+  const int64_t threads = rows * (ld_out / 16);
+  if ((threads + 255) / 256 >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
+  FQT1_CUDA_TRY(launch_k(expand_signs_kernel, dim3((unsigned)((threads + 255) / 256)), dim3(256), 0,
+                         (cudaStream_t)stream, bits, rows, n, fqt1_packed_words(n), out, ld_out));
+  fqt1_count_launches(1);
+  return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_binarize_pack_e4m3(const float* x, int64_t rows, int64_t cols, int64_t ld,
+                                               uint32_t* row_bits, uint32_t* col_bits, int32_t* colsum,
+                                               uint8_t* row_e4m3, int64_t ld_re, uint8_t* col_e4m3, int64_t ld_ce,
+                                               void* stream) {
+  if (!x || rows < 1 || cols < 1 || ld < cols) return FQT1_ERR_INVALID_ARG;
+  if (!row_bits && !col_bits && !colsum && !row_e4m3 && !col_e4m3) return FQT1_ERR_INVALID_ARG;
+  if ((row_e4m3 && (ld_re < cols || ld_re % 16)) || (col_e4m3 && (ld_ce < rows || ld_ce % 16)))
+    return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(x) || (row_bits && !aligned16(row_bits)) || (col_bits && !aligned16(col_bits)) ||
+      (colsum && !aligned16(colsum)) || (row_e4m3 && !aligned16(row_e4m3)) || (col_e4m3 && !aligned16(col_e4m3)))
+    return FQT1_ERR_MISALIGNED;
+  const int64_t bands = (rows + 31) / 32;
+  if (bands > 65535) return FQT1_ERR_UNSUPPORTED;
+  if (cols % 4 != 0 || ld % 4 != 0) {
+    // no shared-memory tile for these rows: the packed signs, then their byte expansion
+    uint32_t* rb = row_bits;
+    uint32_t* cbits = col_bits;
+    if ((row_e4m3 && !rb) || (col_e4m3 && !cbits)) return FQT1_ERR_INVALID_ARG;
+    fqt1_status st = fqt1_binarize_pack(x, rows, cols, ld, rb, cbits, colsum, stream);
+    if (st != FQT1_OK) return st;
+    if (row_e4m3 && (st = fqt1_expand_signs_e4m3(rb, rows, cols, row_e4m3, ld_re, stream)) != FQT1_OK) return st;
+    if (col_e4m3 && (st = fqt1_expand_signs_e4m3(cbits, cols, rows, col_e4m3, ld_ce, stream)) != FQT1_OK) return st;
+    return FQT1_OK;
+  }
+  cudaStream_t s = (cudaStream_t)stream;
+  const int64_t row_words = fqt1_packed_words(cols), col_words = fqt1_packed_words(rows);
+  if (colsum) FQT1_CUDA_TRY(cudaMemsetAsync(colsum, 0, sizeof(int32_t) * cols, s));
+  FQT1_CUDA_TRY(launch_k(pack_tile_kernel, dim3((unsigned)((cols + 32 * kPackTileWarps - 1) / (32 * kPackTileWarps)),
+                                                (unsigned)bands),
+                         dim3(32 * kPackTileWarps), 0, s, x, rows, cols, ld, row_bits, row_words, col_bits, col_words,
+                         colsum, row_e4m3, ld_re, col_e4m3, ld_ce));
+  fqt1_count_launches(1);
+  if (col_bits && col_words > bands) {
+    const int64_t n = cols * (col_words - bands);
+    FQT1_CUDA_TRY(launch_k(zero_col_pad_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, col_bits, cols,
+                           col_words, bands));
+    fqt1_count_launches(1);
+  }
   return FQT1_OK;
 }

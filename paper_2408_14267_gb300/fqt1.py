@@ -51,6 +51,10 @@ _SIGS = {
     "fqt1_ste_clip": (C.c_int, [_VP, _VP, _I64, C.c_float, _VP]),
     "fqt1_agp_quantize_grad": (C.c_int, [_VP, _I64, _I64, _I32, _VP, _VP, _VP, _VP, C.c_size_t, _VP, _VP]),
     "fqt1_scq_workspace_init": (C.c_int, [_VP, C.c_size_t, _VP]),
+    "fqt1_expand_signs_e4m3": (C.c_int, [_VP, _I64, _I64, _VP, _I64, _VP]),
+    "fqt1_binarize_pack_e4m3": (C.c_int, [_VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP, _I64, _VP, _I64, _VP]),
+    "fqt1_fwd_gemm_e4m3w": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _I64, _VP, _VP, _VP, _VP, _VP]),
+    "fqt1_bwd_input_fold_e4m3w": (C.c_int, [_VP, _VP, _I64, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP]),
     "fqt1_pack_pixels": (C.c_int, [_VP, _I32, _I32, _I32, _I32, _VP, _VP]),
     "fqt1_pack_weight_taps": (C.c_int, [_VP, _I64, _I32, _I32, _I32, _VP, _VP]),
     "fqt1_conv_implicit_supported": (_I32, [_I32] * 8),
@@ -155,6 +159,29 @@ def im2col(x, N, Cin, H, W, kh, kw, stride, pad, row_bits=None, col_bits=None, c
 def fwd_gemm(sx_row, sw_row, M, D, K, gamma, acc, y, stream=None):
     _check(lib().fqt1_fwd_gemm(_p(sx_row), _p(sw_row), M, D, K, _p(gamma), _p(acc), _p(y), _s(stream)),
            "fqt1_fwd_gemm")
+
+
+def expand_signs_e4m3(bits, rows, n, out, stream=None):
+    _check(lib().fqt1_expand_signs_e4m3(_p(bits), rows, n, _p(out), out.shape[-1], _s(stream)),
+           "fqt1_expand_signs_e4m3")
+
+
+def binarize_pack_e4m3(x, rows, cols, ld, row_bits, col_bits, colsum, row_e4m3, col_e4m3, stream=None):
+    _check(lib().fqt1_binarize_pack_e4m3(_p(x), rows, cols, ld, _p(row_bits), _p(col_bits), _p(colsum), _p(row_e4m3),
+                                         row_e4m3.shape[-1] if row_e4m3 is not None else 0, _p(col_e4m3),
+                                         col_e4m3.shape[-1] if col_e4m3 is not None else 0, _s(stream)),
+           "fqt1_binarize_pack_e4m3")
+
+
+def fwd_gemm_e4m3w(sx_row, w_e4m3, M, D, K, gamma, bias, acc, y, stream=None):
+    _check(lib().fqt1_fwd_gemm_e4m3w(_p(sx_row), _p(w_e4m3), w_e4m3.shape[-1], M, D, K, _p(gamma), _p(bias),
+                                     _p(acc), _p(y), _s(stream)), "fqt1_fwd_gemm_e4m3w")
+
+
+def bwd_input_fold_e4m3w(psq, wt_e4m3, colsum_w, N, Cin, H, W, kh, kw, stride, pad, D, p, dx, stream=None):
+    _check(lib().fqt1_bwd_input_fold_e4m3w(C.byref(psq.c), _p(wt_e4m3), wt_e4m3.shape[-1], _p(colsum_w), N, Cin, H,
+                                           W, kh, kw, stride, pad, D, C.byref(p), _p(dx), _s(stream)),
+           "fqt1_bwd_input_fold_e4m3w")
 
 
 def pack_pixels(x, N, Cin, H, W, x_pix, stream=None):

@@ -31,7 +31,7 @@ class LayerStep:
     """Buffers and launches of one layer step.  keep_acc=False skips the optional
     int32 copy of the forward accumulators (the benchmark's configuration)."""
 
-    def __init__(self, wl, device="cuda", keep_acc=True, fold=None, implicit=False):
+    def __init__(self, wl, device="cuda", keep_acc=True, fold=None, implicit=False, e4m3_weights=False):
         dev = torch.device(device)
         self.kind = wl["kind"]
         self.keep_acc = keep_acc
@@ -76,6 +76,15 @@ class LayerStep:
         self.sx_col = torch.empty(K, wM, **i32)
         self.cs_x = torch.empty(K, **i32)
         self.sw_row = None if self.implicit else torch.empty(D, wK, **i32)
+        # e4m3 copies of sign(W) (rows for the forward product, columns for the fused Folder's
+        # product): B then goes to the tensor cores by TMA instead of being expanded per CTA.
+        # Off by default: on the 8 x 8, 256-channel layer the step graph is as fast either way
+        # e4m3_weights: True (both products), "fwd" or "fold" (one of them), False
+        e_fwd = e4m3_weights is True or e4m3_weights == "fwd"
+        e_fold = e4m3_weights is True or e4m3_weights == "fold"
+        u8 = dict(dtype=torch.uint8, device=dev)
+        self.w8 = torch.empty(D, fqt1.codes_ld(K), **u8) if e_fwd and not self.implicit else None
+        self.wt8 = torch.empty(K, fqt1.codes_ld(D), **u8) if e_fold and self.fold else None
         self.sw_col = torch.empty(K, wD, **i32)
         self.cs_w = torch.empty(K, **i32)
         self.acc_y = torch.empty(M, D, **i32) if keep_acc else None
@@ -108,7 +117,11 @@ class LayerStep:
             N, Cin, H, W, kh, kw = self.conv
 
             def pack_w(s):
-                fqt1.binarize_pack(self.w, self.D, self.K, self.K, None, self.sw_col, self.cs_w, s)
+                if self.wt8 is not None:
+                    fqt1.binarize_pack_e4m3(self.w, self.D, self.K, self.K, None, self.sw_col, self.cs_w, None,
+                                            self.wt8, s)
+                else:
+                    fqt1.binarize_pack(self.w, self.D, self.K, self.K, None, self.sw_col, self.cs_w, s)
                 fqt1.pack_weight_taps(self.w, self.D, Cin, kh, kw, self.w_taps, s)
 
             st = [("pack_w", pack_w),
@@ -119,8 +132,14 @@ class LayerStep:
                                                                 self.stride, self.pad, self.D, self.gamma_fwd, None,
                                                                 self.acc_y, self.y, s))]
         else:
-            st = [("pack_w", lambda s: fqt1.binarize_pack(self.w, self.D, self.K, self.K, self.sw_row, self.sw_col,
-                                                           self.cs_w, s))]
+            def pack_w(s):
+                if self.w8 is not None or self.wt8 is not None:  # the e4m3 copies from the same pass
+                    fqt1.binarize_pack_e4m3(self.w, self.D, self.K, self.K, self.sw_row, self.sw_col, self.cs_w,
+                                            self.w8, self.wt8, s)
+                else:
+                    fqt1.binarize_pack(self.w, self.D, self.K, self.K, self.sw_row, self.sw_col, self.cs_w, s)
+
+            st = [("pack_w", pack_w)]
             if self.kind == "conv":
                 N, Cin, H, W, kh, kw = self.conv
                 st.append(("im2col", lambda s: fqt1.im2col(self.x, N, Cin, H, W, kh, kw, self.stride, self.pad,
@@ -128,16 +147,25 @@ class LayerStep:
             else:
                 st.append(("pack_x", lambda s: fqt1.binarize_pack(self.x, self.M, self.K, self.K, self.sx_row,
                                                                   self.sx_col, self.cs_x, s)))
-            st.append(("fwd_gemm", lambda s: fqt1.fwd_gemm(self.sx_row, self.sw_row, self.M, self.D, self.K,
-                                                           self.gamma_fwd, self.acc_y, self.y, s)))
+            if self.w8 is not None:
+                st.append(("fwd_gemm", lambda s: fqt1.fwd_gemm_e4m3w(self.sx_row, self.w8, self.M, self.D, self.K,
+                                                                     self.gamma_fwd, None, self.acc_y, self.y, s)))
+            else:
+                st.append(("fwd_gemm", lambda s: fqt1.fwd_gemm(self.sx_row, self.sw_row, self.M, self.D, self.K,
+                                                               self.gamma_fwd, self.acc_y, self.y, s)))
         st.append(("scq_quantize", lambda s: fqt1.scq_quantize(self.gy, self.M, self.D, self.gamma, self.p_s,
                                                                self.p_c, self.psq, self.pcq, self.ws,
                                                                self.dev_status, s)))
         if self.kind == "conv" and self.fold:
             N, Cin, H, W, kh, kw = self.conv
-            st.append(("bwd_input_fold", lambda s: fqt1.bwd_input_fold(self.psq, self.sw_col, self.cs_w, N, Cin, H, W,
-                                                                       kh, kw, self.stride, self.pad, self.D,
-                                                                       self.p_s, self.dx, s)))
+            if self.wt8 is not None:
+                st.append(("bwd_input_fold", lambda s: fqt1.bwd_input_fold_e4m3w(self.psq, self.wt8, self.cs_w, N, Cin,
+                                                                                 H, W, kh, kw, self.stride, self.pad,
+                                                                                 self.D, self.p_s, self.dx, s)))
+            else:
+                st.append(("bwd_input_fold", lambda s: fqt1.bwd_input_fold(self.psq, self.sw_col, self.cs_w, N, Cin,
+                                                                           H, W, kh, kw, self.stride, self.pad,
+                                                                           self.D, self.p_s, self.dx, s)))
         elif self.kind == "conv":
             N, Cin, H, W, kh, kw = self.conv
             st.append(("bwd_input_gemm", lambda s: fqt1.bwd_input_gemm(self.psq, self.sw_col, self.cs_w, self.M,

@@ -385,6 +385,93 @@ def test_scq_matches_single_branch_calls(M, D, rpg, bits, mode):
         assert torch.equal(a.scale[:c], b.scale[:c]) and torch.equal(a.zero[:c], b.zero[:c])
 
 
+@pytest.mark.parametrize("rows,n", [(3, 5), (256, 2304), (17, 128), (40, 300), (1, 16), (70, 44), (33, 1000)])
+def test_binarize_pack_e4m3_bytes(rows, n):
+    """e4m3 bytes of the signs from the sign-pack pass (tile path for rows of a multiple of 4
+    floats, packing + expansion otherwise) and from the expansion of packed signs: 0x38 for
+    +1, 0xB8 for -1, zeros past the data, both orientations; the packed outputs unchanged."""
+    from paper_2408_14267_gb300 import fqt1
+    rng = np.random.default_rng(rows * 3 + n)
+    x = rng.standard_normal((rows, n)).astype(np.float32)
+    x[-1, -1] = 0.0
+    xt = torch.from_numpy(x).cuda()
+    rb = torch.empty(rows, fqt1.packed_words(n), dtype=torch.int32, device="cuda")
+    cbits = torch.empty(n, fqt1.packed_words(rows), dtype=torch.int32, device="cuda")
+    cs = torch.empty(n, dtype=torch.int32, device="cuda")
+    re = torch.full((rows, fqt1.codes_ld(n)), 0x5A, dtype=torch.uint8, device="cuda")
+    ce = torch.full((n, fqt1.codes_ld(rows)), 0x5A, dtype=torch.uint8, device="cuda")
+    fqt1.binarize_pack_e4m3(xt, rows, n, n, rb, cbits, cs, re, ce)
+    torch.cuda.synchronize()
+    sgn = np.where(om.sign(x) > 0, 0x38, 0xB8).astype(np.uint8)
+    r_, c_ = re.cpu().numpy(), ce.cpu().numpy()
+    assert np.array_equal(r_[:, :n], sgn) and not r_[:, n:].any()
+    assert np.array_equal(c_[:, :rows], sgn.T) and not c_[:, rows:].any()
+    bits, _ = unpack_bits(rb, n)
+    assert np.array_equal(bits, om.sign(x))
+    assert np.array_equal(cs.cpu().numpy(), om.colsum_sign(x))
+
+
+@pytest.mark.parametrize("rows,n", [(3, 5), (256, 2304), (17, 128), (40, 300), (1, 16)])
+def test_expand_signs_e4m3_bytes(rows, n):
+    """Packed signs -> e4m3 bytes: 0x38 for +1, 0xB8 for -1, zeros past the n columns."""
+    from paper_2408_14267_gb300 import fqt1
+    rng = np.random.default_rng(rows * 7 + n)
+    x = rng.standard_normal((rows, n)).astype(np.float32)
+    x[0, 0] = 0.0
+    bits = torch.empty(rows, fqt1.packed_words(n), dtype=torch.int32, device="cuda")
+    fqt1.binarize_pack(torch.from_numpy(x).cuda(), rows, n, n, bits, None, None)
+    out = torch.full((rows, fqt1.codes_ld(n)), 0x5A, dtype=torch.uint8, device="cuda")
+    fqt1.expand_signs_e4m3(bits, rows, n, out)
+    torch.cuda.synchronize()
+    o = out.cpu().numpy()
+    assert np.array_equal(o[:, :n], np.where(om.sign(x) > 0, 0x38, 0xB8).astype(np.uint8))
+    assert not o[:, n:].any()
+
+
+@pytest.mark.parametrize("M,K,D,bias", [(8192, 2304, 256, False), (300, 200, 136, True), (64, 512, 512, True),
+                                        (129, 1000, 40, False)])
+def test_fwd_e4m3_weights_equal_packed(M, K, D, bias):
+    """The forward product with sign(W) as e4m3 bytes loaded by TMA equals the packed-bit
+    product bit for bit (acc and y), with ragged K, D and M."""
+    from paper_2408_14267_gb300 import fqt1
+    rng = np.random.default_rng(M + K + D)
+    x = torch.from_numpy(rng.standard_normal((M, K)).astype(np.float32)).cuda()
+    w = torch.from_numpy(rng.standard_normal((D, K)).astype(np.float32)).cuda()
+    g = torch.from_numpy(rng.uniform(0.5, 2.0, D).astype(np.float32)).cuda()
+    b = torch.from_numpy(rng.standard_normal(D).astype(np.float32)).cuda() if bias else None
+    pk = lambda r: torch.empty(r, fqt1.packed_words(K), dtype=torch.int32, device="cuda")
+    sx, sw = pk(M), pk(D)
+    fqt1.binarize_pack(x, M, K, K, sx, None, None)
+    fqt1.binarize_pack(w, D, K, K, sw, None, None)
+    w8 = torch.empty(D, fqt1.codes_ld(K), dtype=torch.uint8, device="cuda")
+    fqt1.expand_signs_e4m3(sw, D, K, w8)
+    acc0, y0 = torch.empty(M, D, dtype=torch.int32, device="cuda"), torch.empty(M, D, device="cuda")
+    acc1, y1 = torch.full((M, D), 3, dtype=torch.int32, device="cuda"), torch.full((M, D), 3.0, device="cuda")
+    fqt1.fwd_gemm_bias(sx, sw, M, D, K, g, b, acc0, y0)
+    fqt1.fwd_gemm_e4m3w(sx, w8, M, D, K, g, b, acc1, y1)
+    torch.cuda.synchronize()
+    assert torch.equal(acc0, acc1) and torch.equal(y0, y1)
+    acc_ref, _ = om.forward(x.cpu().numpy(), w.cpu().numpy(), None)
+    assert np.array_equal(acc1.cpu().numpy(), acc_ref)
+
+
+@pytest.mark.parametrize("name,make", [CASES[1], FOLD_CASES[1], FOLD_CASES[2], FOLD_CASES[5]],
+                         ids=[CASES[1][0], FOLD_CASES[1][0], FOLD_CASES[2][0], FOLD_CASES[5][0]])
+def test_e4m3_weights_step_equals_packed_step(name, make):
+    """A whole step with the e4m3 copies of sign(W) (forward and fused Folder products) equals
+    the step on packed signs bit for bit."""
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    a = LayerStep(w, keep_acc=False, e4m3_weights=True)
+    b = LayerStep(w, keep_acc=False)
+    assert a.w8 is not None and b.w8 is None
+    for st in (a, b):
+        st.dev_status.zero_()
+        st.step()
+    torch.cuda.synchronize()
+    assert torch.equal(a.y, b.y) and torch.equal(a.dx, b.dx) and torch.equal(a.dw, b.dw)
+
+
 def test_nonfinite_gradient_sets_status():
     from paper_2408_14267_gb300.layer import LayerStep
     w = linear_case(32, 32, 16, 1, 2, SYS, seed=10)
