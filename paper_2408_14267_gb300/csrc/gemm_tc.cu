@@ -772,20 +772,29 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
           off[t] = v ? (di * a.fW + dj) * TS + t : 0;
           msk |= v ? 1u << t : 0u;
         }
+        // two channels per iteration: their 18 shared loads are issued before either sum
+        const int cstep = 256 / HW;
         for (int img = 0; img < imgs; ++img) {
           const int n = s_n[img];
           if (n < 0) break;
           const float sc = s_scale[img], ze = s_zero[img];
-          for (int cl = tt / HW; cl < nc; cl += 256 / HW) {
+          for (int cl = tt / HW; cl < nc; cl += 2 * cstep) {
+            const int cl2 = cl + cstep < nc ? cl + cstep : cl;  // a lone last channel is summed twice
             const int32_t* tp = T + (img * rpg + pos) * TS + cl * 9;
-            int32_t v[9];
+            const int32_t* tp2 = T + (img * rpg + pos) * TS + cl2 * 9;
+            int32_t v[9], v2[9];
 #pragma unroll
-            for (int t = 0; t < 9; ++t) v[t] = tp[off[t]];
-            int32_t acc = 0;
+            for (int t = 0; t < 9; ++t) { v[t] = tp[off[t]]; v2[t] = tp2[off[t]]; }
+            const int32_t cf = csf[cl * HW + pos], cf2 = csf[cl2 * HW + pos];
+            int32_t acc = 0, acc2 = 0;
 #pragma unroll
-            for (int t = 0; t < 9; ++t) acc += (msk >> t) & 1u ? v[t] : 0;
-            a.y[((int64_t)n * a.fC + c_first + cl) * HW + pos] =
-                __fadd_rn(__fmul_rn(sc, (float)acc), __fmul_rn(ze, (float)csf[cl * HW + pos]));
+            for (int t = 0; t < 9; ++t) {
+              acc += (msk >> t) & 1u ? v[t] : 0;
+              acc2 += (msk >> t) & 1u ? v2[t] : 0;
+            }
+            float* yo = a.y + ((int64_t)n * a.fC + c_first) * HW + pos;
+            yo[(int64_t)cl * HW] = __fadd_rn(__fmul_rn(sc, (float)acc), __fmul_rn(ze, (float)cf));
+            if (cl2 != cl) yo[(int64_t)cl2 * HW] = __fadd_rn(__fmul_rn(sc, (float)acc2), __fmul_rn(ze, (float)cf2));
           }
         }
       }
