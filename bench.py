@@ -40,10 +40,10 @@ STAGE_SOURCES = {"pack": ("common.cuh", "pack.cu"), "gemm": ("api.cu", "common.c
                  "scq": ("common.cuh", "quantize.cu")}
 STAGE_GROUP = {"pack_w": "pack", "pack_xp": "pack", "im2col": "pack", "fwd_gemm": "gemm", "scq_quantize": "scq",
                "bwd_input_fold": "gemm", "bwd_weight_gemm": "gemm"}
-TRAFFIC_SOURCES = {"pack": "8df06b7aa9f13c7d", "gemm": "85572ab8238d2e95", "scq": "4c3011fadca46d05"}
-TRAFFIC_BYTES = {"pack_w": 2.379008e+06, "im2col": 8.418304e+06, "fwd_gemm": 2.511872e+06,
-                 "scq_quantize": 1.693030e+07, "bwd_input_fold": 6.840320e+05,
-                 "bwd_weight_gemm": 2.979840e+06}
+TRAFFIC_SOURCES = {"pack": "64316be064e8fe62", "gemm": "73fd5628ecffecdc", "scq": "4c3011fadca46d05"}
+TRAFFIC_BYTES = {"pack_w": 2.384128e+06, "im2col": 8.418304e+06, "fwd_gemm": 2.513408e+06,
+                 "scq_quantize": 1.692979e+07, "bwd_input_fold": 6.858240e+05,
+                 "bwd_weight_gemm": 2.981120e+06}
 
 
 def sources_sha(group):
