@@ -160,7 +160,21 @@ fqt1_status fqt1_conv_fwd_implicit(const uint32_t* x_pix, const uint32_t* w_taps
                                    int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad, int64_t D,
                                    const float* gamma, const float* bias, int32_t* acc, float* y, void* stream);
 
-/* Binarized forward GEMM (Sec. 5.1, App. C "binary multiplication"):/* Binarized forward GEMM (Sec. 5.1, App. C "binary multiplication"):
+/* Channels-last inputs (no counterpart in the paper; the layout of x only).
+ * fqt1_pack_planes_nhwc: x with memory order N, H, W, C (a channels-last
+ *   [N, C, H, W] tensor), C a multiple of 32 -> planes [N][C][ceil(H W / 32)]
+ *   words: bit e of word q of plane (n, c) is set iff x[n, c, pixel 32 q + e] > 0
+ *   (pixel = h W + w), bits past H W clear.  x 16-byte aligned.
+ * fqt1_im2col_planes: fqt1_im2col from those plane bits instead of x, same
+ *   outputs bit for bit.  FQT1_ERR_UNSUPPORTED for shapes whose tiles read
+ *   more input than fits in shared memory (fqt1_im2col then reads x itself). */
+fqt1_status fqt1_pack_planes_nhwc(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, uint32_t* planes,
+                                  void* stream);
+fqt1_status fqt1_im2col_planes(const uint32_t* planes, int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh,
+                               int32_t kw, int32_t stride, int32_t pad, uint32_t* row_bits, uint32_t* col_bits,
+                               int32_t* colsum, void* stream);
+
+/* Binarized forward GEMM (Sec. 5.1, App. C "binary multiplication"):
  * acc[m, j] = sum_k sign(X)[m, k] sign(W)[j, k], y[m, j] = gamma[j] * acc[m, j] (fp32).
  * sx_row: [M][words(K)], sw_row: [D][words(K)], gamma: [D].
  * acc: [M][D] int32 or NULL; y: [M][D] fp32 (row stride D). */

@@ -56,7 +56,12 @@ class _BinaryProduct(torch.autograd.Function):
     @staticmethod
     def forward(ctx, x, weight, gamma, bias, layer):
         dev = x.device
-        x = x.contiguous()
+        # a channels-last convolution input (32k channels) is read in place: its signs are packed
+        # into channel planes, which the Unfolder reads instead of x; otherwise x is made contiguous
+        nhwc = (layer.conv is not None and x.dim() == 4 and x.shape[1] % 32 == 0 and not x.is_contiguous()
+                and x.is_contiguous(memory_format=torch.channels_last))
+        if not nhwc:
+            x = x.contiguous()
         D = weight.shape[0]
         w2 = weight.detach().reshape(D, -1).contiguous()
         K = w2.shape[1]
@@ -75,6 +80,15 @@ class _BinaryProduct(torch.autograd.Function):
         cs_x = torch.empty(K, dtype=torch.int32, device=dev)
         if layer.conv is None:
             fqt1.binarize_pack(x.detach(), M, K, K, sx_row, sx_col, cs_x)
+        elif nhwc:
+            planes = torch.empty(N * C * fqt1.plane_words(H, W), dtype=torch.int32, device=dev)
+            fqt1.pack_planes_nhwc(x.detach(), N, C, H, W, planes)
+            try:
+                fqt1.im2col_planes(planes, N, C, H, W, kh, kw, stride, pad, sx_row, sx_col, cs_x)
+            except fqt1.Fqt1Error as e:
+                if "UNSUPPORTED" not in str(e):
+                    raise
+                fqt1.im2col(x.detach().contiguous(), N, C, H, W, kh, kw, stride, pad, sx_row, sx_col, cs_x)
         else:
             fqt1.im2col(x.detach(), N, C, H, W, kh, kw, stride, pad, sx_row, sx_col, cs_x)
         g = gamma.detach().contiguous()
@@ -125,8 +139,8 @@ class _BinaryProduct(torch.autograd.Function):
                     acc_dx = torch.empty(max(cap_s * rpg, 1), K, dtype=torch.int32, device=dev)
                     fqt1.bwd_input_gemm(psq, sw_col, cs_w, M, D, K, p_s, acc_dx, None)
                     fqt1.col2im(acc_dx, psq, cs_w, N, C, H, W, kh, kw, stride, pad, dx)
-            if q.ste_clip is not None:
-                fqt1.ste_clip(x, dx, dx.numel(), q.ste_clip)
+            if q.ste_clip is not None:  # x and dx elementwise in the same (contiguous) layout
+                fqt1.ste_clip(x.contiguous(), dx, dx.numel(), q.ste_clip)
         if ctx.needs_input_grad[1]:
             acc_dw = torch.empty(max(cap_c, 1), K, dtype=torch.int32, device=dev)
             dw = torch.empty(D, K, dtype=torch.float32, device=dev)

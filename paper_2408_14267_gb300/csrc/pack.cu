@@ -178,6 +178,8 @@ constexpr int kUnfoldMaxStreamWords = 24576;  // 96 KB of input bit streams per 
 
 struct UnfoldArgs {
   const float* x;
+  const uint32_t* planes;  // or the sign bits of x as planes [N][C][pw] words (then x is unused)
+  int pw;                  // words per plane, ceil(H W / 32)
   uint32_t* row_bits;
   uint32_t* col_bits;
   int32_t* colsum;
@@ -352,7 +354,23 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
   //    warp, warp + 8, ... with 16 loads in flight per lane (unconditional, from clamped
   //    indices), so the region costs one memory round trip per 128 words, not one per plane
   const int plane_bits = nrows * a.W, data_words = plane_words - 2 * a.guard, gbits = 32 * a.guard;
-  {
+  if (a.planes) {
+    // the signs are given as plane bits: word q of a region plane is the 32 bits from bit
+    // h_lo W + 32 q of the full plane (a funnel shift of two words), zero past its rows
+    const int total = nplanes * data_words, bit0 = h_lo * a.W;
+    const FastDiv div_dw((uint32_t)max(data_words, 1)), div_nc((uint32_t)nc);
+    for (int f = threadIdx.x; f < total; f += 256) {
+      const int pl = (int)div_dw.div((uint32_t)f), q = f - pl * data_words;
+      const int nn = (int)div_nc.div((uint32_t)pl), c = pl - nn * nc;
+      const uint32_t* src = a.planes + ((int64_t)(n_lo + nn) * a.C + c_lo + c) * a.pw;
+      const int b = bit0 + 32 * q, w0 = b >> 5;
+      const uint32_t lo = __ldg(src + min(w0, a.pw - 1)), hi = __ldg(src + min(w0 + 1, a.pw - 1));
+      uint32_t word = __funnelshift_r(lo, hi, b & 31);
+      const int left = plane_bits - 32 * q;
+      if (left < 32) word &= left <= 0 ? 0u : ((1u << left) - 1u);
+      stream[pl * plane_words + a.guard + q] = word;
+    }
+  } else {
     const int total = nplanes * data_words;
     const FastDiv div_dw((uint32_t)max(data_words, 1)), div_nc((uint32_t)nc);
     const int64_t img_stride = (int64_t)a.C * a.H * a.W;
@@ -528,6 +546,7 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
 //     32-lane writes) and leave as 16-byte stores; the column sums come from the same reads.
 struct UnfoldSameArgs {
   const float* x;
+  const uint32_t* planes;  // or the sign bits of x as planes [N][C][dw] words (then x is unused)
   uint32_t* row_bits;
   uint32_t* col_bits;
   int32_t* colsum;
@@ -579,7 +598,15 @@ __global__ void __launch_bounds__(256) unfold_same_kernel(UnfoldSameArgs a) {
     const uint32_t inv = (uint32_t)(0xFFFFFFFFu / (uint32_t)span) + 1u;
     const float* src = a.x + ((int64_t)n_lo * a.C + c_lo) * a.HW + lane;
     const int64_t img_stride = (int64_t)a.C * a.HW;
-    for (int f0 = warp; f0 < total; f0 += 8 * 16) {
+    if (a.planes) {  // the signs given as plane bits: the region is a copy of plane words
+      const uint32_t* ps = a.planes + ((int64_t)n_lo * a.C + c_lo) * a.dw;
+      const int64_t img_w = (int64_t)a.C * a.dw;
+      for (int f = threadIdx.x; f < total; f += 256) {
+        const int img = (int)__umulhi((uint32_t)f, inv);
+        st[f] = __ldg(ps + img * img_w + (f - img * span));
+      }
+    }
+    for (int f0 = warp; !a.planes && f0 < total; f0 += 8 * 16) {
       // unconditional loads from clamped word indices (the ballots of words past the region are
       // not stored): a load under a condition is not hoisted, and the 16 round trips serialize
       float v[16];
@@ -794,6 +821,37 @@ __global__ void __launch_bounds__(256) expand_signs_kernel(const uint32_t* __res
   }
   *reinterpret_cast<uint4*>(out + r * ld_out + e0) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
 }
+
+// ------------------------------------------------------------------ channels-last input
+// Sign bits of a channels-last x (N, H, W, C in memory) as planes [N][C][pw], pw = ceil(H W / 32):
+// bit e of word q of plane (n, c) is sign(x[n, c, pixel 32 q + e]) > 0.  A warp takes 32 pixels x
+// 32 channels: lane p reads its pixel's 32 channels (128 contiguous bytes), forms their sign
+// word, and the warp transpose turns the 32 pixel words into the 32 plane words.
+__global__ void __launch_bounds__(256) pack_planes_nhwc_kernel(const float* __restrict__ x, int N, int C, int HW,
+                                                               int pw, uint32_t* __restrict__ planes) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int cbs = C / 32;
+  const int64_t units = (int64_t)N * pw * cbs;
+  for (int64_t u = (int64_t)blockIdx.x * 8 + warp; u < units; u += (int64_t)gridDim.x * 8) {  // warp-uniform
+    const int64_t n = u / ((int64_t)pw * cbs);
+    const int rem = (int)(u - n * pw * cbs), q = rem / cbs, cb = rem - q * cbs;
+    const int p = 32 * q + lane;
+    const float4* src = reinterpret_cast<const float4*>(x + ((n * HW + min(p, HW - 1)) * C + 32 * cb));
+    float4 v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = __ldg(src + k);
+    uint32_t wd = 0;
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      wd |= (v[k].x > 0.f ? 1u : 0u) << (4 * k) | (v[k].y > 0.f ? 2u : 0u) << (4 * k) |
+            (v[k].z > 0.f ? 4u : 0u) << (4 * k) | (v[k].w > 0.f ? 8u : 0u) << (4 * k);
+    if (p >= HW) wd = 0u;
+    const uint32_t pwd = warp_transpose32(wd, lane);  // lane c: channel 32 cb + c over the 32 pixels
+    planes[(n * C + 32 * cb + lane) * pw + q] = pwd;
+  }
+}
 }  // namespace fqt1
 
 using namespace fqt1;
@@ -831,15 +889,17 @@ extern "C" fqt1_status fqt1_binarize_pack(const float* x, int64_t rows, int64_t 
   return FQT1_OK;
 }
 
-extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh,
-                                   int32_t kw, int32_t stride, int32_t pad, uint32_t* row_bits, uint32_t* col_bits,
-                                   int32_t* colsum, void* stream) {
-  if (!x || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 || pad < 0)
+// The Unfolder of fqt1_im2col (x given) and of fqt1_im2col_planes (planes given: the sign bits of x
+// as [N][C][ceil(H W / 32)] words; shapes that only the gather path serves are unsupported there).
+static fqt1_status im2col_impl(const float* x, const uint32_t* planes, int32_t N, int32_t C, int32_t H, int32_t W,
+                               int32_t kh, int32_t kw, int32_t stride, int32_t pad, uint32_t* row_bits,
+                               uint32_t* col_bits, int32_t* colsum, void* stream) {
+  if ((!x && !planes) || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 || pad < 0)
     return FQT1_ERR_INVALID_ARG;
   if (!row_bits && !col_bits && !colsum) return FQT1_ERR_INVALID_ARG;
   const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
   if (H + 2 * pad < kh || W + 2 * pad < kw || Ho < 1 || Wo < 1) return FQT1_ERR_INVALID_ARG;
-  if (!aligned16(x) || (row_bits && !aligned16(row_bits)) || (col_bits && !aligned16(col_bits)) ||
+  if ((x && !aligned16(x)) || (row_bits && !aligned16(row_bits)) || (col_bits && !aligned16(col_bits)) ||
       (colsum && !aligned16(colsum)))
     return FQT1_ERR_MISALIGNED;
   if ((int64_t)N * C * H * W >= (1ll << 31) || (int64_t)N * Ho * Wo >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
@@ -851,7 +911,7 @@ extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t
   if (same && pad <= 32 && Ki < (1ll << 31) && (128 % (H * W) == 0 || H * W == 256)) {
     // whole images per tile: the contiguous-region Unfolder
     UnfoldSameArgs u;
-    u.x = x; u.row_bits = row_bits; u.col_bits = col_bits; u.colsum = colsum;
+    u.x = x; u.planes = planes; u.row_bits = row_bits; u.col_bits = col_bits; u.colsum = colsum;
     u.row_words = fqt1_packed_words(Ki); u.col_words = fqt1_packed_words(Mi);
     u.N = N; u.C = C; u.H = H; u.W = W; u.pad = pad; u.kw = kw; u.khw = kh * kw; u.K = (int)Ki; u.HW = H * W;
     u.dw = H * W / 32;
@@ -894,7 +954,8 @@ extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t
       const int64_t words = imgs * chans * (((int64_t)H * W + 31) / 32 + 2 * guard);
       if (words > kUnfoldMaxStreamWords) continue;
       UnfoldArgs u;
-      u.x = x; u.row_bits = row_bits; u.col_bits = col_bits; u.colsum = colsum;
+      u.x = x; u.planes = planes; u.pw = (H * W + 31) / 32;
+      u.row_bits = row_bits; u.col_bits = col_bits; u.colsum = colsum;
       u.row_words = fqt1_packed_words(Ki); u.col_words = fqt1_packed_words(Mi);
       u.C = C; u.H = H; u.W = W; u.kh = kh; u.kw = kw; u.stride = stride; u.pad = pad; u.Wo = Wo;
       u.M = (int)Mi; u.K = (int)Ki; u.khw = kh * kw; u.HWo = Ho * Wo; u.tm = tm;
@@ -923,6 +984,7 @@ extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t
       return FQT1_OK;
     }
   }
+  if (!x) return FQT1_ERR_UNSUPPORTED;  // the gather path reads x itself
   Im2colLoader L;
   L.x = x; L.rows = (int64_t)N * Ho * Wo; L.cols = (int64_t)C * kh * kw;
   L.H = H; L.W = W; L.stride = stride; L.pad = pad; L.CHW = C * H * W; L.HW = H * W;
@@ -1010,5 +1072,34 @@ extern "C" fqt1_status fqt1_binarize_pack_e4m3(const float* x, int64_t rows, int
                            col_words, bands));
     fqt1_count_launches(1);
   }
+  return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh,
+                                   int32_t kw, int32_t stride, int32_t pad, uint32_t* row_bits, uint32_t* col_bits,
+                                   int32_t* colsum, void* stream) {
+  if (!x) return FQT1_ERR_INVALID_ARG;
+  return im2col_impl(x, nullptr, N, C, H, W, kh, kw, stride, pad, row_bits, col_bits, colsum, stream);
+}
+
+extern "C" fqt1_status fqt1_im2col_planes(const uint32_t* planes, int32_t N, int32_t C, int32_t H, int32_t W,
+                                          int32_t kh, int32_t kw, int32_t stride, int32_t pad, uint32_t* row_bits,
+                                          uint32_t* col_bits, int32_t* colsum, void* stream) {
+  if (!planes) return FQT1_ERR_INVALID_ARG;
+  return im2col_impl(nullptr, planes, N, C, H, W, kh, kw, stride, pad, row_bits, col_bits, colsum, stream);
+}
+
+extern "C" fqt1_status fqt1_pack_planes_nhwc(const float* x, int32_t N, int32_t C, int32_t H, int32_t W,
+                                             uint32_t* planes, void* stream) {
+  if (!x || !planes || N < 1 || C < 1 || H < 1 || W < 1) return FQT1_ERR_INVALID_ARG;
+  if (C % 32 != 0) return FQT1_ERR_UNSUPPORTED;
+  if (!aligned16(x)) return FQT1_ERR_MISALIGNED;
+  if ((int64_t)N * C * H * W >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
+  const int pw = (H * W + 31) / 32;
+  const int64_t units = (int64_t)N * pw * (C / 32);
+  const unsigned blocks = (unsigned)std::min<int64_t>((units + 7) / 8, 152 * 16);
+  FQT1_CUDA_TRY(launch_k(pack_planes_nhwc_kernel, dim3(blocks), dim3(256), 0, (cudaStream_t)stream, x, N, C, H * W,
+                         pw, planes));
+  fqt1_count_launches(1);
   return FQT1_OK;
 }

@@ -56,6 +56,8 @@ _SIGS = {
     "fqt1_fwd_gemm_e4m3w": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _I64, _VP, _VP, _VP, _VP, _VP]),
     "fqt1_bwd_input_fold_e4m3w": (C.c_int, [_VP, _VP, _I64, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP]),
     "fqt1_pack_pixels": (C.c_int, [_VP, _I32, _I32, _I32, _I32, _VP, _VP]),
+    "fqt1_pack_planes_nhwc": (C.c_int, [_VP, _I32, _I32, _I32, _I32, _VP, _VP]),
+    "fqt1_im2col_planes": (C.c_int, [_VP] + [_I32] * 8 + [_VP, _VP, _VP, _VP]),
     "fqt1_pack_weight_taps": (C.c_int, [_VP, _I64, _I32, _I32, _I32, _VP, _VP]),
     "fqt1_conv_implicit_supported": (_I32, [_I32] * 8),
     "fqt1_conv_fwd_implicit": (C.c_int, [_VP, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP, _VP, _VP]),
@@ -182,6 +184,19 @@ def bwd_input_fold_e4m3w(psq, wt_e4m3, colsum_w, N, Cin, H, W, kh, kw, stride, p
     _check(lib().fqt1_bwd_input_fold_e4m3w(C.byref(psq.c), _p(wt_e4m3), wt_e4m3.shape[-1], _p(colsum_w), N, Cin, H,
                                            W, kh, kw, stride, pad, D, C.byref(p), _p(dx), _s(stream)),
            "fqt1_bwd_input_fold_e4m3w")
+
+
+def plane_words(H, W):
+    return (H * W + 31) // 32
+
+
+def pack_planes_nhwc(x, N, Cin, H, W, planes, stream=None):
+    _check(lib().fqt1_pack_planes_nhwc(_p(x), N, Cin, H, W, _p(planes), _s(stream)), "fqt1_pack_planes_nhwc")
+
+
+def im2col_planes(planes, N, Cin, H, W, kh, kw, stride, pad, row_bits=None, col_bits=None, colsum=None, stream=None):
+    _check(lib().fqt1_im2col_planes(_p(planes), N, Cin, H, W, kh, kw, stride, pad, _p(row_bits), _p(col_bits),
+                                    _p(colsum), _s(stream)), "fqt1_im2col_planes")
 
 
 def pack_pixels(x, N, Cin, H, W, x_pix, stream=None):

@@ -154,3 +154,24 @@ def test_layers_compose_with_torch():
             assert p.grad is not None and torch.isfinite(p.grad).all()
         grads.append(net[0].weight.grad.clone())
     assert not torch.equal(grads[0], grads[1])
+
+
+def test_conv2d_channels_last_input_matches_nchw():
+    """A channels-last input takes the plane-bit Unfolder path (no copy of x) and gives the
+    same output and gradients as the same input in NCHW layout."""
+    from paper_2408_14267_gb300 import binop
+    torch.manual_seed(3)
+    layer = binop.Conv2d(64, 32, 3, padding=1, bias=True)
+    x = torch.randn(4, 64, 16, 16, device="cuda")
+    gy = torch.randn(4, 32, 16, 16, device="cuda") * 1e-3
+    res = []
+    for fmt in (torch.contiguous_format, torch.channels_last):
+        xi = x.clone().contiguous(memory_format=fmt).requires_grad_(True)
+        layer.zero_grad()
+        layer.next_seeds = (11, 12)
+        y = layer(xi)
+        y.backward(gy)
+        res.append((y.detach().clone(), xi.grad.clone(), layer.weight.grad.clone(), layer.gamma.grad.clone(),
+                    layer.bias.grad.clone()))
+    for a, b in zip(*res):
+        assert torch.equal(a, b)

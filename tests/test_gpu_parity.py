@@ -561,3 +561,48 @@ def test_host_copy_step_matches_serial(name, make):
     torch.cuda.synchronize()
     for h, r, what in zip(h_out, ref, ("y", "dx", "dw")):
         assert torch.equal(h, r.cpu()), what
+
+
+@pytest.mark.parametrize("N,C,H,W,k,s,p", [(3, 64, 8, 8, 3, 1, 1), (2, 64, 32, 32, 3, 1, 1), (2, 32, 16, 16, 3, 2, 1),
+                                           (2, 96, 7, 9, 3, 1, 1), (3, 64, 4, 4, 1, 1, 0), (2, 32, 20, 20, 7, 2, 3)])
+def test_im2col_from_channels_last_planes(N, C, H, W, k, s, p):
+    """Channels-last input: the plane bits equal the signs of x, and the Unfolder reading them
+    writes the same rows, columns and column sums as the Unfolder reading x."""
+    from paper_2408_14267_gb300 import fqt1
+    rng = np.random.default_rng(N * C + H + k)
+    x = rng.standard_normal((N, C, H, W)).astype(np.float32)
+    x[0, :2, 0, 0] = 0.0
+    xt = torch.from_numpy(x).cuda()
+    xl = xt.contiguous(memory_format=torch.channels_last)
+    pw = fqt1.plane_words(H, W)
+    planes = torch.full((N * C * pw,), -1, dtype=torch.int32, device="cuda")
+    fqt1.pack_planes_nhwc(xl, N, C, H, W, planes)
+    Ho, Wo = om.conv_out_hw(H, W, k, k, s, p)
+    M, K = N * Ho * Wo, C * k * k
+    outs = []
+    for use_planes in (False, True):
+        rb = torch.full((M, fqt1.packed_words(K)), 7, dtype=torch.int32, device="cuda")
+        cbits = torch.full((K, fqt1.packed_words(M)), 7, dtype=torch.int32, device="cuda")
+        cs = torch.empty(K, dtype=torch.int32, device="cuda")
+        if use_planes:
+            fqt1.im2col_planes(planes, N, C, H, W, k, k, s, p, rb, cbits, cs)
+        else:
+            fqt1.im2col(xt, N, C, H, W, k, k, s, p, rb, cbits, cs)
+        outs.append((rb, cbits, cs))
+    torch.cuda.synchronize()
+    w = planes.cpu().numpy().view(np.uint32).reshape(N, C, pw)
+    bits = ((w[:, :, :, None] >> np.arange(32, dtype=np.uint32)) & 1).reshape(N, C, -1)
+    assert np.array_equal(bits[:, :, :H * W].astype(np.int8) * 2 - 1, om.sign(x).reshape(N, C, H * W))
+    assert not bits[:, :, H * W:].any()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+
+
+def test_im2col_planes_rejects_gather_shapes():
+    """Shapes served only by the gather Unfolder (which reads x itself) are unsupported from planes."""
+    from paper_2408_14267_gb300 import fqt1
+    N, C, H, W = 2, 256, 56, 56
+    planes = torch.zeros(N * C * fqt1.plane_words(H, W), dtype=torch.int32, device="cuda")
+    rb = torch.empty(N * H * W, fqt1.packed_words(C), dtype=torch.int32, device="cuda")
+    with pytest.raises(fqt1.Fqt1Error, match="UNSUPPORTED"):
+        fqt1.im2col_planes(planes, N, C, H, W, 1, 1, 1, 0, rb, None, None)
