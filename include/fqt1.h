@@ -173,6 +173,17 @@ fqt1_status fqt1_pack_planes_nhwc(const float* x, int32_t N, int32_t C, int32_t 
 fqt1_status fqt1_im2col_planes(const uint32_t* planes, int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh,
                                int32_t kw, int32_t stride, int32_t pad, uint32_t* row_bits, uint32_t* col_bits,
                                int32_t* colsum, void* stream);
+/* fqt1_col2im and fqt1_bwd_input_fold with dx in channels-last memory order
+ * (N, H, W, C): the same values, element (n, c, h, w) at ((n H + h) W + w) C + c.
+ * fqt1_col2im_nhwc returns FQT1_ERR_UNSUPPORTED for shapes that fqt1_col2im
+ * serves with its untiled kernel. */
+fqt1_status fqt1_col2im_nhwc(const int32_t* acc, const fqt1_qgrad* psq, const int32_t* colsum_w, int32_t N,
+                             int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad,
+                             float* dx, void* stream);
+fqt1_status fqt1_bwd_input_fold_nhwc(const fqt1_qgrad* psq, const uint32_t* sw_col, const int32_t* colsum_w,
+                                     int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw,
+                                     int32_t stride, int32_t pad, int64_t D, const fqt1_agp_params* p, float* dx,
+                                     void* stream);
 
 /* Binarized forward GEMM (Sec. 5.1, App. C "binary multiplication"):
  * acc[m, j] = sum_k sign(X)[m, k] sign(W)[j, k], y[m, j] = gamma[j] * acc[m, j] (fp32).

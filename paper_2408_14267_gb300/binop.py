@@ -98,6 +98,7 @@ class _BinaryProduct(torch.autograd.Function):
         fqt1.fwd_gemm_bias(sx_row, sw_row, M, D, K, g, b, acc, y)
         ctx.layer, ctx.shape = layer, (M, K, D, rpg)
         ctx.in_shape = tuple(x.shape)
+        ctx.nhwc = nhwc
         ctx.has_bias = bias is not None
         ctx.save_for_backward(x if layer.qcfg.ste_clip is not None else None,
                               weight if layer.qcfg.ste_clip is not None else None, g, acc, sx_col, cs_x, sw_col, cs_w)
@@ -132,15 +133,32 @@ class _BinaryProduct(torch.autograd.Function):
                 N, C, H, W = ctx.in_shape
                 kh, kw, stride, pad = layer.conv
                 Ho, Wo = conv_out_hw(H, W, kh, kw, stride, pad)
-                dx = torch.empty(N, C, H, W, dtype=torch.float32, device=dev)
+                # a channels-last input gets its gradient channels-last too (returned as an NCHW
+                # view of NHWC memory), so that the layers before it need no layout copy
+                nhwc = ctx.nhwc
+                dx = torch.empty((N, H, W, C) if nhwc else (N, C, H, W), dtype=torch.float32, device=dev)
                 if fqt1.fold_supported(Ho, Wo, kh, kw, H, W):
-                    fqt1.bwd_input_fold(psq, sw_col, cs_w, N, C, H, W, kh, kw, stride, pad, D, p_s, dx)
+                    fqt1.bwd_input_fold(psq, sw_col, cs_w, N, C, H, W, kh, kw, stride, pad, D, p_s, dx, nhwc=nhwc)
                 else:
                     acc_dx = torch.empty(max(cap_s * rpg, 1), K, dtype=torch.int32, device=dev)
                     fqt1.bwd_input_gemm(psq, sw_col, cs_w, M, D, K, p_s, acc_dx, None)
-                    fqt1.col2im(acc_dx, psq, cs_w, N, C, H, W, kh, kw, stride, pad, dx)
-            if q.ste_clip is not None:  # x and dx elementwise in the same (contiguous) layout
-                fqt1.ste_clip(x.contiguous(), dx, dx.numel(), q.ste_clip)
+                    try:
+                        fqt1.col2im(acc_dx, psq, cs_w, N, C, H, W, kh, kw, stride, pad, dx, nhwc=nhwc)
+                    except fqt1.Fqt1Error as e:  # untiled Folder shapes write NCHW only
+                        if not nhwc or "UNSUPPORTED" not in str(e):
+                            raise
+                        nhwc = False
+                        dx = torch.empty(N, C, H, W, dtype=torch.float32, device=dev)
+                        fqt1.col2im(acc_dx, psq, cs_w, N, C, H, W, kh, kw, stride, pad, dx)
+                if nhwc:
+                    dx = dx.permute(0, 3, 1, 2)
+            if q.ste_clip is not None:  # x and dx elementwise in the same memory order
+                if dx.is_contiguous():
+                    fqt1.ste_clip(x.contiguous(), dx, dx.numel(), q.ste_clip)
+                else:  # channels-last dx: x in the same order
+                    xm = x.contiguous(memory_format=torch.channels_last)
+                    fqt1.ste_clip(xm.permute(0, 2, 3, 1).contiguous(), dx.permute(0, 2, 3, 1), dx.numel(),
+                                  q.ste_clip)
         if ctx.needs_input_grad[1]:
             acc_dw = torch.empty(max(cap_c, 1), K, dtype=torch.int32, device=dev)
             dw = torch.empty(D, K, dtype=torch.float32, device=dev)

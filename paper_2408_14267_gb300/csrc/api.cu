@@ -144,6 +144,7 @@ struct FoldArgs {
   int N, C, H, W, kh, kw, stride, pad, Ho, Wo;
   int cb, hb, ncb, max_rows, kstride;
   int64_t K;
+  int nhwc;  // dx in memory order N, H, W, C (outputs walked channels fastest) instead of NCHW
 };
 
 __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
@@ -212,9 +213,16 @@ __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
   }
   __syncthreads();
   const float sc = __ldg(a.scale + slot), ze = __ldg(a.zero + slot);
-  const FastDiv div_plane((uint32_t)plane), div_w((uint32_t)a.W);
+  const FastDiv div_plane((uint32_t)plane), div_w((uint32_t)a.W), div_nc((uint32_t)nc);
   for (int e = threadIdx.x; e < nc * plane; e += blockDim.x) {  // output (channel, row, column) of the block
-    const int cl = (int)div_plane.div((uint32_t)e), pos = e - cl * plane;
+    int cl, pos;
+    if (a.nhwc) {  // channels fastest: a pixel's nc channels are contiguous in dx
+      pos = (int)div_nc.div((uint32_t)e);
+      cl = e - pos * nc;
+    } else {
+      cl = (int)div_plane.div((uint32_t)e);
+      pos = e - cl * plane;
+    }
     const int hl = (int)div_w.div((uint32_t)pos), w = pos - hl * a.W;
     const int kc = cl * khw;
     int32_t acc = 0, csum = 0;
@@ -229,8 +237,11 @@ __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
         csum += css[kc + i * a.kw + j];
       }
     }
-    a.dx[(((int64_t)n * a.C + c0 + cl) * a.H + h0 + hl) * a.W + w] =
-        __fadd_rn(__fmul_rn(sc, __int2float_rn(acc)), __fmul_rn(ze, __int2float_rn(csum)));
+    const float v = __fadd_rn(__fmul_rn(sc, __int2float_rn(acc)), __fmul_rn(ze, __int2float_rn(csum)));
+    if (a.nhwc)
+      a.dx[(((int64_t)n * a.H + h0 + hl) * a.W + w) * a.C + c0 + cl] = v;
+    else
+      a.dx[(((int64_t)n * a.C + c0 + cl) * a.H + h0 + hl) * a.W + w] = v;
   }
 }
 
@@ -339,9 +350,10 @@ extern "C" fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t
   return FQT1_OK;
 }
 
-extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, const int32_t* colsum_w, int32_t N,
-                                   int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,
-                                   int32_t pad, float* dx, void* stream) {
+// nhwc: dx in memory order N, H, W, C; only the tiled Folder writes it (else FQT1_ERR_UNSUPPORTED).
+static fqt1_status col2im_impl(const int32_t* acc, const fqt1_qgrad* psq, const int32_t* colsum_w, int32_t N,
+                               int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad,
+                               float* dx, int nhwc, void* stream) {
   if (!acc || !psq || !colsum_w || !dx || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 ||
       pad < 0)
     return FQT1_ERR_INVALID_ARG;
@@ -379,6 +391,7 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
     fa.cs = colsum_w; fa.dx = dx; fa.N = N; fa.C = C; fa.H = H; fa.W = W; fa.kh = kh; fa.kw = kw;
     fa.stride = stride; fa.pad = pad; fa.Ho = Ho; fa.Wo = Wo; fa.cb = cb; fa.hb = hb;
     fa.ncb = (C + cb - 1) / cb; fa.max_rows = max_rows; fa.kstride = kstride; fa.K = (int64_t)C * khw;
+    fa.nhwc = nhwc;
     const int64_t nblk = (int64_t)fa.ncb * ((H + hb - 1) / hb);
     if (nblk > 0x7FFFFFFF || N > 65535) return FQT1_ERR_UNSUPPORTED;
     const size_t smem =
@@ -388,6 +401,7 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
     const int64_t cap = fqt1_kept_capacity(N, 8, FQT1_SEL_BERNOULLI);  // upper bound: all samples
     launch_k(col2im_tiled_kernel, dim3((unsigned)nblk, (unsigned)cap), dim3(256), smem, (cudaStream_t)stream, fa);
   } else {
+    if (nhwc) return FQT1_ERR_UNSUPPORTED;
     const int64_t n = (int64_t)N * C * H * W;
     launch_k(col2im_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, (cudaStream_t)stream, 
         acc, psq->slot_of_group, psq->scale, psq->zero, colsum_w, N, C, H, W, kh, kw, stride, pad, Ho, Wo, dx);
@@ -397,12 +411,24 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
   return FQT1_OK;
 }
 
+extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, const int32_t* colsum_w, int32_t N,
+                                   int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,
+                                   int32_t pad, float* dx, void* stream) {
+  return col2im_impl(acc, psq, colsum_w, N, C, H, W, kh, kw, stride, pad, dx, 0, stream);
+}
+
+extern "C" fqt1_status fqt1_col2im_nhwc(const int32_t* acc, const fqt1_qgrad* psq, const int32_t* colsum_w, int32_t N,
+                                        int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,
+                                        int32_t pad, float* dx, void* stream) {
+  return col2im_impl(acc, psq, colsum_w, N, C, H, W, kh, kw, stride, pad, dx, 1, stream);
+}
+
 // Shared by the two Folder entry points: B is the packed sign(W) columns sw_col, or (wt_e4m3
 // non-null) the e4m3 bytes of sign(W)^T with rows of ld_wt bytes.
 static fqt1_status bwd_input_fold_impl(const fqt1_qgrad* psq, const uint32_t* sw_col, const uint8_t* wt_e4m3,
                                        int64_t ld_wt, const int32_t* colsum_w, int32_t N, int32_t C, int32_t H,
                                        int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad, int64_t D,
-                                       const fqt1_agp_params* p, float* dx, void* stream) {
+                                       const fqt1_agp_params* p, float* dx, int nhwc, void* stream) {
   if (!psq || (!sw_col && !wt_e4m3) || !colsum_w || !p || !dx || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 ||
       kw < 1 || stride < 1 || pad < 0 || D < 1)
     return FQT1_ERR_INVALID_ARG;
@@ -427,7 +453,7 @@ static fqt1_status bwd_input_fold_impl(const fqt1_qgrad* psq, const uint32_t* sw
   FQT1_CUDA_TRY(launch_fold_tc(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, sw_col,
                                (int64_t)C * kh * kw, D, psq->kept_idx, psq->scale, psq->zero, colsum_w,
                                psq->slot_of_group, dx, N, C, H, W, kh, kw, stride, pad, Ho, Wo, nullptr, s,
-                               wt_e4m3, ld_wt));
+                               wt_e4m3, ld_wt, nhwc));
   return FQT1_OK;
 }
 
@@ -436,7 +462,15 @@ extern "C" fqt1_status fqt1_bwd_input_fold(const fqt1_qgrad* psq, const uint32_t
                                            int32_t stride, int32_t pad, int64_t D, const fqt1_agp_params* p,
                                            float* dx, void* stream) {
   if (!sw_col) return FQT1_ERR_INVALID_ARG;
-  return bwd_input_fold_impl(psq, sw_col, nullptr, 0, colsum_w, N, C, H, W, kh, kw, stride, pad, D, p, dx, stream);
+  return bwd_input_fold_impl(psq, sw_col, nullptr, 0, colsum_w, N, C, H, W, kh, kw, stride, pad, D, p, dx, 0, stream);
+}
+
+extern "C" fqt1_status fqt1_bwd_input_fold_nhwc(const fqt1_qgrad* psq, const uint32_t* sw_col,
+                                                const int32_t* colsum_w, int32_t N, int32_t C, int32_t H, int32_t W,
+                                                int32_t kh, int32_t kw, int32_t stride, int32_t pad, int64_t D,
+                                                const fqt1_agp_params* p, float* dx, void* stream) {
+  if (!sw_col) return FQT1_ERR_INVALID_ARG;
+  return bwd_input_fold_impl(psq, sw_col, nullptr, 0, colsum_w, N, C, H, W, kh, kw, stride, pad, D, p, dx, 1, stream);
 }
 
 extern "C" fqt1_status fqt1_bwd_input_fold_e4m3w(const fqt1_qgrad* psq, const uint8_t* wt_e4m3, int64_t ld_wt,
@@ -445,7 +479,7 @@ extern "C" fqt1_status fqt1_bwd_input_fold_e4m3w(const fqt1_qgrad* psq, const ui
                                                  const fqt1_agp_params* p, float* dx, void* stream) {
   if (!wt_e4m3) return FQT1_ERR_INVALID_ARG;
   return bwd_input_fold_impl(psq, nullptr, wt_e4m3, ld_wt, colsum_w, N, C, H, W, kh, kw, stride, pad, D, p, dx,
-                             stream);
+                             0, stream);
 }
 
 extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_t* sx_col, const int32_t* colsum_x,

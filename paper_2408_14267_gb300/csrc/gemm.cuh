@@ -29,11 +29,12 @@ cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int6
                                    int32_t* status, cudaStream_t s);
 enum : int { GEMM_EPI_ACC32 = 1, GEMM_EPI_RED = 2, GEMM_EPI_DX = 3 };
 // Bte: e4m3 sign(W)^T rows [K][ldbte] bytes, or null for the packed sign(W) columns Sg.
+// nhwc: dx in memory order N, H, W, C.
 cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
                            const uint32_t* Sg, int64_t K, int64_t D, const int32_t* kept_idx, const float* scale,
                            const float* zero, const int32_t* cs, const int32_t* slot_of_group, float* dx, int N, int C,
                            int H, int W, int kh, int kw, int stride, int pad, int Ho, int Wo, int32_t* status,
-                           cudaStream_t s, const uint8_t* Bte = nullptr, int64_t ldbte = 0);
+                           cudaStream_t s, const uint8_t* Bte = nullptr, int64_t ldbte = 0, int nhwc = 0);
 // Forward with B = e4m3 sign(W) rows [D][ldbe] bytes (+1 = 0x38, -1 = 0xB8, bytes past K zero).
 cudaError_t launch_fwd_e4m3w_tc(const uint32_t* A, const uint8_t* Be, int64_t ldbe, int64_t M, int64_t D, int64_t K,
                                 const float* gamma, const float* bias, int32_t* acc, float* y, int32_t* status,

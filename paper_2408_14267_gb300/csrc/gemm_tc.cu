@@ -67,6 +67,7 @@ struct TcArgs {
   // EPI_FWD / EPI_ACC32: bit 0 = y, bit 1 = acc leave through TMA stores (tmY / tmAcc)
   int tma_out;
   int fN;  // EPI_FOLD: samples (pruned ones are zeroed by the kernel)
+  int fnhwc;  // EPI_FOLD: dx in memory order N, H, W, C instead of NCHW
   // implicit-GEMM forward of a stride-1 "same" convolution (impl = 1): A comes from the
   // pixel-major sign words [N][H][W][C / 32] through a 4-D tensor map, one box per 128-channel
   // sub-tile of one kernel tap, shifted by the tap; the contraction index is k' = t C + c.
@@ -628,8 +629,14 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       const int32_t kid = __ldg(a.kept_idx + slot);
       const float ksc = __ldg(a.scale + slot), kze = __ldg(a.zero + slot);
       const int nsamp = a.fN > (int)blockIdx.y ? (a.fN - (int)blockIdx.y + (int)gridDim.y - 1) / (int)gridDim.y : 0;
-      const int64_t blk_bytes = (int64_t)f_nc * f_HW * 4;
-      const int pieces = (int)((blk_bytes + kFoldZero - 1) / kFoldZero);
+      // zeroing of a pruned sample: NCHW, this CTA's channel block (nc H W contiguous floats);
+      // NHWC, the whole sample (C H W contiguous floats), its 4 KB pieces dealt round-robin over
+      // the gridDim.x CTAs of the sample's row tile
+      const int64_t blk_bytes = a.fnhwc ? (int64_t)a.fC * f_HW * 4 : (int64_t)f_nc * f_HW * 4;
+      const int pieces_all = (int)((blk_bytes + kFoldZero - 1) / kFoldZero);
+      const int pieces = !a.fnhwc ? pieces_all
+                         : (pieces_all > (int)blockIdx.x
+                                ? (pieces_all - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x : 0);
       int32_t sl[4];
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
@@ -692,10 +699,11 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
           for (int u = 0; u < 4; ++u) {
             const int e = e0 + 256 * u;
             if (e >= nsamp * pieces || sl[u] >= 0) continue;
-            const int k = e / pieces, pc = e - k * pieces;
+            const int k = e / pieces, pj = e - k * pieces;
+            const int pc = a.fnhwc ? (int)blockIdx.x + pj * (int)gridDim.x : pj;
             const int64_t n = (int64_t)blockIdx.y + (int64_t)k * gridDim.y;
-            unsigned char* dst = reinterpret_cast<unsigned char*>(a.y + ((int64_t)n * a.fC + f_c0) * f_HW) +
-                                 (int64_t)pc * kFoldZero;
+            const int64_t first = a.fnhwc ? (int64_t)n * a.fC * f_HW : ((int64_t)n * a.fC + f_c0) * f_HW;
+            unsigned char* dst = reinterpret_cast<unsigned char*>(a.y + first) + (int64_t)pc * kFoldZero;
             const int64_t left = blk_bytes - (int64_t)pc * kFoldZero;
             bulk_store(dst, zb, (uint32_t)(left < kFoldZero ? left : kFoldZero));
             fold_zero_issued = true;
@@ -792,9 +800,12 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
               acc += (msk >> t) & 1u ? v[t] : 0;
               acc2 += (msk >> t) & 1u ? v2[t] : 0;
             }
-            float* yo = a.y + ((int64_t)n * a.fC + c_first) * HW + pos;
-            yo[(int64_t)cl * HW] = __fadd_rn(__fmul_rn(sc, (float)acc), __fmul_rn(ze, (float)cf));
-            if (cl2 != cl) yo[(int64_t)cl2 * HW] = __fadd_rn(__fmul_rn(sc, (float)acc2), __fmul_rn(ze, (float)cf2));
+            // channel cl of this input position: NCHW stride H W, NHWC stride 1
+            float* yo = a.fnhwc ? a.y + ((int64_t)n * HW + pos) * a.fC + c_first
+                                : a.y + ((int64_t)n * a.fC + c_first) * HW + pos;
+            const int64_t cst = a.fnhwc ? 1 : HW;
+            yo[cl * cst] = __fadd_rn(__fmul_rn(sc, (float)acc), __fmul_rn(ze, (float)cf));
+            if (cl2 != cl) yo[cl2 * cst] = __fadd_rn(__fmul_rn(sc, (float)acc2), __fmul_rn(ze, (float)cf2));
           }
         }
       }
@@ -831,8 +842,11 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
             if (o >= 0) acc += tim[o];
           }
         }
-        a.y[((int64_t)n * a.fC + c_first + cl) * HW + pos] =
-            __fadd_rn(__fmul_rn(s_scale[img], (float)acc), __fmul_rn(s_zero[img], (float)csf[rem]));
+        const float v = __fadd_rn(__fmul_rn(s_scale[img], (float)acc), __fmul_rn(s_zero[img], (float)csf[rem]));
+        if (a.fnhwc)
+          a.y[((int64_t)n * HW + pos) * a.fC + c_first + cl] = v;
+        else
+          a.y[((int64_t)n * a.fC + c_first + cl) * HW + pos] = v;
       }
       // the bulk stores of zeros must have read the zero buffer before the CTA exits
       if (fold_zero_issued) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
@@ -1270,7 +1284,7 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
                            const uint32_t* Sg, int64_t K, int64_t D, const int32_t* kept_idx, const float* scale,
                            const float* zero, const int32_t* cs, const int32_t* slot_of_group, float* dx, int N, int C,
                            int H, int W, int kh, int kw, int stride, int pad, int Ho, int Wo, int32_t* status,
-                           cudaStream_t s, const uint8_t* Bte, int64_t ldbte) {
+                           cudaStream_t s, const uint8_t* Bte, int64_t ldbte, int nhwc) {
   const int64_t lds = fqt1_packed_words(D);
   CUtensorMap ma, mb;
   if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, D, max_rows, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B))
@@ -1284,6 +1298,7 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
   }
   TcArgs a{};
   a.b_tma = Bte ? 1 : 0;
+  a.fnhwc = nhwc;
   const int khw = kh * kw, cb = 128 / khw;
   a.M = max_rows; a.N = K; a.L = D; a.count = count; a.rows_per_count = (int64_t)Ho * Wo;
   a.k_tiles = (int)((D + kCodesStageK - 1) / kCodesStageK); a.tiles_per_split = a.k_tiles;

@@ -65,6 +65,8 @@ _SIGS = {
     "fqt1_scq_quantize_noalloc": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, _VP]),
     "fqt1_bwd_input_gemm": (C.c_int, [_VP, _VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
     "fqt1_col2im": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
+    "fqt1_col2im_nhwc": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
+    "fqt1_bwd_input_fold_nhwc": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP]),
     "fqt1_bwd_input_fold": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP]),
     "fqt1_bwd_weight_gemm": (C.c_int, [_VP, _VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP, C.c_size_t, _VP]),
 }
@@ -259,14 +261,17 @@ def bwd_input_gemm(psq, sw_col, colsum_w, M, D, K, params, acc, dx, stream=None)
                                      _p(dx), _s(stream)), "fqt1_bwd_input_gemm")
 
 
-def col2im(acc, psq, colsum_w, N, Cin, H, W, kh, kw, stride, pad, dx, stream=None):
-    _check(lib().fqt1_col2im(_p(acc), C.byref(psq.c), _p(colsum_w), N, Cin, H, W, kh, kw, stride, pad, _p(dx),
-                             _s(stream)), "fqt1_col2im")
+def col2im(acc, psq, colsum_w, N, Cin, H, W, kh, kw, stride, pad, dx, stream=None, nhwc=False):
+    fn = lib().fqt1_col2im_nhwc if nhwc else lib().fqt1_col2im
+    _check(fn(_p(acc), C.byref(psq.c), _p(colsum_w), N, Cin, H, W, kh, kw, stride, pad, _p(dx), _s(stream)),
+           "fqt1_col2im_nhwc" if nhwc else "fqt1_col2im")
 
 
-def bwd_input_fold(psq, sw_col, colsum_w, N, Cin, H, W, kh, kw, stride, pad, D, params, dx, stream=None):
-    _check(lib().fqt1_bwd_input_fold(C.byref(psq.c), _p(sw_col), _p(colsum_w), N, Cin, H, W, kh, kw, stride, pad, D,
-                                     C.byref(params), _p(dx), _s(stream)), "fqt1_bwd_input_fold")
+def bwd_input_fold(psq, sw_col, colsum_w, N, Cin, H, W, kh, kw, stride, pad, D, params, dx, stream=None,
+                   nhwc=False):
+    fn = lib().fqt1_bwd_input_fold_nhwc if nhwc else lib().fqt1_bwd_input_fold
+    _check(fn(C.byref(psq.c), _p(sw_col), _p(colsum_w), N, Cin, H, W, kh, kw, stride, pad, D, C.byref(params),
+              _p(dx), _s(stream)), "fqt1_bwd_input_fold_nhwc" if nhwc else "fqt1_bwd_input_fold")
 
 
 def fold_supported(Ho, Wo, kh, kw, H, W):

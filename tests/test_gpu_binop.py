@@ -164,6 +164,12 @@ def test_conv2d_channels_last_input_matches_nchw():
     layer = binop.Conv2d(64, 32, 3, padding=1, bias=True)
     x = torch.randn(4, 64, 16, 16, device="cuda")
     gy = torch.randn(4, 32, 16, 16, device="cuda") * 1e-3
+    _check_layouts(layer, x, gy)
+    small = binop.Conv2d(32, 16, 3, padding=1, qcfg=binop.QuantConfig(4, ste_clip=1.0))  # 8 x 8: fused Folder
+    _check_layouts(small, torch.randn(6, 32, 8, 8, device="cuda"), torch.randn(6, 16, 8, 8, device="cuda") * 1e-3)
+
+
+def _check_layouts(layer, x, gy):
     res = []
     for fmt in (torch.contiguous_format, torch.channels_last):
         xi = x.clone().contiguous(memory_format=fmt).requires_grad_(True)
@@ -171,7 +177,9 @@ def test_conv2d_channels_last_input_matches_nchw():
         layer.next_seeds = (11, 12)
         y = layer(xi)
         y.backward(gy)
+        if fmt is torch.channels_last:  # the gradient comes back in the input's layout
+            assert xi.grad.is_contiguous(memory_format=torch.channels_last)
         res.append((y.detach().clone(), xi.grad.clone(), layer.weight.grad.clone(), layer.gamma.grad.clone(),
-                    layer.bias.grad.clone()))
+                    layer.bias.grad.clone() if layer.bias is not None else layer.gamma.grad.clone()))
     for a, b in zip(*res):
         assert torch.equal(a, b)

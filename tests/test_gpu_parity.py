@@ -606,3 +606,36 @@ def test_im2col_planes_rejects_gather_shapes():
     rb = torch.empty(N * H * W, fqt1.packed_words(C), dtype=torch.int32, device="cuda")
     with pytest.raises(fqt1.Fqt1Error, match="UNSUPPORTED"):
         fqt1.im2col_planes(planes, N, C, H, W, 1, 1, 1, 0, rb, None, None)
+
+
+@pytest.mark.parametrize("name,make", FOLD_CASES, ids=[c[0] for c in FOLD_CASES])
+def test_fold_channels_last_output(name, make):
+    """The fused Folder writing dx channels-last (N, H, W, C) gives the NCHW result's values,
+    pruned samples included."""
+    from paper_2408_14267_gb300 import fqt1
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    st = LayerStep(w, keep_acc=False)
+    assert st.fold
+    st.step()
+    N, C, H, W, kh, kw = st.conv
+    dx = torch.full((N, H, W, C), 3.0, device="cuda")
+    fqt1.bwd_input_fold(st.psq, st.sw_col, st.cs_w, N, C, H, W, kh, kw, st.stride, st.pad, st.D, st.p_s, dx,
+                        nhwc=True)
+    torch.cuda.synchronize()
+    assert torch.equal(dx.permute(0, 3, 1, 2), st.dx)
+
+
+@pytest.mark.parametrize("name,make", [CASES[12], CASES[15], CASES[8]], ids=[CASES[12][0], CASES[15][0], CASES[8][0]])
+def test_col2im_channels_last_output(name, make):
+    """The two-call Folder writing dx channels-last gives the NCHW result's values."""
+    from paper_2408_14267_gb300 import fqt1
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    st = LayerStep(w, keep_acc=True, fold=False)
+    st.step()
+    N, C, H, W, kh, kw = st.conv
+    dx = torch.full((N, H, W, C), 3.0, device="cuda")
+    fqt1.col2im(st.acc_dx, st.psq, st.cs_w, N, C, H, W, kh, kw, st.stride, st.pad, dx, nhwc=True)
+    torch.cuda.synchronize()
+    assert torch.equal(dx.permute(0, 3, 1, 2), st.dx)
