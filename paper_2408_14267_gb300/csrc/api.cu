@@ -506,13 +506,21 @@ extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_
     int64_t cs = wgrad_cluster_size(p->bits, out_tiles_c, k_tiles);
     int64_t tps = (k_tiles + cs - 1) / cs;
     cs = (k_tiles + tps - 1) / tps;
-    if (tps * kCodesStageK <= exact_chunk(p->bits)) {
+    // few output tiles over a long contraction (e.g. 16 kept channels x 576 columns over 131072
+    // rows) leave most SMs idle with clusters of at most 8 splits: the atomic reduction below then
+    // spreads the contraction over about one wave of CTAs instead
+    const int64_t red_splits = std::min<int64_t>(k_tiles, std::max<int64_t>((152 + out_tiles_c - 1) / out_tiles_c,
+                                                                            (M + exact_chunk(p->bits) - 1) /
+                                                                                exact_chunk(p->bits)));
+    const bool spread = tps > 8 && red_splits >= 2 * cs;
+    if (!spread && tps * kCodesStageK <= exact_chunk(p->bits)) {
       FQT1_CUDA_TRY(launch_wgrad_cluster_tc(p->bits, pcq->codes, pcq->ld_codes, cap, pcq->kept_count, sx_col, K, M,
                                             (int)cs, acc, dw, D, pcq->kept_idx, pcq->slot_of_group, pcq->scale,
                                             pcq->zero, colsum_x, nullptr, s));
       return FQT1_OK;
     }
-    // contractions too long for eight exact splits: int32 atomics across CTAs, then dequantize
+    // contractions too long for eight exact splits, or too long for so few clusters: int32
+    // atomics across CTAs, then dequantize
     const int64_t out_tiles = ((K + 127) / 128) * ((cap + 127) / 128);
     int64_t splits = (152 + out_tiles - 1) / out_tiles;  // about one wave on 152 SMs
     const int64_t min_splits = (M + exact_chunk(p->bits) - 1) / exact_chunk(p->bits);
