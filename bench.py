@@ -115,7 +115,10 @@ class ClockSampler:
     def __init__(self, gpu_index):
         self.gpu = gpu_index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_gpu{gpu_index}.csv")
+        # the raw samples go to FQT1_CLOCKS_DIR (default: the system temporary directory)
+        import tempfile
+        out_dir = os.environ.get("FQT1_CLOCKS_DIR") or tempfile.gettempdir()
+        self.path = os.path.join(out_dir, f"clocks_gpu{gpu_index}.csv")
 
     def __enter__(self):
         try:
@@ -667,7 +670,7 @@ def variance_study(args):
 
 
 def reference_arm(args, world, rank):
-    """The oracle, as it stands, timed on the host cores (the reference for this build)."""
+    """The reference arm: the oracle, as it stands, timed on the host cores."""
     if rank != 0:
         return
     batch = 32  # a bounded sample of the workload per step (32 of 128 samples)
