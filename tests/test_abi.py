@@ -110,3 +110,38 @@ def test_implicit_conv_validation_without_launch(lib):
     assert lib.fqt1_conv_fwd_implicit(*args) == 1                                  # no gamma
     args[11] = odd
     assert lib.fqt1_conv_fwd_implicit(*args) == 2                                  # misaligned gamma
+
+
+def test_layout_and_e4m3_entry_points_validate_without_launch(lib):
+    """Channels-last, e4m3 and workspace entry points reject bad arguments before any launch."""
+    from paper_2408_14267_gb300 import fqt1
+    fake = C.c_void_p(0x10000)
+    odd = C.c_void_p(0x10004)
+    s = C.c_void_p(0)
+    # channels-last packing and the Unfolder from planes
+    assert lib.fqt1_pack_planes_nhwc(fake, 2, 48, 8, 8, fake, s) == 3                     # C % 32
+    assert lib.fqt1_pack_planes_nhwc(odd, 2, 64, 8, 8, fake, s) == 2                      # misaligned x
+    assert lib.fqt1_pack_planes_nhwc(None, 2, 64, 8, 8, fake, s) == 1
+    assert lib.fqt1_im2col_planes(None, 1, 32, 8, 8, 3, 3, 1, 1, fake, None, None, s) == 1
+    assert lib.fqt1_im2col_planes(fake, 1, 32, 2, 2, 5, 5, 1, 0, fake, None, None, s) == 1  # kernel > image
+    # e4m3 copies of the signs
+    assert lib.fqt1_expand_signs_e4m3(fake, 4, 40, fake, C.c_int64(40), s) == 1            # ld % 16
+    assert lib.fqt1_expand_signs_e4m3(fake, 4, 40, fake, C.c_int64(32), s) == 1            # ld < n
+    assert lib.fqt1_expand_signs_e4m3(fake, 4, 40, odd, C.c_int64(48), s) == 2
+    assert lib.fqt1_binarize_pack_e4m3(fake, 4, 40, 40, None, None, None, fake, C.c_int64(40), None, C.c_int64(0),
+                                       s) == 1                                                  # ld_re % 16
+    assert lib.fqt1_binarize_pack_e4m3(fake, 4, 40, 40, None, None, None, None, C.c_int64(0), None, C.c_int64(0),
+                                       s) == 1                                                  # no output
+    assert lib.fqt1_fwd_gemm_e4m3w(fake, fake, C.c_int64(32), 8, 8, 40, fake, None, None, fake, s) == 1  # ld < K
+    assert lib.fqt1_fwd_gemm_e4m3w(fake, fake, C.c_int64(48), 8, 8, 40, None, None, None, fake, s) == 1  # gamma
+    # channels-last Folders
+    q = fqt1.QGrad(*(0x10000 for _ in range(9)), 64)
+    p_ok = fqt1.AgpParams(4, 0, 1, 64)
+    assert lib.fqt1_col2im_nhwc(None, C.byref(q), fake, 2, 8, 8, 8, 3, 3, 1, 1, fake, s) == 1
+    assert lib.fqt1_bwd_input_fold_nhwc(C.byref(q), None, fake, 2, 8, 8, 8, 3, 3, 1, 1, C.c_int64(16), C.byref(p_ok),
+                                        fake, s) == 1
+    assert lib.fqt1_bwd_input_fold_e4m3w(C.byref(q), fake, C.c_int64(8), fake, 2, 8, 8, 8, 3, 3, 1, 1, C.c_int64(16),
+                                         C.byref(p_ok), fake, s) == 1                           # ld_wt < D
+    # workspace preparation
+    assert lib.fqt1_scq_workspace_init(None, 64, s) == 1
+    assert lib.fqt1_scq_workspace_init(fake, 0, s) == 1
