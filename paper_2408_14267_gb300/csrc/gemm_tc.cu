@@ -66,17 +66,15 @@ struct TcArgs {
   int fC, fH, fW, fkh, fkw, fstride, fpad, fHo, fWo, fcb;
   // EPI_FWD / EPI_ACC32: bit 0 = y, bit 1 = acc leave through TMA stores (tmY / tmAcc)
   int tma_out;
-  int fN;  // EPI_FOLD: samples (pruned ones are zeroed by the kernel)
-  int fnhwc;  // EPI_FOLD: dx in memory order N, H, W, C instead of NCHW
-  // implicit-GEMM forward of a stride-1 "same" convolution (impl = 1): A comes from the
+  int fN;  // EPI_FOLD: samples (pruned ones are zeroed by the kernel; mode bit 2: dx in NHWC order)
+  // implicit-GEMM forward of a stride-1 "same" convolution (mode bit 0): A comes from the
   // pixel-major sign words [N][H][W][C / 32] through a 4-D tensor map, one box per 128-channel
   // sub-tile of one kernel tap, shifted by the tap; the contraction index is k' = t C + c.
   // A box covers 2^isb consecutive sub-tiles of one tap (rows of 16 * 2^isb bytes).
-  int impl, iC, ikw, ikhw, ipad, iW, iHW, isb;
-  // b_tma = 1: B is given as e4m3 bytes (+1 = 0x38, -1 = 0xB8, K-major rows, tmB a 128B-swizzled
-  // map of 128 x 128 boxes) and goes by TMA straight into the operand ring; all eight expansion
-  // warps then expand A, each half of a stage's sub-tiles.
-  int b_tma;
+  // (Mode bit 1: B is given as e4m3 bytes, +1 = 0x38, -1 = 0xB8, K-major rows, tmB a
+  // 128B-swizzled map of 128 x 128 boxes, and goes by TMA straight into the operand ring; all
+  // eight expansion warps then expand A, each half of a stage's sub-tiles.)
+  int iC, ikw, ikhw, ipad, iW, iHW, isb;
   // EPI_FOLD divisors (host-built): kh kw, W, kw, H W, stride, fcb H W
   FastDiv fd_khw, fd_w, fd_kw, fd_hw, fd_s, fd_cbhw;
   // EPI_CRED: the cluster's partial tiles are summed into acc (int32, ldo) and dequantized into
@@ -317,11 +315,15 @@ struct TcSmem {
 };
 
 // SHORT tiles run two CTAs per SM, which caps the registers at 65536 / (2 * 320) per thread.
-template <bool A_CODES, bool BITS8, int BN, bool SHORT>
+// X selects the optional datapaths at compile time, so that the default kernels carry none of
+// their code: bit 0 the implicit-convolution A operand, bit 1 B as e4m3 bytes by TMA (b_tma),
+// bit 2 the Folder's NHWC output.
+template <bool A_CODES, bool BITS8, int BN, bool SHORT, int X = 0>
 __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmAcc, TcArgs a) {
   using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
+  constexpr bool kImpl = (X & 1) != 0, kBtma = (X & 2) != 0, kNhwc = (X & 4) != 0;
   constexpr int OS = S::kOpStages, RS = S::kRawStages, KSUB = S::KSUB;
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t raw_full[kMaxStages], raw_empty[kMaxStages], op_full[kMaxStages],
@@ -405,7 +407,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   const int64_t valid_rows = a.count ? (int64_t)__ldg(a.count) * a.rows_per_count : a.M;
   const int nk = m0 < valid_rows ? kt1 - kt0 : 0;  // a tile past the kept rows has no work
 
-  const uint32_t kTx = a.b_tma ? (uint32_t)S::kRawA : (uint32_t)S::kRawStage;
+  const uint32_t kTx = kBtma ? (uint32_t)S::kRawA : (uint32_t)S::kRawStage;
 
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer (raw ring)
@@ -420,7 +422,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
 #pragma unroll
           for (int h = 0; h < KSUB; ++h)  // one 128-byte-swizzled box per sub-tile
             tma_load_2d(rawA(s) + h * (kBM * kBK), &tmA, &raw_full[s], (kt * KSUB + h) * kBK, (int)m0);
-        } else if (!A_CODES && a.impl) {
+        } else if (!A_CODES && kImpl) {
           // implicit convolution: box b = sub-tiles b 2^isb .. + 2^isb - 1, 128 2^isb channels
           // of one tap t; the box of the tile's output pixels shifted by (i - pad, j - pad), so
           // that a tap in the padding reads the fill value 0 (sign -1).  Boxes past the
@@ -438,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         } else {
           tma_load_2d(rawA(s), &tmA, &raw_full[s], kt * KSUB * (kBK / 32), (int)m0);
         }
-        if (!a.b_tma) tma_load_2d(rawB(s), &tmB, &raw_full[s], kt * KSUB * (kBK / 32), (int)n0);
+        if (!kBtma) tma_load_2d(rawB(s), &tmB, &raw_full[s], kt * KSUB * (kBK / 32), (int)n0);
         ++issued;
       }
       // drain: every issued copy must land before the CTA may exit
@@ -456,7 +458,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       for (int i = 0; i < nk; ++i) {
         const int s = i % OS, it = i / OS;
         if (!mbar_wait(&op_full[s], it & 1, &abort_flag, a.status)) break;
-        if (a.b_tma && !mbar_wait(&b_full[s], it & 1, &abort_flag, a.status)) break;
+        if (kBtma && !mbar_wait(&b_full[s], it & 1, &abort_flag, a.status)) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const uint32_t acol = tmem + BN + s * S::kAcols, baddr = smem_u32(opB(s));
         const int nsub = valid_subtiles<KSUB>(a.L, kt0 + i);
@@ -485,9 +487,9 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     const int64_t tile_rows = valid_rows - m0;  // may exceed kBM or be negative
     const int live_q = tile_rows >= kBM ? 4 : (tile_rows <= 0 ? 0 : (int)((tile_rows + 31) / 32));
     const bool split = KSUB == 2 && live_q <= 2;
-    const bool a_warp = a.b_tma ? true : split ? (warp == 4 || warp == 5 || warp >= 8) : warp < 6;
-    const int a_h0 = a.b_tma ? (warp >= 6 ? KSUB / 2 : 0) : (split && warp >= 8 ? 1 : 0);
-    const int a_h1 = a.b_tma ? a_h0 + KSUB / 2 : (split ? a_h0 + 1 : KSUB);
+    const bool a_warp = kBtma ? true : split ? (warp == 4 || warp == 5 || warp >= 8) : warp < 6;
+    const int a_h0 = kBtma ? (warp >= 6 ? KSUB / 2 : 0) : (split && warp >= 8 ? 1 : 0);
+    const int a_h1 = kBtma ? a_h0 + KSUB / 2 : (split ? a_h0 + 1 : KSUB);
     const int bblk = split ? (warp == 2 ? 0 : warp == 3 ? 1 : warp == 6 ? 2 : 3) : warp - 6;
     const int quarter = warp & 3;
     const int arow = 32 * quarter + lane, brow = 32 * bblk + lane;
@@ -499,7 +501,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     for (int i = 0; i < nk; ++i) {
       const int so = i % OS, ito = i / OS, sr = i % RS, itr = i / RS;
       if (ito > 0 && !mbar_wait(&op_empty[so], (ito - 1) & 1, &abort_flag, a.status)) break;
-      if (a.b_tma) {  // the stage's B boxes, as soon as the MMAs of its previous use are done
+      if (kBtma) {  // the stage's B boxes, as soon as the MMAs of its previous use are done
         if (warp == 2 && lane == 0) {
           mbar_expect_tx(&b_full[so], (uint32_t)S::kOpB);
 #pragma unroll
@@ -545,7 +547,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
               // raw rows: 16 bytes per sub-tile, interleaved per row (2-D box), or per row of a
               // box of 2^isb sub-tiles (implicit convolution)
               const int hb = (h >> a.isb) << a.isb;
-              const unsigned char* rp = a.impl ? rawA(sr) + hb * (kBM * 16) + (arow << (4 + a.isb)) + 16 * (h - hb)
+              const unsigned char* rp = kImpl ? rawA(sr) + hb * (kBM * 16) + (arow << (4 + a.isb)) + 16 * (h - hb)
                                                : rawA(sr) + arow * S::kRawRow + 16 * h;
               const uint4 w4 = *reinterpret_cast<const uint4*>(rp);
               const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
@@ -591,7 +593,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
 
     // every B box this thread issued must land before the epilogue reuses the ring or the CTA
     // exits (normally the MMA issuer has already seen them land)
-    if (a.b_tma && warp == 2 && lane == 0) {
+    if (kBtma && warp == 2 && lane == 0) {
       for (int i = (b_issued > OS ? b_issued - OS : 0); i < b_issued; ++i) {
         const int so = i % OS, ito = i / OS;
         const uint64_t t0 = gtimer();
@@ -632,9 +634,9 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       // zeroing of a pruned sample: NCHW, this CTA's channel block (nc H W contiguous floats);
       // NHWC, the whole sample (C H W contiguous floats), its 4 KB pieces dealt round-robin over
       // the gridDim.x CTAs of the sample's row tile
-      const int64_t blk_bytes = a.fnhwc ? (int64_t)a.fC * f_HW * 4 : (int64_t)f_nc * f_HW * 4;
+      const int64_t blk_bytes = kNhwc ? (int64_t)a.fC * f_HW * 4 : (int64_t)f_nc * f_HW * 4;
       const int pieces_all = (int)((blk_bytes + kFoldZero - 1) / kFoldZero);
-      const int pieces = !a.fnhwc ? pieces_all
+      const int pieces = !kNhwc ? pieces_all
                          : (pieces_all > (int)blockIdx.x
                                 ? (pieces_all - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x : 0);
       int32_t sl[4];
@@ -700,9 +702,9 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
             const int e = e0 + 256 * u;
             if (e >= nsamp * pieces || sl[u] >= 0) continue;
             const int k = e / pieces, pj = e - k * pieces;
-            const int pc = a.fnhwc ? (int)blockIdx.x + pj * (int)gridDim.x : pj;
+            const int pc = kNhwc ? (int)blockIdx.x + pj * (int)gridDim.x : pj;
             const int64_t n = (int64_t)blockIdx.y + (int64_t)k * gridDim.y;
-            const int64_t first = a.fnhwc ? (int64_t)n * a.fC * f_HW : ((int64_t)n * a.fC + f_c0) * f_HW;
+            const int64_t first = kNhwc ? (int64_t)n * a.fC * f_HW : ((int64_t)n * a.fC + f_c0) * f_HW;
             unsigned char* dst = reinterpret_cast<unsigned char*>(a.y + first) + (int64_t)pc * kFoldZero;
             const int64_t left = blk_bytes - (int64_t)pc * kFoldZero;
             bulk_store(dst, zb, (uint32_t)(left < kFoldZero ? left : kFoldZero));
@@ -801,9 +803,9 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
               acc2 += (msk >> t) & 1u ? v2[t] : 0;
             }
             // channel cl of this input position: NCHW stride H W, NHWC stride 1
-            float* yo = a.fnhwc ? a.y + ((int64_t)n * HW + pos) * a.fC + c_first
+            float* yo = kNhwc ? a.y + ((int64_t)n * HW + pos) * a.fC + c_first
                                 : a.y + ((int64_t)n * a.fC + c_first) * HW + pos;
-            const int64_t cst = a.fnhwc ? 1 : HW;
+            const int64_t cst = kNhwc ? 1 : HW;
             yo[cl * cst] = __fadd_rn(__fmul_rn(sc, (float)acc), __fmul_rn(ze, (float)cf));
             if (cl2 != cl) yo[cl2 * cst] = __fadd_rn(__fmul_rn(sc, (float)acc2), __fmul_rn(ze, (float)cf2));
           }
@@ -843,7 +845,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
           }
         }
         const float v = __fadd_rn(__fmul_rn(s_scale[img], (float)acc), __fmul_rn(s_zero[img], (float)csf[rem]));
-        if (a.fnhwc)
+        if (kNhwc)
           a.y[((int64_t)n * HW + pos) * a.fC + c_first + cl] = v;
         else
           a.y[((int64_t)n * a.fC + c_first + cl) * HW + pos] = v;
@@ -1135,7 +1137,7 @@ static bool make_map(CUtensorMap* m, const void* ptr, CUtensorMapDataType type, 
             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <bool A_CODES, bool BITS8, int BN, bool SHORT = false>
+template <bool A_CODES, bool BITS8, int BN, bool SHORT = false, int X = 0>
 static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const TcArgs& a, int splits,
                              cudaStream_t s, const CUtensorMap* my = nullptr, const CUtensorMap* macc = nullptr,
                              bool cluster = false) {
@@ -1143,7 +1145,7 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
   using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT>,
+    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT, X>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes);
     if (e != cudaSuccess) return e;
     attr = true;
@@ -1151,10 +1153,10 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
   dim3 grid((unsigned)(a.grid_x > 0 ? a.grid_x : (a.N + BN - 1) / BN), (unsigned)((a.M + kBM - 1) / kBM),
             (unsigned)splits);
   if (cluster)
-    launch_k_cluster(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT>, dim3(grid), dim3(kThreads), S::kBytes, s,
+    launch_k_cluster(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT, X>, dim3(grid), dim3(kThreads), S::kBytes, s,
                      (unsigned)splits, ma, mb, my ? *my : unused, macc ? *macc : unused, a);
   else
-    launch_k(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT>, dim3(grid), dim3(kThreads), S::kBytes, s, ma, mb,
+    launch_k(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT, X>, dim3(grid), dim3(kThreads), S::kBytes, s, ma, mb,
              my ? *my : unused, macc ? *macc : unused, a);
   fqt1_count_launches(1);
   return cudaGetLastError();
@@ -1164,14 +1166,14 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
 // convolution fields (impl = 0 for a plain A = sign(X) rows map).
 static cudaError_t launch_fwd_common(const CUtensorMap& ma, TcArgs a, const uint32_t* B, int64_t M, int64_t D,
                                      int64_t K, const float* gamma, const float* bias, int32_t* acc, float* y,
-                                     int32_t* status, cudaStream_t s, const uint8_t* Be = nullptr, int64_t ldbe = 0) {
+                                     int32_t* status, cudaStream_t s, const uint8_t* Be = nullptr, int64_t ldbe = 0,
+                                     bool implicit = false) {
   using S = TcSmem<false, false, 128>;
   const int64_t ldw = fqt1_packed_words(K);
   CUtensorMap mb;
   if (Be) {  // e4m3 sign(W) rows [D][ldbe] bytes: 128 x 128 boxes, 128-byte swizzle
     if (!make_map(&mb, Be, CU_TENSOR_MAP_DATA_TYPE_UINT8, K, D, ldbe, kBK, 128, CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
-    a.b_tma = 1;
   } else if (!make_map(&mb, B, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, D, ldw * 4, 4 * S::KSUB, 128,
                        CU_TENSOR_MAP_SWIZZLE_NONE)) {
     return cudaErrorInvalidValue;
@@ -1191,6 +1193,8 @@ static cudaError_t launch_fwd_common(const CUtensorMap& ma, TcArgs a, const uint
         a.tma_out = 0;
     }
   }
+  if (implicit) return launch_tc<false, false, 128, false, 1>(ma, mb, a, 1, s, &my, &macc);
+  if (Be) return launch_tc<false, false, 128, false, 2>(ma, mb, a, 1, s, &my, &macc);
   return launch_tc<false, false, 128>(ma, mb, a, 1, s, &my, &macc);
 }
 
@@ -1254,8 +1258,9 @@ cudaError_t launch_fwd_implicit_tc(const uint32_t* xp, const uint32_t* wt, int N
          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
   TcArgs a{};
-  a.impl = 1; a.iC = C; a.ikw = k; a.ikhw = k * k; a.ipad = pad; a.iW = W; a.iHW = (int)HW; a.isb = isb;
-  return launch_fwd_common(ma, a, wt, (int64_t)N * HW, D, (int64_t)C * k * k, gamma, bias, acc, y, status, s);
+  a.iC = C; a.ikw = k; a.ikhw = k * k; a.ipad = pad; a.iW = W; a.iHW = (int)HW; a.isb = isb;
+  return launch_fwd_common(ma, a, wt, (int64_t)N * HW, D, (int64_t)C * k * k, gamma, bias, acc, y, status, s,
+                           nullptr, 0, true);
 }
 
 // Codes x signs: out[r, n] = sum_j Q[r, j] S[n, j], Q [rows][ld] uint8 (valid rows *count * rpc),
@@ -1297,8 +1302,6 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
     return cudaErrorInvalidValue;
   }
   TcArgs a{};
-  a.b_tma = Bte ? 1 : 0;
-  a.fnhwc = nhwc;
   const int khw = kh * kw, cb = 128 / khw;
   a.M = max_rows; a.N = K; a.L = D; a.count = count; a.rows_per_count = (int64_t)Ho * Wo;
   a.k_tiles = (int)((D + kCodesStageK - 1) / kCodesStageK); a.tiles_per_split = a.k_tiles;
@@ -1309,6 +1312,14 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
   a.fcb = cb; a.fN = N; a.slot_of_group = slot_of_group;
   a.fd_khw = FastDiv((uint32_t)khw); a.fd_w = FastDiv((uint32_t)W); a.fd_kw = FastDiv((uint32_t)kw);
   a.fd_hw = FastDiv((uint32_t)(H * W)); a.fd_s = FastDiv((uint32_t)stride); a.fd_cbhw = FastDiv((uint32_t)(cb * H * W));
+  if (Bte) {  // the e4m3 B path writes NCHW
+    if (bits == 8) return launch_tc<true, true, 128, true, 2>(ma, mb, a, 1, s);
+    return launch_tc<true, false, 128, true, 2>(ma, mb, a, 1, s);
+  }
+  if (nhwc) {
+    if (bits == 8) return launch_tc<true, true, 128, true, 4>(ma, mb, a, 1, s);
+    return launch_tc<true, false, 128, true, 4>(ma, mb, a, 1, s);
+  }
   if (bits == 8) return launch_tc<true, true, 128, true>(ma, mb, a, 1, s);
   return launch_tc<true, false, 128, true>(ma, mb, a, 1, s);
 }
