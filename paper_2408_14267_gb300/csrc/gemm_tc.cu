@@ -1312,7 +1312,8 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
   a.fcb = cb; a.fN = N; a.slot_of_group = slot_of_group;
   a.fd_khw = FastDiv((uint32_t)khw); a.fd_w = FastDiv((uint32_t)W); a.fd_kw = FastDiv((uint32_t)kw);
   a.fd_hw = FastDiv((uint32_t)(H * W)); a.fd_s = FastDiv((uint32_t)stride); a.fd_cbhw = FastDiv((uint32_t)(cb * H * W));
-  if (Bte) {  // the e4m3 B path writes NCHW
+  if (Bte) {  // the e4m3 B path writes NCHW only
+    if (nhwc) return cudaErrorNotSupported;
     if (bits == 8) return launch_tc<true, true, 128, true, 2>(ma, mb, a, 1, s);
     return launch_tc<true, false, 128, true, 2>(ma, mb, a, 1, s);
   }
