@@ -83,3 +83,22 @@ def test_rescale_of_a_kept_group_by_hand():
     s, z = om.group_scale(np.array([1.0], np.float32), np.array([-0.5], np.float32), np.array([0.375]), 2)
     assert s[0] == np.float32(8.0 / 9.0)
     assert z[0] == np.float32(-4.0 / 3.0)
+
+
+def test_bernoulli_masks_by_hand():
+    """The paper-literal mode draws m_i ~ Bern(p_i) independently: group i is kept iff its own
+    32-bit word is below P_i. R = [2, 0, 1] with b = 1 keeps all (plain PSQ); with P built for
+    b = 2 (n / b = 1.5): p = 1.5 R / 3 = [1, 0, 0.5] with no cap binding, so group 0 is always
+    kept, group 1 never, and group 2 iff its word is below 2^31."""
+    r = np.array([2, 0, 1], dtype=np.float32)
+    kept, p_hat, _ = om.select_groups(r, 1, om.BERNOULLI, 0, 2)
+    assert kept.tolist() == [0, 1, 2] and p_hat.tolist() == [1.0, 1.0, 1.0]
+    P, _ = om.agp_probabilities(r, 2, om.BERNOULLI)
+    assert P == [TWO32, 0, 1 << 31]
+    seen = set()
+    for seed in range(200):
+        w2 = int(uniform_u32(seed, 3, np.uint64(2)))
+        kept, _, _ = om.select_groups(r, 2, om.BERNOULLI, seed, 3)
+        assert kept.tolist() == ([0, 2] if w2 < 1 << 31 else [0]), seed
+        seen.add(len(kept))
+    assert seen == {1, 2}
