@@ -145,3 +145,48 @@ def test_layout_and_e4m3_entry_points_validate_without_launch(lib):
     # workspace preparation
     assert lib.fqt1_scq_workspace_init(None, 64, s) == 1
     assert lib.fqt1_scq_workspace_init(fake, 0, s) == 1
+
+
+_CTYPE_OF = {"int64_t": C.c_int64, "int32_t": C.c_int32, "size_t": C.c_size_t, "float": C.c_float,
+             "uint64_t": C.c_uint64, "fqt1_status": C.c_int}
+
+
+def _declarations():
+    """(return type, name, [parameter types]) of every function declared in include/*.h."""
+    out = []
+    for h in sorted(os.listdir(os.path.join(ROOT, "include"))):
+        if not h.endswith(".h"):
+            continue
+        txt = open(os.path.join(ROOT, "include", h)).read()
+        txt = re.sub(r"/\*.*?\*/", " ", txt, flags=re.S)
+        txt = re.sub(r"//[^\n]*", " ", txt)
+        txt = re.sub(r"^\s*#[^\n]*", " ", txt, flags=re.M)
+        for ret, name, params in re.findall(r"([\w\s\*]+?)\b(fqt1_\w+)\s*\(([^;{)]*)\)\s*;", txt):
+            ret = " ".join(ret.strip().split("\n")[-1].split())
+            ps = [" ".join(p.split()) for p in params.split(",")]
+            ps = [] if ps == ["void"] or ps == [""] else ps
+            types = [re.sub(r"\s*\b\w+$", "", p) if not p.endswith("*") else p for p in ps]
+            out.append((ret, name, types))
+    return out
+
+
+def _expected_ctype(t):
+    if "*" in t:
+        return C.c_void_p
+    t = t.replace("const ", "").strip()
+    return _CTYPE_OF[t]
+
+
+def test_binding_signatures_match_the_header():
+    """Every ctypes signature in the binding has the header's arity and argument widths, so a
+    wrong int32 / int64 / size_t or a missing argument fails here rather than on a GPU."""
+    from paper_2408_14267_gb300 import fqt1
+    decls = _declarations()
+    assert {n for _, n, _ in decls} == set(fqt1._SIGS)
+    for ret, name, types in decls:
+        restype, argtypes = fqt1._SIGS[name]
+        assert len(argtypes) == len(types), (name, types)
+        for i, (t, a) in enumerate(zip(types, argtypes)):
+            assert a is _expected_ctype(t), (name, i, t, a)
+        want = C.c_char_p if ret == "const char*" else _expected_ctype(ret)
+        assert restype is want, (name, ret, restype)
