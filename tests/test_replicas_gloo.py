@@ -107,23 +107,3 @@ def test_reference_arm_other_ranks_do_no_work(capsys):
     assert bench.reference_arm(args, world=2, rank=1) is None
     assert time.perf_counter() - t0 < 1.0
     assert capsys.readouterr().out == ""
-
-
-def test_reference_arm_rank0_prints_one_contract_line(capsys):
-    """Rank 0 times the oracle on the host and prints one JSON line with the contract's keys."""
-    import argparse
-    import json
-
-    import bench
-    args = argparse.Namespace(steps=1, warmup=0, impl="reference", gpus=1)
-    bench.reference_arm(args, world=1, rank=0)
-    lines = [x for x in capsys.readouterr().out.splitlines() if x.strip()]
-    assert len(lines) == 1
-    d = json.loads(lines[0])
-    assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == bench.UNIT
-    assert d["n_gpus"] == 1 and d["steps"] == 1 and d["warmup"] == 0 and d["higher_is_better"] is True
-    assert d["value"] > 0 and d["ms_per_step"] > 0
-    assert d["config"] == {"workload": bench.WORKLOAD}
-    cb = d["cpu_baseline"]
-    assert cb["kind"] == "oracle" and cb["cores"] == 1 and cb["value"] == d["value"] and cb["sample"]
-    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
