@@ -1,4 +1,6 @@
-"""Host logic of bench.py that needs no GPU: the reference arm's JSON line and the clock record."""
+"""Host logic of bench.py that needs no GPU: the reference arm's JSON line, the clock record and
+the validity of stored DRAM-traffic figures."""
+import os
 
 
 def test_reference_arm_rank0_prints_one_contract_line(capsys):
@@ -43,3 +45,28 @@ def test_clock_record_summary_from_a_fake_nvidia_smi_log(tmp_path, monkeypatch):
     cs2 = bench.ClockSampler(3)
     cs2.proc = object()
     assert cs2.summary()["reasons"] == ["hw_thermal_slowdown"]
+
+
+def test_stage_traffic_is_null_once_its_kernel_sources_change(tmp_path, monkeypatch):
+    """A stored DRAM-traffic figure stands only for the kernel sources it was captured on."""
+    import shutil
+
+    import bench
+    csrc = tmp_path / "paper_2408_14267_gb300" / "csrc"
+    shutil.copytree(os.path.join(bench.ROOT, "paper_2408_14267_gb300", "csrc"), csrc,
+                    ignore=shutil.ignore_patterns("*.o", "_build"))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    sha = bench.sources_sha("scq")
+    monkeypatch.setitem(bench.TRAFFIC_SOURCES, "scq", sha)
+    assert bench.stage_traffic("scq_quantize") == bench.TRAFFIC_BYTES["scq_quantize"]
+    assert bench.stage_traffic("no_such_stage") is None
+    # one byte more in a file of the group: a new hash, and no traffic figure
+    with open(csrc / "quantize.cu", "ab") as f:
+        f.write(b"\n")
+    assert bench.sources_sha("scq") != sha
+    assert bench.stage_traffic("scq_quantize") is None
+    # files outside the group do not matter
+    monkeypatch.setitem(bench.TRAFFIC_SOURCES, "scq", bench.sources_sha("scq"))
+    with open(csrc / "gemm_tc.cu", "ab") as f:
+        f.write(b"\n")
+    assert bench.stage_traffic("scq_quantize") == bench.TRAFFIC_BYTES["scq_quantize"]
