@@ -71,18 +71,28 @@ from paper_2408_14267_gb300 import workloads as wl
 from oracle import method as om
 w = wl.resnet18_cifar_conv()
 batch, steps = int(sys.argv[2]), int(sys.argv[3])
+first = int(sys.argv[4]) if len(sys.argv) > 4 else 0
 N, C, H, W = w["x"].shape
 Ho = Wo = H
-x = w["x"][:batch]
-gy = w["gy"][: batch * Ho * Wo]
-times = []
-for _ in range(steps):
-    t0 = time.perf_counter()
+x = w["x"][first:first + batch]
+gy = w["gy"][first * Ho * Wo:(first + batch) * Ho * Wo]
+def step():
     om.layer_step_conv(x, w["w"], w["gamma"], gy, w["stride"], w["pad"], w["bits_s"], w["mode_s"], w["seed_s"],
                        w["bits_c"], w["mode_c"], w["seed_c"])
+if len(sys.argv) > 5:  # one untimed step, then start together with the other processes
+    step()
+    print("ready", flush=True)
+    sys.stdin.readline()
+times = []
+t_start = time.time()
+for _ in range(steps):
+    t0 = time.perf_counter()
+    step()
     times.append(time.perf_counter() - t0)
+t_end = time.time()
 M, K, D = batch * Ho * Wo, C * 9, w["w"].shape[0]
-print(json.dumps({"times": times, "ops": 6.0 * M * K * D, "M": M, "K": K, "D": D}))
+print(json.dumps({"times": times, "ops": 6.0 * M * K * D, "M": M, "K": K, "D": D, "t_start": t_start,
+                  "t_end": t_end}))
 """
 
 
@@ -95,6 +105,52 @@ def run_oracle_sample(batch, steps):
     if p.returncode != 0:
         raise RuntimeError("oracle sample failed: " + p.stderr[-2000:])
     return json.loads(p.stdout.strip().splitlines()[-1])
+
+
+def host_cores():
+    """Cores this process may run on: its CPU affinity, capped by a cgroup v2 CPU quota."""
+    n = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+    try:
+        with open("/sys/fs/cgroup/cpu.max") as f:
+            quota, period = f.read().split()[:2]
+        if quota != "max":
+            n = min(n, max(1, int(quota) // int(period)))
+    except (OSError, ValueError):
+        pass
+    return n
+
+
+def run_oracle_parallel(batch, procs, steps=1):
+    """The oracle on `procs` host cores at once: one single-threaded process per core, each on
+    its own slice of `batch` samples, all started together once every process has drawn its
+    inputs.  Throughput = all processes' operations / (last end - first start)."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               NUMEXPR_NUM_THREADS="1")
+    ps = [subprocess.Popen([sys.executable, "-c", CPU_SAMPLE_SCRIPT, ROOT, str(batch), str(steps),
+                            str((i * batch) % 128), "together"], env=env, stdin=subprocess.PIPE,
+                           stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True) for i in range(procs)]
+    try:
+        for p in ps:
+            if p.stdout.readline().strip() != "ready":
+                raise RuntimeError("oracle process failed: " + p.stderr.read()[-2000:])
+        for p in ps:
+            p.stdin.write("go\n")
+            p.stdin.flush()
+        outs = [p.communicate(timeout=1800) for p in ps]
+    finally:
+        for p in ps:
+            if p.poll() is None:
+                p.kill()
+                p.wait()
+    rs = []
+    for p, (out, err) in zip(ps, outs):
+        if p.returncode != 0:
+            raise RuntimeError("oracle process failed: " + err[-2000:])
+        rs.append(json.loads(out.strip().splitlines()[-1]))
+    wall = max(r["t_end"] for r in rs) - min(r["t_start"] for r in rs)
+    ops = sum(r["ops"] * len(r["times"]) for r in rs)
+    return {"value": ops / wall / 1e12, "cores": procs, "wall_s": wall, "M": rs[0]["M"], "K": rs[0]["K"],
+            "D": rs[0]["D"]}
 
 
 def load_peaks():
@@ -381,11 +437,19 @@ def main():
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        r = run_oracle_sample(batch=32, steps=2)
-        t = statistics.mean(r["times"])
+        r = run_oracle_sample(batch=32, steps=3)
+        t = statistics.mean(r["times"][1:])  # the first step runs cold (page faults, caches)
         cpu = {"value": r["ops"] / t / 1e12, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": f"oracle layer step on 32 of the 128 samples (M={r['M']} K={r['K']} D={r['D']}), "
-                         f"mean of 2 runs, {t:.2f} s each, one thread"}
+                         f"mean of 2 runs after one untimed run, {t:.2f} s each, one thread"}
+        ncores = min(host_cores(), 16)
+        if ncores > 1:
+            ra = run_oracle_parallel(batch=32, procs=ncores)
+            cpu["all_cores"] = {"value": ra["value"], "unit": UNIT, "cores": ncores, "kind": "oracle",
+                                "sample": f"{ncores} single-threaded oracle processes started together after one "
+                                          f"untimed step each, each one layer step on its own 32 of the 128 "
+                                          f"samples (M={ra['M']} K={ra['K']} D={ra['D']}), {ra['wall_s']:.2f} s "
+                                          f"first start to last end"}
 
     if world > 1:
         dist.barrier()

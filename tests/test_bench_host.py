@@ -70,3 +70,12 @@ def test_stage_traffic_is_null_once_its_kernel_sources_change(tmp_path, monkeypa
     with open(csrc / "gemm_tc.cu", "ab") as f:
         f.write(b"\n")
     assert bench.stage_traffic("scq_quantize") == bench.TRAFFIC_BYTES["scq_quantize"]
+
+
+def test_all_cores_oracle_timing():
+    """The all-cores CPU baseline: one single-threaded oracle process per core, started together."""
+    import bench
+    assert bench.host_cores() >= 1
+    r = bench.run_oracle_parallel(batch=4, procs=2)
+    assert r["cores"] == 2 and r["value"] > 0 and r["wall_s"] > 0
+    assert (r["M"], r["K"], r["D"]) == (4 * 64, 2304, 256)
