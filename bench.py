@@ -276,6 +276,8 @@ def main():
                     help="GEMM-only comparison of average 1-bit and 1-bit products on the Table 5 shapes")
     ap.add_argument("--model", choices=["vgg16", "resnet18"],
                     help="training step of a synthetic model built from binop layers against FP32 PyTorch")
+    ap.add_argument("--layers", choices=["vgg16", "resnet18", "all"],
+                    help="the layer step on every VGG-16 / ResNet-18 layer shape")
     ap.add_argument("--variance", action="store_true",
                     help="empirical variance of the AGP quantizer (b = 2, 4, 8) and of 1-bit PSQ against Eq. 24")
     ap.add_argument("--res", type=int, default=32, help="input resolution of --model")
@@ -293,6 +295,8 @@ def main():
         return model_step(args)
     if args.variance:
         return variance_study(args)
+    if args.layers:
+        return layer_sweep(args)
 
     import torch
     import torch.distributed as dist
@@ -542,6 +546,61 @@ def table5(args):
                                  "l2": "flushed before every timed launch (256 MiB write)",
                                  "timing": "one graph-captured launch, CUDA events, median"},
                       "shapes": rows}))
+
+
+def layer_sweep(args):
+    """The layer step on every VGG-16 (32x32, batch 128) and ResNet-18 (224x224, batch 64) layer
+    shape, b = 4 on both SCQ branches: per layer the three-branch step (LayerStep.step_concurrent)
+    as one CUDA graph, the L2 flushed before every replay, CUDA events on the launching stream,
+    median over `steps` replays.  Reports 6 M K D / time per layer, the fp32 bytes the step reads
+    and writes (x, W, gY in; y, dx, dW out) over the same time, and the whole set's 6 M K D sum
+    over the sum of the layer times."""
+    import torch
+    from paper_2408_14267_gb300 import build, workloads
+    build.build()
+    from paper_2408_14267_gb300.layer import LayerStep
+    dev = torch.device("cuda")
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)  # 256 MiB > 129 MB L2
+    stream = torch.cuda.Stream()
+    sets = {"vgg16": lambda: workloads.vgg16_layers(bits=4), "resnet18": workloads.resnet18_imagenet_layers}
+    rows = []
+    for net in (["vgg16", "resnet18"] if args.layers == "all" else [args.layers]):
+        for wl in sets[net]():
+            st = LayerStep(wl, device=dev, keep_acc=False)
+            with torch.cuda.stream(stream):
+                for _ in range(3):
+                    st.step()
+                stream.synchronize()
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    st.step_concurrent(stream)
+                for _ in range(max(args.warmup, 3)):
+                    g.replay()
+                ts = []
+                for _ in range(args.steps):
+                    flush.zero_()
+                    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    e0.record(stream)
+                    g.replay()
+                    e1.record(stream)
+                    ts.append((e0, e1))
+                stream.synchronize()
+            ms = statistics.median(a.elapsed_time(b) for a, b in ts)
+            io = 4 * sum(t.numel() for t in (st.x, st.w, st.gy, st.y, st.dx, st.dw))
+            rows.append({"layer": wl["name"], "M": st.M, "K": st.K, "D": st.D, "ms": round(ms, 5),
+                         "tops": round(st.dense_ops() / (ms * 1e-3) / 1e12, 2),
+                         "fp32_io_gbs": round(io / (ms * 1e-3) / 1e9, 1)})
+            del g, st
+            torch.cuda.empty_cache()
+    total_ms = sum(r["ms"] for r in rows)
+    total_ops = sum(6.0 * r["M"] * r["K"] * r["D"] for r in rows)
+    print(json.dumps({"metric": "effective TOPS of the 1-bit FQT layer step over VGG-16 / ResNet-18 layer shapes",
+                      "value": total_ops / (total_ms * 1e-3) / 1e12, "unit": "TOPS", "higher_is_better": True,
+                      "steps": args.steps, "warmup": args.warmup, "dtype": "e4m3", "data": "synthetic",
+                      "config": {"workload": f"{args.layers} layer shapes, b = 4, keep 1/4, SCQ",
+                                 "l2": "flushed before every timed replay (256 MiB write)",
+                                 "timing": "one CUDA graph of the three-branch step per layer, CUDA events, median"},
+                      "layers": rows}))
 
 
 def build_model(name, res, binary, classes=10):
