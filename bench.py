@@ -31,8 +31,8 @@ FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS = 6800.0, 1900.0
 SMS, POPC_PER_CLK_SM = 152, 16
 
 # DRAM bytes (read + write) per launch of each stage's kernels, from one ncu capture of
-# `bench.py --profile 2 --warmup 1` (profiles/kernels_resnet18_cifar_conv_full.md; the SCQ
-# stage is the sum of its range, selection and quantize kernels).  A figure is valid only for
+# `bench.py --profile 2 --warmup 1` (the SCQ stage is the sum of its range, selection and
+# quantize kernels).  A figure is valid only for
 # the kernel sources it was taken on: TRAFFIC_SOURCES holds, per stage, the sha256 prefix of the
 # files that define that stage's kernels (STAGE_SOURCES) at the capture; a stage whose sources
 # have changed since reports traffic = null.

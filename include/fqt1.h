@@ -188,7 +188,8 @@ fqt1_status fqt1_bwd_input_fold_nhwc(const fqt1_qgrad* psq, const uint32_t* sw_c
 /* Binarized forward GEMM (Sec. 5.1, App. C "binary multiplication"):
  * acc[m, j] = sum_k sign(X)[m, k] sign(W)[j, k], y[m, j] = gamma[j] * acc[m, j] (fp32).
  * sx_row: [M][words(K)], sw_row: [D][words(K)], gamma: [D].
- * acc: [M][D] int32 or NULL; y: [M][D] fp32 (row stride D). */
+ * acc: [M][D] int32 or NULL; y: [M][D] fp32 (row stride D) or NULL, at least one of
+ * the two given (gamma may be NULL when y is). */
 fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D, int64_t K,
                           const float* gamma, int32_t* acc, float* y, void* stream);
 
@@ -294,13 +295,13 @@ fqt1_status fqt1_scq_quantize(const float* g, int64_t M, int64_t D, const float*
  *    FQT1_NOALLOC_SCRATCH_KEYS; larger calls return FQT1_ERR_UNSUPPORTED and
  *    fqt1_last_cuda_error() names the limit.
  *  - The first call on a device (the device current on the calling thread,
- *    which must own `stream`) looks up the array's device address; make that
- *    first call before any stream capture.
- *  - The array is filled with 0xFF by the first call on the device that is not
- *    captured into a graph (until then by each captured call, as a node of its
- *    graph); every call leaves the part it used at 0xFF, as a workspace after
- *    fqt1_scq_workspace_init.  Calls whose work overlaps on the GPU (concurrent
- *    streams) race on it.
+ *    which must own `stream`) looks up the array's device address and fills
+ *    the array with 0xFF on `stream`; make that first call before any stream
+ *    capture.  Every call that returns FQT1_OK leaves the part it used at
+ *    0xFF, as a workspace after fqt1_scq_workspace_init.  A call that returns
+ *    an error may leave keys behind, so the next call on that device fills the
+ *    array again (one extra fill).  Calls whose work overlaps on the GPU
+ *    (concurrent streams) race on the array.
  *  - Allocates nothing: no cudaMalloc / cudaFree or allocating library call.
  * All other arguments, results and errors are those of fqt1_scq_quantize. */
 #define FQT1_NOALLOC_SCRATCH_KEYS 16384

@@ -34,15 +34,6 @@ extern "C" int64_t fqt1_codes_ld(int64_t n) { return n < 1 ? 0 : ((n + 15) / 16)
 
 namespace fqt1 {
 
-bool use_popcount_path() {
-  static int v = -1;
-  if (v < 0) {
-    const char* e = getenv("FQT1_GEMM_PATH");
-    v = (e && strcmp(e, "popcount") == 0) ? 1 : 0;
-  }
-  return v == 1;
-}
-
 // Rows of pruned groups of an [M][K] fp32 output are exactly zero.  Grid: x covers a row in
 // chunks of 1024 floats, y (and z for more than 65535 rows) the rows.
 __global__ void zero_pruned_rows_kernel(const int32_t* __restrict__ slot_of_group, int64_t M, int64_t K, int64_t rpg,
@@ -261,11 +252,7 @@ extern "C" fqt1_status fqt1_fwd_gemm_bias(const uint32_t* sx_row, const uint32_t
       (gamma && !aligned16(gamma)) || (bias && !aligned16(bias)))
     return FQT1_ERR_MISALIGNED;
   if (K >= (1ll << 24) || (M + 63) / 64 > 65535) return FQT1_ERR_UNSUPPORTED;
-  if (use_popcount_path() || !y) {
-    FQT1_CUDA_TRY(launch_xnor_gemm_simt(sx_row, sw_row, M, D, K, gamma, bias, acc, y, (cudaStream_t)stream));
-  } else {
-    FQT1_CUDA_TRY(launch_fwd_tc(sx_row, sw_row, M, D, K, gamma, bias, acc, y, nullptr, (cudaStream_t)stream));
-  }
+  FQT1_CUDA_TRY(launch_fwd_tc(sx_row, sw_row, M, D, K, gamma, bias, acc, y, nullptr, (cudaStream_t)stream));
   return FQT1_OK;
 }
 
@@ -277,7 +264,7 @@ extern "C" fqt1_status fqt1_fwd_gemm_e4m3w(const uint32_t* sx_row, const uint8_t
   if (!aligned16(sx_row) || !aligned16(w_e4m3) || (acc && !aligned16(acc)) || !aligned16(y) || !aligned16(gamma) ||
       (bias && !aligned16(bias)))
     return FQT1_ERR_MISALIGNED;
-  if (K >= (1ll << 24) || (M + 63) / 64 > 65535 || use_popcount_path()) return FQT1_ERR_UNSUPPORTED;
+  if (K >= (1ll << 24) || (M + 63) / 64 > 65535) return FQT1_ERR_UNSUPPORTED;
   FQT1_CUDA_TRY(launch_fwd_e4m3w_tc(sx_row, w_e4m3, ld_w, M, D, K, gamma, bias, acc, y, nullptr, (cudaStream_t)stream));
   return FQT1_OK;
 }
@@ -302,7 +289,7 @@ extern "C" fqt1_status fqt1_conv_fwd_implicit(const uint32_t* x_pix, const uint3
   if (!aligned16(x_pix) || !aligned16(w_taps) || !aligned16(gamma) || !aligned16(y) || (acc && !aligned16(acc)) ||
       (bias && !aligned16(bias)))
     return FQT1_ERR_MISALIGNED;
-  if (use_popcount_path() || !implicit_conv_supported(N, C, H, W, kh, kw, stride, pad)) return FQT1_ERR_UNSUPPORTED;
+  if (!implicit_conv_supported(N, C, H, W, kh, kw, stride, pad)) return FQT1_ERR_UNSUPPORTED;
   FQT1_CUDA_TRY(launch_fwd_implicit_tc(x_pix, w_taps, N, C, H, W, kh, pad, D, gamma, bias, acc, y, nullptr,
                                        (cudaStream_t)stream));
   return FQT1_OK;
@@ -323,7 +310,7 @@ extern "C" fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t
   const int64_t cap_rows = fqt1_kept_capacity(M / rpg, p->bits, p->mode) * rpg;
   if ((cap_rows + 63) / 64 > 65535) return FQT1_ERR_UNSUPPORTED;
   cudaStream_t s = (cudaStream_t)stream;
-  if (!use_popcount_path() && !acc) {
+  if (!acc) {
     // dequantization fused into the tensor-core epilogue; pruned rows written as zeros
     FQT1_CUDA_TRY(launch_codes_tc_simple(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, rpg, sw_col,
                                          K, D, GEMM_EPI_DX, 1, nullptr, dx, K, psq->kept_idx, psq->scale,
@@ -332,14 +319,9 @@ extern "C" fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t
     FQT1_CUDA_TRY(cudaGetLastError());
     return FQT1_OK;
   }
-  if (use_popcount_path()) {
-    FQT1_CUDA_TRY(launch_codes_gemm_simt(p->bits, psq->codes, psq->ld_codes, psq->kept_count, rpg, cap_rows, sw_col,
-                                         K, D, acc, K, s));
-  } else {
-    FQT1_CUDA_TRY(launch_codes_tc_simple(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, rpg, sw_col,
-                                         K, D, GEMM_EPI_ACC32, 1, acc, nullptr, K, nullptr, nullptr, nullptr,
-                                         nullptr, rpg, nullptr, s));
-  }
+  FQT1_CUDA_TRY(launch_codes_tc_simple(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, rpg, sw_col,
+                                       K, D, GEMM_EPI_ACC32, 1, acc, nullptr, K, nullptr, nullptr, nullptr,
+                                       nullptr, rpg, nullptr, s));
   if (dx) {
     const int64_t n = M * K;
     launch_k(dequant_rows_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, acc, K, psq->slot_of_group, psq->scale,
@@ -379,12 +361,8 @@ static fqt1_status col2im_impl(const int32_t* acc, const fqt1_qgrad* psq, const 
     if (cb) break;
   }
   if (cb > 0) {
-    static bool attr = false;
-    if (!attr) {
-      FQT1_CUDA_TRY(cudaFuncSetAttribute(col2im_tiled_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kMaxTile));
-      attr = true;
-    }
+    static std::atomic<uint64_t> attr{0};
+    FQT1_CUDA_TRY(smem_attr_once((const void*)col2im_tiled_kernel, (int)kMaxTile, attr));
     FoldArgs fa;
     fa.acc = acc; fa.kept_idx = psq->kept_idx; fa.kept_count = psq->kept_count; fa.scale = psq->scale;
     fa.zero = psq->zero;
@@ -494,10 +472,7 @@ extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_
   if (!aligned16(sx_col) || !aligned16(acc) || !aligned16(dw) || !aligned16(colsum_x)) return FQT1_ERR_MISALIGNED;
   const int64_t cap = fqt1_kept_capacity(D, p->bits, p->mode);
   cudaStream_t s = (cudaStream_t)stream;
-  if (use_popcount_path()) {
-    FQT1_CUDA_TRY(launch_codes_gemm_simt(p->bits, pcq->codes, pcq->ld_codes, pcq->kept_count, 1, cap, sx_col, K, M,
-                                         acc, K, s));
-  } else {
+  {
     // split the long contraction over M across a cluster of CTAs that reduce their int32
     // partial tiles in shared memory and dequantize in the same kernel; each CTA's fp32 partial
     // sum stays below 2^24 and no split is empty (every CTA of a cluster takes part)

@@ -4,12 +4,6 @@
 
 namespace fqt1 {
 
-cudaError_t launch_xnor_gemm_simt(const uint32_t* A, const uint32_t* B, int64_t M, int64_t N, int64_t K,
-                                  const float* gamma, const float* bias, int32_t* acc, float* y, cudaStream_t s);
-cudaError_t launch_codes_gemm_simt(int bits, const uint8_t* Q, int64_t ldq, const int32_t* count,
-                                   int64_t rows_per_count, int64_t max_rows, const uint32_t* S, int64_t n_s,
-                                   int64_t L, int32_t* out, int64_t ldo, cudaStream_t s);
-
 // tcgen05 path (gemm_tc.cu)
 struct TcArgs;
 cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64_t D, int64_t K, const float* gamma,
@@ -62,7 +56,5 @@ int wgrad_cluster_size(int bits, int64_t out_tiles, int64_t k_tiles);
 constexpr int kCodesStageK = 256;
 // Largest contraction one CTA may sum in fp32 and stay exact: partial sums below 2^24.
 inline int64_t exact_chunk(int bits) { return (int64_t)((1 << 24) / ((1 << bits) - 1)); }
-// 1 if FQT1_GEMM_PATH=popcount selects the CUDA-core kernels (datapath comparison only).
-bool use_popcount_path();
 
 }  // namespace fqt1

@@ -940,7 +940,15 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
           sc = __ldg(a.scale + slot);
           ze = __ldg(a.zero + slot);
         }
-        if (a.epi == EPI_FWD) {
+        if (a.epi == EPI_FWD && !a.y) {  // the integer accumulators alone
+          int32_t* orow = a.acc + out_row * a.ldo + nb;
+          if (full) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) *reinterpret_cast<int4*>(orow + j) = make_int4(iv[j], iv[j + 1], iv[j + 2], iv[j + 3]);
+          } else {
+            for (int j = 0; j < 32 && nb + j < a.N; ++j) orow[j] = iv[j];
+          }
+        } else if (a.epi == EPI_FWD) {
           float* yrow = a.y + out_row * a.ldo + nb;
           if (full) {
 #pragma unroll
@@ -1143,13 +1151,9 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
                              bool cluster = false) {
   static const CUtensorMap unused{};  // never read: the matching tma_out bit is clear
   using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT, X>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  static std::atomic<uint64_t> attr{0};
+  const cudaError_t ea = smem_attr_once((const void*)tc_gemm_kernel<A_CODES, BITS8, BN, SHORT, X>, S::kBytes, attr);
+  if (ea != cudaSuccess) return ea;
   dim3 grid((unsigned)(a.grid_x > 0 ? a.grid_x : (a.N + BN - 1) / BN), (unsigned)((a.M + kBM - 1) / kBM),
             (unsigned)splits);
   if (cluster)
@@ -1181,17 +1185,15 @@ static cudaError_t launch_fwd_common(const CUtensorMap& ma, TcArgs a, const uint
   a.M = M; a.N = D; a.L = K; a.count = nullptr; a.rows_per_count = 1;
   a.k_tiles = (int)((K + kBK * S::KSUB - 1) / (kBK * S::KSUB)); a.tiles_per_split = a.k_tiles;
   a.epi = EPI_FWD; a.gamma = gamma; a.bias = bias; a.y = y; a.acc = acc; a.ldo = D; a.status = status;
-  // outputs leave through TMA stores when their rows are 16-byte multiples
+  // outputs leave through TMA stores when their rows are 16-byte multiples (y may be null: the
+  // integer accumulators alone)
   CUtensorMap my{}, macc{};
-  if (D % 4 == 0 && make_map(&my, y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, D, M, D * 4, 32, 32,
-                             CU_TENSOR_MAP_SWIZZLE_128B)) {
-    a.tma_out = 1;
-    if (acc) {
-      if (make_map(&macc, acc, CU_TENSOR_MAP_DATA_TYPE_INT32, D, M, D * 4, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B))
-        a.tma_out |= 2;
-      else
-        a.tma_out = 0;
-    }
+  if (D % 4 == 0) {
+    bool ok = true;
+    if (y) ok = make_map(&my, y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, D, M, D * 4, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (ok && acc)
+      ok = make_map(&macc, acc, CU_TENSOR_MAP_DATA_TYPE_INT32, D, M, D * 4, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (ok) a.tma_out = (y ? 1 : 0) | (acc ? 2 : 0);
   }
   if (implicit) return launch_tc<false, false, 128, false, 1>(ma, mb, a, 1, s, &my, &macc);
   if (Be) return launch_tc<false, false, 128, false, 2>(ma, mb, a, 1, s, &my, &macc);
@@ -1329,11 +1331,15 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
 template <bool BITS8>
 static int max_active_clusters(int cs) {
   using S = TcSmem<true, BITS8, 128>;
-  static int cache[9] = {-1, -1, -1, -1, -1, -1, -1, -1, -1};
-  if (cs < 1 || cs > 8) return 0;
-  if (cache[cs] >= 0) return cache[cs];
+  // per device ordinal and cluster size: the number of clusters + 1 (0 = not yet known)
+  static std::atomic<int> cache[64][9];
+  static std::atomic<uint64_t> attr_bits{0};
+  int dev = 0;
+  if (cs < 1 || cs > 8 || cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  const int known = cache[dev][cs].load(std::memory_order_acquire);
+  if (known > 0) return known - 1;
   auto kern = tc_gemm_kernel<true, BITS8, 128, false>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes) != cudaSuccess) return 0;
+  if (smem_attr_once((const void*)kern, S::kBytes, attr_bits) != cudaSuccess) return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(1, 1, (unsigned)cs);
   cfg.blockDim = dim3(kThreads);
@@ -1350,7 +1356,7 @@ static int max_active_clusters(int cs) {
     cudaGetLastError();
     n = 0;
   }
-  cache[cs] = n;
+  cache[dev][cs].store(n + 1, std::memory_order_release);
   return n;
 }
 

@@ -964,12 +964,8 @@ static fqt1_status im2col_impl(const float* x, const uint32_t* planes, int32_t N
       u.div_hwo = FastDiv((uint32_t)(Ho * Wo)); u.div_wo = FastDiv((uint32_t)Wo);
       const int64_t row_tiles = (Mi + tm - 1) / tm, word_tiles = (u.row_words + 7) / 8;
       if (row_tiles > 65535) break;
-      static bool attr = false;
-      if (!attr) {
-        FQT1_CUDA_TRY(cudaFuncSetAttribute(unfold_bits_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           kUnfoldMaxStreamWords * 4));
-        attr = true;
-      }
+      static std::atomic<uint64_t> attr{0};
+      FQT1_CUDA_TRY(smem_attr_once((const void*)unfold_bits_kernel, kUnfoldMaxStreamWords * 4, attr));
       if (colsum) FQT1_CUDA_TRY(cudaMemsetAsync(colsum, 0, sizeof(int32_t) * Ki, s));
       launch_k(unfold_bits_kernel, dim3((unsigned)word_tiles, (unsigned)row_tiles), dim3(256), (size_t)words * 4, s, u);
       fqt1_count_launches(1);

@@ -742,14 +742,9 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
   if (psq) add_sel(ps, psq, smin, smax, (int)ns, kStreamSelSample);
   if (pcq) add_sel(pc, pcq, cmin, cmax, (int)D, kStreamSelChannel);
   const size_t smem = (size_t)npad_max * 8 + (size_t)npad_max * 4;
-  static bool attr_done = false;
-  if (!attr_done) {
-    FQT1_CUDA_TRY(cudaFuncSetAttribute(select_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (size_t)kMaxGroups * 12));
-    FQT1_CUDA_TRY(cudaFuncSetAttribute(select_kernel<kSelThreads>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (size_t)kMaxGroups * 12));
-    attr_done = true;
-  }
+  static std::atomic<uint64_t> attr_small{0}, attr_large{0};
+  FQT1_CUDA_TRY(smem_attr_once((const void*)select_kernel<256>, kMaxGroups * 12, attr_small));
+  FQT1_CUDA_TRY(smem_attr_once((const void*)select_kernel<kSelThreads>, kMaxGroups * 12, attr_large));
   if (npad_max <= 256)  // fewer warps per barrier when every grouping has at most 256 groups
     launch_k(select_kernel<256>, dim3(nsel), dim3(256), smem, s, sa[0], nsel > 1 ? sa[1] : sa[0]);
   else
@@ -811,11 +806,11 @@ extern "C" fqt1_status fqt1_scq_quantize(const float* g, int64_t M, int64_t D, c
 // the step path.  For them the scratch of the range pass (the ordered min / max
 // keys of every sample group and channel) lives in a fixed array compiled into
 // this library instead of a caller buffer.  The array is shared by every call on
-// a device; it is filled with 0xFF once (by the first call on the device that is
-// not being captured into a graph, or by each captured call until then) and every
-// call leaves it so, like a workspace after fqt1_scq_workspace_init.  Only calls
-// that overlap on the GPU (e.g. on two streams at once) interfere, and such calls
-// race.
+// a device; the first call on the device fills it with 0xFF and every call that
+// succeeds leaves it so, like a workspace after fqt1_scq_workspace_init.  A call
+// that fails may leave keys behind, so it marks the array for a refill by the next
+// call.  Only calls that overlap on the GPU (e.g. on two streams at once)
+// interfere, and such calls race.
 static __device__ __align__(256) uint32_t g_scq_scratch[FQT1_NOALLOC_SCRATCH_KEYS];
 
 static std::mutex g_scq_scratch_mu;
@@ -824,10 +819,11 @@ static bool g_scq_scratch_ready[64];  // filled with 0xFF outside a graph captur
 
 // Device address of the scratch array on the calling thread's current device, filled with
 // 0xFF on stream s until a fill has run outside a graph capture.  The first call on a device
-// looks the address up (cudaGetSymbolAddress) and caches it.
-static fqt1_status scq_scratch_address(void** out, cudaStream_t s) {
+// looks the address up (cudaGetSymbolAddress) and caches it.  *dev_out is the device ordinal.
+static fqt1_status scq_scratch_address(void** out, int* dev_out, cudaStream_t s) {
   int dev = -1;
   FQT1_CUDA_TRY(cudaGetDevice(&dev));
+  *dev_out = dev;
   if (dev < 0 || dev >= 64) return FQT1_ERR_UNSUPPORTED;
   std::lock_guard<std::mutex> lock(g_scq_scratch_mu);
   if (!g_scq_scratch_dev[dev]) {
@@ -861,8 +857,17 @@ extern "C" fqt1_status fqt1_scq_quantize_noalloc(const float* g, int64_t M, int6
     return FQT1_ERR_UNSUPPORTED;
   }
   void* scratch = nullptr;
-  const fqt1_status st = scq_scratch_address(&scratch, (cudaStream_t)stream);
+  int dev = -1;
+  const fqt1_status st = scq_scratch_address(&scratch, &dev, (cudaStream_t)stream);
   if (st != FQT1_OK) return st;
-  return quantize_impl(g, M, D, gamma, p_sample, psq, p_channel, pcq, scratch,
-                       sizeof(uint32_t) * FQT1_NOALLOC_SCRATCH_KEYS, dev_status, (cudaStream_t)stream);
+  const fqt1_status q = quantize_impl(g, M, D, gamma, p_sample, psq, p_channel, pcq, scratch,
+                                      sizeof(uint32_t) * FQT1_NOALLOC_SCRATCH_KEYS, dev_status,
+                                      (cudaStream_t)stream);
+  if (q != FQT1_OK) {
+    // the range kernel may have run and left keys that no selection kernel reset: the next
+    // call on this device fills the array again
+    std::lock_guard<std::mutex> lock(g_scq_scratch_mu);
+    g_scq_scratch_ready[dev] = false;
+  }
+  return q;
 }

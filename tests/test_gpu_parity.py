@@ -540,6 +540,29 @@ def test_table5_shapes_exact(M, K, N):
     assert np.array_equal(acc4.cpu().numpy()[:cnt], om.int_matmul(ref["codes"], om.sign(b)))
 
 
+@pytest.mark.parametrize("M,K,D", [(300, 1000, 64), (257, 129, 70), (128, 2304, 256)])
+def test_fwd_acc_only(M, K, D):
+    """fqt1_fwd_gemm with y = NULL (and no Gamma) writes the int32 accumulators alone, on the
+    tensor-core kernel: exact against the oracle (TMA stores when D is a multiple of 4, direct
+    stores otherwise)."""
+    from paper_2408_14267_gb300 import fqt1
+    rng = np.random.default_rng(M * 7 + D)
+    a = rng.standard_normal((M, K)).astype(np.float32)
+    b = rng.standard_normal((D, K)).astype(np.float32)
+    dev = torch.device("cuda")
+    wK = fqt1.packed_words(K)
+    sa = torch.empty(M, wK, dtype=torch.int32, device=dev)
+    sb = torch.empty(D, wK, dtype=torch.int32, device=dev)
+    fqt1.binarize_pack(torch.from_numpy(a).cuda(), M, K, K, sa, None, None)
+    fqt1.binarize_pack(torch.from_numpy(b).cuda(), D, K, K, sb, None, None)
+    acc = torch.full((M, D), 7777, dtype=torch.int32, device=dev)
+    n0 = fqt1.kernel_launches()
+    fqt1.fwd_gemm(sa, sb, M, D, K, None, acc, None)
+    torch.cuda.synchronize()
+    assert fqt1.kernel_launches() == n0 + 1
+    assert np.array_equal(acc.cpu().numpy(), om.int_matmul(om.sign(a), om.sign(b)))
+
+
 @pytest.mark.parametrize("name,make", [CASES[0], CASES[1]], ids=[CASES[0][0], CASES[1][0]])
 def test_host_copy_step_matches_serial(name, make):
     """The step with its host copies (LayerStep.step_concurrent_host, the end-to-end form) gives
