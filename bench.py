@@ -261,6 +261,54 @@ def stage_work(st, name):
     return "hbm", 0
 
 
+def stage_times(st, stream, flush, reps):
+    """Mean device time (ms) of each stage of the step, eager: the L2 is flushed, a sleep kernel
+    holds the stream while all launches are queued, and CUDA events on the launching stream
+    bracket every stage."""
+    import torch
+    stages = st.stages()
+    per_stage = {n: [] for n, _ in stages}
+    with torch.cuda.stream(stream):
+        for _ in range(reps):
+            flush.zero_()
+            torch.cuda._sleep(2_000_000)
+            evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)]
+            evs[0].record(stream)
+            for i, (n, fn) in enumerate(stages):
+                fn(stream)
+                evs[i + 1].record(stream)
+            stream.synchronize()
+            for i, (n, _) in enumerate(stages):
+                per_stage[n].append(evs[i].elapsed_time(evs[i + 1]))
+    return {n: statistics.mean(v) for n, v in per_stage.items()}
+
+
+GEMM_STAGES = (("fwd", ("fwd_gemm",)), ("bwd_input", ("bwd_input_fold", "bwd_input_gemm")),
+               ("bwd_weight", ("bwd_weight_gemm",)))
+
+
+def gemm_rooflines(st, stage_ms, bf16_peak, peak_src):
+    """Tensor roofline of each of the three products: algorithmic operations (2 M K D for the
+    forward, 2 (kept rows) D K for grad_input, 2 (kept channels) M K for grad_weight) over the
+    stage's device time, against the fp8 dense peak (2 x the bf16 peak: the nominal fp8/bf16
+    ratio; the products run on e4m3 tensor cores)."""
+    out = {}
+    peak = 2.0 * bf16_peak
+    for key, names in GEMM_STAGES:
+        name = next((n for n in names if n in stage_ms), None)
+        if name is None:
+            continue
+        _, ops = stage_work(st, name)
+        us = stage_ms[name] * 1e3
+        tf = ops / (us * 1e-6) / 1e12
+        out[key] = {"kernel_stage": name, "ops": ops, "time_us": round(us, 3), "achieved": round(tf, 2),
+                    "peak": peak, "unit": "TFLOP/s", "frac": tf / peak,
+                    "peak_note": f"fp8 dense = 2 x {peak_src} bf16 (nominal fp8/bf16 ratio)"}
+        if name == "bwd_input_fold":
+            out[key]["note"] = "the Folder and the dequantization run in the same kernel's epilogue"
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -270,6 +318,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--implicit", action="store_true",
                     help="implicit-GEMM forward (pixel-major sign(X), no unfolded row packing)")
+    ap.add_argument("--e4m3-weights", choices=["on", "off"], default="off",
+                    help="e4m3 copies of sign(W) written by the weight packing and loaded by TMA as the "
+                         "B operand of the forward and grad_input products")
     ap.add_argument("--profile", type=int, default=0, metavar="N",
                     help="only run --warmup + N eager steps (for ncu), print nothing")
     ap.add_argument("--table5", action="store_true",
@@ -280,6 +331,9 @@ def main():
                     help="the layer step on every VGG-16 / ResNet-18 layer shape")
     ap.add_argument("--variance", action="store_true",
                     help="empirical variance of the AGP quantizer (b = 2, 4, 8) and of 1-bit PSQ against Eq. 24")
+    ap.add_argument("--sweep", choices=["routine", "diag", "full"],
+                    help="GEMM-shaped layer sweep: routine = M=D=K=4096, 256 groups, b = 1, 2, 4, 8; "
+                         "diag = M=D=K in 1024..16384, 256 groups, b = 4; full = the whole grid")
     ap.add_argument("--res", type=int, default=32, help="input resolution of --model")
     ap.add_argument("--batch", type=int, default=128, help="batch of --model")
     args = ap.parse_args()
@@ -297,6 +351,8 @@ def main():
         return variance_study(args)
     if args.layers:
         return layer_sweep(args)
+    if args.sweep:
+        return gemm_sweep(args)
 
     import torch
     import torch.distributed as dist
@@ -311,7 +367,8 @@ def main():
     from paper_2408_14267_gb300.layer import LayerStep
 
     wl = workloads.resnet18_cifar_conv()
-    st = LayerStep(wl, device=f"cuda:{local_rank}", keep_acc=False, implicit=args.implicit)
+    st = LayerStep(wl, device=f"cuda:{local_rank}", keep_acc=False, implicit=args.implicit,
+                   e4m3_weights=args.e4m3_weights == "on")
     stream = torch.cuda.Stream()
     if args.profile:
         with torch.cuda.stream(stream):
@@ -320,7 +377,6 @@ def main():
         torch.cuda.synchronize()
         return
     flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device="cuda")  # 256 MiB > 129 MB L2
-    stages = st.stages()
     with torch.cuda.stream(stream):
         for _ in range(max(args.warmup, 3)):
             st.step()
@@ -372,20 +428,7 @@ def main():
     value = job_tops(ops, args.steps, world, total_ms)
 
     # per-stage device time (eager; the stream is held by a sleep kernel while all launches are queued)
-    per_stage = {n: [] for n, _ in stages}
-    with torch.cuda.stream(stream):
-        for _ in range(max(10, min(args.steps, 50))):
-            flush.zero_()
-            torch.cuda._sleep(2_000_000)
-            evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)]
-            evs[0].record(stream)
-            for i, (n, fn) in enumerate(stages):
-                fn(stream)
-                evs[i + 1].record(stream)
-            stream.synchronize()
-            for i, (n, _) in enumerate(stages):
-                per_stage[n].append(evs[i].elapsed_time(evs[i + 1]))
-    stage_ms = {n: statistics.mean(v) for n, v in per_stage.items()}
+    stage_ms = stage_times(st, stream, flush, max(10, min(args.steps, 50)))
     dom = max(stage_ms, key=stage_ms.get)
     hbm_peak, bf16_peak, peak_src = load_peaks()
     bound, work = stage_work(st, dom)
@@ -403,6 +446,7 @@ def main():
     roof["traffic"] = stage_traffic(dom)
     roof["kernel"] = dom
     roof["peak_source"] = peak_src if bound != "alu" else "derived: 152 SMs x 16 popc/clk x 32 bit x 2 x max clock"
+    roof["gemms"] = gemm_rooflines(st, stage_ms, bf16_peak, peak_src)
 
     # end to end: pinned host inputs -> device, step, outputs -> pinned host, all inside the timed region
     h_in = [t.detach().cpu().pin_memory() for t in (st.x, st.w, st.gy)]
@@ -446,7 +490,7 @@ def main():
         cpu = {"value": r["ops"] / t / 1e12, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": f"oracle layer step on 32 of the 128 samples (M={r['M']} K={r['K']} D={r['D']}), "
                          f"mean of 2 runs after one untimed run, {t:.2f} s each, one thread"}
-        ncores = min(host_cores(), 16)
+        ncores = host_cores()
         if ncores > 1:
             ra = run_oracle_parallel(batch=32, procs=ncores)
             cpu["all_cores"] = {"value": ra["value"], "unit": UNIT, "cores": ncores, "kind": "oracle",
@@ -467,7 +511,9 @@ def main():
                                      "epilogue), CUDA events on the launching stream",
                            "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU",
                            "forward": "implicit GEMM (pixel-major sign(X))" if st.implicit
-                           else "1-bit unfolded X_u"},
+                           else "1-bit unfolded X_u",
+                           "weights": "e4m3 copies of sign(W) by TMA" if (st.w8 is not None or st.wt8 is not None)
+                           else "packed sign(W) expanded per CTA"},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
                 "clocks": clocks, "stage_ms": {k: round(v, 5) for k, v in stage_ms.items()}}
         print(json.dumps(line))
@@ -601,6 +647,118 @@ def layer_sweep(args):
                                  "l2": "flushed before every timed replay (256 MiB write)",
                                  "timing": "one CUDA graph of the three-branch step per layer, CUDA events, median"},
                       "layers": rows}))
+
+
+SWEEP_SIZES = (1024, 2048, 4096, 8192, 16384)
+SWEEP_GROUPS = (64, 128, 256, 512, 1024)
+SWEEP_BITS = (1, 2, 4, 8)
+SWEEP_ORACLE_MAX = 4096  # the oracle is timed on sweep points up to M = K = D = 4096
+
+SWEEP_ORACLE_SCRIPT = r"""
+import json, sys, time
+sys.path.insert(0, sys.argv[1])
+from paper_2408_14267_gb300 import workloads as wl
+from oracle import method as om
+M, K, D, G, b, gs = (int(v) for v in sys.argv[2:8])
+w = wl.sweep_point(M, K, D, G, b)
+rpg = M // G
+rows = gs * rpg
+x, gy = w["x"][:rows], w["gy"][:rows]
+om.layer_step_linear(x[:rpg * b], w["w"], w["gamma"], gy[:rpg * b], b, w["mode_s"], w["seed_s"], b, w["mode_c"],
+                     w["seed_c"], rpg)
+t0 = time.perf_counter()
+om.layer_step_linear(x, w["w"], w["gamma"], gy, b, w["mode_s"], w["seed_s"], b, w["mode_c"], w["seed_c"], rpg)
+t = time.perf_counter() - t0
+print(json.dumps({"s": t, "ops": 6.0 * rows * K * D, "rows": rows}))
+"""
+
+
+def sweep_points(which):
+    if which == "routine":
+        return [(4096, 4096, 4096, 256, b) for b in SWEEP_BITS]
+    if which == "diag":
+        return [(n, n, n, 256, 4) for n in SWEEP_SIZES]
+    return [(n, k, n, g, b) for n in SWEEP_SIZES for k in SWEEP_SIZES for g in SWEEP_GROUPS for b in SWEEP_BITS]
+
+
+def gemm_sweep(args):
+    """The throughput sweep over GEMM-shaped linear layers (M = D rows and output channels, K
+    input features, `groups` sample groups of M / groups rows, AGP b on both SCQ branches with
+    keep ratio 1/b).  Per point one JSON line: the three-branch step as one CUDA graph (L2
+    flushed before every replay, CUDA events, mean over `steps` replays), its effective TOPS
+    (6 M K D / time), the step's fraction of the fp8 tensor peak (issued product operations
+    2 M K D + 2 (kept rows) D K + 2 (kept channels) M K over the time), its fraction of the HBM
+    peak counting only the fp32 inputs and outputs (x, W, gY read; y, dx, dW written), each
+    product's own tensor fraction from an eager per-stage pass, and, up to 4096, the oracle timed
+    on one host core over the first 16 sample groups of the point."""
+    import torch
+    from paper_2408_14267_gb300 import build, workloads
+    build.build()
+    from paper_2408_14267_gb300.layer import LayerStep
+    dev = torch.device("cuda")
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)  # 256 MiB > 129 MB L2
+    stream = torch.cuda.Stream()
+    hbm_peak, bf16_peak, peak_src = load_peaks()
+    fp8_peak = 2.0 * bf16_peak
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               NUMEXPR_NUM_THREADS="1")
+    for (M, K, D, G, b) in sweep_points(args.sweep):
+        wl = workloads.sweep_point_device(M, K, D, G, b, dev)
+        st = LayerStep(wl, device=dev, keep_acc=False)
+        del wl
+        with torch.cuda.stream(stream):
+            st.dev_status.zero_()
+            for _ in range(3):
+                st.step()
+            stream.synchronize()
+            if int(st.dev_status[0].item()) != 0:
+                raise RuntimeError(f"sweep point {(M, K, D, G, b)}: device status {int(st.dev_status[0].item()):#x}")
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                st.step_concurrent(stream)
+            for _ in range(max(args.warmup, 3)):
+                g.replay()
+            ts = []
+            for _ in range(args.steps):
+                flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                g.replay()
+                e1.record(stream)
+                ts.append((e0, e1))
+            stream.synchronize()
+        ms = statistics.mean(a.elapsed_time(e) for a, e in ts)
+        stage_ms = stage_times(st, stream, flush, 5)
+        ks, kc = st.psq.count() * st.rpg, st.pcq.count()
+        issued = 2.0 * M * K * D + 2.0 * ks * D * K + 2.0 * kc * M * K
+        io = 4.0 * (2 * M * K + 2 * D * K + 2 * M * D)
+        sec = ms * 1e-3
+        line = {"point": {"M": M, "K": K, "D": D, "groups": G, "bits": b, "kept_rows": ks, "kept_channels": kc},
+                "ms": round(ms, 5), "tops": 6.0 * M * K * D / sec / 1e12, "unit": "TOPS",
+                "tensor_frac": issued / sec / 1e12 / fp8_peak, "hbm_frac": io / sec / 1e9 / hbm_peak,
+                "peaks": {"fp8_tflops": fp8_peak, "hbm_gbs": hbm_peak, "source": peak_src,
+                          "note": "fp8 = 2 x bf16 (nominal ratio); HBM fraction counts fp32 I/O only"},
+                "gemms": gemm_rooflines(st, stage_ms, bf16_peak, peak_src),
+                "stage_ms": {k: round(v, 5) for k, v in stage_ms.items()},
+                "config": {"l2": "flushed before every timed replay (256 MiB write)",
+                           "timing": "one CUDA graph of the three-branch step, CUDA events, mean",
+                           "steps": args.steps, "warmup": args.warmup, "data": "synthetic (device draw)"}}
+        if max(M, K, D) <= SWEEP_ORACLE_MAX and not args.no_cpu_baseline:
+            gs = 16
+            p = subprocess.run([sys.executable, "-c", SWEEP_ORACLE_SCRIPT, ROOT, str(M), str(K), str(D), str(G),
+                                str(b), str(gs)], env=env, capture_output=True, text=True, timeout=1800)
+            if p.returncode == 0:
+                r = json.loads(p.stdout.strip().splitlines()[-1])
+                line["cpu_baseline"] = {"value": r["ops"] / r["s"] / 1e12, "unit": "TOPS", "cores": 1,
+                                        "kind": "oracle",
+                                        "sample": f"oracle layer step on the first {gs} of {G} sample groups "
+                                                  f"({r['rows']} rows), full K and D, one thread, after one "
+                                                  f"untimed step on {b} groups"}
+            else:
+                line["cpu_baseline"] = {"error": p.stderr[-300:]}
+        print(json.dumps(line), flush=True)
+        del g, st
+        torch.cuda.empty_cache()
 
 
 def build_model(name, res, binary, classes=10):

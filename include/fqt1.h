@@ -193,6 +193,16 @@ fqt1_status fqt1_bwd_input_fold_nhwc(const fqt1_qgrad* psq, const uint32_t* sw_c
 fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D, int64_t K,
                           const float* gamma, int32_t* acc, float* y, void* stream);
 
+/* Test of the failure path (no counterpart in the paper): the kernel of fqt1_fwd_gemm
+ * with every bounded wait cut to 20 ms and the arrive that hands its first operand stage to
+ * the tensor cores withheld, so the wait for it runs out.  The kernel then sets
+ * FQT1_DEV_TIMEOUT in *dev_status (int32, zeroed by the caller), waits for its in-flight copies,
+ * frees its tensor memory and returns; the context stays usable.  y receives unspecified
+ * values.  Arguments as fqt1_fwd_gemm (gamma and y required, no acc).  Meant for tests that
+ * check that a caller sees an expired wait as a status, not as a hang. */
+fqt1_status fqt1_test_expired_wait(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D, int64_t K,
+                                   const float* gamma, float* y, int32_t* dev_status, void* stream);
+
 /* fqt1_fwd_gemm with a per-channel bias: y[m, j] = gamma[j] * acc[m, j] + bias[j]
  * (fp32 multiply, then fp32 add).  The paper's layer (Sec. 5.1) has the scale
  * Gamma only; the bias is the usual extension of a linear or convolution layer

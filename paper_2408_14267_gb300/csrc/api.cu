@@ -269,6 +269,16 @@ extern "C" fqt1_status fqt1_fwd_gemm_e4m3w(const uint32_t* sx_row, const uint8_t
   return FQT1_OK;
 }
 
+extern "C" fqt1_status fqt1_test_expired_wait(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D,
+                                              int64_t K, const float* gamma, float* y, int32_t* dev_status,
+                                              void* stream) {
+  if (!sx_row || !sw_row || !gamma || !y || !dev_status || M < 1 || D < 1 || K < 1) return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(sx_row) || !aligned16(sw_row) || !aligned16(gamma) || !aligned16(y)) return FQT1_ERR_MISALIGNED;
+  if (K >= (1ll << 24) || (M + 127) / 128 > 65535) return FQT1_ERR_UNSUPPORTED;
+  FQT1_CUDA_TRY(launch_fwd_lost_arrive_tc(sx_row, sw_row, M, D, K, gamma, y, dev_status, (cudaStream_t)stream));
+  return FQT1_OK;
+}
+
 extern "C" fqt1_status fqt1_fwd_gemm(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D,
                                      int64_t K, const float* gamma, int32_t* acc, float* y, void* stream) {
   return fqt1_fwd_gemm_bias(sx_row, sw_row, M, D, K, gamma, nullptr, acc, y, stream);

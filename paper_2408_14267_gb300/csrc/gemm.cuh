@@ -29,6 +29,10 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
                            const float* zero, const int32_t* cs, const int32_t* slot_of_group, float* dx, int N, int C,
                            int H, int W, int kh, int kw, int stride, int pad, int Ho, int Wo, int32_t* status,
                            cudaStream_t s, const uint8_t* Bte = nullptr, int64_t ldbte = 0, int nhwc = 0);
+// fqt1_fwd_gemm's kernel with the first operand stage's arrive withheld: its bounded waits
+// (20 ms) expire, FQT1_DEV_TIMEOUT is set in *status and the kernel returns normally.
+cudaError_t launch_fwd_lost_arrive_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64_t D, int64_t K,
+                                      const float* gamma, float* y, int32_t* status, cudaStream_t s);
 // Forward with B = e4m3 sign(W) rows [D][ldbe] bytes (+1 = 0x38, -1 = 0xB8, bytes past K zero).
 cudaError_t launch_fwd_e4m3w_tc(const uint32_t* A, const uint8_t* Be, int64_t ldbe, int64_t M, int64_t D, int64_t K,
                                 const float* gamma, const float* bias, int32_t* acc, float* y, int32_t* status,

@@ -111,14 +111,15 @@ __device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
 }
 // Bounded wait for phase `parity` of barrier b; false (and the timeout status) if it expired
 // or another role already gave up.
-__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, volatile int* abort_flag, int32_t* status) {
+__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, volatile int* abort_flag, int32_t* status,
+                                          uint64_t limit_ns = kWaitNs) {
   if (mbar_test(b, parity)) return true;
   const uint64_t t0 = gtimer();
   for (uint32_t n = 1;; ++n) {
     if (mbar_test(b, parity)) return true;
     if ((n & 1023u) == 0) {  // the timer and the abort flag are checked every 1024 polls
       if (*abort_flag) return false;
-      if (gtimer() - t0 > kWaitNs) {
+      if (gtimer() - t0 > limit_ns) {
         *abort_flag = 1;
         if (status) atomicOr(status, FQT1_DEV_TIMEOUT);
         return false;
@@ -219,6 +220,23 @@ __device__ __forceinline__ void mma_e4m3_ta(uint32_t tmem_d, uint32_t tmem_a, ui
       "r"(tmem_a), "l"(bd), "r"(idesc), "r"(acc));
 }
 
+// A and B both from shared-memory descriptors.
+__device__ __forceinline__ void mma_e4m3_ss(uint32_t tmem_d, uint64_t ad, uint64_t bd, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "l"(ad), "l"(bd), "r"(idesc), "r"(acc));
+}
+
+// An fp32 accumulator word -> the exact int32 sum.  With A_DIRECT the A operand was the code
+// bytes themselves, read as e4m3: byte q < 16 is the e4m3 number q 2^-9 (subnormals 0..7,
+// then the first binade 8..15), so the accumulator holds sum 2^-9 and 512 rescales it exactly.
+template <bool A_DIRECT>
+__device__ __forceinline__ int32_t acc_int(uint32_t v) {
+  if constexpr (A_DIRECT) return __float2int_rn(__fmul_rn(__uint_as_float(v), 512.0f));
+  else return __float2int_rn(__uint_as_float(v));
+}
+
 // 32 consecutive TMEM columns of this thread's lane <- v (the warp writes its 32 lanes).
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
   asm volatile(
@@ -317,13 +335,23 @@ struct TcSmem {
 // SHORT tiles run two CTAs per SM, which caps the registers at 65536 / (2 * 320) per thread.
 // X selects the optional datapaths at compile time, so that the default kernels carry none of
 // their code: bit 0 the implicit-convolution A operand, bit 1 B as e4m3 bytes by TMA (b_tma),
-// bit 2 the Folder's NHWC output.
+// bit 2 the Folder's NHWC output, bit 3 codes of at most 4 bits as the A operand straight from
+// the raw ring (A_DIRECT: the MMA reads the TMA-written code tile as e4m3, nothing expands A;
+// the raw stage is released by the MMA's commit), bit 4 the failure-path test: the expansion
+// warps withhold their arrive on the first operand stage, so the MMA issuer's bounded wait
+// (20 ms in this instantiation) expires and the kernel takes its timeout exit.
 template <bool A_CODES, bool BITS8, int BN, bool SHORT, int X = 0>
 __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmAcc, TcArgs a) {
   using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
-  constexpr bool kImpl = (X & 1) != 0, kBtma = (X & 2) != 0, kNhwc = (X & 4) != 0;
+  constexpr bool kImpl = (X & 1) != 0, kBtma = (X & 2) != 0, kNhwc = (X & 4) != 0, kAdir = (X & 8) != 0;
+  static_assert(!kAdir || (A_CODES && !BITS8), "A_DIRECT takes codes below 16");
+  constexpr bool kLose = (X & 16) != 0;
+  constexpr uint64_t kLimit = kLose ? 20000000ull : kWaitNs;  // bound of every wait below
+  // arrivals that free a raw stage: the expansion warps (when they read it) and, with A_DIRECT,
+  // the commit of the MMAs that read its A tile
+  constexpr uint32_t kRawEmpty = kAdir ? (kBtma ? 1u : (uint32_t)kExpWarps + 1u) : (uint32_t)kExpWarps;
   constexpr int OS = S::kOpStages, RS = S::kRawStages, KSUB = S::KSUB;
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t raw_full[kMaxStages], raw_empty[kMaxStages], op_full[kMaxStages],
@@ -355,7 +383,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
-    for (int s = 0; s < RS; ++s) { mbar_init(&raw_full[s], 1); mbar_init(&raw_empty[s], kExpWarps); }
+    for (int s = 0; s < RS; ++s) { mbar_init(&raw_full[s], 1); mbar_init(&raw_empty[s], kRawEmpty); }
     for (int s = 0; s < OS; ++s) { mbar_init(&op_full[s], kExpWarps); mbar_init(&op_empty[s], 1); mbar_init(&b_full[s], 1); }
     mbar_init(&acc_full, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -415,7 +443,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       int issued = 0;
       for (int i = 0; i < nk; ++i) {
         const int s = i % RS, it = i / RS;
-        if (it > 0 && !mbar_wait(&raw_empty[s], (it - 1) & 1, &abort_flag, a.status)) break;
+        if (it > 0 && !mbar_wait(&raw_empty[s], (it - 1) & 1, &abort_flag, a.status, kLimit)) break;
         const int kt = kt0 + i;
         mbar_expect_tx(&raw_full[s], kTx);
         if (A_CODES) {
@@ -456,11 +484,13 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_e4m3(BN);
       for (int i = 0; i < nk; ++i) {
-        const int s = i % OS, it = i / OS;
-        if (!mbar_wait(&op_full[s], it & 1, &abort_flag, a.status)) break;
-        if (kBtma && !mbar_wait(&b_full[s], it & 1, &abort_flag, a.status)) break;
+        const int s = i % OS, it = i / OS, sr = i % RS, itr = i / RS;
+        if (!mbar_wait(&op_full[s], it & 1, &abort_flag, a.status, kLimit)) break;
+        if (kBtma && !mbar_wait(&b_full[s], it & 1, &abort_flag, a.status, kLimit)) break;
+        if (kAdir && !mbar_wait(&raw_full[sr], itr & 1, &abort_flag, a.status, kLimit)) break;  // the A codes landed
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const uint32_t acol = tmem + BN + s * S::kAcols, baddr = smem_u32(opB(s));
+        const uint32_t aaddr = smem_u32(rawA(sr));
         const int nsub = valid_subtiles<KSUB>(a.L, kt0 + i);
 #pragma unroll
         for (int h = 0; h < KSUB; ++h) {
@@ -468,11 +498,17 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
 #pragma unroll
           for (int k = 0; k < kBK / 32; ++k) {
             const uint64_t bd = sw128_desc(baddr + h * S::kSub + 32 * k);
-            mma_e4m3_ta(tmem, acol + (kBK / 4) * h + 8 * k, bd, idesc, (i > 0 || h > 0 || k > 0) ? 1u : 0u);
-            if (BITS8) mma_e4m3_ta(tmem, acol + (kBK / 4) * (KSUB + h) + 8 * k, bd, idesc, 1u);
+            const uint32_t first = (i > 0 || h > 0 || k > 0) ? 1u : 0u;
+            if (kAdir) {
+              mma_e4m3_ss(tmem, sw128_desc(aaddr + h * (kBM * kBK) + 32 * k), bd, idesc, first);
+            } else {
+              mma_e4m3_ta(tmem, acol + (kBK / 4) * h + 8 * k, bd, idesc, first);
+              if (BITS8) mma_e4m3_ta(tmem, acol + (kBK / 4) * (KSUB + h) + 8 * k, bd, idesc, 1u);
+            }
           }
         }
         mma_commit(&op_empty[s]);
+        if (kAdir) mma_commit(&raw_empty[sr]);  // the A tile is free once these MMAs are done
       }
       mma_commit(&acc_full);
     }
@@ -486,11 +522,15 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     // 5 / 9); warps 2, 3, 6 and 7 then take the B rows.
     const int64_t tile_rows = valid_rows - m0;  // may exceed kBM or be negative
     const int live_q = tile_rows >= kBM ? 4 : (tile_rows <= 0 ? 0 : (int)((tile_rows + 31) / 32));
-    const bool split = KSUB == 2 && live_q <= 2;
-    const bool a_warp = kBtma ? true : split ? (warp == 4 || warp == 5 || warp >= 8) : warp < 6;
+    // A_DIRECT: no A expansion; all eight warps expand B (or, with b_tma, nothing), warps 2..5
+    // the first half of a stage's sub-tiles and warps 6..9 the second half, each warp the 32 B
+    // rows of its lane quarter
+    const bool split = !kAdir && KSUB == 2 && live_q <= 2;
+    const bool a_warp = kAdir ? false : kBtma ? true : split ? (warp == 4 || warp == 5 || warp >= 8) : warp < 6;
     const int a_h0 = kBtma ? (warp >= 6 ? KSUB / 2 : 0) : (split && warp >= 8 ? 1 : 0);
     const int a_h1 = kBtma ? a_h0 + KSUB / 2 : (split ? a_h0 + 1 : KSUB);
-    const int bblk = split ? (warp == 2 ? 0 : warp == 3 ? 1 : warp == 6 ? 2 : 3) : warp - 6;
+    const int bblk = kAdir ? (warp & 3) : split ? (warp == 2 ? 0 : warp == 3 ? 1 : warp == 6 ? 2 : 3) : warp - 6;
+    const int b_h0 = kAdir ? (warp >= 6 ? KSUB / 2 : 0) : 0, b_h1 = kAdir ? b_h0 + KSUB / 2 : KSUB;
     const int quarter = warp & 3;
     const int arow = 32 * quarter + lane, brow = 32 * bblk + lane;
     // a warp whose 32 A rows all lie past the kept rows skips its work: an accumulator row
@@ -500,7 +540,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     int b_issued = 0;  // b_tma: operand stages whose B boxes this thread (warp 2, lane 0) issued
     for (int i = 0; i < nk; ++i) {
       const int so = i % OS, ito = i / OS, sr = i % RS, itr = i / RS;
-      if (ito > 0 && !mbar_wait(&op_empty[so], (ito - 1) & 1, &abort_flag, a.status)) break;
+      if (ito > 0 && !mbar_wait(&op_empty[so], (ito - 1) & 1, &abort_flag, a.status, kLimit)) break;
       if (kBtma) {  // the stage's B boxes, as soon as the MMAs of its previous use are done
         if (warp == 2 && lane == 0) {
           mbar_expect_tx(&b_full[so], (uint32_t)S::kOpB);
@@ -511,9 +551,12 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         }
         __syncwarp();
       }
-      if (!mbar_wait(&raw_full[sr], itr & 1, &abort_flag, a.status)) break;
+      // with A_DIRECT and b_tma the expansion warps read nothing from the raw stage
+      if (!(kAdir && kBtma) && !mbar_wait(&raw_full[sr], itr & 1, &abort_flag, a.status, kLimit)) break;
       const int kt = kt0 + i;
-      if (a_warp) {
+      if (kAdir && kBtma) {
+        // nothing to expand: the arrive below only hands the B stage's issue to the MMA
+      } else if (a_warp) {
         if (a_live) {
           const uint32_t acol = a_lanes + BN + so * S::kAcols;
           const int nsub = min(valid_subtiles<KSUB>(a.L, kt), a_h1);
@@ -569,9 +612,9 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         }
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       } else {
-        const int nsub = valid_subtiles<KSUB>(a.L, kt);
+        const int nsub = min(valid_subtiles<KSUB>(a.L, kt), b_h1);
 #pragma unroll
-        for (int h = 0; h < KSUB; ++h) {
+        for (int h = b_h0; h < KSUB; ++h) {
           if (h >= nsub) break;
           const uint4 w4 = *reinterpret_cast<const uint4*>(rawB(sr) + brow * S::kRawRow + 16 * h);
           const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
@@ -586,8 +629,8 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       }
       __syncwarp();
       if (lane == 0) {
-        mbar_arrive(&op_full[so]);
-        mbar_arrive(&raw_empty[sr]);
+        if (!(kLose && i == 0)) mbar_arrive(&op_full[so]);
+        if (!(kAdir && kBtma)) mbar_arrive(&raw_empty[sr]);
       }
     }
 
@@ -729,7 +772,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       if (a.bias && tt < BN) bias_s[tt] = n0 + tt < a.N ? __ldg(a.bias + n0 + tt) : 0.f;
       asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
     }
-    const bool have_acc = mbar_wait(&acc_full, 0, &abort_flag, a.status);
+    const bool have_acc = mbar_wait(&acc_full, 0, &abort_flag, a.status, kLimit);
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     if (a.epi == EPI_FOLD) {
       // 1. the whole 128 x BN accumulator tile -> shared memory as int32 (rings are idle);
@@ -752,7 +795,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
         int32_t* trow = T + (32 * qf + lane) * TS + c0;
 #pragma unroll
-        for (int j = 0; j < 32; ++j) trow[j] = __float2int_rn(__uint_as_float(v[j]));
+        for (int j = 0; j < 32; ++j) trow[j] = acc_int<kAdir>(v[j]);
       }
       const int rpg = (int)a.rpg, imgs = f_imgs, khw = f_khw, HW = f_HW;
       const int c_first = f_c0, nc = f_nc;
@@ -876,10 +919,10 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
           int4 w;
-          w.x = __float2int_rn(__uint_as_float(v[4 * c + 0]));
-          w.y = __float2int_rn(__uint_as_float(v[4 * c + 1]));
-          w.z = __float2int_rn(__uint_as_float(v[4 * c + 2]));
-          w.w = __float2int_rn(__uint_as_float(v[4 * c + 3]));
+          w.x = acc_int<kAdir>(v[4 * c + 0]);
+          w.y = acc_int<kAdir>(v[4 * c + 1]);
+          w.z = acc_int<kAdir>(v[4 * c + 2]);
+          w.w = acc_int<kAdir>(v[4 * c + 3]);
           *reinterpret_cast<int4*>(base + ptile_off(r, (c0 >> 2) + c)) = w;
         }
         continue;
@@ -896,10 +939,10 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         const int64_t nb = n0 + c0;
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
-          const int32_t i0 = __float2int_rn(__uint_as_float(v[4 * c + 0]));
-          const int32_t i1 = __float2int_rn(__uint_as_float(v[4 * c + 1]));
-          const int32_t i2 = __float2int_rn(__uint_as_float(v[4 * c + 2]));
-          const int32_t i3 = __float2int_rn(__uint_as_float(v[4 * c + 3]));
+          const int32_t i0 = acc_int<kAdir>(v[4 * c + 0]);
+          const int32_t i1 = acc_int<kAdir>(v[4 * c + 1]);
+          const int32_t i2 = acc_int<kAdir>(v[4 * c + 2]);
+          const int32_t i3 = acc_int<kAdir>(v[4 * c + 3]);
           const int off = lane * 32 + ((c ^ (lane & 7)) << 2);
           if (a.tma_out & 1) {
             const float4 g4 = *reinterpret_cast<const float4*>(gamma_s + c0 + 4 * c);
@@ -930,7 +973,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         if (r >= valid_rows || r >= a.M || nb >= a.N) continue;
         int32_t iv[32];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) iv[j] = __float2int_rn(__uint_as_float(v[j]));
+        for (int j = 0; j < 32; ++j) iv[j] = acc_int<kAdir>(v[j]);
         const bool full = nb + 32 <= a.N && (a.ldo % 4) == 0;
         int64_t out_row = r;
         float sc = 0.f, ze = 0.f;
@@ -1004,10 +1047,10 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         uint4 w;
-        w.x = (uint32_t)__float2int_rn(__uint_as_float(v[4 * c + 0]));
-        w.y = (uint32_t)__float2int_rn(__uint_as_float(v[4 * c + 1]));
-        w.z = (uint32_t)__float2int_rn(__uint_as_float(v[4 * c + 2]));
-        w.w = (uint32_t)__float2int_rn(__uint_as_float(v[4 * c + 3]));
+        w.x = (uint32_t)acc_int<kAdir>(v[4 * c + 0]);
+        w.y = (uint32_t)acc_int<kAdir>(v[4 * c + 1]);
+        w.z = (uint32_t)acc_int<kAdir>(v[4 * c + 2]);
+        w.w = (uint32_t)acc_int<kAdir>(v[4 * c + 3]);
         *reinterpret_cast<uint4*>(stage + lane * 32 + ((c ^ (lane & 7)) << 2)) = w;
       }
       __syncwarp();
@@ -1212,6 +1255,24 @@ cudaError_t launch_fwd_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64
   return launch_fwd_common(ma, TcArgs{}, B, M, D, K, gamma, bias, acc, y, status, s);
 }
 
+// The failure-path test: fqt1_fwd_gemm's kernel with one operand-stage arrive withheld (bit 4).
+cudaError_t launch_fwd_lost_arrive_tc(const uint32_t* A, const uint32_t* B, int64_t M, int64_t D, int64_t K,
+                                      const float* gamma, float* y, int32_t* status, cudaStream_t s) {
+  using S = TcSmem<false, false, 128>;
+  const int64_t ldw = fqt1_packed_words(K);
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, A, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, M, ldw * 4, 4 * S::KSUB, kBM,
+                CU_TENSOR_MAP_SWIZZLE_NONE) ||
+      !make_map(&mb, B, CU_TENSOR_MAP_DATA_TYPE_UINT32, ldw, D, ldw * 4, 4 * S::KSUB, 128,
+                CU_TENSOR_MAP_SWIZZLE_NONE))
+    return cudaErrorInvalidValue;
+  TcArgs a{};
+  a.M = M; a.N = D; a.L = K; a.count = nullptr; a.rows_per_count = 1;
+  a.k_tiles = (int)((K + kBK * S::KSUB - 1) / (kBK * S::KSUB)); a.tiles_per_split = a.k_tiles;
+  a.epi = EPI_FWD; a.gamma = gamma; a.y = y; a.ldo = D; a.status = status;
+  return launch_tc<false, false, 128, false, 16>(ma, mb, a, 1, s);
+}
+
 // Forward with B = e4m3 sign(W) rows [D][ldbe] bytes (ldbe a multiple of 16, bytes past K zero).
 cudaError_t launch_fwd_e4m3w_tc(const uint32_t* A, const uint8_t* Be, int64_t ldbe, int64_t M, int64_t D, int64_t K,
                                 const float* gamma, const float* bias, int32_t* acc, float* y, int32_t* status,
@@ -1283,7 +1344,7 @@ cudaError_t launch_codes_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max
   a.epi = epi;
   const int z = (a.k_tiles + a.tiles_per_split - 1) / a.tiles_per_split;
   if (bits == 8) return launch_tc<true, true, 128>(ma, mb, a, z, s);
-  return launch_tc<true, false, 128>(ma, mb, a, z, s);
+  return launch_tc<true, false, 128, false, 8>(ma, mb, a, z, s);  // codes < 16: A straight from TMA
 }
 
 // grad_input of a convolution with the Folder in the epilogue (EPI_FOLD, 256-column tiles).
@@ -1314,17 +1375,18 @@ cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_
   a.fcb = cb; a.fN = N; a.slot_of_group = slot_of_group;
   a.fd_khw = FastDiv((uint32_t)khw); a.fd_w = FastDiv((uint32_t)W); a.fd_kw = FastDiv((uint32_t)kw);
   a.fd_hw = FastDiv((uint32_t)(H * W)); a.fd_s = FastDiv((uint32_t)stride); a.fd_cbhw = FastDiv((uint32_t)(cb * H * W));
+  // codes < 16 (b <= 4) go to the tensor cores straight from TMA (A_DIRECT)
   if (Bte) {  // the e4m3 B path writes NCHW only
     if (nhwc) return cudaErrorNotSupported;
     if (bits == 8) return launch_tc<true, true, 128, true, 2>(ma, mb, a, 1, s);
-    return launch_tc<true, false, 128, true, 2>(ma, mb, a, 1, s);
+    return launch_tc<true, false, 128, true, 2 | 8>(ma, mb, a, 1, s);
   }
   if (nhwc) {
     if (bits == 8) return launch_tc<true, true, 128, true, 4>(ma, mb, a, 1, s);
-    return launch_tc<true, false, 128, true, 4>(ma, mb, a, 1, s);
+    return launch_tc<true, false, 128, true, 4 | 8>(ma, mb, a, 1, s);
   }
   if (bits == 8) return launch_tc<true, true, 128, true>(ma, mb, a, 1, s);
-  return launch_tc<true, false, 128, true>(ma, mb, a, 1, s);
+  return launch_tc<true, false, 128, true, 8>(ma, mb, a, 1, s);
 }
 
 // Clusters of `cs` CTAs of this kernel that fit on the GPU at once (0 if unknown).
@@ -1338,7 +1400,7 @@ static int max_active_clusters(int cs) {
   if (cs < 1 || cs > 8 || cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
   const int known = cache[dev][cs].load(std::memory_order_acquire);
   if (known > 0) return known - 1;
-  auto kern = tc_gemm_kernel<true, BITS8, 128, false>;
+  auto kern = tc_gemm_kernel<true, BITS8, 128, false, BITS8 ? 0 : 8>;  // the kernel launch_wgrad_cluster_tc runs
   if (smem_attr_once((const void*)kern, S::kBytes, attr_bits) != cudaSuccess) return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(1, 1, (unsigned)cs);
@@ -1388,7 +1450,7 @@ cudaError_t launch_wgrad_cluster_tc(int bits, const uint8_t* Q, int64_t ldq, int
   a.epi = EPI_CRED; a.acc = acc; a.y = dw; a.ldo = K; a.kept_idx = kept_idx; a.scale = scale; a.zero = zero;
   a.cs = cs; a.status = status; a.slot_of_group = slot_of_group; a.D = D;
   if (bits == 8) return launch_tc<true, true, 128>(ma, mb, a, splits, s, nullptr, nullptr, true);
-  return launch_tc<true, false, 128>(ma, mb, a, splits, s, nullptr, nullptr, true);
+  return launch_tc<true, false, 128, false, 8>(ma, mb, a, splits, s, nullptr, nullptr, true);
 }
 
 cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,

@@ -418,11 +418,16 @@ __global__ void __launch_bounds__(NT) select_kernel(SelectArgs a0, SelectArgs a1
   uint64_t ktot;
   const uint64_t kincl = block_inclusive_scan<NT>((uint64_t)nk, warp_sums, &ktot);
   int slot = (int)(kincl - nk);
+  // Finite gradients never keep more than `capacity` groups (systematic: floor or ceil of
+  // sum p^ <= n / b; top-k: n / b; Bernoulli and b = 1: capacity = n).  A non-finite range
+  // (flagged by the range pass) breaks the fixed-point arithmetic above, so the kept list is
+  // cut at the capacity here: no later kernel reads or writes past the caller's buffers.
+  const int kcap = (int)min(ktot, (uint64_t)a.capacity);
   // the per-slot scale and zero point are computed by the quantize kernel
   for (int i = beg; i < end; ++i) {
     const uint64_t P = key[i];
     o.p_hat[i] = p_hat_of(P);
-    if (kept_bits & (1ull << (i - beg))) {
+    if ((kept_bits & (1ull << (i - beg))) && slot < kcap) {
       o.slot_of_group[i] = slot;
       o.kept_idx[slot] = i;
       ++slot;
@@ -430,8 +435,8 @@ __global__ void __launch_bounds__(NT) select_kernel(SelectArgs a0, SelectArgs a1
       o.slot_of_group[i] = -1;
     }
   }
-  for (int s = (int)ktot + tid; s < a.capacity; s += NT) o.kept_idx[s] = -1;
-  if (tid == 0) *o.kept_count = (int32_t)ktot;
+  for (int s = kcap + tid; s < a.capacity; s += NT) o.kept_idx[s] = -1;
+  if (tid == 0) *o.kept_count = (int32_t)kcap;
 }
 
 // --------------------------------------------------------------- quantize

@@ -46,6 +46,7 @@ _SIGS = {
     "fqt1_im2col": (C.c_int, [_VP] + [_I32] * 8 + [_VP, _VP, _VP, _VP]),
     "fqt1_fwd_gemm": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
     "fqt1_fwd_gemm_bias": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP, _VP]),
+    "fqt1_test_expired_wait": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
     "fqt1_scale_bias_workspace": (C.c_size_t, [_I64, _I64]),
     "fqt1_scale_bias_grad": (C.c_int, [_VP, _VP, _I64, _I64, _VP, _VP, _VP, C.c_size_t, _VP]),
     "fqt1_ste_clip": (C.c_int, [_VP, _VP, _I64, C.c_float, _VP]),
@@ -158,6 +159,11 @@ def binarize_pack(x, rows, cols, ld, row_bits=None, col_bits=None, colsum=None, 
 def im2col(x, N, Cin, H, W, kh, kw, stride, pad, row_bits=None, col_bits=None, colsum=None, stream=None):
     _check(lib().fqt1_im2col(_p(x), N, Cin, H, W, kh, kw, stride, pad, _p(row_bits), _p(col_bits), _p(colsum),
                              _s(stream)), "fqt1_im2col")
+
+
+def test_expired_wait(sx_row, sw_row, M, D, K, gamma, y, dev_status, stream=None):
+    _check(lib().fqt1_test_expired_wait(_p(sx_row), _p(sw_row), M, D, K, _p(gamma), _p(y), _p(dev_status),
+                                        _s(stream)), "fqt1_test_expired_wait")
 
 
 def fwd_gemm(sx_row, sw_row, M, D, K, gamma, acc, y, stream=None):

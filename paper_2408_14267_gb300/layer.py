@@ -37,10 +37,15 @@ class LayerStep:
         self.keep_acc = keep_acc
         f32 = dict(dtype=torch.float32, device=dev)
         i32 = dict(dtype=torch.int32, device=dev)
-        self.x = torch.as_tensor(np.ascontiguousarray(wl["x"]), **f32)
-        self.w = torch.as_tensor(np.ascontiguousarray(wl["w"]), **f32)
-        self.gamma = None if wl.get("gamma") is None else torch.as_tensor(wl["gamma"], **f32)
-        self.gy = torch.as_tensor(np.ascontiguousarray(wl["gy"]), **f32)
+        def dev_tensor(a):  # host arrays are copied in; device tensors are taken as they are
+            if isinstance(a, torch.Tensor):
+                return a.to(**f32).contiguous()
+            return torch.as_tensor(np.ascontiguousarray(a), **f32)
+
+        self.x = dev_tensor(wl["x"])
+        self.w = dev_tensor(wl["w"])
+        self.gamma = None if wl.get("gamma") is None else dev_tensor(wl["gamma"])
+        self.gy = dev_tensor(wl["gy"])
         if self.kind == "conv":
             N, Cin, H, W = self.x.shape
             D, _, kh, kw = self.w.shape

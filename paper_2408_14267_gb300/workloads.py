@@ -123,3 +123,22 @@ def sweep_point(M, K, D, groups, bits, seed=1004, qseed=0xF075):
     gy = (rng.laplace(0.0, 1e-3, size=(groups, M // groups, D)) * s).reshape(M, D).astype(np.float32)
     return dict(name=f"sweep M{M} K{K} D{D} G{groups} b{bits}", kind="linear", x=x, w=w,
                 gamma=np.ones(D, dtype=np.float32), gy=gy, rows_per_group=M // groups, **_agp(bits, bits, qseed))
+
+
+def sweep_point_device(M, K, D, groups, bits, device, seed=1004, qseed=0xF075):
+    """The sweep recipe of `sweep_point`, drawn on the device with torch's generator (the large
+    points do not fit a host draw in reasonable time): X, W ~ N(0,1), gY = Laplace(0, 1e-3) x
+    10^U(-2,2) per group of M/groups rows, Gamma = 1.  Timing only: parity tests draw their
+    sweep points with `sweep_point` so that the oracle sees the same numbers."""
+    import torch
+    g = torch.Generator(device=device).manual_seed(seed)
+    x = torch.randn(M, K, generator=g, device=device)
+    w = torch.randn(D, K, generator=g, device=device)
+    # u strictly inside (-1/2, 1/2): rand() can return 0, and u = -1/2 would give -inf
+    u = torch.rand(M, D, generator=g, device=device) + (0.5 * 2.0 ** -24 - 0.5)
+    lap = -1e-3 * torch.sign(u) * torch.log1p(-2.0 * u.abs())
+    s = 10.0 ** (torch.rand(groups, 1, 1, generator=g, device=device) * 4.0 - 2.0)
+    gy = (lap.view(groups, M // groups, D) * s).view(M, D).contiguous()
+    return dict(name=f"sweep M{M} K{K} D{D} G{groups} b{bits}", kind="linear", x=x, w=w,
+                gamma=torch.ones(D, device=device), gy=gy, rows_per_group=M // groups, **_agp(bits, bits, qseed))
+

@@ -483,6 +483,28 @@ def test_nonfinite_gradient_sets_status():
     assert int(st.dev_status[0].item()) & 0x100
 
 
+@pytest.mark.parametrize("val", [float("-inf"), float("inf")])
+def test_infinite_gradient_stays_in_bounds(val):
+    """An infinite gradient value gives an infinite range, which breaks the fixed-point keep
+    probabilities (every group would be kept).  The step must still flag the input, keep at
+    most `capacity` groups per branch, and keep every kept id and slot in range."""
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = linear_case(64, 64, 64, 1, 4, SYS, seed=12)
+    w["gy"][5, 3] = val
+    st = LayerStep(w)
+    st.dev_status.zero_()
+    st.step()
+    torch.cuda.synchronize()
+    assert int(st.dev_status[0].item()) & 0x100
+    for q in (st.psq, st.pcq):
+        cnt = q.count()
+        assert 0 <= cnt <= q.capacity
+        kid = q.kept_idx.cpu().numpy()
+        assert np.all((kid[:cnt] >= 0) & (kid[:cnt] < q.n)) and np.all(kid[cnt:q.capacity] == -1)
+        slots = q.slot_of_group.cpu().numpy()
+        assert np.all((slots >= -1) & (slots < cnt))
+
+
 @pytest.mark.parametrize("rows,cols,ld", [(77, 300, 304), (40, 128, 132), (3, 4, 8), (64, 256, 256), (33, 100, 103),
                                           (70, 45, 45)])
 def test_binarize_pack_strided(rows, cols, ld):
