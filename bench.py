@@ -318,7 +318,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--implicit", action="store_true",
                     help="implicit-GEMM forward (pixel-major sign(X), no unfolded row packing)")
-    ap.add_argument("--e4m3-weights", choices=["on", "off"], default="off",
+    ap.add_argument("--e4m3-weights", choices=["on", "off"], default="on",
                     help="e4m3 copies of sign(W) written by the weight packing and loaded by TMA as the "
                          "B operand of the forward and grad_input products")
     ap.add_argument("--profile", type=int, default=0, metavar="N",
@@ -371,8 +371,12 @@ def main():
                    e4m3_weights=args.e4m3_weights == "on")
     stream = torch.cuda.Stream()
     if args.profile:
+        # eager steps, each after an L2 flush as in the timed loop (with ncu --cache-control none
+        # the counters then show the step's own DRAM traffic)
+        flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device="cuda")
         with torch.cuda.stream(stream):
             for _ in range(args.warmup + args.profile):
+                flush.zero_()
                 st.step()
         torch.cuda.synchronize()
         return
@@ -704,8 +708,9 @@ def gemm_sweep(args):
                NUMEXPR_NUM_THREADS="1")
     for (M, K, D, G, b) in sweep_points(args.sweep):
         wl = workloads.sweep_point_device(M, K, D, G, b, dev)
-        st = LayerStep(wl, device=dev, keep_acc=False)
+        st = LayerStep(wl, device=dev, keep_acc=False, e4m3_weights=args.e4m3_weights == "on")
         del wl
+        torch.cuda.synchronize()  # the inputs are drawn on the default stream; the step runs on `stream`
         with torch.cuda.stream(stream):
             st.dev_status.zero_()
             for _ in range(3):
