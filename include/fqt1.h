@@ -160,6 +160,23 @@ fqt1_status fqt1_conv_fwd_implicit(const uint32_t* x_pix, const uint32_t* w_taps
                                    int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad, int64_t D,
                                    const float* gamma, const float* bias, int32_t* acc, float* y, void* stream);
 
+/* Sign planes of a contiguous x (App. C Unfolder, in two passes).
+ * fqt1_pack_planes: x [N, C, H, W] fp32 (contiguous, 16-byte aligned) -> planes
+ *   [N][C][ceil(H W / 32)] words: bit e of word q of plane (n, c) is set iff
+ *   x[n, c, pixel 32 q + e] > 0 (pixel = h W + w), bits past H W clear; the
+ *   layout fqt1_pack_planes_nhwc writes and fqt1_im2col_planes reads.  One
+ *   streaming pass over x.
+ * fqt1_im2col_path: how fqt1_im2col serves the shape.  2: tiles of whole images
+ *   (stride-1 "same" convolutions whose H W divides 128 or is 256), one pass over
+ *   x.  1: tiles of up to 128 output pixels, each reading its input region; then
+ *   fqt1_pack_planes followed by fqt1_im2col_planes gives the same outputs from
+ *   32 times fewer bytes.  0: a per-element gather (regions too large; x must be
+ *   given).  -1: invalid shape. */
+fqt1_status fqt1_pack_planes(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, uint32_t* planes,
+                             void* stream);
+int32_t fqt1_im2col_path(int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,
+                         int32_t pad);
+
 /* Channels-last inputs (no counterpart in the paper; the layout of x only).
  * fqt1_pack_planes_nhwc: x with memory order N, H, W, C (a channels-last
  *   [N, C, H, W] tensor), C a multiple of 32 -> planes [N][C][ceil(H W / 32)]

@@ -357,18 +357,33 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
   if (a.planes) {
     // the signs are given as plane bits: word q of a region plane is the 32 bits from bit
     // h_lo W + 32 q of the full plane (a funnel shift of two words), zero past its rows
+    // 8 region words per thread per batch, their 16 loads in flight together (unconditional,
+    // from clamped indices)
     const int total = nplanes * data_words, bit0 = h_lo * a.W;
     const FastDiv div_dw((uint32_t)max(data_words, 1)), div_nc((uint32_t)nc);
-    for (int f = threadIdx.x; f < total; f += 256) {
-      const int pl = (int)div_dw.div((uint32_t)f), q = f - pl * data_words;
-      const int nn = (int)div_nc.div((uint32_t)pl), c = pl - nn * nc;
-      const uint32_t* src = a.planes + ((int64_t)(n_lo + nn) * a.C + c_lo + c) * a.pw;
-      const int b = bit0 + 32 * q, w0 = b >> 5;
-      const uint32_t lo = __ldg(src + min(w0, a.pw - 1)), hi = __ldg(src + min(w0 + 1, a.pw - 1));
-      uint32_t word = __funnelshift_r(lo, hi, b & 31);
-      const int left = plane_bits - 32 * q;
-      if (left < 32) word &= left <= 0 ? 0u : ((1u << left) - 1u);
-      stream[pl * plane_words + a.guard + q] = word;
+    for (int f0 = threadIdx.x; f0 < total; f0 += 256 * 8) {
+      uint32_t lo[8], hi[8];
+      int pos[8], sh[8], left[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int f = min(f0 + 256 * u, total - 1);
+        const int pl = (int)div_dw.div((uint32_t)f), q = f - pl * data_words;
+        const int nn = (int)div_nc.div((uint32_t)pl), c = pl - nn * nc;
+        const uint32_t* src = a.planes + ((int64_t)(n_lo + nn) * a.C + c_lo + c) * a.pw;
+        const int b = bit0 + 32 * q, w0 = b >> 5;
+        lo[u] = __ldg(src + min(w0, a.pw - 1));
+        hi[u] = __ldg(src + min(w0 + 1, a.pw - 1));
+        pos[u] = pl * plane_words + a.guard + q;
+        sh[u] = b & 31;
+        left[u] = plane_bits - 32 * q;
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        if (f0 + 256 * u >= total) break;
+        uint32_t word = __funnelshift_r(lo[u], hi[u], sh[u]);
+        if (left[u] < 32) word &= left[u] <= 0 ? 0u : ((1u << left[u]) - 1u);
+        stream[pos[u]] = word;
+      }
     }
   } else {
     const int total = nplanes * data_words;
@@ -852,6 +867,33 @@ __global__ void __launch_bounds__(256) pack_planes_nhwc_kernel(const float* __re
     planes[(n * C + 32 * cb + lane) * pw + q] = pwd;
   }
 }
+// Sign bits of a contiguous [N, C, H, W] x as channel planes [N C][pw] words, pw = ceil(H W / 32):
+// bit e of word q of plane p is x[p H W + 32 q + e] > 0, bits past H W clear.  A warp takes 8
+// consecutive words of one plane and has its 8 coalesced 128-byte loads in flight together; a
+// word is the ballot of its 32 floats.
+__global__ void __launch_bounds__(256) pack_planes_nchw_kernel(const float* __restrict__ x, int64_t planes_n, int HW,
+                                                               int pw, uint32_t* __restrict__ planes) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int blocks = (pw + 7) / 8;
+  const int64_t units = planes_n * blocks;
+  for (int64_t u = (int64_t)blockIdx.x * 8 + warp; u < units; u += (int64_t)gridDim.x * 8) {  // warp-uniform
+    const int64_t pl = u / blocks;
+    const int q0 = 8 * (int)(u - pl * blocks);
+    const float* src = x + pl * HW;
+    float v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = __ldg(src + min(32 * (q0 + k) + lane, HW - 1));
+    uint32_t mine = 0u;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const uint32_t wd = __ballot_sync(0xFFFFFFFFu, v[k] > 0.0f && 32 * (q0 + k) + lane < HW);
+      if (lane == k) mine = wd;
+    }
+    if (lane < 8 && q0 + lane < pw) planes[pl * pw + q0 + lane] = mine;
+  }
+}
 }  // namespace fqt1
 
 using namespace fqt1;
@@ -889,6 +931,41 @@ extern "C" fqt1_status fqt1_binarize_pack(const float* x, int64_t rows, int64_t 
   return FQT1_OK;
 }
 
+// Whether the whole-image Unfolder (unfold_same_kernel) serves the shape: a stride-1 "same"
+// convolution whose tiles hold whole images (H W divides 128, or is 256), with its region and
+// guards in 32 KB of shared memory.
+static bool unfold_same_fits(int N, int C, int H, int W, int kh, int kw, int stride, int pad) {
+  const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
+  const int64_t Ki = (int64_t)C * kh * kw;
+  const bool same = stride == 1 && kh == kw && kh == 2 * pad + 1 && (Ho * Wo) % 32 == 0;
+  if (!(same && pad <= 32 && Ki < (1ll << 31) && (128 % (H * W) == 0 || H * W == 256))) return false;
+  const int dw = H * W / 32, nsub = H * W == 256 ? 8 : 4, ipt = 32 * nsub / (H * W);
+  const int guard = (pad * W + pad + 63) / 32;
+  const int64_t nc_max = std::min<int64_t>(C, 256 / (kh * kw) + 2);
+  const size_t smem = (size_t)(2 * guard + ipt * nc_max * dw) * 4;
+  const int64_t row_tiles = (N + ipt - 1) / ipt;
+  return row_tiles <= 65535 && smem <= 32 * 1024;
+}
+
+// Pixels per tile of the region Unfolder (unfold_bits_kernel): the largest of 128, 64, 32 whose
+// input region bound (images a tile may touch x channels of 256 columns x whole planes with
+// guards) fits kUnfoldMaxStreamWords, with at most 65535 row tiles; 0 if none (gather path).
+static int unfold_bits_tm(int N, int C, int H, int W, int kh, int kw, int stride, int pad) {
+  const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
+  const int64_t Mi = (int64_t)N * Ho * Wo, Ki = (int64_t)C * kh * kw;
+  if (!(pad <= 32 && Ki < (1ll << 31))) return 0;
+  const bool same = stride == 1 && kh == kw && kh == 2 * pad + 1 && (Ho * Wo) % 32 == 0;
+  const int guard = same ? (pad * W + pad + 63) / 32 : 1;
+  for (int tm = 128; tm >= 32; tm /= 2) {
+    const int64_t imgs = std::min<int64_t>(N, tm / (Ho * Wo) + 2);
+    const int64_t chans = std::min<int64_t>(C, 256 / (kh * kw) + 2);
+    const int64_t words = imgs * chans * (((int64_t)H * W + 31) / 32 + 2 * guard);
+    if (words > kUnfoldMaxStreamWords) continue;
+    return (Mi + tm - 1) / tm > 65535 ? 0 : tm;
+  }
+  return 0;
+}
+
 // The Unfolder of fqt1_im2col (x given) and of fqt1_im2col_planes (planes given: the sign bits of x
 // as [N][C][ceil(H W / 32)] words; shapes that only the gather path serves are unsupported there).
 static fqt1_status im2col_impl(const float* x, const uint32_t* planes, int32_t N, int32_t C, int32_t H, int32_t W,
@@ -908,7 +985,7 @@ static fqt1_status im2col_impl(const float* x, const uint32_t* planes, int32_t N
   // region of a tile of tm pixels: images it may touch x channels of 256 columns x whole planes.
   const int64_t Mi = (int64_t)N * Ho * Wo, Ki = (int64_t)C * kh * kw;
   const bool same = stride == 1 && kh == kw && kh == 2 * pad + 1 && (Ho * Wo) % 32 == 0;
-  if (same && pad <= 32 && Ki < (1ll << 31) && (128 % (H * W) == 0 || H * W == 256)) {
+  if (unfold_same_fits(N, C, H, W, kh, kw, stride, pad)) {
     // whole images per tile: the contiguous-region Unfolder
     UnfoldSameArgs u;
     u.x = x; u.planes = planes; u.row_bits = row_bits; u.col_bits = col_bits; u.colsum = colsum;
@@ -942,17 +1019,15 @@ static fqt1_status im2col_impl(const float* x, const uint32_t* planes, int32_t N
       return FQT1_OK;
     }
   }
-  if (pad <= 32 && Ki < (1ll << 31)) {
+  if (const int tm = unfold_bits_tm(N, C, H, W, kh, kw, stride, pad)) {
     // 128-pixel tiles (smaller only when the input region does not fit): fewer CTAs, each
     // amortizing its region set-up over more output words
-    const int tm_first = 128;
     // the fast path reads a 32-bit window up to pad W + pad bits before or after the plane
     const int guard = same ? (pad * W + pad + 63) / 32 : 1;
-    for (int tm = tm_first; tm >= 32; tm /= 2) {
+    {
       const int64_t imgs = std::min<int64_t>(N, tm / (Ho * Wo) + 2);
       const int64_t chans = std::min<int64_t>(C, 256 / (kh * kw) + 2);
       const int64_t words = imgs * chans * (((int64_t)H * W + 31) / 32 + 2 * guard);
-      if (words > kUnfoldMaxStreamWords) continue;
       UnfoldArgs u;
       u.x = x; u.planes = planes; u.pw = (H * W + 31) / 32;
       u.row_bits = row_bits; u.col_bits = col_bits; u.colsum = colsum;
@@ -963,7 +1038,6 @@ static fqt1_status im2col_impl(const float* x, const uint32_t* planes, int32_t N
       u.div_khw = FastDiv((uint32_t)(kh * kw)); u.div_kw = FastDiv((uint32_t)kw);
       u.div_hwo = FastDiv((uint32_t)(Ho * Wo)); u.div_wo = FastDiv((uint32_t)Wo);
       const int64_t row_tiles = (Mi + tm - 1) / tm, word_tiles = (u.row_words + 7) / 8;
-      if (row_tiles > 65535) break;
       static std::atomic<uint64_t> attr{0};
       FQT1_CUDA_TRY(smem_attr_once((const void*)unfold_bits_kernel, kUnfoldMaxStreamWords * 4, attr));
       if (colsum) FQT1_CUDA_TRY(cudaMemsetAsync(colsum, 0, sizeof(int32_t) * Ki, s));
@@ -1083,6 +1157,27 @@ extern "C" fqt1_status fqt1_im2col_planes(const uint32_t* planes, int32_t N, int
                                           uint32_t* col_bits, int32_t* colsum, void* stream) {
   if (!planes) return FQT1_ERR_INVALID_ARG;
   return im2col_impl(nullptr, planes, N, C, H, W, kh, kw, stride, pad, row_bits, col_bits, colsum, stream);
+}
+
+extern "C" fqt1_status fqt1_pack_planes(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, uint32_t* planes,
+                                        void* stream) {
+  if (!x || !planes || N < 1 || C < 1 || H < 1 || W < 1) return FQT1_ERR_INVALID_ARG;
+  if ((int64_t)N * C * H * W >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
+  const int pw = (H * W + 31) / 32;
+  const int64_t units = (int64_t)N * C * ((pw + 7) / 8);
+  const unsigned blocks = (unsigned)std::min<int64_t>((units + 7) / 8, 152 * 16);
+  FQT1_CUDA_TRY(launch_k(pack_planes_nchw_kernel, dim3(blocks), dim3(256), 0, (cudaStream_t)stream, x,
+                         (int64_t)N * C, H * W, pw, planes));
+  fqt1_count_launches(1);
+  return FQT1_OK;
+}
+
+extern "C" int32_t fqt1_im2col_path(int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw,
+                                    int32_t stride, int32_t pad) {
+  if (N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 || pad < 0) return -1;
+  if (H + 2 * pad < kh || W + 2 * pad < kw) return -1;
+  if (unfold_same_fits(N, C, H, W, kh, kw, stride, pad)) return 2;
+  return unfold_bits_tm(N, C, H, W, kh, kw, stride, pad) ? 1 : 0;
 }
 
 extern "C" fqt1_status fqt1_pack_planes_nhwc(const float* x, int32_t N, int32_t C, int32_t H, int32_t W,

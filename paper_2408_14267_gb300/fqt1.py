@@ -58,6 +58,8 @@ _SIGS = {
     "fqt1_bwd_input_fold_e4m3w": (C.c_int, [_VP, _VP, _I64, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP]),
     "fqt1_pack_pixels": (C.c_int, [_VP, _I32, _I32, _I32, _I32, _VP, _VP]),
     "fqt1_pack_planes_nhwc": (C.c_int, [_VP, _I32, _I32, _I32, _I32, _VP, _VP]),
+    "fqt1_pack_planes": (C.c_int, [_VP, _I32, _I32, _I32, _I32, _VP, _VP]),
+    "fqt1_im2col_path": (_I32, [_I32] * 8),
     "fqt1_im2col_planes": (C.c_int, [_VP] + [_I32] * 8 + [_VP, _VP, _VP, _VP]),
     "fqt1_pack_weight_taps": (C.c_int, [_VP, _I64, _I32, _I32, _I32, _VP, _VP]),
     "fqt1_conv_implicit_supported": (_I32, [_I32] * 8),
@@ -196,6 +198,15 @@ def bwd_input_fold_e4m3w(psq, wt_e4m3, colsum_w, N, Cin, H, W, kh, kw, stride, p
 
 def plane_words(H, W):
     return (H * W + 31) // 32
+
+
+def pack_planes(x, N, Cin, H, W, planes, stream=None):
+    _check(lib().fqt1_pack_planes(_p(x), N, Cin, H, W, _p(planes), _s(stream)), "fqt1_pack_planes")
+
+
+def im2col_path(N, Cin, H, W, kh, kw, stride, pad):
+    """2: whole-image tiles from x; 1: region tiles (planes first read 32x fewer bytes); 0: gather."""
+    return lib().fqt1_im2col_path(N, Cin, H, W, kh, kw, stride, pad)
 
 
 def pack_planes_nhwc(x, N, Cin, H, W, planes, stream=None):

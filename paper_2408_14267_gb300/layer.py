@@ -74,6 +74,12 @@ class LayerStep:
         else:
             self.implicit = False
         wK, wM, wD = fqt1.packed_words(K), fqt1.packed_words(M), fqt1.packed_words(D)
+        # shapes whose Unfolder reads an input region per tile: sign-pack x into planes first
+        # (one streaming pass), so that the regions are read as bits
+        self.x_planes = None
+        if self.kind == "conv" and not self.implicit and fqt1.im2col_path(N, Cin, H, W, kh, kw, self.stride,
+                                                                          self.pad) == 1:
+            self.x_planes = torch.empty(N * Cin * fqt1.plane_words(H, W), **i32)
         if self.implicit:
             self.x_pix = torch.empty(N * H * W, fqt1.packed_words(Cin), **i32)
             self.w_taps = torch.empty(D, wK, **i32)
@@ -145,7 +151,15 @@ class LayerStep:
                     fqt1.binarize_pack(self.w, self.D, self.K, self.K, self.sw_row, self.sw_col, self.cs_w, s)
 
             st = [("pack_w", pack_w)]
-            if self.kind == "conv":
+            if self.kind == "conv" and self.x_planes is not None:
+                N, Cin, H, W, kh, kw = self.conv
+
+                def unfold(s):
+                    fqt1.pack_planes(self.x, N, Cin, H, W, self.x_planes, s)
+                    fqt1.im2col_planes(self.x_planes, N, Cin, H, W, kh, kw, self.stride, self.pad, self.sx_row,
+                                       self.sx_col, self.cs_x, s)
+                st.append(("im2col", unfold))
+            elif self.kind == "conv":
                 N, Cin, H, W, kh, kw = self.conv
                 st.append(("im2col", lambda s: fqt1.im2col(self.x, N, Cin, H, W, kh, kw, self.stride, self.pad,
                                                            self.sx_row, self.sx_col, self.cs_x, s)))

@@ -643,6 +643,58 @@ def test_im2col_from_channels_last_planes(N, C, H, W, k, s, p):
         assert torch.equal(a, b)
 
 
+@pytest.mark.parametrize("N,C,H,W,k,s,p", [(2, 3, 30, 30, 7, 2, 3), (2, 64, 28, 28, 1, 2, 0), (3, 16, 14, 14, 3, 2, 1),
+                                           (2, 5, 13, 11, 3, 1, 1), (1, 32, 56, 56, 3, 1, 1), (4, 8, 9, 7, 1, 1, 0)])
+def test_pack_planes_nchw_and_unfold_from_planes(N, C, H, W, k, s, p):
+    """Contiguous x: fqt1_pack_planes writes the signs of x as channel planes (any C, H W not a
+    multiple of 32, bits past H W clear), and the Unfolder reading those planes writes the same
+    rows, columns and column sums as the Unfolder reading x (the region-tile shapes of the
+    ResNet-18 stem and downsamples among them)."""
+    from paper_2408_14267_gb300 import fqt1
+    rng = np.random.default_rng(N * C + H * 3 + k)
+    x = rng.standard_normal((N, C, H, W)).astype(np.float32)
+    x[0, 0, 0, :3] = 0.0
+    xt = torch.from_numpy(x).cuda()
+    pw = fqt1.plane_words(H, W)
+    planes = torch.full((N * C * pw,), -1, dtype=torch.int32, device="cuda")
+    fqt1.pack_planes(xt, N, C, H, W, planes)
+    Ho, Wo = om.conv_out_hw(H, W, k, k, s, p)
+    M, K = N * Ho * Wo, C * k * k
+    path = fqt1.im2col_path(N, C, H, W, k, k, s, p)
+    assert path in (1, 2)
+    outs = []
+    for use_planes in (False, True):
+        rb = torch.full((M, fqt1.packed_words(K)), 7, dtype=torch.int32, device="cuda")
+        cbits = torch.full((K, fqt1.packed_words(M)), 7, dtype=torch.int32, device="cuda")
+        cs = torch.empty(K, dtype=torch.int32, device="cuda")
+        if use_planes:
+            fqt1.im2col_planes(planes, N, C, H, W, k, k, s, p, rb, cbits, cs)
+        else:
+            fqt1.im2col(xt, N, C, H, W, k, k, s, p, rb, cbits, cs)
+        outs.append((rb, cbits, cs))
+    torch.cuda.synchronize()
+    w = planes.cpu().numpy().view(np.uint32).reshape(N, C, pw)
+    bits = ((w[:, :, :, None] >> np.arange(32, dtype=np.uint32)) & 1).reshape(N, C, -1)
+    assert np.array_equal(bits[:, :, :H * W].astype(np.int8) * 2 - 1, om.sign(x).reshape(N, C, H * W))
+    assert not bits[:, :, H * W:].any()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+    # and both against the oracle's unfolded signs
+    su, pad = unpack_bits(outs[1][0], K)
+    assert np.array_equal(su, om.sign(om.unfold(x, k, k, s, p))) and not pad.any()
+
+
+def test_im2col_path_query():
+    """fqt1_im2col_path: whole-image tiles for the bench layer, region tiles for the ResNet-18
+    ImageNet stem and downsamples, the gather for regions too large, -1 for invalid shapes."""
+    from paper_2408_14267_gb300 import fqt1
+    assert fqt1.im2col_path(128, 256, 8, 8, 3, 3, 1, 1) == 2
+    assert fqt1.im2col_path(64, 3, 224, 224, 7, 7, 2, 3) == 1
+    assert fqt1.im2col_path(64, 64, 56, 56, 1, 1, 2, 0) == 1
+    assert fqt1.im2col_path(2, 256, 56, 56, 1, 1, 1, 0) == 0
+    assert fqt1.im2col_path(2, 4, 3, 3, 7, 7, 1, 0) == -1
+
+
 def test_im2col_planes_rejects_gather_shapes():
     """Shapes served only by the gather Unfolder (which reads x itself) are unsupported from planes."""
     from paper_2408_14267_gb300 import fqt1
