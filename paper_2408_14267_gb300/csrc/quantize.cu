@@ -7,6 +7,7 @@
 //   quantize_kernel  second read of G: stochastic rounding of the kept sample
 //                    groups (PSQ codes, row-major) and kept channels (PCQ codes,
 //                    written transposed through shared memory).
+#include <algorithm>
 #include <mutex>
 #include <stdio.h>
 
@@ -15,7 +16,18 @@
 namespace fqt1 {
 
 // ------------------------------------------------------------------ ranges
-constexpr int kRangeRows = 32, kRangeCols = 128;  // 8 warps x 4 rows x (32 lanes x 4 columns)
+constexpr int kRangeLoads = 4;  // float4 loads per thread per chunk
+
+// Lane layout of the range pass: LPR lanes of 4 columns each span the CTA's column tile and a
+// warp-wide load covers 32 / LPR rows.  The narrow layouts (LPR 16 or 8) keep every lane busy
+// when D <= 64, where the full-width one would leave half or three quarters of them idle.
+template <int LPR>
+struct RangeShape {
+  static constexpr int kRW = 32 / LPR;              // rows of one warp-wide load
+  static constexpr int kChunk = kRangeLoads * kRW;  // rows of one warp per row tile
+  static constexpr int kTile = 8 * kChunk;          // rows of one CTA per row tile
+  static constexpr int kCols = 4 * LPR;             // columns of one CTA
+};
 
 struct RangeArgs {
   const float* g;
@@ -37,14 +49,112 @@ __device__ __forceinline__ T ldg_sel(const T* p, int64_t i, bool ok, T dflt, con
   return ok ? v : dflt;
 }
 
-template <bool VEC>
+// One chunk of a lane: rows r, r + kRW, ... (clamped to the last row, so every address is valid)
+// and columns c0 .. c0 + 3 (clamped likewise; the caller masks what lies outside G).
+template <int LPR, bool VEC>
+__device__ __forceinline__ void range_load(const RangeArgs& a, int64_t r, int64_t c0, bool cv0,
+                                           float (&v)[kRangeLoads][4]) {
+#pragma unroll
+  for (int i = 0; i < kRangeLoads; ++i) {
+    const int64_t ri = min(r + i * RangeShape<LPR>::kRW, a.M - 1);
+    if (VEC) {
+      const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + ri * a.D + (cv0 ? c0 : 0)));
+      v[i][0] = t.x; v[i][1] = t.y; v[i][2] = t.z; v[i][3] = t.w;
+    } else {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) v[i][q] = __ldg(a.g + ri * a.D + min(c0 + q, a.D - 1));
+    }
+  }
+}
+
+// The range pass is bound by instructions and load latency per element, not by memory, so its
+// loop is lean: float minima / maxima per thread (ordered integer keys only for the atomics),
+// one finite test per element, the Gamma product only when there is a Gamma (the loop exists
+// in both forms), and the sample-group bookkeeping once per chunk of a warp when the chunk lies
+// in one group (the usual case: a group is a whole sample).  rc is the chunk's first row
+// (warp-uniform), sub the lane's row within a warp-wide load.
+template <int LPR, bool GAMMA>
+__device__ __forceinline__ void range_chunk(const RangeArgs& a, int64_t rc, int sub, const bool (&cv)[4],
+                                            const float (&gam)[4], const float (&v)[kRangeLoads][4],
+                                            float (&cmn)[4], float (&cmx)[4], float& gmn, float& gmx,
+                                            int64_t& cur, bool& bad, int lane) {
+  using S = RangeShape<LPR>;
+  const int nrows = (int)min((int64_t)S::kChunk, a.M - rc);  // >= 1
+  const int64_t g0 = a.div_rpg.div((uint32_t)rc), g1 = a.div_rpg.div((uint32_t)(rc + nrows - 1));
+  auto flush = [&](int64_t next) {  // the warp's group minimum / maximum, when its rows move on
+    if (a.smin && next != cur) {
+      if (cur >= 0) {
+        const uint32_t mn = __reduce_min_sync(0xFFFFFFFFu, float_to_ordered(gmn));
+        const uint32_t mx = __reduce_max_sync(0xFFFFFFFFu, float_to_ordered(gmx));
+        if (lane == 0) { atomicMin(a.smin + cur, mn); atomicMin(a.smax + cur, ~mx); }
+      }
+      cur = next;
+      gmn = __int_as_float(0x7F800000);   // +inf
+      gmx = __int_as_float(0xFF800000);   // -inf
+    }
+  };
+  auto take = [&](float g, int q) {
+    const float x = GAMMA ? __fmul_rn(g, gam[q]) : g;
+    bad |= !(fabsf(x) <= 3.402823466e38f);  // NaN or +-Inf
+    cmn[q] = fminf(cmn[q], x); cmx[q] = fmaxf(cmx[q], x);
+    return x;
+  };
+  if (g0 == g1) {
+    flush(g0);
+#pragma unroll
+    for (int i = 0; i < kRangeLoads; ++i) {
+      const bool rv = i * S::kRW + sub < nrows;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        if (!cv[q] || !rv) continue;
+        const float x = take(v[i][q], q);
+        gmn = fminf(gmn, x); gmx = fmaxf(gmx, x);
+      }
+    }
+  } else if (LPR == 32) {  // one row per load: the warp follows the group boundary row by row
+    int64_t gi = g0, grem = rc - g0 * a.rpg;
+#pragma unroll
+    for (int i = 0; i < kRangeLoads; ++i) {
+      if (i >= nrows) break;
+      if (i > 0 && ++grem == a.rpg) { grem = 0; ++gi; }
+      flush(gi);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        if (!cv[q]) continue;
+        const float x = take(v[i][q], q);
+        gmn = fminf(gmn, x); gmx = fmaxf(gmx, x);
+      }
+    }
+  } else {  // lanes of one load in different groups (the host avoids this layout then): per element
+    flush(-1);
+#pragma unroll
+    for (int i = 0; i < kRangeLoads; ++i) {
+      if (i * S::kRW + sub >= nrows) continue;
+      const int64_t gi = a.div_rpg.div((uint32_t)(rc + i * S::kRW + sub));
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        if (!cv[q]) continue;
+        const float x = take(v[i][q], q);
+        if (a.smin) { atomicMin(a.smin + gi, float_to_ordered(x)); atomicMin(a.smax + gi, ~float_to_ordered(x)); }
+      }
+    }
+  }
+}
+
+// A contiguous run of row tiles per CTA: the host sizes gridDim.y to one resident wave, so that a
+// tall gradient (the ResNet-18 stem: 12544 row tiles) updates each channel key once per CTA
+// rather than once per row tile, and a warp's rows leave a sample group at most a few times
+// (strided tiles would change group on every tile and flood the group keys with atomics).  The
+// next chunk's loads are issued before the current chunk is reduced, so that every lane keeps
+// two chunks of G in flight.
+template <int LPR, bool VEC>
 __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
+  using S = RangeShape<LPR>;
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
-  __shared__ uint32_t cmin_s[8][kRangeCols], cmax_s[8][kRangeCols];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t c0 = (int64_t)blockIdx.x * kRangeCols + lane * 4;
-  const int64_t r0 = (int64_t)blockIdx.y * kRangeRows + warp * (kRangeRows / 8);
+  __shared__ uint32_t cmin_s[8][S::kCols], cmax_s[8][S::kCols];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, sub = lane / LPR;
+  const int64_t c0 = (int64_t)blockIdx.x * S::kCols + (lane % LPR) * 4;
   float gam[4];
   bool cv[4];
 #pragma unroll
@@ -52,65 +162,55 @@ __global__ void __launch_bounds__(256) range_kernel(RangeArgs a) {
     cv[q] = c0 + q < a.D;
     gam[q] = ldg_sel(a.gamma, c0 + q, a.gamma && cv[q], 1.0f, a.g);
   }
-  uint32_t colmin[4] = {0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu}, colmax[4] = {0u, 0u, 0u, 0u};
-  uint32_t gmin = 0xFFFFFFFFu, gmax = 0u;
+  const float pinf = __int_as_float(0x7F800000), ninf = __int_as_float(0xFF800000);
+  float cmn[4] = {pinf, pinf, pinf, pinf}, cmx[4] = {ninf, ninf, ninf, ninf};
+  float gmn = pinf, gmx = ninf;
   int64_t cur = -1;
   bool bad = false;
-  constexpr int kR = kRangeRows / 8;  // rows per warp
-  float v[kR][4];
+  const int64_t row_tiles = (a.M + S::kTile - 1) / S::kTile;
+  const int64_t per_cta = (row_tiles + gridDim.y - 1) / gridDim.y;
+  const int64_t rt0 = (int64_t)blockIdx.y * per_cta, rt1 = min(row_tiles, rt0 + per_cta);
+  const int64_t wrow = (int64_t)warp * S::kChunk;
+  float v[kRangeLoads][4], nv[kRangeLoads][4];
+  if (rt0 < rt1) range_load<LPR, VEC>(a, rt0 * S::kTile + wrow + sub, c0, cv[0], v);
+#pragma unroll 1
+  for (int64_t rt = rt0; rt < rt1; ++rt) {
+    const int64_t rc = rt * S::kTile + wrow;
+    if (rc >= a.M) break;  // warp-uniform; later tiles start further on
+    if (rt + 1 < rt1) range_load<LPR, VEC>(a, rc + S::kTile + sub, c0, cv[0], nv);
+    if (a.gamma) range_chunk<LPR, true>(a, rc, sub, cv, gam, v, cmn, cmx, gmn, gmx, cur, bad, lane);
+    else range_chunk<LPR, false>(a, rc, sub, cv, gam, v, cmn, cmx, gmn, gmx, cur, bad, lane);
 #pragma unroll
-  for (int i = 0; i < kR; ++i) {  // all loads of this warp's rows first, unconditional (clamped)
-    const int64_t r = min(r0 + i, a.M - 1);
-    if (VEC) {
-      const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + (cv[0] ? c0 : 0)));
-      v[i][0] = t.x; v[i][1] = t.y; v[i][2] = t.z; v[i][3] = t.w;
-    } else {
+    for (int i = 0; i < kRangeLoads; ++i)
 #pragma unroll
-      for (int q = 0; q < 4; ++q) v[i][q] = __ldg(a.g + r * a.D + min(c0 + q, a.D - 1));
-    }
+      for (int q = 0; q < 4; ++q) v[i][q] = nv[i][q];
   }
-  // sample group of the first row; the next rows step through it
-  int64_t gi = a.div_rpg.div((uint32_t)min(r0, a.M - 1)), grem = min(r0, a.M - 1) - gi * a.rpg;
-#pragma unroll
-  for (int i = 0; i < kR; ++i) {
-    const int64_t r = r0 + i;
-    if (r >= a.M) break;
-    if (i > 0 && ++grem == a.rpg) { grem = 0; ++gi; }
-    if (a.smin && gi != cur) {
-      if (cur >= 0) {
-        const uint32_t mn = __reduce_min_sync(0xFFFFFFFFu, gmin), mx = __reduce_max_sync(0xFFFFFFFFu, gmax);
-        if (lane == 0) { atomicMin(a.smin + cur, mn); atomicMin(a.smax + cur, ~mx); }
-      }
-      cur = gi;
-      gmin = 0xFFFFFFFFu;
-      gmax = 0u;
-    }
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      if (!cv[q]) continue;
-      const float x = a.gamma ? __fmul_rn(v[i][q], gam[q]) : v[i][q];
-      bad |= !isfinite(x);
-      const uint32_t k = float_to_ordered(x);
-      colmin[q] = min(colmin[q], k);
-      colmax[q] = max(colmax[q], k);
-      gmin = min(gmin, k);
-      gmax = max(gmax, k);
-    }
-  }
+  // rc is warp-uniform, so every lane of a warp that has rows reaches this flush together
   if (a.smin && cur >= 0) {
-    const uint32_t mn = __reduce_min_sync(0xFFFFFFFFu, gmin), mx = __reduce_max_sync(0xFFFFFFFFu, gmax);
+    const uint32_t mn = __reduce_min_sync(0xFFFFFFFFu, float_to_ordered(gmn));
+    const uint32_t mx = __reduce_max_sync(0xFFFFFFFFu, float_to_ordered(gmx));
     if (lane == 0) { atomicMin(a.smin + cur, mn); atomicMin(a.smax + cur, ~mx); }
   }
   if (__any_sync(0xFFFFFFFFu, bad) && lane == 0) atomicOr(a.dev_status, FQT1_DEV_NONFINITE);
   if (a.cmin) {
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      cmin_s[warp][lane * 4 + q] = colmin[q];
-      cmax_s[warp][lane * 4 + q] = colmax[q];
+    for (int q = 0; q < 4; ++q) {  // lanes that hold the same columns (other rows) first
+#pragma unroll
+      for (int o = LPR; o < 32; o <<= 1) {
+        cmn[q] = fminf(cmn[q], __shfl_xor_sync(0xFFFFFFFFu, cmn[q], o));
+        cmx[q] = fmaxf(cmx[q], __shfl_xor_sync(0xFFFFFFFFu, cmx[q], o));
+      }
+    }
+    if (lane < LPR) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {  // no rows: +inf / -inf map to keys that leave the atomics below idle
+        cmin_s[warp][lane * 4 + q] = float_to_ordered(cmn[q]);
+        cmax_s[warp][lane * 4 + q] = cmx[q] == ninf ? 0u : float_to_ordered(cmx[q]);
+      }
     }
     __syncthreads();
-    if (threadIdx.x < kRangeCols) {
-      const int64_t c = (int64_t)blockIdx.x * kRangeCols + threadIdx.x;
+    if (threadIdx.x < S::kCols) {
+      const int64_t c = (int64_t)blockIdx.x * S::kCols + threadIdx.x;
       uint32_t mn = 0xFFFFFFFFu, mx = 0u;
 #pragma unroll
       for (int w = 0; w < 8; ++w) { mn = min(mn, cmin_s[w][threadIdx.x]); mx = max(mx, cmax_s[w][threadIdx.x]); }
@@ -690,6 +790,21 @@ extern "C" size_t fqt1_workspace_size(int32_t which, int64_t M, int64_t D, int64
   return 0;
 }
 
+// Resident range CTAs on the whole GPU (SMs x CTAs per SM) for each kernel variant, per device.
+static int range_wave(void (*rk)(RangeArgs), int variant) {
+  static std::atomic<int> cache[64][4];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
+  int w = cache[dev][variant].load(std::memory_order_relaxed);
+  if (w > 0) return w;
+  int sms = 152, per_sm = 4;
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rk, 256, 0) != cudaSuccess || per_sm < 1) per_sm = 1;
+  w = sms * per_sm;
+  cache[dev][variant].store(w, std::memory_order_relaxed);
+  return w;
+}
+
 // Shared driver of both entry points.
 static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const float* gamma,
                                  const fqt1_agp_params* ps, fqt1_qgrad* psq, const fqt1_agp_params* pc,
@@ -712,7 +827,7 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
   if (!ws || ws_bytes < need) return FQT1_ERR_WORKSPACE;
   if (!aligned16(ws)) return FQT1_ERR_MISALIGNED;
   if (M * D >= (1ll << 46)) return FQT1_ERR_UNSUPPORTED;
-  if ((M + kQRows - 1) / kQRows > 65535 || (M + kRangeRows - 1) / kRangeRows > 65535) return FQT1_ERR_UNSUPPORTED;
+  if ((M + kQRows - 1) / kQRows > 65535) return FQT1_ERR_UNSUPPORTED;
 
   uint32_t* smin = static_cast<uint32_t*>(ws);
   uint32_t* cmin = smin + ns;
@@ -724,9 +839,19 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
   const bool vec = (D % 4) == 0;
   RangeArgs ra{g, gamma, M, D, rpg, psq ? smin : nullptr, psq ? smax : nullptr, pcq ? cmin : nullptr,
                pcq ? cmax : nullptr, dev_status, FastDiv((uint32_t)rpg)};
-  dim3 rgrid((unsigned)((D + kRangeCols - 1) / kRangeCols), (unsigned)((M + kRangeRows - 1) / kRangeRows));
-  if (vec) launch_k(range_kernel<true>, dim3(rgrid), dim3(256), 0, s, ra);
-  else launch_k(range_kernel<false>, dim3(rgrid), dim3(256), 0, s, ra);
+  // lane layout: rows of 8 or 16 lanes when D is that narrow and no warp chunk straddles two
+  // sample groups; one resident wave of CTAs at most, each looping over its run of row tiles
+  int lpr = 32;
+  if (vec && D <= 32 && (!psq || rpg % RangeShape<8>::kChunk == 0)) lpr = 8;
+  else if (vec && D <= 64 && (!psq || rpg % RangeShape<16>::kChunk == 0)) lpr = 16;
+  void (*rk)(RangeArgs) = lpr == 8 ? range_kernel<8, true>
+                        : lpr == 16 ? range_kernel<16, true>
+                        : vec ? range_kernel<32, true> : range_kernel<32, false>;
+  const int tile = lpr == 8 ? RangeShape<8>::kTile : lpr == 16 ? RangeShape<16>::kTile : RangeShape<32>::kTile;
+  const int64_t rcols = (D + 4 * lpr - 1) / (4 * lpr), rtiles = (M + tile - 1) / tile;
+  const int wave = range_wave(rk, lpr == 8 ? 0 : lpr == 16 ? 1 : vec ? 2 : 3);
+  dim3 rgrid((unsigned)rcols, (unsigned)std::min<int64_t>(rtiles, std::max<int64_t>(1, wave / rcols)));
+  launch_k(rk, rgrid, dim3(256), 0, s, ra);
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
 
