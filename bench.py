@@ -321,6 +321,9 @@ def main():
     ap.add_argument("--e4m3-weights", choices=["on", "off"], default="on",
                     help="e4m3 copies of sign(W) written by the weight packing and loaded by TMA as the "
                          "B operand of the forward and grad_input products")
+    ap.add_argument("--e4m3-x", choices=["on", "off"], default="off",
+                    help="e4m3 copies of sign(X_u) written by the Unfolder and loaded by TMA as the sign "
+                         "operand of the forward and grad_weight products")
     ap.add_argument("--profile", type=int, default=0, metavar="N",
                     help="only run --warmup + N eager steps (for ncu), print nothing")
     ap.add_argument("--table5", action="store_true",
@@ -368,7 +371,7 @@ def main():
 
     wl = workloads.resnet18_cifar_conv()
     st = LayerStep(wl, device=f"cuda:{local_rank}", keep_acc=False, implicit=args.implicit,
-                   e4m3_weights=args.e4m3_weights == "on")
+                   e4m3_weights=args.e4m3_weights == "on", e4m3_x=args.e4m3_x == "on")
     stream = torch.cuda.Stream()
     if args.profile:
         # eager steps, each after an L2 flush as in the timed loop (with ncu --cache-control none
@@ -515,6 +518,7 @@ def main():
                                      "epilogue), CUDA events on the launching stream",
                            "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU",
                            "forward": "implicit GEMM (pixel-major sign(X))" if st.implicit
+                           else "e4m3 copies of sign(X_u) by TMA (forward and grad_weight)" if st.e4m3_x
                            else "1-bit unfolded X_u",
                            "weights": "e4m3 copies of sign(W) by TMA" if (st.w8 is not None or st.wt8 is not None)
                            else "packed sign(W) expanded per CTA"},

@@ -260,6 +260,36 @@ fqt1_status fqt1_bwd_input_fold_e4m3w(const fqt1_qgrad* psq, const uint8_t* wt_e
                                       int32_t kh, int32_t kw, int32_t stride, int32_t pad, int64_t D,
                                       const fqt1_agp_params* p, float* dx, void* stream);
 
+/* e4m3 copies of sign(X_u) for the forward and grad_weight products (no
+ * counterpart in the paper: the Unfolder's +-1 values of App. C in the tensor
+ * cores' byte format, so that both products load their sign operand with TMA
+ * and expand nothing; 8 times the bytes of the packed signs).
+ * fqt1_im2col_e4m3: the Unfolder of fqt1_im2col writing x_row [M][ld_row]
+ *   (row m = output pixel, byte k = column of X_u; ld_row >= K rounded up to 16)
+ *   and x_col [K][ld_col] (the transpose; ld_col >= M rounded up to 16) instead
+ *   of the packed words: 0x38 (+1), 0xB8 (-1), and 0 from the valid length to
+ *   the next multiple of 16; colsum [K] as in fqt1_im2col.  Each output may be
+ *   NULL (x_row or x_col must be given); pointers 16-byte aligned.  Serves the
+ *   shapes for which fqt1_im2col_path returns 2; others give
+ *   FQT1_ERR_UNSUPPORTED before any launch.
+ * fqt1_fwd_gemm_e4m3x: the forward product of Sec. 5.1 with both operands as
+ *   e4m3 signs: x_e4m3 [M][ld_x] (from fqt1_im2col_e4m3, or the row_e4m3 of
+ *   fqt1_binarize_pack_e4m3 for a linear X) and w_e4m3 [D][ld_w]; bytes past K
+ *   must be 0 in at least one of them.  gamma, bias, acc and y as in
+ *   fqt1_fwd_gemm_bias; results equal it bit for bit.
+ * fqt1_bwd_weight_gemm_e4m3x: fqt1_bwd_weight_gemm with sign(X_u)^T given as
+ *   x_col_e4m3 [K][ld_xc] bytes (ld_xc >= M rounded up to 16); results equal it
+ *   bit for bit. */
+fqt1_status fqt1_im2col_e4m3(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw,
+                             int32_t stride, int32_t pad, uint8_t* x_row, int64_t ld_row, uint8_t* x_col,
+                             int64_t ld_col, int32_t* colsum, void* stream);
+fqt1_status fqt1_fwd_gemm_e4m3x(const uint8_t* x_e4m3, int64_t ld_x, const uint8_t* w_e4m3, int64_t ld_w, int64_t M,
+                                int64_t D, int64_t K, const float* gamma, const float* bias, int32_t* acc, float* y,
+                                void* stream);
+fqt1_status fqt1_bwd_weight_gemm_e4m3x(const fqt1_qgrad* pcq, const uint8_t* x_col_e4m3, int64_t ld_xc,
+                                       const int32_t* colsum_x, int64_t M, int64_t D, int64_t K,
+                                       const fqt1_agp_params* p, int32_t* acc, float* dw, void* stream);
+
 /* ------------------------------------------------ layer parameters and STE */
 /* Gradients of the layer's scale Gamma (Sec. 5.1: y = (sign(X) sign(W)^T) (.)
  * Gamma, Gamma learnable) and of its bias:

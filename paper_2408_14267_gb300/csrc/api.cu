@@ -119,11 +119,11 @@ __global__ void col2im_kernel(const int32_t* __restrict__ acc, const int32_t* __
   dx[idx] = v;
 }
 
-// Folder with the accumulators staged in shared memory.  A CTA owns sample n, channels
-// [c0, c0+cb) and input rows [h0, h0+hb): it loads, coalesced, the int32 accumulator rows of
-// every output pixel whose window touches those input rows (their k-range of the block's
-// channels), then sums the taps of each input pixel from shared memory.  Row stride of the
-// tile is odd so that neighbouring pixels fall in different banks.
+// Folder with the accumulators staged in shared memory (two kernels).  A CTA owns one kept
+// sample, a block of channels and a block of input pixels: it loads, coalesced, the int32
+// accumulators of every output pixel whose window touches that block (the k-range of the
+// block's channels), then sums the taps of each input pixel from shared memory.  The tile's
+// row stride is odd so that neighbouring pixels fall in different banks.
 struct FoldArgs {
   const int32_t* acc;
   const int32_t* kept_idx;
@@ -133,12 +133,17 @@ struct FoldArgs {
   const int32_t* cs;
   float* dx;
   int N, C, H, W, kh, kw, stride, pad, Ho, Wo;
-  int cb, hb, ncb, max_rows, kstride;
+  int cb, hb, wb, ncb, nwb, max_rows, max_cols, kstride;
   int64_t K;
   int nhwc;  // dx in memory order N, H, W, C (outputs walked channels fastest) instead of NCHW
 };
 
-__global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
+constexpr int kFoldLoads = 8;  // accumulator loads in flight per thread while staging
+
+// Folder over whole input rows (blocks of at least min(C, 4) channels): a CTA owns channels
+// [c0, c0+cb) and input rows [h0, h0+hb) of its sample; each warp copies the accumulator
+// k-range of one output pixel at a time, which is coalesced when that range is long.
+__global__ void __launch_bounds__(256) col2im_rows_kernel(FoldArgs a) {
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
   extern __shared__ int32_t fold_smem[];
@@ -233,6 +238,115 @@ __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
       a.dx[(((int64_t)n * a.H + h0 + hl) * a.W + w) * a.C + c0 + cl] = v;
     else
       a.dx[(((int64_t)n * a.C + c0 + cl) * a.H + h0 + hl) * a.W + w] = v;
+  }
+}
+
+// Folder over blocks of input rows and columns (shapes whose whole-row blocks would hold fewer
+// than min(C, 4) channels, such as the 7 x 7 stride-2 stem on 3 channels): a CTA owns channels
+// [c0, c0+cb), rows [h0, h0+hb) and columns [w0, w0+wb) of its sample, which keeps the staged
+// halo of large, strided windows small; the staging loop walks the (pixel, k) elements of the
+// halo with every thread's loads in flight together, whatever the length of a pixel's k-range.
+__global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  extern __shared__ int32_t fold_smem[];
+  const int32_t slot = (int32_t)blockIdx.y;  // one kept sample per grid row
+  if (slot >= __ldg(a.kept_count)) return;
+  const int n = __ldg(a.kept_idx + slot);
+  const int cblk = blockIdx.x % a.ncb, rest = blockIdx.x / a.ncb;
+  const int wblk = rest % a.nwb, hblk = rest / a.nwb;
+  const int c0 = cblk * a.cb, h0 = hblk * a.hb, w0 = wblk * a.wb;
+  const int c1 = min(a.C, c0 + a.cb), h1 = min(a.H, h0 + a.hb), w1 = min(a.W, w0 + a.wb);
+  const int nc = c1 - c0, nh = h1 - h0, nw = w1 - w0;
+  const int khw = a.kh * a.kw;
+  // output rows / columns whose windows reach the block
+  int oh_lo = h0 + a.pad - (a.kh - 1);
+  oh_lo = oh_lo <= 0 ? 0 : (oh_lo + a.stride - 1) / a.stride;
+  const int oh_hi = min(a.Ho - 1, (h1 - 1 + a.pad) / a.stride);
+  int ow_lo = w0 + a.pad - (a.kw - 1);
+  ow_lo = ow_lo <= 0 ? 0 : (ow_lo + a.stride - 1) / a.stride;
+  const int ow_hi = min(a.Wo - 1, (w1 - 1 + a.pad) / a.stride);
+  const int nrows = oh_hi - oh_lo + 1, ncols = ow_hi - ow_lo + 1;
+  const int kb = nc * khw;
+  int32_t* tile = fold_smem;                                   // [max_rows * max_cols][kstride]
+  int32_t* hrow = tile + a.max_rows * a.max_cols * a.kstride;  // [hb * kh]: tile pixel-row offset or -1
+  int32_t* wcol = hrow + a.hb * a.kh;                          // [wb * kw]: tile column or -1
+  int32_t* css = wcol + a.wb * a.kw;                           // [cb * khw]: colsum of the block
+  for (int x = threadIdx.x; x < nh * a.kh; x += blockDim.x) {
+    const int hl = x / a.kh, i = x - hl * a.kh;
+    const int hn = h0 + hl + a.pad - i;
+    int v = -1;
+    if (hn >= 0 && hn % a.stride == 0) {
+      const int oh = hn / a.stride;
+      if (oh >= oh_lo && oh <= oh_hi) v = (oh - oh_lo) * a.max_cols;
+    }
+    hrow[x] = v;
+  }
+  for (int x = threadIdx.x; x < nw * a.kw; x += blockDim.x) {
+    const int wl = x / a.kw, j = x - wl * a.kw;
+    const int wn = w0 + wl + a.pad - j;
+    int v = -1;
+    if (wn >= 0 && wn % a.stride == 0) {
+      const int ow = wn / a.stride;
+      if (ow >= ow_lo && ow <= ow_hi) v = ow - ow_lo;
+    }
+    wcol[x] = v;
+  }
+  const int64_t kbase = (int64_t)c0 * khw;
+  for (int x = threadIdx.x; x < kb; x += blockDim.x) css[x] = __ldg(a.cs + kbase + x);
+  if (nrows > 0 && ncols > 0) {
+    // the (pixel, k) elements of the halo, kFoldLoads loads in flight per thread whatever kb is
+    const int total = nrows * ncols * kb;
+    const FastDiv div_kb((uint32_t)kb), div_cols((uint32_t)ncols);
+    const int64_t rbase = (int64_t)slot * a.Ho * a.Wo + (int64_t)oh_lo * a.Wo + ow_lo;
+    for (int e0 = threadIdx.x; e0 < total; e0 += blockDim.x * kFoldLoads) {
+      int32_t v[kFoldLoads];
+      int dsti[kFoldLoads];
+#pragma unroll
+      for (int u = 0; u < kFoldLoads; ++u) {
+        const int e = min(e0 + u * (int)blockDim.x, total - 1);  // clamped: every load is valid
+        const int pix = (int)div_kb.div((uint32_t)e), kk = e - pix * kb;
+        const int r = (int)div_cols.div((uint32_t)pix), cl = pix - r * ncols;
+        v[u] = __ldg(a.acc + (rbase + (int64_t)r * a.Wo + cl) * a.K + kbase + kk);
+        dsti[u] = (r * a.max_cols + cl) * a.kstride + kk;
+      }
+#pragma unroll
+      for (int u = 0; u < kFoldLoads; ++u)
+        if (e0 + u * (int)blockDim.x < total) tile[dsti[u]] = v[u];
+    }
+  }
+  __syncthreads();
+  const float sc = __ldg(a.scale + slot), ze = __ldg(a.zero + slot);
+  const int plane = nh * nw;
+  const FastDiv div_plane((uint32_t)plane), div_w((uint32_t)nw), div_nc((uint32_t)nc);
+  for (int e = threadIdx.x; e < nc * plane; e += blockDim.x) {  // output (channel, row, column) of the block
+    int cl, pos;
+    if (a.nhwc) {  // channels fastest: a pixel's nc channels are contiguous in dx
+      pos = (int)div_nc.div((uint32_t)e);
+      cl = e - pos * nc;
+    } else {
+      cl = (int)div_plane.div((uint32_t)e);
+      pos = e - cl * plane;
+    }
+    const int hl = (int)div_w.div((uint32_t)pos), wl = pos - hl * nw;
+    const int kc = cl * khw;
+    int32_t acc = 0, csum = 0;
+    for (int i = 0; i < a.kh; ++i) {
+      const int ro = hrow[hl * a.kh + i];
+      if (ro < 0) continue;
+      const int32_t* trow = tile + kc + i * a.kw;
+      for (int j = 0; j < a.kw; ++j) {
+        const int co = wcol[wl * a.kw + j];
+        if (co < 0) continue;
+        acc += trow[(ro + co) * a.kstride + j];
+        csum += css[kc + i * a.kw + j];
+      }
+    }
+    const float v = __fadd_rn(__fmul_rn(sc, __int2float_rn(acc)), __fmul_rn(ze, __int2float_rn(csum)));
+    if (a.nhwc)
+      a.dx[(((int64_t)n * a.H + h0 + hl) * a.W + w0 + wl) * a.C + c0 + cl] = v;
+    else
+      a.dx[(((int64_t)n * a.C + c0 + cl) * a.H + h0 + hl) * a.W + w0 + wl] = v;
   }
 }
 
@@ -354,15 +468,15 @@ static fqt1_status col2im_impl(const int32_t* acc, const fqt1_qgrad* psq, const 
   const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
   if (H + 2 * pad < kh || W + 2 * pad < kw) return FQT1_ERR_INVALID_ARG;
   if (!aligned16(acc) || !aligned16(dx)) return FQT1_ERR_MISALIGNED;
-  // tiled Folder: choose input rows and channels per CTA so that the staged accumulators fit
   constexpr int64_t kMaxTile = 96 * 1024;
   constexpr int64_t kPreferTile = 48 * 1024;  // >= 4 resident CTAs per SM
   const int khw = kh * kw;
-  int hb = H < 8 ? H : 8, cb = 0;
-  int max_rows = 0, kstride = 0;
+  // whole-row Folder: up to 8 input rows per CTA and the most channels whose staged
+  // accumulators fit (<= 48 KB, or 96 KB for a single channel)
+  int hb = H < 8 ? H : 8, wb = W, cb = 0;
+  int max_rows = 0, max_cols = Wo, kstride = 0;
   for (; hb >= 1 && cb == 0; hb /= 2) {
-    max_rows = (hb - 1 + kh - 1) / stride + 1;
-    if (max_rows > Ho) max_rows = Ho;
+    max_rows = std::min(Ho, (hb - 1 + kh - 1) / stride + 1);
     for (int c = (C < 32 ? C : 32); c >= 1; c = (c > 1 ? c / 2 : 0)) {
       const int ks = (c * khw) | 1;
       const int64_t words = (int64_t)max_rows * Wo * ks + (int64_t)hb * kh + (int64_t)W * kw + (int64_t)c * khw;
@@ -370,24 +484,62 @@ static fqt1_status col2im_impl(const int32_t* acc, const fqt1_qgrad* psq, const 
     }
     if (cb) break;
   }
+  // blocks of rows and columns when whole rows leave fewer than min(C, 4) channels per CTA:
+  // chosen for the least staging cost per output (the halo of the windows and the partial
+  // 32-byte sectors of each pixel's k-range, plus a fixed cost per CTA), with about 16 CTAs
+  // per SM over all samples
+  bool tiled = false;
+  if (cb < std::min(C, 4)) {
+    double best = 0.0;
+    int tcb = 0;
+    const int hbs[6] = {32, 16, 8, 4, 2, 1}, wbs[5] = {0, 64, 32, 16, 8};  // wb 0: whole rows
+    for (int pass = 0; pass < 2 && tcb == 0; ++pass) {
+      const int64_t cap = pass == 0 ? kPreferTile : kMaxTile;
+      for (int hi = 0; hi < 6; ++hi) {
+        const int hbc = hbs[hi] < H ? hbs[hi] : H;
+        for (int wi = 0; wi < 5; ++wi) {
+          const int wbc = (wbs[wi] == 0 || wbs[wi] > W) ? W : wbs[wi];
+          const int mr = std::min(Ho, (hbc - 1 + kh - 1) / stride + 1);
+          const int mc = std::min(Wo, (wbc - 1 + kw - 1) / stride + 1);
+          for (int c = (C < 32 ? C : 32); c >= 1; c = (c > 1 ? c / 2 : 0)) {
+            const int ks = (c * khw) | 1;
+            const int64_t words =
+                (int64_t)mr * mc * ks + (int64_t)hbc * kh + (int64_t)wbc * kw + (int64_t)c * khw;
+            if (words * 4 > cap) continue;
+            const double sectors = (double)(((int64_t)c * khw * 4 + 31) / 32 + 1) * 32.0;
+            double cost = ((double)mr * mc * sectors + 8192.0) / ((double)hbc * wbc * c);
+            const double ctas = (double)N * ((C + c - 1) / c) * ((H + hbc - 1) / hbc) * ((W + wbc - 1) / wbc);
+            if (ctas < 16.0 * 152) cost *= 16.0 * 152 / ctas;
+            if (tcb == 0 || cost < best) {
+              best = cost; hb = hbc; wb = wbc; tcb = c; max_rows = mr; max_cols = mc; kstride = ks;
+            }
+          }
+        }
+      }
+    }
+    if (tcb > 0) { cb = tcb; tiled = true; }
+  }
   if (cb > 0) {
-    static std::atomic<uint64_t> attr{0};
-    FQT1_CUDA_TRY(smem_attr_once((const void*)col2im_tiled_kernel, (int)kMaxTile, attr));
+    static std::atomic<uint64_t> attr_rows{0}, attr_tiled{0};
+    FQT1_CUDA_TRY(smem_attr_once((const void*)col2im_rows_kernel, (int)kMaxTile, attr_rows));
+    FQT1_CUDA_TRY(smem_attr_once((const void*)col2im_tiled_kernel, (int)kMaxTile, attr_tiled));
     FoldArgs fa;
     fa.acc = acc; fa.kept_idx = psq->kept_idx; fa.kept_count = psq->kept_count; fa.scale = psq->scale;
     fa.zero = psq->zero;
     fa.cs = colsum_w; fa.dx = dx; fa.N = N; fa.C = C; fa.H = H; fa.W = W; fa.kh = kh; fa.kw = kw;
-    fa.stride = stride; fa.pad = pad; fa.Ho = Ho; fa.Wo = Wo; fa.cb = cb; fa.hb = hb;
-    fa.ncb = (C + cb - 1) / cb; fa.max_rows = max_rows; fa.kstride = kstride; fa.K = (int64_t)C * khw;
+    fa.stride = stride; fa.pad = pad; fa.Ho = Ho; fa.Wo = Wo; fa.cb = cb; fa.hb = hb; fa.wb = wb;
+    fa.ncb = (C + cb - 1) / cb; fa.nwb = (W + wb - 1) / wb; fa.max_rows = max_rows; fa.max_cols = max_cols;
+    fa.kstride = kstride; fa.K = (int64_t)C * khw;
     fa.nhwc = nhwc;
-    const int64_t nblk = (int64_t)fa.ncb * ((H + hb - 1) / hb);
+    const int64_t nblk = (int64_t)fa.ncb * fa.nwb * ((H + hb - 1) / hb);
     if (nblk > 0x7FFFFFFF || N > 65535) return FQT1_ERR_UNSUPPORTED;
     const size_t smem =
-        ((size_t)max_rows * Wo * kstride + (size_t)hb * kh + (size_t)W * kw + (size_t)cb * khw) * 4;
+        ((size_t)max_rows * max_cols * kstride + (size_t)hb * kh + (size_t)wb * kw + (size_t)cb * khw) * 4;
     // pruned samples: zeros; kept samples: the tiled fold (one grid row per kept slot)
     launch_zero_pruned_rows(psq->slot_of_group, N, (int64_t)C * H * W, 1, dx, (cudaStream_t)stream);
     const int64_t cap = fqt1_kept_capacity(N, 8, FQT1_SEL_BERNOULLI);  // upper bound: all samples
-    launch_k(col2im_tiled_kernel, dim3((unsigned)nblk, (unsigned)cap), dim3(256), smem, (cudaStream_t)stream, fa);
+    launch_k(tiled ? col2im_tiled_kernel : col2im_rows_kernel, dim3((unsigned)nblk, (unsigned)cap), dim3(256), smem,
+             (cudaStream_t)stream, fa);
   } else {
     if (nhwc) return FQT1_ERR_UNSUPPORTED;
     const int64_t n = (int64_t)N * C * H * W;
@@ -470,16 +622,20 @@ extern "C" fqt1_status fqt1_bwd_input_fold_e4m3w(const fqt1_qgrad* psq, const ui
                              0, stream);
 }
 
-extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_t* sx_col, const int32_t* colsum_x,
-                                            int64_t M, int64_t D, int64_t K, const fqt1_agp_params* p, int32_t* acc,
-                                            float* dw, void* ws, size_t ws_bytes, void* stream) {
-  (void)ws; (void)ws_bytes;
-  if (!pcq || !sx_col || !colsum_x || !p || !acc || !dw || M < 1 || D < 1 || K < 1) return FQT1_ERR_INVALID_ARG;
+// grad_weight with B = packed sign(X_u)^T words (sx_col) or e4m3 sign bytes (xe, ldxe).
+static fqt1_status bwd_weight_impl(const fqt1_qgrad* pcq, const uint32_t* sx_col, const uint8_t* xe, int64_t ldxe,
+                                   const int32_t* colsum_x, int64_t M, int64_t D, int64_t K,
+                                   const fqt1_agp_params* p, int32_t* acc, float* dw, void* stream) {
+  if (!pcq || (!sx_col && !xe) || !colsum_x || !p || !acc || !dw || M < 1 || D < 1 || K < 1)
+    return FQT1_ERR_INVALID_ARG;
   if (!valid_bits(p->bits)) return FQT1_ERR_INVALID_ARG;
   if (!pcq->codes || !pcq->kept_count || !pcq->slot_of_group || !pcq->scale || !pcq->zero ||
       pcq->ld_codes < fqt1_codes_ld(M) || pcq->ld_codes % 16)
     return FQT1_ERR_INVALID_ARG;
-  if (!aligned16(sx_col) || !aligned16(acc) || !aligned16(dw) || !aligned16(colsum_x)) return FQT1_ERR_MISALIGNED;
+  if (xe && (ldxe < fqt1_codes_ld(M) || ldxe % 16)) return FQT1_ERR_INVALID_ARG;
+  if ((sx_col && !aligned16(sx_col)) || (xe && !aligned16(xe)) || !aligned16(acc) || !aligned16(dw) ||
+      !aligned16(colsum_x))
+    return FQT1_ERR_MISALIGNED;
   const int64_t cap = fqt1_kept_capacity(D, p->bits, p->mode);
   cudaStream_t s = (cudaStream_t)stream;
   {
@@ -501,7 +657,7 @@ extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_
     if (!spread && tps * kCodesStageK <= exact_chunk(p->bits)) {
       FQT1_CUDA_TRY(launch_wgrad_cluster_tc(p->bits, pcq->codes, pcq->ld_codes, cap, pcq->kept_count, sx_col, K, M,
                                             (int)cs, acc, dw, D, pcq->kept_idx, pcq->slot_of_group, pcq->scale,
-                                            pcq->zero, colsum_x, nullptr, s));
+                                            pcq->zero, colsum_x, nullptr, s, xe, ldxe));
       return FQT1_OK;
     }
     // contractions too long for eight exact splits, or too long for so few clusters: int32
@@ -515,7 +671,7 @@ extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_
     FQT1_CUDA_TRY(cudaMemsetAsync(acc, 0, sizeof(int32_t) * cap * K, s));
     FQT1_CUDA_TRY(launch_codes_tc_simple(p->bits, pcq->codes, pcq->ld_codes, cap, pcq->kept_count, 1, sx_col, K, M,
                                          GEMM_EPI_RED, (int)splits, acc, nullptr, K, nullptr, nullptr, nullptr,
-                                         nullptr, 1, nullptr, s));
+                                         nullptr, 1, nullptr, s, xe, ldxe));
   }
   const int64_t n = D * K;
   launch_k(dequant_rows_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, acc, K, pcq->slot_of_group, pcq->scale, pcq->zero,
@@ -524,3 +680,34 @@ extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_
   FQT1_CUDA_TRY(cudaGetLastError());
   return FQT1_OK;
 }
+
+extern "C" fqt1_status fqt1_bwd_weight_gemm(const fqt1_qgrad* pcq, const uint32_t* sx_col, const int32_t* colsum_x,
+                                            int64_t M, int64_t D, int64_t K, const fqt1_agp_params* p, int32_t* acc,
+                                            float* dw, void* ws, size_t ws_bytes, void* stream) {
+  (void)ws; (void)ws_bytes;
+  if (!sx_col) return FQT1_ERR_INVALID_ARG;
+  return bwd_weight_impl(pcq, sx_col, nullptr, 0, colsum_x, M, D, K, p, acc, dw, stream);
+}
+
+extern "C" fqt1_status fqt1_bwd_weight_gemm_e4m3x(const fqt1_qgrad* pcq, const uint8_t* x_col_e4m3, int64_t ld_xc,
+                                                  const int32_t* colsum_x, int64_t M, int64_t D, int64_t K,
+                                                  const fqt1_agp_params* p, int32_t* acc, float* dw, void* stream) {
+  if (!x_col_e4m3) return FQT1_ERR_INVALID_ARG;
+  return bwd_weight_impl(pcq, nullptr, x_col_e4m3, ld_xc, colsum_x, M, D, K, p, acc, dw, stream);
+}
+
+extern "C" fqt1_status fqt1_fwd_gemm_e4m3x(const uint8_t* x_e4m3, int64_t ld_x, const uint8_t* w_e4m3, int64_t ld_w,
+                                           int64_t M, int64_t D, int64_t K, const float* gamma, const float* bias,
+                                           int32_t* acc, float* y, void* stream) {
+  if (!x_e4m3 || !w_e4m3 || M < 1 || D < 1 || K < 1 || (!acc && !y) || (y && !gamma) || (bias && !y))
+    return FQT1_ERR_INVALID_ARG;
+  if (ld_x < fqt1_codes_ld(K) || ld_x % 16 || ld_w < fqt1_codes_ld(K) || ld_w % 16) return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(x_e4m3) || !aligned16(w_e4m3) || (acc && !aligned16(acc)) || (y && !aligned16(y)) ||
+      (gamma && !aligned16(gamma)) || (bias && !aligned16(bias)))
+    return FQT1_ERR_MISALIGNED;
+  if (K >= (1ll << 24) || (M + 127) / 128 > 65535) return FQT1_ERR_UNSUPPORTED;
+  FQT1_CUDA_TRY(launch_fwd_e4m3x_tc(x_e4m3, ld_x, w_e4m3, ld_w, M, D, K, gamma, bias, acc, y, nullptr,
+                                    (cudaStream_t)stream));
+  return FQT1_OK;
+}
+

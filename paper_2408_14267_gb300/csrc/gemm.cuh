@@ -20,7 +20,8 @@ cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int6
                                    int64_t rows_per_count, const uint32_t* Sg, int64_t n_s, int64_t L, int epi,
                                    int splits, int32_t* acc, float* out, int64_t ldo, const int32_t* kept_idx,
                                    const float* scale, const float* zero, const int32_t* cs, int64_t rpg,
-                                   int32_t* status, cudaStream_t s);
+                                   int32_t* status, cudaStream_t s, const uint8_t* Be = nullptr,
+                                   int64_t ldbe = 0);
 enum : int { GEMM_EPI_ACC32 = 1, GEMM_EPI_RED = 2, GEMM_EPI_DX = 3 };
 // Bte: e4m3 sign(W)^T rows [K][ldbte] bytes, or null for the packed sign(W) columns Sg.
 // nhwc: dx in memory order N, H, W, C.
@@ -46,12 +47,18 @@ inline int64_t fold_table_bytes(int64_t H, int64_t W, int64_t kh, int64_t kw, in
 // grad_weight with the split-K reduction and the dequantization in the kernel: the splits of
 // an output tile form a thread-block cluster of `splits` (<= 8) CTAs that add their partial
 // tiles through distributed shared memory.  acc [capacity][K] receives the int32 sums (rows past
-// the kept count 0), dw [D][K] the dequantized rows (pruned channels 0).
+// the kept count 0), dw [D][K] the dequantized rows (pruned channels 0).  Be (optional): the
+// signs of X_u^T as e4m3 bytes [K][ldbe] (by TMA into the operand ring) instead of Sx.
 cudaError_t launch_wgrad_cluster_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t capacity, const int32_t* count,
                                     const uint32_t* Sx, int64_t K, int64_t M, int splits, int32_t* acc, float* dw,
                                     int64_t D, const int32_t* kept_idx, const int32_t* slot_of_group,
                                     const float* scale, const float* zero, const int32_t* cs, int32_t* status,
-                                    cudaStream_t s);
+                                    cudaStream_t s, const uint8_t* Be = nullptr, int64_t ldbe = 0);
+// Forward with A = e4m3 sign(X_u) rows [M][ldxe] and B = e4m3 sign(W) rows [D][ldbe] bytes
+// (+1 = 0x38, -1 = 0xB8, bytes past K zero), both straight from TMA.
+cudaError_t launch_fwd_e4m3x_tc(const uint8_t* Xe, int64_t ldxe, const uint8_t* Be, int64_t ldbe, int64_t M, int64_t D,
+                                int64_t K, const float* gamma, const float* bias, int32_t* acc, float* y,
+                                int32_t* status, cudaStream_t s);
 // Cluster size for launch_wgrad_cluster_tc: the largest (<= 8, <= k_tiles) whose out_tiles
 // clusters fit on the GPU at once.
 int wgrad_cluster_size(int bits, int64_t out_tiles, int64_t k_tiles);

@@ -231,6 +231,7 @@ __device__ __forceinline__ void mma_e4m3_ss(uint32_t tmem_d, uint64_t ad, uint64
 // An fp32 accumulator word -> the exact int32 sum.  With A_DIRECT the A operand was the code
 // bytes themselves, read as e4m3: byte q < 16 is the e4m3 number q 2^-9 (subnormals 0..7,
 // then the first binade 8..15), so the accumulator holds sum 2^-9 and 512 rescales it exactly.
+// (A operands of e4m3 signs, +-1, need no rescale: A_DIRECT is false for them.)
 template <bool A_DIRECT>
 __device__ __forceinline__ int32_t acc_int(uint32_t v) {
   if constexpr (A_DIRECT) return __float2int_rn(__fmul_rn(__uint_as_float(v), 512.0f));
@@ -339,14 +340,19 @@ struct TcSmem {
 // the raw ring (A_DIRECT: the MMA reads the TMA-written code tile as e4m3, nothing expands A;
 // the raw stage is released by the MMA's commit), bit 4 the failure-path test: the expansion
 // warps withhold their arrive on the first operand stage, so the MMA issuer's bounded wait
-// (20 ms in this instantiation) expires and the kernel takes its timeout exit.
+// (20 ms in this instantiation) expires and the kernel takes its timeout exit, bit 5 e4m3
+// signs (+1 = 0x38, -1 = 0xB8) as the A operand straight from the raw ring (the A_DIRECT
+// datapath with a unit scale: the forward product of e4m3 X_u rows).
 template <bool A_CODES, bool BITS8, int BN, bool SHORT, int X = 0>
 __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmAcc, TcArgs a) {
   using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
-  constexpr bool kImpl = (X & 1) != 0, kBtma = (X & 2) != 0, kNhwc = (X & 4) != 0, kAdir = (X & 8) != 0;
-  static_assert(!kAdir || (A_CODES && !BITS8), "A_DIRECT takes codes below 16");
+  constexpr bool kImpl = (X & 1) != 0, kBtma = (X & 2) != 0, kNhwc = (X & 4) != 0;
+  // bit 3: codes below 16 as the A operand straight from TMA (scale 2^-9); bit 5: e4m3 signs
+  // (+-1) as the A operand straight from TMA (scale 1).  Both take the A_DIRECT datapath.
+  constexpr bool kA512 = (X & 8) != 0, kAdir = (X & 8) != 0 || (X & 32) != 0;
+  static_assert(!kAdir || (A_CODES && !BITS8), "A_DIRECT takes byte operands of one digit");
   constexpr bool kLose = (X & 16) != 0;
   constexpr uint64_t kLimit = kLose ? 20000000ull : kWaitNs;  // bound of every wait below
   // arrivals that free a raw stage: the expansion warps (when they read it) and, with A_DIRECT,
@@ -795,7 +801,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
         int32_t* trow = T + (32 * qf + lane) * TS + c0;
 #pragma unroll
-        for (int j = 0; j < 32; ++j) trow[j] = acc_int<kAdir>(v[j]);
+        for (int j = 0; j < 32; ++j) trow[j] = acc_int<kA512>(v[j]);
       }
       const int rpg = (int)a.rpg, imgs = f_imgs, khw = f_khw, HW = f_HW;
       const int c_first = f_c0, nc = f_nc;
@@ -919,10 +925,10 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
           int4 w;
-          w.x = acc_int<kAdir>(v[4 * c + 0]);
-          w.y = acc_int<kAdir>(v[4 * c + 1]);
-          w.z = acc_int<kAdir>(v[4 * c + 2]);
-          w.w = acc_int<kAdir>(v[4 * c + 3]);
+          w.x = acc_int<kA512>(v[4 * c + 0]);
+          w.y = acc_int<kA512>(v[4 * c + 1]);
+          w.z = acc_int<kA512>(v[4 * c + 2]);
+          w.w = acc_int<kA512>(v[4 * c + 3]);
           *reinterpret_cast<int4*>(base + ptile_off(r, (c0 >> 2) + c)) = w;
         }
         continue;
@@ -939,10 +945,10 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         const int64_t nb = n0 + c0;
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
-          const int32_t i0 = acc_int<kAdir>(v[4 * c + 0]);
-          const int32_t i1 = acc_int<kAdir>(v[4 * c + 1]);
-          const int32_t i2 = acc_int<kAdir>(v[4 * c + 2]);
-          const int32_t i3 = acc_int<kAdir>(v[4 * c + 3]);
+          const int32_t i0 = acc_int<kA512>(v[4 * c + 0]);
+          const int32_t i1 = acc_int<kA512>(v[4 * c + 1]);
+          const int32_t i2 = acc_int<kA512>(v[4 * c + 2]);
+          const int32_t i3 = acc_int<kA512>(v[4 * c + 3]);
           const int off = lane * 32 + ((c ^ (lane & 7)) << 2);
           if (a.tma_out & 1) {
             const float4 g4 = *reinterpret_cast<const float4*>(gamma_s + c0 + 4 * c);
@@ -973,7 +979,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         if (r >= valid_rows || r >= a.M || nb >= a.N) continue;
         int32_t iv[32];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) iv[j] = acc_int<kAdir>(v[j]);
+        for (int j = 0; j < 32; ++j) iv[j] = acc_int<kA512>(v[j]);
         const bool full = nb + 32 <= a.N && (a.ldo % 4) == 0;
         int64_t out_row = r;
         float sc = 0.f, ze = 0.f;
@@ -1047,10 +1053,10 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         uint4 w;
-        w.x = (uint32_t)acc_int<kAdir>(v[4 * c + 0]);
-        w.y = (uint32_t)acc_int<kAdir>(v[4 * c + 1]);
-        w.z = (uint32_t)acc_int<kAdir>(v[4 * c + 2]);
-        w.w = (uint32_t)acc_int<kAdir>(v[4 * c + 3]);
+        w.x = (uint32_t)acc_int<kA512>(v[4 * c + 0]);
+        w.y = (uint32_t)acc_int<kA512>(v[4 * c + 1]);
+        w.z = (uint32_t)acc_int<kA512>(v[4 * c + 2]);
+        w.w = (uint32_t)acc_int<kA512>(v[4 * c + 3]);
         *reinterpret_cast<uint4*>(stage + lane * 32 + ((c ^ (lane & 7)) << 2)) = w;
       }
       __syncwarp();
@@ -1286,6 +1292,30 @@ cudaError_t launch_fwd_e4m3w_tc(const uint32_t* A, const uint8_t* Be, int64_t ld
   return launch_fwd_common(ma, TcArgs{}, nullptr, M, D, K, gamma, bias, acc, y, status, s, Be, ldbe);
 }
 
+// Forward with A = e4m3 sign(X_u) rows [M][ldxe] and B = e4m3 sign(W) rows [D][ldbe] (bytes
+// +1 = 0x38, -1 = 0xB8): both operands go by TMA straight into the MMA, nothing is expanded.
+cudaError_t launch_fwd_e4m3x_tc(const uint8_t* Xe, int64_t ldxe, const uint8_t* Be, int64_t ldbe, int64_t M, int64_t D,
+                                int64_t K, const float* gamma, const float* bias, int32_t* acc, float* y,
+                                int32_t* status, cudaStream_t s) {
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, Xe, CU_TENSOR_MAP_DATA_TYPE_UINT8, K, M, ldxe, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&mb, Be, CU_TENSOR_MAP_DATA_TYPE_UINT8, K, D, ldbe, kBK, 128, CU_TENSOR_MAP_SWIZZLE_128B))
+    return cudaErrorInvalidValue;
+  TcArgs a{};
+  a.M = M; a.N = D; a.L = K; a.count = nullptr; a.rows_per_count = 1;
+  a.k_tiles = (int)((K + kCodesStageK - 1) / kCodesStageK); a.tiles_per_split = a.k_tiles;
+  a.epi = EPI_FWD; a.gamma = gamma; a.bias = bias; a.y = y; a.acc = acc; a.ldo = D; a.status = status;
+  CUtensorMap my{}, macc{};
+  if (D % 4 == 0) {
+    bool ok = true;
+    if (y) ok = make_map(&my, y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, D, M, D * 4, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (ok && acc)
+      ok = make_map(&macc, acc, CU_TENSOR_MAP_DATA_TYPE_INT32, D, M, D * 4, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (ok) a.tma_out = (y ? 1 : 0) | (acc ? 2 : 0);
+  }
+  return launch_tc<true, false, 128, false, 2 | 32>(ma, mb, a, 1, s, &my, &macc);
+}
+
 // Implicit-GEMM forward of a stride-1 "same" convolution (kh = kw = 2 pad + 1, C a multiple of
 // 128).  A tile of 128 output pixels is whole images (H W divides 128) or whole image rows (W
 // divides 128 and the rows of a tile divide H); its A sub-tiles are 4-D boxes of the pixel-major
@@ -1328,21 +1358,32 @@ cudaError_t launch_fwd_implicit_tc(const uint32_t* xp, const uint32_t* wt, int N
 
 // Codes x signs: out[r, n] = sum_j Q[r, j] S[n, j], Q [rows][ld] uint8 (valid rows *count * rpc),
 // S [n_s][words(L)] packed signs.  epi: EPI_ACC32 (store), EPI_RED (split-K add), EPI_DX (dequantize).
+// Be (optional): S as e4m3 sign bytes [n_s][ldbe] instead of packed words, by TMA into the
+// operand ring.
 cudaError_t launch_codes_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
                             int64_t rows_per_count, const uint32_t* Sg, int64_t n_s, int64_t L, int epi, int splits,
-                            const TcArgs& epi_args, cudaStream_t s) {
+                            const TcArgs& epi_args, cudaStream_t s, const uint8_t* Be = nullptr, int64_t ldbe = 0) {
   const int64_t lds = fqt1_packed_words(L);
   CUtensorMap ma, mb;
-  if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, L, max_rows, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, n_s, lds * 4, kCodesStageK / 32, 128,
-                CU_TENSOR_MAP_SWIZZLE_NONE))
+  if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, L, max_rows, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B))
     return cudaErrorInvalidValue;
+  if (Be) {
+    if (!make_map(&mb, Be, CU_TENSOR_MAP_DATA_TYPE_UINT8, L, n_s, ldbe, kBK, 128, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+  } else if (!make_map(&mb, Sg, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, n_s, lds * 4, kCodesStageK / 32, 128,
+                       CU_TENSOR_MAP_SWIZZLE_NONE)) {
+    return cudaErrorInvalidValue;
+  }
   TcArgs a = epi_args;
   a.M = max_rows; a.N = n_s; a.L = L; a.count = count; a.rows_per_count = rows_per_count;
   a.k_tiles = (int)((L + kCodesStageK - 1) / kCodesStageK);
   a.tiles_per_split = (a.k_tiles + splits - 1) / splits;
   a.epi = epi;
   const int z = (a.k_tiles + a.tiles_per_split - 1) / a.tiles_per_split;
+  if (Be) {
+    if (bits == 8) return launch_tc<true, true, 128, false, 2>(ma, mb, a, z, s);
+    return launch_tc<true, false, 128, false, 2 | 8>(ma, mb, a, z, s);
+  }
   if (bits == 8) return launch_tc<true, true, 128>(ma, mb, a, z, s);
   return launch_tc<true, false, 128, false, 8>(ma, mb, a, z, s);  // codes < 16: A straight from TMA
 }
@@ -1436,19 +1477,28 @@ cudaError_t launch_wgrad_cluster_tc(int bits, const uint8_t* Q, int64_t ldq, int
                                     const uint32_t* Sx, int64_t K, int64_t M, int splits, int32_t* acc, float* dw,
                                     int64_t D, const int32_t* kept_idx, const int32_t* slot_of_group,
                                     const float* scale, const float* zero, const int32_t* cs, int32_t* status,
-                                    cudaStream_t s) {
+                                    cudaStream_t s, const uint8_t* Be, int64_t ldbe) {
   const int64_t lds = fqt1_packed_words(M);
   CUtensorMap ma, mb;
-  if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, M, capacity, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&mb, Sx, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, kCodesStageK / 32, 128,
-                CU_TENSOR_MAP_SWIZZLE_NONE))
+  if (!make_map(&ma, Q, CU_TENSOR_MAP_DATA_TYPE_UINT8, M, capacity, ldq, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B))
     return cudaErrorInvalidValue;
+  if (Be) {  // e4m3 sign(X_u)^T rows [K][ldbe] bytes: 128 x 128 boxes, 128-byte swizzle
+    if (!make_map(&mb, Be, CU_TENSOR_MAP_DATA_TYPE_UINT8, M, K, ldbe, kBK, 128, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+  } else if (!make_map(&mb, Sx, CU_TENSOR_MAP_DATA_TYPE_UINT32, lds, K, lds * 4, kCodesStageK / 32, 128,
+                       CU_TENSOR_MAP_SWIZZLE_NONE)) {
+    return cudaErrorInvalidValue;
+  }
   TcArgs a{};
   a.M = capacity; a.N = K; a.L = M; a.count = count; a.rows_per_count = 1;
   a.k_tiles = (int)((M + kCodesStageK - 1) / kCodesStageK);
   a.tiles_per_split = (a.k_tiles + splits - 1) / splits;
   a.epi = EPI_CRED; a.acc = acc; a.y = dw; a.ldo = K; a.kept_idx = kept_idx; a.scale = scale; a.zero = zero;
   a.cs = cs; a.status = status; a.slot_of_group = slot_of_group; a.D = D;
+  if (Be) {
+    if (bits == 8) return launch_tc<true, true, 128, false, 2>(ma, mb, a, splits, s, nullptr, nullptr, true);
+    return launch_tc<true, false, 128, false, 2 | 8>(ma, mb, a, splits, s, nullptr, nullptr, true);
+  }
   if (bits == 8) return launch_tc<true, true, 128>(ma, mb, a, splits, s, nullptr, nullptr, true);
   return launch_tc<true, false, 128, false, 8>(ma, mb, a, splits, s, nullptr, nullptr, true);
 }
@@ -1457,11 +1507,11 @@ cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int6
                                    int64_t rows_per_count, const uint32_t* Sg, int64_t n_s, int64_t L, int epi,
                                    int splits, int32_t* acc, float* out, int64_t ldo, const int32_t* kept_idx,
                                    const float* scale, const float* zero, const int32_t* cs, int64_t rpg,
-                                   int32_t* status, cudaStream_t s) {
+                                   int32_t* status, cudaStream_t s, const uint8_t* Be, int64_t ldbe) {
   TcArgs a{};
   a.acc = acc; a.y = out; a.ldo = ldo; a.kept_idx = kept_idx; a.scale = scale; a.zero = zero; a.cs = cs;
   a.rpg = rpg; a.status = status;
-  return launch_codes_tc(bits, Q, ldq, max_rows, count, rows_per_count, Sg, n_s, L, epi, splits, a, s);
+  return launch_codes_tc(bits, Q, ldq, max_rows, count, rows_per_count, Sg, n_s, L, epi, splits, a, s, Be, ldbe);
 }
 
 }  // namespace fqt1

@@ -572,7 +572,28 @@ struct UnfoldSameArgs {
   int guard;     // zero words before and after the region
   uint32_t rep;  // W divides 32: replicates a W-bit row pattern over 32 bits (1 for W = 32); else 0
   FastDiv div_khw, div_kw;
+  // optional e4m3 copies of the signs (+1 = 0x38, -1 = 0xB8): rows [M][ld_row_e] (row r = pixel,
+  // byte k) and columns [K][ld_col_e] (row k, byte r); the bytes from the valid length to the
+  // next multiple of 16 are written as 0
+  uint8_t* row_e4m3;
+  uint8_t* col_e4m3;
+  int64_t ld_row_e, ld_col_e, M;
 };
+
+// 16 signs (bits 0..15 of w) as 16 e4m3 bytes, the bytes at or past `valid` zero.
+__device__ __forceinline__ uint4 e4m3_signs16(uint32_t w, int valid) {
+  uint4 v = make_uint4(e4m3_signs4(w & 15u), e4m3_signs4((w >> 4) & 15u), e4m3_signs4((w >> 8) & 15u),
+                       e4m3_signs4((w >> 12) & 15u));
+  if (valid < 16) {
+    uint32_t* p = &v.x;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int keep = min(max(valid - 4 * q, 0), 4);  // bytes of word q that stay
+      p[q] &= keep == 4 ? 0xFFFFFFFFu : ((1u << (8 * keep)) - 1u);
+    }
+  }
+  return v;
+}
 
 __device__ __forceinline__ uint32_t bit_range(int lo, int hi) {  // bits lo .. hi - 1 of a word
   lo = max(lo, 0);
@@ -672,7 +693,7 @@ __global__ void __launch_bounds__(256) unfold_same_kernel(UnfoldSameArgs a) {
       }
       colw = (uint32_t)(v >> o) & bit_range(plo - p0, phi - p0) & cmask;
     }
-    if (a.row_bits) {  // uniform: a caller that needs only the column packing skips the transposes
+    if (a.row_bits || a.row_e4m3) {  // uniform: a caller that needs only the column packing skips the transposes
       const uint32_t roww = warp_transpose32(colw, lane);
       const int px = 32 * s + lane;
       rw_s[px * 8 + (warp ^ ((px >> 2) & 7))] = roww;
@@ -695,6 +716,33 @@ __global__ void __launch_bounds__(256) unfold_same_kernel(UnfoldSameArgs a) {
       if (px < nimg * a.HW && wbase + 4 * h < a.row_words) {
         const uint4 v = unswizzle4(*reinterpret_cast<const uint4*>(rw_s + px * 8 + 4 * (h ^ (sw >> 2))), sw & 3);
         *reinterpret_cast<uint4*>(a.row_bits + ((int64_t)n_lo * a.HW + px) * a.row_words + wbase + 4 * h) = v;
+      }
+    }
+  }
+  if (a.row_e4m3) {  // 16 bytes per chunk, 16 chunks (256 columns) per pixel
+    for (int e = threadIdx.x; e < 16 * TM; e += 256) {
+      const int px = e >> 4, ch = e & 15;
+      const int64_t kc = (int64_t)k0 + 16 * ch;
+      if (px < nimg * a.HW && kc < a.K) {
+        const int sw = (px >> 2) & 7;
+        const uint32_t word = rw_s[px * 8 + ((ch >> 1) ^ sw)] >> (16 * (ch & 1));
+        const uint4 v = e4m3_signs16(word, (int)(a.K - kc < 16 ? a.K - kc : 16));
+        *reinterpret_cast<uint4*>(a.row_e4m3 + ((int64_t)n_lo * a.HW + px) * a.ld_row_e + kc) = v;
+      }
+    }
+  }
+  if (a.col_e4m3) {  // TM bytes per column k: a warp writes four columns' contiguous runs
+    constexpr int kChunks = TM / 16;
+    const int64_t p0 = (int64_t)blockIdx.y * TM;
+    for (int e = threadIdx.x; e < 256 * kChunks; e += 256) {
+      const int kl = e / kChunks, ch = e % kChunks;
+      const int64_t pc = p0 + 16 * ch;
+      if (k0 + kl < k1 && pc < a.M) {
+        const int z = (kl >> kZShift) & (NSUB - 1);
+        const int wi = ch >> 1;  // pixel word of the chunk
+        const uint32_t word = cw_s[kl * NSUB + (wi ^ z)] >> (16 * (ch & 1));
+        const uint4 v = e4m3_signs16(word, (int)(a.M - pc < 16 ? a.M - pc : 16));
+        *reinterpret_cast<uint4*>(a.col_e4m3 + (int64_t)(k0 + kl) * a.ld_col_e + pc) = v;
       }
     }
   }
@@ -970,10 +1018,11 @@ static int unfold_bits_tm(int N, int C, int H, int W, int kh, int kw, int stride
 // as [N][C][ceil(H W / 32)] words; shapes that only the gather path serves are unsupported there).
 static fqt1_status im2col_impl(const float* x, const uint32_t* planes, int32_t N, int32_t C, int32_t H, int32_t W,
                                int32_t kh, int32_t kw, int32_t stride, int32_t pad, uint32_t* row_bits,
-                               uint32_t* col_bits, int32_t* colsum, void* stream) {
+                               uint32_t* col_bits, int32_t* colsum, void* stream, uint8_t* row_e4m3 = nullptr,
+                               int64_t ld_re = 0, uint8_t* col_e4m3 = nullptr, int64_t ld_ce = 0) {
   if ((!x && !planes) || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 || pad < 0)
     return FQT1_ERR_INVALID_ARG;
-  if (!row_bits && !col_bits && !colsum) return FQT1_ERR_INVALID_ARG;
+  if (!row_bits && !col_bits && !colsum && !row_e4m3 && !col_e4m3) return FQT1_ERR_INVALID_ARG;
   const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
   if (H + 2 * pad < kh || W + 2 * pad < kw || Ho < 1 || Wo < 1) return FQT1_ERR_INVALID_ARG;
   if ((x && !aligned16(x)) || (row_bits && !aligned16(row_bits)) || (col_bits && !aligned16(col_bits)) ||
@@ -985,10 +1034,19 @@ static fqt1_status im2col_impl(const float* x, const uint32_t* planes, int32_t N
   // region of a tile of tm pixels: images it may touch x channels of 256 columns x whole planes.
   const int64_t Mi = (int64_t)N * Ho * Wo, Ki = (int64_t)C * kh * kw;
   const bool same = stride == 1 && kh == kw && kh == 2 * pad + 1 && (Ho * Wo) % 32 == 0;
+  const bool e4m3 = row_e4m3 || col_e4m3;
+  if (e4m3) {  // only the whole-image Unfolder writes the byte copies
+    if (!unfold_same_fits(N, C, H, W, kh, kw, stride, pad)) return FQT1_ERR_UNSUPPORTED;
+    if ((row_e4m3 && (ld_re < (Ki + 15) / 16 * 16 || ld_re % 16)) ||
+        (col_e4m3 && (ld_ce < (Mi + 15) / 16 * 16 || ld_ce % 16)))
+      return FQT1_ERR_INVALID_ARG;
+    if ((row_e4m3 && !aligned16(row_e4m3)) || (col_e4m3 && !aligned16(col_e4m3))) return FQT1_ERR_MISALIGNED;
+  }
   if (unfold_same_fits(N, C, H, W, kh, kw, stride, pad)) {
     // whole images per tile: the contiguous-region Unfolder
     UnfoldSameArgs u;
     u.x = x; u.planes = planes; u.row_bits = row_bits; u.col_bits = col_bits; u.colsum = colsum;
+    u.row_e4m3 = row_e4m3; u.col_e4m3 = col_e4m3; u.ld_row_e = ld_re; u.ld_col_e = ld_ce; u.M = Mi;
     u.row_words = fqt1_packed_words(Ki); u.col_words = fqt1_packed_words(Mi);
     u.N = N; u.C = C; u.H = H; u.W = W; u.pad = pad; u.kw = kw; u.khw = kh * kw; u.K = (int)Ki; u.HW = H * W;
     u.dw = H * W / 32;
@@ -1019,6 +1077,7 @@ static fqt1_status im2col_impl(const float* x, const uint32_t* planes, int32_t N
       return FQT1_OK;
     }
   }
+  if (e4m3) return FQT1_ERR_UNSUPPORTED;
   if (const int tm = unfold_bits_tm(N, C, H, W, kh, kw, stride, pad)) {
     // 128-pixel tiles (smaller only when the input region does not fit): fewer CTAs, each
     // amortizing its region set-up over more output words
@@ -1150,6 +1209,14 @@ extern "C" fqt1_status fqt1_im2col(const float* x, int32_t N, int32_t C, int32_t
                                    int32_t* colsum, void* stream) {
   if (!x) return FQT1_ERR_INVALID_ARG;
   return im2col_impl(x, nullptr, N, C, H, W, kh, kw, stride, pad, row_bits, col_bits, colsum, stream);
+}
+
+extern "C" fqt1_status fqt1_im2col_e4m3(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh,
+                                        int32_t kw, int32_t stride, int32_t pad, uint8_t* x_row, int64_t ld_row,
+                                        uint8_t* x_col, int64_t ld_col, int32_t* colsum, void* stream) {
+  if (!x || (!x_row && !x_col)) return FQT1_ERR_INVALID_ARG;
+  return im2col_impl(x, nullptr, N, C, H, W, kh, kw, stride, pad, nullptr, nullptr, colsum, stream, x_row, ld_row,
+                     x_col, ld_col);
 }
 
 extern "C" fqt1_status fqt1_im2col_planes(const uint32_t* planes, int32_t N, int32_t C, int32_t H, int32_t W,

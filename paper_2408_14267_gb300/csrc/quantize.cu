@@ -540,8 +540,6 @@ __global__ void __launch_bounds__(NT) select_kernel(SelectArgs a0, SelectArgs a1
 }
 
 // --------------------------------------------------------------- quantize
-constexpr int kQRows = 32, kQCols = 128;
-
 struct QBranch {
   const float* zmin;     // [n] group minima
   const float* range;    // [n] group ranges
@@ -586,41 +584,110 @@ struct QuantArgs {
   FastDiv div_rpg;  // row -> sample group (rows < 2^31)
 };
 
-// Quantization of one 32 x 128 tile of G = gY * gamma for both branches (Sec. 5.3).
-//  - Warps 0-7 load the tile (warp w: rows 4w .. 4w+3, lane l: columns 4l .. 4l+3) and the
-//    per-row and per-column constants, every load unconditional so that all are in flight
-//    together.
+// Tile shape of the quantize pass: LPC lanes of 4 columns span kCols columns of G, a warp-wide
+// load covers kRW = 32 / LPC rows, and each quantizing thread holds 4 x 4 values of a tile
+// (kRows x kCols = 4096 elements for every LPC).  The narrow shapes (LPC 16 or 8) keep every
+// lane busy when D <= 64, where the full-width one would leave half or three quarters idle.
+template <int LPC>
+struct QShape {
+  static constexpr int kCols = 4 * LPC;
+  static constexpr int kRW = 32 / LPC;       // rows of one warp-wide load
+  static constexpr int kWarpRows = 4 * kRW;  // rows of one warp per tile
+  static constexpr int kRows = kQWarps * kWarpRows;
+};
+
+// The values one lane holds for one tile: rows rw + kRW i (i < 4), columns c0 .. c0 + 3.
+struct QRows {
+  float v[4][4];
+};
+
+// Every load of a lane's tile, unconditional (clamped rows and columns), so that all of them
+// are in flight together.
+template <bool VEC, int RW>
+__device__ __forceinline__ void quant_load(const QuantArgs& a, int64_t rw, int64_t c0, bool cv0, QRows& t) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int64_t rc = min(rw + (int64_t)i * RW, a.M - 1);
+    if (VEC) {
+      const float4 x = __ldg(reinterpret_cast<const float4*>(a.g + rc * a.D + (cv0 ? c0 : 0)));
+      t.v[i][0] = x.x; t.v[i][1] = x.y; t.v[i][2] = x.z; t.v[i][3] = x.w;
+    } else {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) t.v[i][q] = __ldg(a.g + rc * a.D + min(c0 + q, a.D - 1));
+    }
+  }
+}
+
+// The sample-branch constants of a lane's rows rw + RW i: slot (-1: pruned, or past M), row in
+// its group, range and zero point.  The loads are issued together and hit L1 / L2.
+template <int RW>
+__device__ __forceinline__ void quant_rows(const QuantArgs& a, int64_t rw, int32_t (&slot)[4], int32_t (&rem)[4],
+                                           float (&rg)[4], float (&zm)[4]) {
+  // one division for the first row; the next rows step by RW (at most one group boundary per
+  // step when rpg >= RW, else a division each)
+  const uint32_t r0 = (uint32_t)min(rw, a.M - 1);
+  uint32_t gi = a.div_rpg.div(r0), rr = r0 - gi * (uint32_t)a.rpg;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int64_t r = rw + (int64_t)i * RW;
+    if (i > 0) {
+      if (a.rpg >= RW) {
+        rr += RW;
+        if (rr >= (uint32_t)a.rpg) { rr -= (uint32_t)a.rpg; ++gi; }
+      } else {
+        const uint32_t rc = (uint32_t)min(r, a.M - 1);
+        gi = a.div_rpg.div(rc);
+        rr = rc - gi * (uint32_t)a.rpg;
+      }
+    }
+    rem[i] = (int32_t)rr;
+    const bool ls = r < a.M;
+    slot[i] = ldg_sel(a.s.slot, (int64_t)gi, ls, -1, a.g);
+    rg[i] = ldg_sel(a.s.range, (int64_t)gi, ls, 0.f, a.g);
+    zm[i] = ldg_sel(a.s.zmin, (int64_t)gi, ls, 0.f, a.g);
+  }
+}
+
+// Codes of the tiles of G = gY * gamma for both branches (Sec. 5.3).
+//  - Warps 0-7 quantize.  A CTA takes one column tile and every gridDim.y-th row tile (the
+//    host sizes the grid to about one resident wave), and issues the next tile's loads before
+//    it rounds the current one, so that every lane keeps two tiles of G in flight.
 //  - PSQ: rows of kept sample groups; element (m, j) takes word m D + j of stream 0, so one
 //    Philox block gives a lane's 4 columns of a row.
-//  - PCQ: the tile goes to shared memory and the kept columns of the tile are listed; one
-//    thread per (kept column, 4 rows) draws one Philox block (words j M + m .. + 3 of stream
-//    1) and forms the 4 codes, so no rounding is spent on pruned channels.
-//  - Warp 8 lists the kept columns with their constants (and signals barrier 1 without
-//    waiting), then computes the per-slot S' and Z' in float64 beside the quantizing warps.
-template <bool VEC>
-__global__ void __launch_bounds__(32 * (kQWarps + 1), 4) quantize_kernel(QuantArgs a) {
+//  - PCQ: the tile goes to shared memory; one thread per (kept column, 4 rows) draws one
+//    Philox block (words j M + m .. + 3 of stream 1) and forms the 4 codes, so no rounding is
+//    spent on pruned channels.  The codes are staged in shared memory and written with the
+//    samples contiguous.
+//  - Warp 8 lists the kept columns of the column tile with their constants once (the list is
+//    the same for every row tile), signals barrier 1 without waiting, then computes the
+//    per-slot S' and Z' in float64 beside the quantizing warps.
+//  - PIPE (row tiles beyond one resident wave): the next tile's loads are issued before the
+//    current tile is rounded; the extra registers leave two CTAs per SM.  Without it a CTA
+//    takes one tile at a time and four CTAs fit on an SM.
+template <int LPC, bool VEC, bool PIPE>
+__global__ void __launch_bounds__(32 * (kQWarps + 1), PIPE ? 2 : 4) quantize_kernel(QuantArgs a) {
+  using S = QShape<LPC>;
   // the dependent (the grad_input product, a leaf of the step) is not released early either:
   // its CTAs would wait on SMs that the grad_weight product, which also waits for this
   // kernel, can use
   FQT1_PDL_WAIT();
-  __shared__ __align__(16) float gt[kQRows][kQCols + 4];  // the tile of G * gamma
-  __shared__ uint32_t tile[kQCols][kQRows / 4 + 1];       // codes of kept column j, 4 rows per word
-  __shared__ int32_t klist[kQCols], kslot[kQCols];        // kept column j: tile column, slot
-  __shared__ float kz[kQCols], kinv[kQCols];              // its Z and B / R (negative: degenerate)
+  __shared__ __align__(16) float gt[S::kRows][S::kCols + 4];  // the tile of G * gamma
+  __shared__ uint32_t tile[S::kCols][S::kRows / 4 + 1];       // codes of kept column j, 4 rows per word
+  __shared__ int32_t klist[S::kCols], kslot[S::kCols];        // kept column j: tile column, slot
+  __shared__ float kz[S::kCols], kinv[S::kCols];              // its Z and B / R (negative: degenerate)
   __shared__ int32_t nk_s;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t cb = (int64_t)blockIdx.x * kQCols;
-  const int64_t c0 = cb + lane * 4;
-  const int64_t r0 = (int64_t)blockIdx.y * kQRows;
+  const int64_t cb = (int64_t)blockIdx.x * S::kCols;
   if (warp == kQWarps) {
     if (a.do_pcq) {
-      // the kept columns of the tile in ascending order (lane l: columns 4l .. 4l+3)
+      // the kept columns of the tile in ascending order (lane l: tile columns 4l .. 4l+3)
+      const int64_t c0 = cb + lane * 4;
       int32_t cslot[4];
       float crg[4], zc[4];
       int mine = 0;
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const bool lc = c0 + q < a.D;
+        const bool lc = 4 * lane + q < S::kCols && c0 + q < a.D;
         cslot[q] = ldg_sel(a.c.slot, c0 + q, lc, -1, a.g);
         crg[q] = ldg_sel(a.c.range, c0 + q, lc, 0.f, a.g);
         zc[q] = ldg_sel(a.c.zmin, c0 + q, lc, 0.f, a.g);
@@ -652,8 +719,8 @@ __global__ void __launch_bounds__(32 * (kQWarps + 1), 4) quantize_kernel(QuantAr
     slot_constants(a.s, a.c, a.do_psq != 0, a.do_pcq != 0, cta, ncta, lane);
     return;
   }
-  // every load first (gamma, the row slots, ranges and zero points, the 4 x 4 gradient
-  // values), so that they are in flight together instead of one dependent round trip each
+  const int sub = lane / LPC;
+  const int64_t c0 = cb + (lane % LPC) * 4;
   float gam[4];
   bool cv[4];
 #pragma unroll
@@ -662,108 +729,110 @@ __global__ void __launch_bounds__(32 * (kQWarps + 1), 4) quantize_kernel(QuantAr
     cv[q] = c < a.D;
     gam[q] = ldg_sel(a.gamma, c, a.gamma && cv[q], 1.0f, a.g);
   }
-  const int64_t rb = r0 + warp * 4;  // this warp's 4 rows
-  int32_t sslots[4];
-  int32_t srem[4];  // row within its sample group
-  float srg[4], szm[4];
-  {
-    const int64_t rc = min(rb, a.M - 1);
-    int64_t gi = a.div_rpg.div((uint32_t)rc), rem = rc - gi * a.rpg;
+  // row tiles blockIdx.y, + gridDim.y, ...: strided, so that every CTA gets its share of the
+  // kept sample groups (their PSQ rounding costs several times a pruned tile's work)
+  const int64_t row_tiles = (a.M + S::kRows - 1) / S::kRows;
+  const int64_t rt0 = blockIdx.y, rstep = gridDim.y;
+  const int64_t lrow = (int64_t)warp * S::kWarpRows + sub;  // this lane's first row in a tile
+  // without PIPE the host launches one CTA per row tile, and the tile is not a loop
+  QRows cur, nxt;
+  auto do_tile = [&](int64_t rt) {
+    const int64_t r0 = rt * S::kRows, rw = r0 + lrow;
+    int32_t sslot[4], srem[4];
+    float srg[4], szm[4];
+    if (a.do_psq) quant_rows<S::kRW>(a, rw, sslot, srem, srg, szm);
+    if (PIPE && rt + rstep < row_tiles) quant_load<VEC, S::kRW>(a, rw + rstep * S::kRows, c0, cv[0], nxt);
+    if (a.gamma) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      if (i > 0 && ++rem == a.rpg) { rem = 0; ++gi; }
-      srem[i] = (int32_t)rem;
-      const bool ls = a.do_psq && rb + i < a.M;
-      sslots[i] = ldg_sel(a.s.slot, gi, ls, -1, a.g);
-      srg[i] = ldg_sel(a.s.range, gi, ls, 0.f, a.g);
-      szm[i] = ldg_sel(a.s.zmin, gi, ls, 0.f, a.g);
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) cur.v[i][q] = __fmul_rn(cur.v[i][q], gam[q]);
     }
-  }
-  float vv[4][4];
+    // PSQ: kept rows; element (m, j) takes word m*D + j of stream 0 (one block = 4 columns)
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {  // unconditional loads from clamped rows / columns
-    const int64_t r = min(rb + i, a.M - 1);
-    if (VEC) {
-      const float4 t = __ldg(reinterpret_cast<const float4*>(a.g + r * a.D + (cv[0] ? c0 : 0)));
-      vv[i][0] = t.x; vv[i][1] = t.y; vv[i][2] = t.z; vv[i][3] = t.w;
-    } else {
+    for (int i = 0; i < 4 && a.do_psq; ++i) {
+      if (sslot[i] < 0) continue;
+      const int64_t r = rw + (int64_t)i * S::kRW;
+      const float rs = srg[i], zs = szm[i];
+      const float inv = __fdiv_rn(a.s.B, rs);
+      const bool deg = !(rs > 0.0f) || !isfinite(inv);
+      const uint64_t e0 = (uint64_t)r * (uint64_t)a.D + (uint64_t)c0;
+      uint8_t* dst = a.s.codes + ((int64_t)sslot[i] * a.rpg + srem[i]) * a.s.ld + c0;
+      if (VEC) {
+        if (cv[0]) {
+          const U32x4 p = philox_block(a.s.seed, kStreamSrPsq, e0 >> 2);
+          const uint32_t packed = sr_code(cur.v[i][0], zs, inv, a.s.B, deg, p.x) |
+                                  (sr_code(cur.v[i][1], zs, inv, a.s.B, deg, p.y) << 8) |
+                                  (sr_code(cur.v[i][2], zs, inv, a.s.B, deg, p.z) << 16) |
+                                  (sr_code(cur.v[i][3], zs, inv, a.s.B, deg, p.w) << 24);
+          *reinterpret_cast<uint32_t*>(dst) = packed;
+        }
+      } else {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) vv[i][q] = __ldg(a.g + r * a.D + min(c0 + q, a.D - 1));
-    }
-  }
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-#pragma unroll
-    for (int q = 0; q < 4; ++q) vv[i][q] = a.gamma ? __fmul_rn(vv[i][q], gam[q]) : vv[i][q];
-  }
-  // PSQ: kept rows; element (m, j) takes word m*D + j of stream 0 (one block = 4 columns)
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int64_t r = rb + i;
-    const int32_t sslot = sslots[i];
-    if (sslot < 0) continue;
-    const float rs = srg[i], zs = szm[i];
-    const float inv = __fdiv_rn(a.s.B, rs);
-    const bool deg = !(rs > 0.0f) || !isfinite(inv);
-    const uint64_t e0 = (uint64_t)r * (uint64_t)a.D + (uint64_t)c0;
-    uint8_t* dst = a.s.codes + ((int64_t)sslot * a.rpg + srem[i]) * a.s.ld + c0;
-    if (VEC) {
-      if (cv[0]) {
-        const U32x4 p = philox_block(a.s.seed, kStreamSrPsq, e0 >> 2);
-        const uint32_t packed = sr_code(vv[i][0], zs, inv, a.s.B, deg, p.x) |
-                                (sr_code(vv[i][1], zs, inv, a.s.B, deg, p.y) << 8) |
-                                (sr_code(vv[i][2], zs, inv, a.s.B, deg, p.z) << 16) |
-                                (sr_code(vv[i][3], zs, inv, a.s.B, deg, p.w) << 24);
-        *reinterpret_cast<uint32_t*>(dst) = packed;
+        for (int q = 0; q < 4; ++q)
+          if (cv[q])
+            dst[q] = (uint8_t)sr_code(cur.v[i][q], zs, inv, a.s.B, deg, philox_word(a.s.seed, kStreamSrPsq, e0 + q));
       }
-    } else {
-#pragma unroll
-      for (int q = 0; q < 4; ++q)
-        if (cv[q]) dst[q] = (uint8_t)sr_code(vv[i][q], zs, inv, a.s.B, deg, philox_word(a.s.seed, kStreamSrPsq, e0 + q));
     }
-  }
-  if (!a.do_pcq) return;
-  // stage the tile; barrier 1 also waits for warp 8's list of kept columns
+    if (a.do_pcq) {
+      // stage the tile; on the first tile barrier 1 also waits for warp 8's list of kept
+      // columns, later tiles need only the quantizing warps (barrier 3)
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
-    *reinterpret_cast<float4*>(&gt[4 * warp + i][4 * lane]) = make_float4(vv[i][0], vv[i][1], vv[i][2], vv[i][3]);
-  asm volatile("bar.sync 1, %0;" ::"n"(32 * (kQWarps + 1)) : "memory");
-  const int nk = nk_s;
-  for (int u = threadIdx.x; u < nk * (kQRows / 4); u += 32 * kQWarps) {
-    const int j = u / (kQRows / 4), g = u % (kQRows / 4);
-    const int col = klist[j];
-    const int64_t rq = r0 + 4 * g;
-    const float z = kz[j], inv = kinv[j];
-    const bool deg = !(inv > 0.0f);
-    const uint64_t e = (uint64_t)(cb + col) * (uint64_t)a.M + (uint64_t)rq;
-    uint32_t w[4];
-    if ((a.M & 3) == 0) {
-      const U32x4 p = philox_block(a.c.seed, kStreamSrPcq, e >> 2);
-      w[0] = p.x; w[1] = p.y; w[2] = p.z; w[3] = p.w;
-    } else {
+      for (int i = 0; i < 4; ++i)
+        *reinterpret_cast<float4*>(&gt[lrow + i * S::kRW][4 * (lane % LPC)]) =
+            make_float4(cur.v[i][0], cur.v[i][1], cur.v[i][2], cur.v[i][3]);
+      if (rt == rt0) asm volatile("bar.sync 1, %0;" ::"n"(32 * (kQWarps + 1)) : "memory");
+      else asm volatile("bar.sync 3, %0;" ::"n"(32 * kQWarps) : "memory");
+      const int nk = nk_s;
+      for (int u = threadIdx.x; u < nk * (S::kRows / 4); u += 32 * kQWarps) {
+        const int j = u / (S::kRows / 4), g = u % (S::kRows / 4);
+        const int col = klist[j];
+        const int64_t rq = r0 + 4 * g;
+        const float z = kz[j], inv = kinv[j];
+        const bool deg = !(inv > 0.0f);
+        const uint64_t e = (uint64_t)(cb + col) * (uint64_t)a.M + (uint64_t)rq;
+        uint32_t w[4];
+        if ((a.M & 3) == 0) {
+          const U32x4 p = philox_block(a.c.seed, kStreamSrPcq, e >> 2);
+          w[0] = p.x; w[1] = p.y; w[2] = p.z; w[3] = p.w;
+        } else {
 #pragma unroll
-      for (int i = 0; i < 4; ++i) w[i] = philox_word(a.c.seed, kStreamSrPcq, e + i);
+          for (int i = 0; i < 4; ++i) w[i] = philox_word(a.c.seed, kStreamSrPcq, e + i);
+        }
+        uint32_t word = 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (rq + i < a.M) word |= sr_code(gt[4 * g + i][col], z, inv, a.c.B, deg, w[i]) << (8 * i);
+        tile[j][g] = word;
+      }
+      asm volatile("bar.sync 2, %0;" ::"n"(32 * kQWarps) : "memory");
+      // kept column j: the codes of rows r0 .. r0 + kRows - 1 as 16-byte stores
+      for (int t = threadIdx.x; t < nk * (S::kRows / 16); t += 32 * kQWarps) {
+        const int j = t / (S::kRows / 16), h = t % (S::kRows / 16);
+        const int64_t rb = r0 + 16 * h;
+        if (rb < a.M && rb + 16 <= a.c.ld) {
+          uint4 val;
+          val.x = tile[j][4 * h + 0];
+          val.y = tile[j][4 * h + 1];
+          val.z = tile[j][4 * h + 2];
+          val.w = tile[j][4 * h + 3];
+          *reinterpret_cast<uint4*>(a.c.codes + (int64_t)kslot[j] * a.c.ld + rb) = val;
+        }
+      }
     }
-    uint32_t word = 0;
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-      if (rq + i < a.M) word |= sr_code(gt[4 * g + i][col], z, inv, a.c.B, deg, w[i]) << (8 * i);
-    tile[j][g] = word;
-  }
-  asm volatile("bar.sync 2, %0;" ::"n"(32 * kQWarps) : "memory");
-  // kept column j: the codes of rows r0 .. r0 + 31 as two 16-byte stores
-  for (int t = threadIdx.x; t < 2 * nk; t += 32 * kQWarps) {
-    const int j = t >> 1, half = t & 1;
-    const int64_t rb = r0 + 16 * half;
-    if (rb < a.M && rb + 16 <= a.c.ld) {
-      uint4 val;
-      val.x = tile[j][4 * half + 0];
-      val.y = tile[j][4 * half + 1];
-      val.z = tile[j][4 * half + 2];
-      val.w = tile[j][4 * half + 3];
-      *reinterpret_cast<uint4*>(a.c.codes + (int64_t)kslot[j] * a.c.ld + rb) = val;
+  };
+  if (rt0 < row_tiles) quant_load<VEC, S::kRW>(a, rt0 * S::kRows + lrow, c0, cv[0], cur);
+  if (PIPE) {
+#pragma unroll 1
+    for (int64_t rt = rt0; rt < row_tiles; rt += rstep) {
+      do_tile(rt);
+      cur = nxt;
     }
+  } else if (rt0 < row_tiles) {
+    do_tile(rt0);
   }
+  // a CTA without row tiles (the host never launches one) still meets warp 8's arrive
+  if (a.do_pcq && rt0 >= row_tiles) asm volatile("bar.sync 1, %0;" ::"n"(32 * (kQWarps + 1)) : "memory");
 }
 
 }  // namespace fqt1
@@ -790,19 +859,31 @@ extern "C" size_t fqt1_workspace_size(int32_t which, int64_t M, int64_t D, int64
   return 0;
 }
 
-// Resident range CTAs on the whole GPU (SMs x CTAs per SM) for each kernel variant, per device.
-static int range_wave(void (*rk)(RangeArgs), int variant) {
-  static std::atomic<int> cache[64][4];
+// Resident CTAs on the whole GPU (SMs x CTAs per SM) of a kernel variant, per device; `slot`
+// names the variant in the cache (0-3 range pass, 4-7 pipelined quantize pass, 8-11 quantize
+// pass one tile per CTA).
+template <class Args>
+static int resident_wave(void (*k)(Args), int threads, int slot) {
+  static std::atomic<int> cache[64][12];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
-  int w = cache[dev][variant].load(std::memory_order_relaxed);
+  int w = cache[dev][slot].load(std::memory_order_relaxed);
   if (w > 0) return w;
-  int sms = 152, per_sm = 4;
+  int sms = 152, per_sm = 1;
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rk, 256, 0) != cudaSuccess || per_sm < 1) per_sm = 1;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, threads, 0) != cudaSuccess || per_sm < 1) per_sm = 1;
   w = sms * per_sm;
-  cache[dev][variant].store(w, std::memory_order_relaxed);
+  cache[dev][slot].store(w, std::memory_order_relaxed);
   return w;
+}
+
+// Rows of a contiguous run per CTA so that the CTAs of `cols` column tiles fill about one
+// resident wave; the grid's row extent then leaves no CTA without a tile.
+static void row_runs(int64_t tiles, int64_t cols, int wave, int64_t* per_cta, int64_t* ctas) {
+  const int64_t want = std::max<int64_t>(1, wave / std::max<int64_t>(1, cols));
+  *per_cta = (tiles + want - 1) / want;
+  if (*per_cta < 1) *per_cta = 1;
+  *ctas = std::max<int64_t>(1, (tiles + *per_cta - 1) / *per_cta);
 }
 
 // Shared driver of both entry points.
@@ -827,7 +908,7 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
   if (!ws || ws_bytes < need) return FQT1_ERR_WORKSPACE;
   if (!aligned16(ws)) return FQT1_ERR_MISALIGNED;
   if (M * D >= (1ll << 46)) return FQT1_ERR_UNSUPPORTED;
-  if ((M + kQRows - 1) / kQRows > 65535) return FQT1_ERR_UNSUPPORTED;
+  if (M >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;  // rows go through 32-bit multiply-high division
 
   uint32_t* smin = static_cast<uint32_t*>(ws);
   uint32_t* cmin = smin + ns;
@@ -849,8 +930,10 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
                         : vec ? range_kernel<32, true> : range_kernel<32, false>;
   const int tile = lpr == 8 ? RangeShape<8>::kTile : lpr == 16 ? RangeShape<16>::kTile : RangeShape<32>::kTile;
   const int64_t rcols = (D + 4 * lpr - 1) / (4 * lpr), rtiles = (M + tile - 1) / tile;
-  const int wave = range_wave(rk, lpr == 8 ? 0 : lpr == 16 ? 1 : vec ? 2 : 3);
-  dim3 rgrid((unsigned)rcols, (unsigned)std::min<int64_t>(rtiles, std::max<int64_t>(1, wave / rcols)));
+  const int wave = resident_wave(rk, 256, lpr == 8 ? 0 : lpr == 16 ? 1 : vec ? 2 : 3);
+  int64_t rper = 0, rctas = 0;
+  row_runs(rtiles, rcols, wave, &rper, &rctas);
+  dim3 rgrid((unsigned)rcols, (unsigned)rctas);
   launch_k(rk, rgrid, dim3(256), 0, s, ra);
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
@@ -894,9 +977,25 @@ static fqt1_status quantize_impl(const float* g, int64_t M, int64_t D, const flo
                           (float)((1 << pc->bits) - 1), pc->seed, pcq->kept_idx, pcq->kept_count, pcq->p_hat,
                           pcq->scale, pcq->zero};
   else qa.c = QBranch{};
-  dim3 qgrid((unsigned)((D + kQCols - 1) / kQCols), (unsigned)((M + kQRows - 1) / kQRows));
-  if (vec) launch_k(quantize_kernel<true>, dim3(qgrid), dim3(32 * (kQWarps + 1)), 0, s, qa);
-  else launch_k(quantize_kernel<false>, dim3(qgrid), dim3(32 * (kQWarps + 1)), 0, s, qa);
+  // tile shape: 16 or 8 lanes per row when D is that narrow.  Tiles that fit in one wave of
+  // four CTAs per SM go one per CTA; more tiles go to about one resident wave of pipelined CTAs,
+  // each over every gridDim.y-th row tile
+  const int lpc = !vec ? 32 : D <= 32 ? 8 : D <= 64 ? 16 : 32;
+  const int qrows = lpc == 8 ? QShape<8>::kRows : lpc == 16 ? QShape<16>::kRows : QShape<32>::kRows;
+  const int64_t qcols = (D + 4 * lpc - 1) / (4 * lpc), qtiles = (M + qrows - 1) / qrows;
+  void (*qk1)(QuantArgs) = lpc == 8 ? quantize_kernel<8, true, false>
+                         : lpc == 16 ? quantize_kernel<16, true, false>
+                         : vec ? quantize_kernel<32, true, false> : quantize_kernel<32, false, false>;
+  void (*qkp)(QuantArgs) = lpc == 8 ? quantize_kernel<8, true, true>
+                         : lpc == 16 ? quantize_kernel<16, true, true>
+                         : vec ? quantize_kernel<32, true, true> : quantize_kernel<32, false, true>;
+  const int vslot = lpc == 8 ? 0 : lpc == 16 ? 1 : vec ? 2 : 3;
+  const int wave1 = resident_wave(qk1, 32 * (kQWarps + 1), 8 + vslot);
+  const bool pipe = qtiles * qcols > wave1;
+  void (*qk)(QuantArgs) = pipe ? qkp : qk1;
+  const int qwave = pipe ? resident_wave(qkp, 32 * (kQWarps + 1), 4 + vslot) : wave1;
+  const int64_t qctas = std::min<int64_t>(qtiles, std::max<int64_t>(1, qwave / qcols));
+  launch_k(qk, dim3((unsigned)qcols, (unsigned)qctas), dim3(32 * (kQWarps + 1)), 0, s, qa);
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
   return FQT1_OK;

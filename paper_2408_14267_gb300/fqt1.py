@@ -56,6 +56,9 @@ _SIGS = {
     "fqt1_binarize_pack_e4m3": (C.c_int, [_VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP, _I64, _VP, _I64, _VP]),
     "fqt1_fwd_gemm_e4m3w": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _I64, _VP, _VP, _VP, _VP, _VP]),
     "fqt1_bwd_input_fold_e4m3w": (C.c_int, [_VP, _VP, _I64, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP]),
+    "fqt1_im2col_e4m3": (C.c_int, [_VP] + [_I32] * 8 + [_VP, _I64, _VP, _I64, _VP, _VP]),
+    "fqt1_fwd_gemm_e4m3x": (C.c_int, [_VP, _I64, _VP, _I64, _I64, _I64, _I64, _VP, _VP, _VP, _VP, _VP]),
+    "fqt1_bwd_weight_gemm_e4m3x": (C.c_int, [_VP, _VP, _I64, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
     "fqt1_pack_pixels": (C.c_int, [_VP, _I32, _I32, _I32, _I32, _VP, _VP]),
     "fqt1_pack_planes_nhwc": (C.c_int, [_VP, _I32, _I32, _I32, _I32, _VP, _VP]),
     "fqt1_pack_planes": (C.c_int, [_VP, _I32, _I32, _I32, _I32, _VP, _VP]),
@@ -183,6 +186,24 @@ def binarize_pack_e4m3(x, rows, cols, ld, row_bits, col_bits, colsum, row_e4m3, 
                                          row_e4m3.shape[-1] if row_e4m3 is not None else 0, _p(col_e4m3),
                                          col_e4m3.shape[-1] if col_e4m3 is not None else 0, _s(stream)),
            "fqt1_binarize_pack_e4m3")
+
+
+def im2col_e4m3(x, N, Cin, H, W, kh, kw, stride, pad, x_row=None, x_col=None, colsum=None, stream=None):
+    _check(lib().fqt1_im2col_e4m3(_p(x), N, Cin, H, W, kh, kw, stride, pad, _p(x_row),
+                                  0 if x_row is None else x_row.shape[-1], _p(x_col),
+                                  0 if x_col is None else x_col.shape[-1], _p(colsum), _s(stream)),
+           "fqt1_im2col_e4m3")
+
+
+def fwd_gemm_e4m3x(x_e4m3, w_e4m3, M, D, K, gamma, bias, acc, y, stream=None):
+    _check(lib().fqt1_fwd_gemm_e4m3x(_p(x_e4m3), x_e4m3.shape[-1], _p(w_e4m3), w_e4m3.shape[-1], M, D, K, _p(gamma),
+                                     _p(bias), _p(acc), _p(y), _s(stream)), "fqt1_fwd_gemm_e4m3x")
+
+
+def bwd_weight_gemm_e4m3x(pcq, x_col_e4m3, colsum_x, M, D, K, params, acc, dw, stream=None):
+    _check(lib().fqt1_bwd_weight_gemm_e4m3x(C.byref(pcq.c), _p(x_col_e4m3), x_col_e4m3.shape[-1], _p(colsum_x), M, D,
+                                            K, C.byref(params), _p(acc), _p(dw), _s(stream)),
+           "fqt1_bwd_weight_gemm_e4m3x")
 
 
 def fwd_gemm_e4m3w(sx_row, w_e4m3, M, D, K, gamma, bias, acc, y, stream=None):

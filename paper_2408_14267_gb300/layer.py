@@ -31,7 +31,8 @@ class LayerStep:
     """Buffers and launches of one layer step.  keep_acc=False skips the optional
     int32 copy of the forward accumulators (the benchmark's configuration)."""
 
-    def __init__(self, wl, device="cuda", keep_acc=True, fold=None, implicit=False, e4m3_weights=False):
+    def __init__(self, wl, device="cuda", keep_acc=True, fold=None, implicit=False, e4m3_weights=False,
+                 e4m3_x=False):
         dev = torch.device(device)
         self.kind = wl["kind"]
         self.keep_acc = keep_acc
@@ -83,8 +84,25 @@ class LayerStep:
         if self.implicit:
             self.x_pix = torch.empty(N * H * W, fqt1.packed_words(Cin), **i32)
             self.w_taps = torch.empty(D, wK, **i32)
-        self.sx_row = None if self.implicit else torch.empty(M, wK, **i32)
-        self.sx_col = torch.empty(K, wM, **i32)
+        # e4m3 copies of sign(X_u) (rows for the forward product, columns for grad_weight's),
+        # written by the Unfolder instead of the packed words: both products then load their
+        # sign operand by TMA and expand nothing.  Where the whole-image Unfolder serves the
+        # convolution (fqt1_im2col_path 2), or for a linear layer whose rows are a multiple of 4
+        # floats; the forward then takes the e4m3 copy of sign(W) too
+        u8 = dict(dtype=torch.uint8, device=dev)
+        self.e4m3_x = False
+        if e4m3_x and not self.implicit:
+            if self.kind == "conv":
+                self.e4m3_x = fqt1.im2col_path(N, Cin, H, W, kh, kw, self.stride, self.pad) == 2
+            else:
+                self.e4m3_x = K % 4 == 0
+        if self.e4m3_x:
+            self.x_planes = None
+            self.x8_row = torch.empty(M, fqt1.codes_ld(K), **u8)
+            self.x8_col = torch.empty(K, fqt1.codes_ld(M), **u8)
+            e4m3_weights = True if e4m3_weights is True or e4m3_weights == "fold" else "fwd"
+        self.sx_row = None if self.implicit or self.e4m3_x else torch.empty(M, wK, **i32)
+        self.sx_col = None if self.e4m3_x else torch.empty(K, wM, **i32)
         self.cs_x = torch.empty(K, **i32)
         self.sw_row = None if self.implicit else torch.empty(D, wK, **i32)
         # e4m3 copies of sign(W) (rows for the forward product, columns for the fused Folder's
@@ -93,7 +111,6 @@ class LayerStep:
         # e4m3_weights: True (both products), "fwd" or "fold" (one of them), False
         e_fwd = e4m3_weights is True or e4m3_weights == "fwd"
         e_fold = e4m3_weights is True or e4m3_weights == "fold"
-        u8 = dict(dtype=torch.uint8, device=dev)
         self.w8 = torch.empty(D, fqt1.codes_ld(K), **u8) if e_fwd and not self.implicit else None
         self.wt8 = torch.empty(K, fqt1.codes_ld(D), **u8) if e_fold and self.fold else None
         self.sw_col = torch.empty(K, wD, **i32)
@@ -151,7 +168,14 @@ class LayerStep:
                     fqt1.binarize_pack(self.w, self.D, self.K, self.K, self.sw_row, self.sw_col, self.cs_w, s)
 
             st = [("pack_w", pack_w)]
-            if self.kind == "conv" and self.x_planes is not None:
+            if self.e4m3_x and self.kind == "conv":
+                N, Cin, H, W, kh, kw = self.conv
+                st.append(("im2col", lambda s: fqt1.im2col_e4m3(self.x, N, Cin, H, W, kh, kw, self.stride, self.pad,
+                                                                self.x8_row, self.x8_col, self.cs_x, s)))
+            elif self.e4m3_x:
+                st.append(("pack_x", lambda s: fqt1.binarize_pack_e4m3(self.x, self.M, self.K, self.K, None, None,
+                                                                       self.cs_x, self.x8_row, self.x8_col, s)))
+            elif self.kind == "conv" and self.x_planes is not None:
                 N, Cin, H, W, kh, kw = self.conv
 
                 def unfold(s):
@@ -166,7 +190,10 @@ class LayerStep:
             else:
                 st.append(("pack_x", lambda s: fqt1.binarize_pack(self.x, self.M, self.K, self.K, self.sx_row,
                                                                   self.sx_col, self.cs_x, s)))
-            if self.w8 is not None:
+            if self.e4m3_x:
+                st.append(("fwd_gemm", lambda s: fqt1.fwd_gemm_e4m3x(self.x8_row, self.w8, self.M, self.D, self.K,
+                                                                     self.gamma_fwd, None, self.acc_y, self.y, s)))
+            elif self.w8 is not None:
                 st.append(("fwd_gemm", lambda s: fqt1.fwd_gemm_e4m3w(self.sx_row, self.w8, self.M, self.D, self.K,
                                                                      self.gamma_fwd, None, self.acc_y, self.y, s)))
             else:
@@ -197,9 +224,14 @@ class LayerStep:
             acc = self.acc_dx if self.keep_acc else None
             st.append(("bwd_input_gemm", lambda s: fqt1.bwd_input_gemm(self.psq, self.sw_col, self.cs_w, self.M,
                                                                        self.D, self.K, self.p_s, acc, self.dx, s)))
-        st.append(("bwd_weight_gemm", lambda s: fqt1.bwd_weight_gemm(self.pcq, self.sx_col, self.cs_x, self.M,
-                                                                     self.D, self.K, self.p_c, self.acc_dw, self.dw,
-                                                                     None, s)))
+        if self.e4m3_x:
+            st.append(("bwd_weight_gemm", lambda s: fqt1.bwd_weight_gemm_e4m3x(self.pcq, self.x8_col, self.cs_x,
+                                                                               self.M, self.D, self.K, self.p_c,
+                                                                               self.acc_dw, self.dw, s)))
+        else:
+            st.append(("bwd_weight_gemm", lambda s: fqt1.bwd_weight_gemm(self.pcq, self.sx_col, self.cs_x, self.M,
+                                                                         self.D, self.K, self.p_c, self.acc_dw,
+                                                                         self.dw, None, s)))
         return st
 
     def forward(self, stream=None):

@@ -33,6 +33,14 @@ def unpack_bits(words_i32, n):
     return bits[:, :n].astype(np.int8) * 2 - 1, bits[:, n:]
 
 
+def unpack_e4m3(t, n):
+    """e4m3 sign bytes [rows][ld] -> (+-1 int8 [rows][n], the bytes n .. next multiple of 16)."""
+    b = t.cpu().numpy()
+    v = b[:, :n]
+    assert np.isin(v, (0x38, 0xB8)).all(), "bytes other than +-1 in e4m3 signs"
+    return np.where(v == 0x38, 1, -1).astype(np.int8), b[:, n:(n + 15) // 16 * 16]
+
+
 def linear_case(M, K, D, rpg, bits, mode, seed=0, gamma=True, bits_c=None, mode_c=None):
     rng = np.random.default_rng(seed)
     x = rng.standard_normal((M, K)).astype(np.float32)
@@ -96,13 +104,22 @@ def check_step(w, st, ref):
         assert np.array_equal(sp, om.pixel_signs(w["x"])) and not pad_bits.any(), "sign(X) pixel bits"
         swt, pad_bits = unpack_bits(st.w_taps, K)
         assert np.array_equal(swt, om.tap_major_signs(w["w"])) and not pad_bits.any(), "sign(W) tap-major bits"
+    elif st.e4m3_x:  # e4m3 bytes of sign(X_u): 0x38 (+1), 0xB8 (-1), zeros to the next 16 bytes
+        xr, pad_r = unpack_e4m3(st.x8_row, K)
+        assert np.array_equal(xr, om.sign(x_u)) and not pad_r.any(), "sign(X) e4m3 rows"
+        sw, _ = unpack_bits(st.sw_row, K)
+        assert np.array_equal(sw, om.sign(w_u)), "sign(W) row bits"
     else:
         sx, pad_bits = unpack_bits(st.sx_row, K)
         assert np.array_equal(sx, om.sign(x_u)) and not pad_bits.any(), "sign(X) row bits"
         sw, _ = unpack_bits(st.sw_row, K)
         assert np.array_equal(sw, om.sign(w_u)), "sign(W) row bits"
-    sxc, pad_bits = unpack_bits(st.sx_col, M)
-    assert np.array_equal(sxc, om.sign(x_u).T) and not pad_bits.any(), "sign(X) col bits"
+    if st.e4m3_x:
+        xc, pad_c = unpack_e4m3(st.x8_col, M)
+        assert np.array_equal(xc, om.sign(x_u).T) and not pad_c.any(), "sign(X) e4m3 columns"
+    else:
+        sxc, pad_bits = unpack_bits(st.sx_col, M)
+        assert np.array_equal(sxc, om.sign(x_u).T) and not pad_bits.any(), "sign(X) col bits"
     swc, _ = unpack_bits(st.sw_col, D)
     assert np.array_equal(swc, om.sign(w_u).T), "sign(W) col bits"
     assert np.array_equal(st.cs_x.cpu().numpy(), om.colsum_sign(x_u)), "colsum X"
@@ -465,6 +482,44 @@ def test_e4m3_weights_step_equals_packed_step(name, make):
     a = LayerStep(w, keep_acc=False, e4m3_weights=True)
     b = LayerStep(w, keep_acc=False)
     assert a.w8 is not None and b.w8 is None
+    for st in (a, b):
+        st.dev_status.zero_()
+        st.step()
+    torch.cuda.synchronize()
+    assert torch.equal(a.y, b.y) and torch.equal(a.dx, b.dx) and torch.equal(a.dw, b.dw)
+
+
+E4M3X_CASES = [c for c in CASES if c[0] in ("linear-64x512x512-b2", "conv-resnet18-cifar-8192x2304x256-b4",
+                                             "conv-same-8x8-ragged", "conv-same-16x16-5x5", "conv-same-4x8-1x1",
+                                             "conv-same-8x16-7x7", "conv-same-4x64", "linear-b8-bernoulli",
+                                             "linear-mixed-bits")]
+
+
+@pytest.mark.parametrize("name,make", E4M3X_CASES, ids=[c[0] for c in E4M3X_CASES])
+def test_e4m3_x_step_parity(name, make):
+    """The step with e4m3 copies of sign(X_u) (the Unfolder's byte output, both products' sign
+    operand straight from TMA) against the oracle: bytes, integer sums and outputs."""
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    ref = run_oracle(w)
+    st = LayerStep(w, keep_acc=True, fold=False, e4m3_x=True)
+    assert st.e4m3_x and st.sx_row is None and st.sx_col is None
+    st.dev_status.zero_()
+    st.step()
+    torch.cuda.synchronize()
+    check_step(w, st, ref)
+
+
+@pytest.mark.parametrize("name,make", [CASES[1], CASES[0], FOLD_CASES[2]], ids=[CASES[1][0], CASES[0][0],
+                                                                             FOLD_CASES[2][0]])
+def test_e4m3_x_step_equals_packed_step(name, make):
+    """The benchmark's configuration (fused Folder, no int32 copies) with and without the e4m3
+    copies of sign(X_u): identical y, dx and dW."""
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    a = LayerStep(w, keep_acc=False, e4m3_weights=True, e4m3_x=True)
+    b = LayerStep(w, keep_acc=False)
+    assert a.e4m3_x and not b.e4m3_x
     for st in (a, b):
         st.dev_status.zero_()
         st.step()

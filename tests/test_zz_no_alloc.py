@@ -71,3 +71,14 @@ def test_noalloc_rejects_sizes_beyond_the_scratch():
                                      C.c_void_p(0))
     assert st == 3
     assert b"exceed the built-in scratch" in L.fqt1_last_cuda_error()
+
+
+def test_noalloc_wide_grouping_then_small_call():
+    """A channel grouping of 6000 (the selection needs more than 48 KB of shared memory) with
+    two sample groups, then a small call: the second call must find every key it reads reset."""
+    from test_gpu_parity import linear_case
+    from paper_2408_14267_gb300 import workloads as wl
+    from oracle import method as om
+    _run_both(linear_case(64, 40, 6000, 32, 4, om.SYSTEMATIC, seed=21))
+    _run_both(wl.linear_small())
+    _run_both(linear_case(96, 50, 200, 3, 2, om.BERNOULLI, seed=22))
