@@ -301,7 +301,8 @@ __device__ __forceinline__ uint32_t codes4_x16(uint32_t h) {
   return e + nz;
 }
 
-template <bool A_CODES, bool BITS8, int BN, bool SHORT = false>
+// TAB: SHORT tiles of the fused Folder keep its tables after the rings; other SHORT tiles do not.
+template <bool A_CODES, bool BITS8, int BN, bool SHORT = false, bool TAB = SHORT>
 struct TcSmem {
   static_assert(BN == 128, "one B row per expansion thread");
   // a stage carries KSUB sub-tiles of kBK contraction elements (fewer ring hand-offs per element)
@@ -324,7 +325,7 @@ struct TcSmem {
   // Folder's tables have a region of their own after the rings (built while the rings are busy)
   static constexpr int kEpi = SHORT ? kFoldTile : kExpWarps * 16384;
   static constexpr int kMain = kRing > kEpi ? kRing : kEpi;
-  static constexpr int kTab = SHORT ? kFoldTab : 0;
+  static constexpr int kTab = SHORT && TAB ? kFoldTab : 0;
   static constexpr int kBytes = kMain + kTab + 1024;  // + alignment slack
   static_assert(kSub % 1024 == 0 && kRawStage % 1024 == 0, "stages keep 1024-byte alignment");
   static_assert(kTmemUsed <= 512, "TMEM holds 512 columns");
@@ -340,14 +341,16 @@ struct TcSmem {
 // the raw ring (A_DIRECT: the MMA reads the TMA-written code tile as e4m3, nothing expands A;
 // the raw stage is released by the MMA's commit), bit 4 the failure-path test: the expansion
 // warps withhold their arrive on the first operand stage, so the MMA issuer's bounded wait
-// (20 ms in this instantiation) expires and the kernel takes its timeout exit, bit 5 e4m3
+// (20 ms in this instantiation) expires and the kernel takes its timeout exit, bit 6 a SHORT
+// tile without the Folder's tables (two CTAs per SM for short contractions; a TMA-stored
+// output is y alone), bit 5 e4m3
 // signs (+1 = 0x38, -1 = 0xB8) as the A operand straight from the raw ring (the A_DIRECT
 // datapath with a unit scale: the forward product of e4m3 X_u rows).
 template <bool A_CODES, bool BITS8, int BN, bool SHORT, int X = 0>
 __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmAcc, TcArgs a) {
-  using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
+  using S = TcSmem<A_CODES, BITS8, BN, SHORT, (X & 64) == 0>;
   constexpr bool kImpl = (X & 1) != 0, kBtma = (X & 2) != 0, kNhwc = (X & 4) != 0;
   // bit 3: codes below 16 as the A operand straight from TMA (scale 2^-9); bit 5: e4m3 signs
   // (+-1) as the A operand straight from TMA (scale 1).  Both take the A_DIRECT datapath.
@@ -939,7 +942,9 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         // c ^ (row & 7), the 128-byte swizzle of the output maps), then one TMA store per
         // output; TMA clips columns past the tensor
         // 8 KB per warp and 32-column chunk (y then acc): no wait between the warp's chunks
-        unsigned char* stg = base + (warp - 2) * 16384 + ((c0 - cbeg) >> 5) * 8192;
+        // (SHORT tiles store y alone: 4 KB per chunk, within the smaller ring)
+        unsigned char* stg = SHORT ? base + (warp - 2) * 8192 + ((c0 - cbeg) >> 5) * 4096
+                                   : base + (warp - 2) * 16384 + ((c0 - cbeg) >> 5) * 8192;
         float* sy = reinterpret_cast<float*>(stg);
         int32_t* sacc = reinterpret_cast<int32_t*>(stg + 4096);
         const int64_t nb = n0 + c0;
@@ -1199,7 +1204,7 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
                              cudaStream_t s, const CUtensorMap* my = nullptr, const CUtensorMap* macc = nullptr,
                              bool cluster = false) {
   static const CUtensorMap unused{};  // never read: the matching tma_out bit is clear
-  using S = TcSmem<A_CODES, BITS8, BN, SHORT>;
+  using S = TcSmem<A_CODES, BITS8, BN, SHORT, (X & 64) == 0>;
   static std::atomic<uint64_t> attr{0};
   const cudaError_t ea = smem_attr_once((const void*)tc_gemm_kernel<A_CODES, BITS8, BN, SHORT, X>, S::kBytes, attr);
   if (ea != cudaSuccess) return ea;
@@ -1245,7 +1250,14 @@ static cudaError_t launch_fwd_common(const CUtensorMap& ma, TcArgs a, const uint
     if (ok) a.tma_out = (y ? 1 : 0) | (acc ? 2 : 0);
   }
   if (implicit) return launch_tc<false, false, 128, false, 1>(ma, mb, a, 1, s, &my, &macc);
-  if (Be) return launch_tc<false, false, 128, false, 2>(ma, mb, a, 1, s, &my, &macc);
+  // one operand stage without int32 outputs (tall, short layers such as the 7 x 7 stem): SHORT
+  // tiles, two CTAs per SM, so that one CTA's set-up and epilogue overlap the other's products
+  const bool short_tile = a.k_tiles == 1 && !acc;
+  if (Be) {
+    if (short_tile) return launch_tc<false, false, 128, true, 2 | 64>(ma, mb, a, 1, s, &my, &macc);
+    return launch_tc<false, false, 128, false, 2>(ma, mb, a, 1, s, &my, &macc);
+  }
+  if (short_tile) return launch_tc<false, false, 128, true, 64>(ma, mb, a, 1, s, &my, &macc);
   return launch_tc<false, false, 128>(ma, mb, a, 1, s, &my, &macc);
 }
 
@@ -1313,6 +1325,7 @@ cudaError_t launch_fwd_e4m3x_tc(const uint8_t* Xe, int64_t ldxe, const uint8_t* 
       ok = make_map(&macc, acc, CU_TENSOR_MAP_DATA_TYPE_INT32, D, M, D * 4, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B);
     if (ok) a.tma_out = (y ? 1 : 0) | (acc ? 2 : 0);
   }
+  if (a.k_tiles <= 2 && !acc) return launch_tc<true, false, 128, true, 2 | 32 | 64>(ma, mb, a, 1, s, &my, &macc);
   return launch_tc<true, false, 128, false, 2 | 32>(ma, mb, a, 1, s, &my, &macc);
 }
 
@@ -1380,11 +1393,16 @@ cudaError_t launch_codes_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max
   a.tiles_per_split = (a.k_tiles + splits - 1) / splits;
   a.epi = epi;
   const int z = (a.k_tiles + a.tiles_per_split - 1) / a.tiles_per_split;
+  // short contractions per CTA (the grad_input product of layers with few output channels):
+  // SHORT tiles, two CTAs per SM (their epilogues store directly, without TMA staging)
+  const bool short_tile = a.tiles_per_split == 1 && !a.tma_out;
   if (Be) {
     if (bits == 8) return launch_tc<true, true, 128, false, 2>(ma, mb, a, z, s);
+    if (short_tile) return launch_tc<true, false, 128, true, 2 | 8 | 64>(ma, mb, a, z, s);
     return launch_tc<true, false, 128, false, 2 | 8>(ma, mb, a, z, s);
   }
   if (bits == 8) return launch_tc<true, true, 128>(ma, mb, a, z, s);
+  if (short_tile) return launch_tc<true, false, 128, true, 8 | 64>(ma, mb, a, z, s);
   return launch_tc<true, false, 128, false, 8>(ma, mb, a, z, s);  // codes < 16: A straight from TMA
 }
 
