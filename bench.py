@@ -607,8 +607,8 @@ def layer_sweep(args):
     shape, b = 4 on both SCQ branches: per layer the three-branch step (LayerStep.step_concurrent)
     as one CUDA graph, the L2 flushed before every replay, CUDA events on the launching stream,
     median over `steps` replays.  Reports 6 M K D / time per layer, the fp32 bytes the step reads
-    and writes (x, W, gY in; y, dx, dW out) over the same time, and the whole set's 6 M K D sum
-    over the sum of the layer times."""
+    and writes (x, W, gY in; y, dx, dW out) over the same time, each stage's eager device time
+    (stage_times), and the whole set's 6 M K D sum over the sum of the layer times."""
     import torch
     from paper_2408_14267_gb300 import build, workloads
     build.build()
@@ -641,9 +641,11 @@ def layer_sweep(args):
                 stream.synchronize()
             ms = statistics.median(a.elapsed_time(b) for a, b in ts)
             io = 4 * sum(t.numel() for t in (st.x, st.w, st.gy, st.y, st.dx, st.dw))
+            stage_ms = stage_times(st, stream, flush, 5)  # eager, serial: where the step's time goes
             rows.append({"layer": wl["name"], "M": st.M, "K": st.K, "D": st.D, "ms": round(ms, 5),
                          "tops": round(st.dense_ops() / (ms * 1e-3) / 1e12, 2),
-                         "fp32_io_gbs": round(io / (ms * 1e-3) / 1e9, 1)})
+                         "fp32_io_gbs": round(io / (ms * 1e-3) / 1e9, 1),
+                         "stage_us": {k: round(v * 1e3, 1) for k, v in stage_ms.items()}})
             del g, st
             torch.cuda.empty_cache()
     total_ms = sum(r["ms"] for r in rows)
