@@ -140,6 +140,66 @@ struct FoldArgs {
 
 constexpr int kFoldLoads = 8;  // accumulator loads in flight per thread while staging
 
+// Compact tap lists of a Folder block, so that an input pixel visits only the taps that land on
+// it (about (kh / stride) x (kw / stride) of them) instead of testing all kh x kw.  Local row hl
+// (input row h0 + hl): taps i whose output row oh = (h0 + hl + pad - i) / stride exists and lies
+// in [oh_lo, oh_hi], stored as h_off = (oh - oh_lo) row_pix kstride + i kw (tile offset) and
+// h_cs = i kw (column-sum offset), hcnt of them; local column wl likewise: w_off = (ow - ow_lo)
+// kstride + j, w_cs = j.  Row wl of the lists holds kh (kw) slots.
+__device__ __forceinline__ void fold_tap_lists(const FoldArgs& a, int h0, int nh, int oh_lo, int oh_hi, int row_pix,
+                                               int w0, int nw, int ow_lo, int ow_hi, int32_t* h_off, int32_t* h_cs,
+                                               int32_t* hcnt, int32_t* w_off, int32_t* w_cs, int32_t* wcnt) {
+  for (int hl = threadIdx.x; hl < nh; hl += blockDim.x) {
+    int cnt = 0;
+    for (int i = 0; i < a.kh; ++i) {
+      const int hn = h0 + hl + a.pad - i;
+      if (hn < 0 || hn % a.stride) continue;
+      const int oh = hn / a.stride;
+      if (oh < oh_lo || oh > oh_hi) continue;
+      h_off[hl * a.kh + cnt] = (oh - oh_lo) * row_pix * a.kstride + i * a.kw;
+      h_cs[hl * a.kh + cnt] = i * a.kw;
+      ++cnt;
+    }
+    hcnt[hl] = cnt;
+  }
+  for (int wl = threadIdx.x; wl < nw; wl += blockDim.x) {
+    int cnt = 0;
+    for (int j = 0; j < a.kw; ++j) {
+      const int wn = w0 + wl + a.pad - j;
+      if (wn < 0 || wn % a.stride) continue;
+      const int ow = wn / a.stride;
+      if (ow < ow_lo || ow > ow_hi) continue;
+      w_off[wl * a.kw + cnt] = (ow - ow_lo) * a.kstride + j;
+      w_cs[wl * a.kw + cnt] = j;
+      ++cnt;
+    }
+    wcnt[wl] = cnt;
+  }
+}
+
+// The integer sum and the folded column sum of one input pixel (local row hl, column wl) of
+// channel block offset kc, over its compact tap lists.
+__device__ __forceinline__ void fold_pixel(const int32_t* tile, const int32_t* css, const int32_t* h_off,
+                                           const int32_t* h_cs, const int32_t* hcnt, const int32_t* w_off,
+                                           const int32_t* w_cs, const int32_t* wcnt, int kh, int kw, int hl, int wl,
+                                           int kc, int32_t& acc, int32_t& csum) {
+  const int hc = hcnt[hl], wc = wcnt[wl];
+  const int32_t* ho = h_off + hl * kh;
+  const int32_t* hs = h_cs + hl * kh;
+  const int32_t* wo = w_off + wl * kw;
+  const int32_t* ws = w_cs + wl * kw;
+  acc = 0;
+  csum = 0;
+  for (int p = 0; p < hc; ++p) {
+    const int32_t* trow = tile + kc + ho[p];
+    const int32_t* crow = css + kc + hs[p];
+    for (int q = 0; q < wc; ++q) {
+      acc += trow[wo[q]];
+      csum += crow[ws[q]];
+    }
+  }
+}
+
 // Folder over whole input rows (blocks of at least min(C, 4) channels): a CTA owns channels
 // [c0, c0+cb) and input rows [h0, h0+hb) of its sample; each warp copies the accumulator
 // k-range of one output pixel at a time, which is coalesced when that range is long.
@@ -163,26 +223,14 @@ __global__ void __launch_bounds__(256) col2im_rows_kernel(FoldArgs a) {
   const int nrows = oh_hi - oh_lo + 1;
   const int kb = nc * khw;
   int32_t* tile = fold_smem;                                   // [max_rows * Wo][kstride]
-  int32_t* hrow = tile + a.max_rows * a.Wo * a.kstride;        // [hb * kh]: pixel-row offset or -1
-  int32_t* wcol = hrow + a.hb * a.kh;                          // [W * kw]: output column or -1
-  int32_t* css = wcol + a.W * a.kw;                            // [cb * khw]: colsum of the block
-  for (int x = threadIdx.x; x < nh * a.kh; x += blockDim.x) {
-    const int hl = x / a.kh, i = x - hl * a.kh;
-    const int hn = h0 + hl + a.pad - i;
-    int v = -1;
-    if (hn >= 0 && hn % a.stride == 0) {
-      const int oh = hn / a.stride;
-      if (oh >= oh_lo && oh <= oh_hi) v = (oh - oh_lo) * a.Wo;
-    }
-    hrow[x] = v;
-  }
-  for (int x = threadIdx.x; x < a.W * a.kw; x += blockDim.x) {
-    const int w = x / a.kw, j = x - w * a.kw;
-    const int wn = w + a.pad - j;
-    int v = -1;
-    if (wn >= 0 && wn % a.stride == 0 && wn / a.stride < a.Wo) v = wn / a.stride;
-    wcol[x] = v;
-  }
+  int32_t* h_off = tile + a.max_rows * a.Wo * a.kstride;       // [hb][kh] tap lists of the rows
+  int32_t* h_cs = h_off + a.hb * a.kh;
+  int32_t* hcnt = h_cs + a.hb * a.kh;                          // [hb]
+  int32_t* w_off = hcnt + a.hb;                                // [W][kw] tap lists of the columns
+  int32_t* w_cs = w_off + a.W * a.kw;
+  int32_t* wcnt = w_cs + a.W * a.kw;                           // [W]
+  int32_t* css = wcnt + a.W;                                   // [cb * khw]: colsum of the block
+  fold_tap_lists(a, h0, nh, oh_lo, oh_hi, a.Wo, 0, a.W, 0, a.Wo - 1, h_off, h_cs, hcnt, w_off, w_cs, wcnt);
   const int64_t kbase = (int64_t)c0 * khw;
   for (int x = threadIdx.x; x < kb; x += blockDim.x) css[x] = __ldg(a.cs + kbase + x);
   if (nrows > 0) {
@@ -220,19 +268,8 @@ __global__ void __launch_bounds__(256) col2im_rows_kernel(FoldArgs a) {
       pos = e - cl * plane;
     }
     const int hl = (int)div_w.div((uint32_t)pos), w = pos - hl * a.W;
-    const int kc = cl * khw;
-    int32_t acc = 0, csum = 0;
-    for (int i = 0; i < a.kh; ++i) {
-      const int ro = hrow[hl * a.kh + i];
-      if (ro < 0) continue;
-      const int32_t* trow = tile + kc + i * a.kw;
-      for (int j = 0; j < a.kw; ++j) {
-        const int co = wcol[w * a.kw + j];
-        if (co < 0) continue;
-        acc += trow[(ro + co) * a.kstride + j];
-        csum += css[kc + i * a.kw + j];
-      }
-    }
+    int32_t acc, csum;
+    fold_pixel(tile, css, h_off, h_cs, hcnt, w_off, w_cs, wcnt, a.kh, a.kw, hl, w, cl * khw, acc, csum);
     const float v = __fadd_rn(__fmul_rn(sc, __int2float_rn(acc)), __fmul_rn(ze, __int2float_rn(csum)));
     if (a.nhwc)
       a.dx[(((int64_t)n * a.H + h0 + hl) * a.W + w) * a.C + c0 + cl] = v;
@@ -269,36 +306,24 @@ __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
   const int nrows = oh_hi - oh_lo + 1, ncols = ow_hi - ow_lo + 1;
   const int kb = nc * khw;
   int32_t* tile = fold_smem;                                   // [max_rows * max_cols][kstride]
-  int32_t* hrow = tile + a.max_rows * a.max_cols * a.kstride;  // [hb * kh]: tile pixel-row offset or -1
-  int32_t* wcol = hrow + a.hb * a.kh;                          // [wb * kw]: tile column or -1
-  int32_t* css = wcol + a.wb * a.kw;                           // [cb * khw]: colsum of the block
-  for (int x = threadIdx.x; x < nh * a.kh; x += blockDim.x) {
-    const int hl = x / a.kh, i = x - hl * a.kh;
-    const int hn = h0 + hl + a.pad - i;
-    int v = -1;
-    if (hn >= 0 && hn % a.stride == 0) {
-      const int oh = hn / a.stride;
-      if (oh >= oh_lo && oh <= oh_hi) v = (oh - oh_lo) * a.max_cols;
-    }
-    hrow[x] = v;
-  }
-  for (int x = threadIdx.x; x < nw * a.kw; x += blockDim.x) {
-    const int wl = x / a.kw, j = x - wl * a.kw;
-    const int wn = w0 + wl + a.pad - j;
-    int v = -1;
-    if (wn >= 0 && wn % a.stride == 0) {
-      const int ow = wn / a.stride;
-      if (ow >= ow_lo && ow <= ow_hi) v = ow - ow_lo;
-    }
-    wcol[x] = v;
-  }
+  int32_t* h_off = tile + a.max_rows * a.max_cols * a.kstride; // [hb][kh] tap lists of the rows
+  int32_t* h_cs = h_off + a.hb * a.kh;
+  int32_t* hcnt = h_cs + a.hb * a.kh;                          // [hb]
+  int32_t* w_off = hcnt + a.hb;                                // [wb][kw] tap lists of the columns
+  int32_t* w_cs = w_off + a.wb * a.kw;
+  int32_t* wcnt = w_cs + a.wb * a.kw;                          // [wb]
+  int32_t* css = wcnt + a.wb;                                  // [cb * khw]: colsum of the block
+  fold_tap_lists(a, h0, nh, oh_lo, oh_hi, a.max_cols, w0, nw, ow_lo, ow_hi, h_off, h_cs, hcnt, w_off, w_cs, wcnt);
   const int64_t kbase = (int64_t)c0 * khw;
   for (int x = threadIdx.x; x < kb; x += blockDim.x) css[x] = __ldg(a.cs + kbase + x);
   if (nrows > 0 && ncols > 0) {
     // the (pixel, k) elements of the halo, kFoldLoads loads in flight per thread whatever kb is
     const int total = nrows * ncols * kb;
     const FastDiv div_kb((uint32_t)kb), div_cols((uint32_t)ncols);
-    const int64_t rbase = (int64_t)slot * a.Ho * a.Wo + (int64_t)oh_lo * a.Wo + ow_lo;
+    // the halo's first accumulator of the block: offsets from it fit 32 bits (a halo row of
+    // pixels spans at most Wo K words)
+    const int32_t* src0 = a.acc + ((int64_t)slot * a.Ho * a.Wo + (int64_t)oh_lo * a.Wo + ow_lo) * a.K + kbase;
+    const int rowK = a.Wo * (int)a.K, K32 = (int)a.K;
     for (int e0 = threadIdx.x; e0 < total; e0 += blockDim.x * kFoldLoads) {
       int32_t v[kFoldLoads];
       int dsti[kFoldLoads];
@@ -307,7 +332,7 @@ __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
         const int e = min(e0 + u * (int)blockDim.x, total - 1);  // clamped: every load is valid
         const int pix = (int)div_kb.div((uint32_t)e), kk = e - pix * kb;
         const int r = (int)div_cols.div((uint32_t)pix), cl = pix - r * ncols;
-        v[u] = __ldg(a.acc + (rbase + (int64_t)r * a.Wo + cl) * a.K + kbase + kk);
+        v[u] = __ldg(src0 + r * rowK + cl * K32 + kk);
         dsti[u] = (r * a.max_cols + cl) * a.kstride + kk;
       }
 #pragma unroll
@@ -329,19 +354,8 @@ __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
       pos = e - cl * plane;
     }
     const int hl = (int)div_w.div((uint32_t)pos), wl = pos - hl * nw;
-    const int kc = cl * khw;
-    int32_t acc = 0, csum = 0;
-    for (int i = 0; i < a.kh; ++i) {
-      const int ro = hrow[hl * a.kh + i];
-      if (ro < 0) continue;
-      const int32_t* trow = tile + kc + i * a.kw;
-      for (int j = 0; j < a.kw; ++j) {
-        const int co = wcol[wl * a.kw + j];
-        if (co < 0) continue;
-        acc += trow[(ro + co) * a.kstride + j];
-        csum += css[kc + i * a.kw + j];
-      }
-    }
+    int32_t acc, csum;
+    fold_pixel(tile, css, h_off, h_cs, hcnt, w_off, w_cs, wcnt, a.kh, a.kw, hl, wl, cl * khw, acc, csum);
     const float v = __fadd_rn(__fmul_rn(sc, __int2float_rn(acc)), __fmul_rn(ze, __int2float_rn(csum)));
     if (a.nhwc)
       a.dx[(((int64_t)n * a.H + h0 + hl) * a.W + w0 + wl) * a.C + c0 + cl] = v;
@@ -456,6 +470,12 @@ extern "C" fqt1_status fqt1_bwd_input_gemm(const fqt1_qgrad* psq, const uint32_t
   return FQT1_OK;
 }
 
+// Words of a Folder CTA's tables after its accumulator tile: tap lists of hb rows and wb columns
+// (offsets, column-sum offsets, counts) and the column sums of cb channels.
+static int64_t fold_table_words(int64_t hb, int64_t wb, int64_t kh, int64_t kw, int64_t cb) {
+  return 2 * hb * kh + hb + 2 * wb * kw + wb + cb * kh * kw;
+}
+
 // nhwc: dx in memory order N, H, W, C; only the tiled Folder writes it (else FQT1_ERR_UNSUPPORTED).
 static fqt1_status col2im_impl(const int32_t* acc, const fqt1_qgrad* psq, const int32_t* colsum_w, int32_t N,
                                int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad,
@@ -479,7 +499,7 @@ static fqt1_status col2im_impl(const int32_t* acc, const fqt1_qgrad* psq, const 
     max_rows = std::min(Ho, (hb - 1 + kh - 1) / stride + 1);
     for (int c = (C < 32 ? C : 32); c >= 1; c = (c > 1 ? c / 2 : 0)) {
       const int ks = (c * khw) | 1;
-      const int64_t words = (int64_t)max_rows * Wo * ks + (int64_t)hb * kh + (int64_t)W * kw + (int64_t)c * khw;
+      const int64_t words = (int64_t)max_rows * Wo * ks + fold_table_words(hb, W, kh, kw, c);
       if (words * 4 <= (c > 1 ? kPreferTile : kMaxTile)) { cb = c; kstride = ks; break; }
     }
     if (cb) break;
@@ -503,9 +523,9 @@ static fqt1_status col2im_impl(const int32_t* acc, const fqt1_qgrad* psq, const 
           const int mc = std::min(Wo, (wbc - 1 + kw - 1) / stride + 1);
           for (int c = (C < 32 ? C : 32); c >= 1; c = (c > 1 ? c / 2 : 0)) {
             const int ks = (c * khw) | 1;
-            const int64_t words =
-                (int64_t)mr * mc * ks + (int64_t)hbc * kh + (int64_t)wbc * kw + (int64_t)c * khw;
+            const int64_t words = (int64_t)mr * mc * ks + fold_table_words(hbc, wbc, kh, kw, c);
             if (words * 4 > cap) continue;
+            if ((int64_t)mr * Wo * C * khw >= (1ll << 31)) continue;  // the kernel's 32-bit halo offsets
             const double sectors = (double)(((int64_t)c * khw * 4 + 31) / 32 + 1) * 32.0;
             double cost = ((double)mr * mc * sectors + 8192.0) / ((double)hbc * wbc * c);
             const double ctas = (double)N * ((C + c - 1) / c) * ((H + hbc - 1) / hbc) * ((W + wbc - 1) / wbc);
@@ -533,8 +553,7 @@ static fqt1_status col2im_impl(const int32_t* acc, const fqt1_qgrad* psq, const 
     fa.nhwc = nhwc;
     const int64_t nblk = (int64_t)fa.ncb * fa.nwb * ((H + hb - 1) / hb);
     if (nblk > 0x7FFFFFFF || N > 65535) return FQT1_ERR_UNSUPPORTED;
-    const size_t smem =
-        ((size_t)max_rows * max_cols * kstride + (size_t)hb * kh + (size_t)wb * kw + (size_t)cb * khw) * 4;
+    const size_t smem = ((size_t)max_rows * max_cols * kstride + (size_t)fold_table_words(hb, wb, kh, kw, cb)) * 4;
     // pruned samples: zeros; kept samples: the tiled fold (one grid row per kept slot)
     launch_zero_pruned_rows(psq->slot_of_group, N, (int64_t)C * H * W, 1, dx, (cudaStream_t)stream);
     const int64_t cap = fqt1_kept_capacity(N, 8, FQT1_SEL_BERNOULLI);  // upper bound: all samples

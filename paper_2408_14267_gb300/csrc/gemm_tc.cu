@@ -910,6 +910,9 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     uint32_t* stage = reinterpret_cast<uint32_t*>(base) + (warp - 2) * 1024;  // 4 KB per warp (operand ring is idle)
     const int64_t row_base = m0 + 32 * q;
     for (int c0 = cbeg; c0 < cbeg + BN / 2; c0 += 32) {
+      // accumulator columns past N hold no output (warp-uniform; the cluster reduction reads
+      // every column of its partial tiles)
+      if (a.epi != EPI_CRED && n0 + c0 >= a.N) break;
       __syncwarp();
       uint32_t v[32];
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)c0;
