@@ -980,6 +980,23 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         }
         continue;
       }
+      if (a.epi == EPI_ACC32) {
+        // the int32 accumulators through the warp's 4 KB staging block (row = lane, word j at
+        // j ^ lane), then one coalesced 128-byte row segment per store (lanes over columns)
+        // instead of each lane writing its own row
+        __syncwarp();  // the previous chunk's reads of the block are done
+#pragma unroll
+        for (int j = 0; j < 32; ++j) stage[lane * 32 + (j ^ lane)] = (uint32_t)acc_int<kA512>(v[j]);
+        __syncwarp();
+        const int64_t col = n0 + c0 + lane;
+        const int64_t left = (valid_rows < a.M ? valid_rows : a.M) - row_base;
+        const int rows = left <= 0 ? 0 : (left >= 32 ? 32 : (int)left);
+        if (col < a.N) {
+          int32_t* dst = a.acc + row_base * a.ldo + col;
+          for (int rr = 0; rr < rows; ++rr) dst[rr * a.ldo] = (int32_t)stage[rr * 32 + (lane ^ rr)];
+        }
+        continue;
+      }
       if (a.epi != EPI_RED) {
         // direct stores: this thread's row, 32 consecutive columns
         const int64_t r = row_base + lane;
