@@ -59,6 +59,8 @@ struct TcArgs {
   const int32_t* cs;
   int64_t rpg;
   int32_t* status;
+  // persistent tile loop (mode bit 7): output tiles p_tiles, p_tiles_n of them along N
+  int64_t p_tiles, p_tiles_n;
   // EPI_FOLD: grad_input of a convolution with the Folder in the epilogue.  A CTA's rows are
   // whole samples (rpg = Ho*Wo divides 128) and its columns the kernel taps of fcb channels
   // starting at channel blockIdx.x * fcb (column offset n_step = fcb * kh * kw).
@@ -357,6 +359,11 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   constexpr bool kA512 = (X & 8) != 0, kAdir = (X & 8) != 0 || (X & 32) != 0;
   static_assert(!kAdir || (A_CODES && !BITS8), "A_DIRECT takes byte operands of one digit");
   constexpr bool kLose = (X & 16) != 0;
+  // bit 7: a persistent CTA takes output tiles blockIdx.x, + gridDim.x, ... (EPI_FWD / EPI_ACC32 /
+  // EPI_DX without splits): the set-up is paid once, the producer loads the next tile's stages
+  // while the epilogue of the current one runs, and the rings' positions and phases continue
+  // across tiles
+  constexpr bool kPersist = (X & 128) != 0;
   constexpr uint64_t kLimit = kLose ? 20000000ull : kWaitNs;  // bound of every wait below
   // arrivals that free a raw stage: the expansion warps (when they read it) and, with A_DIRECT,
   // the commit of the MMAs that read its A tile
@@ -373,7 +380,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   __shared__ __align__(16) float bias_s[BN];   // EPI_FWD with a bias: the bias of those columns
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t m0 = (int64_t)blockIdx.y * kBM, n0 = (int64_t)blockIdx.x * (a.n_step > 0 ? a.n_step : BN);
+  int64_t m0 = (int64_t)blockIdx.y * kBM, n0 = (int64_t)blockIdx.x * (a.n_step > 0 ? a.n_step : BN);
   const int kt0 = blockIdx.z * a.tiles_per_split;
   const int kt1 = min(a.k_tiles, kt0 + a.tiles_per_split);
   if (kt0 >= kt1) {
@@ -442,16 +449,24 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
   const int64_t valid_rows = a.count ? (int64_t)__ldg(a.count) * a.rows_per_count : a.M;
-  const int nk = m0 < valid_rows ? kt1 - kt0 : 0;  // a tile past the kept rows has no work
 
   const uint32_t kTx = kBtma ? (uint32_t)S::kRawA : (uint32_t)S::kRawStage;
+  int gbase = 0;     // operand stages of this CTA's earlier tiles
+  int issued = 0;    // producer: raw stages issued
+  int b_issued = 0;  // b_tma: operand stages whose B boxes this thread (warp 2, lane 0) issued
+  const int64_t ptiles = kPersist ? a.p_tiles : 1;
+  for (int64_t pt = kPersist ? (int64_t)blockIdx.x : 0, tj = 0; pt < ptiles; pt += kPersist ? gridDim.x : 1, ++tj) {
+  if (kPersist) {
+    m0 = (pt / a.p_tiles_n) * kBM;
+    n0 = (pt % a.p_tiles_n) * BN;
+  }
+  const int nk = m0 < valid_rows ? kt1 - kt0 : 0;  // a tile past the kept rows has no work
 
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer (raw ring)
     if (lane == 0) {
-      int issued = 0;
       for (int i = 0; i < nk; ++i) {
-        const int s = i % RS, it = i / RS;
+        const int g = gbase + i, s = g % RS, it = g / RS;
         if (it > 0 && !mbar_wait(&raw_empty[s], (it - 1) & 1, &abort_flag, a.status, kLimit)) break;
         const int kt = kt0 + i;
         mbar_expect_tx(&raw_full[s], kTx);
@@ -480,20 +495,13 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         if (!kBtma) tma_load_2d(rawB(s), &tmB, &raw_full[s], kt * KSUB * (kBK / 32), (int)n0);
         ++issued;
       }
-      // drain: every issued copy must land before the CTA may exit
-      for (int i = (issued > RS ? issued - RS : 0); i < issued; ++i) {
-        const int s = i % RS, it = i / RS;
-        const uint64_t t0 = gtimer();
-        while (!mbar_test(&raw_full[s], it & 1) && gtimer() - t0 < kWaitNs) {
-        }
-      }
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer (operand ring)
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_e4m3(BN);
       for (int i = 0; i < nk; ++i) {
-        const int s = i % OS, it = i / OS, sr = i % RS, itr = i / RS;
+        const int g = gbase + i, s = g % OS, it = g / OS, sr = g % RS, itr = g / RS;
         if (!mbar_wait(&op_full[s], it & 1, &abort_flag, a.status, kLimit)) break;
         if (kBtma && !mbar_wait(&b_full[s], it & 1, &abort_flag, a.status, kLimit)) break;
         if (kAdir && !mbar_wait(&raw_full[sr], itr & 1, &abort_flag, a.status, kLimit)) break;  // the A codes landed
@@ -546,9 +554,8 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     // depends only on its own A row, and the epilogue drops those rows
     const bool a_live = a_warp && m0 + 32 * quarter < valid_rows;
     const uint32_t a_lanes = tmem + ((uint32_t)(32 * quarter) << 16);
-    int b_issued = 0;  // b_tma: operand stages whose B boxes this thread (warp 2, lane 0) issued
     for (int i = 0; i < nk; ++i) {
-      const int so = i % OS, ito = i / OS, sr = i % RS, itr = i / RS;
+      const int g = gbase + i, so = g % OS, ito = g / OS, sr = g % RS, itr = g / RS;
       if (ito > 0 && !mbar_wait(&op_empty[so], (ito - 1) & 1, &abort_flag, a.status, kLimit)) break;
       if (kBtma) {  // the stage's B boxes, as soon as the MMAs of its previous use are done
         if (warp == 2 && lane == 0) {
@@ -781,7 +788,7 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       if (a.bias && tt < BN) bias_s[tt] = n0 + tt < a.N ? __ldg(a.bias + n0 + tt) : 0.f;
       asm volatile("bar.sync 1, 256;" ::: "memory");  // the 256 epilogue threads
     }
-    const bool have_acc = mbar_wait(&acc_full, 0, &abort_flag, a.status, kLimit);
+    const bool have_acc = mbar_wait(&acc_full, (uint32_t)(tj & 1), &abort_flag, a.status, kLimit);
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     if (a.epi == EPI_FOLD) {
       // 1. the whole 128 x BN accumulator tile -> shared memory as int32 (rings are idle);
@@ -1098,6 +1105,24 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
     // the stores must have read the staging buffers before the CTA exits
     if (a.tma_out && lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
     }  // epilogue modes other than EPI_FOLD
+    if (kPersist) {
+      // every epilogue warp has read its staging block and its accumulator columns before the
+      // next tile's operands go into the ring (also by TMA) and its products into TMEM
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+    }
+  }
+  gbase += nk;
+  }  // output tiles
+  if (warp == 0 && lane == 0) {
+    // drain: every issued copy must land before the CTA may exit
+    for (int i = (issued > RS ? issued - RS : 0); i < issued; ++i) {
+      const int s = i % RS, it = i / RS;
+      const uint64_t t0 = gtimer();
+      while (!mbar_test(&raw_full[s], it & 1) && gtimer() - t0 < kWaitNs) {
+      }
+    }
   }
 
   // The producer and MMA roles ran on lane 0 only; reconverge before the aligned barriers
@@ -1219,8 +1244,24 @@ static bool make_map(CUtensorMap* m, const void* ptr, CUtensorMapDataType type, 
             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// SMs of the current device (cached per device ordinal).
+static int sm_count() {
+  static std::atomic<int> cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152;
+  int n = cache[dev].load(std::memory_order_relaxed);
+  if (n > 0) return n;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 152;
+  cache[dev].store(n, std::memory_order_relaxed);
+  return n;
+}
+
+// Output tiles of a launch and the resident CTAs of one wave (1 per SM, 2 for SHORT tiles).
+static int64_t out_tiles(const TcArgs& a, int bn) { return ((a.N + bn - 1) / bn) * ((a.M + kBM - 1) / kBM); }
+static int64_t tile_wave(bool short_tile) { return (int64_t)sm_count() * (short_tile ? 2 : 1); }
+
 template <bool A_CODES, bool BITS8, int BN, bool SHORT = false, int X = 0>
-static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const TcArgs& a, int splits,
+static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const TcArgs& a_in, int splits,
                              cudaStream_t s, const CUtensorMap* my = nullptr, const CUtensorMap* macc = nullptr,
                              bool cluster = false) {
   static const CUtensorMap unused{};  // never read: the matching tma_out bit is clear
@@ -1228,8 +1269,14 @@ static cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const
   static std::atomic<uint64_t> attr{0};
   const cudaError_t ea = smem_attr_once((const void*)tc_gemm_kernel<A_CODES, BITS8, BN, SHORT, X>, S::kBytes, attr);
   if (ea != cudaSuccess) return ea;
+  TcArgs a = a_in;
   dim3 grid((unsigned)(a.grid_x > 0 ? a.grid_x : (a.N + BN - 1) / BN), (unsigned)((a.M + kBM - 1) / kBM),
             (unsigned)splits);
+  if constexpr ((X & 128) != 0) {  // persistent: one wave of CTAs over all output tiles
+    a.p_tiles_n = (a.N + BN - 1) / BN;
+    a.p_tiles = out_tiles(a, BN);
+    grid = dim3((unsigned)std::min<int64_t>(a.p_tiles, tile_wave(SHORT)), 1, 1);
+  }
   if (cluster)
     launch_k_cluster(tc_gemm_kernel<A_CODES, BITS8, BN, SHORT, X>, dim3(grid), dim3(kThreads), S::kBytes, s,
                      (unsigned)splits, ma, mb, my ? *my : unused, macc ? *macc : unused, a);
@@ -1272,12 +1319,18 @@ static cudaError_t launch_fwd_common(const CUtensorMap& ma, TcArgs a, const uint
   if (implicit) return launch_tc<false, false, 128, false, 1>(ma, mb, a, 1, s, &my, &macc);
   // one operand stage without int32 outputs (tall, short layers such as the 7 x 7 stem): SHORT
   // tiles, two CTAs per SM, so that one CTA's set-up and epilogue overlap the other's products
+  // more output tiles than one wave of CTAs: persistent CTAs over the tiles (mode bit 7)
   const bool short_tile = a.k_tiles == 1 && !acc;
+  const bool persist = out_tiles(a, 128) > tile_wave(short_tile);
   if (Be) {
+    if (short_tile && persist) return launch_tc<false, false, 128, true, 2 | 64 | 128>(ma, mb, a, 1, s, &my, &macc);
     if (short_tile) return launch_tc<false, false, 128, true, 2 | 64>(ma, mb, a, 1, s, &my, &macc);
+    if (persist) return launch_tc<false, false, 128, false, 2 | 128>(ma, mb, a, 1, s, &my, &macc);
     return launch_tc<false, false, 128, false, 2>(ma, mb, a, 1, s, &my, &macc);
   }
+  if (short_tile && persist) return launch_tc<false, false, 128, true, 64 | 128>(ma, mb, a, 1, s, &my, &macc);
   if (short_tile) return launch_tc<false, false, 128, true, 64>(ma, mb, a, 1, s, &my, &macc);
+  if (persist) return launch_tc<false, false, 128, false, 128>(ma, mb, a, 1, s, &my, &macc);
   return launch_tc<false, false, 128>(ma, mb, a, 1, s, &my, &macc);
 }
 
@@ -1422,7 +1475,11 @@ cudaError_t launch_codes_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max
     return launch_tc<true, false, 128, false, 2 | 8>(ma, mb, a, z, s);
   }
   if (bits == 8) return launch_tc<true, true, 128>(ma, mb, a, z, s);
+  // more output tiles than one wave, without splits: persistent CTAs over the tiles (mode bit 7)
+  const bool persist = z == 1 && out_tiles(a, 128) > tile_wave(short_tile);
+  if (short_tile && persist) return launch_tc<true, false, 128, true, 8 | 64 | 128>(ma, mb, a, z, s);
   if (short_tile) return launch_tc<true, false, 128, true, 8 | 64>(ma, mb, a, z, s);
+  if (persist) return launch_tc<true, false, 128, false, 8 | 128>(ma, mb, a, z, s);
   return launch_tc<true, false, 128, false, 8>(ma, mb, a, z, s);  // codes < 16: A straight from TMA
 }
 
