@@ -324,6 +324,30 @@ __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
     // pixels spans at most Wo K words)
     const int32_t* src0 = a.acc + ((int64_t)slot * a.Ho * a.Wo + (int64_t)oh_lo * a.Wo + ow_lo) * a.K + kbase;
     const int rowK = a.Wo * (int)a.K, K32 = (int)a.K;
+    if ((kb & 3) == 0 && (K32 & 3) == 0 && (kbase & 3) == 0) {
+      // k-ranges of whole 16-byte groups: one 16-byte load per four elements (a quarter of the
+      // index arithmetic), stored as four words (the tile's row stride is odd)
+      const int kb4 = kb >> 2, total4 = total >> 2;
+      const FastDiv div_kb4((uint32_t)kb4);
+      for (int e0 = threadIdx.x; e0 < total4; e0 += blockDim.x * kFoldLoads) {
+        int4 v[kFoldLoads];
+        int dsti[kFoldLoads];
+#pragma unroll
+        for (int u = 0; u < kFoldLoads; ++u) {
+          const int e = min(e0 + u * (int)blockDim.x, total4 - 1);  // clamped: every load is valid
+          const int pix = (int)div_kb4.div((uint32_t)e), kk = 4 * (e - pix * kb4);
+          const int r = (int)div_cols.div((uint32_t)pix), cl = pix - r * ncols;
+          v[u] = __ldg(reinterpret_cast<const int4*>(src0 + r * rowK + cl * K32 + kk));
+          dsti[u] = (r * a.max_cols + cl) * a.kstride + kk;
+        }
+#pragma unroll
+        for (int u = 0; u < kFoldLoads; ++u) {
+          if (e0 + u * (int)blockDim.x >= total4) break;
+          int32_t* d = tile + dsti[u];
+          d[0] = v[u].x; d[1] = v[u].y; d[2] = v[u].z; d[3] = v[u].w;
+        }
+      }
+    } else
     for (int e0 = threadIdx.x; e0 < total; e0 += blockDim.x * kFoldLoads) {
       int32_t v[kFoldLoads];
       int dsti[kFoldLoads];

@@ -942,6 +942,32 @@ __global__ void __launch_bounds__(256) pack_planes_nchw_kernel(const float* __re
     if (lane < 8 && q0 + lane < pw) planes[pl * pw + q0 + lane] = mine;
   }
 }
+// Planes of fewer than 32 pixels that divide 32 (4 x 4, 2 x 2, 1 x 1 maps): 32 consecutive floats
+// of x are all the pixels of 32 / HW consecutive planes, so one ballot gives the words of all of
+// them (one word per plane).  A warp takes 8 such chunks at a time, their loads in flight
+// together.
+__global__ void __launch_bounds__(256) pack_planes_small_kernel(const float* __restrict__ x, int64_t total, int HW,
+                                                                uint32_t* __restrict__ planes) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int per = 32 / HW;  // planes per chunk
+  const uint32_t mask = (1u << HW) - 1u;
+  const int64_t chunks = (total + 31) / 32;
+  for (int64_t c0 = ((int64_t)blockIdx.x * 8 + warp) * 8; c0 < chunks; c0 += (int64_t)gridDim.x * 64) {
+    float v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = __ldg(x + min((c0 + k) * 32 + lane, total - 1));
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      if (c0 + k >= chunks) break;  // warp-uniform
+      const int64_t f = (c0 + k) * 32 + lane;
+      const uint32_t wd = __ballot_sync(0xFFFFFFFFu, v[k] > 0.0f && f < total);
+      const int64_t pl = (c0 + k) * per + lane;
+      if (lane < per && pl * HW < total) planes[pl] = (wd >> (lane * HW)) & mask;
+    }
+  }
+}
 }  // namespace fqt1
 
 using namespace fqt1;
@@ -995,16 +1021,21 @@ static bool unfold_same_fits(int N, int C, int H, int W, int kh, int kw, int str
   return row_tiles <= 65535 && smem <= 32 * 1024;
 }
 
-// Pixels per tile of the region Unfolder (unfold_bits_kernel): the largest of 128, 64, 32 whose
-// input region bound (images a tile may touch x channels of 256 columns x whole planes with
+// Pixels per tile of the region Unfolder (unfold_bits_kernel): the largest of 256 (see below),
+// 128, 64, 32 whose input region bound (images a tile may touch x channels of 256 columns x whole planes with
 // guards) fits kUnfoldMaxStreamWords, with at most 65535 row tiles; 0 if none (gather path).
+// Larger tiles pay the region set-up, its divisions and its barrier over more output words.
 static int unfold_bits_tm(int N, int C, int H, int W, int kh, int kw, int stride, int pad) {
   const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
   const int64_t Mi = (int64_t)N * Ho * Wo, Ki = (int64_t)C * kh * kw;
   if (!(pad <= 32 && Ki < (1ll << 31))) return 0;
   const bool same = stride == 1 && kh == kw && kh == 2 * pad + 1 && (Ho * Wo) % 32 == 0;
   const int guard = same ? (pad * W + pad + 63) / 32 : 1;
-  for (int tm = 128; tm >= 32; tm /= 2) {
+  // 256-pixel tiles only for maps of 256 or more output pixels and windows larger than one tap
+  // (measured: they speed up the stem, layer1 and the 32 x 32 layers, and slow down the 1 x 1
+  // downsamples and the small maps)
+  const int tm_max = (Ho * Wo >= 256 && kh * kw > 1) ? 256 : 128;
+  for (int tm = tm_max; tm >= 32; tm /= 2) {
     const int64_t imgs = std::min<int64_t>(N, tm / (Ho * Wo) + 2);
     const int64_t chans = std::min<int64_t>(C, 256 / (kh * kw) + 2);
     const int64_t words = imgs * chans * (((int64_t)H * W + 31) / 32 + 2 * guard);
@@ -1231,6 +1262,14 @@ extern "C" fqt1_status fqt1_pack_planes(const float* x, int32_t N, int32_t C, in
   if (!x || !planes || N < 1 || C < 1 || H < 1 || W < 1) return FQT1_ERR_INVALID_ARG;
   if ((int64_t)N * C * H * W >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
   const int pw = (H * W + 31) / 32;
+  if (H * W < 32 && 32 % (H * W) == 0) {  // several planes per 32 floats
+    const int64_t total = (int64_t)N * C * H * W, chunks = (total + 31) / 32;
+    const unsigned blocks = (unsigned)std::min<int64_t>((chunks + 63) / 64, 152 * 16);
+    FQT1_CUDA_TRY(launch_k(pack_planes_small_kernel, dim3(blocks), dim3(256), 0, (cudaStream_t)stream, x, total,
+                           H * W, planes));
+    fqt1_count_launches(1);
+    return FQT1_OK;
+  }
   const int64_t units = (int64_t)N * C * ((pw + 7) / 8);
   const unsigned blocks = (unsigned)std::min<int64_t>((units + 7) / 8, 152 * 16);
   FQT1_CUDA_TRY(launch_k(pack_planes_nchw_kernel, dim3(blocks), dim3(256), 0, (cudaStream_t)stream, x,

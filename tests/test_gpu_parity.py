@@ -699,7 +699,8 @@ def test_im2col_from_channels_last_planes(N, C, H, W, k, s, p):
 
 
 @pytest.mark.parametrize("N,C,H,W,k,s,p", [(2, 3, 30, 30, 7, 2, 3), (2, 64, 28, 28, 1, 2, 0), (3, 16, 14, 14, 3, 2, 1),
-                                           (2, 5, 13, 11, 3, 1, 1), (1, 32, 56, 56, 3, 1, 1), (4, 8, 9, 7, 1, 1, 0)])
+                                           (2, 5, 13, 11, 3, 1, 1), (1, 32, 56, 56, 3, 1, 1), (4, 8, 9, 7, 1, 1, 0),
+                                           (5, 37, 4, 4, 3, 1, 1), (9, 50, 2, 2, 3, 1, 1), (3, 11, 2, 4, 3, 1, 1)])
 def test_pack_planes_nchw_and_unfold_from_planes(N, C, H, W, k, s, p):
     """Contiguous x: fqt1_pack_planes writes the signs of x as channel planes (any C, H W not a
     multiple of 32, bits past H W clear), and the Unfolder reading those planes writes the same
