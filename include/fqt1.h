@@ -170,7 +170,9 @@ fqt1_status fqt1_conv_fwd_implicit(const uint32_t* x_pix, const uint32_t* w_taps
  *   (stride-1 "same" convolutions whose H W divides 128 or is 256), one pass over
  *   x.  1: tiles of up to 128 output pixels, each reading its input region; then
  *   fqt1_pack_planes followed by fqt1_im2col_planes gives the same outputs from
- *   32 times fewer bytes.  0: a per-element gather (regions too large; x must be
+ *   32 times fewer bytes.  3: a pointwise convolution (1 x 1 window, no padding):
+ *   one pass over x, which fqt1_im2col reads directly (fqt1_im2col_planes serves
+ *   it with region tiles).  0: a per-element gather (regions too large; x must be
  *   given).  -1: invalid shape. */
 fqt1_status fqt1_pack_planes(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, uint32_t* planes,
                              void* stream);

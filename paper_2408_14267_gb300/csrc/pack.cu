@@ -942,6 +942,73 @@ __global__ void __launch_bounds__(256) pack_planes_nchw_kernel(const float* __re
     if (lane < 8 && q0 + lane < pw) planes[pl * pw + q0 + lane] = mine;
   }
 }
+// Unfolder of a pointwise convolution (1 x 1 window, no padding, any stride): X_u[m][c] is
+// sign(x[n][c][s oh][s ow]), a strided subsample of x.  A warp takes 32 output pixels x 32
+// channels (lane = channel): its 32 loads per lane (one per pixel) are in flight together, a
+// ballot per pixel gives that pixel's row word, and each lane's own 32 compares give its
+// channel's column word.  Pixel groups run up to the padded column words and channel groups up
+// to the padded row words, so the padding words are written as zeros.  The column sums are
+// reduced over the CTA's 8 warps (same channels) before one atomic per channel.
+struct UnfoldPointArgs {
+  const float* x;
+  uint32_t* row_bits;
+  uint32_t* col_bits;
+  int32_t* colsum;
+  int64_t row_words, col_words;
+  int C, H, W, stride, Ho, Wo, M;
+  FastDiv div_hwo, div_wo;
+};
+
+__global__ void __launch_bounds__(256) unfold_pointwise_kernel(UnfoldPointArgs a) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  __shared__ int32_t cs_s[8][32];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t pg = (int64_t)blockIdx.x * 8 + warp;  // pixel group (32 pixels)
+  const int cw = blockIdx.y;                           // channel word
+  const int c = cw * 32 + lane;
+  const bool cvalid = c < a.C;
+  const int64_t m0 = pg * 32;
+  int32_t cnt = 0;
+  if (pg < a.col_words) {  // warp-uniform
+    // input offset of pixel m0 (clamped) for channel c; later pixels step along the output row
+    const int mc = (int)(m0 < a.M - 1 ? m0 : a.M - 1);
+    int n = (int)a.div_hwo.div((uint32_t)mc), rem = mc - n * a.Ho * a.Wo;
+    int oh = (int)a.div_wo.div((uint32_t)rem), ow = rem - oh * a.Wo;
+    const int64_t plane = (int64_t)a.H * a.W, cc = cvalid ? c : a.C - 1;
+    float v[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      v[j] = __ldg(a.x + ((int64_t)n * a.C + cc) * plane + (int64_t)oh * a.stride * a.W + (int64_t)ow * a.stride);
+      if (m0 + j + 1 < a.M) {  // the next pixel (uniform); past M the last one is loaded again
+        if (++ow == a.Wo) { ow = 0; if (++oh == a.Ho) { oh = 0; ++n; } }
+      }
+    }
+    uint32_t roww = 0u, colw = 0u;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const bool pvalid = m0 + j < a.M;
+      const bool pos = v[j] > 0.0f && pvalid;
+      const uint32_t b = __ballot_sync(0xFFFFFFFFu, pos && cvalid);
+      if (lane == j) roww = b;
+      colw |= (pos ? 1u : 0u) << j;
+    }
+    if (a.row_bits && m0 + lane < a.M && cw < a.row_words) a.row_bits[(m0 + lane) * a.row_words + cw] = roww;
+    if (a.col_bits && cvalid) a.col_bits[(int64_t)c * a.col_words + pg] = colw;
+    const int64_t left = a.M - m0;
+    const int valid = left <= 0 ? 0 : (left >= 32 ? 32 : (int)left);
+    cnt = cvalid ? 2 * __popc(colw) - valid : 0;
+  }
+  cs_s[warp][lane] = cnt;
+  __syncthreads();
+  if (a.colsum && warp == 0) {
+    int32_t sum = 0;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) sum += cs_s[w][lane];
+    if (cvalid && sum != 0) atomicAdd(a.colsum + c, sum);
+  }
+}
+
 // Planes of fewer than 32 pixels that divide 32 (4 x 4, 2 x 2, 1 x 1 maps): 32 consecutive floats
 // of x are all the pixels of 32 / HW consecutive planes, so one ballot gives the words of all of
 // them (one word per plane).  A warp takes 8 such chunks at a time, their loads in flight
@@ -1020,6 +1087,9 @@ static bool unfold_same_fits(int N, int C, int H, int W, int kh, int kw, int str
   const int64_t row_tiles = (N + ipt - 1) / ipt;
   return row_tiles <= 65535 && smem <= 32 * 1024;
 }
+
+// A 1 x 1 window without padding: the pointwise Unfolder reads x directly.
+static bool pointwise_conv(int kh, int kw, int pad) { return kh == 1 && kw == 1 && pad == 0; }
 
 // Pixels per tile of the region Unfolder (unfold_bits_kernel): the largest of 256 (see below),
 // 128, 64, 32 whose input region bound (images a tile may touch x channels of 256 columns x whole planes with
@@ -1109,6 +1179,21 @@ static fqt1_status im2col_impl(const float* x, const uint32_t* planes, int32_t N
     }
   }
   if (e4m3) return FQT1_ERR_UNSUPPORTED;
+  if (x && pointwise_conv(kh, kw, pad) && Mi < (1ll << 31)) {
+    // pointwise convolution: a strided subsample of x, read once per element
+    UnfoldPointArgs u;
+    u.x = x; u.row_bits = row_bits; u.col_bits = col_bits; u.colsum = colsum;
+    u.row_words = fqt1_packed_words(Ki); u.col_words = fqt1_packed_words(Mi);
+    u.C = C; u.H = H; u.W = W; u.stride = stride; u.Ho = Ho; u.Wo = Wo; u.M = (int)Mi;
+    u.div_hwo = FastDiv((uint32_t)(Ho * Wo)); u.div_wo = FastDiv((uint32_t)Wo);
+    if (colsum) FQT1_CUDA_TRY(cudaMemsetAsync(colsum, 0, sizeof(int32_t) * Ki, s));
+    const int64_t gx = (u.col_words + 7) / 8;
+    if (gx > 0x7FFFFFFF || u.row_words > 65535) return FQT1_ERR_UNSUPPORTED;
+    launch_k(unfold_pointwise_kernel, dim3((unsigned)gx, (unsigned)u.row_words), dim3(256), 0, s, u);
+    fqt1_count_launches(1);
+    FQT1_CUDA_TRY(cudaGetLastError());
+    return FQT1_OK;
+  }
   if (const int tm = unfold_bits_tm(N, C, H, W, kh, kw, stride, pad)) {
     // 128-pixel tiles (smaller only when the input region does not fit): fewer CTAs, each
     // amortizing its region set-up over more output words
@@ -1283,6 +1368,8 @@ extern "C" int32_t fqt1_im2col_path(int32_t N, int32_t C, int32_t H, int32_t W, 
   if (N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 || pad < 0) return -1;
   if (H + 2 * pad < kh || W + 2 * pad < kw) return -1;
   if (unfold_same_fits(N, C, H, W, kh, kw, stride, pad)) return 2;
+  if (pointwise_conv(kh, kw, pad) && (int64_t)N * ((H - 1) / stride + 1) * ((W - 1) / stride + 1) < (1ll << 31))
+    return 3;
   return unfold_bits_tm(N, C, H, W, kh, kw, stride, pad) ? 1 : 0;
 }
 

@@ -700,12 +700,13 @@ def test_im2col_from_channels_last_planes(N, C, H, W, k, s, p):
 
 @pytest.mark.parametrize("N,C,H,W,k,s,p", [(2, 3, 30, 30, 7, 2, 3), (2, 64, 28, 28, 1, 2, 0), (3, 16, 14, 14, 3, 2, 1),
                                            (2, 5, 13, 11, 3, 1, 1), (1, 32, 56, 56, 3, 1, 1), (4, 8, 9, 7, 1, 1, 0),
-                                           (5, 37, 4, 4, 3, 1, 1), (9, 50, 2, 2, 3, 1, 1), (3, 11, 2, 4, 3, 1, 1)])
+                                           (5, 37, 4, 4, 3, 1, 1), (9, 50, 2, 2, 3, 1, 1), (3, 11, 2, 4, 3, 1, 1),
+                                           (3, 40, 15, 13, 1, 3, 0), (2, 33, 8, 9, 1, 1, 0), (5, 70, 7, 7, 1, 2, 0)])
 def test_pack_planes_nchw_and_unfold_from_planes(N, C, H, W, k, s, p):
     """Contiguous x: fqt1_pack_planes writes the signs of x as channel planes (any C, H W not a
     multiple of 32, bits past H W clear), and the Unfolder reading those planes writes the same
-    rows, columns and column sums as the Unfolder reading x (the region-tile shapes of the
-    ResNet-18 stem and downsamples among them)."""
+    rows, columns and column sums as the Unfolder reading x (the region-tile shape of the
+    ResNet-18 stem, and the 1 x 1 downsamples, which the pointwise pass serves from x)."""
     from paper_2408_14267_gb300 import fqt1
     rng = np.random.default_rng(N * C + H * 3 + k)
     x = rng.standard_normal((N, C, H, W)).astype(np.float32)
@@ -717,7 +718,7 @@ def test_pack_planes_nchw_and_unfold_from_planes(N, C, H, W, k, s, p):
     Ho, Wo = om.conv_out_hw(H, W, k, k, s, p)
     M, K = N * Ho * Wo, C * k * k
     path = fqt1.im2col_path(N, C, H, W, k, k, s, p)
-    assert path in (1, 2)
+    assert path in (1, 2, 3)
     outs = []
     for use_planes in (False, True):
         rb = torch.full((M, fqt1.packed_words(K)), 7, dtype=torch.int32, device="cuda")
@@ -742,12 +743,14 @@ def test_pack_planes_nchw_and_unfold_from_planes(N, C, H, W, k, s, p):
 
 def test_im2col_path_query():
     """fqt1_im2col_path: whole-image tiles for the bench layer, region tiles for the ResNet-18
-    ImageNet stem and downsamples, the gather for regions too large, -1 for invalid shapes."""
+    ImageNet stem, the pointwise pass for 1 x 1 windows without padding (the downsamples), the
+    gather for regions too large, -1 for invalid shapes."""
     from paper_2408_14267_gb300 import fqt1
     assert fqt1.im2col_path(128, 256, 8, 8, 3, 3, 1, 1) == 2
     assert fqt1.im2col_path(64, 3, 224, 224, 7, 7, 2, 3) == 1
-    assert fqt1.im2col_path(64, 64, 56, 56, 1, 1, 2, 0) == 1
-    assert fqt1.im2col_path(2, 256, 56, 56, 1, 1, 1, 0) == 0
+    assert fqt1.im2col_path(64, 64, 56, 56, 1, 1, 2, 0) == 3
+    assert fqt1.im2col_path(2, 256, 56, 56, 1, 1, 1, 0) == 3
+    assert fqt1.im2col_path(1, 64, 512, 512, 3, 3, 1, 1) == 0
     assert fqt1.im2col_path(2, 4, 3, 3, 7, 7, 1, 0) == -1
 
 
