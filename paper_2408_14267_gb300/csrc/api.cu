@@ -200,6 +200,50 @@ __device__ __forceinline__ void fold_pixel(const int32_t* tile, const int32_t* c
   }
 }
 
+// Folder of a pointwise convolution (1 x 1 window, no padding, stride s): input pixel (h, w)
+// receives the tap of output pixel (h / s, w / s) when s divides both, and nothing otherwise.
+// A CTA owns one kept sample, one output row oh and 32 channels: it stages the accumulator rows
+// of that output row ([Wo][32] ints, coalesced) in shared memory and writes the s input rows
+// s oh .. s oh + s - 1 of its channels completely (zeros where no tap lands).
+__global__ void __launch_bounds__(256) col2im_pointwise_kernel(FoldArgs a) {
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  extern __shared__ int32_t pw_tile[];  // [32][Wo + 1]
+  const int32_t slot = (int32_t)blockIdx.y;
+  if (slot >= __ldg(a.kept_count)) return;
+  const int n = __ldg(a.kept_idx + slot);
+  const int ncb = (a.C + 31) / 32;
+  const int oh = blockIdx.x / ncb, c0 = (blockIdx.x - oh * ncb) * 32;
+  const int nc = min(32, a.C - c0);
+  const int ts = a.Wo + 1;
+  const int32_t* src = a.acc + ((int64_t)slot * a.Ho * a.Wo + (int64_t)oh * a.Wo) * a.K + c0;
+  for (int e = threadIdx.x; e < a.Wo * 32; e += blockDim.x) {
+    const int ow = e >> 5, cl = e & 31;
+    pw_tile[cl * ts + ow] = cl < nc ? __ldg(src + (int64_t)ow * a.K + cl) : 0;
+  }
+  __syncthreads();
+  const float sc = __ldg(a.scale + slot), ze = __ldg(a.zero + slot);
+  const int h0 = oh * a.stride, h1 = min(a.H, h0 + a.stride);
+  const int per = (h1 - h0) * a.W;  // floats of one channel in this CTA's rows
+  for (int e = threadIdx.x; e < nc * per; e += blockDim.x) {
+    int cl, pos;
+    if (a.nhwc) { pos = e / nc; cl = e - pos * nc; }
+    else { cl = e / per; pos = e - cl * per; }
+    const int hl = pos / a.W, w = pos - hl * a.W;
+    float v = 0.0f;
+    if (hl == 0 && w % a.stride == 0) {
+      const int ow = w / a.stride;
+      if (ow < a.Wo)
+        v = __fadd_rn(__fmul_rn(sc, __int2float_rn(pw_tile[cl * ts + ow])),
+                      __fmul_rn(ze, __int2float_rn(__ldg(a.cs + c0 + cl))));
+    }
+    if (a.nhwc)
+      a.dx[(((int64_t)n * a.H + h0 + hl) * a.W + w) * a.C + c0 + cl] = v;
+    else
+      a.dx[(((int64_t)n * a.C + c0 + cl) * a.H + h0 + hl) * a.W + w] = v;
+  }
+}
+
 // Folder over whole input rows (blocks of at least min(C, 4) channels): a CTA owns channels
 // [c0, c0+cb) and input rows [h0, h0+hb) of its sample; each warp copies the accumulator
 // k-range of one output pixel at a time, which is coalesced when that range is long.
@@ -515,6 +559,20 @@ static fqt1_status col2im_impl(const int32_t* acc, const fqt1_qgrad* psq, const 
   constexpr int64_t kMaxTile = 96 * 1024;
   constexpr int64_t kPreferTile = 48 * 1024;  // >= 4 resident CTAs per SM
   const int khw = kh * kw;
+  if (kh == 1 && kw == 1 && pad == 0 && Wo <= 256 && (int64_t)Ho * ((C + 31) / 32) <= 0x7FFFFFFF && N <= 65535) {
+    // pointwise convolution: one output row of 32 channels per CTA
+    FoldArgs fa{};
+    fa.acc = acc; fa.kept_idx = psq->kept_idx; fa.kept_count = psq->kept_count; fa.scale = psq->scale;
+    fa.zero = psq->zero; fa.cs = colsum_w; fa.dx = dx; fa.N = N; fa.C = C; fa.H = H; fa.W = W; fa.kh = 1; fa.kw = 1;
+    fa.stride = stride; fa.pad = 0; fa.Ho = Ho; fa.Wo = Wo; fa.K = C; fa.nhwc = nhwc;
+    launch_zero_pruned_rows(psq->slot_of_group, N, (int64_t)C * H * W, 1, dx, (cudaStream_t)stream);
+    const size_t smem = (size_t)32 * (Wo + 1) * 4;
+    launch_k(col2im_pointwise_kernel, dim3((unsigned)((int64_t)Ho * ((C + 31) / 32)), (unsigned)N), dim3(256), smem,
+             (cudaStream_t)stream, fa);
+    fqt1_count_launches(1);
+    FQT1_CUDA_TRY(cudaGetLastError());
+    return FQT1_OK;
+  }
   // whole-row Folder: up to 8 input rows per CTA and the most channels whose staged
   // accumulators fit (<= 48 KB, or 96 KB for a single channel)
   int hb = H < 8 ? H : 8, wb = W, cb = 0;

@@ -782,7 +782,8 @@ def test_fold_channels_last_output(name, make):
     assert torch.equal(dx.permute(0, 3, 1, 2), st.dx)
 
 
-@pytest.mark.parametrize("name,make", [CASES[12], CASES[15], CASES[8]], ids=[CASES[12][0], CASES[15][0], CASES[8][0]])
+@pytest.mark.parametrize("name,make", [CASES[12], CASES[15], CASES[8], CASES[10], CASES[11]],
+                         ids=[CASES[12][0], CASES[15][0], CASES[8][0], CASES[10][0], CASES[11][0]])
 def test_col2im_channels_last_output(name, make):
     """The two-call Folder writing dx channels-last gives the NCHW result's values."""
     from paper_2408_14267_gb300 import fqt1
