@@ -332,6 +332,9 @@ def main():
                     help="training step of a synthetic model built from binop layers against FP32 PyTorch")
     ap.add_argument("--layers", choices=["vgg16", "resnet18", "all"],
                     help="the layer step on every VGG-16 / ResNet-18 layer shape")
+    ap.add_argument("--colmajor", choices=["auto", "on", "off"], default="auto",
+                    help="--layers: grad_input of convolutions without the fused Folder through column-major "
+                         "int32 accumulators and the column-major Folder (auto: the library's default)")
     ap.add_argument("--variance", action="store_true",
                     help="empirical variance of the AGP quantizer (b = 2, 4, 8) and of 1-bit PSQ against Eq. 24")
     ap.add_argument("--sweep", choices=["routine", "diag", "full"],
@@ -620,7 +623,8 @@ def layer_sweep(args):
     rows = []
     for net in (["vgg16", "resnet18"] if args.layers == "all" else [args.layers]):
         for wl in sets[net]():
-            st = LayerStep(wl, device=dev, keep_acc=False)
+            opts = {} if args.colmajor == "auto" else {"colmajor": args.colmajor == "on"}
+            st = LayerStep(wl, device=dev, keep_acc=False, **opts)
             with torch.cuda.stream(stream):
                 for _ in range(3):
                     st.step()
@@ -643,6 +647,8 @@ def layer_sweep(args):
             io = 4 * sum(t.numel() for t in (st.x, st.w, st.gy, st.y, st.dx, st.dw))
             stage_ms = stage_times(st, stream, flush, 5)  # eager, serial: where the step's time goes
             rows.append({"layer": wl["name"], "M": st.M, "K": st.K, "D": st.D, "ms": round(ms, 5),
+                         "grad_input": "fused Folder" if st.fold else ("column-major Folder" if st.colmajor
+                                                                        else "row-major Folder"),
                          "tops": round(st.dense_ops() / (ms * 1e-3) / 1e12, 2),
                          "fp32_io_gbs": round(io / (ms * 1e-3) / 1e9, 1),
                          "stage_us": {k: round(v * 1e3, 1) for k, v in stage_ms.items()}})

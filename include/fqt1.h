@@ -386,6 +386,28 @@ fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, const int32_t
                         int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride, int32_t pad, float* dx,
                         void* stream);
 
+/* grad_input of a convolution for any window, stride and map size, as two calls
+ * through column-major int32 accumulators (Eq. 21 with Sec. 5.3's per-sample
+ * scales, App. C Folder).  The first call is fqt1_bwd_input_gemm's integer
+ * product with acc stored column-major:
+ *   acc[k * ld_acc + r] = sum_j q[r, j] sign(W)[j, k] for the kept rows r (kept
+ *   order, r < kept_count * rows_per_group); entries of other rows are not written.
+ * ld_acc >= capacity * rows_per_group and a multiple of 4 (a multiple of 32 keeps
+ * every column 128-byte aligned); acc: [K][ld_acc] int32, 16-byte aligned. */
+fqt1_status fqt1_bwd_input_gemm_colmajor(const fqt1_qgrad* psq, const uint32_t* sw_col, int64_t M, int64_t D,
+                                         int64_t K, const fqt1_agp_params* p, int32_t* acc, int64_t ld_acc,
+                                         void* stream);
+
+/* The Folder of App. C on those accumulators, then the per-sample
+ * dequantization: the same dx as fqt1_col2im (bit for bit), read with every
+ * tap of a warp's 32 consecutive outputs as one contiguous run of a column.
+ * acc: [C kh kw][ld_acc] from fqt1_bwd_input_gemm_colmajor (the row of output
+ * pixel (oh, ow) of kept slot s is s Ho Wo + oh Wo + ow); dx: [N, C, H, W],
+ * pruned samples 0.  N <= 65535 and C H W < 2^31, else FQT1_ERR_UNSUPPORTED. */
+fqt1_status fqt1_col2im_colmajor(const int32_t* acc, int64_t ld_acc, const fqt1_qgrad* psq, const int32_t* colsum_w,
+                                 int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,
+                                 int32_t pad, float* dx, void* stream);
+
 /* grad_input of a convolution with the Folder fused into the product (Eq. 21 with
  * Sec. 5.3's per-sample scales, App. C Folder): the same dx as fqt1_bwd_input_gemm
  * followed by fqt1_col2im, without the int32 accumulators in memory.  A tile of 128

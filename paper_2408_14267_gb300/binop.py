@@ -144,6 +144,12 @@ class _BinaryProduct(torch.autograd.Function):
                 dx = torch.empty((N, H, W, C) if nhwc else (N, C, H, W), dtype=torch.float32, device=dev)
                 if fqt1.fold_supported(Ho, Wo, kh, kw, H, W):
                     fqt1.bwd_input_fold(psq, sw_col, cs_w, N, C, H, W, kh, kw, stride, pad, D, p_s, dx, nhwc=nhwc)
+                elif not nhwc:
+                    # column-major int32 accumulators: the Folder reads every tap as contiguous runs
+                    ld = (max(cap_s * rpg, 1) + 31) // 32 * 32
+                    acc_cm = torch.empty(K, ld, dtype=torch.int32, device=dev)
+                    fqt1.bwd_input_gemm_colmajor(psq, sw_col, M, D, K, p_s, acc_cm, ld)
+                    fqt1.col2im_colmajor(acc_cm, ld, psq, cs_w, N, C, H, W, kh, kw, stride, pad, dx)
                 else:
                     acc_dx = torch.empty(max(cap_s * rpg, 1), K, dtype=torch.int32, device=dev)
                     fqt1.bwd_input_gemm(psq, sw_col, cs_w, M, D, K, p_s, acc_dx, None)

@@ -432,11 +432,179 @@ __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
   }
 }
 
+// Folder on column-major int32 accumulators (the layout fqt1_bwd_input_gemm_colmajor writes):
+// acc[k * ld + r] for kept row r = slot Ho Wo + oh Wo + ow and column k = c kh kw + i kw + j.
+// A thread owns elements e = c H W + h W + w of one kept sample's dx plane; tap (i, j) of input
+// pixel (h, w) is the accumulator of output pixel oh = (h + pad - i) / stride,
+// ow = (w + pad - j) / stride when both divisions are exact and land in the output map.  The 32
+// lanes of a warp hold consecutive elements, so for each tap they read consecutive rows of one
+// column: every load is coalesced and nothing is staged.  KH, KW, S: compile-time window and
+// stride (0: taken from the arguments).
+struct FoldCmArgs {
+  const int32_t* acc;
+  int64_t ld;
+  const int32_t* kept_idx;
+  const int32_t* kept_count;
+  const float* scale;
+  const float* zero;
+  const int32_t* cs;
+  float* dx;
+  int H, W, kh, kw, stride, pad, Ho, Wo;
+  int64_t plane;  // C H W floats of one sample
+  FastDiv div_hw, div_w;
+  int K;          // C kh kw columns
+  int cs_smem;    // 1: the column sums are staged in shared memory (K <= 12288)
+};
+
+// Elements per thread of col2im_colmajor_kernel<KH, KW, S>: 4 for a runtime window, else by the
+// number c of tap candidates (a thread holds U c loaded accumulators): 1 for c >= 16, 2 for
+// c >= 4, 4 below (64 registers, 4 CTAs per SM).  The launcher sizes its grid with the same
+// function.
+__host__ __device__ constexpr int fold_cm_cand(int KH, int KW, int S) {
+  return ((KH + S - 1) / S) * ((KW + S - 1) / S);
+}
+__host__ __device__ constexpr int fold_cm_per(int KH, int KW, int S) {
+  return KH == 0 ? 4
+                 : (fold_cm_cand(KH, KW, S) >= 16 ? 1 : (fold_cm_cand(KH, KW, S) >= 4 ? 2 : 4));
+}
+
+template <int KH, int KW, int S>
+__global__ void __launch_bounds__(256, 4) col2im_colmajor_kernel(FoldCmArgs a) {
+  // With a compile-time window, an input pixel's taps are enumerated by residue: row taps
+  // i = rh + S mi (rh = (h + pad) mod S) land on output row oh = qh - mi (qh = (h + pad) / S),
+  // columns likewise, so only ceil(KH / S) ceil(KW / S) candidates exist (3 x 3 stride 1: 9,
+  // 7 x 7 stride 2: 16).  Every candidate's load is issued unconditionally from a clamped,
+  // valid address and masked afterwards, so a thread's loads are all in flight together; the
+  // column sums of the taps come from shared memory afterwards.
+  constexpr int SS = S > 0 ? S : 1;  // the compile-time stride (1 for a runtime window)
+  constexpr int CI = KH ? (KH + SS - 1) / SS : 1, CJ = KW ? (KW + SS - 1) / SS : 1;
+  constexpr int U = fold_cm_per(KH, KW, SS);  // elements per thread
+  extern __shared__ int32_t fold_cs[];        // [K] column sums when a.cs_smem
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  const int kh = KH ? KH : a.kh, kw = KW ? KW : a.kw, st = S ? S : a.stride;
+  const int khw = kh * kw, HW = a.H * a.W;
+  const int32_t* csb = a.cs;
+  if (a.cs_smem) {
+    for (int k = threadIdx.x; k < a.K; k += blockDim.x) fold_cs[k] = __ldg(a.cs + k);
+    __syncthreads();
+    csb = fold_cs;
+  }
+  // grid rows loop over the kept slots (the grid is sized by occupancy, not by the samples, so
+  // few CTAs are launched only to find their sample pruned)
+  const int kept = __ldg(a.kept_count);
+  for (int slot = (int)blockIdx.y; slot < kept; slot += (int)gridDim.y) {
+    const int n = __ldg(a.kept_idx + slot);
+    const int32_t* accs = a.acc + (int64_t)slot * a.Ho * a.Wo;
+    const float sc = __ldg(a.scale + slot), ze = __ldg(a.zero + slot);
+    const int64_t e0 = (int64_t)blockIdx.x * (256 * U) + threadIdx.x;
+    int32_t av[U], cv[U];
+    if (KH) {
+      int32_t va[U][CI * CJ];
+      uint32_t ok[U];
+      int cbase[U], rhv[U], rwv[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int64_t e = min(e0 + u * 256, a.plane - 1);  // clamped: every address is valid
+        const int c = (int)a.div_hw.div((uint32_t)e), pix = (int)e - c * HW;
+        const int h = (int)a.div_w.div((uint32_t)pix), w = pix - h * a.W;
+        const int32_t* col = accs + (int64_t)c * khw * a.ld;
+        const int hp = h + a.pad, wp = w + a.pad;
+        const int rh = SS == 1 ? 0 : hp % SS, qh = SS == 1 ? hp : hp / SS;
+        const int rw = SS == 1 ? 0 : wp % SS, qw = SS == 1 ? wp : wp / SS;
+        cbase[u] = c * khw;
+        rhv[u] = rh;
+        rwv[u] = rw;
+        uint32_t m = 0;
+#pragma unroll
+        for (int mi = 0; mi < CI; ++mi) {
+          const int i = rh + SS * mi, oh = qh - mi;
+          const bool vi = i < KH && oh >= 0 && oh < a.Ho;
+#pragma unroll
+          for (int mj = 0; mj < CJ; ++mj) {
+            const int j = rw + SS * mj, ow = qw - mj;
+            const bool v = vi && j < KW && ow >= 0 && ow < a.Wo;
+            m |= v ? 1u << (mi * CJ + mj) : 0u;
+            va[u][mi * CJ + mj] = __ldg(col + (v ? (int64_t)(i * KW + j) * a.ld + oh * a.Wo + ow : 0));
+          }
+        }
+        ok[u] = m;
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        int32_t sa = 0, sc_ = 0;
+#pragma unroll
+        for (int mi = 0; mi < CI; ++mi) {
+#pragma unroll
+          for (int mj = 0; mj < CJ; ++mj) {
+            const bool v = (ok[u] >> (mi * CJ + mj)) & 1u;
+            const int t = (rhv[u] + SS * mi) * KW + rwv[u] + SS * mj;
+            sa += v ? va[u][mi * CJ + mj] : 0;
+            sc_ += v ? csb[cbase[u] + t] : 0;
+          }
+        }
+        av[u] = sa;
+        cv[u] = sc_;
+      }
+    } else {
+      // runtime window: every tap tested in turn
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        av[u] = 0;
+        cv[u] = 0;
+        const int64_t e = e0 + u * 256;
+        if (e >= a.plane) continue;
+        const int c = (int)a.div_hw.div((uint32_t)e), pix = (int)e - c * HW;
+        const int h = (int)a.div_w.div((uint32_t)pix), w = pix - h * a.W;
+        const int32_t* col = accs + (int64_t)c * khw * a.ld;
+        const int32_t* csc = csb + c * khw;
+#pragma unroll 1
+        for (int i = 0; i < kh; ++i) {
+          const int hn = h + a.pad - i;
+          if (hn < 0) break;  // decreasing in i
+          if (hn % st) continue;
+          const int oh = hn / st;
+          if (oh >= a.Ho) continue;
+#pragma unroll 1
+          for (int j = 0; j < kw; ++j) {
+            const int wn = w + a.pad - j;
+            if (wn < 0) break;
+            if (wn % st) continue;
+            const int ow = wn / st;
+            if (ow >= a.Wo) continue;
+            const int t = i * kw + j;
+            av[u] += __ldg(col + (int64_t)t * a.ld + oh * a.Wo + ow);
+            cv[u] += csc[t];
+          }
+        }
+      }
+    }
+    float* out = a.dx + (int64_t)n * a.plane;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t e = e0 + u * 256;
+      if (e < a.plane)
+        out[e] = __fadd_rn(__fmul_rn(sc, __int2float_rn(av[u])), __fmul_rn(ze, __int2float_rn(cv[u])));
+    }
+  }  // kept slots
+}
+
 }  // namespace fqt1
 
 using namespace fqt1;
 
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+// SMs of the current device (cached per device ordinal; 152 if the query fails)
+static int sm_count_api() {
+  static std::atomic<int> cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152;
+  int v = cache[dev].load(std::memory_order_relaxed);
+  if (v > 0) return v;
+  if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v < 1) v = 152;
+  cache[dev].store(v, std::memory_order_relaxed);
+  return v;
+}
 static bool valid_bits(int b) { return b == 1 || b == 2 || b == 4 || b == 8; }
 
 extern "C" fqt1_status fqt1_fwd_gemm_bias(const uint32_t* sx_row, const uint32_t* sw_row, int64_t M, int64_t D,
@@ -656,6 +824,74 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
                                    int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,
                                    int32_t pad, float* dx, void* stream) {
   return col2im_impl(acc, psq, colsum_w, N, C, H, W, kh, kw, stride, pad, dx, 0, stream);
+}
+
+extern "C" fqt1_status fqt1_bwd_input_gemm_colmajor(const fqt1_qgrad* psq, const uint32_t* sw_col, int64_t M,
+                                                    int64_t D, int64_t K, const fqt1_agp_params* p, int32_t* acc,
+                                                    int64_t ld_acc, void* stream) {
+  if (!psq || !sw_col || !p || !acc || M < 1 || D < 1 || K < 1) return FQT1_ERR_INVALID_ARG;
+  if (!valid_bits(p->bits) || p->rows_per_group < 1 || M % p->rows_per_group) return FQT1_ERR_INVALID_ARG;
+  if (!psq->codes || !psq->kept_count || psq->ld_codes < fqt1_codes_ld(D) || psq->ld_codes % 16)
+    return FQT1_ERR_INVALID_ARG;
+  const int64_t rpg = p->rows_per_group;
+  const int64_t cap_rows = fqt1_kept_capacity(M / rpg, p->bits, p->mode) * rpg;
+  if (ld_acc < cap_rows || ld_acc % 4) return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(sw_col) || !aligned16(acc)) return FQT1_ERR_MISALIGNED;
+  if ((cap_rows + 63) / 64 > 65535) return FQT1_ERR_UNSUPPORTED;
+  FQT1_CUDA_TRY(launch_codes_tc_colmajor(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, rpg, sw_col,
+                                         K, D, acc, ld_acc, nullptr, (cudaStream_t)stream));
+  return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_col2im_colmajor(const int32_t* acc, int64_t ld_acc, const fqt1_qgrad* psq,
+                                            const int32_t* colsum_w, int32_t N, int32_t C, int32_t H, int32_t W,
+                                            int32_t kh, int32_t kw, int32_t stride, int32_t pad, float* dx,
+                                            void* stream) {
+  if (!acc || !psq || !colsum_w || !dx || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 ||
+      pad < 0 || kh > 64 || kw > 64)
+    return FQT1_ERR_INVALID_ARG;
+  if (!psq->slot_of_group || !psq->scale || !psq->zero || !psq->kept_idx || !psq->kept_count)
+    return FQT1_ERR_INVALID_ARG;
+  if (H + 2 * pad < kh || W + 2 * pad < kw) return FQT1_ERR_INVALID_ARG;
+  const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
+  if (ld_acc < (int64_t)Ho * Wo || ld_acc % 4) return FQT1_ERR_INVALID_ARG;
+  if (!aligned16(acc) || !aligned16(dx)) return FQT1_ERR_MISALIGNED;
+  const int64_t plane = (int64_t)C * H * W;
+  if (plane >= (1ll << 31) || N > 65535) return FQT1_ERR_UNSUPPORTED;
+  FoldCmArgs fa;
+  fa.acc = acc; fa.ld = ld_acc; fa.kept_idx = psq->kept_idx; fa.kept_count = psq->kept_count;
+  fa.scale = psq->scale; fa.zero = psq->zero; fa.cs = colsum_w; fa.dx = dx;
+  fa.H = H; fa.W = W; fa.kh = kh; fa.kw = kw; fa.stride = stride; fa.pad = pad; fa.Ho = Ho; fa.Wo = Wo;
+  fa.plane = plane; fa.div_hw = FastDiv((uint32_t)(H * W)); fa.div_w = FastDiv((uint32_t)W);
+  const int64_t K = (int64_t)C * kh * kw;
+  fa.K = (int)std::min<int64_t>(K, 0x7FFFFFFF);
+  fa.cs_smem = K <= 12288;
+  const size_t cs_bytes = fa.cs_smem ? (size_t)K * 4 : 0;
+  cudaStream_t s = (cudaStream_t)stream;
+  // pruned samples: zeros; kept samples: one grid row per slot (slots past the kept count exit)
+  launch_zero_pruned_rows(psq->slot_of_group, N, plane, 1, dx, s);
+  // grid: the plane's CTAs along x; along y about 16 CTAs per SM in all (a few resident waves),
+  // each grid row looping over kept slots y, y + gridDim.y, ...
+  auto grid = [&](int per) {
+    const int64_t gx = (plane + 256 * per - 1) / (256 * per);
+    const int64_t gy = std::max<int64_t>(1, std::min<int64_t>(N, (16 * (int64_t)sm_count_api() + gx - 1) / gx));
+    return dim3((unsigned)gx, (unsigned)gy);
+  };
+  if (kh == 3 && kw == 3 && stride == 1)
+    launch_k(col2im_colmajor_kernel<3, 3, 1>, grid(fold_cm_per(3, 3, 1)), dim3(256), cs_bytes, s, fa);
+  else if (kh == 3 && kw == 3 && stride == 2)
+    launch_k(col2im_colmajor_kernel<3, 3, 2>, grid(fold_cm_per(3, 3, 2)), dim3(256), cs_bytes, s, fa);
+  else if (kh == 1 && kw == 1 && stride == 1)
+    launch_k(col2im_colmajor_kernel<1, 1, 1>, grid(fold_cm_per(1, 1, 1)), dim3(256), cs_bytes, s, fa);
+  else if (kh == 1 && kw == 1 && stride == 2)
+    launch_k(col2im_colmajor_kernel<1, 1, 2>, grid(fold_cm_per(1, 1, 2)), dim3(256), cs_bytes, s, fa);
+  else if (kh == 7 && kw == 7 && stride == 2)
+    launch_k(col2im_colmajor_kernel<7, 7, 2>, grid(fold_cm_per(7, 7, 2)), dim3(256), cs_bytes, s, fa);
+  else
+    launch_k(col2im_colmajor_kernel<0, 0, 0>, grid(fold_cm_per(0, 0, 1)), dim3(256), cs_bytes, s, fa);
+  fqt1_count_launches(1);
+  FQT1_CUDA_TRY(cudaGetLastError());
+  return FQT1_OK;
 }
 
 extern "C" fqt1_status fqt1_col2im_nhwc(const int32_t* acc, const fqt1_qgrad* psq, const int32_t* colsum_w, int32_t N,

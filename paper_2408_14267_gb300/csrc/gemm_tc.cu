@@ -83,6 +83,9 @@ struct TcArgs {
   // y = dw[D][ldo] (kept channel kept_idx[r]: scale[r] acc + zero[r] cs[n]; pruned channels 0)
   const int32_t* slot_of_group;
   int64_t D;
+  // EPI_ACC32: 1 = acc is column-major, acc[col * ldo + row]; a warp's 32 rows of one column
+  // are then one 128-byte line, stored straight from the TMEM registers
+  int acc_cm;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -987,6 +990,17 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         }
         continue;
       }
+      if (a.epi == EPI_ACC32 && a.acc_cm) {
+        // column-major: lane = row, so each column's 32 rows leave as one coalesced line
+        const int64_t r = row_base + lane;
+        const bool rv = r < valid_rows && r < a.M;
+        int32_t* dst = a.acc + (n0 + c0) * a.ldo + r;
+        const int64_t ncol = a.N - (n0 + c0);  // > 0 here
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (rv && j < ncol) dst[j * a.ldo] = acc_int<kA512>(v[j]);
+        continue;
+      }
       if (a.epi == EPI_ACC32) {
         // the int32 accumulators through the warp's 4 KB staging block (row = lane, word j at
         // j ^ lane), then one coalesced 128-byte row segment per store (lanes over columns)
@@ -1596,6 +1610,16 @@ cudaError_t launch_wgrad_cluster_tc(int bits, const uint8_t* Q, int64_t ldq, int
   }
   if (bits == 8) return launch_tc<true, true, 128>(ma, mb, a, splits, s, nullptr, nullptr, true);
   return launch_tc<true, false, 128, false, 8>(ma, mb, a, splits, s, nullptr, nullptr, true);
+}
+
+// grad_input product with its int32 accumulators column-major: acc[k * ld + r] for the kept
+// rows r (EPI_ACC32 with acc_cm; ld >= max_rows).
+cudaError_t launch_codes_tc_colmajor(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
+                                     int64_t rows_per_count, const uint32_t* Sg, int64_t n_s, int64_t L,
+                                     int32_t* acc, int64_t ld, int32_t* status, cudaStream_t s) {
+  TcArgs a{};
+  a.acc = acc; a.ldo = ld; a.acc_cm = 1; a.rpg = rows_per_count; a.status = status;
+  return launch_codes_tc(bits, Q, ldq, max_rows, count, rows_per_count, Sg, n_s, L, EPI_ACC32, 1, a, s);
 }
 
 cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,

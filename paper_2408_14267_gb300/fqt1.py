@@ -71,6 +71,8 @@ _SIGS = {
     "fqt1_scq_quantize_noalloc": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, _VP]),
     "fqt1_bwd_input_gemm": (C.c_int, [_VP, _VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
     "fqt1_col2im": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
+    "fqt1_bwd_input_gemm_colmajor": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _I64, _VP]),
+    "fqt1_col2im_colmajor": (C.c_int, [_VP, _I64, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
     "fqt1_col2im_nhwc": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
     "fqt1_bwd_input_fold_nhwc": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP]),
     "fqt1_bwd_input_fold": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP]),
@@ -303,6 +305,16 @@ def col2im(acc, psq, colsum_w, N, Cin, H, W, kh, kw, stride, pad, dx, stream=Non
     fn = lib().fqt1_col2im_nhwc if nhwc else lib().fqt1_col2im
     _check(fn(_p(acc), C.byref(psq.c), _p(colsum_w), N, Cin, H, W, kh, kw, stride, pad, _p(dx), _s(stream)),
            "fqt1_col2im_nhwc" if nhwc else "fqt1_col2im")
+
+
+def bwd_input_gemm_colmajor(psq, sw_col, M, D, K, params, acc, ld_acc, stream=None):
+    _check(lib().fqt1_bwd_input_gemm_colmajor(C.byref(psq.c), _p(sw_col), M, D, K, C.byref(params), _p(acc), ld_acc,
+                                              _s(stream)), "fqt1_bwd_input_gemm_colmajor")
+
+
+def col2im_colmajor(acc, ld_acc, psq, colsum_w, N, Cin, H, W, kh, kw, stride, pad, dx, stream=None):
+    _check(lib().fqt1_col2im_colmajor(_p(acc), ld_acc, C.byref(psq.c), _p(colsum_w), N, Cin, H, W, kh, kw, stride,
+                                      pad, _p(dx), _s(stream)), "fqt1_col2im_colmajor")
 
 
 def bwd_input_fold(psq, sw_col, colsum_w, N, Cin, H, W, kh, kw, stride, pad, D, params, dx, stream=None,

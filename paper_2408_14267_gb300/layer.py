@@ -32,7 +32,7 @@ class LayerStep:
     int32 copy of the forward accumulators (the benchmark's configuration)."""
 
     def __init__(self, wl, device="cuda", keep_acc=True, fold=None, implicit=False, e4m3_weights=False,
-                 e4m3_x=False):
+                 e4m3_x=False, colmajor=None):
         dev = torch.device(device)
         self.kind = wl["kind"]
         self.keep_acc = keep_acc
@@ -66,6 +66,13 @@ class LayerStep:
             self.fold = (not keep_acc and ok) if fold is None else (fold and ok)
         else:
             self.fold = False
+        # convolutions without the fused Folder: grad_input through column-major int32
+        # accumulators and the column-major Folder (every tap read as contiguous runs), unless
+        # the row-major accumulators are kept (keep_acc) or colmajor is forced off
+        if self.kind == "conv" and not self.fold:
+            self.colmajor = (not keep_acc) if colmajor is None else bool(colmajor)
+        else:
+            self.colmajor = False
         # implicit-GEMM forward on request, where the library supports the convolution (off by
         # default: on the 8 x 8, 256-channel layer its two extra packing kernels cost more than
         # the Unfolder's row packing they replace)
@@ -129,6 +136,10 @@ class LayerStep:
         self.ws = fqt1.scq_workspace(M, D, K, rpg, dev)
         self.dev_status = torch.zeros(4, **i32)
         self.acc_dx = torch.empty(max(self.cap_s * rpg, 1), K, **i32)
+        # column-major copy for the column-major Folder: [K][ld_cm], ld_cm >= kept rows, a
+        # multiple of 32 so that every column starts on a 128-byte line
+        self.ld_cm = (max(self.cap_s * rpg, 1) + 31) // 32 * 32
+        self.acc_dx_cm = torch.empty(K, self.ld_cm, **i32) if self.colmajor else None
         self.dx = torch.empty(*(self.x.shape), **f32)
         self.acc_dw = torch.empty(max(self.cap_c, 1), K, **i32)
         self.dw = torch.empty(D, K, **f32)
@@ -212,6 +223,14 @@ class LayerStep:
                 st.append(("bwd_input_fold", lambda s: fqt1.bwd_input_fold(self.psq, self.sw_col, self.cs_w, N, Cin,
                                                                            H, W, kh, kw, self.stride, self.pad,
                                                                            self.D, self.p_s, self.dx, s)))
+        elif self.kind == "conv" and self.colmajor:
+            N, Cin, H, W, kh, kw = self.conv
+            st.append(("bwd_input_gemm", lambda s: fqt1.bwd_input_gemm_colmajor(self.psq, self.sw_col, self.M, self.D,
+                                                                                self.K, self.p_s, self.acc_dx_cm,
+                                                                                self.ld_cm, s)))
+            st.append(("col2im", lambda s: fqt1.col2im_colmajor(self.acc_dx_cm, self.ld_cm, self.psq, self.cs_w, N,
+                                                                Cin, H, W, kh, kw, self.stride, self.pad, self.dx,
+                                                                s)))
         elif self.kind == "conv":
             N, Cin, H, W, kh, kw = self.conv
             st.append(("bwd_input_gemm", lambda s: fqt1.bwd_input_gemm(self.psq, self.sw_col, self.cs_w, self.M,

@@ -74,6 +74,17 @@ def test_argument_validation_without_launch(lib):
     assert lib.fqt1_bwd_input_gemm(C.byref(q), fake, fake, 8, 8, 8, C.byref(bad_bits), fake, fake, s) == 1
     assert lib.fqt1_bwd_weight_gemm(C.byref(q), fake, fake, 8, 8, 8, C.byref(ok), None, fake, None, 0, s) == 1
     assert lib.fqt1_col2im(fake, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 0, 1, fake, s) == 1  # stride 0
+    # column-major grad_input: ld below the kept rows (capacity 4 of 8 groups, 1 row each) or
+    # not a multiple of 4; the Folder: stride 0, ld below Ho Wo, ld not a multiple of 4, and
+    # an unaligned accumulator pointer
+    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(ok), fake, 2, s) == 1
+    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(ok), fake, 6, s) == 1
+    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(bad_bits), fake, 8, s) == 1
+    assert lib.fqt1_col2im_colmajor(fake, 16, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 0, 1, fake, s) == 1
+    assert lib.fqt1_col2im_colmajor(fake, 12, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake, s) == 1
+    assert lib.fqt1_col2im_colmajor(fake, 18, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake, s) == 1
+    assert lib.fqt1_col2im_colmajor(C.c_void_p(0x10004), 16, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake,
+                                    s) == 2
 
 
 def test_implicit_conv_support_rules(lib):
