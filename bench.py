@@ -624,7 +624,7 @@ def layer_sweep(args):
     for net in (["vgg16", "resnet18"] if args.layers == "all" else [args.layers]):
         for wl in sets[net]():
             opts = {} if args.colmajor == "auto" else {"colmajor": args.colmajor == "on"}
-            st = LayerStep(wl, device=dev, keep_acc=False, **opts)
+            st = LayerStep(wl, device=dev, keep_acc=False, e4m3_weights=args.e4m3_weights == "on", **opts)
             with torch.cuda.stream(stream):
                 for _ in range(3):
                     st.step()
@@ -660,6 +660,8 @@ def layer_sweep(args):
                       "value": total_ops / (total_ms * 1e-3) / 1e12, "unit": "TOPS", "higher_is_better": True,
                       "steps": args.steps, "warmup": args.warmup, "dtype": "e4m3", "data": "synthetic",
                       "config": {"workload": f"{args.layers} layer shapes, b = 4, keep 1/4, SCQ",
+                                 "weights": ("e4m3 copies of sign(W) by TMA" if args.e4m3_weights == "on"
+                                             else "packed sign(W) expanded in the products"),
                                  "l2": "flushed before every timed replay (256 MiB write)",
                                  "timing": "one CUDA graph of the three-branch step per layer, CUDA events, median"},
                       "layers": rows}))

@@ -35,25 +35,34 @@ extern "C" int64_t fqt1_codes_ld(int64_t n) { return n < 1 ? 0 : ((n + 15) / 16)
 namespace fqt1 {
 
 // Rows of pruned groups of an [M][K] fp32 output are exactly zero.  Grid: x covers a row in
-// chunks of 1024 floats, y (and z for more than 65535 rows) the rows.
-__global__ void zero_pruned_rows_kernel(const int32_t* __restrict__ slot_of_group, int64_t M, int64_t K, int64_t rpg,
-                                        float* __restrict__ out) {
+// chunks of kZeroChunk floats (each thread kZeroVec float4 stores, strided by the block so
+// that every store instruction is coalesced), y (and z for more than 65535 rows) the rows.
+constexpr int kZeroVec = 8;
+constexpr int kZeroChunk = 256 * 4 * kZeroVec;
+__global__ void __launch_bounds__(256) zero_pruned_rows_kernel(const int32_t* __restrict__ slot_of_group, int64_t M,
+                                                               int64_t K, int64_t rpg, float* __restrict__ out) {
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
   const int64_t row = (int64_t)blockIdx.z * 65535 + blockIdx.y;
   if (row >= M || __ldg(slot_of_group + row / rpg) >= 0) return;
   float* dst = out + row * K;
-  const int64_t c = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 4;
-  if (c + 4 <= K && (K % 4) == 0) {
-    *reinterpret_cast<float4*>(dst + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+  const int64_t c0 = (int64_t)blockIdx.x * kZeroChunk + threadIdx.x * 4;
+  if ((K % 4) == 0) {
+#pragma unroll
+    for (int v = 0; v < kZeroVec; ++v) {
+      const int64_t c = c0 + v * 1024;
+      if (c < K) *reinterpret_cast<float4*>(dst + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
   } else {
-    for (int64_t j = c; j < c + 4 && j < K; ++j) dst[j] = 0.0f;
+    for (int v = 0; v < kZeroVec; ++v)
+      for (int64_t j = c0 + v * 1024; j < c0 + v * 1024 + 4 && j < K; ++j) dst[j] = 0.0f;
   }
 }
 
 static void launch_zero_pruned_rows(const int32_t* slot_of_group, int64_t M, int64_t K, int64_t rpg, float* out,
                                     cudaStream_t s) {
-  const dim3 grid((unsigned)((K + 1023) / 1024), (unsigned)(M < 65535 ? M : 65535), (unsigned)((M + 65534) / 65535));
+  const dim3 grid((unsigned)((K + kZeroChunk - 1) / kZeroChunk), (unsigned)(M < 65535 ? M : 65535),
+                  (unsigned)((M + 65534) / 65535));
   launch_k(zero_pruned_rows_kernel, dim3(grid), dim3(256), 0, s, slot_of_group, M, K, rpg, out);
   fqt1_count_launches(1);
 }
