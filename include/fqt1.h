@@ -387,24 +387,36 @@ fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, const int32_t
                         void* stream);
 
 /* grad_input of a convolution for any window, stride and map size, as two calls
- * through column-major int32 accumulators (Eq. 21 with Sec. 5.3's per-sample
+ * through column-major integer accumulators (Eq. 21 with Sec. 5.3's per-sample
  * scales, App. C Folder).  The first call is fqt1_bwd_input_gemm's integer
  * product with acc stored column-major:
  *   acc[k * ld_acc + r] = sum_j q[r, j] sign(W)[j, k] for the kept rows r (kept
  *   order, r < kept_count * rows_per_group); entries of other rows are not written.
- * ld_acc >= capacity * rows_per_group and a multiple of 4 (a multiple of 32 keeps
- * every column 128-byte aligned); acc: [K][ld_acc] int32, 16-byte aligned. */
+ * acc_bits: 32 (int32) or 16 (int16, exact when (2^bits - 1) * D <= 32767, else
+ * FQT1_ERR_INVALID_ARG; it halves the accumulators' traffic).  ld_acc >= capacity
+ * * rows_per_group and a multiple of 4 (int32) or 8 (int16); a multiple of 32
+ * keeps every column 128-byte aligned.  acc: [K][ld_acc], 16-byte aligned. */
 fqt1_status fqt1_bwd_input_gemm_colmajor(const fqt1_qgrad* psq, const uint32_t* sw_col, int64_t M, int64_t D,
-                                         int64_t K, const fqt1_agp_params* p, int32_t* acc, int64_t ld_acc,
-                                         void* stream);
+                                         int64_t K, const fqt1_agp_params* p, void* acc, int32_t acc_bits,
+                                         int64_t ld_acc, void* stream);
+
+/* The same product with sign(W)^T given as e4m3 bytes (+1 = 0x38, -1 = 0xB8, bytes
+ * past D zero), wt_e4m3: [K][ld_wt], ld_wt >= fqt1_codes_ld(D) and a multiple of 16
+ * (fqt1_binarize_pack_e4m3's transposed output): the B operand then goes to the
+ * tensor cores by TMA, unexpanded.  Same acc, bit for bit. */
+fqt1_status fqt1_bwd_input_gemm_colmajor_e4m3w(const fqt1_qgrad* psq, const uint8_t* wt_e4m3, int64_t ld_wt,
+                                               int64_t M, int64_t D, int64_t K, const fqt1_agp_params* p,
+                                               void* acc, int32_t acc_bits, int64_t ld_acc, void* stream);
 
 /* The Folder of App. C on those accumulators, then the per-sample
  * dequantization: the same dx as fqt1_col2im (bit for bit), read with every
  * tap of a warp's 32 consecutive outputs as one contiguous run of a column.
- * acc: [C kh kw][ld_acc] from fqt1_bwd_input_gemm_colmajor (the row of output
- * pixel (oh, ow) of kept slot s is s Ho Wo + oh Wo + ow); dx: [N, C, H, W],
- * pruned samples 0.  N <= 65535 and C H W < 2^31, else FQT1_ERR_UNSUPPORTED. */
-fqt1_status fqt1_col2im_colmajor(const int32_t* acc, int64_t ld_acc, const fqt1_qgrad* psq, const int32_t* colsum_w,
+ * acc: [C kh kw][ld_acc] from fqt1_bwd_input_gemm_colmajor with the same acc_bits
+ * (the row of output pixel (oh, ow) of kept slot s is s Ho Wo + oh Wo + ow); dx:
+ * [N, C, H, W], pruned samples 0.  N <= 65535 and C H W < 2^31, else
+ * FQT1_ERR_UNSUPPORTED. */
+fqt1_status fqt1_col2im_colmajor(const void* acc, int32_t acc_bits, int64_t ld_acc, const fqt1_qgrad* psq,
+                                 const int32_t* colsum_w,
                                  int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,
                                  int32_t pad, float* dx, void* stream);
 

@@ -147,9 +147,10 @@ class _BinaryProduct(torch.autograd.Function):
                 elif not nhwc:
                     # column-major int32 accumulators: the Folder reads every tap as contiguous runs
                     ld = (max(cap_s * rpg, 1) + 31) // 32 * 32
-                    acc_cm = torch.empty(K, ld, dtype=torch.int32, device=dev)
-                    fqt1.bwd_input_gemm_colmajor(psq, sw_col, M, D, K, p_s, acc_cm, ld)
-                    fqt1.col2im_colmajor(acc_cm, ld, psq, cs_w, N, C, H, W, kh, kw, stride, pad, dx)
+                    acc_t = torch.int16 if fqt1.colmajor_acc_bits(q.bits_s, D) == 16 else torch.int32
+                    acc_cm = torch.empty(K, ld, dtype=acc_t, device=dev)
+                    fqt1.bwd_input_gemm_colmajor(psq, sw_col, M, D, K, p_s, acc_cm)
+                    fqt1.col2im_colmajor(acc_cm, psq, cs_w, N, C, H, W, kh, kw, stride, pad, dx)
                 else:
                     acc_dx = torch.empty(max(cap_s * rpg, 1), K, dtype=torch.int32, device=dev)
                     fqt1.bwd_input_gemm(psq, sw_col, cs_w, M, D, K, p_s, acc_dx, None)

@@ -450,7 +450,7 @@ __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
 // column: every load is coalesced and nothing is staged.  KH, KW, S: compile-time window and
 // stride (0: taken from the arguments).
 struct FoldCmArgs {
-  const int32_t* acc;
+  const void* acc;  // int32 or int16 (the kernel's T)
   int64_t ld;
   const int32_t* kept_idx;
   const int32_t* kept_count;
@@ -477,7 +477,7 @@ __host__ __device__ constexpr int fold_cm_per(int KH, int KW, int S) {
                  : (fold_cm_cand(KH, KW, S) >= 16 ? 1 : (fold_cm_cand(KH, KW, S) >= 4 ? 2 : 4));
 }
 
-template <int KH, int KW, int S>
+template <int KH, int KW, int S, class T>
 __global__ void __launch_bounds__(256, 4) col2im_colmajor_kernel(FoldCmArgs a) {
   // With a compile-time window, an input pixel's taps are enumerated by residue: row taps
   // i = rh + S mi (rh = (h + pad) mod S) land on output row oh = qh - mi (qh = (h + pad) / S),
@@ -504,7 +504,7 @@ __global__ void __launch_bounds__(256, 4) col2im_colmajor_kernel(FoldCmArgs a) {
   const int kept = __ldg(a.kept_count);
   for (int slot = (int)blockIdx.y; slot < kept; slot += (int)gridDim.y) {
     const int n = __ldg(a.kept_idx + slot);
-    const int32_t* accs = a.acc + (int64_t)slot * a.Ho * a.Wo;
+    const T* accs = static_cast<const T*>(a.acc) + (int64_t)slot * a.Ho * a.Wo;
     const float sc = __ldg(a.scale + slot), ze = __ldg(a.zero + slot);
     const int64_t e0 = (int64_t)blockIdx.x * (256 * U) + threadIdx.x;
     int32_t av[U], cv[U];
@@ -517,7 +517,7 @@ __global__ void __launch_bounds__(256, 4) col2im_colmajor_kernel(FoldCmArgs a) {
         const int64_t e = min(e0 + u * 256, a.plane - 1);  // clamped: every address is valid
         const int c = (int)a.div_hw.div((uint32_t)e), pix = (int)e - c * HW;
         const int h = (int)a.div_w.div((uint32_t)pix), w = pix - h * a.W;
-        const int32_t* col = accs + (int64_t)c * khw * a.ld;
+        const T* col = accs + (int64_t)c * khw * a.ld;
         const int hp = h + a.pad, wp = w + a.pad;
         const int rh = SS == 1 ? 0 : hp % SS, qh = SS == 1 ? hp : hp / SS;
         const int rw = SS == 1 ? 0 : wp % SS, qw = SS == 1 ? wp : wp / SS;
@@ -534,7 +534,7 @@ __global__ void __launch_bounds__(256, 4) col2im_colmajor_kernel(FoldCmArgs a) {
             const int j = rw + SS * mj, ow = qw - mj;
             const bool v = vi && j < KW && ow >= 0 && ow < a.Wo;
             m |= v ? 1u << (mi * CJ + mj) : 0u;
-            va[u][mi * CJ + mj] = __ldg(col + (v ? (int64_t)(i * KW + j) * a.ld + oh * a.Wo + ow : 0));
+            va[u][mi * CJ + mj] = (int32_t)__ldg(col + (v ? (int64_t)(i * KW + j) * a.ld + oh * a.Wo + ow : 0));
           }
         }
         ok[u] = m;
@@ -565,7 +565,7 @@ __global__ void __launch_bounds__(256, 4) col2im_colmajor_kernel(FoldCmArgs a) {
         if (e >= a.plane) continue;
         const int c = (int)a.div_hw.div((uint32_t)e), pix = (int)e - c * HW;
         const int h = (int)a.div_w.div((uint32_t)pix), w = pix - h * a.W;
-        const int32_t* col = accs + (int64_t)c * khw * a.ld;
+        const T* col = accs + (int64_t)c * khw * a.ld;
         const int32_t* csc = csb + c * khw;
 #pragma unroll 1
         for (int i = 0; i < kh; ++i) {
@@ -582,7 +582,7 @@ __global__ void __launch_bounds__(256, 4) col2im_colmajor_kernel(FoldCmArgs a) {
             const int ow = wn / st;
             if (ow >= a.Wo) continue;
             const int t = i * kw + j;
-            av[u] += __ldg(col + (int64_t)t * a.ld + oh * a.Wo + ow);
+            av[u] += (int32_t)__ldg(col + (int64_t)t * a.ld + oh * a.Wo + ow);
             cv[u] += csc[t];
           }
         }
@@ -835,24 +835,43 @@ extern "C" fqt1_status fqt1_col2im(const int32_t* acc, const fqt1_qgrad* psq, co
   return col2im_impl(acc, psq, colsum_w, N, C, H, W, kh, kw, stride, pad, dx, 0, stream);
 }
 
-extern "C" fqt1_status fqt1_bwd_input_gemm_colmajor(const fqt1_qgrad* psq, const uint32_t* sw_col, int64_t M,
-                                                    int64_t D, int64_t K, const fqt1_agp_params* p, int32_t* acc,
-                                                    int64_t ld_acc, void* stream) {
-  if (!psq || !sw_col || !p || !acc || M < 1 || D < 1 || K < 1) return FQT1_ERR_INVALID_ARG;
+static fqt1_status bwd_input_colmajor_impl(const fqt1_qgrad* psq, const uint32_t* sw_col, const uint8_t* wt_e4m3,
+                                           int64_t ld_wt, int64_t M, int64_t D, int64_t K, const fqt1_agp_params* p,
+                                           void* acc, int32_t acc_bits, int64_t ld_acc, void* stream) {
+  if (!psq || !(sw_col || wt_e4m3) || !p || !acc || M < 1 || D < 1 || K < 1) return FQT1_ERR_INVALID_ARG;
+  if (acc_bits != 16 && acc_bits != 32) return FQT1_ERR_INVALID_ARG;
+  if (wt_e4m3 && (ld_wt < fqt1_codes_ld(D) || ld_wt % 16)) return FQT1_ERR_INVALID_ARG;
   if (!valid_bits(p->bits) || p->rows_per_group < 1 || M % p->rows_per_group) return FQT1_ERR_INVALID_ARG;
   if (!psq->codes || !psq->kept_count || psq->ld_codes < fqt1_codes_ld(D) || psq->ld_codes % 16)
     return FQT1_ERR_INVALID_ARG;
   const int64_t rpg = p->rows_per_group;
   const int64_t cap_rows = fqt1_kept_capacity(M / rpg, p->bits, p->mode) * rpg;
-  if (ld_acc < cap_rows || ld_acc % 4) return FQT1_ERR_INVALID_ARG;
-  if (!aligned16(sw_col) || !aligned16(acc)) return FQT1_ERR_MISALIGNED;
+  if (ld_acc < cap_rows || ld_acc % (acc_bits == 16 ? 8 : 4)) return FQT1_ERR_INVALID_ARG;
+  // int16 sums: every |acc| <= (2^b - 1) D must fit
+  if (acc_bits == 16 && ((1ll << p->bits) - 1) * D > 32767) return FQT1_ERR_INVALID_ARG;
+  if ((sw_col && !aligned16(sw_col)) || (wt_e4m3 && !aligned16(wt_e4m3)) || !aligned16(acc))
+    return FQT1_ERR_MISALIGNED;
   if ((cap_rows + 63) / 64 > 65535) return FQT1_ERR_UNSUPPORTED;
   FQT1_CUDA_TRY(launch_codes_tc_colmajor(p->bits, psq->codes, psq->ld_codes, cap_rows, psq->kept_count, rpg, sw_col,
-                                         K, D, acc, ld_acc, nullptr, (cudaStream_t)stream));
+                                         K, D, acc, acc_bits, ld_acc, nullptr, (cudaStream_t)stream, wt_e4m3, ld_wt));
   return FQT1_OK;
 }
 
-extern "C" fqt1_status fqt1_col2im_colmajor(const int32_t* acc, int64_t ld_acc, const fqt1_qgrad* psq,
+extern "C" fqt1_status fqt1_bwd_input_gemm_colmajor(const fqt1_qgrad* psq, const uint32_t* sw_col, int64_t M,
+                                                    int64_t D, int64_t K, const fqt1_agp_params* p, void* acc,
+                                                    int32_t acc_bits, int64_t ld_acc, void* stream) {
+  if (!sw_col) return FQT1_ERR_INVALID_ARG;
+  return bwd_input_colmajor_impl(psq, sw_col, nullptr, 0, M, D, K, p, acc, acc_bits, ld_acc, stream);
+}
+
+extern "C" fqt1_status fqt1_bwd_input_gemm_colmajor_e4m3w(const fqt1_qgrad* psq, const uint8_t* wt_e4m3, int64_t ld_wt,
+                                                          int64_t M, int64_t D, int64_t K, const fqt1_agp_params* p,
+                                                          void* acc, int32_t acc_bits, int64_t ld_acc, void* stream) {
+  if (!wt_e4m3) return FQT1_ERR_INVALID_ARG;
+  return bwd_input_colmajor_impl(psq, nullptr, wt_e4m3, ld_wt, M, D, K, p, acc, acc_bits, ld_acc, stream);
+}
+
+extern "C" fqt1_status fqt1_col2im_colmajor(const void* acc, int32_t acc_bits, int64_t ld_acc, const fqt1_qgrad* psq,
                                             const int32_t* colsum_w, int32_t N, int32_t C, int32_t H, int32_t W,
                                             int32_t kh, int32_t kw, int32_t stride, int32_t pad, float* dx,
                                             void* stream) {
@@ -863,7 +882,8 @@ extern "C" fqt1_status fqt1_col2im_colmajor(const int32_t* acc, int64_t ld_acc, 
     return FQT1_ERR_INVALID_ARG;
   if (H + 2 * pad < kh || W + 2 * pad < kw) return FQT1_ERR_INVALID_ARG;
   const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
-  if (ld_acc < (int64_t)Ho * Wo || ld_acc % 4) return FQT1_ERR_INVALID_ARG;
+  if (acc_bits != 16 && acc_bits != 32) return FQT1_ERR_INVALID_ARG;
+  if (ld_acc < (int64_t)Ho * Wo || ld_acc % (acc_bits == 16 ? 8 : 4)) return FQT1_ERR_INVALID_ARG;
   if (!aligned16(acc) || !aligned16(dx)) return FQT1_ERR_MISALIGNED;
   const int64_t plane = (int64_t)C * H * W;
   if (plane >= (1ll << 31) || N > 65535) return FQT1_ERR_UNSUPPORTED;
@@ -886,18 +906,25 @@ extern "C" fqt1_status fqt1_col2im_colmajor(const int32_t* acc, int64_t ld_acc, 
     const int64_t gy = std::max<int64_t>(1, std::min<int64_t>(N, (16 * (int64_t)sm_count_api() + gx - 1) / gx));
     return dim3((unsigned)gx, (unsigned)gy);
   };
-  if (kh == 3 && kw == 3 && stride == 1)
-    launch_k(col2im_colmajor_kernel<3, 3, 1>, grid(fold_cm_per(3, 3, 1)), dim3(256), cs_bytes, s, fa);
-  else if (kh == 3 && kw == 3 && stride == 2)
-    launch_k(col2im_colmajor_kernel<3, 3, 2>, grid(fold_cm_per(3, 3, 2)), dim3(256), cs_bytes, s, fa);
-  else if (kh == 1 && kw == 1 && stride == 1)
-    launch_k(col2im_colmajor_kernel<1, 1, 1>, grid(fold_cm_per(1, 1, 1)), dim3(256), cs_bytes, s, fa);
-  else if (kh == 1 && kw == 1 && stride == 2)
-    launch_k(col2im_colmajor_kernel<1, 1, 2>, grid(fold_cm_per(1, 1, 2)), dim3(256), cs_bytes, s, fa);
-  else if (kh == 7 && kw == 7 && stride == 2)
-    launch_k(col2im_colmajor_kernel<7, 7, 2>, grid(fold_cm_per(7, 7, 2)), dim3(256), cs_bytes, s, fa);
+  auto launch = [&](auto zero) {  // zero: a value of the accumulator type
+    using T = decltype(zero);
+    if (kh == 3 && kw == 3 && stride == 1)
+      launch_k(col2im_colmajor_kernel<3, 3, 1, T>, grid(fold_cm_per(3, 3, 1)), dim3(256), cs_bytes, s, fa);
+    else if (kh == 3 && kw == 3 && stride == 2)
+      launch_k(col2im_colmajor_kernel<3, 3, 2, T>, grid(fold_cm_per(3, 3, 2)), dim3(256), cs_bytes, s, fa);
+    else if (kh == 1 && kw == 1 && stride == 1)
+      launch_k(col2im_colmajor_kernel<1, 1, 1, T>, grid(fold_cm_per(1, 1, 1)), dim3(256), cs_bytes, s, fa);
+    else if (kh == 1 && kw == 1 && stride == 2)
+      launch_k(col2im_colmajor_kernel<1, 1, 2, T>, grid(fold_cm_per(1, 1, 2)), dim3(256), cs_bytes, s, fa);
+    else if (kh == 7 && kw == 7 && stride == 2)
+      launch_k(col2im_colmajor_kernel<7, 7, 2, T>, grid(fold_cm_per(7, 7, 2)), dim3(256), cs_bytes, s, fa);
+    else
+      launch_k(col2im_colmajor_kernel<0, 0, 0, T>, grid(fold_cm_per(0, 0, 1)), dim3(256), cs_bytes, s, fa);
+  };
+  if (acc_bits == 16)
+    launch(int16_t{0});
   else
-    launch_k(col2im_colmajor_kernel<0, 0, 0>, grid(fold_cm_per(0, 0, 1)), dim3(256), cs_bytes, s, fa);
+    launch(int32_t{0});
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
   return FQT1_OK;

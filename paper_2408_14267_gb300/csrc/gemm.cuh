@@ -24,10 +24,13 @@ cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int6
                                    int64_t ldbe = 0);
 enum : int { GEMM_EPI_ACC32 = 1, GEMM_EPI_RED = 2, GEMM_EPI_DX = 3 };
 // The same product with EPI_ACC32 accumulators column-major: acc[n * ld + r] (ld >= max_rows),
-// each warp's 32 rows of a column stored as one line straight from the TMEM registers.
+// each warp's 32 rows of a column stored as one line straight from the TMEM registers; acc_bits
+// 32 (int32) or 16 (int16, when every sum fits).  Be (optional): e4m3 sign(W)^T rows [n_s][ldbe]
+// bytes by TMA instead of the packed columns Sg.
 cudaError_t launch_codes_tc_colmajor(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
                                      int64_t rows_per_count, const uint32_t* Sg, int64_t n_s, int64_t L,
-                                     int32_t* acc, int64_t ld, int32_t* status, cudaStream_t s);
+                                     void* acc, int acc_bits, int64_t ld, int32_t* status, cudaStream_t s,
+                                     const uint8_t* Be = nullptr, int64_t ldbe = 0);
 // Bte: e4m3 sign(W)^T rows [K][ldbte] bytes, or null for the packed sign(W) columns Sg.
 // nhwc: dx in memory order N, H, W, C.
 cudaError_t launch_fold_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,

@@ -83,8 +83,9 @@ struct TcArgs {
   // y = dw[D][ldo] (kept channel kept_idx[r]: scale[r] acc + zero[r] cs[n]; pruned channels 0)
   const int32_t* slot_of_group;
   int64_t D;
-  // EPI_ACC32: 1 = acc is column-major, acc[col * ldo + row]; a warp's 32 rows of one column
-  // are then one 128-byte line, stored straight from the TMEM registers
+  // EPI_ACC32: 1 = acc is column-major int32, acc[col * ldo + row]; a warp's 32 rows of one
+  // column are then one 128-byte line, stored straight from the TMEM registers; 2 = the same
+  // as int16 (the host checks that every sum fits: (2^b - 1) * contraction < 2^15)
   int acc_cm;
 };
 
@@ -996,6 +997,13 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
         const bool rv = r < valid_rows && r < a.M;
         int32_t* dst = a.acc + (n0 + c0) * a.ldo + r;
         const int64_t ncol = a.N - (n0 + c0);  // > 0 here
+        if (a.acc_cm == 2) {
+          int16_t* dst16 = reinterpret_cast<int16_t*>(a.acc) + (n0 + c0) * a.ldo + r;
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (rv && j < ncol) dst16[j * a.ldo] = (int16_t)acc_int<kA512>(v[j]);
+          continue;
+        }
 #pragma unroll
         for (int j = 0; j < 32; ++j)
           if (rv && j < ncol) dst[j * a.ldo] = acc_int<kA512>(v[j]);
@@ -1485,6 +1493,8 @@ cudaError_t launch_codes_tc(int bits, const uint8_t* Q, int64_t ldq, int64_t max
   const bool short_tile = a.tiles_per_split == 1 && !a.tma_out;
   if (Be) {
     if (bits == 8) return launch_tc<true, true, 128, false, 2>(ma, mb, a, z, s);
+    const bool persist_b = short_tile && z == 1 && out_tiles(a, 128) > tile_wave(true);
+    if (persist_b) return launch_tc<true, false, 128, true, 2 | 8 | 64 | 128>(ma, mb, a, z, s);
     if (short_tile) return launch_tc<true, false, 128, true, 2 | 8 | 64>(ma, mb, a, z, s);
     return launch_tc<true, false, 128, false, 2 | 8>(ma, mb, a, z, s);
   }
@@ -1616,10 +1626,12 @@ cudaError_t launch_wgrad_cluster_tc(int bits, const uint8_t* Q, int64_t ldq, int
 // rows r (EPI_ACC32 with acc_cm; ld >= max_rows).
 cudaError_t launch_codes_tc_colmajor(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,
                                      int64_t rows_per_count, const uint32_t* Sg, int64_t n_s, int64_t L,
-                                     int32_t* acc, int64_t ld, int32_t* status, cudaStream_t s) {
+                                     void* acc, int acc_bits, int64_t ld, int32_t* status, cudaStream_t s,
+                                     const uint8_t* Be, int64_t ldbe) {
   TcArgs a{};
-  a.acc = acc; a.ldo = ld; a.acc_cm = 1; a.rpg = rows_per_count; a.status = status;
-  return launch_codes_tc(bits, Q, ldq, max_rows, count, rows_per_count, Sg, n_s, L, EPI_ACC32, 1, a, s);
+  a.acc = reinterpret_cast<int32_t*>(acc); a.ldo = ld; a.acc_cm = acc_bits == 16 ? 2 : 1;
+  a.rpg = rows_per_count; a.status = status;
+  return launch_codes_tc(bits, Q, ldq, max_rows, count, rows_per_count, Sg, n_s, L, EPI_ACC32, 1, a, s, Be, ldbe);
 }
 
 cudaError_t launch_codes_tc_simple(int bits, const uint8_t* Q, int64_t ldq, int64_t max_rows, const int32_t* count,

@@ -71,8 +71,10 @@ _SIGS = {
     "fqt1_scq_quantize_noalloc": (C.c_int, [_VP, _I64, _I64, _VP, _VP, _VP, _VP, _VP, _VP, _VP]),
     "fqt1_bwd_input_gemm": (C.c_int, [_VP, _VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _VP]),
     "fqt1_col2im": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
-    "fqt1_bwd_input_gemm_colmajor": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _I64, _VP]),
-    "fqt1_col2im_colmajor": (C.c_int, [_VP, _I64, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
+    "fqt1_bwd_input_gemm_colmajor": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _I32, _I64, _VP]),
+    "fqt1_col2im_colmajor": (C.c_int, [_VP, _I32, _I64, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
+    "fqt1_bwd_input_gemm_colmajor_e4m3w": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _I64, _VP, _VP, _I32, _I64,
+                                                     _VP]),
     "fqt1_col2im_nhwc": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
     "fqt1_bwd_input_fold_nhwc": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP]),
     "fqt1_bwd_input_fold": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_I64, _VP, _VP, _VP]),
@@ -307,14 +309,31 @@ def col2im(acc, psq, colsum_w, N, Cin, H, W, kh, kw, stride, pad, dx, stream=Non
            "fqt1_col2im_nhwc" if nhwc else "fqt1_col2im")
 
 
-def bwd_input_gemm_colmajor(psq, sw_col, M, D, K, params, acc, ld_acc, stream=None):
-    _check(lib().fqt1_bwd_input_gemm_colmajor(C.byref(psq.c), _p(sw_col), M, D, K, C.byref(params), _p(acc), ld_acc,
-                                              _s(stream)), "fqt1_bwd_input_gemm_colmajor")
+def _acc_bits(acc):
+    return {torch.int16: 16, torch.int32: 32}[acc.dtype]
 
 
-def col2im_colmajor(acc, ld_acc, psq, colsum_w, N, Cin, H, W, kh, kw, stride, pad, dx, stream=None):
-    _check(lib().fqt1_col2im_colmajor(_p(acc), ld_acc, C.byref(psq.c), _p(colsum_w), N, Cin, H, W, kh, kw, stride,
-                                      pad, _p(dx), _s(stream)), "fqt1_col2im_colmajor")
+def bwd_input_gemm_colmajor(psq, sw_col, M, D, K, params, acc, stream=None):
+    """acc: [K][ld] int32 or int16 (its dtype selects the accumulator width)."""
+    _check(lib().fqt1_bwd_input_gemm_colmajor(C.byref(psq.c), _p(sw_col), M, D, K, C.byref(params), _p(acc),
+                                              _acc_bits(acc), acc.shape[1], _s(stream)),
+           "fqt1_bwd_input_gemm_colmajor")
+
+
+def bwd_input_gemm_colmajor_e4m3w(psq, wt8, M, D, K, params, acc, stream=None):
+    _check(lib().fqt1_bwd_input_gemm_colmajor_e4m3w(C.byref(psq.c), _p(wt8), wt8.shape[1], M, D, K, C.byref(params),
+                                                    _p(acc), _acc_bits(acc), acc.shape[1], _s(stream)),
+           "fqt1_bwd_input_gemm_colmajor_e4m3w")
+
+
+def col2im_colmajor(acc, psq, colsum_w, N, Cin, H, W, kh, kw, stride, pad, dx, stream=None):
+    _check(lib().fqt1_col2im_colmajor(_p(acc), _acc_bits(acc), acc.shape[1], C.byref(psq.c), _p(colsum_w), N, Cin, H,
+                                      W, kh, kw, stride, pad, _p(dx), _s(stream)), "fqt1_col2im_colmajor")
+
+
+def colmajor_acc_bits(bits, D):
+    """16 when every grad_input accumulator fits int16 ((2^bits - 1) D <= 32767), else 32."""
+    return 16 if ((1 << bits) - 1) * D <= 32767 else 32
 
 
 def bwd_input_fold(psq, sw_col, colsum_w, N, Cin, H, W, kh, kw, stride, pad, D, params, dx, stream=None,

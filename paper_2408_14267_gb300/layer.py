@@ -32,7 +32,7 @@ class LayerStep:
     int32 copy of the forward accumulators (the benchmark's configuration)."""
 
     def __init__(self, wl, device="cuda", keep_acc=True, fold=None, implicit=False, e4m3_weights=False,
-                 e4m3_x=False, colmajor=None):
+                 e4m3_x=False, colmajor=None, acc16=True):
         dev = torch.device(device)
         self.kind = wl["kind"]
         self.keep_acc = keep_acc
@@ -120,6 +120,10 @@ class LayerStep:
         e_fold = e4m3_weights is True or e4m3_weights == "fold"
         self.w8 = torch.empty(D, fqt1.codes_ld(K), **u8) if e_fwd and not self.implicit else None
         self.wt8 = torch.empty(K, fqt1.codes_ld(D), **u8) if e_fold and self.fold else None
+        # e4m3 sign(W)^T for the column-major product on request only (e4m3_weights="colmajor"):
+        # measured no faster than the packed signs there
+        if e4m3_weights == "colmajor" and self.colmajor:
+            self.wt8 = torch.empty(K, fqt1.codes_ld(D), **u8)
         self.sw_col = torch.empty(K, wD, **i32)
         self.cs_w = torch.empty(K, **i32)
         self.acc_y = torch.empty(M, D, **i32) if keep_acc else None
@@ -136,10 +140,13 @@ class LayerStep:
         self.ws = fqt1.scq_workspace(M, D, K, rpg, dev)
         self.dev_status = torch.zeros(4, **i32)
         self.acc_dx = torch.empty(max(self.cap_s * rpg, 1), K, **i32)
-        # column-major copy for the column-major Folder: [K][ld_cm], ld_cm >= kept rows, a
-        # multiple of 32 so that every column starts on a 128-byte line
+        # column-major accumulators for the column-major Folder: [K][ld_cm], ld_cm >= kept rows, a
+        # multiple of 32 so that every column starts on a 128-byte line; int16 where every sum
+        # fits (acc_bits_cm: (2^b - 1) D <= 32767), which halves their traffic, else int32
         self.ld_cm = (max(self.cap_s * rpg, 1) + 31) // 32 * 32
-        self.acc_dx_cm = torch.empty(K, self.ld_cm, **i32) if self.colmajor else None
+        self.acc_bits_cm = fqt1.colmajor_acc_bits(wl["bits_s"], D) if acc16 else 32
+        cm_type = torch.int16 if self.acc_bits_cm == 16 else torch.int32
+        self.acc_dx_cm = torch.empty(K, self.ld_cm, dtype=cm_type, device=dev) if self.colmajor else None
         self.dx = torch.empty(*(self.x.shape), **f32)
         self.acc_dw = torch.empty(max(self.cap_c, 1), K, **i32)
         self.dw = torch.empty(D, K, **f32)
@@ -225,12 +232,14 @@ class LayerStep:
                                                                            self.D, self.p_s, self.dx, s)))
         elif self.kind == "conv" and self.colmajor:
             N, Cin, H, W, kh, kw = self.conv
-            st.append(("bwd_input_gemm", lambda s: fqt1.bwd_input_gemm_colmajor(self.psq, self.sw_col, self.M, self.D,
-                                                                                self.K, self.p_s, self.acc_dx_cm,
-                                                                                self.ld_cm, s)))
-            st.append(("col2im", lambda s: fqt1.col2im_colmajor(self.acc_dx_cm, self.ld_cm, self.psq, self.cs_w, N,
-                                                                Cin, H, W, kh, kw, self.stride, self.pad, self.dx,
-                                                                s)))
+            if self.wt8 is not None:
+                st.append(("bwd_input_gemm", lambda s: fqt1.bwd_input_gemm_colmajor_e4m3w(
+                    self.psq, self.wt8, self.M, self.D, self.K, self.p_s, self.acc_dx_cm, s)))
+            else:
+                st.append(("bwd_input_gemm", lambda s: fqt1.bwd_input_gemm_colmajor(
+                    self.psq, self.sw_col, self.M, self.D, self.K, self.p_s, self.acc_dx_cm, s)))
+            st.append(("col2im", lambda s: fqt1.col2im_colmajor(self.acc_dx_cm, self.psq, self.cs_w, N, Cin, H, W, kh,
+                                                                kw, self.stride, self.pad, self.dx, s)))
         elif self.kind == "conv":
             N, Cin, H, W, kh, kw = self.conv
             st.append(("bwd_input_gemm", lambda s: fqt1.bwd_input_gemm(self.psq, self.sw_col, self.cs_w, self.M,

@@ -77,13 +77,21 @@ def test_argument_validation_without_launch(lib):
     # column-major grad_input: ld below the kept rows (capacity 4 of 8 groups, 1 row each) or
     # not a multiple of 4; the Folder: stride 0, ld below Ho Wo, ld not a multiple of 4, and
     # an unaligned accumulator pointer
-    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(ok), fake, 2, s) == 1
-    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(ok), fake, 6, s) == 1
-    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(bad_bits), fake, 8, s) == 1
-    assert lib.fqt1_col2im_colmajor(fake, 16, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 0, 1, fake, s) == 1
-    assert lib.fqt1_col2im_colmajor(fake, 12, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake, s) == 1
-    assert lib.fqt1_col2im_colmajor(fake, 18, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake, s) == 1
-    assert lib.fqt1_col2im_colmajor(C.c_void_p(0x10004), 16, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake,
+    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(ok), fake, 32, 2, s) == 1
+    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(ok), fake, 32, 6, s) == 1
+    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(bad_bits), fake, 32, 8, s) == 1
+    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(ok), fake, 8, 8, s) == 1  # width 8
+    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(ok), fake, 16, 4, s) == 1  # ld % 8
+    big_d = fqt1.AgpParams(4, 0, 1, 1)  # 15 * 4096 > 32767: int16 cannot hold the sums
+    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 4096, 8, C.byref(big_d), fake, 16, 8, s) == 1
+    assert lib.fqt1_bwd_input_gemm_colmajor_e4m3w(C.byref(q), fake, 8, 8, 8, 8, C.byref(ok), fake, 32, 8, s) == 1
+    assert lib.fqt1_bwd_input_gemm_colmajor_e4m3w(C.byref(q), None, 16, 8, 8, 8, C.byref(ok), fake, 32, 8, s) == 1
+    assert lib.fqt1_col2im_colmajor(fake, 32, 16, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 0, 1, fake, s) == 1
+    assert lib.fqt1_col2im_colmajor(fake, 32, 12, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake, s) == 1
+    assert lib.fqt1_col2im_colmajor(fake, 32, 18, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake, s) == 1
+    assert lib.fqt1_col2im_colmajor(fake, 16, 20, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake, s) == 1
+    assert lib.fqt1_col2im_colmajor(fake, 24, 16, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake, s) == 1
+    assert lib.fqt1_col2im_colmajor(C.c_void_p(0x10004), 32, 16, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake,
                                     s) == 2
 
 

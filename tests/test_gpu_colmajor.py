@@ -76,8 +76,8 @@ def test_colmajor_grad_input_matches_oracle_and_row_major_folder(name, make):
     psq = ref["psq"]
     rows = len(psq["kept"]) * cm.rpg
     assert cm.psq.count() == len(psq["kept"])
-    acc = cm.acc_dx_cm.cpu().numpy()[:, :rows].T
-    assert np.array_equal(acc, ref["acc_dx"]), "column-major int32 accumulators"
+    acc = cm.acc_dx_cm.cpu().numpy()[:, :rows].T.astype(np.int64)
+    assert np.array_equal(acc, ref["acc_dx"]), f"column-major int{cm.acc_bits_cm} accumulators"
     assert torch.equal(cm.dx, rm.dx), "column-major Folder against the row-major Folder"
     a_mag = np.zeros(ref["dx"].shape)
     c_mag = np.zeros(ref["dx"].shape)
@@ -104,3 +104,48 @@ def test_colmajor_is_the_default_without_fused_folder():
     st = LayerStep(wl.resnet18_cifar_conv(), keep_acc=False)
     assert st.fold and not st.colmajor
     assert not LayerStep(COLMAJOR_CASES[0][1](), keep_acc=True).colmajor
+
+
+@pytest.mark.parametrize("name,make", [COLMAJOR_CASES[i] for i in (0, 2, 6, 8)],
+                         ids=[COLMAJOR_CASES[i][0] for i in (0, 2, 6, 8)])
+def test_colmajor_e4m3_weights_equal_packed(name, make):
+    """fqt1_bwd_input_gemm_colmajor_e4m3w (sign(W)^T bytes by TMA) gives the packed-sign
+    product's accumulators and dx bit for bit."""
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    a = LayerStep(w, keep_acc=False, fold=False, colmajor=True, e4m3_weights="colmajor")
+    b = LayerStep(w, keep_acc=False, fold=False, colmajor=True, e4m3_weights=False)
+    assert a.wt8 is not None and b.wt8 is None
+    a.step()
+    b.step()
+    torch.cuda.synchronize()
+    rows = a.psq.count() * a.rpg
+    assert rows == b.psq.count() * b.rpg
+    assert torch.equal(a.acc_dx_cm[:, :rows], b.acc_dx_cm[:, :rows])
+    assert torch.equal(a.dx, b.dx)
+
+
+@pytest.mark.parametrize("name,make", [COLMAJOR_CASES[i] for i in (0, 3, 6, 8, 10)],
+                         ids=[COLMAJOR_CASES[i][0] for i in (0, 3, 6, 8, 10)])
+def test_colmajor_int16_equals_int32(name, make):
+    """int16 column-major accumulators (chosen where (2^b - 1) D fits) give the int32 path's
+    accumulators and dx bit for bit."""
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    a = LayerStep(w, keep_acc=False, fold=False, colmajor=True, acc16=True)
+    b = LayerStep(w, keep_acc=False, fold=False, colmajor=True, acc16=False)
+    assert a.acc_bits_cm == 16 and b.acc_bits_cm == 32
+    a.step()
+    b.step()
+    torch.cuda.synchronize()
+    rows = a.psq.count() * a.rpg
+    assert torch.equal(a.acc_dx_cm[:, :rows].to(torch.int32), b.acc_dx_cm[:, :rows])
+    assert torch.equal(a.dx, b.dx)
+
+
+def test_colmajor_int16_bound():
+    """int16 is taken exactly when every accumulator fits: (2^b - 1) D <= 32767."""
+    from paper_2408_14267_gb300 import fqt1
+    assert fqt1.colmajor_acc_bits(4, 2184) == 16 and fqt1.colmajor_acc_bits(4, 2185) == 32
+    assert fqt1.colmajor_acc_bits(8, 128) == 16 and fqt1.colmajor_acc_bits(8, 129) == 32
+    assert fqt1.colmajor_acc_bits(1, 32767) == 16 and fqt1.colmajor_acc_bits(1, 32768) == 32
