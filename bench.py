@@ -326,6 +326,9 @@ def main():
                          "operand of the forward and grad_weight products")
     ap.add_argument("--profile", type=int, default=0, metavar="N",
                     help="only run --warmup + N eager steps (for ncu), print nothing")
+    ap.add_argument("--profile-layer", metavar="NAME",
+                    help="with --profile: the eager steps run this layer of the --layers sweep instead "
+                         "(e.g. resnet18.stem, resnet18.layer1, vgg16.conv2)")
     ap.add_argument("--table5", action="store_true",
                     help="GEMM-only comparison of average 1-bit and 1-bit products on the Table 5 shapes")
     ap.add_argument("--model", choices=["vgg16", "resnet18"],
@@ -373,6 +376,11 @@ def main():
     from paper_2408_14267_gb300.layer import LayerStep
 
     wl = workloads.resnet18_cifar_conv()
+    if args.profile and args.profile_layer:  # another layer shape of the sweep, for ncu
+        named = {w["name"].split()[0]: w for w in workloads.vgg16_layers(bits=4) + workloads.resnet18_imagenet_layers()}
+        if args.profile_layer not in named:
+            raise SystemExit(f"--profile-layer: one of {sorted(named)}")
+        wl = named[args.profile_layer]
     st = LayerStep(wl, device=f"cuda:{local_rank}", keep_acc=False, implicit=args.implicit,
                    e4m3_weights=args.e4m3_weights == "on", e4m3_x=args.e4m3_x == "on")
     stream = torch.cuda.Stream()
