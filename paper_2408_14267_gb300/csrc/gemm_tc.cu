@@ -917,10 +917,16 @@ __global__ void __launch_bounds__(kThreads, SHORT ? 2 : 1)
       if (fold_zero_issued) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
     } else {
     const int q = warp & 3;                         // TMEM lane quarter of this warp
-    const int cbeg = ((warp - 2) >> 2) * (BN / 2);  // its half of the accumulator columns
+    // its share of the accumulator columns: the tile's 32-column chunks below N (all BN for the
+    // cluster reduction, which reads every column of its partial tiles), the first half to warps
+    // 2..5 and the rest to warps 6..9, so that a tile narrower than BN (64 output channels)
+    // still spreads its epilogue over all eight warps (at most BN / 64 chunks per warp)
+    const int nchunks = a.epi == EPI_CRED ? BN / 32 : (int)min((int64_t)(BN / 32), (a.N - n0 + 31) / 32);
+    const int half = (nchunks + 1) >> 1;
+    const int cbeg = (warp >= 6 ? half : 0) * 32, cend = (warp >= 6 ? nchunks : half) * 32;
     uint32_t* stage = reinterpret_cast<uint32_t*>(base) + (warp - 2) * 1024;  // 4 KB per warp (operand ring is idle)
     const int64_t row_base = m0 + 32 * q;
-    for (int c0 = cbeg; c0 < cbeg + BN / 2; c0 += 32) {
+    for (int c0 = cbeg; c0 < cend; c0 += 32) {
       // accumulator columns past N hold no output (warp-uniform; the cluster reduction reads
       // every column of its partial tiles)
       if (a.epi != EPI_CRED && n0 + c0 >= a.N) break;
