@@ -773,7 +773,8 @@ def gemm_sweep(args):
                NUMEXPR_NUM_THREADS="1")
     for (M, K, D, G, b) in sweep_points(args.sweep):
         wl = workloads.sweep_point_device(M, K, D, G, b, dev)
-        st = LayerStep(wl, device=dev, keep_acc=False, e4m3_weights=args.e4m3_weights == "on")
+        st = LayerStep(wl, device=dev, keep_acc=False, e4m3_weights=args.e4m3_weights == "on",
+                       e4m3_x=args.e4m3_x == "on")
         del wl
         torch.cuda.synchronize()  # the inputs are drawn on the default stream; the step runs on `stream`
         with torch.cuda.stream(stream):
@@ -811,6 +812,8 @@ def gemm_sweep(args):
                 "gemms": gemm_rooflines(st, stage_ms, bf16_peak, peak_src),
                 "stage_ms": {k: round(v, 5) for k, v in stage_ms.items()},
                 "config": {"l2": "flushed before every timed replay (256 MiB write)",
+                           "x_operand": ("e4m3 copies of sign(X) by TMA" if st.e4m3_x
+                                         else "packed sign(X) expanded in the products"),
                            "timing": "one CUDA graph of the three-branch step, CUDA events, mean",
                            "steps": args.steps, "warmup": args.warmup, "data": "synthetic (device draw)"}}
         if max(M, K, D) <= SWEEP_ORACLE_MAX and not args.no_cpu_baseline:
