@@ -420,6 +420,13 @@ fqt1_status fqt1_col2im_colmajor(const void* acc, int32_t acc_bits, int64_t ld_a
                                  int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,
                                  int32_t pad, float* dx, void* stream);
 
+/* fqt1_col2im_colmajor with dx channels-last: dx[n, h, w, c] (memory order N, H, W, C),
+ * the same values.  Each CTA reads its taps along 32 positions and writes 128-byte runs
+ * of channels through shared memory. */
+fqt1_status fqt1_col2im_colmajor_nhwc(const void* acc, int32_t acc_bits, int64_t ld_acc, const fqt1_qgrad* psq,
+                                      const int32_t* colsum_w, int32_t N, int32_t C, int32_t H, int32_t W,
+                                      int32_t kh, int32_t kw, int32_t stride, int32_t pad, float* dx, void* stream);
+
 /* grad_input of a convolution with the Folder fused into the product (Eq. 21 with
  * Sec. 5.3's per-sample scales, App. C Folder): the same dx as fqt1_bwd_input_gemm
  * followed by fqt1_col2im, without the int32 accumulators in memory.  A tile of 128

@@ -144,24 +144,14 @@ class _BinaryProduct(torch.autograd.Function):
                 dx = torch.empty((N, H, W, C) if nhwc else (N, C, H, W), dtype=torch.float32, device=dev)
                 if fqt1.fold_supported(Ho, Wo, kh, kw, H, W):
                     fqt1.bwd_input_fold(psq, sw_col, cs_w, N, C, H, W, kh, kw, stride, pad, D, p_s, dx, nhwc=nhwc)
-                elif not nhwc:
-                    # column-major int32 accumulators: the Folder reads every tap as contiguous runs
+                else:
+                    # column-major accumulators (int16 where every sum fits): the Folder reads
+                    # every tap as contiguous runs of a column; dx in the input's memory order
                     ld = (max(cap_s * rpg, 1) + 31) // 32 * 32
                     acc_t = torch.int16 if fqt1.colmajor_acc_bits(q.bits_s, D) == 16 else torch.int32
                     acc_cm = torch.empty(K, ld, dtype=acc_t, device=dev)
                     fqt1.bwd_input_gemm_colmajor(psq, sw_col, M, D, K, p_s, acc_cm)
-                    fqt1.col2im_colmajor(acc_cm, psq, cs_w, N, C, H, W, kh, kw, stride, pad, dx)
-                else:
-                    acc_dx = torch.empty(max(cap_s * rpg, 1), K, dtype=torch.int32, device=dev)
-                    fqt1.bwd_input_gemm(psq, sw_col, cs_w, M, D, K, p_s, acc_dx, None)
-                    try:
-                        fqt1.col2im(acc_dx, psq, cs_w, N, C, H, W, kh, kw, stride, pad, dx, nhwc=nhwc)
-                    except fqt1.Fqt1Error as e:  # untiled Folder shapes write NCHW only
-                        if not nhwc or "UNSUPPORTED" not in str(e):
-                            raise
-                        nhwc = False
-                        dx = torch.empty(N, C, H, W, dtype=torch.float32, device=dev)
-                        fqt1.col2im(acc_dx, psq, cs_w, N, C, H, W, kh, kw, stride, pad, dx)
+                    fqt1.col2im_colmajor(acc_cm, psq, cs_w, N, C, H, W, kh, kw, stride, pad, dx, nhwc=nhwc)
                 if nhwc:
                     dx = dx.permute(0, 3, 1, 2)
             if q.ste_clip is not None:  # x and dx elementwise in the same memory order

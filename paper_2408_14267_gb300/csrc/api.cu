@@ -598,6 +598,134 @@ __global__ void __launch_bounds__(256, 4) col2im_colmajor_kernel(FoldCmArgs a) {
   }  // kept slots
 }
 
+// The same Folder with dx channels-last (dx[n, h, w, c]): a CTA owns 32 consecutive positions
+// p = h W + w of a kept sample's plane and 32 channels.  Lane l of warp w holds position l and
+// channels 4 w .. 4 w + 3, so each position's tap candidates and their validity are worked out
+// once, and each tap's loads run along the 32 positions of a column (coalesced); the 32 x 32
+// block of results then turns through shared memory into 128-byte channel runs.
+template <int KH, int KW, int S, class T>
+__global__ void __launch_bounds__(256, 2) col2im_colmajor_nhwc_kernel(FoldCmArgs a) {
+  constexpr int SS = S > 0 ? S : 1;
+  constexpr int CI = KH ? (KH + SS - 1) / SS : 1, CJ = KW ? (KW + SS - 1) / SS : 1;
+  constexpr int NCAND = CI * CJ;
+  constexpr int CPW = 4;   // channels per warp
+  constexpr int CB = 2;    // channels whose loads are in flight together
+  extern __shared__ int32_t fold_cs[];  // [K] column sums when a.cs_smem
+  __shared__ float blk[32][33];         // [channel in block][position in block]
+  FQT1_PDL_WAIT();
+  FQT1_PDL_TRIGGER();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int kh = KH ? KH : a.kh, kw = KW ? KW : a.kw, st = S ? S : a.stride;
+  const int khw = kh * kw, HW = a.H * a.W, C = (int)(a.plane / HW);
+  const int32_t* csb = a.cs;
+  if (a.cs_smem) {
+    for (int k = threadIdx.x; k < a.K; k += blockDim.x) fold_cs[k] = __ldg(a.cs + k);
+    __syncthreads();
+    csb = fold_cs;
+  }
+  const int npb = (HW + 31) / 32;
+  const int pb = (int)(blockIdx.x % npb), cblk = (int)(blockIdx.x / npb);
+  const int pos = min(pb * 32 + lane, HW - 1);  // clamped: every address below is valid
+  const int h = (int)a.div_w.div((uint32_t)pos), w = pos - h * a.W;
+  // this position's tap candidates (compile-time window: by residue, as the NCHW kernel)
+  int toff[NCAND], tix[NCAND];
+  uint32_t ok = 0;
+  if (KH) {
+    const int hp = h + a.pad, wp = w + a.pad;
+    const int rh = SS == 1 ? 0 : hp % SS, qh = SS == 1 ? hp : hp / SS;
+    const int rw = SS == 1 ? 0 : wp % SS, qw = SS == 1 ? wp : wp / SS;
+#pragma unroll
+    for (int mi = 0; mi < CI; ++mi) {
+      const int i = rh + SS * mi, oh = qh - mi;
+      const bool vi = i < KH && oh >= 0 && oh < a.Ho;
+#pragma unroll
+      for (int mj = 0; mj < CJ; ++mj) {
+        const int j = rw + SS * mj, ow = qw - mj;
+        const bool v = vi && j < KW && ow >= 0 && ow < a.Wo;
+        ok |= v ? 1u << (mi * CJ + mj) : 0u;
+        toff[mi * CJ + mj] = v ? oh * a.Wo + ow : 0;
+        tix[mi * CJ + mj] = v ? i * KW + j : 0;
+      }
+    }
+  }
+  const int c_base = cblk * 32 + warp * CPW;
+  const int kept = __ldg(a.kept_count);
+  for (int slot = (int)blockIdx.y; slot < kept; slot += (int)gridDim.y) {
+    const int n = __ldg(a.kept_idx + slot);
+    const T* accs = static_cast<const T*>(a.acc) + (int64_t)slot * a.Ho * a.Wo;
+    const float sc = __ldg(a.scale + slot), ze = __ldg(a.zero + slot);
+#pragma unroll
+    for (int u0 = 0; u0 < CPW; u0 += CB) {
+      int32_t av[CB], cv[CB];
+      if (KH) {
+        int32_t va[CB][NCAND];
+#pragma unroll
+        for (int u = 0; u < CB; ++u) {
+          const int c = min(c_base + u0 + u, C - 1);
+          const T* col = accs + (int64_t)c * khw * a.ld;
+#pragma unroll
+          for (int x = 0; x < NCAND; ++x) va[u][x] = (int32_t)__ldg(col + (int64_t)tix[x] * a.ld + toff[x]);
+        }
+#pragma unroll
+        for (int u = 0; u < CB; ++u) {
+          const int c = min(c_base + u0 + u, C - 1);
+          int32_t sa = 0, sc_ = 0;
+#pragma unroll
+          for (int x = 0; x < NCAND; ++x) {
+            const bool v = (ok >> x) & 1u;
+            sa += v ? va[u][x] : 0;
+            sc_ += v ? csb[c * khw + tix[x]] : 0;
+          }
+          av[u] = sa;
+          cv[u] = sc_;
+        }
+      } else {
+        // runtime window: every tap tested in turn
+#pragma unroll
+        for (int u = 0; u < CB; ++u) {
+          av[u] = 0;
+          cv[u] = 0;
+          const int c = min(c_base + u0 + u, C - 1);
+          const T* col = accs + (int64_t)c * khw * a.ld;
+#pragma unroll 1
+          for (int i = 0; i < kh; ++i) {
+            const int hn = h + a.pad - i;
+            if (hn < 0) break;
+            if (hn % st) continue;
+            const int oh = hn / st;
+            if (oh >= a.Ho) continue;
+#pragma unroll 1
+            for (int j = 0; j < kw; ++j) {
+              const int wn = w + a.pad - j;
+              if (wn < 0) break;
+              if (wn % st) continue;
+              const int ow = wn / st;
+              if (ow >= a.Wo) continue;
+              const int t = i * kw + j;
+              av[u] += (int32_t)__ldg(col + (int64_t)t * a.ld + oh * a.Wo + ow);
+              cv[u] += csb[c * khw + t];
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < CB; ++u)
+        blk[warp * CPW + u0 + u][lane] =
+            __fadd_rn(__fmul_rn(sc, __int2float_rn(av[u])), __fmul_rn(ze, __int2float_rn(cv[u])));
+    }
+    __syncthreads();
+    // positions 4 w .. 4 w + 3 of the block, lane = channel: 128-byte runs of dx[n, p, :]
+    float* out = a.dx + (int64_t)n * a.plane;
+    const int c = cblk * 32 + lane;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int p = pb * 32 + warp * 4 + q;
+      if (p < HW && c < C) out[(int64_t)p * C + c] = blk[lane][warp * 4 + q];
+    }
+    __syncthreads();
+  }
+}
+
 }  // namespace fqt1
 
 using namespace fqt1;
@@ -871,10 +999,10 @@ extern "C" fqt1_status fqt1_bwd_input_gemm_colmajor_e4m3w(const fqt1_qgrad* psq,
   return bwd_input_colmajor_impl(psq, nullptr, wt_e4m3, ld_wt, M, D, K, p, acc, acc_bits, ld_acc, stream);
 }
 
-extern "C" fqt1_status fqt1_col2im_colmajor(const void* acc, int32_t acc_bits, int64_t ld_acc, const fqt1_qgrad* psq,
-                                            const int32_t* colsum_w, int32_t N, int32_t C, int32_t H, int32_t W,
-                                            int32_t kh, int32_t kw, int32_t stride, int32_t pad, float* dx,
-                                            void* stream) {
+static fqt1_status col2im_colmajor_impl(const void* acc, int32_t acc_bits, int64_t ld_acc, const fqt1_qgrad* psq,
+                                       const int32_t* colsum_w, int32_t N, int32_t C, int32_t H, int32_t W,
+                                       int32_t kh, int32_t kw, int32_t stride, int32_t pad, float* dx, bool nhwc,
+                                       void* stream) {
   if (!acc || !psq || !colsum_w || !dx || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 ||
       pad < 0 || kh > 64 || kw > 64)
     return FQT1_ERR_INVALID_ARG;
@@ -906,6 +1034,32 @@ extern "C" fqt1_status fqt1_col2im_colmajor(const void* acc, int32_t acc_bits, i
     const int64_t gy = std::max<int64_t>(1, std::min<int64_t>(N, (16 * (int64_t)sm_count_api() + gx - 1) / gx));
     return dim3((unsigned)gx, (unsigned)gy);
   };
+  if (nhwc) {  // 32 positions x 32 channels per CTA, the same grid rows over kept slots
+    const int64_t gx = ((int64_t)H * W + 31) / 32 * ((C + 31) / 32);
+    if (gx > 0x7FFFFFFF) return FQT1_ERR_UNSUPPORTED;
+    const dim3 g((unsigned)gx,
+                 (unsigned)std::max<int64_t>(1, std::min<int64_t>(N, (16 * (int64_t)sm_count_api() + gx - 1) / gx)));
+    auto launch_nhwc = [&](auto zero) {
+      using T = decltype(zero);
+      if (kh == 3 && kw == 3 && stride == 1)
+        launch_k(col2im_colmajor_nhwc_kernel<3, 3, 1, T>, g, dim3(256), cs_bytes, s, fa);
+      else if (kh == 3 && kw == 3 && stride == 2)
+        launch_k(col2im_colmajor_nhwc_kernel<3, 3, 2, T>, g, dim3(256), cs_bytes, s, fa);
+      else if (kh == 1 && kw == 1 && stride == 1)
+        launch_k(col2im_colmajor_nhwc_kernel<1, 1, 1, T>, g, dim3(256), cs_bytes, s, fa);
+      else if (kh == 1 && kw == 1 && stride == 2)
+        launch_k(col2im_colmajor_nhwc_kernel<1, 1, 2, T>, g, dim3(256), cs_bytes, s, fa);
+      else
+        launch_k(col2im_colmajor_nhwc_kernel<0, 0, 0, T>, g, dim3(256), cs_bytes, s, fa);
+    };
+    if (acc_bits == 16)
+      launch_nhwc(int16_t{0});
+    else
+      launch_nhwc(int32_t{0});
+    fqt1_count_launches(1);
+    FQT1_CUDA_TRY(cudaGetLastError());
+    return FQT1_OK;
+  }
   auto launch = [&](auto zero) {  // zero: a value of the accumulator type
     using T = decltype(zero);
     if (kh == 3 && kw == 3 && stride == 1)
@@ -928,6 +1082,22 @@ extern "C" fqt1_status fqt1_col2im_colmajor(const void* acc, int32_t acc_bits, i
   fqt1_count_launches(1);
   FQT1_CUDA_TRY(cudaGetLastError());
   return FQT1_OK;
+}
+
+extern "C" fqt1_status fqt1_col2im_colmajor(const void* acc, int32_t acc_bits, int64_t ld_acc, const fqt1_qgrad* psq,
+                                            const int32_t* colsum_w, int32_t N, int32_t C, int32_t H, int32_t W,
+                                            int32_t kh, int32_t kw, int32_t stride, int32_t pad, float* dx,
+                                            void* stream) {
+  return col2im_colmajor_impl(acc, acc_bits, ld_acc, psq, colsum_w, N, C, H, W, kh, kw, stride, pad, dx, false,
+                              stream);
+}
+
+extern "C" fqt1_status fqt1_col2im_colmajor_nhwc(const void* acc, int32_t acc_bits, int64_t ld_acc,
+                                                 const fqt1_qgrad* psq, const int32_t* colsum_w, int32_t N,
+                                                 int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw,
+                                                 int32_t stride, int32_t pad, float* dx, void* stream) {
+  return col2im_colmajor_impl(acc, acc_bits, ld_acc, psq, colsum_w, N, C, H, W, kh, kw, stride, pad, dx, true,
+                              stream);
 }
 
 extern "C" fqt1_status fqt1_col2im_nhwc(const int32_t* acc, const fqt1_qgrad* psq, const int32_t* colsum_w, int32_t N,

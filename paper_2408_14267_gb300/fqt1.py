@@ -73,6 +73,7 @@ _SIGS = {
     "fqt1_col2im": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
     "fqt1_bwd_input_gemm_colmajor": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _I32, _I64, _VP]),
     "fqt1_col2im_colmajor": (C.c_int, [_VP, _I32, _I64, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
+    "fqt1_col2im_colmajor_nhwc": (C.c_int, [_VP, _I32, _I64, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
     "fqt1_bwd_input_gemm_colmajor_e4m3w": (C.c_int, [_VP, _VP, _I64, _I64, _I64, _I64, _VP, _VP, _I32, _I64,
                                                      _VP]),
     "fqt1_col2im_nhwc": (C.c_int, [_VP, _VP, _VP] + [_I32] * 8 + [_VP, _VP]),
@@ -326,9 +327,10 @@ def bwd_input_gemm_colmajor_e4m3w(psq, wt8, M, D, K, params, acc, stream=None):
            "fqt1_bwd_input_gemm_colmajor_e4m3w")
 
 
-def col2im_colmajor(acc, psq, colsum_w, N, Cin, H, W, kh, kw, stride, pad, dx, stream=None):
-    _check(lib().fqt1_col2im_colmajor(_p(acc), _acc_bits(acc), acc.shape[1], C.byref(psq.c), _p(colsum_w), N, Cin, H,
-                                      W, kh, kw, stride, pad, _p(dx), _s(stream)), "fqt1_col2im_colmajor")
+def col2im_colmajor(acc, psq, colsum_w, N, Cin, H, W, kh, kw, stride, pad, dx, stream=None, nhwc=False):
+    fn = lib().fqt1_col2im_colmajor_nhwc if nhwc else lib().fqt1_col2im_colmajor
+    _check(fn(_p(acc), _acc_bits(acc), acc.shape[1], C.byref(psq.c), _p(colsum_w), N, Cin, H, W, kh, kw, stride, pad,
+              _p(dx), _s(stream)), "fqt1_col2im_colmajor_nhwc" if nhwc else "fqt1_col2im_colmajor")
 
 
 def colmajor_acc_bits(bits, D):

@@ -149,3 +149,21 @@ def test_colmajor_int16_bound():
     assert fqt1.colmajor_acc_bits(4, 2184) == 16 and fqt1.colmajor_acc_bits(4, 2185) == 32
     assert fqt1.colmajor_acc_bits(8, 128) == 16 and fqt1.colmajor_acc_bits(8, 129) == 32
     assert fqt1.colmajor_acc_bits(1, 32767) == 16 and fqt1.colmajor_acc_bits(1, 32768) == 32
+
+
+@pytest.mark.parametrize("name,make", [COLMAJOR_CASES[i] for i in (0, 2, 4, 6, 8, 9)],
+                         ids=[COLMAJOR_CASES[i][0] for i in (0, 2, 4, 6, 8, 9)])
+def test_colmajor_channels_last_output(name, make):
+    """fqt1_col2im_colmajor_nhwc writes the NCHW Folder's values in N, H, W, C order (pruned
+    samples included), from int16 and from int32 accumulators."""
+    from paper_2408_14267_gb300 import fqt1
+    from paper_2408_14267_gb300.layer import LayerStep
+    w = make()
+    for acc16 in (True, False):
+        st = LayerStep(w, keep_acc=False, fold=False, colmajor=True, acc16=acc16)
+        st.step()
+        N, C, H, W, kh, kw = st.conv
+        dx = torch.full((N, H, W, C), 3.0, device="cuda")
+        fqt1.col2im_colmajor(st.acc_dx_cm, st.psq, st.cs_w, N, C, H, W, kh, kw, st.stride, st.pad, dx, nhwc=True)
+        torch.cuda.synchronize()
+        assert torch.equal(dx.permute(0, 3, 1, 2), st.dx)
