@@ -441,8 +441,9 @@ __global__ void __launch_bounds__(256) col2im_tiled_kernel(FoldArgs a) {
   }
 }
 
-// Folder on column-major int32 accumulators (the layout fqt1_bwd_input_gemm_colmajor writes):
-// acc[k * ld + r] for kept row r = slot Ho Wo + oh Wo + ow and column k = c kh kw + i kw + j.
+// Folder on column-major accumulators (the layout fqt1_bwd_input_gemm_colmajor writes; T int32,
+// or int16 where every sum fits): acc[k * ld + r] for kept row r = slot Ho Wo + oh Wo + ow and
+// column k = c kh kw + i kw + j; the tap sums are taken in int32.
 // A thread owns elements e = c H W + h W + w of one kept sample's dx plane; tap (i, j) of input
 // pixel (h, w) is the accumulator of output pixel oh = (h + pad - i) / stride,
 // ow = (w + pad - j) / stride when both divisions are exact and land in the output map.  The 32
