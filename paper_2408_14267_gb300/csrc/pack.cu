@@ -320,6 +320,28 @@ __device__ __forceinline__ uint32_t stream_bits(const uint32_t* st, int pos, int
   return cnt >= 32 ? bits : bits & ((1u << cnt) - 1u);
 }
 
+// The even bits of 32 bits, packed into the low 16 (bit 2 t -> bit t).
+__device__ __forceinline__ uint32_t even_bits16(uint32_t x) {
+  x &= 0x55555555u;
+  x = (x | (x >> 1)) & 0x33333333u;
+  x = (x | (x >> 2)) & 0x0F0F0F0Fu;
+  x = (x | (x >> 4)) & 0x00FF00FFu;
+  x = (x | (x >> 8)) & 0x0000FFFFu;
+  return x;
+}
+
+// cnt (1..32) bits of a stream at bit positions pos, pos + 2, ..., pos + 2 (cnt - 1): only the
+// words holding those bits are read (at most three), so the read stays inside the bits it needs.
+__device__ __forceinline__ uint32_t stream_even_bits(const uint32_t* st, int pos, int cnt) {
+  const int w = pos >> 5, o = pos & 31, last = (pos + 2 * cnt - 2) >> 5;
+  const uint32_t x0 = st[w];
+  const uint32_t x1 = last > w ? st[w + 1] : 0u;
+  const uint32_t x2 = last > w + 1 ? st[w + 2] : 0u;
+  const uint32_t lo = __funnelshift_r(x0, x1, o), hi = __funnelshift_r(x1, x2, o);
+  const uint32_t bits = even_bits16(lo) | (even_bits16(hi) << 16);
+  return cnt >= 32 ? bits : bits & ((1u << cnt) - 1u);
+}
+
 __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
   FQT1_PDL_WAIT();
   FQT1_PDL_TRIGGER();
@@ -472,6 +494,35 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
           if (kvalid && h >= 0 && h < a.H && hi > lo) {
             const uint32_t* st = st_c + (n - n_lo) * nc * plane_words;
             colw |= stream_bits(st, gbits + (h - h_lo) * a.W + wa + lo, hi - lo) << (m - ms + lo);
+          }
+          m += cnt;
+          ow += cnt;
+          if (ow == a.Wo) {
+            ow = 0;
+            if (++oh == Ho) { oh = 0; ++n; }
+          }
+        }
+        roww = warp_transpose32(colw, lane);
+      } else if (a.stride == 2) {
+        // stride 2: the column word of k = kb + lane over pixels ms .. ms + 31, by runs along
+        // output rows as for stride 1; a run of pixels ow .. ow + cnt - 1 reads every other bit
+        // of its input row from input column 2 ow - pad + j, so its bits are the even bits of a
+        // stream window of at most 63 bits (stream_even_bits)
+        const int mend = min(a.M, ms + 32);
+        int n = (int)a.div_hwo.div((uint32_t)ms), rem = ms - n * a.HWo;
+        int oh = (int)a.div_wo.div((uint32_t)rem), ow = rem - oh * a.Wo;
+        const uint32_t* st_c = stream + (cl_ - c_lo) * plane_words;
+        const bool kvalid = kb + lane < a.K;
+        for (int m = ms; m < mend;) {
+          const int cnt = min(a.Wo - ow, mend - m);  // pixels left on this output row
+          const int h = 2 * oh - a.pad + il_;
+          const int wa = 2 * ow - a.pad + jl_;  // input column of the run's first pixel
+          // pixels t of the run whose input column wa + 2 t lies in [0, W)
+          const int lo = wa >= 0 ? 0 : (1 - wa) / 2;
+          const int hi = wa <= a.W - 1 ? min(cnt, (a.W - 1 - wa) / 2 + 1) : 0;
+          if (kvalid && h >= 0 && h < a.H && hi > lo) {
+            const uint32_t* st = st_c + (n - n_lo) * nc * plane_words;
+            colw |= stream_even_bits(st, gbits + (h - h_lo) * a.W + wa + 2 * lo, hi - lo) << (m - ms + lo);
           }
           m += cnt;
           ow += cnt;
