@@ -58,6 +58,8 @@ COLMAJOR_CASES = [
     ("5x5-s3-p2-runtime-window", lambda: conv_case(3, 6, 17, 13, 8, 5, 3, 2, 4, SYS, seed=39)),
     ("2x4-window-s1-p0", lambda: _rect_case(3, 7, 11, 10, 12, 2, 4, 1, 0, 4, SYS, seed=40)),
     ("single-sample-b1", lambda: conv_case(1, 9, 12, 12, 10, 3, 1, 1, 1, SYS, seed=41)),
+    # 255 x 200 > 32767: the accumulators stay int32 (chosen by LayerStep, checked below)
+    ("b8-wide-D-int32", lambda: conv_case(3, 10, 12, 12, 200, 3, 1, 1, 8, SYS, seed=42)),
 ]
 
 
@@ -69,6 +71,8 @@ def test_colmajor_grad_input_matches_oracle_and_row_major_folder(name, make):
     cm = LayerStep(w, keep_acc=False, fold=False, colmajor=True)
     rm = LayerStep(w, keep_acc=True, fold=False, colmajor=False)
     assert cm.colmajor and not rm.colmajor
+    # int16 exactly where every sum fits: (2^b - 1) D <= 32767
+    assert cm.acc_bits_cm == (16 if ((1 << w["bits_s"]) - 1) * cm.D <= 32767 else 32)
     cm.dx.fill_(7.0)  # pruned samples must be overwritten with zeros
     cm.step()
     rm.step()
