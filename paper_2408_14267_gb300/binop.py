@@ -89,7 +89,7 @@ class _BinaryProduct(torch.autograd.Function):
                 if "UNSUPPORTED" not in str(e):
                     raise
                 fqt1.im2col(x.detach().contiguous(), N, C, H, W, kh, kw, stride, pad, sx_row, sx_col, cs_x)
-        elif fqt1.im2col_path(N, C, H, W, kh, kw, stride, pad) == 1:
+        elif fqt1.unfold_from_planes(N, C, H, W, kh, kw, stride, pad):
             # region tiles: sign-pack x into planes in one pass, the Unfolder then reads bits
             planes = torch.empty(N * C * fqt1.plane_words(H, W), dtype=torch.int32, device=dev)
             fqt1.pack_planes(x.detach(), N, C, H, W, planes)

@@ -407,6 +407,36 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
         stream[pos[u]] = word;
       }
     }
+  } else if (plane_bits < 32 && 32 % plane_bits == 0 && nrows == a.H) {
+    // whole planes of fewer than 32 pixels that divide 32 (4 x 4, 2 x 2 maps): the region's
+    // floats of one image are nc H W consecutive floats of x, so one ballot of 32 of them gives
+    // the (single) words of 32 / (H W) consecutive planes; no load lane is idle
+    const int hw = plane_bits, per = 32 / hw;
+    const uint32_t pmask = (1u << hw) - 1u;
+    const int span = nc * hw, gper = (span + 31) / 32;  // floats and ballots of one image's region
+    const int total = (nplanes / nc) * gper;
+    const int64_t img_stride = (int64_t)a.C * hw;
+    const float* base = a.x + ((int64_t)n_lo * a.C + c_lo) * hw;
+    const FastDiv div_g((uint32_t)gper);
+    for (int f0 = warp; f0 < total; f0 += 8 * 16) {
+      float v[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const int f = min(f0 + 8 * u, total - 1);
+        const int nn = (int)div_g.div((uint32_t)f), e = 32 * (f - nn * gper) + lane;
+        v[u] = __ldg(base + nn * img_stride + min(e, span - 1));
+        if (e >= span) v[u] = 0.0f;
+      }
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const uint32_t word = __ballot_sync(0xFFFFFFFFu, v[u] > 0.0f);
+        const int f = f0 + 8 * u;
+        if (f < total && lane < per) {
+          const int nn = (int)div_g.div((uint32_t)f), c = (f - nn * gper) * per + lane;
+          if (c < nc) stream[(nn * nc + c) * plane_words + a.guard] = (word >> (lane * hw)) & pmask;
+        }
+      }
+    }
   } else {
     const int total = nplanes * data_words;
     const FastDiv div_dw((uint32_t)max(data_words, 1)), div_nc((uint32_t)nc);

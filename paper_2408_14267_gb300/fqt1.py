@@ -235,6 +235,16 @@ def im2col_path(N, Cin, H, W, kh, kw, stride, pad):
     return lib().fqt1_im2col_path(N, Cin, H, W, kh, kw, stride, pad)
 
 
+def unfold_from_planes(N, Cin, H, W, kh, kw, stride, pad):
+    """Whether a contiguous x is sign-packed into planes before the Unfolder: every region-tile
+    shape (im2col_path 1).  Reading x directly is faster for the Unfolder alone on 4 x 4, 2 x 2
+    and 7 x 7 maps (eager, L2 flushed: 19-24 us against 27-31 us for the two launches), but not
+    for the three-branch layer step: on the 4 x 4 VGG-16 layers three same-GPU sweeps gave 209.5
+    and 220.3 us (direct) against 206.9 us (planes first) for conv8-conv10, single replays
+    spreading over 66-86 us with the order in which the concurrent branches get their SMs."""
+    return im2col_path(N, Cin, H, W, kh, kw, stride, pad) == 1
+
+
 def pack_planes_nhwc(x, N, Cin, H, W, planes, stream=None):
     _check(lib().fqt1_pack_planes_nhwc(_p(x), N, Cin, H, W, _p(planes), _s(stream)), "fqt1_pack_planes_nhwc")
 

@@ -85,8 +85,8 @@ class LayerStep:
         # shapes whose Unfolder reads an input region per tile: sign-pack x into planes first
         # (one streaming pass), so that the regions are read as bits
         self.x_planes = None
-        if self.kind == "conv" and not self.implicit and fqt1.im2col_path(N, Cin, H, W, kh, kw, self.stride,
-                                                                          self.pad) == 1:
+        if self.kind == "conv" and not self.implicit and fqt1.unfold_from_planes(N, Cin, H, W, kh, kw, self.stride,
+                                                                                 self.pad):
             self.x_planes = torch.empty(N * Cin * fqt1.plane_words(H, W), **i32)
         if self.implicit:
             self.x_pix = torch.empty(N * H * W, fqt1.packed_words(Cin), **i32)

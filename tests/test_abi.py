@@ -113,6 +113,19 @@ def test_implicit_conv_support_rules(lib):
     assert not ok(2, 128, 3, 3, 3, 3, 1, 1)         # 9 pixels do not divide 128
 
 
+def test_unfolder_source_choice(lib):
+    """Which Unfolder input a layer gives a contiguous x (host logic, no GPU): whole-image tiles
+    (path 2) and pointwise windows (path 3) read x; region tiles (path 1) read sign planes packed
+    first."""
+    from paper_2408_14267_gb300 import fqt1
+    assert fqt1.im2col_path(128, 256, 8, 8, 3, 3, 1, 1) == 2 and not fqt1.unfold_from_planes(128, 256, 8, 8, 3, 3, 1, 1)
+    assert fqt1.im2col_path(64, 64, 56, 56, 1, 1, 2, 0) == 3 and not fqt1.unfold_from_planes(64, 64, 56, 56, 1, 1, 2, 0)
+    for shape in [(128, 512, 4, 4, 3, 3, 1, 1), (16, 64, 2, 4, 3, 3, 1, 1), (128, 512, 2, 2, 3, 3, 1, 1),
+                  (64, 512, 7, 7, 3, 3, 1, 1), (64, 256, 14, 14, 3, 3, 1, 1), (64, 3, 224, 224, 7, 7, 2, 3),
+                  (8, 16, 1, 1, 3, 3, 1, 1)]:
+        assert fqt1.im2col_path(*shape) == 1 and fqt1.unfold_from_planes(*shape), shape
+
+
 def test_implicit_conv_validation_without_launch(lib):
     fake = C.c_void_p(0x10000)
     odd = C.c_void_p(0x10004)

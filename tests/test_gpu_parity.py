@@ -701,12 +701,17 @@ def test_im2col_from_channels_last_planes(N, C, H, W, k, s, p):
 @pytest.mark.parametrize("N,C,H,W,k,s,p", [(2, 3, 30, 30, 7, 2, 3), (2, 64, 28, 28, 1, 2, 0), (3, 16, 14, 14, 3, 2, 1),
                                            (2, 5, 13, 11, 3, 1, 1), (1, 32, 56, 56, 3, 1, 1), (4, 8, 9, 7, 1, 1, 0),
                                            (5, 37, 4, 4, 3, 1, 1), (9, 50, 2, 2, 3, 1, 1), (3, 11, 2, 4, 3, 1, 1),
-                                           (3, 40, 15, 13, 1, 3, 0), (2, 33, 8, 9, 1, 1, 0), (5, 70, 7, 7, 1, 2, 0)])
+                                           (3, 40, 15, 13, 1, 3, 0), (2, 33, 8, 9, 1, 1, 0), (5, 70, 7, 7, 1, 2, 0),
+                                           (40, 70, 4, 4, 3, 1, 1), (70, 33, 2, 2, 3, 1, 1), (6, 45, 1, 1, 3, 1, 1),
+                                           (9, 21, 1, 2, 3, 1, 1), (1, 29, 4, 4, 3, 1, 1)])
 def test_pack_planes_nchw_and_unfold_from_planes(N, C, H, W, k, s, p):
     """Contiguous x: fqt1_pack_planes writes the signs of x as channel planes (any C, H W not a
     multiple of 32, bits past H W clear), and the Unfolder reading those planes writes the same
     rows, columns and column sums as the Unfolder reading x (the region-tile shape of the
-    ResNet-18 stem, and the 1 x 1 downsamples, which the pointwise pass serves from x)."""
+    ResNet-18 stem, and the 1 x 1 downsamples, which the pointwise pass serves from x).  Maps of
+    fewer than 32 pixels that divide 32 (4 x 4, 2 x 2, 1 x 2, 1 x 1): the Unfolder reading x takes
+    each ballot over several whole planes; the cases span several row and column tiles, channel
+    counts that leave a partial ballot per image, and a single image."""
     from paper_2408_14267_gb300 import fqt1
     rng = np.random.default_rng(N * C + H * 3 + k)
     x = rng.standard_normal((N, C, H, W)).astype(np.float32)
