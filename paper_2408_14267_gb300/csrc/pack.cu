@@ -407,7 +407,7 @@ __global__ void __launch_bounds__(256) unfold_bits_kernel(UnfoldArgs a) {
         stream[pos[u]] = word;
       }
     }
-  } else if (plane_bits < 32 && 32 % plane_bits == 0 && nrows == a.H) {
+  } else if (nrows == a.H && plane_bits < 32 && 32 % plane_bits == 0) {  // plane_bits = H W >= 1 here
     // whole planes of fewer than 32 pixels that divide 32 (4 x 4, 2 x 2 maps): the region's
     // floats of one image are nc H W consecutive floats of x, so one ballot of 32 of them gives
     // the (single) words of 32 / (H W) consecutive planes; no load lane is idle
