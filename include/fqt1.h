@@ -413,8 +413,8 @@ fqt1_status fqt1_bwd_input_gemm_colmajor_e4m3w(const fqt1_qgrad* psq, const uint
  * tap of a warp's 32 consecutive outputs as one contiguous run of a column.
  * acc: [C kh kw][ld_acc] from fqt1_bwd_input_gemm_colmajor with the same acc_bits
  * (the row of output pixel (oh, ow) of kept slot s is s Ho Wo + oh Wo + ow); dx:
- * [N, C, H, W], pruned samples 0.  N <= 65535 and C H W < 2^31, else
- * FQT1_ERR_UNSUPPORTED. */
+ * [N, C, H, W], pruned samples 0.  N <= 65535, C H W < 2^31 and C kh kw < 2^31,
+ * else FQT1_ERR_UNSUPPORTED. */
 fqt1_status fqt1_col2im_colmajor(const void* acc, int32_t acc_bits, int64_t ld_acc, const fqt1_qgrad* psq,
                                  const int32_t* colsum_w,
                                  int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,

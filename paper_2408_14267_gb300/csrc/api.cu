@@ -1022,7 +1022,8 @@ static fqt1_status col2im_colmajor_impl(const void* acc, int32_t acc_bits, int64
   fa.H = H; fa.W = W; fa.kh = kh; fa.kw = kw; fa.stride = stride; fa.pad = pad; fa.Ho = Ho; fa.Wo = Wo;
   fa.plane = plane; fa.div_hw = FastDiv((uint32_t)(H * W)); fa.div_w = FastDiv((uint32_t)W);
   const int64_t K = (int64_t)C * kh * kw;
-  fa.K = (int)std::min<int64_t>(K, 0x7FFFFFFF);
+  if (K >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;  // column indices are 32-bit in the kernels
+  fa.K = (int)K;
   fa.cs_smem = K <= 12288;
   const size_t cs_bytes = fa.cs_smem ? (size_t)K * 4 : 0;
   cudaStream_t s = (cudaStream_t)stream;

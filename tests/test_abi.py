@@ -93,6 +93,8 @@ def test_argument_validation_without_launch(lib):
     assert lib.fqt1_col2im_colmajor(fake, 24, 16, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake, s) == 1
     assert lib.fqt1_col2im_colmajor(C.c_void_p(0x10004), 32, 16, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 1, 1, fake,
                                     s) == 2
+    # C kh kw = 2^19 x 64 x 64 = 2^31 columns (C H W = 2^29): refused before any launch
+    assert lib.fqt1_col2im_colmajor(fake, 32, 4, C.byref(q), fake, 1, 1 << 19, 32, 32, 64, 64, 1, 16, fake, s) == 3
 
 
 def test_implicit_conv_support_rules(lib):
