@@ -82,8 +82,14 @@ def test_argument_validation_without_launch(lib):
     assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(bad_bits), fake, 32, 8, s) == 1
     assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(ok), fake, 8, 8, s) == 1  # width 8
     assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 8, 8, C.byref(ok), fake, 16, 4, s) == 1  # ld % 8
-    big_d = fqt1.AgpParams(4, 0, 1, 1)  # 15 * 4096 > 32767: int16 cannot hold the sums
-    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q), fake, 8, 4096, 8, C.byref(big_d), fake, 16, 8, s) == 1
+    # int16 cannot hold the sums: 15 * 4096 and 15 * 2185 = 32775 > 32767 (the first width past
+    # the bound, the binding's rule agreeing); q_wide's codes rows have room for D = 4096, so the
+    # int16 bound is the only check these calls fail
+    big_d = fqt1.AgpParams(4, 0, 1, 1)
+    q_wide = fqt1.QGrad(*(0x10000 for _ in range(9)), 4096)
+    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q_wide), fake, 8, 4096, 8, C.byref(big_d), fake, 16, 8, s) == 1
+    assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q_wide), fake, 8, 2185, 8, C.byref(big_d), fake, 16, 8, s) == 1
+    assert fqt1.colmajor_acc_bits(4, 2185) == 32 and fqt1.colmajor_acc_bits(4, 2184) == 16
     assert lib.fqt1_bwd_input_gemm_colmajor_e4m3w(C.byref(q), fake, 8, 8, 8, 8, C.byref(ok), fake, 32, 8, s) == 1
     assert lib.fqt1_bwd_input_gemm_colmajor_e4m3w(C.byref(q), None, 16, 8, 8, 8, C.byref(ok), fake, 32, 8, s) == 1
     assert lib.fqt1_col2im_colmajor(fake, 32, 16, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 0, 1, fake, s) == 1
