@@ -71,8 +71,8 @@ def test_argument_validation_without_launch(lib):
     qbig = fqt1.QGrad(*(0x10000 for _ in range(9)), 1 << 16)
     assert lib.fqt1_agp_quantize_grad(fake, 20000, 16, 0, None, C.byref(big), C.byref(qbig), fake, 1 << 20, st,
                                       s) == 3                                          # > 16384 groups
-    assert lib.fqt1_bwd_input_gemm(C.byref(q), fake, fake, 8, 8, 8, C.byref(bad_bits), fake, fake, s) == 1
-    assert lib.fqt1_bwd_weight_gemm(C.byref(q), fake, fake, 8, 8, 8, C.byref(ok), None, fake, None, 0, s) == 1
+    assert lib.fqt1_bwd_input_gemm(C.byref(q), fake, fake, 8, 8, 8, C.byref(bad_bits), fake, fake, s) == 1  # b = 3
+    assert lib.fqt1_bwd_weight_gemm(C.byref(q), fake, fake, 8, 8, 8, C.byref(ok), None, fake, None, 0, s) == 1  # no acc
     assert lib.fqt1_col2im(fake, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 0, 1, fake, s) == 1  # stride 0
     # column-major grad_input: ld below the kept rows (capacity 4 of 8 groups, 1 row each) or
     # not a multiple of 4; the Folder: stride 0, ld below Ho Wo, ld not a multiple of 4, and
@@ -90,6 +90,7 @@ def test_argument_validation_without_launch(lib):
     assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q_wide), fake, 8, 4096, 8, C.byref(big_d), fake, 16, 8, s) == 1
     assert lib.fqt1_bwd_input_gemm_colmajor(C.byref(q_wide), fake, 8, 2185, 8, C.byref(big_d), fake, 16, 8, s) == 1
     assert fqt1.colmajor_acc_bits(4, 2185) == 32 and fqt1.colmajor_acc_bits(4, 2184) == 16
+    # sign(W)^T rows of 8 bytes, below codes_ld(D = 8) = 16; no sign(W)^T at all
     assert lib.fqt1_bwd_input_gemm_colmajor_e4m3w(C.byref(q), fake, 8, 8, 8, 8, C.byref(ok), fake, 32, 8, s) == 1
     assert lib.fqt1_bwd_input_gemm_colmajor_e4m3w(C.byref(q), None, 16, 8, 8, 8, C.byref(ok), fake, 32, 8, s) == 1
     assert lib.fqt1_col2im_colmajor(fake, 32, 16, C.byref(q), fake, 1, 1, 4, 4, 3, 3, 0, 1, fake, s) == 1
