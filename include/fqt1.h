@@ -173,7 +173,8 @@ fqt1_status fqt1_conv_fwd_implicit(const uint32_t* x_pix, const uint32_t* w_taps
  *   32 times fewer bytes.  3: a pointwise convolution (1 x 1 window, no padding):
  *   one pass over x, which fqt1_im2col reads directly (fqt1_im2col_planes serves
  *   it with region tiles).  0: a per-element gather (regions too large; x must be
- *   given).  -1: invalid shape. */
+ *   given).  -1: a shape fqt1_im2col rejects (invalid, or N C H W, N Ho Wo or
+ *   H + 2 pad reaching 2^31). */
 fqt1_status fqt1_pack_planes(const float* x, int32_t N, int32_t C, int32_t H, int32_t W, uint32_t* planes,
                              void* stream);
 int32_t fqt1_im2col_path(int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw, int32_t stride,

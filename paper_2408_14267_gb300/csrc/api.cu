@@ -732,6 +732,15 @@ __global__ void __launch_bounds__(256, 2) col2im_colmajor_nhwc_kernel(FoldCmArgs
 using namespace fqt1;
 
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+// Output extent of a convolution along one axis, (n + 2 pad - k) / stride + 1 for n, k, stride
+// >= 1 and pad >= 0, computed in 64 bits: 0 when the window does not fit, -1 when n + 2 pad
+// does not fit an int (the kernels' index arithmetic is 32-bit).
+static int64_t conv_extent(int32_t n, int32_t k, int32_t stride, int32_t pad) {
+  const int64_t span = (int64_t)n + 2 * (int64_t)pad;
+  if (span >= (1ll << 31)) return -1;
+  return span < k ? 0 : (span - k) / stride + 1;
+}
 // SMs of the current device (cached per device ordinal; 152 if the query fails)
 static int sm_count_api() {
   static std::atomic<int> cache[64];
@@ -859,8 +868,10 @@ static fqt1_status col2im_impl(const int32_t* acc, const fqt1_qgrad* psq, const 
     return FQT1_ERR_INVALID_ARG;
   if (!psq->slot_of_group || !psq->scale || !psq->zero || !psq->kept_idx || !psq->kept_count)
     return FQT1_ERR_INVALID_ARG;
-  const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
-  if (H + 2 * pad < kh || W + 2 * pad < kw) return FQT1_ERR_INVALID_ARG;
+  const int64_t Ho64 = conv_extent(H, kh, stride, pad), Wo64 = conv_extent(W, kw, stride, pad);
+  if (Ho64 == 0 || Wo64 == 0) return FQT1_ERR_INVALID_ARG;
+  if (Ho64 < 0 || Wo64 < 0 || Ho64 * Wo64 >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
+  const int Ho = (int)Ho64, Wo = (int)Wo64;
   if (!aligned16(acc) || !aligned16(dx)) return FQT1_ERR_MISALIGNED;
   constexpr int64_t kMaxTile = 96 * 1024;
   constexpr int64_t kPreferTile = 48 * 1024;  // >= 4 resident CTAs per SM
@@ -1009,8 +1020,10 @@ static fqt1_status col2im_colmajor_impl(const void* acc, int32_t acc_bits, int64
     return FQT1_ERR_INVALID_ARG;
   if (!psq->slot_of_group || !psq->scale || !psq->zero || !psq->kept_idx || !psq->kept_count)
     return FQT1_ERR_INVALID_ARG;
-  if (H + 2 * pad < kh || W + 2 * pad < kw) return FQT1_ERR_INVALID_ARG;
-  const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
+  const int64_t Ho64 = conv_extent(H, kh, stride, pad), Wo64 = conv_extent(W, kw, stride, pad);
+  if (Ho64 == 0 || Wo64 == 0) return FQT1_ERR_INVALID_ARG;
+  if (Ho64 < 0 || Wo64 < 0 || Ho64 * Wo64 >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
+  const int Ho = (int)Ho64, Wo = (int)Wo64;
   if (acc_bits != 16 && acc_bits != 32) return FQT1_ERR_INVALID_ARG;
   if (ld_acc < (int64_t)Ho * Wo || ld_acc % (acc_bits == 16 ? 8 : 4)) return FQT1_ERR_INVALID_ARG;
   if (!aligned16(acc) || !aligned16(dx)) return FQT1_ERR_MISALIGNED;
@@ -1122,8 +1135,10 @@ static fqt1_status bwd_input_fold_impl(const fqt1_qgrad* psq, const uint32_t* sw
   if (!valid_bits(p->bits) || !psq->codes || !psq->kept_count || !psq->kept_idx || !psq->slot_of_group ||
       !psq->scale || !psq->zero || psq->ld_codes < fqt1_codes_ld(D) || psq->ld_codes % 16)
     return FQT1_ERR_INVALID_ARG;
-  if (H + 2 * pad < kh || W + 2 * pad < kw) return FQT1_ERR_INVALID_ARG;
-  const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
+  const int64_t Ho64 = conv_extent(H, kh, stride, pad), Wo64 = conv_extent(W, kw, stride, pad);
+  if (Ho64 == 0 || Wo64 == 0) return FQT1_ERR_INVALID_ARG;
+  if (Ho64 < 0 || Wo64 < 0 || Ho64 * Wo64 >= (1ll << 31)) return FQT1_ERR_UNSUPPORTED;
+  const int Ho = (int)Ho64, Wo = (int)Wo64;
   if (p->rows_per_group != (int64_t)Ho * Wo) return FQT1_ERR_INVALID_ARG;
   if ((sw_col && !aligned16(sw_col)) || !aligned16(dx) || !aligned16(colsum_w)) return FQT1_ERR_MISALIGNED;
   // whole samples per 128-row tile, at least one channel's taps per tile, and the Folder's

@@ -1122,6 +1122,15 @@ using namespace fqt1;
 
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
+// Output extent of a convolution along one axis, (n + 2 pad - k) / stride + 1 for n, k, stride
+// >= 1 and pad >= 0, computed in 64 bits: 0 when the window does not fit, -1 when n + 2 pad
+// does not fit an int (the kernels' index arithmetic is 32-bit).
+static int64_t conv_extent(int32_t n, int32_t k, int32_t stride, int32_t pad) {
+  const int64_t span = (int64_t)n + 2 * (int64_t)pad;
+  if (span >= (1ll << 31)) return -1;
+  return span < k ? 0 : (span - k) / stride + 1;
+}
+
 extern "C" fqt1_status fqt1_binarize_pack(const float* x, int64_t rows, int64_t cols, int64_t ld,
                                           uint32_t* row_bits, uint32_t* col_bits, int32_t* colsum,
                                           void* stream) {
@@ -1205,8 +1214,10 @@ static fqt1_status im2col_impl(const float* x, const uint32_t* planes, int32_t N
   if ((!x && !planes) || N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 || pad < 0)
     return FQT1_ERR_INVALID_ARG;
   if (!row_bits && !col_bits && !colsum && !row_e4m3 && !col_e4m3) return FQT1_ERR_INVALID_ARG;
-  const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
-  if (H + 2 * pad < kh || W + 2 * pad < kw || Ho < 1 || Wo < 1) return FQT1_ERR_INVALID_ARG;
+  const int64_t Ho64 = conv_extent(H, kh, stride, pad), Wo64 = conv_extent(W, kw, stride, pad);
+  if (Ho64 == 0 || Wo64 == 0) return FQT1_ERR_INVALID_ARG;
+  if (Ho64 < 0 || Wo64 < 0) return FQT1_ERR_UNSUPPORTED;
+  const int Ho = (int)Ho64, Wo = (int)Wo64;
   if ((x && !aligned16(x)) || (row_bits && !aligned16(row_bits)) || (col_bits && !aligned16(col_bits)) ||
       (colsum && !aligned16(colsum)))
     return FQT1_ERR_MISALIGNED;
@@ -1447,7 +1458,9 @@ extern "C" fqt1_status fqt1_pack_planes(const float* x, int32_t N, int32_t C, in
 extern "C" int32_t fqt1_im2col_path(int32_t N, int32_t C, int32_t H, int32_t W, int32_t kh, int32_t kw,
                                     int32_t stride, int32_t pad) {
   if (N < 1 || C < 1 || H < 1 || W < 1 || kh < 1 || kw < 1 || stride < 1 || pad < 0) return -1;
-  if (H + 2 * pad < kh || W + 2 * pad < kw) return -1;
+  const int64_t Ho = conv_extent(H, kh, stride, pad), Wo = conv_extent(W, kw, stride, pad);
+  if (Ho < 1 || Wo < 1) return -1;
+  if ((int64_t)N * C * H * W >= (1ll << 31) || N * Ho * Wo >= (1ll << 31)) return -1;  // fqt1_im2col refuses these
   if (unfold_same_fits(N, C, H, W, kh, kw, stride, pad)) return 2;
   if (pointwise_conv(kh, kw, pad) && (int64_t)N * ((H - 1) / stride + 1) * ((W - 1) / stride + 1) < (1ll << 31))
     return 3;

@@ -102,6 +102,17 @@ def test_argument_validation_without_launch(lib):
                                     s) == 2
     # C kh kw = 2^19 x 64 x 64 = 2^31 columns (C H W = 2^29): refused before any launch
     assert lib.fqt1_col2im_colmajor(fake, 32, 4, C.byref(q), fake, 1, 1 << 19, 32, 32, 64, 64, 1, 16, fake, s) == 3
+    # shapes whose 32-bit index arithmetic would overflow are refused before any launch:
+    # H + 2 pad >= 2^31, or Ho Wo >= 2^31 (a 1 x 1 input padded by 30000: 60001^2 outputs)
+    huge, wide = 1 << 30, 30000
+    p8 = fqt1.AgpParams(2, 0, 1, 1)
+    for pad in (huge, wide):
+        assert lib.fqt1_col2im_colmajor(fake, 32, 4, C.byref(q), fake, 1, 1, 1, 1, 1, 1, 1, pad, fake, s) == 3
+        assert lib.fqt1_col2im(fake, C.byref(q), fake, 1, 1, 1, 1, 1, 1, 1, pad, fake, s) == 3
+        assert lib.fqt1_bwd_input_fold(C.byref(q), fake, fake, 1, 1, 1, 1, 1, 1, 1, pad, C.c_int64(8), C.byref(p8),
+                                       fake, s) == 3
+        assert lib.fqt1_im2col(fake, 1, 1, 1, 1, 1, 1, 1, pad, fake, None, None, s) == 3
+        assert lib.fqt1_im2col_path(1, 1, 1, 1, 1, 1, 1, pad) == -1
 
 
 def test_implicit_conv_support_rules(lib):
