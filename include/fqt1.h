@@ -413,7 +413,9 @@ fqt1_status fqt1_bwd_input_gemm_colmajor_e4m3w(const fqt1_qgrad* psq, const uint
  * dequantization: the same dx as fqt1_col2im (bit for bit), read with every
  * tap of a warp's 32 consecutive outputs as one contiguous run of a column.
  * acc: [C kh kw][ld_acc] from fqt1_bwd_input_gemm_colmajor with the same acc_bits
- * (the row of output pixel (oh, ow) of kept slot s is s Ho Wo + oh Wo + ow); dx:
+ * and ld_acc (the row of output pixel (oh, ow) of kept slot s is s Ho Wo + oh Wo + ow;
+ * this call reads rows up to kept count x Ho Wo, which the product's rule ld_acc >=
+ * capacity x rows_per_group keeps inside each column; it checks only ld_acc >= Ho Wo); dx:
  * [N, C, H, W], pruned samples 0.  N <= 65535, C H W < 2^31 and C kh kw < 2^31,
  * else FQT1_ERR_UNSUPPORTED. */
 fqt1_status fqt1_col2im_colmajor(const void* acc, int32_t acc_bits, int64_t ld_acc, const fqt1_qgrad* psq,
