@@ -197,7 +197,6 @@ def implicit_conv_acc(x, w, pad):
 
 
 # --------------------------------------------------------------------------
-# Backward, step 1: group ranges# --------------------------------------------------------------------------
 # Backward, step 1: group ranges (Sec. 3.2, PSQ Sec. 5.2, PCQ Sec. 5.3)
 # --------------------------------------------------------------------------
 def grad_to_quantize(gy, gamma):
