@@ -40,7 +40,7 @@ STAGE_SOURCES = {"pack": ("common.cuh", "pack.cu"), "gemm": ("api.cu", "common.c
                  "scq": ("common.cuh", "quantize.cu")}
 STAGE_GROUP = {"pack_w": "pack", "pack_xp": "pack", "im2col": "pack", "fwd_gemm": "gemm", "scq_quantize": "scq",
                "bwd_input_fold": "gemm", "bwd_weight_gemm": "gemm"}
-TRAFFIC_SOURCES = {"pack": "152daac4263996dc", "gemm": "589331ac6aa45757", "scq": "42a74653e8857164"}
+TRAFFIC_SOURCES = {"pack": "152daac4263996dc", "gemm": "59e795348d529633", "scq": "42a74653e8857164"}
 TRAFFIC_BYTES = {"pack_w": 2.383872e+06, "im2col": 8.423680e+06, "fwd_gemm": 3.029504e+06,
                  "scq_quantize": 1.6950016e+07, "bwd_input_fold": 1.205504e+06,
                  "bwd_weight_gemm": 2.982144e+06}

@@ -741,6 +741,7 @@ static int64_t conv_extent(int32_t n, int32_t k, int32_t stride, int32_t pad) {
   if (span >= (1ll << 31)) return -1;
   return span < k ? 0 : (span - k) / stride + 1;
 }
+
 // SMs of the current device (cached per device ordinal; 152 if the query fails)
 static int sm_count_api() {
   static std::atomic<int> cache[64];
